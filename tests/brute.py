@@ -1,0 +1,68 @@
+"""Brute-force allocation by enumeration (pure Python, tiny instances only).
+
+Independent of the C oracle: it enumerates every allocation of Section 3,
+Eqs. 1-5 (per class: nothing, or one SLO-feasible cell with 1 <= n <= G/tau
+replicas), keeps those within the GPU budget G, and maximises the minimum
+fulfilment r_i = min(lambda_i, n c) / lambda_i over classes. Fulfilment is
+computed in IEEE float32 (numpy scalars), one rounding per operation.
+"""
+
+from __future__ import annotations
+
+import itertools
+
+import numpy as np
+
+TP = (1, 2, 4, 8)
+
+
+def f32_fulfil(n, c, lam):
+    served = np.float32(n) * np.float32(c)
+    r = np.float32(served / np.float32(lam))
+    return np.float32(1.0) if r > np.float32(1.0) else r
+
+
+def options(K, B, G, cap, tail, demand, slo):
+    cap = np.asarray(cap, np.float32).reshape(K, 4, B)
+    tail = np.asarray(tail, np.float32).reshape(K, 4, B)
+    out = []
+    for i in range(K):
+        opts = []
+        for j, tau in enumerate(TP):
+            for b in range(B):
+                if not tail[i, j, b] <= slo[i]:
+                    continue
+                for n in range(1, G // tau + 1):
+                    f = f32_fulfil(n, cap[i, j, b], demand[i])
+                    opts.append((n * tau, j, n, float(cap[i, j, b]), b, float(f)))
+        out.append(opts)
+    return out
+
+
+def best_max_min(K, B, G, cap, tail, demand, slo):
+    """Largest min_i r_i over every feasible allocation (0 if a class must be empty)."""
+    opts = options(K, B, G, cap, tail, demand, slo)
+    best = 0.0
+    for combo in itertools.product(*[[None] + o for o in opts]):
+        cost = sum(c[0] for c in combo if c is not None)
+        if cost > G:
+            continue
+        if any(c is None for c in combo):
+            val = 0.0
+        else:
+            val = min(c[5] for c in combo)
+        best = max(best, val)
+    return best
+
+
+def choice_at(K, B, G, cap, tail, demand, slo, t):
+    """Per class, the preferred option covering t: (cost, TP, n, -capacity, bin) minimal."""
+    opts = options(K, B, G, cap, tail, demand, slo)
+    res = []
+    for o in opts:
+        cov = [x for x in o if x[5] >= t]
+        if not cov:
+            res.append(None)
+            continue
+        res.append(min(cov, key=lambda x: (x[0], x[1], x[2], -x[3], x[4])))
+    return res
