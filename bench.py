@@ -1,0 +1,366 @@
+"""Benchmark of the GB300 decision-gap scorer.
+
+One step = one fs_score_candidates pass over the paper-scale workload
+(2 classes, TP in {1,2,4,8}, G = 16, 8 load bins; 64 candidates x 8 outcomes x
+4096 samples = 2,097,152 scenarios, each solving the allocation under both
+realisations): base solves, per-candidate tables, the Monte-Carlo kernel and
+the reduction. Inputs are resident in HBM when the timed region starts; L2 is
+flushed (256 MiB write) between timed steps. Prints one JSON line.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload I] [--impl reference]
+
+--impl reference times the CPU oracle (single-threaded C) on a bounded
+sample of the same workload. Under torchrun (N > 1) every rank scores its own
+independent problem (stream id = rank): weak scaling, no collective on the
+data path.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+from paper_2608_19659_gb300 import workloads  # noqa: E402
+
+METRIC = "scenario allocation-solves/s"
+UNIT = "allocation-solves/s"
+SMS = 152
+ISSUE_PER_SM_CLK = 4 * 32  # 4 schedulers x 32 lanes, one warp instruction each per clock
+
+# Algorithmic thread-operations per scenario of the Monte-Carlo kernel (the
+# instruction-level minimum of the method's arithmetic; derivation in the
+# design notes): half a Philox4x32-10 call (10 rounds x 2 wide multiplies +
+# 2 three-input XORs) = 20, two quantile positions + lookups = 4, two affine
+# maps with clamps = 8, tail gate and two row patches = 5, two fulfilments
+# f = min(1, m C / lambda) with an IEEE division (>= 7 each) and the
+# max with the table threshold (2 each) = 18, gap and fixed-point add = 5.
+# The table searches (3 per probe) are not counted: a lower bound.
+OPS_PER_SCENARIO = 60
+
+
+def _env_int(name, default):
+    try:
+        return int(os.environ.get(name, default))
+    except ValueError:
+        return default
+
+
+def _measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f)
+    except OSError:
+        return {}
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle samples during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = str(gpu_index)
+        try:  # name the GPU by UUID: CUDA and nvidia-smi may number devices differently
+            import torch
+
+            u = str(torch.cuda.get_device_properties(gpu_index).uuid)
+            self.gpu = u if u.startswith("GPU-") else "GPU-" + u
+        except Exception:
+            pass
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(prefix="fs_clocks_", suffix=".csv")
+        os.close(fd)
+        try:
+            self.out = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.out, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+        self.out.close()
+
+    def summary(self):
+        try:
+            lines = [ln.split(",") for ln in open(self.path).read().strip().splitlines() if ln.strip()]
+            os.unlink(self.path)
+        except OSError:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for f in lines:
+            f = [x.strip() for x in f]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_setup(n_gpus: int):
+    world = _env_int("WORLD_SIZE", 1)
+    rank = _env_int("RANK", 0)
+    local = _env_int("LOCAL_RANK", 0)
+    if world > 1:
+        import torch.distributed as dist
+
+        backend = "nccl" if os.environ.get("FS_BENCH_BACKEND", "nccl") == "nccl" else "gloo"
+        dist.init_process_group(backend=backend)
+        return dist, rank, world, local
+    return None, 0, 1, 0
+
+
+def max_over_ranks(dist, value: float, device=None) -> float:
+    if dist is None:
+        return value
+    import torch
+
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(dist, value: float, device=None) -> float:
+    if dist is None:
+        return value
+    import torch
+
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+def config_of(w, extra=None):
+    c = {"workload": w.name, "classes": w.K, "load_bins": w.B, "gpu_budget": w.G,
+         "candidates": int(len(w.candidates)), "outcomes": w.O, "samples": w.S,
+         "scenarios_per_step": w.scenarios, "solves_per_scenario": 2,
+         "l2": "flushed between timed steps (256 MiB write)"}
+    if extra:
+        c.update(extra)
+    return c
+
+
+def cpu_baseline(w, seconds_target: float = 15.0):
+    """The oracle, single-threaded, on the first candidates of the workload (whole O x S each)."""
+    import oracle
+
+    qn = oracle.triangular_table(4096)
+    t0 = time.perf_counter()
+    oracle.score(w, qn, candidates=w.candidates[:1])
+    one = time.perf_counter() - t0
+    n = int(max(1, min(len(w.candidates), seconds_target / max(one, 1e-6))))
+    t0 = time.perf_counter()
+    oracle.score(w, qn, candidates=w.candidates[:n])
+    dt = time.perf_counter() - t0
+    scen = n * w.O * w.S
+    return {"value": 2 * scen / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"first {n} of {len(w.candidates)} candidates, all {w.O}x{w.S} scenarios each "
+                      f"({scen} scenarios, {dt:.1f} s)",
+            "candidate_scores_per_s": n / dt}
+
+
+def run_reference(args, w, rank):
+    if rank != 0:
+        return 0
+    import oracle
+
+    qn = oracle.triangular_table(4096)
+    # a bounded sample per step: enough candidates for about 1 s of CPU work
+    t0 = time.perf_counter()
+    oracle.score(w, qn, candidates=w.candidates[:1])
+    one = time.perf_counter() - t0
+    n = int(max(1, min(len(w.candidates), 1.0 / max(one, 1e-6))))
+    for _ in range(args.warmup):
+        oracle.score(w, qn, candidates=w.candidates[:n])
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        oracle.score(w, qn, candidates=w.candidates[:n])
+        times.append(time.perf_counter() - t0)
+    total = sum(times)
+    scen = n * w.O * w.S
+    value = 2 * scen * args.steps / total
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * total / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic", "config": config_of(w, {"reference_sample_candidates": n}),
+            "candidate_scores_per_s": n * args.steps / total,
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                             "sample": f"first {n} of {len(w.candidates)} candidates per step"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--workload", type=int, default=1)
+    ap.add_argument("--impl", default="native", choices=["native", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        args.warmup = 3
+
+    dist, rank, world, local = dist_setup(args.gpus)
+    w = workloads.make_workload(args.workload)
+    if args.impl == "reference":
+        rc = run_reference(args, w, rank)
+        if dist is not None:
+            dist.destroy_process_group()
+        return rc
+
+    import torch
+
+    from paper_2608_19659_gb300 import fleetsieve as fsb
+
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    fsb.lib()
+    stream = torch.cuda.current_stream()
+    n = len(w.candidates)
+    model = fsb.fs_load_model(w.cap_lo, w.cap_hi, w.tail_lo, w.tail_hi, w.slo, w.demand, w.G, w.K, w.B,
+                              stream=stream)
+    cand = torch.from_numpy(w.candidates).to(dev)
+    gap = torch.zeros(n, dtype=torch.float64, device=dev)
+    score = torch.zeros(n, dtype=torch.float64, device=dev)
+    gt = torch.zeros(1, dtype=torch.float32, device=dev)
+    best = torch.zeros(1, dtype=torch.int32, device=dev)
+    flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device=dev)  # 256 MiB > 129 MB L2
+    stream_id = rank
+
+    def step():
+        fsb.fs_score_candidates_async(model, cand, w.O, w.S, w.seed, stream_id, 0, gap_dev=gap,
+                                      score_dev=score, gamma_t_dev=gt, best_dev=best, stream=stream)
+
+    for _ in range(args.warmup):
+        flush.zero_()
+        step()
+    fsb.fs_check(model, stream)
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    fsb.fs_timing_read(model)
+    fsb.fs_timing_enable(model, True)
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    launches0 = fsb.fs_launch_count()
+    with ClockSampler(local) as clocks:
+        for k in range(args.steps):
+            flush.zero_()
+            starts[k].record(stream)
+            step()
+            ends[k].record(stream)
+        torch.cuda.synchronize()
+    launches = fsb.fs_launch_count() - launches0
+    if dist is not None:
+        dist.barrier()
+    fsb.fs_check(model, stream)
+    kernel_ms, kernel_n = fsb.fs_timing_read(model)
+    fsb.fs_timing_enable(model, False)
+    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    total_ms = max_over_ranks(dist, sum(step_ms), dev)
+    scen_all = sum_over_ranks(dist, float(w.scenarios) * args.steps, dev)
+    value = 2.0 * scen_all / (total_ms / 1000.0)
+
+    # end to end through the public host API: bounds in from pinned host memory,
+    # scores out to host memory, every step
+    pinned = {k: torch.from_numpy(getattr(w, k).reshape(-1).copy()).pin_memory().numpy()
+              for k in ("cap_lo", "cap_hi", "tail_lo", "tail_hi")}
+    cand_h = torch.from_numpy(w.candidates.copy()).pin_memory().numpy()
+    outs = (torch.zeros(n, dtype=torch.float64).pin_memory().numpy(),
+            torch.zeros(n, dtype=torch.float64).pin_memory().numpy(),
+            torch.zeros(1, dtype=torch.float32).pin_memory().numpy(),
+            torch.zeros(1, dtype=torch.int32).pin_memory().numpy(), None)
+
+    def e2e_step():
+        fsb.fs_update_bounds(model, pinned["cap_lo"], pinned["cap_hi"], pinned["tail_lo"], pinned["tail_hi"])
+        return fsb.fs_score_candidates(model, cand_h, w.O, w.S, w.seed, stream_id, 0, outputs=outs)
+
+    for _ in range(args.warmup):
+        e2e_step()
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        res = e2e_step()
+    torch.cuda.synchronize()
+    e2e_s = max_over_ranks(dist, time.perf_counter() - t0, dev)
+    e2e_value = 2.0 * scen_all / e2e_s
+    h2d = 16 * w.cells + w.cells + 4 * n
+    d2h = 8 * n + 8 * n + 4 + 4
+
+    peaks = _measured_peaks()
+    clk = clocks.summary()
+    sm_max = float(peaks.get("sm_max_mhz", 2070.0))
+    alu_peak = SMS * ISSUE_PER_SM_CLK * sm_max * 1e6  # thread-ops/s at the maximum SM clock
+    kern_s = kernel_ms / 1000.0 / max(kernel_n, 1)
+    achieved = OPS_PER_SCENARIO * w.scenarios / kern_s if kernel_n else None
+    roofline = {"bound": "alu", "kernel": "k_score (Monte-Carlo sampler + parametric re-solve)",
+                "achieved": achieved / 1e12 if achieved else None,
+                "peak": alu_peak / 1e12, "unit": "Tops/s (32-bit thread operations)",
+                "frac": (achieved / alu_peak) if achieved else None,
+                "traffic": None, "kernel_ms_per_launch": kern_s * 1000.0,
+                "ops_per_scenario": OPS_PER_SCENARIO,
+                "peak_basis": f"{SMS} SMs x 4 issue slots x 32 lanes x {sm_max:.0f} MHz (max SM clock)",
+                "kernel_share_of_step": (kernel_ms / max(sum(step_ms), 1e-9)) if kernel_n else None}
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w)
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": config_of(w, {"parallelism": f"replicas x{world} (independent problems)"}),
+            "candidate_scores_per_s": len(w.candidates) * args.steps * world / (total_ms / 1000.0),
+            "scenarios_per_s": scen_all / (total_ms / 1000.0),
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                    "api": "fs_update_bounds + fs_score_candidates (pinned host buffers)",
+                    "best": int(res.best)},
+            "gpu_launches": int(launches), "roofline": roofline, "clocks": clk,
+            "cpu_baseline": cpu}
+    if rank == 0:
+        print(json.dumps(line))
+    fsb.fs_free_model(model)
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

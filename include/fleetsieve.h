@@ -1,0 +1,276 @@
+/*
+ * fleetsieve.h -- C ABI of the GB300 decision-gap scorer.
+ *
+ * FleetSieve (decision-critical profiling for SLO-aware LLM fleet
+ * configuration) chooses which serving configuration to measure next by the
+ * expected reduction of the gap between a conservative and an optimistic
+ * fleet allocation. This library evaluates that expectation by Monte Carlo
+ * on one GPU (sm_103a):
+ *
+ *   fs_load_model         bounds, SLOs, demands, G  -> device-resident model
+ *   fs_score_candidates   samples                   -> E[Gamma_{t+1} | e], score, argmax
+ *   fs_solve(_batch)      realisation               -> allocation
+ *   fs_solve_bounds       conservative / optimistic allocations and Gamma_t
+ *   fs_reveal, fs_certificate, fs_replay            the profiling loop
+ *
+ * Notation (paper, Section 3): class i has demand lambda_i (req/s) and an SLO
+ * L_i (s) on its binding tail metric. A configuration is a TP degree
+ * tau in {1, 2, 4, 8} (index j = 0..3) and a load bin b; a replica of it uses
+ * tau GPUs and serves c req/s with tail l. Cells are indexed
+ * cell = (i * 4 + j) * B + b and every per-cell array is [K][4][B] row-major.
+ *
+ * Conventions for every call:
+ *   - returns FS_OK (0) or a negative FS_E* code; fs_last_error() gives a
+ *     thread-local message for the last failure of the calling thread;
+ *   - no exception or abort crosses the ABI;
+ *   - the caller owns every buffer it passes; inputs are copied (host inputs
+ *     before the call returns, device inputs in stream order);
+ *   - calls taking host output pointers are synchronous; calls named
+ *     *_async / *_batch take device pointers and a cudaStream_t (as void*),
+ *     enqueue their work and return; fs_check() synchronises such a stream and
+ *     reports device-side errors;
+ *   - one fs_model is not thread-safe; separate models are independent.
+ */
+#ifndef FLEETSIEVE_H
+#define FLEETSIEVE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum {
+    FS_OK = 0,
+    FS_EINVAL = -1,   /* bad argument: NaN/inf, lo > hi, sizes out of range, ... */
+    FS_ENOMEM = -2,   /* device or host allocation failed */
+    FS_ECUDA = -3,    /* a CUDA runtime call failed */
+    FS_ETIMEOUT = -4, /* a bounded device wait ran out (watchdog) */
+    FS_EDEVICE = -5   /* a kernel reported an inconsistency in its status word */
+};
+
+#define FS_TP_COUNT 4        /* TP degrees {1, 2, 4, 8} */
+#define FS_MAX_CLASSES 64    /* K */
+#define FS_MAX_BINS 4096     /* B */
+#define FS_MAX_GPUS 32767    /* G */
+#define FS_MAX_THRESHOLDS 16384 /* K * sum_tau floor(G / tau) must not exceed this */
+#define FS_MAX_SAMPLES_PER_CAND (1 << 22) /* O * S */
+
+typedef struct fs_model fs_model;
+
+/*
+ * Per-cell uncertainty state after round t (Section 4.1): capacity interval
+ * [cap_lo, cap_hi] (req/s per replica) and tail interval [tail_lo, tail_hi]
+ * (s). All four arrays are host pointers to [K][4][B] floats, finite, >= 0,
+ * lo <= hi. quantile: optional host table Qn[Q] in [0, 1], nondecreasing,
+ * of the posterior inside an interval (value v = lo + (hi - lo) * Qn[k]);
+ * NULL selects the built-in symmetric triangular table with Q = 4096.
+ * Q must be a power of two >= 4.
+ */
+typedef struct {
+    int32_t K;
+    int32_t B;
+    const float *cap_lo;
+    const float *cap_hi;
+    const float *tail_lo;
+    const float *tail_hi;
+    const float *quantile;
+    int32_t Q;
+    int32_t reserved;
+} fs_bounds;
+
+/*
+ * fs_load_model -- upload bounds, SLOs L_i (s, > 0), demands lambda_i
+ * (req/s, > 0) and the GPU budget G (Section 3, Eqs. 1-5) into a new model.
+ * cuda_stream: stream used by the synchronous calls of this model (NULL =
+ * default stream). Limits: 1 <= K <= 64, 1 <= B <= 4096, 1 <= G <= 32767,
+ * K * (floor(G/1) + floor(G/2) + floor(G/4) + floor(G/8)) <= 16384.
+ * All cells start unrevealed. *out is set only on success.
+ */
+int fs_load_model(const fs_bounds *bounds, const float *slo, const float *demand, int32_t G,
+                  void *cuda_stream, fs_model **out);
+
+/*
+ * fs_update_bounds -- replace the four bound arrays (host, [K][4][B]) of a
+ * model, e.g. after the intervals were refit (Algorithm 1, "fit joint
+ * capacity and tail intervals"). Revealed flags are kept. Synchronous.
+ */
+int fs_update_bounds(fs_model *m, const float *cap_lo, const float *cap_hi,
+                     const float *tail_lo, const float *tail_hi);
+
+/*
+ * Monte-Carlo plan of one scoring call (Section 4.3).
+ *   cand[n_cand]: candidate cell ids (host pointer for fs_score_candidates,
+ *     device pointer for fs_score_candidates_async); duplicates allowed;
+ *     revealed cells are allowed and score 0.
+ *   O: outcome strata, a power of two dividing Q; S >= 1 samples per
+ *     (candidate, outcome); O * S <= 2^22.
+ *   Draws: Philox4x32-10 (Salmon et al., SC'11) with key (seed_lo,
+ *     seed_hi XOR stream_id) and counter (s/2, o, cell, round); sample s uses
+ *     words 2(s&1) (capacity) and 2(s&1)+1 (tail); the top log2(Q/O) bits pick
+ *     a quantile inside stratum o.
+ */
+typedef struct {
+    uint64_t seed;
+    uint32_t stream_id;
+    uint32_t round;
+    int32_t n_cand;
+    int32_t O;
+    int32_t S;
+    int32_t reserved;
+    const int32_t *cand;
+} fs_samples;
+
+/*
+ * Per-scenario parity record written by the dump mode, one per scenario in
+ * (candidate, outcome, sample) order, record stride fs_dump_stride(m) bytes:
+ *   float c_y, l_y;          drawn capacity and tail of the candidate cell
+ *   float t_star[2];         t* of the patched conservative [0] / optimistic [1] realisation
+ *   int32_t total_gpus[2];
+ *   uint32_t choice[2][K];   per class: replicas n (bits 0-15), TP index j
+ *                            (bits 16-17), bin (bits 18-30); 0 = no replicas
+ */
+typedef struct {
+    float c_y;
+    float l_y;
+    float t_star[2];
+    int32_t total_gpus[2];
+} fs_scenario_head;
+
+/* Record stride of the dump for this model (bytes, a multiple of 8). */
+int32_t fs_dump_stride(const fs_model *m);
+
+/*
+ * fs_score_candidates -- score_t(e) = E[Gamma_t - Gamma_{t+1} | e] for every
+ * candidate (Section 4.3) with Gamma = t*(A+) - t*(A-) (Section 4.2, the
+ * max-min gap). For every candidate e, outcome o and sample s the drawn
+ * (c_y, l_y) replaces cell e in both the conservative (cap_lo, tail_hi) and
+ * the optimistic (cap_hi, tail_lo) realisation, both allocations are solved,
+ * and the gaps are summed in int64 fixed point (g = rint(Gamma' * 2^40)).
+ * Host outputs (each nullable):
+ *   gap_out[n_cand]   E[Gamma_{t+1} | e] = (sum g * 2^-40) / (O S)
+ *   score_out[n_cand] (rint(Gamma_t 2^40) O S - sum g) * 2^-40 / (O S)
+ *   gamma_t[1]        Gamma_t
+ *   best[1]           argmax cell: largest score, then lower TP (fewer
+ *                     profiling GPU-seconds, 300 s x TP), then earlier in cand;
+ *                     -1 if n_cand == 0
+ *   sum_eo[n_cand*O]  the int64 fixed-point sums per (candidate, outcome)
+ * dump_dev: optional DEVICE buffer of n_cand*O*S*fs_dump_stride(m) bytes.
+ */
+int fs_score_candidates(fs_model *m, const fs_samples *samples, double *gap_out,
+                        double *score_out, float *gamma_t, int32_t *best, int64_t *sum_eo,
+                        void *dump_dev);
+
+/* Same with samples->cand and every output on the device, enqueued on cuda_stream. */
+int fs_score_candidates_async(fs_model *m, const fs_samples *samples, double *gap_dev,
+                              double *score_dev, float *gamma_t_dev, int32_t *best_dev,
+                              int64_t *sum_eo_dev, void *dump_dev, void *cuda_stream);
+
+/*
+ * One allocation (Section 3): per class the chosen TP degree (0 = none),
+ * bin (-1 = none), replica count and fulfilment r_i; t_star = min_i r_i
+ * reached (the tier-2 objective), ok = t_star > 0.
+ */
+typedef struct {
+    float t_star;
+    int32_t total_gpus;
+    uint64_t has_option_mask; /* bit i: class i has an SLO-feasible cell */
+    int32_t ok;
+    int32_t reserved;
+    int8_t tp[FS_MAX_CLASSES];
+    int16_t bin[FS_MAX_CLASSES];
+    int16_t replicas[FS_MAX_CLASSES];
+    float fulfil[FS_MAX_CLASSES];
+} fs_allocation;
+
+/*
+ * fs_solve -- allocation of one realisation (host arrays cap, tail
+ * [K][4][B]) under the model's SLOs, demands and G. Tier 2 of the objective
+ * (Section 3): t* is the largest option fulfilment t for which every class's
+ * cheapest SLO-feasible option with fulfilment >= t fits in G together;
+ * ties: lower TP, then fewer replicas, then larger capacity, then lower bin;
+ * nothing fits -> t* = 0 and no class gets replicas.
+ */
+int fs_solve(fs_model *m, const float *cap, const float *tail, fs_allocation *out);
+
+/* n realisations, device arrays cap_dev/tail_dev [n][K][4][B], out_dev [n]. */
+int fs_solve_batch(fs_model *m, int32_t n, const float *cap_dev, const float *tail_dev,
+                   fs_allocation *out_dev, void *cuda_stream);
+
+/* A- and A+ at the current bounds (Section 4.1) and Gamma_t (host outputs, nullable). */
+int fs_solve_bounds(fs_model *m, fs_allocation *minus, fs_allocation *plus, float *gamma_t);
+
+/* Measurement of one cell: lo = hi = the measured value, marks it revealed. */
+int fs_reveal(fs_model *m, int32_t cell, float cap, float tail);
+
+/*
+ * Decision certificate (Section 4.2) without critical classes:
+ * *state = 1 (certified feasible) when Gamma_t <= eps and every cell to which
+ * A- commits replicas is revealed; else 0 (undecided). 2 (certified
+ * infeasible) is reserved for critical floors. gamma_t nullable.
+ */
+int fs_certificate(fs_model *m, float eps, int32_t *state, float *gamma_t);
+
+/*
+ * fs_replay -- Algorithm 1 on n_streams independent reveal orders over the
+ * model's bounds, batched on the device. Stream k: hidden truth
+ * truth_cap/truth_tail[k][cells], order perm[k][cells] (its first r0 cells
+ * are the common initial design; perm position breaks exact score ties).
+ * Each round: A-, A+, certificate (eps); if undecided, score the unrevealed
+ * cells (perm order) with O x S samples, Philox stream id k and round r,
+ * then reveal the argmax. Stops on the certificate, when no cell is left, or
+ * after max_rounds. All inputs are host pointers; outputs host, nullable:
+ *   rounds[k], state[k], gpu_seconds[k] (300 s x TP per revealed cell),
+ *   reveal_order[k][cells] (-1 padded), gamma_trace[k][max_rounds+1],
+ *   final_minus[k] (A- at the end).
+ */
+typedef struct {
+    int32_t n_streams;
+    int32_t r0;
+    float eps;
+    int32_t O;
+    int32_t S;
+    int32_t max_rounds;
+    uint64_t seed;
+    const float *truth_cap;
+    const float *truth_tail;
+    const int32_t *perm;
+} fs_replay_spec;
+
+int fs_replay(fs_model *m, const fs_replay_spec *spec, int32_t *rounds, int32_t *state,
+              double *gpu_seconds, int32_t *reveal_order, float *gamma_trace,
+              fs_allocation *final_minus);
+
+/* Synchronise cuda_stream (NULL = the model's) and report device-side errors. */
+int fs_check(fs_model *m, void *cuda_stream);
+
+/*
+ * Kernel timing for measurement. With on != 0, every later scoring call of
+ * this model records a pair of CUDA events around its Monte-Carlo kernel on
+ * the stream it launches on (up to 4096 pairs are kept). fs_timing_read waits
+ * for the recorded events, returns the summed kernel time (ms) and the number
+ * of timed launches, and clears the record. Not part of the method.
+ */
+int fs_timing_enable(fs_model *m, int32_t on);
+int fs_timing_read(fs_model *m, double *kernel_ms, int32_t *launches);
+
+/* Kernels this library has launched since it was loaded (all models). */
+uint64_t fs_launch_count(void);
+
+/*
+ * Watchdog self-test: one kernel waits on a shared-memory barrier that no
+ * copy ever completes, gives up after timeout_ns (clamped to [1 ms, 5 s]),
+ * records the timeout in a status word and returns; the call then returns
+ * FS_ETIMEOUT. Nothing is left running and the context stays usable.
+ */
+int fs_watchdog_selftest(int64_t timeout_ns);
+
+void fs_free_model(fs_model *m);
+
+const char *fs_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif

@@ -1,0 +1,683 @@
+// C ABI of the decision-gap scorer: model lifetime, argument checks, device
+// buffers and the launch sequence of each call. See include/fleetsieve.h for
+// the contract of every entry point.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <atomic>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "fs_internal.cuh"
+
+namespace fs {
+
+static std::atomic<uint64_t> g_launches{0};
+void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+
+static thread_local std::string g_err;
+
+static int fail(int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_err = buf;
+  return code;
+}
+
+static int cuda_fail(cudaError_t e, const char* what) {
+  return fail(e == cudaErrorMemoryAllocation ? FS_ENOMEM : FS_ECUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+#define FS_CUDA(call, what)                          \
+  do {                                               \
+    cudaError_t e_ = (call);                         \
+    if (e_ != cudaSuccess) return cuda_fail(e_, what); \
+  } while (0)
+
+static bool is_pow2(long long x) { return x > 0 && (x & (x - 1)) == 0; }
+
+static int log2i(long long x) {
+  int v = 0;
+  while ((1LL << v) < x) ++v;
+  return v;
+}
+
+// One device allocation that is grown on demand (never shrunk).
+struct Buf {
+  void* p = nullptr;
+  size_t bytes = 0;
+  int ensure(size_t want, const char* what) {
+    if (want <= bytes) return FS_OK;
+    if (p) cudaFree(p);
+    p = nullptr;
+    bytes = 0;
+    size_t b = std::max<size_t>(want, 256);
+    cudaError_t e = cudaMalloc(&p, b);
+    if (e != cudaSuccess) {
+      p = nullptr;
+      return cuda_fail(e, what);
+    }
+    bytes = b;
+    return FS_OK;
+  }
+  void release() {
+    if (p) cudaFree(p);
+    p = nullptr;
+    bytes = 0;
+  }
+};
+
+}  // namespace fs
+
+using namespace fs;
+
+struct fs_model {
+  Dims d{};
+  int device = 0;
+  int sm_count = 0;
+  cudaStream_t stream = nullptr;
+  // device state of the single problem (P = 1)
+  Buf fixed;      // lam, slo, qn, bounds, revealed, theta, ntheta, rowC, rowB, base, status
+  Set set{};
+  // per-call scratch
+  Buf cand, tables, sums, outs, real;
+  // host mirrors
+  std::vector<float> h_bounds;      // [4][cells]
+  std::vector<uint8_t> h_revealed;  // [cells]
+  std::vector<float> h_lam, h_slo;
+  // optional event pairs around the Monte-Carlo kernel
+  bool timing = false;
+  std::vector<cudaEvent_t> ev;      // 2 per timed launch
+  size_t ev_used = 0;
+};
+
+namespace {
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+constexpr size_t kMaxTimedEvents = 2 * 4096;
+
+int check_cells(const float* a, int n, const char* name) {
+  if (!a) return fail(FS_EINVAL, "%s is NULL", name);
+  for (int i = 0; i < n; ++i)
+    if (!std::isfinite(a[i]) || a[i] < 0.0f) return fail(FS_EINVAL, "%s[%d] = %g is not finite and >= 0", name, i, (double)a[i]);
+  return FS_OK;
+}
+
+int check_bounds4(const float* clo, const float* chi, const float* tlo, const float* thi, int cells) {
+  int rc;
+  if ((rc = check_cells(clo, cells, "cap_lo")) || (rc = check_cells(chi, cells, "cap_hi")) ||
+      (rc = check_cells(tlo, cells, "tail_lo")) || (rc = check_cells(thi, cells, "tail_hi")))
+    return rc;
+  for (int c = 0; c < cells; ++c) {
+    if (clo[c] > chi[c]) return fail(FS_EINVAL, "cap_lo[%d] > cap_hi[%d]", c, c);
+    if (tlo[c] > thi[c]) return fail(FS_EINVAL, "tail_lo[%d] > tail_hi[%d]", c, c);
+  }
+  return FS_OK;
+}
+
+// +0 for -0, so that nonnegative floats order like their bit patterns.
+inline float canon(float v) { return v == 0.0f ? 0.0f : v; }
+
+int upload_bounds(fs_model* m) {
+  FS_CUDA(cudaMemcpyAsync(m->set.bounds, m->h_bounds.data(), m->h_bounds.size() * 4, cudaMemcpyHostToDevice,
+                          m->stream),
+          "upload bounds");
+  FS_CUDA(cudaMemcpyAsync(m->set.revealed, m->h_revealed.data(), m->h_revealed.size(), cudaMemcpyHostToDevice,
+                          m->stream),
+          "upload revealed");
+  FS_CUDA(cudaStreamSynchronize(m->stream), "upload sync");
+  return FS_OK;
+}
+
+int read_status(fs_model* m, cudaStream_t s) {
+  FS_CUDA(cudaStreamSynchronize(s), "synchronize");
+  uint32_t st = 0;
+  FS_CUDA(cudaMemcpy(&st, m->set.status, 4, cudaMemcpyDeviceToHost), "read status");
+  if (st) {
+    uint32_t z = 0;
+    cudaMemcpy(m->set.status, &z, 4, cudaMemcpyHostToDevice);
+    if (st & ST_TIMEOUT) return fail(FS_ETIMEOUT, "a device wait timed out (status 0x%x)", st);
+    return fail(FS_EDEVICE, "device status word 0x%x", st);
+  }
+  return FS_OK;
+}
+
+int check_samples(const fs_model* m, const fs_samples* s, bool host_cand) {
+  if (!s) return fail(FS_EINVAL, "samples is NULL");
+  if (s->n_cand < 0) return fail(FS_EINVAL, "n_cand < 0");
+  if (s->n_cand > 0 && !s->cand) return fail(FS_EINVAL, "cand is NULL");
+  if (!is_pow2(s->O) || s->O > m->d.Q) return fail(FS_EINVAL, "O = %d must be a power of two <= Q = %d", s->O, m->d.Q);
+  if (s->S < 1) return fail(FS_EINVAL, "S = %d < 1", s->S);
+  if ((long long)s->O * s->S > FS_MAX_SAMPLES_PER_CAND) return fail(FS_EINVAL, "O * S exceeds 2^22");
+  if ((long long)s->n_cand * s->O > (1LL << 30)) return fail(FS_EINVAL, "n_cand * O too large");
+  if (host_cand)
+    for (int e = 0; e < s->n_cand; ++e)
+      if (s->cand[e] < 0 || s->cand[e] >= m->d.cells) return fail(FS_EINVAL, "cand[%d] = %d out of range", e, s->cand[e]);
+  return FS_OK;
+}
+
+Plan make_plan(const fs_model* m, const fs_samples* s, int n_items) {
+  Plan pl{};
+  pl.key0 = (uint32_t)s->seed;
+  pl.key1 = (uint32_t)(s->seed >> 32);
+  pl.stream_base = s->stream_id;
+  pl.round = s->round;
+  pl.O = s->O;
+  pl.S = s->S;
+  pl.W = m->d.Q / s->O;
+  pl.w = log2i(pl.W);
+  pl.pairs = (s->S + 1) / 2;
+  const long long all_pairs = (long long)n_items * s->O * pl.pairs;
+  const long long slots = (long long)m->sm_count * 2048 * 2;  // two waves of resident threads
+  long long ppt = (all_pairs + slots - 1) / std::max<long long>(slots, 1);
+  ppt = std::min<long long>(std::max<long long>(ppt, 1), 16);
+  pl.ppt = (int)ppt;
+  const long long per_tile = (long long)kScoreThreads * pl.ppt;
+  pl.chunks = (int)((pl.pairs + per_tile - 1) / per_tile);
+  return pl;
+}
+
+int ensure_items(fs_model* m, int n, int O) {
+  int rc;
+  if ((rc = m->cand.ensure((size_t)std::max(n, 1) * 4, "candidate list"))) return rc;
+  if ((rc = m->tables.ensure((size_t)std::max(n, 1) * 2 * m->d.slot_floats * 4, "candidate tables"))) return rc;
+  if ((rc = m->sums.ensure((size_t)std::max(n, 1) * O * 8, "sums"))) return rc;
+  if ((rc = m->outs.ensure((size_t)std::max(n, 1) * 16 + 64, "outputs"))) return rc;
+  return FS_OK;
+}
+
+// The scoring sequence on stream s; cand_dev holds n_cand cell ids.
+int run_score(fs_model* m, const fs_samples* smp, const int32_t* cand_dev, double* gap, double* score,
+              float* gamma_t, int32_t* best, void* dump, cudaStream_t s) {
+  const int n = smp->n_cand;
+  Items it{};
+  it.n = n;
+  it.p = nullptr;
+  it.cell = cand_dev;
+  it.off = nullptr;
+  const Plan pl = make_plan(m, smp, n);
+  FS_CUDA(launch_solve(m->set, 2, nullptr, nullptr, nullptr, true, s), "launch solve");
+  FS_CUDA(launch_prep(m->set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, s), "launch prep");
+  const bool timed = m->timing && n > 0 && m->ev_used + 2 <= kMaxTimedEvents;
+  if (timed) {
+    while (m->ev.size() < m->ev_used + 2) {
+      cudaEvent_t e;
+      FS_CUDA(cudaEventCreate(&e), "create timing event");
+      m->ev.push_back(e);
+    }
+    FS_CUDA(cudaEventRecord(m->ev[m->ev_used], s), "record timing event");
+  }
+  FS_CUDA(launch_score(m->set, it, pl, (const float*)m->tables.p, (uint64_t*)m->sums.p, dump,
+                       fs_dump_stride(m), m->sm_count, s),
+          "launch score");
+  if (timed) {
+    FS_CUDA(cudaEventRecord(m->ev[m->ev_used + 1], s), "record timing event");
+    m->ev_used += 2;
+  }
+  FS_CUDA(launch_finalize(m->set, it, pl, (const uint64_t*)m->sums.p, gap, score, gamma_t, best, s),
+          "launch finalize");
+  return FS_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* fs_last_error(void) { return g_err.c_str(); }
+
+uint64_t fs_launch_count(void) { return g_launches.load(); }
+
+int32_t fs_dump_stride(const fs_model* m) {
+  if (!m) return 0;
+  return (int32_t)align_up(sizeof(fs_scenario_head) + 8 * (size_t)m->d.K, 8);
+}
+
+int fs_load_model(const fs_bounds* b, const float* slo, const float* demand, int32_t G, void* cuda_stream,
+                  fs_model** out) {
+  if (!out) return fail(FS_EINVAL, "out is NULL");
+  if (!b) return fail(FS_EINVAL, "bounds is NULL");
+  if (b->K < 1 || b->K > FS_MAX_CLASSES) return fail(FS_EINVAL, "K = %d outside [1, %d]", b->K, FS_MAX_CLASSES);
+  if (b->B < 1 || b->B > FS_MAX_BINS) return fail(FS_EINVAL, "B = %d outside [1, %d]", b->B, FS_MAX_BINS);
+  if (G < 1 || G > FS_MAX_GPUS) return fail(FS_EINVAL, "G = %d outside [1, %d]", G, FS_MAX_GPUS);
+  const int K = b->K, B = b->B, cells = K * 4 * B;
+  const long long theta_cap = (long long)K * ((G >> 0) + (G >> 1) + (G >> 2) + (G >> 3));
+  if (theta_cap > FS_MAX_THRESHOLDS)
+    return fail(FS_EINVAL, "K * sum floor(G/tau) = %lld exceeds %d", theta_cap, FS_MAX_THRESHOLDS);
+  int rc = check_bounds4(b->cap_lo, b->cap_hi, b->tail_lo, b->tail_hi, cells);
+  if (rc) return rc;
+  if (!slo || !demand) return fail(FS_EINVAL, "slo / demand is NULL");
+  for (int i = 0; i < K; ++i) {
+    if (!std::isfinite(slo[i]) || !(slo[i] > 0.0f)) return fail(FS_EINVAL, "slo[%d] must be finite and > 0", i);
+    if (!std::isfinite(demand[i]) || !(demand[i] > 0.0f)) return fail(FS_EINVAL, "demand[%d] must be finite and > 0", i);
+  }
+  int Q = 4096;
+  if (b->quantile) {
+    Q = b->Q;
+    if (!is_pow2(Q) || Q < 4 || Q > (1 << 24)) return fail(FS_EINVAL, "Q = %d must be a power of two in [4, 2^24]", Q);
+    for (int k = 0; k < Q; ++k) {
+      const float v = b->quantile[k];
+      if (!(v >= 0.0f && v <= 1.0f)) return fail(FS_EINVAL, "quantile[%d] = %g outside [0, 1]", k, (double)v);
+      if (k && v < b->quantile[k - 1]) return fail(FS_EINVAL, "quantile table decreases at %d", k);
+    }
+  }
+
+  fs_model* m = new (std::nothrow) fs_model();
+  if (!m) return fail(FS_ENOMEM, "host allocation");
+  m->stream = (cudaStream_t)cuda_stream;
+  cudaError_t e = cudaGetDevice(&m->device);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&m->sm_count, cudaDevAttrMultiProcessorCount, m->device);
+  if (e != cudaSuccess) {
+    delete m;
+    return cuda_fail(e, "device query");
+  }
+  Dims& d = m->d;
+  d.K = K;
+  d.B = B;
+  d.G = G;
+  d.Q = Q;
+  d.cells = cells;
+  d.K4 = 4 * K;
+  for (int j = 0; j < kT; ++j) d.M[j] = G >> j;
+  d.theta_cap = (int)theta_cap;
+  d.lcap = (d.theta_cap + 3) & ~3;
+  d.slot_floats = kTableHeader + 3 * d.lcap;
+
+  // fixed device state, one allocation carved into 256-byte aligned pieces
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    size_t o = off;
+    off = align_up(off + bytes, 256);
+    return o;
+  };
+  const size_t o_lam = take(4 * K), o_slo = take(4 * K), o_qn = take(4 * (size_t)Q);
+  const size_t o_bounds = take(16 * (size_t)cells), o_rev = take(cells);
+  const size_t o_theta = take(8 * (size_t)d.theta_cap), o_nth = take(8);
+  const size_t o_rowc = take(8 * (size_t)d.K4), o_rowb = take(8 * (size_t)d.K4);
+  const size_t o_base = take(2 * sizeof(fs_allocation)), o_status = take(4);
+  rc = m->fixed.ensure(off, "model state");
+  if (rc) {
+    delete m;
+    return rc;
+  }
+  char* base = (char*)m->fixed.p;
+  Set& s = m->set;
+  s.d = d;
+  s.P = 1;
+  s.lam = (const float*)(base + o_lam);
+  s.slo = (const float*)(base + o_slo);
+  s.qn = (const float*)(base + o_qn);
+  s.bounds = (float*)(base + o_bounds);
+  s.revealed = (uint8_t*)(base + o_rev);
+  s.theta = (float*)(base + o_theta);
+  s.ntheta = (int*)(base + o_nth);
+  s.rowC = (float*)(base + o_rowc);
+  s.rowB = (int*)(base + o_rowb);
+  s.base = (fs_allocation*)(base + o_base);
+  s.status = (uint32_t*)(base + o_status);
+  s.skip = nullptr;
+
+  m->h_lam.assign(demand, demand + K);
+  m->h_slo.assign(slo, slo + K);
+  m->h_bounds.resize(4 * (size_t)cells);
+  const float* src[4] = {b->cap_lo, b->cap_hi, b->tail_lo, b->tail_hi};
+  for (int r = 0; r < 4; ++r)
+    for (int c = 0; c < cells; ++c) m->h_bounds[(size_t)r * cells + c] = canon(src[r][c]);
+  m->h_revealed.assign(cells, 0);
+
+  auto bail = [&](int code) {
+    fs_free_model(m);
+    return code;
+  };
+  e = cudaMemsetAsync(m->fixed.p, 0, off, m->stream);
+  if (e == cudaSuccess) e = cudaMemcpyAsync((void*)s.lam, demand, 4 * K, cudaMemcpyHostToDevice, m->stream);
+  if (e == cudaSuccess) e = cudaMemcpyAsync((void*)s.slo, slo, 4 * K, cudaMemcpyHostToDevice, m->stream);
+  if (e == cudaSuccess) {
+    if (b->quantile) e = cudaMemcpyAsync((void*)s.qn, b->quantile, 4 * (size_t)Q, cudaMemcpyHostToDevice, m->stream);
+    else e = launch_qtable((float*)s.qn, Q, m->stream);
+  }
+  if (e != cudaSuccess) return bail(cuda_fail(e, "model upload"));
+  rc = upload_bounds(m);
+  if (rc) return bail(rc);
+  *out = m;
+  return FS_OK;
+}
+
+int fs_update_bounds(fs_model* m, const float* cap_lo, const float* cap_hi, const float* tail_lo,
+                     const float* tail_hi) {
+  if (!m) return fail(FS_EINVAL, "model is NULL");
+  const int cells = m->d.cells;
+  int rc = check_bounds4(cap_lo, cap_hi, tail_lo, tail_hi, cells);
+  if (rc) return rc;
+  const float* src[4] = {cap_lo, cap_hi, tail_lo, tail_hi};
+  for (int r = 0; r < 4; ++r)
+    for (int c = 0; c < cells; ++c) m->h_bounds[(size_t)r * cells + c] = canon(src[r][c]);
+  return upload_bounds(m);
+}
+
+int fs_score_candidates(fs_model* m, const fs_samples* smp, double* gap_out, double* score_out, float* gamma_t,
+                        int32_t* best, int64_t* sum_eo, void* dump_dev) {
+  if (!m) return fail(FS_EINVAL, "model is NULL");
+  int rc = check_samples(m, smp, true);
+  if (rc) return rc;
+  const int n = smp->n_cand;
+  if ((rc = ensure_items(m, n, smp->O))) return rc;
+  double* d_gap = (double*)m->outs.p;
+  double* d_score = d_gap + std::max(n, 1);
+  float* d_gt = (float*)(d_score + std::max(n, 1));
+  int32_t* d_best = (int32_t*)(d_gt + 4);
+  cudaStream_t s = m->stream;
+  if (n > 0)
+    FS_CUDA(cudaMemcpyAsync(m->cand.p, smp->cand, 4 * (size_t)n, cudaMemcpyHostToDevice, s), "upload candidates");
+  rc = run_score(m, smp, (const int32_t*)m->cand.p, d_gap, d_score, d_gt, d_best, dump_dev, s);
+  if (rc) return rc;
+  if (gap_out && n) FS_CUDA(cudaMemcpyAsync(gap_out, d_gap, 8 * (size_t)n, cudaMemcpyDeviceToHost, s), "read gap");
+  if (score_out && n) FS_CUDA(cudaMemcpyAsync(score_out, d_score, 8 * (size_t)n, cudaMemcpyDeviceToHost, s), "read score");
+  if (gamma_t) FS_CUDA(cudaMemcpyAsync(gamma_t, d_gt, 4, cudaMemcpyDeviceToHost, s), "read gamma");
+  if (best) FS_CUDA(cudaMemcpyAsync(best, d_best, 4, cudaMemcpyDeviceToHost, s), "read best");
+  if (sum_eo && n)
+    FS_CUDA(cudaMemcpyAsync(sum_eo, m->sums.p, 8 * (size_t)n * smp->O, cudaMemcpyDeviceToHost, s), "read sums");
+  return read_status(m, s);
+}
+
+int fs_score_candidates_async(fs_model* m, const fs_samples* smp, double* gap_dev, double* score_dev,
+                              float* gamma_t_dev, int32_t* best_dev, int64_t* sum_eo_dev, void* dump_dev,
+                              void* cuda_stream) {
+  if (!m) return fail(FS_EINVAL, "model is NULL");
+  int rc = check_samples(m, smp, false);
+  if (rc) return rc;
+  const int n = smp->n_cand;
+  if ((rc = ensure_items(m, n, smp->O))) return rc;
+  cudaStream_t s = (cudaStream_t)cuda_stream;
+  rc = run_score(m, smp, smp->cand, gap_dev, score_dev, gamma_t_dev, best_dev, dump_dev, s);
+  if (rc) return rc;
+  if (sum_eo_dev && n)
+    FS_CUDA(cudaMemcpyAsync(sum_eo_dev, m->sums.p, 8 * (size_t)n * smp->O, cudaMemcpyDeviceToDevice, s),
+            "copy sums");
+  return FS_OK;
+}
+
+int fs_solve(fs_model* m, const float* cap, const float* tail, fs_allocation* out) {
+  if (!m) return fail(FS_EINVAL, "model is NULL");
+  if (!out) return fail(FS_EINVAL, "out is NULL");
+  const int cells = m->d.cells;
+  int rc;
+  if ((rc = check_cells(cap, cells, "cap")) || (rc = check_cells(tail, cells, "tail"))) return rc;
+  if ((rc = m->real.ensure(8 * (size_t)cells + 256 + sizeof(fs_allocation), "realisation"))) return rc;
+  float* d_cap = (float*)m->real.p;
+  float* d_tail = d_cap + cells;
+  fs_allocation* d_out = (fs_allocation*)((char*)m->real.p + align_up(8 * (size_t)cells, 256));
+  cudaStream_t s = m->stream;
+  FS_CUDA(cudaMemcpyAsync(d_cap, cap, 4 * (size_t)cells, cudaMemcpyHostToDevice, s), "upload cap");
+  FS_CUDA(cudaMemcpyAsync(d_tail, tail, 4 * (size_t)cells, cudaMemcpyHostToDevice, s), "upload tail");
+  FS_CUDA(launch_solve(m->set, 1, d_cap, d_tail, d_out, false, s), "launch solve");
+  FS_CUDA(cudaMemcpyAsync(out, d_out, sizeof(fs_allocation), cudaMemcpyDeviceToHost, s), "read allocation");
+  return read_status(m, s);
+}
+
+int fs_solve_batch(fs_model* m, int32_t n, const float* cap_dev, const float* tail_dev, fs_allocation* out_dev,
+                   void* cuda_stream) {
+  if (!m) return fail(FS_EINVAL, "model is NULL");
+  if (n < 0) return fail(FS_EINVAL, "n < 0");
+  if (n == 0) return FS_OK;
+  if (!cap_dev || !tail_dev || !out_dev) return fail(FS_EINVAL, "NULL device pointer");
+  FS_CUDA(launch_solve(m->set, n, cap_dev, tail_dev, out_dev, false, (cudaStream_t)cuda_stream), "launch solve");
+  return FS_OK;
+}
+
+int fs_solve_bounds(fs_model* m, fs_allocation* minus, fs_allocation* plus, float* gamma_t) {
+  if (!m) return fail(FS_EINVAL, "model is NULL");
+  cudaStream_t s = m->stream;
+  FS_CUDA(launch_solve(m->set, 2, nullptr, nullptr, nullptr, true, s), "launch solve");
+  fs_allocation h[2];
+  FS_CUDA(cudaMemcpyAsync(h, m->set.base, sizeof h, cudaMemcpyDeviceToHost, s), "read allocations");
+  int rc = read_status(m, s);
+  if (rc) return rc;
+  if (minus) *minus = h[0];
+  if (plus) *plus = h[1];
+  if (gamma_t) *gamma_t = h[1].t_star - h[0].t_star;
+  return FS_OK;
+}
+
+int fs_reveal(fs_model* m, int32_t cell, float cap, float tail) {
+  if (!m) return fail(FS_EINVAL, "model is NULL");
+  if (cell < 0 || cell >= m->d.cells) return fail(FS_EINVAL, "cell %d out of range", cell);
+  if (!std::isfinite(cap) || cap < 0.0f || !std::isfinite(tail) || tail < 0.0f)
+    return fail(FS_EINVAL, "measured values must be finite and >= 0");
+  const int cells = m->d.cells;
+  m->h_bounds[(size_t)CAP_LO * cells + cell] = canon(cap);
+  m->h_bounds[(size_t)CAP_HI * cells + cell] = canon(cap);
+  m->h_bounds[(size_t)TAIL_LO * cells + cell] = canon(tail);
+  m->h_bounds[(size_t)TAIL_HI * cells + cell] = canon(tail);
+  m->h_revealed[cell] = 1;
+  return upload_bounds(m);
+}
+
+int fs_certificate(fs_model* m, float eps, int32_t* state, float* gamma_t) {
+  if (!m) return fail(FS_EINVAL, "model is NULL");
+  if (!state) return fail(FS_EINVAL, "state is NULL");
+  if (std::isnan(eps)) return fail(FS_EINVAL, "eps is NaN");
+  fs_allocation am, ap;
+  float gt;
+  int rc = fs_solve_bounds(m, &am, &ap, &gt);
+  if (rc) return rc;
+  bool known = true;
+  for (int i = 0; i < m->d.K; ++i) {
+    if (am.replicas[i] <= 0) continue;
+    int j = 0;
+    while (j < kT && (1 << j) != am.tp[i]) ++j;
+    if (!m->h_revealed[(size_t)(i * 4 + j) * m->d.B + am.bin[i]]) known = false;
+  }
+  *state = (gt <= eps && known) ? 1 : 0;
+  if (gamma_t) *gamma_t = gt;
+  return FS_OK;
+}
+
+int fs_replay(fs_model* m, const fs_replay_spec* sp, int32_t* rounds, int32_t* state, double* gpu_seconds,
+              int32_t* reveal_order, float* gamma_trace, fs_allocation* final_minus) {
+  if (!m) return fail(FS_EINVAL, "model is NULL");
+  if (!sp) return fail(FS_EINVAL, "spec is NULL");
+  const Dims d = m->d;
+  const int P = sp->n_streams, cells = d.cells;
+  if (P < 1 || P > 65536) return fail(FS_EINVAL, "n_streams = %d outside [1, 65536]", P);
+  if (sp->r0 < 0 || sp->r0 > cells) return fail(FS_EINVAL, "r0 = %d outside [0, cells]", sp->r0);
+  if (sp->max_rounds < 0 || sp->max_rounds > cells) return fail(FS_EINVAL, "max_rounds outside [0, cells]");
+  if (std::isnan(sp->eps)) return fail(FS_EINVAL, "eps is NaN");
+  if (!sp->truth_cap || !sp->truth_tail || !sp->perm) return fail(FS_EINVAL, "NULL truth / perm");
+  fs_samples probe{sp->seed, 0, 0, 0, sp->O, sp->S, 0, nullptr};
+  int rc = check_samples(m, &probe, false);
+  if (rc) return rc;
+  if ((rc = check_cells(sp->truth_cap, P * cells, "truth_cap")) || (rc = check_cells(sp->truth_tail, P * cells, "truth_tail")))
+    return rc;
+  std::vector<char> seen(cells);
+  for (int k = 0; k < P; ++k) {
+    std::fill(seen.begin(), seen.end(), 0);
+    for (int q = 0; q < cells; ++q) {
+      const int c = sp->perm[(size_t)k * cells + q];
+      if (c < 0 || c >= cells || seen[c]) return fail(FS_EINVAL, "perm[%d] is not a permutation of the cells", k);
+      seen[c] = 1;
+    }
+  }
+
+  // device state of P problems
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    size_t o = off;
+    off = align_up(off + bytes, 256);
+    return o;
+  };
+  const size_t o_bounds = take(16 * (size_t)P * cells), o_rev = take((size_t)P * cells);
+  const size_t o_theta = take(8 * (size_t)P * d.theta_cap), o_nth = take(8 * (size_t)P);
+  const size_t o_rowc = take(8 * (size_t)P * d.K4), o_rowb = take(8 * (size_t)P * d.K4);
+  const size_t o_base = take(2 * (size_t)P * sizeof(fs_allocation));
+  const size_t o_truth = take(8 * (size_t)P * cells), o_perm = take(4 * (size_t)P * cells);
+  const size_t o_rounds = take(4 * (size_t)P), o_state = take(4 * (size_t)P), o_gs = take(8 * (size_t)P);
+  const size_t o_order = take(4 * (size_t)P * cells), o_nrev = take(4 * (size_t)P);
+  const size_t o_trace = take(4 * (size_t)P * (sp->max_rounds + 1));
+  const size_t o_final = take((size_t)P * sizeof(fs_allocation)), o_active = take(4 * (size_t)P), o_nact = take(4);
+  const size_t o_ip = take(4 * (size_t)P * cells), o_ic = take(4 * (size_t)P * cells);
+  Buf all;
+  if ((rc = all.ensure(off, "replay state"))) return rc;
+  char* base = (char*)all.p;
+  Set set = m->set;
+  set.P = P;
+  set.bounds = (float*)(base + o_bounds);
+  set.revealed = (uint8_t*)(base + o_rev);
+  set.theta = (float*)(base + o_theta);
+  set.ntheta = (int*)(base + o_nth);
+  set.rowC = (float*)(base + o_rowc);
+  set.rowB = (int*)(base + o_rowb);
+  set.base = (fs_allocation*)(base + o_base);
+  ReplayState rs{};
+  rs.truth = (const float*)(base + o_truth);
+  rs.perm = (const int*)(base + o_perm);
+  rs.rounds = (int*)(base + o_rounds);
+  rs.state = (int*)(base + o_state);
+  rs.gpu_seconds = (double*)(base + o_gs);
+  rs.reveal_order = (int*)(base + o_order);
+  rs.n_revealed = (int*)(base + o_nrev);
+  rs.gamma_trace = (float*)(base + o_trace);
+  rs.final_minus = (fs_allocation*)(base + o_final);
+  rs.active = (int*)(base + o_active);
+  rs.n_active = (int*)(base + o_nact);
+  rs.item_p = (int*)(base + o_ip);
+  rs.item_cell = (int*)(base + o_ic);
+  rs.item_off = nullptr;
+  rs.max_rounds = sp->max_rounds;
+  rs.eps = sp->eps;
+  set.skip = rs.state;
+
+  cudaStream_t s = m->stream;
+  auto run = [&]() -> int {
+    FS_CUDA(cudaMemsetAsync(all.p, 0, off, s), "clear replay state");
+    for (int k = 0; k < P; ++k) {
+      FS_CUDA(cudaMemcpyAsync(set.bounds + (size_t)k * 4 * cells, m->h_bounds.data(), 16 * (size_t)cells,
+                              cudaMemcpyHostToDevice, s),
+              "upload prior");
+    }
+    std::vector<float> truth(2 * (size_t)P * cells);
+    for (int k = 0; k < P; ++k) {
+      std::memcpy(&truth[(2 * (size_t)k) * cells], sp->truth_cap + (size_t)k * cells, 4 * (size_t)cells);
+      std::memcpy(&truth[(2 * (size_t)k + 1) * cells], sp->truth_tail + (size_t)k * cells, 4 * (size_t)cells);
+    }
+    for (auto& v : truth) v = canon(v);
+    FS_CUDA(cudaMemcpyAsync((void*)rs.truth, truth.data(), 4 * truth.size(), cudaMemcpyHostToDevice, s), "upload truth");
+    FS_CUDA(cudaMemcpyAsync((void*)rs.perm, sp->perm, 4 * (size_t)P * cells, cudaMemcpyHostToDevice, s), "upload perm");
+    FS_CUDA(launch_replay_init(set, rs, sp->r0, s), "launch replay init");
+    const int rc_sync = read_status(m, s);  // truth buffer must outlive the copy
+    if (rc_sync) return rc_sync;
+    for (int r = 0; r <= sp->max_rounds; ++r) {
+      FS_CUDA(launch_solve(set, 2 * P, nullptr, nullptr, nullptr, true, s), "launch solve");
+      FS_CUDA(cudaMemsetAsync(rs.n_active, 0, 4, s), "clear active");
+      FS_CUDA(launch_replay_certify(set, rs, r, s), "launch certify");
+      int n_active = 0;
+      FS_CUDA(cudaMemcpyAsync(&n_active, rs.n_active, 4, cudaMemcpyDeviceToHost, s), "read active");
+      FS_CUDA(cudaStreamSynchronize(s), "round sync");
+      if (n_active == 0) break;
+      const int per = cells - sp->r0 - r;
+      if (per <= 0) break;
+      const int n_items = n_active * per;
+      int rc2 = ensure_items(m, n_items, sp->O);
+      if (rc2) return rc2;
+      FS_CUDA(launch_replay_items(set, rs, n_active, per, s), "launch items");
+      Items it{};
+      it.n = n_items;
+      it.p = rs.item_p;
+      it.cell = rs.item_cell;
+      it.off = nullptr;
+      fs_samples smp{sp->seed, 0, (uint32_t)r, n_items, sp->O, sp->S, 0, nullptr};
+      const Plan pl = make_plan(m, &smp, n_items);
+      FS_CUDA(launch_prep(set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, s), "launch prep");
+      FS_CUDA(launch_score(set, it, pl, (const float*)m->tables.p, (uint64_t*)m->sums.p, nullptr, 0, m->sm_count, s),
+              "launch score");
+      FS_CUDA(launch_replay_reveal(set, rs, it, pl, (const uint64_t*)m->sums.p, n_active, s), "launch reveal");
+    }
+    if (rounds) FS_CUDA(cudaMemcpyAsync(rounds, rs.rounds, 4 * (size_t)P, cudaMemcpyDeviceToHost, s), "read rounds");
+    if (state) FS_CUDA(cudaMemcpyAsync(state, rs.state, 4 * (size_t)P, cudaMemcpyDeviceToHost, s), "read state");
+    if (gpu_seconds)
+      FS_CUDA(cudaMemcpyAsync(gpu_seconds, rs.gpu_seconds, 8 * (size_t)P, cudaMemcpyDeviceToHost, s), "read gpu-s");
+    if (reveal_order)
+      FS_CUDA(cudaMemcpyAsync(reveal_order, rs.reveal_order, 4 * (size_t)P * cells, cudaMemcpyDeviceToHost, s),
+              "read order");
+    if (gamma_trace)
+      FS_CUDA(cudaMemcpyAsync(gamma_trace, rs.gamma_trace, 4 * (size_t)P * (sp->max_rounds + 1),
+                              cudaMemcpyDeviceToHost, s),
+              "read trace");
+    if (final_minus)
+      FS_CUDA(cudaMemcpyAsync(final_minus, rs.final_minus, sizeof(fs_allocation) * (size_t)P, cudaMemcpyDeviceToHost,
+                              s),
+              "read allocations");
+    return read_status(m, s);
+  };
+  rc = run();
+  cudaStreamSynchronize(s);
+  all.release();
+  return rc;
+}
+
+int fs_check(fs_model* m, void* cuda_stream) {
+  if (!m) return fail(FS_EINVAL, "model is NULL");
+  return read_status(m, cuda_stream ? (cudaStream_t)cuda_stream : m->stream);
+}
+
+int fs_timing_enable(fs_model* m, int32_t on) {
+  if (!m) return fail(FS_EINVAL, "model is NULL");
+  m->timing = on != 0;
+  m->ev_used = 0;
+  return FS_OK;
+}
+
+int fs_timing_read(fs_model* m, double* kernel_ms, int32_t* launches) {
+  if (!m) return fail(FS_EINVAL, "model is NULL");
+  double total = 0.0;
+  const size_t n = m->ev_used / 2;
+  for (size_t k = 0; k < n; ++k) {
+    FS_CUDA(cudaEventSynchronize(m->ev[2 * k + 1]), "wait timing event");
+    float ms = 0.0f;
+    FS_CUDA(cudaEventElapsedTime(&ms, m->ev[2 * k], m->ev[2 * k + 1]), "elapsed time");
+    total += ms;
+  }
+  m->ev_used = 0;
+  if (kernel_ms) *kernel_ms = total;
+  if (launches) *launches = (int32_t)n;
+  return FS_OK;
+}
+
+int fs_watchdog_selftest(int64_t timeout_ns) {
+  const int64_t t = std::min<int64_t>(std::max<int64_t>(timeout_ns, 1000000), 5000000000LL);
+  uint32_t* st = nullptr;
+  FS_CUDA(cudaMalloc(&st, 4), "watchdog status");
+  cudaError_t e = cudaMemset(st, 0, 4);
+  if (e == cudaSuccess) e = launch_watchdog(st, (uint64_t)t, nullptr);
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  uint32_t v = 0;
+  if (e == cudaSuccess) e = cudaMemcpy(&v, st, 4, cudaMemcpyDeviceToHost);
+  cudaFree(st);
+  if (e != cudaSuccess) return cuda_fail(e, "watchdog self-test");
+  if (v & ST_TIMEOUT) return fail(FS_ETIMEOUT, "watchdog: the barrier wait gave up after %lld ns", (long long)t);
+  return fail(FS_EDEVICE, "watchdog: the wait did not report a timeout (status 0x%x)", v);
+}
+
+void fs_free_model(fs_model* m) {
+  if (!m) return;
+  if (m->stream) cudaStreamSynchronize(m->stream);
+  else cudaDeviceSynchronize();
+  m->fixed.release();
+  m->cand.release();
+  m->tables.release();
+  m->sums.release();
+  m->outs.release();
+  m->real.release();
+  for (cudaEvent_t e : m->ev) cudaEventDestroy(e);
+  delete m;
+}
+
+}  // extern "C"

@@ -1,0 +1,229 @@
+// Internal device-side definitions of the decision-gap scorer (sm_103a).
+//
+// Layout of a problem set in HBM (all problems share K, B, G, SLOs, demands
+// and the quantile table; the replay batches one problem per reveal order):
+//   bounds   [P][4][cells] f32   rows CAP_LO, CAP_HI, TAIL_LO, TAIL_HI
+//   revealed [P][cells]    u8
+//   theta    [P][2][theta_cap] f32  sorted option fulfilments of the base
+//                                   realisation sigma (0 = A-, 1 = A+)
+//   ntheta   [P][2]        i32
+//   rowC     [P][2][K*4]   f32   best SLO-feasible capacity per (class, TP)
+//   rowB     [P][2][K*4]   i32   its bin (-1: none)
+//   base     [P][2]        fs_allocation
+// Per scoring call (items = (problem, candidate cell) pairs):
+//   tables   [items][2][slot_floats] f32   per-candidate threshold tables
+//   sums     [items][O]    u64 (int64 fixed point, 2^-40)
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "../../include/fleetsieve.h"
+
+namespace fs {
+
+constexpr int kT = 4;                 // TP degrees {1, 2, 4, 8}
+constexpr int kCostInf = 0x3FFFFFFF;  // "no option covers the threshold"
+constexpr int kSolveThreads = 256;
+constexpr int kPrepThreads = 128;
+constexpr int kScoreThreads = 256;
+constexpr int kTableHeader = 8;       // floats before the three table arrays
+constexpr int kSmemTableCap = 1024;   // table entries staged in shared memory per realisation
+
+enum : int { CAP_LO = 0, CAP_HI = 1, TAIL_LO = 2, TAIL_HI = 3 };
+
+// status word bits (device -> host)
+enum : uint32_t {
+  ST_TIMEOUT = 1u,       // a bounded mbarrier wait gave up
+  ST_THETA = 2u,         // threshold count above the model's capacity
+  ST_TABLE = 4u,         // candidate table longer than its slot
+  ST_CELL = 8u,          // a device-side candidate id outside [0, cells)
+};
+
+struct Dims {
+  int K, B, G, Q, cells, K4;
+  int M[kT];            // floor(G / tau)
+  int theta_cap;        // K * sum M: most thresholds one realisation can have
+  int slot_floats;      // stride of one (item, sigma) table
+  int lcap;             // table entries a slot can hold (multiple of 4)
+};
+
+struct Set {
+  Dims d;
+  int P;
+  const float* lam;     // [K]
+  const float* slo;     // [K]
+  const float* qn;      // [Q]
+  float* bounds;        // [P][4][cells]
+  uint8_t* revealed;    // [P][cells]
+  float* theta;         // [P][2][theta_cap]
+  int* ntheta;          // [P][2]
+  float* rowC;          // [P][2][K4]
+  int* rowB;            // [P][2][K4] bin of rowC, -1 = no SLO-feasible bin
+  fs_allocation* base;  // [P][2]
+  uint32_t* status;
+  const int* skip;      // [P] or nullptr: base solves skip problems with skip[p] >= 0
+};
+
+// Scenario plan shared by a launch.
+struct Plan {
+  uint32_t key0;        // low word of the seed
+  uint32_t key1;        // high word of the seed (stream id XORed per problem)
+  uint32_t stream_base; // stream id of problem 0 (problem p uses stream_base + p)
+  uint32_t round;
+  int O, S, W, w;       // W = Q / O quantiles per stratum, w = log2(W)
+  int pairs;            // ceil(S / 2) Philox calls per (candidate, outcome)
+  int ppt;              // Philox calls per thread per tile
+  int chunks;           // tiles per (candidate, outcome)
+};
+
+struct Items {
+  int n;
+  const int* p;         // [n] problem of the item, nullptr = all problem 0
+  const int* cell;      // [n] candidate cell
+  const int* off;       // [P + 1] item range of each problem (grouped by problem)
+};
+
+// ---------------------------------------------------------------- arithmetic
+
+// Fulfilment of n replicas of capacity c: min(1, (n c) / lambda), Section 3
+// (Eqs. 2 and 4, r_i = x_i / lambda_i). One IEEE rounding per step, no FMA.
+__device__ __forceinline__ float fulfil(float n, float c, float lam) {
+  float r = __fdiv_rn(__fmul_rn(n, c), lam);
+  return fminf(r, 1.0f);
+}
+
+// Smallest n in [1, M] with fulfil(n, c) >= t, or 0 if none (fulfil is
+// nondecreasing in n under round-to-nearest).
+__device__ __forceinline__ int min_replicas(float t, float c, float lam, int M) {
+  if (M < 1 || fulfil((float)M, c, lam) < t) return 0;
+  int lo = 1, hi = M;
+  while (lo < hi) {
+    int mid = (lo + hi) >> 1;
+    if (fulfil((float)mid, c, lam) >= t) hi = mid; else lo = mid + 1;
+  }
+  return lo;
+}
+
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11): ten rounds of the 4x32
+// S-box (two 32x32->64 products) with the Weyl key schedule.
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    const uint32_t hi0 = __umulhi(0xD2511F53u, c.x);
+    const uint32_t lo0 = 0xD2511F53u * c.x;
+    const uint32_t hi1 = __umulhi(0xCD9E8D57u, c.z);
+    const uint32_t lo1 = 0xCD9E8D57u * c.z;
+    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+    k0 += 0x9E3779B9u;
+    k1 += 0xBB67AE85u;
+  }
+  return c;
+}
+
+// lo + (hi - lo) q rounded step by step, clamped into [lo, hi]; d = hi - lo.
+__device__ __forceinline__ float map_into(float lo, float d, float hi, float q) {
+  float v = __fadd_rn(lo, __fmul_rn(d, q));
+  return fminf(fmaxf(v, lo), hi);
+}
+
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// ---------------------------------------------------------------- TMA bulk copy
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Global -> shared bulk copy (no tensor map, no multicast); dst, src and
+// bytes must be multiples of 16. Completion is counted on bar.
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// Bounded wait for phase `parity` of bar: true when it completed, false when
+// limit_ns elapsed (or an iteration cap was hit) first.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
+  const uint32_t a = smem_u32(bar);
+  const uint64_t t0 = global_ns();
+  for (uint32_t it = 0; it < (1u << 28); ++it) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(ok)
+        : "r"(a), "r"(parity)
+        : "memory");
+    if (ok) return true;
+    if ((it & 15u) == 15u && global_ns() - t0 > limit_ns) return false;
+  }
+  return false;
+}
+
+constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s
+
+// ---------------------------------------------------------------- launchers (host)
+
+void note_launch();
+cudaError_t launch_qtable(float* qn, int Q, cudaStream_t s);
+// Base or explicit realisations: realisation r of `n` reads cap/tail either
+// from the problem set's bounds (explicit == nullptr: r = 2 p + sigma) or from
+// cap_x / tail_x [n][cells].
+cudaError_t launch_solve(const Set& set, int n, const float* cap_x, const float* tail_x,
+                         fs_allocation* out, bool write_theta, cudaStream_t s);
+cudaError_t launch_prep(const Set& set, const Items& it, const Plan& pl, float* tables,
+                        uint64_t* sums, cudaStream_t s);
+cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const float* tables,
+                         uint64_t* sums, void* dump, int dump_stride, int sm_count, cudaStream_t s);
+cudaError_t launch_finalize(const Set& set, const Items& it, const Plan& pl, const uint64_t* sums,
+                            double* gap, double* score, float* gamma_t, int32_t* best, cudaStream_t s);
+cudaError_t launch_watchdog(uint32_t* status, uint64_t limit_ns, cudaStream_t s);
+
+// replay
+struct ReplayState {
+  const float* truth;     // [P][2][cells] cap, tail
+  const int* perm;        // [P][cells]
+  int* rounds;            // [P]
+  int* state;             // [P]  -1 running, 0 undecided stop, 1 certified
+  double* gpu_seconds;    // [P]
+  int* reveal_order;      // [P][cells]
+  int* n_revealed;        // [P]
+  float* gamma_trace;     // [P][max_rounds + 1]
+  fs_allocation* final_minus;  // [P]
+  int* active;            // [P] compact list of running problems
+  int* n_active;          // [1]
+  int* item_p;            // [P * cells]
+  int* item_cell;         // [P * cells]
+  int* item_off;          // [P + 1]
+  int max_rounds;
+  float eps;
+};
+cudaError_t launch_replay_init(const Set& set, const ReplayState& rs, int r0, cudaStream_t s);
+cudaError_t launch_replay_certify(const Set& set, const ReplayState& rs, int round, cudaStream_t s);
+cudaError_t launch_replay_items(const Set& set, const ReplayState& rs, int n_active, int per,
+                                cudaStream_t s);
+cudaError_t launch_replay_reveal(const Set& set, const ReplayState& rs, const Items& it,
+                                 const Plan& pl, const uint64_t* sums, int n_active, cudaStream_t s);
+
+}  // namespace fs

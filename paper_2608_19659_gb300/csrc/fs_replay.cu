@@ -1,0 +1,120 @@
+// Profiling loop (Algorithm 1) batched over many reveal orders, for sm_103a.
+//
+// Every stream k is one problem of the set: its own bounds, revealed flags
+// and hidden truth. A round runs, for all streams still going:
+//   A-, A+ (k_solve) -> certificate (Section 4.2) -> candidate list (the
+//   unrevealed cells in the stream's reveal order) -> k_prep / k_score
+//   (Section 4.3) -> argmax -> reveal (interval collapses to the truth).
+// The host only reads the number of streams still going once per round.
+#include <cuda_runtime.h>
+
+#include "fs_internal.cuh"
+#include "fs_finalize.cuh"
+
+namespace fs {
+
+__device__ __forceinline__ void reveal_cell(const Set& set, const ReplayState& rs, int p, int c) {
+  const Dims& d = set.d;
+  float* bp = set.bounds + (size_t)p * 4 * d.cells;
+  const float tc = rs.truth[((size_t)p * 2) * d.cells + c];
+  const float tl = rs.truth[((size_t)p * 2 + 1) * d.cells + c];
+  bp[(size_t)CAP_LO * d.cells + c] = tc;
+  bp[(size_t)CAP_HI * d.cells + c] = tc;
+  bp[(size_t)TAIL_LO * d.cells + c] = tl;
+  bp[(size_t)TAIL_HI * d.cells + c] = tl;
+  set.revealed[(size_t)p * d.cells + c] = 1;
+  const int q = rs.n_revealed[p]++;
+  rs.reveal_order[(size_t)p * d.cells + q] = c;
+  rs.gpu_seconds[p] += 300.0 * (double)(1 << ((c / d.B) & 3));  // 300 s per cell x TP GPUs
+}
+
+__global__ void k_replay_init(Set set, ReplayState rs, int r0) {
+  const int p = blockIdx.x * blockDim.x + threadIdx.x;
+  if (p >= set.P) return;
+  rs.n_revealed[p] = 0;
+  rs.gpu_seconds[p] = 0.0;
+  rs.rounds[p] = 0;
+  rs.state[p] = -1;
+  for (int q = 0; q < set.d.cells; ++q) rs.reveal_order[(size_t)p * set.d.cells + q] = -1;
+  for (int q = 0; q < r0; ++q) reveal_cell(set, rs, p, rs.perm[(size_t)p * set.d.cells + q]);
+}
+
+// Certificate of every running stream; collects the ones that go on.
+__global__ void k_replay_certify(Set set, ReplayState rs, int round) {
+  const int p = blockIdx.x * blockDim.x + threadIdx.x;
+  if (p >= set.P || rs.state[p] >= 0) return;
+  const Dims& d = set.d;
+  const fs_allocation& am = set.base[2 * p];
+  const fs_allocation& ap = set.base[2 * p + 1];
+  const float gt = __fsub_rn(ap.t_star, am.t_star);
+  rs.gamma_trace[(size_t)p * (rs.max_rounds + 1) + round] = gt;
+  bool known = true;
+  for (int i = 0; i < d.K; ++i) {
+    if (am.replicas[i] <= 0) continue;
+    const int j = __ffs(am.tp[i]) - 1;
+    const int c = (i * 4 + j) * d.B + am.bin[i];
+    if (!set.revealed[(size_t)p * d.cells + c]) known = false;
+  }
+  int st = -1;
+  if (gt <= rs.eps && known) st = 1;
+  else if (round >= rs.max_rounds || rs.n_revealed[p] >= d.cells) st = 0;
+  if (st >= 0) {
+    rs.state[p] = st;
+    rs.rounds[p] = round;
+    rs.final_minus[p] = am;
+  } else {
+    rs.active[atomicAdd(rs.n_active, 1)] = p;
+  }
+}
+
+// Candidates of running stream slot a: its unrevealed cells in reveal order.
+__global__ void k_replay_items(Set set, ReplayState rs, int n_active, int per) {
+  const int a = blockIdx.x * blockDim.x + threadIdx.x;
+  if (a >= n_active) return;
+  const int p = rs.active[a];
+  const Dims& d = set.d;
+  int q = 0;
+  for (int k = 0; k < d.cells && q < per; ++k) {
+    const int c = rs.perm[(size_t)p * d.cells + k];
+    if (!set.revealed[(size_t)p * d.cells + c]) {
+      rs.item_p[a * per + q] = p;
+      rs.item_cell[a * per + q] = c;
+      ++q;
+    }
+  }
+  if (q != per) atomicOr(set.status, ST_TABLE);
+}
+
+__global__ void k_replay_reveal(Set set, ReplayState rs, Items it, Plan pl, const uint64_t* sums, int per) {
+  const int a = blockIdx.x;
+  const int p = rs.active[a];
+  const Best b = finalize_problem(set, it, pl, sums, p, a * per, (a + 1) * per, nullptr, nullptr, nullptr);
+  if (threadIdx.x == 0 && b.pos >= 0) reveal_cell(set, rs, p, it.cell[a * per + b.pos]);
+}
+
+cudaError_t launch_replay_init(const Set& set, const ReplayState& rs, int r0, cudaStream_t s) {
+  note_launch();
+  k_replay_init<<<(set.P + 127) / 128, 128, 0, s>>>(set, rs, r0);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_replay_certify(const Set& set, const ReplayState& rs, int round, cudaStream_t s) {
+  note_launch();
+  k_replay_certify<<<(set.P + 127) / 128, 128, 0, s>>>(set, rs, round);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_replay_items(const Set& set, const ReplayState& rs, int n_active, int per, cudaStream_t s) {
+  note_launch();
+  k_replay_items<<<(n_active + 127) / 128, 128, 0, s>>>(set, rs, n_active, per);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_replay_reveal(const Set& set, const ReplayState& rs, const Items& it, const Plan& pl,
+                                 const uint64_t* sums, int n_active, cudaStream_t s) {
+  note_launch();
+  k_replay_reveal<<<n_active, 256, 0, s>>>(set, rs, it, pl, sums, it.n / n_active);
+  return cudaGetLastError();
+}
+
+}  // namespace fs

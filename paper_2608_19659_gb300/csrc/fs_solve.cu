@@ -1,0 +1,308 @@
+// Allocation solver (Section 3, Eqs. 1-5; tier 2 of the objective) and the
+// quantile table, for sm_103a.
+//
+// One CTA solves one realisation (a capacity and a tail value per cell):
+//   1. rows: for every (class i, TP index j) the best SLO-feasible bin
+//      (largest capacity, then lowest bin; Eq. 5 gates l <= L_i) -> C_ij;
+//   2. thresholds: the positive fulfilments f(n, C_ij), n = 1..floor(G/tau_j)
+//      (cut at the first n with f = 1), written to shared memory and
+//      bitonic-sorted;
+//   3. search: the largest threshold t whose cheapest per-class covers fit in
+//      G. Each probe is one warp: lanes hold rows, shuffles take the per-class
+//      minimum over the four TP lanes, a ballot flags classes with no cover,
+//      and a warp reduction sums the GPUs. The CTA's eight warps probe eight
+//      points per step (a 9-ary search);
+//   4. choice at t*: per class the cheapest cover, ties to the lower TP.
+// For a fixed (TP, n) a larger capacity never lowers f, so the best bin of
+// each row is the option the tie rule (larger capacity, then lower bin)
+// picks; and t* is the largest threshold t of the rows' values at which the
+// total fits, as cost(t) is constant between consecutive thresholds.
+#include <cuda_runtime.h>
+
+#include "fs_internal.cuh"
+
+namespace fs {
+
+__global__ void k_qtable(float* qn, int Q) {
+  const int k = blockIdx.x * blockDim.x + threadIdx.x;
+  if (k >= Q) return;
+  // Inverse CDF of the symmetric triangular law on [0, 1] at u = (k + 1/2) / Q:
+  // 2x^2 = u below 1/2, 1 - 2(1-x)^2 = u above.
+  const float u = __fdiv_rn(__fadd_rn(__int2float_rn(k), 0.5f), __int2float_rn(Q));
+  float x;
+  if (u < 0.5f) {
+    x = __fsqrt_rn(__fmul_rn(u, 0.5f));
+  } else {
+    x = __fsub_rn(1.0f, __fsqrt_rn(__fmul_rn(__fsub_rn(1.0f, u), 0.5f)));
+  }
+  qn[k] = x;
+}
+
+// Total GPUs of the cheapest per-class covers of threshold t, or kCostInf if
+// some class has no cover. Called by a whole warp; rows rho = 4 i + j.
+__device__ __forceinline__ int warp_total_cost(float t, const float* sC, const float* lam,
+                                               const Dims& d, int lane) {
+  int total = 0;
+  bool inf = false;
+  for (int base = 0; base < d.K4; base += 32) {
+    const int rho = base + lane;
+    int cost = kCostInf;
+    if (rho < d.K4) {
+      const int j = rho & 3;
+      const int n = min_replicas(t, sC[rho], lam[rho >> 2], d.M[j]);
+      if (n) cost = n << j;
+    }
+    cost = min(cost, __shfl_xor_sync(0xffffffffu, cost, 1));
+    cost = min(cost, __shfl_xor_sync(0xffffffffu, cost, 2));
+    const bool head = rho < d.K4 && (lane & 3) == 0;
+    if (__ballot_sync(0xffffffffu, head && cost >= kCostInf)) inf = true;
+    total += __reduce_add_sync(0xffffffffu, (head && cost < kCostInf) ? cost : 0);
+  }
+  return inf ? kCostInf : total;
+}
+
+__global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, const float* cap_x,
+                                                         const float* tail_x, fs_allocation* out_x,
+                                                         int write_theta) {
+  extern __shared__ __align__(16) unsigned char smraw[];
+  const Dims d = set.d;
+  const int r = blockIdx.x;
+  if (r >= n_real) return;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = blockDim.x >> 5;
+
+  const float* cap;
+  const float* tail;
+  int p = 0, sigma = 0;
+  fs_allocation* out;
+  if (cap_x) {
+    cap = cap_x + (size_t)r * d.cells;
+    tail = tail_x + (size_t)r * d.cells;
+    out = out_x + r;
+  } else {
+    p = r >> 1;
+    sigma = r & 1;
+    if (set.skip && set.skip[p] >= 0) return;
+    const float* bp = set.bounds + (size_t)p * 4 * d.cells;
+    cap = bp + (size_t)(sigma ? CAP_HI : CAP_LO) * d.cells;
+    tail = bp + (size_t)(sigma ? TAIL_LO : TAIL_HI) * d.cells;
+    out = set.base + r;
+  }
+
+  float* sC = reinterpret_cast<float*>(smraw);          // [256]
+  int* sB = reinterpret_cast<int*>(sC + 256);             // [256]
+  int* sN0 = sB + 256;                                    // [256]
+  int* sOff = sN0 + 256;                                  // [260]
+  int* sProbe = sOff + 260;                               // [32]
+  int* sMisc = sProbe + 32;                               // [8]
+  float* sTheta = reinterpret_cast<float*>(sMisc + 8);    // [pow2 >= theta_cap]
+
+  // 1. rows
+  for (int rho = tid; rho < d.K4; rho += blockDim.x) {
+    const int i = rho >> 2, j = rho & 3;
+    const float L = set.slo[i];
+    const float* cr = cap + (size_t)rho * d.B;
+    const float* tr = tail + (size_t)rho * d.B;
+    float best = 0.0f;
+    int bb = -1;
+    for (int b = 0; b < d.B; ++b) {
+      if (tr[b] <= L) {
+        const float c = cr[b];
+        if (bb < 0 || c > best) {
+          best = c;
+          bb = b;
+        }
+      }
+    }
+    sC[rho] = bb >= 0 ? best : 0.0f;
+    sB[rho] = bb;
+    const float lam = set.lam[i];
+    const int M = d.M[j];
+    int n0 = 0, len = 0;
+    if (bb >= 0 && M >= 1) {
+      n0 = min_replicas(__int_as_float(1), best, lam, M);  // first positive fulfilment
+      if (n0) {
+        const int ns = min_replicas(1.0f, best, lam, M);   // first full fulfilment
+        len = ns ? ns : M;
+      }
+    }
+    sN0[rho] = n0;
+    sOff[rho] = n0 ? len - n0 + 1 : 0;  // count, scanned below
+  }
+  __syncthreads();
+  if (tid == 0) {
+    int acc = 0;
+    for (int rho = 0; rho < d.K4; ++rho) {
+      const int c = sOff[rho];
+      sOff[rho] = acc;
+      acc += c;
+    }
+    sOff[d.K4] = acc;
+    uint32_t mask_lo = 0, mask_hi = 0;
+    for (int rho = 0; rho < d.K4; ++rho)
+      if (sB[rho] >= 0) {
+        const int i = rho >> 2;
+        if (i < 32) mask_lo |= 1u << i; else mask_hi |= 1u << (i - 32);
+      }
+    sMisc[2] = (int)mask_lo;
+    sMisc[3] = (int)mask_hi;
+  }
+  __syncthreads();
+  int total = sOff[d.K4];
+  if (total > d.theta_cap) {  // cannot happen: a row holds at most floor(G/tau) values
+    if (tid == 0) atomicOr(set.status, ST_THETA);
+    total = d.theta_cap;
+  }
+  int P2 = 1;
+  while (P2 < total) P2 <<= 1;
+
+  // 2. thresholds, then bitonic sort (ascending, +inf padding)
+  for (int x = tid; x < P2; x += blockDim.x) {
+    float v = __int_as_float(0x7f800000);
+    if (x < total) {
+      int lo = 0, hi = d.K4 - 1;
+      while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (sOff[mid] <= x) lo = mid; else hi = mid - 1;
+      }
+      const int n = sN0[lo] + (x - sOff[lo]);
+      v = fulfil((float)n, sC[lo], set.lam[lo >> 2]);
+    }
+    sTheta[x] = v;
+  }
+  __syncthreads();
+  for (int k = 2; k <= P2; k <<= 1) {
+    for (int jj = k >> 1; jj > 0; jj >>= 1) {
+      for (int x = tid; x < P2; x += blockDim.x) {
+        const int y = x ^ jj;
+        if (y > x) {
+          const float a = sTheta[x], b = sTheta[y];
+          const bool up = (x & k) == 0;
+          if ((a > b) == up && a != b) {
+            sTheta[x] = b;
+            sTheta[y] = a;
+          }
+        }
+      }
+      __syncthreads();
+    }
+  }
+
+  // 3. search: largest index whose threshold fits in G (lo feasible, hi not)
+  if (tid == 0) {
+    sMisc[0] = -1;
+    sMisc[1] = total;
+    sMisc[4] = 0;
+  }
+  __syncthreads();
+  while (sMisc[1] - sMisc[0] > 1) {
+    const int lo = sMisc[0], hi = sMisc[1];
+    const int span = hi - lo;
+    int kp = lo + (int)(((long long)(warp + 1) * span) / (nwarp + 1));
+    kp = max(lo + 1, min(hi - 1, kp));
+    const int cost = warp_total_cost(sTheta[kp], sC, set.lam, d, lane);
+    if (lane == 0) sProbe[warp] = (cost <= d.G) ? kp : -(kp + 1);
+    __syncthreads();
+    if (tid == 0) {
+      int nlo = lo, nhi = hi;
+      for (int w = 0; w < nwarp; ++w) {
+        const int v = sProbe[w];
+        if (v >= 0) nlo = max(nlo, v); else nhi = min(nhi, -v - 1);
+      }
+      sMisc[0] = nlo;
+      sMisc[1] = nhi;
+    }
+    __syncthreads();
+  }
+  const int kstar = sMisc[0];
+  const float tstar = kstar >= 0 ? sTheta[kstar] : 0.0f;
+
+  // 4. choice at t*
+  if (tid < FS_MAX_CLASSES) {
+    const int i = tid;
+    int8_t tp = 0;
+    int16_t bin = -1, reps = 0;
+    float f = 0.0f;
+    int cost_i = 0;
+    if (i < d.K && tstar > 0.0f) {
+      int best = kCostInf, bj = -1, bn = 0;
+      for (int j = 0; j < kT; ++j) {
+        const int n = min_replicas(tstar, sC[4 * i + j], set.lam[i], d.M[j]);
+        if (n && (n << j) < best) {
+          best = n << j;
+          bj = j;
+          bn = n;
+        }
+      }
+      tp = (int8_t)(1 << bj);
+      bin = (int16_t)sB[4 * i + bj];
+      reps = (int16_t)bn;
+      f = fulfil((float)bn, sC[4 * i + bj], set.lam[i]);
+      cost_i = best;
+    }
+    out->tp[i] = tp;
+    out->bin[i] = bin;
+    out->replicas[i] = reps;
+    out->fulfil[i] = f;
+    if (i < d.K) atomicAdd(&sMisc[4], cost_i);
+  }
+  __syncthreads();
+  if (tid == 0) {
+    out->t_star = tstar;
+    out->total_gpus = tstar > 0.0f ? sMisc[4] : 0;
+    out->has_option_mask = (uint64_t)(uint32_t)sMisc[2] | ((uint64_t)(uint32_t)sMisc[3] << 32);
+    out->ok = tstar > 0.0f ? 1 : 0;
+    out->reserved = 0;
+  }
+  if (write_theta && !cap_x) {
+    float* th = set.theta + ((size_t)p * 2 + sigma) * d.theta_cap;
+    for (int x = tid; x < total; x += blockDim.x) th[x] = sTheta[x];
+    float* rc = set.rowC + ((size_t)p * 2 + sigma) * d.K4;
+    int* rb = set.rowB + ((size_t)p * 2 + sigma) * d.K4;
+    for (int rho = tid; rho < d.K4; rho += blockDim.x) {
+      rc[rho] = sC[rho];
+      rb[rho] = sB[rho];
+    }
+    if (tid == 0) set.ntheta[p * 2 + sigma] = total;
+  }
+}
+
+// Watchdog self-test: wait on a barrier phase that nothing completes; the
+// bounded wait gives up, records the timeout and the kernel returns.
+__global__ void k_watchdog(uint32_t* status, uint64_t limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x == 0) mbar_init(&bar, 1);
+  __syncthreads();
+  const bool ok = mbar_wait(&bar, 0u, limit_ns);
+  if (!ok && threadIdx.x == 0) atomicOr(status, ST_TIMEOUT);
+}
+
+cudaError_t launch_watchdog(uint32_t* status, uint64_t limit_ns, cudaStream_t s) {
+  note_launch();
+  k_watchdog<<<1, 32, 0, s>>>(status, limit_ns);
+  return cudaGetLastError();
+}
+
+size_t solve_smem_bytes(const Dims& d) {
+  int P2 = 1;
+  while (P2 < d.theta_cap) P2 <<= 1;
+  return (size_t)(256 * 3 + 260 + 32 + 8) * 4 + (size_t)P2 * 4;
+}
+
+cudaError_t launch_qtable(float* qn, int Q, cudaStream_t s) {
+  note_launch();
+  k_qtable<<<(Q + 255) / 256, 256, 0, s>>>(qn, Q);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_solve(const Set& set, int n, const float* cap_x, const float* tail_x,
+                         fs_allocation* out, bool write_theta, cudaStream_t s) {
+  if (n <= 0) return cudaSuccess;
+  const size_t smem = solve_smem_bytes(set.d);
+  cudaError_t e = cudaFuncSetAttribute(k_solve, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  note_launch();
+  k_solve<<<n, kSolveThreads, smem, s>>>(set, n, cap_x, tail_x, out, write_theta ? 1 : 0);
+  return cudaGetLastError();
+}
+
+}  // namespace fs

@@ -30,3 +30,39 @@ def oracle_lib():
 
     oracle.lib()
     return oracle
+
+
+@pytest.fixture(scope="session")
+def fsb():
+    """The ctypes binding of the CUDA library (built in-tree first)."""
+    from paper_2608_19659_gb300 import _build
+
+    _build.build()
+    from paper_2608_19659_gb300 import fleetsieve
+
+    fleetsieve.lib()
+    return fleetsieve
+
+
+@pytest.fixture(scope="session")
+def cuda():
+    import torch
+
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    torch.cuda.set_device(0)
+    return torch
+
+
+def load_model(fsb, w, quantile=None):
+    return fsb.fs_load_model(w.cap_lo, w.cap_hi, w.tail_lo, w.tail_hi, w.slo, w.demand, w.G, w.K, w.B,
+                             quantile=quantile)
+
+
+def alloc_matches(gpu: dict, ref, K: int) -> bool:
+    """GPU allocation dict equals an oracle Allocation field by field (bit-exact floats)."""
+    import numpy as np
+
+    return (gpu["t_star"] == ref.t_star and gpu["total_gpus"] == ref.total_gpus and gpu["ok"] == ref.ok
+            and gpu["has_option_mask"] == ref.has_option_mask and gpu["tp"] == ref.tp
+            and gpu["bin"] == ref.bin and gpu["replicas"] == ref.replicas
+            and [np.float32(x) for x in gpu["fulfil"]] == [np.float32(x) for x in ref.fulfil])

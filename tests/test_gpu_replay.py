@@ -1,0 +1,81 @@
+"""Batched profiling loop (fs_replay, Algorithm 1) against the oracle's per-stream replay."""
+
+import numpy as np
+import pytest
+
+from conftest import load_model
+from paper_2608_19659_gb300 import workloads
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def qn(oracle_lib):
+    return oracle_lib.triangular_table(4096)
+
+
+def _gpu_replay(fsb, rp, S, seed, max_rounds=None):
+    w = rp.base
+    mr = rp.max_rounds if max_rounds is None else max_rounds
+    with load_model(fsb, w) as m:
+        return fsb.fs_replay(m, rp.truth_cap, rp.truth_tail, rp.perm, rp.r0, rp.eps, w.O, S, seed, mr)
+
+
+def _compare(fsb, res, rp, k, ref, K):
+    assert res.rounds[k] == ref.rounds and res.state[k] == ref.state
+    assert res.gpu_seconds[k] == ref.gpu_seconds
+    n = len(ref.reveal_order)
+    assert np.array_equal(res.reveal_order[k][:n], ref.reveal_order)
+    assert np.all(res.reveal_order[k][n:] == -1)
+    assert np.array_equal(res.gamma_trace[k][: ref.rounds + 1], ref.gamma_trace)
+    f = res.final_minus[k]
+    a = ref.final_minus
+    assert float(f["t_star"]) == a.t_star and int(f["total_gpus"]) == a.total_gpus
+    assert [int(x) for x in f["tp"][:K]] == a.tp and [int(x) for x in f["bin"][:K]] == a.bin
+    assert [int(x) for x in f["replicas"][:K]] == a.replicas
+
+
+def test_replay_small_samples_matches_oracle(fsb, cuda, oracle_lib, qn):
+    rp = workloads.make_replay(n_streams=12)
+    res = _gpu_replay(fsb, rp, S=32, seed=2026)
+    for k in range(12):
+        ref = oracle_lib.replay_stream(rp, k, qn, seed=2026, S=32)
+        _compare(fsb, res, rp, k, ref, rp.base.K)
+
+
+def test_replay_round_cap_and_full_initial_design(fsb, cuda, oracle_lib, qn):
+    import dataclasses
+
+    rp = dataclasses.replace(workloads.make_replay(n_streams=3), eps=-1.0)
+    res = _gpu_replay(fsb, rp, S=8, seed=1, max_rounds=4)
+    for k in range(3):
+        ref = oracle_lib.replay_stream(rp, k, qn, seed=1, S=8, max_rounds=4)
+        assert res.rounds[k] == 4 and res.state[k] == 0
+        _compare(fsb, res, rp, k, ref, rp.base.K)
+    full = dataclasses.replace(workloads.make_replay(n_streams=2), r0=64)
+    res = _gpu_replay(fsb, full, S=8, seed=1)
+    assert np.all(res.rounds == 0) and np.all(res.state == 1) and np.all(res.gamma_trace[:, 0] == 0)
+
+
+def test_replay_full_size(fsb, cuda, oracle_lib, qn):
+    """200 reveal orders x (unrevealed x 8 x 4096) per round; stream 0 replayed by the oracle in full."""
+    rp = workloads.make_replay()
+    res = _gpu_replay(fsb, rp, S=4096, seed=2026)
+    assert np.all(res.state == 1)
+    for k in range(200):
+        tr = res.gamma_trace[k][: res.rounds[k] + 1]
+        assert np.all(np.diff(tr) <= 0) and tr[-1] <= rp.eps
+    ref = oracle_lib.replay_stream(rp, 0, qn, seed=2026, S=4096)
+    _compare(fsb, res, rp, 0, ref, rp.base.K)
+
+
+def test_replay_rejects_bad_specs(fsb, cuda):
+    rp = workloads.make_replay(n_streams=2)
+    bad = rp.perm.copy()
+    bad[1, 3] = bad[1, 4]
+    w = rp.base
+    with load_model(fsb, w) as m:
+        with pytest.raises(fsb.FleetSieveError):
+            fsb.fs_replay(m, rp.truth_cap, rp.truth_tail, bad, 6, 0.01, 8, 16, 1, 64)
+        with pytest.raises(fsb.FleetSieveError):
+            fsb.fs_replay(m, rp.truth_cap, rp.truth_tail, rp.perm, 6, 0.01, 3, 16, 1, 64)
