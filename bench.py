@@ -275,7 +275,7 @@ def main(argv=None):
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     fsb.fs_timing_read(model)
-    fsb.fs_timing_enable(model, True)
+    fsb.fs_timing_enable(model, 1)
     if dist is not None:
         dist.barrier()
     torch.cuda.synchronize()
@@ -291,8 +291,8 @@ def main(argv=None):
     if dist is not None:
         dist.barrier()
     fsb.fs_check(model, stream)
-    kernel_ms, kernel_n = fsb.fs_timing_read(model)
-    fsb.fs_timing_enable(model, False)
+    kernel_ms, kernel_n, _ = fsb.fs_timing_read(model)
+    fsb.fs_timing_enable(model, 0)
     step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     total_ms = max_over_ranks(dist, sum(step_ms), dev)
     scen_all = sum_over_ranks(dist, float(w.scenarios) * args.steps, dev)

@@ -103,12 +103,13 @@ int fs_update_bounds(fs_model *m, const float *cap_lo, const float *cap_hi,
  *   cand[n_cand]: candidate cell ids (host pointer for fs_score_candidates,
  *     device pointer for fs_score_candidates_async); duplicates allowed;
  *     revealed cells are allowed and score 0.
- *   O: outcome strata, a power of two dividing Q; S >= 1 samples per
- *     (candidate, outcome); O * S <= 2^22.
+ *   O: outcome strata, a power of two dividing Q with Q/O <= 16384; S >= 1
+ *     samples per (candidate, outcome); O * S <= 2^22.
  *   Draws: Philox4x32-10 (Salmon et al., SC'11) with key (seed_lo,
- *     seed_hi XOR stream_id) and counter (s/2, o, cell, round); sample s uses
- *     words 2(s&1) (capacity) and 2(s&1)+1 (tail); the top log2(Q/O) bits pick
- *     a quantile inside stratum o.
+ *     seed_hi XOR stream_id) and counter (s/4, o, cell, round); sample s uses
+ *     output word s mod 4, whose upper 16 bits give the capacity and lower 16
+ *     bits the tail: the top log2(Q/O) bits of each half pick a quantile inside
+ *     stratum o.
  */
 typedef struct {
     uint64_t seed;
@@ -245,14 +246,18 @@ int fs_replay(fs_model *m, const fs_replay_spec *spec, int32_t *rounds, int32_t 
 int fs_check(fs_model *m, void *cuda_stream);
 
 /*
- * Kernel timing for measurement. With on != 0, every later scoring call of
- * this model records a pair of CUDA events around its Monte-Carlo kernel on
- * the stream it launches on (up to 4096 pairs are kept). fs_timing_read waits
- * for the recorded events, returns the summed kernel time (ms) and the number
- * of timed launches, and clears the record. Not part of the method.
+ * Kernel timing for measurement (not part of the method). mode 1: every
+ * later scoring call of this model records CUDA events around its
+ * Monte-Carlo kernel on the stream it launches on; mode 2: also around the
+ * base solves, the table preparation and the reduction; 0: off (up to 4096
+ * calls are kept). fs_timing_read waits for the recorded events and returns
+ * the summed Monte-Carlo kernel time (ms), the number of timed calls and,
+ * in mode 2, phase_ms[4] = summed (solve, prep, Monte-Carlo, reduction) time
+ * (nullable); it clears the record. Events between kernels also stop the
+ * next kernel from starting early, so timed calls can take a little longer.
  */
-int fs_timing_enable(fs_model *m, int32_t on);
-int fs_timing_read(fs_model *m, double *kernel_ms, int32_t *launches);
+int fs_timing_enable(fs_model *m, int32_t mode);
+int fs_timing_read(fs_model *m, double *kernel_ms, int32_t *launches, double *phase_ms);
 
 /* Kernels this library has launched since it was loaded (all models). */
 uint64_t fs_launch_count(void);

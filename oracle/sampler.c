@@ -74,11 +74,12 @@ static int ilog2_exact(int x)
 }
 
 /*
- * Quantile indices of scenario (cell, o, s). One Philox call serves two
- * consecutive samples: counter (s/2, o, cell, round), key (seed_lo,
- * seed_hi XOR stream_id); sample s takes words 2(s&1) (capacity) and
- * 2(s&1)+1 (tail). The top log2(Q/O) bits pick the position inside the
- * outcome stratum [o Q/O, (o+1) Q/O).
+ * Quantile indices of scenario (cell, o, s). One Philox call serves four
+ * consecutive samples: counter (s/4, o, cell, round), key (seed_lo,
+ * seed_hi XOR stream_id); sample s takes output word s mod 4. Its upper 16
+ * bits give the capacity position and its lower 16 bits the tail position:
+ * the top log2(Q/O) bits of each half pick the position inside the outcome
+ * stratum [o Q/O, (o+1) Q/O) (Q/O at most 2^16).
  */
 int or_draw_index(uint64_t seed, uint32_t stream_id, uint32_t round, int32_t cell,
                   int Q, int O, int o, int s, int32_t *k_cap, int32_t *k_tail)
@@ -86,17 +87,16 @@ int or_draw_index(uint64_t seed, uint32_t stream_id, uint32_t round, int32_t cel
     if (Q < 1 || O < 1 || Q % O != 0) return -1;
     int W = Q / O;
     int w = ilog2_exact(W);
-    if (w < 0 || o < 0 || o >= O || s < 0) return -1;
-    uint32_t ctr[4] = {(uint32_t)s >> 1, (uint32_t)o, (uint32_t)cell, round};
+    if (w < 0 || w > 16 || o < 0 || o >= O || s < 0) return -1;
+    uint32_t ctr[4] = {(uint32_t)s >> 2, (uint32_t)o, (uint32_t)cell, round};
     uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32) ^ stream_id};
     uint32_t x[4];
     or_philox4x32_10(ctr, key, x);
-    uint32_t xc = x[2 * (s & 1)];
-    uint32_t xl = x[2 * (s & 1) + 1];
-    int32_t off_c = w ? (int32_t)(xc >> (32 - w)) : 0;
-    int32_t off_l = w ? (int32_t)(xl >> (32 - w)) : 0;
-    *k_cap = o * W + off_c;
-    *k_tail = o * W + off_l;
+    uint32_t word = x[s & 3];
+    uint32_t hi16 = word >> 16;
+    uint32_t lo16 = word & 0xFFFFu;
+    *k_cap = o * W + (int32_t)(hi16 >> (16 - w));
+    *k_tail = o * W + (int32_t)(lo16 >> (16 - w));
     return 0;
 }
 

@@ -93,9 +93,11 @@ struct fs_model {
   std::vector<float> h_bounds;      // [4][cells]
   std::vector<uint8_t> h_revealed;  // [cells]
   std::vector<float> h_lam, h_slo;
-  // optional event pairs around the Monte-Carlo kernel
-  bool timing = false;
-  std::vector<cudaEvent_t> ev;      // 2 per timed launch
+  LaunchCache lc;
+  // optional timing events: 5 per timed call (before solve, prep, score,
+  // finalize, and after finalize); mode 1 records only the two around score
+  int timing = 0;
+  std::vector<cudaEvent_t> ev;
   size_t ev_used = 0;
 };
 
@@ -103,7 +105,7 @@ namespace {
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-constexpr size_t kMaxTimedEvents = 2 * 4096;
+constexpr size_t kMaxTimedEvents = 5 * 4096;
 
 int check_cells(const float* a, int n, const char* name) {
   if (!a) return fail(FS_EINVAL, "%s is NULL", name);
@@ -156,6 +158,7 @@ int check_samples(const fs_model* m, const fs_samples* s, bool host_cand) {
   if (s->n_cand < 0) return fail(FS_EINVAL, "n_cand < 0");
   if (s->n_cand > 0 && !s->cand) return fail(FS_EINVAL, "cand is NULL");
   if (!is_pow2(s->O) || s->O > m->d.Q) return fail(FS_EINVAL, "O = %d must be a power of two <= Q = %d", s->O, m->d.Q);
+  if (m->d.Q / s->O > 16384) return fail(FS_EINVAL, "Q / O = %d exceeds 16384 quantiles per stratum", m->d.Q / s->O);
   if (s->S < 1) return fail(FS_EINVAL, "S = %d < 1", s->S);
   if ((long long)s->O * s->S > FS_MAX_SAMPLES_PER_CAND) return fail(FS_EINVAL, "O * S exceeds 2^22");
   if ((long long)s->n_cand * s->O > (1LL << 30)) return fail(FS_EINVAL, "n_cand * O too large");
@@ -175,14 +178,9 @@ Plan make_plan(const fs_model* m, const fs_samples* s, int n_items) {
   pl.S = s->S;
   pl.W = m->d.Q / s->O;
   pl.w = log2i(pl.W);
-  pl.pairs = (s->S + 1) / 2;
-  const long long all_pairs = (long long)n_items * s->O * pl.pairs;
-  const long long slots = (long long)m->sm_count * 2048 * 2;  // two waves of resident threads
-  long long ppt = (all_pairs + slots - 1) / std::max<long long>(slots, 1);
-  ppt = std::min<long long>(std::max<long long>(ppt, 1), 16);
-  pl.ppt = (int)ppt;
-  const long long per_tile = (long long)kScoreThreads * pl.ppt;
-  pl.chunks = (int)((pl.pairs + per_tile - 1) / per_tile);
+  pl.sh = 16 - pl.w;
+  pl.calls = (s->S + 3) / 4;
+  (void)n_items;
   return pl;
 }
 
@@ -205,26 +203,30 @@ int run_score(fs_model* m, const fs_samples* smp, const int32_t* cand_dev, doubl
   it.cell = cand_dev;
   it.off = nullptr;
   const Plan pl = make_plan(m, smp, n);
-  FS_CUDA(launch_solve(m->set, 2, nullptr, nullptr, nullptr, true, s), "launch solve");
-  FS_CUDA(launch_prep(m->set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, s), "launch prep");
-  const bool timed = m->timing && n > 0 && m->ev_used + 2 <= kMaxTimedEvents;
+  const bool timed = m->timing && n > 0 && m->ev_used + 5 <= kMaxTimedEvents;
+  cudaEvent_t* ev = nullptr;
   if (timed) {
-    while (m->ev.size() < m->ev_used + 2) {
+    while (m->ev.size() < m->ev_used + 5) {
       cudaEvent_t e;
       FS_CUDA(cudaEventCreate(&e), "create timing event");
       m->ev.push_back(e);
     }
-    FS_CUDA(cudaEventRecord(m->ev[m->ev_used], s), "record timing event");
+    ev = &m->ev[m->ev_used];
+    m->ev_used += 5;
   }
+  const bool phases = timed && m->timing == 2;
+  if (phases) FS_CUDA(cudaEventRecord(ev[0], s), "record timing event");
+  FS_CUDA(launch_solve(m->set, 2, nullptr, nullptr, nullptr, true, m->lc, s), "launch solve");
+  if (phases) FS_CUDA(cudaEventRecord(ev[1], s), "record timing event");
+  FS_CUDA(launch_prep(m->set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, m->lc, s), "launch prep");
+  if (timed) FS_CUDA(cudaEventRecord(ev[2], s), "record timing event");
   FS_CUDA(launch_score(m->set, it, pl, (const float*)m->tables.p, (uint64_t*)m->sums.p, dump,
-                       fs_dump_stride(m), m->sm_count, s),
+                       fs_dump_stride(m), m->sm_count, m->lc, s),
           "launch score");
-  if (timed) {
-    FS_CUDA(cudaEventRecord(m->ev[m->ev_used + 1], s), "record timing event");
-    m->ev_used += 2;
-  }
+  if (timed) FS_CUDA(cudaEventRecord(ev[3], s), "record timing event");
   FS_CUDA(launch_finalize(m->set, it, pl, (const uint64_t*)m->sums.p, gap, score, gamma_t, best, s),
           "launch finalize");
+  if (phases) FS_CUDA(cudaEventRecord(ev[4], s), "record timing event");
   return FS_OK;
 }
 
@@ -288,7 +290,8 @@ int fs_load_model(const fs_bounds* b, const float* slo, const float* demand, int
   d.K4 = 4 * K;
   for (int j = 0; j < kT; ++j) d.M[j] = G >> j;
   d.theta_cap = (int)theta_cap;
-  d.lcap = (d.theta_cap + 3) & ~3;
+  d.lcap = 4;
+  while (d.lcap < d.theta_cap + 1) d.lcap <<= 1;
   d.slot_floats = kTableHeader + 3 * d.lcap;
 
   // fixed device state, one allocation carved into 256-byte aligned pieces
@@ -302,7 +305,7 @@ int fs_load_model(const fs_bounds* b, const float* slo, const float* demand, int
   const size_t o_bounds = take(16 * (size_t)cells), o_rev = take(cells);
   const size_t o_theta = take(8 * (size_t)d.theta_cap), o_nth = take(8);
   const size_t o_rowc = take(8 * (size_t)d.K4), o_rowb = take(8 * (size_t)d.K4);
-  const size_t o_base = take(2 * sizeof(fs_allocation)), o_status = take(4);
+  const size_t o_base = take(2 * sizeof(fs_allocation)), o_status = take(4), o_lmax = take(4);
   rc = m->fixed.ensure(off, "model state");
   if (rc) {
     delete m;
@@ -323,6 +326,7 @@ int fs_load_model(const fs_bounds* b, const float* slo, const float* demand, int
   s.rowB = (int*)(base + o_rowb);
   s.base = (fs_allocation*)(base + o_base);
   s.status = (uint32_t*)(base + o_status);
+  s.lmax = (int*)(base + o_lmax);
   s.skip = nullptr;
 
   m->h_lam.assign(demand, demand + K);
@@ -418,7 +422,7 @@ int fs_solve(fs_model* m, const float* cap, const float* tail, fs_allocation* ou
   cudaStream_t s = m->stream;
   FS_CUDA(cudaMemcpyAsync(d_cap, cap, 4 * (size_t)cells, cudaMemcpyHostToDevice, s), "upload cap");
   FS_CUDA(cudaMemcpyAsync(d_tail, tail, 4 * (size_t)cells, cudaMemcpyHostToDevice, s), "upload tail");
-  FS_CUDA(launch_solve(m->set, 1, d_cap, d_tail, d_out, false, s), "launch solve");
+  FS_CUDA(launch_solve(m->set, 1, d_cap, d_tail, d_out, false, m->lc, s), "launch solve");
   FS_CUDA(cudaMemcpyAsync(out, d_out, sizeof(fs_allocation), cudaMemcpyDeviceToHost, s), "read allocation");
   return read_status(m, s);
 }
@@ -429,14 +433,15 @@ int fs_solve_batch(fs_model* m, int32_t n, const float* cap_dev, const float* ta
   if (n < 0) return fail(FS_EINVAL, "n < 0");
   if (n == 0) return FS_OK;
   if (!cap_dev || !tail_dev || !out_dev) return fail(FS_EINVAL, "NULL device pointer");
-  FS_CUDA(launch_solve(m->set, n, cap_dev, tail_dev, out_dev, false, (cudaStream_t)cuda_stream), "launch solve");
+  FS_CUDA(launch_solve(m->set, n, cap_dev, tail_dev, out_dev, false, m->lc, (cudaStream_t)cuda_stream),
+          "launch solve");
   return FS_OK;
 }
 
 int fs_solve_bounds(fs_model* m, fs_allocation* minus, fs_allocation* plus, float* gamma_t) {
   if (!m) return fail(FS_EINVAL, "model is NULL");
   cudaStream_t s = m->stream;
-  FS_CUDA(launch_solve(m->set, 2, nullptr, nullptr, nullptr, true, s), "launch solve");
+  FS_CUDA(launch_solve(m->set, 2, nullptr, nullptr, nullptr, true, m->lc, s), "launch solve");
   fs_allocation h[2];
   FS_CUDA(cudaMemcpyAsync(h, m->set.base, sizeof h, cudaMemcpyDeviceToHost, s), "read allocations");
   int rc = read_status(m, s);
@@ -550,7 +555,6 @@ int fs_replay(fs_model* m, const fs_replay_spec* sp, int32_t* rounds, int32_t* s
   rs.n_active = (int*)(base + o_nact);
   rs.item_p = (int*)(base + o_ip);
   rs.item_cell = (int*)(base + o_ic);
-  rs.item_off = nullptr;
   rs.max_rounds = sp->max_rounds;
   rs.eps = sp->eps;
   set.skip = rs.state;
@@ -575,7 +579,7 @@ int fs_replay(fs_model* m, const fs_replay_spec* sp, int32_t* rounds, int32_t* s
     const int rc_sync = read_status(m, s);  // truth buffer must outlive the copy
     if (rc_sync) return rc_sync;
     for (int r = 0; r <= sp->max_rounds; ++r) {
-      FS_CUDA(launch_solve(set, 2 * P, nullptr, nullptr, nullptr, true, s), "launch solve");
+      FS_CUDA(launch_solve(set, 2 * P, nullptr, nullptr, nullptr, true, m->lc, s), "launch solve");
       FS_CUDA(cudaMemsetAsync(rs.n_active, 0, 4, s), "clear active");
       FS_CUDA(launch_replay_certify(set, rs, r, s), "launch certify");
       int n_active = 0;
@@ -595,8 +599,9 @@ int fs_replay(fs_model* m, const fs_replay_spec* sp, int32_t* rounds, int32_t* s
       it.off = nullptr;
       fs_samples smp{sp->seed, 0, (uint32_t)r, n_items, sp->O, sp->S, 0, nullptr};
       const Plan pl = make_plan(m, &smp, n_items);
-      FS_CUDA(launch_prep(set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, s), "launch prep");
-      FS_CUDA(launch_score(set, it, pl, (const float*)m->tables.p, (uint64_t*)m->sums.p, nullptr, 0, m->sm_count, s),
+      FS_CUDA(launch_prep(set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, m->lc, s), "launch prep");
+      FS_CUDA(launch_score(set, it, pl, (const float*)m->tables.p, (uint64_t*)m->sums.p, nullptr, 0, m->sm_count,
+                           m->lc, s),
               "launch score");
       FS_CUDA(launch_replay_reveal(set, rs, it, pl, (const uint64_t*)m->sums.p, n_active, s), "launch reveal");
     }
@@ -630,24 +635,35 @@ int fs_check(fs_model* m, void* cuda_stream) {
 
 int fs_timing_enable(fs_model* m, int32_t on) {
   if (!m) return fail(FS_EINVAL, "model is NULL");
-  m->timing = on != 0;
+  if (on < 0 || on > 2) return fail(FS_EINVAL, "timing mode %d not in {0, 1, 2}", on);
+  m->timing = on;
   m->ev_used = 0;
   return FS_OK;
 }
 
-int fs_timing_read(fs_model* m, double* kernel_ms, int32_t* launches) {
+int fs_timing_read(fs_model* m, double* kernel_ms, int32_t* launches, double* phase_ms) {
   if (!m) return fail(FS_EINVAL, "model is NULL");
-  double total = 0.0;
-  const size_t n = m->ev_used / 2;
+  double total = 0.0, ph[4] = {0.0, 0.0, 0.0, 0.0};
+  const size_t n = m->ev_used / 5;
   for (size_t k = 0; k < n; ++k) {
-    FS_CUDA(cudaEventSynchronize(m->ev[2 * k + 1]), "wait timing event");
+    cudaEvent_t* e = &m->ev[5 * k];
+    FS_CUDA(cudaEventSynchronize(e[3]), "wait timing event");
     float ms = 0.0f;
-    FS_CUDA(cudaEventElapsedTime(&ms, m->ev[2 * k], m->ev[2 * k + 1]), "elapsed time");
+    FS_CUDA(cudaEventElapsedTime(&ms, e[2], e[3]), "elapsed time");
     total += ms;
+    if (m->timing == 2) {
+      FS_CUDA(cudaEventSynchronize(e[4]), "wait timing event");
+      for (int q = 0; q < 4; ++q) {
+        FS_CUDA(cudaEventElapsedTime(&ms, e[q], e[q + 1]), "elapsed time");
+        ph[q] += ms;
+      }
+    }
   }
   m->ev_used = 0;
   if (kernel_ms) *kernel_ms = total;
   if (launches) *launches = (int32_t)n;
+  if (phase_ms)
+    for (int q = 0; q < 4; ++q) phase_ms[q] = ph[q];
   return FS_OK;
 }
 

@@ -10,6 +10,7 @@
 //   rowC     [P][2][K*4]   f32   best SLO-feasible capacity per (class, TP)
 //   rowB     [P][2][K*4]   i32   its bin (-1: none)
 //   base     [P][2]        fs_allocation
+//   lmax     [1]           i32   longest padded candidate table of the call
 // Per scoring call (items = (problem, candidate cell) pairs):
 //   tables   [items][2][slot_floats] f32   per-candidate threshold tables
 //   sums     [items][O]    u64 (int64 fixed point, 2^-40)
@@ -27,8 +28,25 @@ constexpr int kCostInf = 0x3FFFFFFF;  // "no option covers the threshold"
 constexpr int kSolveThreads = 256;
 constexpr int kPrepThreads = 128;
 constexpr int kScoreThreads = 256;
-constexpr int kTableHeader = 8;       // floats before the three table arrays
-constexpr int kSmemTableCap = 1024;   // table entries staged in shared memory per realisation
+constexpr int kTableHeader = 16;      // floats before the three table arrays
+constexpr int kSmemTableCap = 256;    // table entries staged in shared memory per realisation (pow2)
+
+// Table header words (floats unless noted).
+enum : int {
+  H_TH_BASE = 0,  // threshold below the first table entry (0 if none)
+  H_M_FIRST = 1,  // replicas row r may use just above it
+  H_L = 2,        // entries (int)
+  H_LPAD = 3,     // entries padded to 4 (int)
+  H_CX = 4,       // best capacity of row r without the candidate's bin
+  H_BX = 5,       // its bin (int, -1 none)
+  H_CMAX = 6,     // max(Cexcl, cap_hi of the candidate)
+  H_LAM = 7,      // demand of the candidate's class
+  H_LO_C = 8, H_HI_C = 9, H_LO_L = 10, H_HI_L = 11,  // candidate cell bounds
+  H_SLO = 12,     // SLO of the candidate's class
+  H_CELL = 13,    // candidate cell (int)
+  H_P = 14,       // problem (int)
+  H_STEP0 = 15,   // first step of the table search, P/2 with P = pow2 >= L + 1 (int, 0 if L = 0)
+};
 
 enum : int { CAP_LO = 0, CAP_HI = 1, TAIL_LO = 2, TAIL_HI = 3 };
 
@@ -45,7 +63,7 @@ struct Dims {
   int M[kT];            // floor(G / tau)
   int theta_cap;        // K * sum M: most thresholds one realisation can have
   int slot_floats;      // stride of one (item, sigma) table
-  int lcap;             // table entries a slot can hold (multiple of 4)
+  int lcap;             // table entries a slot can hold: pow2 >= theta_cap + 1, at least 4
 };
 
 struct Set {
@@ -62,6 +80,7 @@ struct Set {
   int* rowB;            // [P][2][K4] bin of rowC, -1 = no SLO-feasible bin
   fs_allocation* base;  // [P][2]
   uint32_t* status;
+  int* lmax;            // [1]
   const int* skip;      // [P] or nullptr: base solves skip problems with skip[p] >= 0
 };
 
@@ -71,10 +90,9 @@ struct Plan {
   uint32_t key1;        // high word of the seed (stream id XORed per problem)
   uint32_t stream_base; // stream id of problem 0 (problem p uses stream_base + p)
   uint32_t round;
-  int O, S, W, w;       // W = Q / O quantiles per stratum, w = log2(W)
-  int pairs;            // ceil(S / 2) Philox calls per (candidate, outcome)
-  int ppt;              // Philox calls per thread per tile
-  int chunks;           // tiles per (candidate, outcome)
+  int O, S, W, w;       // W = Q / O quantiles per stratum, w = log2(W) <= 16
+  int sh;               // 16 - w: a 16-bit field's top w bits are field >> sh
+  int calls;            // ceil(S / 4) Philox calls per (candidate, outcome)
 };
 
 struct Items {
@@ -110,13 +128,37 @@ __device__ __forceinline__ int min_replicas(float t, float c, float lam, int M) 
 __device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
 #pragma unroll
   for (int r = 0; r < 10; ++r) {
-    const uint32_t hi0 = __umulhi(0xD2511F53u, c.x);
-    const uint32_t lo0 = 0xD2511F53u * c.x;
-    const uint32_t hi1 = __umulhi(0xCD9E8D57u, c.z);
-    const uint32_t lo1 = 0xCD9E8D57u * c.z;
-    c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
+    const uint64_t p0 = (uint64_t)0xD2511F53u * c.x;  // one wide multiply gives both halves
+    const uint64_t p1 = (uint64_t)0xCD9E8D57u * c.z;
+    c = make_uint4((uint32_t)(p1 >> 32) ^ c.y ^ k0, (uint32_t)p1, (uint32_t)(p0 >> 32) ^ c.w ^ k1, (uint32_t)p0);
     k0 += 0x9E3779B9u;
     k1 += 0xBB67AE85u;
+  }
+  return c;
+}
+
+// The ten round keys of one key, computed once and reused for many counters.
+struct PhiloxKeys {
+  uint32_t k0[10], k1[10];
+};
+
+__device__ __forceinline__ PhiloxKeys philox_keys(uint32_t k0, uint32_t k1) {
+  PhiloxKeys k;
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    k.k0[r] = k0 + (uint32_t)r * 0x9E3779B9u;
+    k.k1[r] = k1 + (uint32_t)r * 0xBB67AE85u;
+  }
+  return k;
+}
+
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, const PhiloxKeys& k) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    const uint64_t p0 = (uint64_t)0xD2511F53u * c.x;
+    const uint64_t p1 = (uint64_t)0xCD9E8D57u * c.z;
+    c = make_uint4((uint32_t)(p1 >> 32) ^ c.y ^ k.k0[r], (uint32_t)p1, (uint32_t)(p0 >> 32) ^ c.w ^ k.k1[r],
+                   (uint32_t)p0);
   }
   return c;
 }
@@ -127,11 +169,30 @@ __device__ __forceinline__ float map_into(float lo, float d, float hi, float q) 
   return fminf(fmaxf(v, lo), hi);
 }
 
+// rint(g * 2^40) for 0 <= g <= 1, round half to even, with integer and fp32
+// ALU operations only (a float-to-int64 conversion would use the FP64 unit).
+// Below 2^23, adding 2^23 rounds to an integer whose value is the bit
+// pattern's offset from that of 2^23; from 2^23 up the product is already
+// an integer: its 24-bit significand shifted by (exponent - 23).
+__device__ __forceinline__ uint64_t fixed40(float g) {
+  const float x = __fmul_rn(g, 0x1p40f);
+  const uint32_t small = __float_as_uint(__fadd_rn(x, 0x1p23f)) - 0x4B000000u;
+  const uint32_t b = __float_as_uint(x);
+  const uint32_t sh = (b >> 23) - 150u;
+  const uint64_t big = (uint64_t)((b & 0x7FFFFFu) | 0x800000u) << (sh & 63u);
+  return x < 0x1p23f ? (uint64_t)small : big;
+}
+
 __device__ __forceinline__ uint64_t global_ns() {
   uint64_t t;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
   return t;
 }
+
+// Programmatic dependent launch: wait for the preceding kernel of the stream
+// (its writes visible), and let the next one start launching.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
 // ---------------------------------------------------------------- TMA bulk copy
 
@@ -186,16 +247,42 @@ constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s
 // ---------------------------------------------------------------- launchers (host)
 
 void note_launch();
+// Launch with programmatic stream serialisation: the kernel may start while
+// its predecessor drains and synchronises with it through pdl_wait().
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                       Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  note_launch();
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
+// Per-model cache of launch shapes (filled on first use).
+struct LaunchCache {
+  size_t solve_smem = 0, prep_smem = 0, score_smem[2] = {0, 0};
+  int score_blocks_per_sm[2] = {0, 0};
+};
+
 cudaError_t launch_qtable(float* qn, int Q, cudaStream_t s);
 // Base or explicit realisations: realisation r of `n` reads cap/tail either
 // from the problem set's bounds (explicit == nullptr: r = 2 p + sigma) or from
 // cap_x / tail_x [n][cells].
 cudaError_t launch_solve(const Set& set, int n, const float* cap_x, const float* tail_x,
-                         fs_allocation* out, bool write_theta, cudaStream_t s);
+                         fs_allocation* out, bool write_theta, LaunchCache& lc, cudaStream_t s);
 cudaError_t launch_prep(const Set& set, const Items& it, const Plan& pl, float* tables,
-                        uint64_t* sums, cudaStream_t s);
+                        uint64_t* sums, LaunchCache& lc, cudaStream_t s);
 cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const float* tables,
-                         uint64_t* sums, void* dump, int dump_stride, int sm_count, cudaStream_t s);
+                         uint64_t* sums, void* dump, int dump_stride, int sm_count, LaunchCache& lc,
+                         cudaStream_t s);
 cudaError_t launch_finalize(const Set& set, const Items& it, const Plan& pl, const uint64_t* sums,
                             double* gap, double* score, float* gamma_t, int32_t* best, cudaStream_t s);
 cudaError_t launch_watchdog(uint32_t* status, uint64_t limit_ns, cudaStream_t s);
@@ -215,7 +302,6 @@ struct ReplayState {
   int* n_active;          // [1]
   int* item_p;            // [P * cells]
   int* item_cell;         // [P * cells]
-  int* item_off;          // [P + 1]
   int max_rounds;
   float eps;
 };

@@ -29,8 +29,8 @@
 // E[Gamma_{t+1} | e], the score and the argmax.
 #include <cuda_runtime.h>
 
-#include "fs_internal.cuh"
 #include "fs_finalize.cuh"
+#include "fs_internal.cuh"
 
 namespace fs {
 
@@ -77,29 +77,36 @@ __device__ __forceinline__ bool feasible_at(const Eval& e, int m, float C, float
 
 __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan pl, float* tables,
                                                        uint64_t* sums) {
-  __shared__ float sC[256];
+  extern __shared__ __align__(16) unsigned char smraw[];
+  float* sC = reinterpret_cast<float*>(smraw);  // [256]
+  float* sTh = sC + 256;                          // [theta_cap]
   __shared__ float s_cx, s_cmax;
   __shared__ int s_bx, s_b0, s_b1;
   const Dims d = set.d;
   const int item = blockIdx.x >> 1, sigma = blockIdx.x & 1;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = blockDim.x >> 5;
+  pdl_wait();     // thresholds, rows and the zeroed lmax come from k_solve
+  pdl_trigger();  // k_score may start launching; it waits for this grid to finish
   const int p = it.p ? it.p[item] : 0;
   const int cell = it.cell[item];
+  float* tab = tables + ((size_t)item * 2 + sigma) * d.slot_floats;
   if (sigma == 0)
     for (int o = tid; o < pl.O; o += blockDim.x) sums[(size_t)item * pl.O + o] = 0ull;
   if (cell < 0 || cell >= d.cells) {  // device-side candidate ids are checked here
     if (tid == 0) {
       atomicOr(set.status, ST_CELL);
-      float* tab = tables + ((size_t)item * 2 + sigma) * d.slot_floats;
       for (int k = 0; k < kTableHeader; ++k) tab[k] = 0.0f;
-      tab[5] = __int_as_float(-1);
+      tab[H_BX] = __int_as_float(-1);
     }
     return;
   }
   const int rr = cell / d.B, be = cell - rr * d.B, ie = rr >> 2, jr = rr & 3;
   const float lam = set.lam[ie], L = set.slo[ie];
   const size_t ps = (size_t)p * 2 + sigma;
+  const int total = set.ntheta[ps];
+  const float* th_g = set.theta + ps * d.theta_cap;
   for (int rho = tid; rho < d.K4; rho += blockDim.x) sC[rho] = set.rowC[ps * d.K4 + rho];
+  for (int k = tid; k < total; k += blockDim.x) sTh[k] = th_g[k];
   const float* bp = set.bounds + (size_t)p * 4 * d.cells;
   const float* capS = bp + (size_t)(sigma ? CAP_HI : CAP_LO) * d.cells;
   const float* tailS = bp + (size_t)(sigma ? TAIL_LO : TAIL_HI) * d.cells;
@@ -135,8 +142,6 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
   }
   __syncthreads();
   const float cx = s_cx, cmax = s_cmax;
-  const int total = set.ntheta[ps];
-  const float* th = set.theta + ps * d.theta_cap;
   const int msent = d.K == 1 ? d.M[jr] : 0;  // above every threshold only a lone class can go on
 
   // b0: last index feasible at Cexcl; b1: last index feasible at max(Cexcl, cap_hi)
@@ -144,15 +149,15 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
     int lo = -1, hi = total;
     while (hi - lo > 1) {
       const int mid = (lo + hi) >> 1;
-      const Eval e = warp_eval_excl(th[mid], sC, set.lam, d, rr, ie, lane);
-      if (feasible_at(e, replicas_left(e, jr, d), cx, th[mid], lam)) lo = mid; else hi = mid;
+      const Eval e = warp_eval_excl(sTh[mid], sC, set.lam, d, rr, ie, lane);
+      if (feasible_at(e, replicas_left(e, jr, d), cx, sTh[mid], lam)) lo = mid; else hi = mid;
     }
     const int b0 = lo;
     hi = total;
     while (hi - lo > 1) {
       const int mid = (lo + hi) >> 1;
-      const Eval e = warp_eval_excl(th[mid], sC, set.lam, d, rr, ie, lane);
-      if (feasible_at(e, replicas_left(e, jr, d), cmax, th[mid], lam)) lo = mid; else hi = mid;
+      const Eval e = warp_eval_excl(sTh[mid], sC, set.lam, d, rr, ie, lane);
+      if (feasible_at(e, replicas_left(e, jr, d), cmax, sTh[mid], lam)) lo = mid; else hi = mid;
     }
     if (lane == 0) {
       s_b0 = b0;
@@ -162,12 +167,15 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
   __syncthreads();
   const int b0 = s_b0, b1 = s_b1;
   const int Lt = b1 - b0;
-  float* tab = tables + ((size_t)item * 2 + sigma) * d.slot_floats;
-  if (Lt > d.lcap) {  // cannot happen: Lt <= total <= theta_cap <= lcap
+  // arrays padded to P = pow2 >= Lt + 1 entries (+inf beyond Lt), so the
+  // scenario search needs no bound checks; at least 4 for 16-byte copies
+  int P = 1;
+  while (P < Lt + 1) P <<= 1;
+  const int Lpad = Lt ? max(P, 4) : 0;
+  if (Lpad > d.lcap) {  // cannot happen: Lt <= total <= theta_cap
     if (tid == 0) atomicOr(set.status, ST_TABLE);
     return;
   }
-  const int Lpad = (Lt + 3) & ~3;
   float* kap = tab + kTableHeader;
   float* tht = kap + Lpad;
   float* mn = tht + Lpad;
@@ -177,7 +185,7 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
     const int k = b0 + 1 + u;
     int m;
     if (k < total) {
-      const Eval e = warp_eval_excl(th[k], sC, set.lam, d, rr, ie, lane);
+      const Eval e = warp_eval_excl(sTh[k], sC, set.lam, d, rr, ie, lane);
       m = replicas_left(e, jr, d);
     } else {
       m = msent;
@@ -185,7 +193,7 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
     if (u < Lt) {
       // smallest capacity in (cx, cmax] at which f(m, C) >= theta_k: 32-ary search on the
       // bit patterns of nonnegative floats (ordered like the values)
-      const float t = th[k];
+      const float t = sTh[k];
       uint32_t lo = __float_as_uint(cx), hi = __float_as_uint(cmax);
       while (hi - lo > 1) {
         const uint32_t span = hi - lo;
@@ -204,7 +212,7 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
       }
     }
     if (lane == 0) {
-      if (u == 0) tab[1] = (float)m; else mn[u - 1] = (float)m;
+      if (u == 0) tab[H_M_FIRST] = (float)m; else mn[u - 1] = (float)m;
     }
   }
   for (int u = Lt + tid; u < Lpad; u += blockDim.x) {
@@ -213,30 +221,36 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
     mn[u] = 0.0f;
   }
   if (tid == 0) {
-    tab[0] = b0 >= 0 ? th[b0] : 0.0f;
-    tab[2] = __int_as_float(Lt);
-    tab[3] = __int_as_float(Lpad);
-    tab[4] = cx;
-    tab[5] = __int_as_float(s_bx);
-    tab[6] = cmax;
-    tab[7] = 0.0f;
+    tab[H_TH_BASE] = b0 >= 0 ? sTh[b0] : 0.0f;
+    tab[H_L] = __int_as_float(Lt);
+    tab[H_LPAD] = __int_as_float(Lpad);
+    tab[H_CX] = cx;
+    tab[H_BX] = __int_as_float(s_bx);
+    tab[H_CMAX] = cmax;
+    tab[H_LAM] = lam;
+    tab[H_LO_C] = bp[(size_t)CAP_LO * d.cells + cell];
+    tab[H_HI_C] = bp[(size_t)CAP_HI * d.cells + cell];
+    tab[H_LO_L] = bp[(size_t)TAIL_LO * d.cells + cell];
+    tab[H_HI_L] = bp[(size_t)TAIL_HI * d.cells + cell];
+    tab[H_SLO] = L;
+    tab[H_CELL] = __int_as_float(cell);
+    tab[H_P] = __int_as_float(p);
+    tab[H_STEP0] = __int_as_float(Lt ? P >> 1 : 0);
+    atomicMax(set.lmax, Lpad);
   }
 }
 
-// t* of one realisation with row capacity C (see the file comment).
+// t* of one realisation with row capacity C (see the file comment). kap is
+// padded with +inf to a power of two above the entry count, so the
+// branch-free search needs no bound checks; step0 = half that power.
 __device__ __forceinline__ float tstar_of(float C, const float* kap, const float* tht, const float* mn,
-                                          int L, int step0, float th_base, float m_first, float lam) {
+                                          int step0, float th_base, float m_first, float lam) {
   int pos = 0;
-  for (int step = step0; step > 0; step >>= 1)
-    if (pos + step <= L && kap[pos + step - 1] <= C) pos += step;
+  for (int step = step0; step > 0; step >>= 1) pos += kap[pos + step - 1] <= C ? step : 0;
   const float thb = pos ? tht[pos - 1] : th_base;
   const float m = pos ? mn[pos - 1] : m_first;
   const float tr = m >= 1.0f ? fulfil(m, C, lam) : 0.0f;
   return tr > thb ? tr : thb;
-}
-
-__device__ __forceinline__ int top_pow2(int L) {
-  return L > 0 ? (1 << (31 - __clz(L))) : 0;
 }
 
 // Per-class choice of one scenario at threshold t (dump mode only): rows from
@@ -272,148 +286,205 @@ __device__ void dump_choices(float t, const Set& set, size_t ps, int rr, float C
   *total_gpus = t > 0.0f ? total : 0;
 }
 
+// Philox calls [q_lo, q_hi) of one (candidate, outcome) segment; call q
+// serves samples 4q..4q+3, sample 4q+h reading output word h (upper 16 bits:
+// capacity position, lower 16 bits: tail position; top log2(W) bits each).
+// h0/h1 point at the staged table headers; kap/tht/mnn at the table arrays
+// (shared memory when TS, else global). Without DUMP, sQ holds the stratum's
+// capacities already mapped into [cap_lo, cap_hi], and the tail gate of
+// Eq. 5 (l_y <= L_i) is the position test kl < kgate (the mapped tail
+// quantiles are nondecreasing in the position); with DUMP, sQ holds the raw
+// quantiles and both values are mapped per sample.
+template <bool DUMP, bool TS>
+__device__ __forceinline__ uint64_t run_piece(const Set& set, const Plan& pl, int item, int o, int q_lo,
+                                              int q_hi, const float* sQ, int qoff, int kgate, const float* h0,
+                                              const float* h1, const float* kap0, const float* tht0,
+                                              const float* mn0, const float* kap1, const float* tht1,
+                                              const float* mn1, unsigned char* dump, int dump_stride) {
+  const int st0 = __float_as_int(h0[H_STEP0]), st1 = __float_as_int(h1[H_STEP0]);
+  const float thb0 = h0[H_TH_BASE], mf0 = h0[H_M_FIRST], cx0 = h0[H_CX];
+  const float thb1 = h1[H_TH_BASE], mf1 = h1[H_M_FIRST], cx1 = h1[H_CX];
+  const float lam = h0[H_LAM];
+  const int cell = __float_as_int(h0[H_CELL]), p = __float_as_int(h0[H_P]);
+  const PhiloxKeys keys = philox_keys(pl.key0, pl.key1 ^ (pl.stream_base + (uint32_t)p));
+  const uint32_t sh = (uint32_t)pl.sh;
+  const int S = pl.S;
+  const uint32_t ctr1 = (uint32_t)o, ctr2 = (uint32_t)cell, ctr3 = pl.round;
+  const float* sQo = sQ + qoff;
+  uint64_t acc = 0;
+  for (int q = q_lo + (int)threadIdx.x; q < q_hi; q += blockDim.x) {
+    const uint4 x = philox4x32_10(make_uint4((uint32_t)q, ctr1, ctr2, ctr3), keys);
+#pragma unroll
+    for (int h = 0; h < 4; ++h) {
+      const int s = 4 * q + h;
+      const uint32_t word = h == 0 ? x.x : h == 1 ? x.y : h == 2 ? x.z : x.w;
+      const int kc = (int)((word >> 16) >> sh);
+      const int kl = (int)((word & 0xFFFFu) >> sh);
+      float cy, ly = 0.0f;
+      bool gate;
+      if (DUMP) {
+        const float lo_c = h0[H_LO_C], hi_c = h0[H_HI_C], lo_l = h0[H_LO_L], hi_l = h0[H_HI_L];
+        cy = map_into(lo_c, __fsub_rn(hi_c, lo_c), hi_c, sQo[kc]);
+        ly = map_into(lo_l, __fsub_rn(hi_l, lo_l), hi_l, sQo[kl]);
+        gate = ly <= h0[H_SLO];
+      } else {
+        cy = sQo[kc];
+        gate = kl < kgate;
+      }
+      const float C0 = gate ? fmaxf(cx0, cy) : cx0;
+      const float C1 = gate ? fmaxf(cx1, cy) : cx1;
+      const float t0 = tstar_of(C0, kap0, tht0, mn0, st0, thb0, mf0, lam);
+      const float t1 = tstar_of(C1, kap1, tht1, mn1, st1, thb1, mf1, lam);
+      const uint64_t gf = fixed40(__fsub_rn(t1, t0));
+      acc += (h == 0 || s < S) ? gf : 0ull;  // the last call may serve fewer than four samples
+      if (DUMP && (h == 0 || s < S)) {
+        const size_t idx = ((size_t)item * pl.O + o) * pl.S + s;
+        unsigned char* rec = dump + idx * dump_stride;
+        fs_scenario_head hd;
+        hd.c_y = cy;
+        hd.l_y = ly;
+        hd.t_star[0] = t0;
+        hd.t_star[1] = t1;
+        const int rr = cell / set.d.B, be = cell - rr * set.d.B;
+        uint32_t* ch = reinterpret_cast<uint32_t*>(rec + sizeof(fs_scenario_head));
+#pragma unroll
+        for (int sg = 0; sg < 2; ++sg) {
+          const float cx = sg ? cx1 : cx0;
+          const int bx = __float_as_int(sg ? h1[H_BX] : h0[H_BX]);
+          int bC;
+          if (!gate) bC = bx;
+          else if (bx < 0 || cy > cx) bC = be;
+          else if (cy == cx) bC = min(be, bx);
+          else bC = bx;
+          dump_choices(sg ? t1 : t0, set, (size_t)p * 2 + sg, rr, sg ? C1 : C0, bC, ch + sg * set.d.K,
+                       &hd.total_gpus[sg]);
+        }
+        *reinterpret_cast<fs_scenario_head*>(rec) = hd;
+      }
+    }
+  }
+  return acc;
+}
+
+// Thread 0: stage segment seg (its quantile window and both candidate tables,
+// header plus lcopy entries each) into dst, completing on bar.
+__device__ __forceinline__ void stage_segment(const Set& set, const Plan& pl, const float* tables, int seg,
+                                              float* dst, uint64_t* bar, int qwin, int tstride, int lcopy) {
+  const Dims& d = set.d;
+  const int item = seg / pl.O, o = seg - item * pl.O;
+  const int q0 = (o * pl.W) & ~3;
+  const int q1 = min(((o + 1) * pl.W + 3) & ~3, d.Q);
+  const float* tab = tables + (size_t)item * 2 * d.slot_floats;
+  const uint32_t tb = (uint32_t)(kTableHeader + 3 * lcopy) * 4u;
+  const uint32_t qb = (uint32_t)(q1 - q0) * 4u;
+  fence_proxy_async();
+  mbar_expect_tx(bar, qb + 2 * tb);
+  bulk_g2s(dst, set.qn + q0, qb, bar);
+  bulk_g2s(dst + qwin, tab, tb, bar);
+  bulk_g2s(dst + qwin + tstride, tab + d.slot_floats, tb, bar);
+}
+
+// Each block owns a contiguous range of the flattened Philox-call index
+// (segment = (candidate, outcome), ceil(S/4) calls each), so the work is
+// balanced to within one call per thread. A segment's quantile window and
+// both candidate tables are staged in shared memory by TMA bulk copies,
+// double-buffered: the next segment's copies fly while this one computes.
 template <bool DUMP>
-__global__ void __launch_bounds__(kScoreThreads) k_score(Set set, Items it, Plan pl, const float* tables,
+__global__ void __launch_bounds__(kScoreThreads, 5) k_score(Set set, Items it, Plan pl, const float* tables,
                                                          uint64_t* sums, unsigned char* dump, int dump_stride,
-                                                         int n_tiles, int lcap_s, int qwin) {
+                                                         long long total_calls, int lcap_s, int qwin) {
   extern __shared__ __align__(16) unsigned char smraw[];
-  uint64_t* bar = reinterpret_cast<uint64_t*>(smraw);
-  float* sQ = reinterpret_cast<float*>(smraw + 16);
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smraw);  // [2]
   const int tstride = kTableHeader + 3 * lcap_s;
-  float* sT[2] = {sQ + qwin, sQ + qwin + tstride};
+  const int stage_floats = qwin + 2 * tstride;
+  float* stage0 = reinterpret_cast<float*>(smraw + 16);
+  __shared__ int s_lcopy;
   const Dims d = set.d;
   const int tid = threadIdx.x, lane = tid & 31;
 
-  if (tid == 0) mbar_init(bar, 1);
+  pdl_wait();  // tables, zeroed sums and lmax come from k_prep
+  const long long g = gridDim.x;
+  const long long r_lo = total_calls * blockIdx.x / g;
+  const long long r_hi = total_calls * (blockIdx.x + 1) / g;
+  if (r_hi <= r_lo) return;
+  const int seg_first = (int)(r_lo / pl.calls);
+  const int seg_last = (int)((r_hi - 1) / pl.calls);
+
+  if (tid == 0) {
+    s_lcopy = min(*set.lmax, lcap_s);
+    mbar_init(&bar[0], 1);
+    mbar_init(&bar[1], 1);
+  }
   __syncthreads();
-  uint32_t phase = 0;
+  const int lcopy = s_lcopy;
+  if (tid == 0) stage_segment(set, pl, tables, seg_first, stage0, bar, qwin, tstride, lcopy);
 
-  for (int tile = blockIdx.x; tile < n_tiles; tile += gridDim.x) {
-    const int chunk = tile % pl.chunks;
-    const int eo = tile / pl.chunks;
-    const int o = eo % pl.O;
-    const int item = eo / pl.O;
-    const int p = it.p ? it.p[item] : 0;
-    const int cell = it.cell[item];
-    if (cell < 0 || cell >= d.cells) continue;  // flagged by k_prep; uniform over the block
-    const float* tab[2] = {tables + (size_t)item * 2 * d.slot_floats,
-                           tables + ((size_t)item * 2 + 1) * d.slot_floats};
-    int Lr[2], Lp[2];
-    bool inS[2];
-#pragma unroll
-    for (int sg = 0; sg < 2; ++sg) {
-      Lr[sg] = __float_as_int(tab[sg][2]);
-      Lp[sg] = __float_as_int(tab[sg][3]);
-      inS[sg] = Lp[sg] <= lcap_s;
-    }
-    const int q0 = (o * pl.W) & ~3;
-    const int q1 = min(((o + 1) * pl.W + 3) & ~3, d.Q);
-
-    __syncthreads();  // every thread is done with the previous tile's staged data
-    if (tid == 0) {
-      fence_proxy_async();
-      uint32_t bytes = (uint32_t)(q1 - q0) * 4u;
-      uint32_t tb[2];
-#pragma unroll
-      for (int sg = 0; sg < 2; ++sg) {
-        tb[sg] = inS[sg] ? (uint32_t)(kTableHeader + 3 * Lp[sg]) * 4u : (uint32_t)kTableHeader * 4u;
-        bytes += tb[sg];
-      }
-      mbar_expect_tx(bar, bytes);
-      bulk_g2s(sQ, set.qn + q0, (uint32_t)(q1 - q0) * 4u, bar);
-      bulk_g2s(sT[0], tab[0], tb[0], bar);
-      bulk_g2s(sT[1], tab[1], tb[1], bar);
-    }
-    const bool ok = mbar_wait(bar, phase, kWaitLimitNs);
-    phase ^= 1u;
+  int j = 0;
+  for (int seg = seg_first; seg <= seg_last; ++seg, ++j) {
+    const int st = j & 1;
+    if (tid == 0 && seg < seg_last)
+      stage_segment(set, pl, tables, seg + 1, stage0 + (size_t)(st ^ 1) * stage_floats, bar + (st ^ 1), qwin,
+                    tstride, lcopy);
+    const bool ok = mbar_wait(&bar[st], (uint32_t)((j >> 1) & 1), kWaitLimitNs);
     if (__syncthreads_or(!ok)) {
       if (tid == 0) atomicOr(set.status, ST_TIMEOUT);
-      mbar_wait(bar, phase ^ 1u, kWaitLimitNs);  // let copies in flight land before exiting
+      // let copies in flight land before the block exits (bounded as well)
+      mbar_wait(&bar[st], (uint32_t)((j >> 1) & 1), kWaitLimitNs);
+      if (seg < seg_last) mbar_wait(&bar[st ^ 1], (uint32_t)(((j + 1) >> 1) & 1), kWaitLimitNs);
       return;
     }
-
-    const float* kap[2];
-    const float* tht[2];
-    const float* mnn[2];
-#pragma unroll
-    for (int sg = 0; sg < 2; ++sg) {
-      const float* base = inS[sg] ? sT[sg] : tab[sg];
-      kap[sg] = base + kTableHeader;
-      tht[sg] = kap[sg] + Lp[sg];
-      mnn[sg] = tht[sg] + Lp[sg];
-    }
-    const float thb0 = sT[0][0], mf0 = sT[0][1], cx0 = sT[0][4];
-    const float thb1 = sT[1][0], mf1 = sT[1][1], cx1 = sT[1][4];
-    const int st0 = top_pow2(Lr[0]), st1 = top_pow2(Lr[1]);
-
-    const int ie = cell / d.B >> 2;
-    const float lam = set.lam[ie], Lslo = set.slo[ie];
-    const float* bp = set.bounds + (size_t)p * 4 * d.cells;
-    const float lo_c = bp[(size_t)CAP_LO * d.cells + cell], hi_c = bp[(size_t)CAP_HI * d.cells + cell];
-    const float lo_l = bp[(size_t)TAIL_LO * d.cells + cell], hi_l = bp[(size_t)TAIL_HI * d.cells + cell];
-    const float d_c = __fsub_rn(hi_c, lo_c), d_l = __fsub_rn(hi_l, lo_l);
-    const uint32_t k0 = pl.key0, k1 = pl.key1 ^ (pl.stream_base + (uint32_t)p);
-    const int qoff = o * pl.W - q0;
-    const uint32_t W = (uint32_t)pl.W;
-
-    uint64_t acc = 0;
-    for (int pp = 0; pp < pl.ppt; ++pp) {
-      const int pair = (chunk * pl.ppt + pp) * blockDim.x + tid;
-      if (pair >= pl.pairs) break;
-      const uint4 x = philox4x32_10(make_uint4((uint32_t)pair, (uint32_t)o, (uint32_t)cell, pl.round), k0, k1);
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int s = 2 * pair + h;
-        if (h == 1 && s >= pl.S) break;
-        const uint32_t xc = h ? x.z : x.x;
-        const uint32_t xl = h ? x.w : x.y;
-        const int kc = qoff + (int)__umulhi(xc, W);  // top log2(W) bits
-        const int kl = qoff + (int)__umulhi(xl, W);
-        const float cy = map_into(lo_c, d_c, hi_c, sQ[kc]);
-        const float ly = map_into(lo_l, d_l, hi_l, sQ[kl]);
-        const bool gate = ly <= Lslo;                       // Eq. 5 for the revealed cell
-        const float C0 = gate ? fmaxf(cx0, cy) : cx0;
-        const float C1 = gate ? fmaxf(cx1, cy) : cx1;
-        const float t0 = tstar_of(C0, kap[0], tht[0], mnn[0], Lr[0], st0, thb0, mf0, lam);
-        const float t1 = tstar_of(C1, kap[1], tht[1], mnn[1], Lr[1], st1, thb1, mf1, lam);
-        const float g = __fsub_rn(t1, t0);
-        acc += (uint64_t)__float2ll_rn(__fmul_rn(g, 0x1p40f));
-        if (DUMP) {
-          const size_t idx = ((size_t)item * pl.O + o) * pl.S + s;
-          unsigned char* rec = dump + idx * dump_stride;
-          fs_scenario_head hd;
-          hd.c_y = cy;
-          hd.l_y = ly;
-          hd.t_star[0] = t0;
-          hd.t_star[1] = t1;
-          const int rr = cell / d.B, be = cell - rr * d.B;
-          uint32_t* ch = reinterpret_cast<uint32_t*>(rec + sizeof(fs_scenario_head));
-#pragma unroll
-          for (int sg = 0; sg < 2; ++sg) {
-            const float cx = sg ? cx1 : cx0;
-            const int bx = __float_as_int(sg ? sT[1][5] : sT[0][5]);
-            const float C = sg ? C1 : C0;
-            int bC;
-            if (!gate) bC = bx;
-            else if (bx < 0 || cy > cx) bC = be;
-            else if (cy == cx) bC = min(be, bx);
-            else bC = bx;
-            dump_choices(sg ? t1 : t0, set, (size_t)p * 2 + sg, rr, C, bC, ch + sg * d.K,
-                         &hd.total_gpus[sg]);
-          }
-          *reinterpret_cast<fs_scenario_head*>(rec) = hd;
+    float* stg = stage0 + (size_t)st * stage_floats;
+    const float* h0 = stg + qwin;
+    const float* h1 = h0 + tstride;
+    const int item = seg / pl.O, o = seg - item * pl.O;
+    const long long sb = (long long)seg * pl.calls;
+    const int q_lo = (int)(max(r_lo, sb) - sb);
+    const int q_hi = (int)(min(r_hi, sb + pl.calls) - sb);
+    const int qoff = o * pl.W - ((o * pl.W) & ~3);
+    const int Lp0 = __float_as_int(h0[H_LPAD]), Lp1 = __float_as_int(h1[H_LPAD]);
+    const int cell = __float_as_int(h0[H_CELL]);
+    const bool cell_ok = cell >= 0 && cell < d.cells;  // a bad device-side id was flagged by k_prep
+    int kgate = 0;
+    if (!DUMP) {
+      // map the stratum's quantiles into this cell's capacity interval in place,
+      // and count the positions whose tail value passes the SLO gate
+      const float lo_c = h0[H_LO_C], hi_c = h0[H_HI_C], lo_l = h0[H_LO_L], hi_l = h0[H_HI_L];
+      const float d_c = __fsub_rn(hi_c, lo_c), d_l = __fsub_rn(hi_l, lo_l), slo = h0[H_SLO];
+      for (int k0 = 0; k0 < pl.W; k0 += blockDim.x) {
+        const int k = k0 + tid;
+        bool pass = false;
+        if (k < pl.W) {
+          const float qv = stg[qoff + k];
+          stg[qoff + k] = map_into(lo_c, d_c, hi_c, qv);
+          pass = map_into(lo_l, d_l, hi_l, qv) <= slo;
         }
+        kgate += __syncthreads_count(pass);
+      }
+    }
+    uint64_t acc = 0;
+    if (cell_ok) {
+      if (Lp0 <= lcopy && Lp1 <= lcopy) {
+        acc = run_piece<DUMP, true>(set, pl, item, o, q_lo, q_hi, stg, qoff, kgate, h0, h1, h0 + kTableHeader,
+                                    h0 + kTableHeader + Lp0, h0 + kTableHeader + 2 * Lp0, h1 + kTableHeader,
+                                    h1 + kTableHeader + Lp1, h1 + kTableHeader + 2 * Lp1, dump, dump_stride);
+      } else {
+        const float* g0 = tables + (size_t)item * 2 * d.slot_floats + kTableHeader;
+        const float* g1 = g0 + d.slot_floats;
+        acc = run_piece<DUMP, false>(set, pl, item, o, q_lo, q_hi, stg, qoff, kgate, h0, h1, g0, g0 + Lp0,
+                                     g0 + 2 * Lp0, g1, g1 + Lp1, g1 + 2 * Lp1, dump, dump_stride);
       }
     }
     for (int off = 16; off; off >>= 1) acc += __shfl_down_sync(0xffffffffu, acc, off);
     if (lane == 0 && acc)
-      atomicAdd(reinterpret_cast<unsigned long long*>(&sums[(size_t)item * pl.O + o]),
-                (unsigned long long)acc);
+      atomicAdd(reinterpret_cast<unsigned long long*>(&sums[(size_t)seg]), (unsigned long long)acc);
+    __syncthreads();  // stage st is free for the copies issued next iteration
   }
+  pdl_trigger();
 }
 
 __global__ void k_finalize(Set set, Items it, Plan pl, const uint64_t* sums, double* gap, double* score,
                            float* gamma_t, int32_t* best) {
+  pdl_wait();
   const int p = blockIdx.x;
   const int beg = it.off ? it.off[p] : 0;
   const int end = it.off ? it.off[p + 1] : it.n;
@@ -421,63 +492,71 @@ __global__ void k_finalize(Set set, Items it, Plan pl, const uint64_t* sums, dou
   if (threadIdx.x == 0 && best) best[p] = b.pos >= 0 ? it.cell[beg + b.pos] : -1;
 }
 
+static size_t prep_smem_bytes(const Dims& d) { return (size_t)(256 + d.theta_cap) * 4; }
+
 cudaError_t launch_prep(const Set& set, const Items& it, const Plan& pl, float* tables, uint64_t* sums,
-                        cudaStream_t s) {
+                        LaunchCache& lc, cudaStream_t s) {
   if (it.n <= 0) return cudaSuccess;
-  note_launch();
-  k_prep<<<it.n * 2, kPrepThreads, 0, s>>>(set, it, pl, tables, sums);
-  return cudaGetLastError();
+  const size_t smem = prep_smem_bytes(set.d);
+  if (smem > lc.prep_smem) {
+    cudaError_t e = cudaFuncSetAttribute(k_prep, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    lc.prep_smem = smem;
+  }
+  return launch_pdl(k_prep, dim3(it.n * 2), dim3(kPrepThreads), smem, s, set, it, pl, tables, sums);
 }
 
-static int score_lcap(const Dims& d) {
-  const int lc = (d.theta_cap + 3) & ~3;
-  return lc < kSmemTableCap ? lc : kSmemTableCap;
-}
+static int score_lcap(const Dims& d) { return d.lcap < kSmemTableCap ? d.lcap : kSmemTableCap; }
 
 static int score_qwin(const Dims& d, const Plan& pl) {
   const int w = ((pl.W + 3) & ~3) + 4;
   return w < d.Q ? w : d.Q;
 }
 
-static size_t score_smem(const Dims& d, const Plan& pl) {
-  return 16 + (size_t)score_qwin(d, pl) * 4 + 2 * (size_t)(kTableHeader + 3 * score_lcap(d)) * 4;
-}
-
 cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const float* tables, uint64_t* sums,
-                         void* dump, int dump_stride, int sm_count, cudaStream_t s) {
+                         void* dump, int dump_stride, int sm_count, LaunchCache& lc, cudaStream_t s) {
   if (it.n <= 0) return cudaSuccess;
-  const long long tiles = (long long)it.n * pl.O * pl.chunks;
-  if (tiles > 0x7fffffffLL) return cudaErrorInvalidValue;
-  const size_t smem = score_smem(set.d, pl);
+  const long long total = (long long)it.n * pl.O * pl.calls;
   const int lcap_s = score_lcap(set.d), qwin = score_qwin(set.d, pl);
-  int per_sm = 0;
-  cudaError_t e;
-  if (dump) {
-    e = cudaFuncSetAttribute(k_score<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_score<true>, kScoreThreads, smem);
-  } else {
-    e = cudaFuncSetAttribute(k_score<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_score<false>, kScoreThreads, smem);
+  const size_t smem = 16 + 2 * (size_t)(qwin + 2 * (kTableHeader + 3 * lcap_s)) * 4;
+  const int v = dump ? 1 : 0;
+  if (smem != lc.score_smem[v]) {
+    cudaError_t e;
+    int per_sm = 0;
+    if (dump) {
+      e = cudaFuncSetAttribute(k_score<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e == cudaSuccess)
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_score<true>, kScoreThreads, smem);
+    } else {
+      e = cudaFuncSetAttribute(k_score<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e == cudaSuccess)
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_score<false>, kScoreThreads, smem);
+    }
+    if (e != cudaSuccess) return e;
+    lc.score_smem[v] = smem;
+    lc.score_blocks_per_sm[v] = per_sm < 1 ? 1 : per_sm;
   }
-  if (e != cudaSuccess) return e;
-  if (per_sm < 1) per_sm = 1;
-  const long long cap = (long long)per_sm * sm_count;
-  const int grid = (int)(tiles < cap ? tiles : cap);
-  note_launch();
+  // One resident wave at least; up to four when every block still gets >= 16
+  // calls per thread, so that the block scheduler evens out segments of
+  // unequal cost (table length, fulfilment divisions).
+  const long long resident = (long long)lc.score_blocks_per_sm[v] * sm_count;
+  const long long by_work = total / ((long long)kScoreThreads * 16);
+  long long grid_l = by_work < 4 * resident ? by_work : 4 * resident;
+  if (grid_l < resident) grid_l = resident;
+  const long long min_blocks = (total + kScoreThreads - 1) / kScoreThreads;
+  if (grid_l > min_blocks) grid_l = min_blocks;
+  const int grid = (int)grid_l;
   if (dump)
-    k_score<true><<<grid, kScoreThreads, smem, s>>>(set, it, pl, tables, sums, (unsigned char*)dump, dump_stride,
-                                                    (int)tiles, lcap_s, qwin);
-  else
-    k_score<false><<<grid, kScoreThreads, smem, s>>>(set, it, pl, tables, sums, nullptr, 0, (int)tiles, lcap_s,
-                                                     qwin);
-  return cudaGetLastError();
+    return launch_pdl(k_score<true>, dim3(grid), dim3(kScoreThreads), smem, s, set, it, pl, tables, sums,
+                      (unsigned char*)dump, dump_stride, total, lcap_s, qwin);
+  return launch_pdl(k_score<false>, dim3(grid), dim3(kScoreThreads), smem, s, set, it, pl, tables, sums,
+                    (unsigned char*)nullptr, 0, total, lcap_s, qwin);
 }
 
 cudaError_t launch_finalize(const Set& set, const Items& it, const Plan& pl, const uint64_t* sums, double* gap,
                             double* score, float* gamma_t, int32_t* best, cudaStream_t s) {
-  note_launch();
-  k_finalize<<<it.off ? set.P : 1, 256, 0, s>>>(set, it, pl, sums, gap, score, gamma_t, best);
-  return cudaGetLastError();
+  return launch_pdl(k_finalize, dim3(it.off ? set.P : 1), dim3(256), 0, s, set, it, pl, sums, gap, score,
+                    gamma_t, best);
 }
 
 }  // namespace fs

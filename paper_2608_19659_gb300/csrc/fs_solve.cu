@@ -3,7 +3,9 @@
 //
 // One CTA solves one realisation (a capacity and a tail value per cell):
 //   1. rows: for every (class i, TP index j) the best SLO-feasible bin
-//      (largest capacity, then lowest bin; Eq. 5 gates l <= L_i) -> C_ij;
+//      (largest capacity, then lowest bin; Eq. 5 gates l <= L_i) -> C_ij.
+//      All cells are read once, coalesced; each feasible cell folds
+//      (capacity, -bin) into its row with a 64-bit shared-memory atomicMax;
 //   2. thresholds: the positive fulfilments f(n, C_ij), n = 1..floor(G/tau_j)
 //      (cut at the first n with f = 1), written to shared memory and
 //      bitonic-sorted;
@@ -67,8 +69,10 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   extern __shared__ __align__(16) unsigned char smraw[];
   const Dims d = set.d;
   const int r = blockIdx.x;
-  if (r >= n_real) return;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = blockDim.x >> 5;
+  if (r == 0 && tid == 0 && set.lmax) *set.lmax = 0;  // before any early exit
+  pdl_trigger();
+  if (r >= n_real) return;
 
   const float* cap;
   const float* tail;
@@ -88,7 +92,8 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
     out = set.base + r;
   }
 
-  float* sC = reinterpret_cast<float*>(smraw);          // [256]
+  unsigned long long* sKey = reinterpret_cast<unsigned long long*>(smraw);  // [256]
+  float* sC = reinterpret_cast<float*>(sKey + 256);       // [256]
   int* sB = reinterpret_cast<int*>(sC + 256);             // [256]
   int* sN0 = sB + 256;                                    // [256]
   int* sOff = sN0 + 256;                                  // [260]
@@ -96,55 +101,57 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   int* sMisc = sProbe + 32;                               // [8]
   float* sTheta = reinterpret_cast<float*>(sMisc + 8);    // [pow2 >= theta_cap]
 
-  // 1. rows
-  for (int rho = tid; rho < d.K4; rho += blockDim.x) {
-    const int i = rho >> 2, j = rho & 3;
-    const float L = set.slo[i];
-    const float* cr = cap + (size_t)rho * d.B;
-    const float* tr = tail + (size_t)rho * d.B;
-    float best = 0.0f;
-    int bb = -1;
-    for (int b = 0; b < d.B; ++b) {
-      if (tr[b] <= L) {
-        const float c = cr[b];
-        if (bb < 0 || c > best) {
-          best = c;
-          bb = b;
-        }
-      }
+  // 1. rows: key = (capacity bits, ~bin) of the best SLO-feasible bin; 0 = none
+  for (int rho = tid; rho < d.K4; rho += blockDim.x) sKey[rho] = 0ull;
+  if (tid < 8) sMisc[tid] = 0;
+  __syncthreads();
+  for (int c = tid; c < d.cells; c += blockDim.x) {
+    const int rho = c / d.B;
+    const int b = c - rho * d.B;
+    if (tail[c] <= set.slo[rho >> 2]) {
+      const uint32_t cb = __float_as_uint(__fadd_rn(cap[c], 0.0f));  // -0 -> +0: bits order like values
+      atomicMax(&sKey[rho], ((unsigned long long)cb << 32) | (0xFFFFFFFFu - (uint32_t)b));
     }
-    sC[rho] = bb >= 0 ? best : 0.0f;
+  }
+  __syncthreads();
+  for (int rho = tid; rho < d.K4; rho += blockDim.x) {
+    const unsigned long long key = sKey[rho];
+    const int bb = key ? (int)(0xFFFFFFFFu - (uint32_t)key) : -1;
+    const float best = key ? __uint_as_float((uint32_t)(key >> 32)) : 0.0f;
+    sC[rho] = best;
     sB[rho] = bb;
+    const int i = rho >> 2, j = rho & 3;
     const float lam = set.lam[i];
     const int M = d.M[j];
     int n0 = 0, len = 0;
-    if (bb >= 0 && M >= 1) {
-      n0 = min_replicas(__int_as_float(1), best, lam, M);  // first positive fulfilment
-      if (n0) {
-        const int ns = min_replicas(1.0f, best, lam, M);   // first full fulfilment
-        len = ns ? ns : M;
+    if (bb >= 0) {
+      atomicOr(reinterpret_cast<unsigned int*>(&sMisc[2 + (i >> 5)]), 1u << (i & 31));
+      if (M >= 1) {
+        n0 = min_replicas(__int_as_float(1), best, lam, M);  // first positive fulfilment
+        if (n0) {
+          const int ns = min_replicas(1.0f, best, lam, M);   // first full fulfilment
+          len = ns ? ns : M;
+        }
       }
     }
     sN0[rho] = n0;
     sOff[rho] = n0 ? len - n0 + 1 : 0;  // count, scanned below
   }
   __syncthreads();
-  if (tid == 0) {
-    int acc = 0;
-    for (int rho = 0; rho < d.K4; ++rho) {
-      const int c = sOff[rho];
-      sOff[rho] = acc;
-      acc += c;
-    }
-    sOff[d.K4] = acc;
-    uint32_t mask_lo = 0, mask_hi = 0;
-    for (int rho = 0; rho < d.K4; ++rho)
-      if (sB[rho] >= 0) {
-        const int i = rho >> 2;
-        if (i < 32) mask_lo |= 1u << i; else mask_hi |= 1u << (i - 32);
+  if (warp == 0) {  // exclusive scan of the row counts
+    int carry = 0;
+    for (int base = 0; base < d.K4; base += 32) {
+      const int rho = base + lane;
+      const int v = rho < d.K4 ? sOff[rho] : 0;
+      int incl = v;
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
       }
-    sMisc[2] = (int)mask_lo;
-    sMisc[3] = (int)mask_hi;
+      if (rho < d.K4) sOff[rho] = carry + incl - v;
+      carry += __shfl_sync(0xffffffffu, incl, 31);
+    }
+    if (lane == 0) sOff[d.K4] = carry;
   }
   __syncthreads();
   int total = sOff[d.K4];
@@ -282,10 +289,10 @@ cudaError_t launch_watchdog(uint32_t* status, uint64_t limit_ns, cudaStream_t s)
   return cudaGetLastError();
 }
 
-size_t solve_smem_bytes(const Dims& d) {
+static size_t solve_smem_bytes(const Dims& d) {
   int P2 = 1;
   while (P2 < d.theta_cap) P2 <<= 1;
-  return (size_t)(256 * 3 + 260 + 32 + 8) * 4 + (size_t)P2 * 4;
+  return 256 * 8 + (size_t)(256 * 3 + 260 + 32 + 8) * 4 + (size_t)P2 * 4;
 }
 
 cudaError_t launch_qtable(float* qn, int Q, cudaStream_t s) {
@@ -295,11 +302,14 @@ cudaError_t launch_qtable(float* qn, int Q, cudaStream_t s) {
 }
 
 cudaError_t launch_solve(const Set& set, int n, const float* cap_x, const float* tail_x,
-                         fs_allocation* out, bool write_theta, cudaStream_t s) {
+                         fs_allocation* out, bool write_theta, LaunchCache& lc, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   const size_t smem = solve_smem_bytes(set.d);
-  cudaError_t e = cudaFuncSetAttribute(k_solve, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
+  if (smem > lc.solve_smem) {
+    cudaError_t e = cudaFuncSetAttribute(k_solve, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    lc.solve_smem = smem;
+  }
   note_launch();
   k_solve<<<n, kSolveThreads, smem, s>>>(set, n, cap_x, tail_x, out, write_theta ? 1 : 0);
   return cudaGetLastError();

@@ -99,7 +99,8 @@ def lib():
         L.fs_check.argtypes = [C.c_void_p, C.c_void_p]
         L.fs_launch_count.restype = C.c_uint64
         L.fs_timing_enable.argtypes = [C.c_void_p, C.c_int32]
-        L.fs_timing_read.argtypes = [C.c_void_p, C.POINTER(C.c_double), C.POINTER(C.c_int32)]
+        L.fs_timing_read.argtypes = [C.c_void_p, C.POINTER(C.c_double), C.POINTER(C.c_int32),
+                                     C.c_void_p]
         L.fs_watchdog_selftest.argtypes = [C.c_int64]
         L.fs_free_model.argtypes = [C.c_void_p]
         L.fs_free_model.restype = None
@@ -293,16 +294,18 @@ def fs_check(m: Model, stream=None) -> None:
     _check(lib().fs_check(m.handle, _stream(stream)))
 
 
-def fs_timing_enable(m: Model, on: bool) -> None:
-    _check(lib().fs_timing_enable(m.handle, 1 if on else 0))
+def fs_timing_enable(m: Model, mode: int) -> None:
+    """0 off, 1 Monte-Carlo kernel only, 2 every phase of a scoring call."""
+    _check(lib().fs_timing_enable(m.handle, int(mode)))
 
 
 def fs_timing_read(m: Model):
-    """(summed Monte-Carlo kernel time in ms, number of timed launches) since the last read."""
+    """(Monte-Carlo kernel ms, timed calls, [solve, prep, Monte-Carlo, reduction] ms) since the last read."""
     ms = C.c_double()
     n = C.c_int32()
-    _check(lib().fs_timing_read(m.handle, C.byref(ms), C.byref(n)))
-    return float(ms.value), int(n.value)
+    ph = np.zeros(4, np.float64)
+    _check(lib().fs_timing_read(m.handle, C.byref(ms), C.byref(n), _vp(ph)))
+    return float(ms.value), int(n.value), ph
 
 
 def fs_launch_count() -> int:

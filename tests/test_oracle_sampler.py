@@ -71,6 +71,21 @@ def test_draw_arguments_validated(oracle_lib):
         oracle_lib.draw_index(0, 0, 0, 0, 96, 8, 0, 0)  # Q/O not a power of two
     with pytest.raises(ValueError):
         oracle_lib.draw_index(0, 0, 0, 0, 4096, 8, 8, 0)  # outcome out of range
+    with pytest.raises(ValueError):
+        oracle_lib.draw_index(0, 0, 0, 0, 1 << 17, 1, 0, 0)  # more than 2^16 positions per stratum
+    assert 0 <= oracle_lib.draw_index(0, 0, 0, 0, 1 << 16, 1, 0, 5)[0] < (1 << 16)
+
+
+def test_four_samples_share_one_philox_call(oracle_lib):
+    """Samples 4m..4m+3 read the four words of the call with counter m (16-bit halves)."""
+    Q, O, o, cell, seed, stream, rnd = 4096, 16, 5, 33, (3 << 32) | 9, 2, 7
+    W = Q // O
+    for m in (0, 1, 77):
+        x = oracle_lib.philox4x32_10([m, o, cell, rnd], [seed & 0xFFFFFFFF, (seed >> 32) ^ stream])
+        for h in range(4):
+            kc, kl = oracle_lib.draw_index(seed, stream, rnd, cell, Q, O, o, 4 * m + h)
+            word = int(x[h])
+            assert kc == o * W + ((word >> 16) >> 8) and kl == o * W + ((word & 0xFFFF) >> 8)
 
 
 def test_map_is_affine_clamped_and_monotone(oracle_lib):
