@@ -168,6 +168,39 @@ int fs_score_candidates_async(fs_model *m, const fs_samples *samples, double *ga
                               int64_t *sum_eo_dev, void *dump_dev, void *cuda_stream);
 
 /*
+ * fs_score_candidates_noalloc -- the same scores as fs_score_candidates, for
+ * callers that cannot allocate device memory while they run: processes whose
+ * device memory is already handed out by their own pool, and latency-critical
+ * paths that must not pay for cudaMalloc/cudaFree (which can synchronise the
+ * device). The paper has no counterpart; this entry point exists for them.
+ * It allocates nothing and needs no fs_model:
+ *   bounds_dev   DEVICE [4][K][4][B] floats: cap_lo, cap_hi, tail_lo, tail_hi
+ *   slo_dev, demand_dev  DEVICE [K] floats
+ *   quantile_dev DEVICE [Q] table, or NULL for the built-in triangular table
+ *                (Q = 4096, rebuilt by every call)
+ *   samples      as for fs_score_candidates_async (cand is a DEVICE pointer)
+ *   gap_dev, score_dev [n_cand] doubles, gamma_t_dev [1], best_dev [1]: DEVICE
+ *                outputs (each nullable)
+ * The same limits as fs_load_model apply, and the values must satisfy its
+ * rules (finite, >= 0, lo <= hi, SLOs and demands > 0): they are on the device
+ * and are not checked here; candidate ids are range-checked by the kernels
+ * (FS_EDEVICE). All intermediates live in one fixed device array of 16 MiB
+ * that every GPU loading this library holds until the process exits; a call
+ * needing more (roughly n_cand * (2 * (16 + 3 * p) * 4 + 8 * O) bytes, p the
+ * power of two above K * sum floor(G/tau)) returns FS_EINVAL without running.
+ * The first call on a device looks up the array's address for that device, so
+ * make it before any stream capture. Every call shares the array: calls whose
+ * GPU work overlaps (other streams or host threads) race. The call enqueues its
+ * kernels on cuda_stream, waits for that stream and reports device-side errors
+ * (FS_ETIMEOUT, FS_EDEVICE).
+ */
+int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, const float *bounds_dev,
+                                const float *slo_dev, const float *demand_dev,
+                                const float *quantile_dev, int32_t Q, const fs_samples *samples,
+                                double *gap_dev, double *score_dev, float *gamma_t_dev,
+                                int32_t *best_dev, void *cuda_stream);
+
+/*
  * One allocation (Section 3): per class the chosen TP degree (0 = none),
  * bin (-1 = none), replica count and fulfilment r_i; t_star = min_i r_i
  * reached (the tier-2 objective), ok = t_star > 0.

@@ -32,6 +32,13 @@ static int fail(int code, const char* fmt, ...) {
   return code;
 }
 
+// Error message for other translation units of the library (thread-local, read
+// back through fs_last_error).
+int record_error(int code, const char* msg) {
+  g_err = msg;
+  return code;
+}
+
 static int cuda_fail(cudaError_t e, const char* what) {
   return fail(e == cudaErrorMemoryAllocation ? FS_ENOMEM : FS_ECUDA, "%s: %s", what, cudaGetErrorString(e));
 }

@@ -24,7 +24,8 @@ FS_MAX_CLASSES = 64
 EXPORTS = ("fs_load_model", "fs_update_bounds", "fs_dump_stride", "fs_score_candidates",
            "fs_score_candidates_async", "fs_solve", "fs_solve_batch", "fs_solve_bounds",
            "fs_reveal", "fs_certificate", "fs_replay", "fs_check", "fs_launch_count",
-           "fs_watchdog_selftest", "fs_free_model", "fs_last_error", "fs_timing_enable",
+           "fs_watchdog_selftest", "fs_free_model", "fs_last_error", "fs_score_candidates_noalloc",
+           "fs_timing_enable",
            "fs_timing_read")
 
 
@@ -87,6 +88,10 @@ def lib():
         L.fs_score_candidates_async.argtypes = [C.c_void_p, C.POINTER(fs_samples), C.c_void_p,
                                                 C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
                                                 C.c_void_p, C.c_void_p]
+        L.fs_score_candidates_noalloc.argtypes = [C.c_int32, C.c_int32, C.c_int32, C.c_void_p,
+                                                  C.c_void_p, C.c_void_p, C.c_void_p, C.c_int32,
+                                                  C.POINTER(fs_samples), C.c_void_p, C.c_void_p,
+                                                  C.c_void_p, C.c_void_p, C.c_void_p]
         L.fs_solve.argtypes = [C.c_void_p, fp, fp, C.POINTER(fs_allocation)]
         L.fs_solve_batch.argtypes = [C.c_void_p, C.c_int32, C.c_void_p, C.c_void_p, C.c_void_p,
                                      C.c_void_p]
@@ -208,6 +213,28 @@ def fs_score_candidates(m: Model, cand, O: int, S: int, seed: int, stream_id: in
     _check(lib().fs_score_candidates(m.handle, C.byref(smp), _vp(gap), _vp(score), _vp(gt),
                                      _vp(best), _vp(sums), _vp(dump_dev)))
     return ScoreResult(gap, score, float(gt[0]), int(best[0]), sums)
+
+
+def fs_score_candidates_noalloc(K: int, B: int, G: int, bounds_dev, slo_dev, demand_dev, cand_dev,
+                                O: int, S: int, seed: int, stream_id: int = 0, rnd: int = 0,
+                                gap_dev=None, score_dev=None, gamma_t_dev=None, best_dev=None,
+                                quantile_dev=None, stream=None) -> None:
+    """Scoring that allocates no device memory (every buffer is the caller's device tensor).
+
+    For callers that cannot allocate while they run (device memory handed out
+    by their own pool, or no room for cudaMalloc's device-wide synchronisation
+    on their path). bounds_dev: float32 [4 * K * 4 * B] (cap_lo, cap_hi,
+    tail_lo, tail_hi); slo_dev, demand_dev: float32 [K]; cand_dev: int32.
+    Intermediates use the library's fixed 16 MiB device array; larger calls
+    raise FS_EINVAL. Returns after the work on ``stream`` has finished.
+    """
+    n = int(cand_dev.numel())
+    smp = _samples(seed, stream_id, rnd, n, O, S, cand_dev.data_ptr() if n else None)
+    Q = int(quantile_dev.numel()) if quantile_dev is not None else 0
+    _check(lib().fs_score_candidates_noalloc(int(K), int(B), int(G), _vp(bounds_dev), _vp(slo_dev),
+                                             _vp(demand_dev), _vp(quantile_dev), Q, C.byref(smp),
+                                             _vp(gap_dev), _vp(score_dev), _vp(gamma_t_dev),
+                                             _vp(best_dev), _stream(stream)))
 
 
 def fs_score_candidates_async(m: Model, cand_dev, O: int, S: int, seed: int, stream_id: int = 0,
