@@ -104,23 +104,90 @@ struct Items {
 
 // ---------------------------------------------------------------- arithmetic
 
+// x / lam, correctly rounded to nearest even, by Markstein's method
+// (P. Markstein, "Computation of elementary functions on the IBM RISC
+// System/6000 processor", IBM J. Res. Dev. 34(1), 1990): with r = RN(1/lam),
+// q0 = RN(x r) is within one unit in the last place of x / lam, the residual
+// x - lam q0 is exact in one fused multiply-add, and RN(q0 + (x - lam q0) r)
+// is the correctly rounded quotient, provided no step overflows or underflows.
+// Callers keep x in {0} or [2^-60, 2^60] and lam in [2^-60, 2^60]. Three inline
+// operations instead of the out-of-line IEEE divide, so independent divisions
+// overlap; the results are the IEEE quotients bit for bit.
+__device__ __forceinline__ float div_markstein(float x, float lam, float rlam) {
+  const float q0 = __fmul_rn(x, rlam);
+  const float e = __fmaf_rn(-lam, q0, x);
+  return __fmaf_rn(e, rlam, q0);
+}
+
+__device__ __forceinline__ bool in_markstein_range(float v) { return v >= 0x1p-60f && v <= 0x1p60f; }
+
 // Fulfilment of n replicas of capacity c: min(1, (n c) / lambda), Section 3
-// (Eqs. 2 and 4, r_i = x_i / lambda_i). One IEEE rounding per step, no FMA.
+// (Eqs. 2 and 4, r_i = x_i / lambda_i): one IEEE rounding for the product, one
+// for the quotient, then the cap at 1.
 __device__ __forceinline__ float fulfil(float n, float c, float lam) {
   float r = __fdiv_rn(__fmul_rn(n, c), lam);
   return fminf(r, 1.0f);
 }
 
+// The same value, the quotient by Markstein's method; rlam = RN(1/lam).
+// Requires n c in {0} or [2^-60, 2^60] and lam in [2^-60, 2^60].
+__device__ __forceinline__ float fulfil_fast(float n, float c, float lam, float rlam) {
+  return fminf(div_markstein(__fmul_rn(n, c), lam, rlam), 1.0f);
+}
+
+// The same value for any inputs: Markstein when the product and lambda are
+// in range, else the IEEE divide.
+__device__ __forceinline__ float fulfil_r(float n, float c, float lam, float rlam) {
+  const float x = __fmul_rn(n, c);
+  if ((x == 0.0f || in_markstein_range(x)) && in_markstein_range(lam))
+    return fminf(div_markstein(x, lam, rlam), 1.0f);
+  return fminf(__fdiv_rn(x, lam), 1.0f);
+}
+
+// Every n c with 1 <= n <= 32767 stays in {0} or [2^-60, 2^60].
+__device__ __forceinline__ bool row_in_range(float c, float lam) {
+  return (c == 0.0f || (c >= 0x1p-60f && c <= 0x1p44f)) && in_markstein_range(lam);
+}
+
 // Smallest n in [1, M] with fulfil(n, c) >= t, or 0 if none (fulfil is
-// nondecreasing in n under round-to-nearest).
-__device__ __forceinline__ int min_replicas(float t, float c, float lam, int M) {
-  if (M < 1 || fulfil((float)M, c, lam) < t) return 0;
+// nondecreasing in n under round-to-nearest). The real-valued answer is
+// t lambda / c; the rounded fulfilment differs from n c / lambda by at most
+// two roundings (relative 2^-22), so for n <= 32767 the answer is within one
+// of ceil(t lambda / c) even with an approximate division. Five candidates
+// around that estimate are tested at once; a plain bisection is kept for the
+// case the bracket does not hold.
+template <bool FAST>
+__device__ __forceinline__ int min_replicas_impl(float t, float c, float lam, float rlam, int M) {
+  auto f = [&](int n) { return FAST ? fulfil_fast((float)n, c, lam, rlam) : fulfil((float)n, c, lam); };
+  const float fM = f(M);
+  const float y = __fdividef(__fmul_rn(t, lam), c);  // estimate only
+  if (!(fM >= t)) return 0;  // also covers c == 0
+  int n = y < (float)M ? (int)ceilf(y) : M;
+  n = max(n, 1);
+  const int a = max(1, n - 2), b = min(M, n + 2);
+  const bool left = a == 1 || f(a - 1) < t;
+  const bool right = f(b) >= t;
+  if (left && right) {
+    int r = b;
+#pragma unroll
+    for (int k = 3; k >= 0; --k) {
+      const int v = a + k;
+      if (v < b && f(v) >= t) r = v;
+    }
+    return r;
+  }
   int lo = 1, hi = M;
   while (lo < hi) {
-    int mid = (lo + hi) >> 1;
-    if (fulfil((float)mid, c, lam) >= t) hi = mid; else lo = mid + 1;
+    const int mid = (lo + hi) >> 1;
+    if (f(mid) >= t) hi = mid; else lo = mid + 1;
   }
   return lo;
+}
+
+__device__ __forceinline__ int min_replicas(float t, float c, float lam, float rlam, int M) {
+  if (M < 1) return 0;
+  return row_in_range(c, lam) ? min_replicas_impl<true>(t, c, lam, rlam, M)
+                              : min_replicas_impl<false>(t, c, lam, rlam, M);
 }
 
 // Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11): ten rounds of the 4x32

@@ -40,7 +40,7 @@ struct Eval {
   int P;   // kCostInf if no other row of class ie covers t
 };
 
-__device__ __forceinline__ Eval warp_eval_excl(float t, const float* sC, const float* lam,
+__device__ __forceinline__ Eval warp_eval_excl(float t, const float* sC, const float* sLam, const float* sRl,
                                                const Dims& d, int rr, int ie, int lane) {
   int R = 0;
   bool rinf = false;
@@ -49,7 +49,7 @@ __device__ __forceinline__ Eval warp_eval_excl(float t, const float* sC, const f
     const int rho = base + lane;
     int cost = kCostInf;
     if (rho < d.K4 && rho != rr) {
-      const int n = min_replicas(t, sC[rho], lam[rho >> 2], d.M[rho & 3]);
+      const int n = min_replicas(t, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.M[rho & 3]);
       if (n) cost = n << (rho & 3);
     }
     cost = min(cost, __shfl_xor_sync(0xffffffffu, cost, 1));
@@ -71,8 +71,8 @@ __device__ __forceinline__ int replicas_left(const Eval& e, int jr, const Dims& 
   return (e.A >= (1 << jr)) ? min(e.A >> jr, d.M[jr]) : 0;
 }
 
-__device__ __forceinline__ bool feasible_at(const Eval& e, int m, float C, float t, float lam) {
-  return (e.P < kCostInf && e.P <= e.A) || (m >= 1 && fulfil((float)m, C, lam) >= t);
+__device__ __forceinline__ bool feasible_at(const Eval& e, int m, float C, float t, float lam, float rl) {
+  return (e.P < kCostInf && e.P <= e.A) || (m >= 1 && fulfil_r((float)m, C, lam, rl) >= t);
 }
 
 __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan pl, float* tables,
@@ -81,8 +81,8 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
   float* sC = reinterpret_cast<float*>(smraw);  // [256]
   float* sTh = sC + 256;                          // [theta_cap]
   __shared__ float s_cx, s_cmax;
-  __shared__ int s_bx, s_b0, s_b1;
-  const Dims d = set.d;
+  __shared__ int s_bx;
+  const Dims& d = set.d;  // kernel-parameter space: d.M[j] reads need no local copy
   const int item = blockIdx.x >> 1, sigma = blockIdx.x & 1;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = blockDim.x >> 5;
   pdl_wait();     // thresholds, rows and the zeroed lmax come from k_solve
@@ -101,7 +101,12 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
     return;
   }
   const int rr = cell / d.B, be = cell - rr * d.B, ie = rr >> 2, jr = rr & 3;
-  const float lam = set.lam[ie], L = set.slo[ie];
+  const float lam = set.lam[ie], L = set.slo[ie], rl = __frcp_rn(lam);
+  __shared__ float sLam[FS_MAX_CLASSES], sRl[FS_MAX_CLASSES];  // demand and RN(1/demand)
+  if (tid < d.K) {
+    sLam[tid] = set.lam[tid];
+    sRl[tid] = __frcp_rn(set.lam[tid]);
+  }
   const size_t ps = (size_t)p * 2 + sigma;
   const int total = set.ntheta[ps];
   const float* th_g = set.theta + ps * d.theta_cap;
@@ -144,28 +149,58 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
   const float cx = s_cx, cmax = s_cmax;
   const int msent = d.K == 1 ? d.M[jr] : 0;  // above every threshold only a lone class can go on
 
-  // b0: last index feasible at Cexcl; b1: last index feasible at max(Cexcl, cap_hi)
-  if (warp == 0) {
-    int lo = -1, hi = total;
-    while (hi - lo > 1) {
-      const int mid = (lo + hi) >> 1;
-      const Eval e = warp_eval_excl(sTh[mid], sC, set.lam, d, rr, ie, lane);
-      if (feasible_at(e, replicas_left(e, jr, d), cx, sTh[mid], lam)) lo = mid; else hi = mid;
-    }
-    const int b0 = lo;
-    hi = total;
-    while (hi - lo > 1) {
-      const int mid = (lo + hi) >> 1;
-      const Eval e = warp_eval_excl(sTh[mid], sC, set.lam, d, rr, ie, lane);
-      if (feasible_at(e, replicas_left(e, jr, d), cmax, sTh[mid], lam)) lo = mid; else hi = mid;
-    }
-    if (lane == 0) {
-      s_b0 = b0;
-      s_b1 = lo;
-    }
+  // b0: last index feasible at Cexcl; b1: last index feasible at max(Cexcl, cap_hi).
+  // Joint search: each round every warp probes one index; a probe answers for
+  // both capacities, and the warps split whichever intervals are still open.
+  __shared__ int s_iv[4], s_probe[8];
+  if (tid == 0) {
+    s_iv[0] = -1;
+    s_iv[1] = total;
+    s_iv[2] = -1;
+    s_iv[3] = total;
   }
   __syncthreads();
-  const int b0 = s_b0, b1 = s_b1;
+  for (;;) {
+    const int lo0 = s_iv[0], hi0 = s_iv[1], lo1 = s_iv[2], hi1 = s_iv[3];
+    const bool open0 = hi0 - lo0 > 1, open1 = hi1 - lo1 > 1;
+    if (!open0 && !open1) break;
+    int lo, hi, part, parts;
+    if (open0 && open1) {
+      const bool first = warp < nwarp / 2;
+      lo = first ? lo0 : lo1;
+      hi = first ? hi0 : hi1;
+      parts = nwarp / 2 + 1;
+      part = (first ? warp : warp - nwarp / 2) + 1;
+    } else {
+      lo = open0 ? lo0 : lo1;
+      hi = open0 ? hi0 : hi1;
+      parts = nwarp + 1;
+      part = warp + 1;
+    }
+    int k = lo + (int)(((long long)part * (hi - lo)) / parts);
+    k = max(lo + 1, min(hi - 1, k));
+    const Eval e = warp_eval_excl(sTh[k], sC, sLam, sRl, d, rr, ie, lane);
+    const int m = replicas_left(e, jr, d);
+    if (lane == 0) {
+      s_probe[2 * warp] = k;
+      s_probe[2 * warp + 1] = (feasible_at(e, m, cx, sTh[k], lam, rl) ? 1 : 0) | (feasible_at(e, m, cmax, sTh[k], lam, rl) ? 2 : 0);
+    }
+    __syncthreads();
+    if (tid == 0) {
+      int a0 = lo0, c0 = hi0, a1 = lo1, c1 = hi1;
+      for (int w = 0; w < nwarp; ++w) {
+        const int kk = s_probe[2 * w], f = s_probe[2 * w + 1];
+        if (f & 1) a0 = max(a0, kk); else c0 = min(c0, kk);
+        if (f & 2) a1 = max(a1, kk); else c1 = min(c1, kk);
+      }
+      s_iv[0] = a0;
+      s_iv[1] = c0;
+      s_iv[2] = a1;
+      s_iv[3] = c1;
+    }
+    __syncthreads();
+  }
+  const int b0 = s_iv[0], b1 = s_iv[2];
   const int Lt = b1 - b0;
   // arrays padded to P = pow2 >= Lt + 1 entries (+inf beyond Lt), so the
   // scenario search needs no bound checks; at least 4 for 16-byte copies
@@ -185,20 +220,32 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
     const int k = b0 + 1 + u;
     int m;
     if (k < total) {
-      const Eval e = warp_eval_excl(sTh[k], sC, set.lam, d, rr, ie, lane);
+      const Eval e = warp_eval_excl(sTh[k], sC, sLam, sRl, d, rr, ie, lane);
       m = replicas_left(e, jr, d);
     } else {
       m = msent;
     }
     if (u < Lt) {
-      // smallest capacity in (cx, cmax] at which f(m, C) >= theta_k: 32-ary search on the
-      // bit patterns of nonnegative floats (ordered like the values)
+      // smallest capacity in (cx, cmax] at which f(m, C) >= theta_k, on the bit
+      // patterns of nonnegative floats (ordered like the values). First the 32
+      // patterns around the real solution t lambda / m, one per lane; if the
+      // answer is not among them, a 32-ary search over the whole interval.
       const float t = sTh[k];
-      uint32_t lo = __float_as_uint(cx), hi = __float_as_uint(cmax);
+      const uint32_t bx = __float_as_uint(cx), bmax = __float_as_uint(cmax);
+      const float c0 = __fdiv_rn(__fmul_rn(t, lam), (float)m);
+      const long long pl_ = (long long)__float_as_uint(c0) - 16 + lane;
+      const uint32_t pt0 = pl_ < 0 ? 0u : (uint32_t)pl_;
+      const bool ok0 = pt0 > bx && (pt0 >= bmax || fulfil_r((float)m, __uint_as_float(pt0), lam, rl) >= t);
+      const uint32_t bal0 = __ballot_sync(0xffffffffu, ok0);
+      uint32_t lo = bx, hi = bmax;
+      if (bal0 != 0u && (bal0 & 1u) == 0u) {  // lane 0 fails, some lane passes: the first passing lane
+        hi = __shfl_sync(0xffffffffu, pt0, __ffs(bal0) - 1);
+        lo = hi - 1;
+      }
       while (hi - lo > 1) {
         const uint32_t span = hi - lo;
         const uint32_t pt = lo + (uint32_t)(((uint64_t)(lane + 1) * span) >> 5);
-        const bool ok = fulfil((float)m, __uint_as_float(pt), lam) >= t;
+        const bool ok = fulfil_r((float)m, __uint_as_float(pt), lam, rl) >= t;
         const uint32_t bal = __ballot_sync(0xffffffffu, ok);
         const int l = __ffs(bal) - 1;  // lane 31 tests hi, which is feasible
         const uint32_t nhi = __shfl_sync(0xffffffffu, pt, l);
@@ -244,11 +291,15 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
 // padded with +inf to a power of two above the entry count, so the
 // branch-free search needs no bound checks; step0 = half that power.
 __device__ __forceinline__ float tstar_of(float C, const float* kap, const float* tht, const float* mn,
-                                          int step0, float th_base, float m_first, float lam) {
+                                          int step0, float th_base, float m_first, float lam,
+                                          float rlam) {
   int pos = 0;
   for (int step = step0; step > 0; step >>= 1) pos += kap[pos + step - 1] <= C ? step : 0;
   const float thb = pos ? tht[pos - 1] : th_base;
   const float m = pos ? mn[pos - 1] : m_first;
+  // the row term is rarely needed; the out-of-line IEEE divide keeps it behind
+  // the branch (an inline quotient would be computed for every scenario)
+  (void)rlam;
   const float tr = m >= 1.0f ? fulfil(m, C, lam) : 0.0f;
   return tr > thb ? tr : thb;
 }
@@ -268,7 +319,7 @@ __device__ void dump_choices(float t, const Set& set, size_t ps, int rr, float C
         const float c = rho == rr ? C : set.rowC[ps * d.K4 + rho];
         const int b = rho == rr ? bC : set.rowB[ps * d.K4 + rho];
         if (b < 0) continue;
-        const int n = min_replicas(t, c, set.lam[i], d.M[j]);
+        const int n = min_replicas(t, c, set.lam[i], __frcp_rn(set.lam[i]), d.M[j]);
         if (n && (n << j) < best) {
           best = n << j;
           bj = j;
@@ -304,7 +355,7 @@ __device__ __forceinline__ uint64_t run_piece(const Set& set, const Plan& pl, in
   const int st0 = __float_as_int(h0[H_STEP0]), st1 = __float_as_int(h1[H_STEP0]);
   const float thb0 = h0[H_TH_BASE], mf0 = h0[H_M_FIRST], cx0 = h0[H_CX];
   const float thb1 = h1[H_TH_BASE], mf1 = h1[H_M_FIRST], cx1 = h1[H_CX];
-  const float lam = h0[H_LAM];
+  const float lam = h0[H_LAM], rlam = __frcp_rn(lam);
   const int cell = __float_as_int(h0[H_CELL]), p = __float_as_int(h0[H_P]);
   const PhiloxKeys keys = philox_keys(pl.key0, pl.key1 ^ (pl.stream_base + (uint32_t)p));
   const uint32_t sh = (uint32_t)pl.sh;
@@ -333,8 +384,8 @@ __device__ __forceinline__ uint64_t run_piece(const Set& set, const Plan& pl, in
       }
       const float C0 = gate ? fmaxf(cx0, cy) : cx0;
       const float C1 = gate ? fmaxf(cx1, cy) : cx1;
-      const float t0 = tstar_of(C0, kap0, tht0, mn0, st0, thb0, mf0, lam);
-      const float t1 = tstar_of(C1, kap1, tht1, mn1, st1, thb1, mf1, lam);
+      const float t0 = tstar_of(C0, kap0, tht0, mn0, st0, thb0, mf0, lam, rlam);
+      const float t1 = tstar_of(C1, kap1, tht1, mn1, st1, thb1, mf1, lam, rlam);
       const uint64_t gf = fixed40(__fsub_rn(t1, t0));
       acc += (h == 0 || s < S) ? gf : 0ull;  // the last call may serve fewer than four samples
       if (DUMP && (h == 0 || s < S)) {
@@ -399,7 +450,7 @@ __global__ void __launch_bounds__(kScoreThreads, 5) k_score(Set set, Items it, P
   const int stage_floats = qwin + 2 * tstride;
   float* stage0 = reinterpret_cast<float*>(smraw + 16);
   __shared__ int s_lcopy;
-  const Dims d = set.d;
+  const Dims& d = set.d;  // kernel-parameter space: d.M[j] reads need no local copy
   const int tid = threadIdx.x, lane = tid & 31;
 
   pdl_wait();  // tables, zeroed sums and lmax come from k_prep

@@ -42,7 +42,7 @@ __global__ void k_qtable(float* qn, int Q) {
 
 // Total GPUs of the cheapest per-class covers of threshold t, or kCostInf if
 // some class has no cover. Called by a whole warp; rows rho = 4 i + j.
-__device__ __forceinline__ int warp_total_cost(float t, const float* sC, const float* lam,
+__device__ __forceinline__ int warp_total_cost(float t, const float* sC, const float* sLam, const float* sRl,
                                                const Dims& d, int lane) {
   int total = 0;
   bool inf = false;
@@ -51,7 +51,7 @@ __device__ __forceinline__ int warp_total_cost(float t, const float* sC, const f
     int cost = kCostInf;
     if (rho < d.K4) {
       const int j = rho & 3;
-      const int n = min_replicas(t, sC[rho], lam[rho >> 2], d.M[j]);
+      const int n = min_replicas(t, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.M[j]);
       if (n) cost = n << j;
     }
     cost = min(cost, __shfl_xor_sync(0xffffffffu, cost, 1));
@@ -67,7 +67,7 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
                                                          const float* tail_x, fs_allocation* out_x,
                                                          int write_theta) {
   extern __shared__ __align__(16) unsigned char smraw[];
-  const Dims d = set.d;
+  const Dims& d = set.d;  // kernel-parameter space: d.M[j] reads need no local copy
   const int r = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = blockDim.x >> 5;
   if (r == 0 && tid == 0 && set.lmax) *set.lmax = 0;  // before any early exit
@@ -102,6 +102,11 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   float* sTheta = reinterpret_cast<float*>(sMisc + 8);    // [pow2 >= theta_cap]
 
   // 1. rows: key = (capacity bits, ~bin) of the best SLO-feasible bin; 0 = none
+  __shared__ float sLam[FS_MAX_CLASSES], sRl[FS_MAX_CLASSES];  // demand and RN(1/demand)
+  if (tid < d.K) {
+    sLam[tid] = set.lam[tid];
+    sRl[tid] = __frcp_rn(set.lam[tid]);
+  }
   for (int rho = tid; rho < d.K4; rho += blockDim.x) sKey[rho] = 0ull;
   if (tid < 8) sMisc[tid] = 0;
   __syncthreads();
@@ -121,15 +126,15 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
     sC[rho] = best;
     sB[rho] = bb;
     const int i = rho >> 2, j = rho & 3;
-    const float lam = set.lam[i];
+    const float lam = sLam[i], rl = sRl[i];
     const int M = d.M[j];
     int n0 = 0, len = 0;
     if (bb >= 0) {
       atomicOr(reinterpret_cast<unsigned int*>(&sMisc[2 + (i >> 5)]), 1u << (i & 31));
       if (M >= 1) {
-        n0 = min_replicas(__int_as_float(1), best, lam, M);  // first positive fulfilment
+        n0 = min_replicas(__int_as_float(1), best, lam, rl, M);  // first positive fulfilment
         if (n0) {
-          const int ns = min_replicas(1.0f, best, lam, M);   // first full fulfilment
+          const int ns = min_replicas(1.0f, best, lam, rl, M);   // first full fulfilment
           len = ns ? ns : M;
         }
       }
@@ -172,25 +177,54 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
         if (sOff[mid] <= x) lo = mid; else hi = mid - 1;
       }
       const int n = sN0[lo] + (x - sOff[lo]);
-      v = fulfil((float)n, sC[lo], set.lam[lo >> 2]);
+      v = fulfil_r((float)n, sC[lo], sLam[lo >> 2], sRl[lo >> 2]);
     }
     sTheta[x] = v;
   }
   __syncthreads();
-  for (int k = 2; k <= P2; k <<= 1) {
-    for (int jj = k >> 1; jj > 0; jj >>= 1) {
-      for (int x = tid; x < P2; x += blockDim.x) {
-        const int y = x ^ jj;
-        if (y > x) {
-          const float a = sTheta[x], b = sTheta[y];
-          const bool up = (x & k) == 0;
-          if ((a > b) == up && a != b) {
-            sTheta[x] = b;
-            sTheta[y] = a;
+  if (P2 <= 64) {
+    // small lists: one warp sorts 64 values held two per lane (bitonic network,
+    // partners by __shfl_xor_sync), with no block barriers
+    if (warp == 0) {
+      const float inf = __int_as_float(0x7f800000);
+      float r[2] = {lane < P2 ? sTheta[lane] : inf, lane + 32 < P2 ? sTheta[lane + 32] : inf};
+      for (int k = 2; k <= 64; k <<= 1) {
+        for (int jj = k >> 1; jj > 0; jj >>= 1) {
+          if (jj == 32) {  // partners share a lane; k == 64, ascending
+            const float lo = fminf(r[0], r[1]), hi = fmaxf(r[0], r[1]);
+            r[0] = lo;
+            r[1] = hi;
+          } else {
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              const int i = lane + 32 * h;
+              const float pv = __shfl_xor_sync(0xffffffffu, r[h], jj);
+              const bool keep_min = ((i & jj) == 0) == ((i & k) == 0);
+              r[h] = keep_min ? fminf(r[h], pv) : fmaxf(r[h], pv);
+            }
           }
         }
       }
-      __syncthreads();
+      if (lane < P2) sTheta[lane] = r[0];
+      if (lane + 32 < P2) sTheta[lane + 32] = r[1];
+    }
+    __syncthreads();
+  } else {
+    for (int k = 2; k <= P2; k <<= 1) {
+      for (int jj = k >> 1; jj > 0; jj >>= 1) {
+        for (int x = tid; x < P2; x += blockDim.x) {
+          const int y = x ^ jj;
+          if (y > x) {
+            const float a = sTheta[x], b = sTheta[y];
+            const bool up = (x & k) == 0;
+            if ((a > b) == up && a != b) {
+              sTheta[x] = b;
+              sTheta[y] = a;
+            }
+          }
+        }
+        __syncthreads();
+      }
     }
   }
 
@@ -206,7 +240,7 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
     const int span = hi - lo;
     int kp = lo + (int)(((long long)(warp + 1) * span) / (nwarp + 1));
     kp = max(lo + 1, min(hi - 1, kp));
-    const int cost = warp_total_cost(sTheta[kp], sC, set.lam, d, lane);
+    const int cost = warp_total_cost(sTheta[kp], sC, sLam, sRl, d, lane);
     if (lane == 0) sProbe[warp] = (cost <= d.G) ? kp : -(kp + 1);
     __syncthreads();
     if (tid == 0) {
@@ -223,34 +257,35 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   const int kstar = sMisc[0];
   const float tstar = kstar >= 0 ? sTheta[kstar] : 0.0f;
 
-  // 4. choice at t*
-  if (tid < FS_MAX_CLASSES) {
-    const int i = tid;
-    int8_t tp = 0;
-    int16_t bin = -1, reps = 0;
-    float f = 0.0f;
-    int cost_i = 0;
-    if (i < d.K && tstar > 0.0f) {
-      int best = kCostInf, bj = -1, bn = 0;
-      for (int j = 0; j < kT; ++j) {
-        const int n = min_replicas(tstar, sC[4 * i + j], set.lam[i], d.M[j]);
-        if (n && (n << j) < best) {
-          best = n << j;
-          bj = j;
-          bn = n;
-        }
-      }
-      tp = (int8_t)(1 << bj);
-      bin = (int16_t)sB[4 * i + bj];
-      reps = (int16_t)bn;
-      f = fulfil((float)bn, sC[4 * i + bj], set.lam[i]);
-      cost_i = best;
+  // 4. choice at t*: every row's cheapest cover in parallel (thread = row), then
+  // per class the cheapest row over its four TP lanes, lower TP on ties
+  {
+    const int rho = tid;  // K4 <= 256 = blockDim
+    int key = 0x7fffffff;
+    if (rho < d.K4 && tstar > 0.0f) {
+      const int n = min_replicas(tstar, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.M[rho & 3]);
+      if (n) key = ((n << (rho & 3)) << 2) | (rho & 3);
     }
-    out->tp[i] = tp;
-    out->bin[i] = bin;
-    out->replicas[i] = reps;
-    out->fulfil[i] = f;
-    if (i < d.K) atomicAdd(&sMisc[4], cost_i);
+    key = min(key, __shfl_xor_sync(0xffffffffu, key, 1));
+    key = min(key, __shfl_xor_sync(0xffffffffu, key, 2));
+    if ((tid & 3) == 0) {
+      const int i = tid >> 2;
+      int8_t tp = 0;
+      int16_t bin = -1, reps = 0;
+      float f = 0.0f;
+      if (i < d.K && key != 0x7fffffff) {
+        const int bj = key & 3, cost_i = key >> 2, bn = cost_i >> bj;
+        tp = (int8_t)(1 << bj);
+        bin = (int16_t)sB[4 * i + bj];
+        reps = (int16_t)bn;
+        f = fulfil_r((float)bn, sC[4 * i + bj], sLam[i], sRl[i]);
+        atomicAdd(&sMisc[4], cost_i);
+      }
+      out->tp[i] = tp;
+      out->bin[i] = bin;
+      out->replicas[i] = reps;
+      out->fulfil[i] = f;
+    }
   }
   __syncthreads();
   if (tid == 0) {
