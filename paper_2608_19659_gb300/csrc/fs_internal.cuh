@@ -61,6 +61,7 @@ enum : uint32_t {
 struct Dims {
   int K, B, G, Q, cells, K4;
   int M[kT];            // floor(G / tau)
+  float Mf[kT];         // the same as floats
   int theta_cap;        // K * sum M: most thresholds one realisation can have
   int slot_floats;      // stride of one (item, sigma) table
   int lcap;             // table entries a slot can hold: pow2 >= theta_cap + 1, at least 4
@@ -156,36 +157,38 @@ __device__ __forceinline__ bool row_in_range(float c, float lam) {
 // of ceil(t lambda / c) even with an approximate division. Five candidates
 // around that estimate are tested at once; a plain bisection is kept for the
 // case the bracket does not hold.
+// Replica counts are handled as floats (integers up to 32767 are exact there),
+// so that no integer/float conversion sits on the dependent chain; M is the
+// replica cap as a float.
 template <bool FAST>
-__device__ __forceinline__ int min_replicas_impl(float t, float c, float lam, float rlam, int M) {
-  auto f = [&](int n) { return FAST ? fulfil_fast((float)n, c, lam, rlam) : fulfil((float)n, c, lam); };
+__device__ __forceinline__ int min_replicas_impl(float t, float c, float lam, float rlam, float M) {
+  auto f = [&](float n) { return FAST ? fulfil_fast(n, c, lam, rlam) : fulfil(n, c, lam); };
   const float fM = f(M);
-  const float y = __fdividef(__fmul_rn(t, lam), c);  // estimate only
+  const float y = ceilf(__fdividef(__fmul_rn(t, lam), c));  // estimate only
   if (!(fM >= t)) return 0;  // also covers c == 0
-  int n = y < (float)M ? (int)ceilf(y) : M;
-  n = max(n, 1);
-  const int a = max(1, n - 2), b = min(M, n + 2);
-  const bool left = a == 1 || f(a - 1) < t;
+  const float n = fminf(fmaxf(y, 1.0f), M);
+  const float a = fmaxf(1.0f, n - 2.0f), b = fminf(M, n + 2.0f);
+  const bool left = a == 1.0f || f(a - 1.0f) < t;
   const bool right = f(b) >= t;
   if (left && right) {
-    int r = b;
+    float r = b;
 #pragma unroll
     for (int k = 3; k >= 0; --k) {
-      const int v = a + k;
+      const float v = a + (float)k;
       if (v < b && f(v) >= t) r = v;
     }
-    return r;
+    return (int)r;
   }
-  int lo = 1, hi = M;
+  int lo = 1, hi = (int)M;
   while (lo < hi) {
     const int mid = (lo + hi) >> 1;
-    if (f(mid) >= t) hi = mid; else lo = mid + 1;
+    if (f((float)mid) >= t) hi = mid; else lo = mid + 1;
   }
   return lo;
 }
 
-__device__ __forceinline__ int min_replicas(float t, float c, float lam, float rlam, int M) {
-  if (M < 1) return 0;
+__device__ __forceinline__ int min_replicas(float t, float c, float lam, float rlam, float M) {
+  if (!(M >= 1.0f)) return 0;
   return row_in_range(c, lam) ? min_replicas_impl<true>(t, c, lam, rlam, M)
                               : min_replicas_impl<false>(t, c, lam, rlam, M);
 }

@@ -49,7 +49,7 @@ __device__ __forceinline__ Eval warp_eval_excl(float t, const float* sC, const f
     const int rho = base + lane;
     int cost = kCostInf;
     if (rho < d.K4 && rho != rr) {
-      const int n = min_replicas(t, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.M[rho & 3]);
+      const int n = min_replicas(t, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[rho & 3]);
       if (n) cost = n << (rho & 3);
     }
     cost = min(cost, __shfl_xor_sync(0xffffffffu, cost, 1));
@@ -319,7 +319,7 @@ __device__ void dump_choices(float t, const Set& set, size_t ps, int rr, float C
         const float c = rho == rr ? C : set.rowC[ps * d.K4 + rho];
         const int b = rho == rr ? bC : set.rowB[ps * d.K4 + rho];
         if (b < 0) continue;
-        const int n = min_replicas(t, c, set.lam[i], __frcp_rn(set.lam[i]), d.M[j]);
+        const int n = min_replicas(t, c, set.lam[i], __frcp_rn(set.lam[i]), d.Mf[j]);
         if (n && (n << j) < best) {
           best = n << j;
           bj = j;

@@ -51,7 +51,7 @@ __device__ __forceinline__ int warp_total_cost(float t, const float* sC, const f
     int cost = kCostInf;
     if (rho < d.K4) {
       const int j = rho & 3;
-      const int n = min_replicas(t, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.M[j]);
+      const int n = min_replicas(t, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[j]);
       if (n) cost = n << j;
     }
     cost = min(cost, __shfl_xor_sync(0xffffffffu, cost, 1));
@@ -128,13 +128,14 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
     const int i = rho >> 2, j = rho & 3;
     const float lam = sLam[i], rl = sRl[i];
     const int M = d.M[j];
+    const float Mf = d.Mf[j];
     int n0 = 0, len = 0;
     if (bb >= 0) {
       atomicOr(reinterpret_cast<unsigned int*>(&sMisc[2 + (i >> 5)]), 1u << (i & 31));
       if (M >= 1) {
-        n0 = min_replicas(__int_as_float(1), best, lam, rl, M);  // first positive fulfilment
+        n0 = min_replicas(__int_as_float(1), best, lam, rl, Mf);  // first positive fulfilment
         if (n0) {
-          const int ns = min_replicas(1.0f, best, lam, rl, M);   // first full fulfilment
+          const int ns = min_replicas(1.0f, best, lam, rl, Mf);   // first full fulfilment
           len = ns ? ns : M;
         }
       }
@@ -263,7 +264,7 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
     const int rho = tid;  // K4 <= 256 = blockDim
     int key = 0x7fffffff;
     if (rho < d.K4 && tstar > 0.0f) {
-      const int n = min_replicas(tstar, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.M[rho & 3]);
+      const int n = min_replicas(tstar, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[rho & 3]);
       if (n) key = ((n << (rho & 3)) << 2) | (rho & 3);
     }
     key = min(key, __shfl_xor_sync(0xffffffffu, key, 1));
