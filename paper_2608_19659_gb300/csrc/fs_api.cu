@@ -187,6 +187,8 @@ Plan make_plan(const fs_model* m, const fs_samples* s, int n_items) {
   pl.w = log2i(pl.W);
   pl.sh = 16 - pl.w;
   pl.calls = (s->S + 3) / 4;
+  pl.Wp = 4 + ((pl.W + 3) & ~3);
+  pl.item_floats = 2LL * m->d.slot_floats + (long long)s->O * pl.Wp;
   (void)n_items;
   return pl;
 }
@@ -194,7 +196,9 @@ Plan make_plan(const fs_model* m, const fs_samples* s, int n_items) {
 int ensure_items(fs_model* m, int n, int O) {
   int rc;
   if ((rc = m->cand.ensure((size_t)std::max(n, 1) * 4, "candidate list"))) return rc;
-  if ((rc = m->tables.ensure((size_t)std::max(n, 1) * 2 * m->d.slot_floats * 4, "candidate tables"))) return rc;
+  const int W = m->d.Q / O, Wp = 4 + ((W + 3) & ~3);
+  const size_t item_floats = 2 * (size_t)m->d.slot_floats + (size_t)O * Wp;
+  if ((rc = m->tables.ensure((size_t)std::max(n, 1) * item_floats * 4, "candidate records"))) return rc;
   if ((rc = m->sums.ensure((size_t)std::max(n, 1) * O * 8, "sums"))) return rc;
   if ((rc = m->outs.ensure((size_t)std::max(n, 1) * 16 + 64, "outputs"))) return rc;
   return FS_OK;
@@ -225,7 +229,7 @@ int run_score(fs_model* m, const fs_samples* smp, const int32_t* cand_dev, doubl
   if (phases) FS_CUDA(cudaEventRecord(ev[0], s), "record timing event");
   FS_CUDA(launch_solve(m->set, 2, nullptr, nullptr, nullptr, true, m->lc, s), "launch solve");
   if (phases) FS_CUDA(cudaEventRecord(ev[1], s), "record timing event");
-  FS_CUDA(launch_prep(m->set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, m->lc, s), "launch prep");
+  FS_CUDA(launch_prep(m->set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, true, m->lc, s), "launch prep");
   if (timed) FS_CUDA(cudaEventRecord(ev[2], s), "record timing event");
   FS_CUDA(launch_score(m->set, it, pl, (const float*)m->tables.p, (uint64_t*)m->sums.p, dump,
                        fs_dump_stride(m), m->sm_count, m->lc, s),
@@ -315,7 +319,7 @@ int fs_load_model(const fs_bounds* b, const float* slo, const float* demand, int
   const size_t o_bounds = take(16 * (size_t)cells), o_rev = take(cells);
   const size_t o_theta = take(8 * (size_t)d.theta_cap), o_nth = take(8);
   const size_t o_rowc = take(8 * (size_t)d.K4), o_rowb = take(8 * (size_t)d.K4);
-  const size_t o_base = take(2 * sizeof(fs_allocation)), o_status = take(4), o_lmax = take(4);
+  const size_t o_base = take(2 * sizeof(fs_allocation)), o_status = take(4), o_work = take(8);
   rc = m->fixed.ensure(off, "model state");
   if (rc) {
     delete m;
@@ -336,7 +340,7 @@ int fs_load_model(const fs_bounds* b, const float* slo, const float* demand, int
   s.rowB = (int*)(base + o_rowb);
   s.base = (fs_allocation*)(base + o_base);
   s.status = (uint32_t*)(base + o_status);
-  s.lmax = (int*)(base + o_lmax);
+  s.work = (unsigned long long*)(base + o_work);
   s.skip = nullptr;
 
   m->h_lam.assign(demand, demand + K);
@@ -609,7 +613,7 @@ int fs_replay(fs_model* m, const fs_replay_spec* sp, int32_t* rounds, int32_t* s
       it.off = nullptr;
       fs_samples smp{sp->seed, 0, (uint32_t)r, n_items, sp->O, sp->S, 0, nullptr};
       const Plan pl = make_plan(m, &smp, n_items);
-      FS_CUDA(launch_prep(set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, m->lc, s), "launch prep");
+      FS_CUDA(launch_prep(set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, false, m->lc, s), "launch prep");
       FS_CUDA(launch_score(set, it, pl, (const float*)m->tables.p, (uint64_t*)m->sums.p, nullptr, 0, m->sm_count,
                            m->lc, s),
               "launch score");

@@ -61,6 +61,7 @@ __device__ inline Best finalize_problem(const Set& set, const Items& it, const P
   Best b{0, 0, -1};
   for (int q = beg + tid; q < end; q += blockDim.x) {
     long long tot = 0;
+#pragma unroll 8
     for (int o = 0; o < pl.O; ++o) tot += (long long)sums[(size_t)q * pl.O + o];
     const long long sc = gfix * n - tot;
     if (gap) gap[q] = fixed_mean((unsigned long long)tot, n, log2n);

@@ -10,9 +10,13 @@
 //   rowC     [P][2][K*4]   f32   best SLO-feasible capacity per (class, TP)
 //   rowB     [P][2][K*4]   i32   its bin (-1: none)
 //   base     [P][2]        fs_allocation
-//   lmax     [1]           i32   longest padded candidate table of the call
-// Per scoring call (items = (problem, candidate cell) pairs):
-//   tables   [items][2][slot_floats] f32   per-candidate threshold tables
+//   work     [1]           u64   chunk counter of the Monte-Carlo kernel
+// Per scoring call (items = (problem, candidate cell) pairs), one record of
+// item_floats = 2 slot_floats + O Wp floats per item:
+//   [2][slot_floats] f32   threshold tables of the two realisations
+//   [O][Wp]          f32   per outcome: the gate position (int) and three pad
+//                          words, then the outcome's W quantiles mapped into the
+//                          candidate's capacity interval (Wp = 4 + W rounded up to 4)
 //   sums     [items][O]    u64 (int64 fixed point, 2^-40)
 #pragma once
 
@@ -28,7 +32,7 @@ constexpr int kCostInf = 0x3FFFFFFF;  // "no option covers the threshold"
 constexpr int kSolveThreads = 256;
 constexpr int kPrepThreads = 128;
 constexpr int kScoreThreads = 256;
-constexpr int kTableHeader = 16;      // floats before the three table arrays
+constexpr int kTableHeader = 20;      // floats before the three table arrays (16-byte multiple)
 constexpr int kSmemTableCap = 256;    // table entries staged in shared memory per realisation (pow2)
 
 // Table header words (floats unless noted).
@@ -46,6 +50,8 @@ enum : int {
   H_CELL = 13,    // candidate cell (int)
   H_P = 14,       // problem (int)
   H_STEP0 = 15,   // first step of the table search, P/2 with P = pow2 >= L + 1 (int, 0 if L = 0)
+  H_ROW = 16,     // 1 if row r can buy a replica at some reachable threshold (int)
+  H_FAST = 17,    // 1 if every reachable row-term quotient is in Markstein's range (int)
 };
 
 enum : int { CAP_LO = 0, CAP_HI = 1, TAIL_LO = 2, TAIL_HI = 3 };
@@ -81,7 +87,7 @@ struct Set {
   int* rowB;            // [P][2][K4] bin of rowC, -1 = no SLO-feasible bin
   fs_allocation* base;  // [P][2]
   uint32_t* status;
-  int* lmax;            // [1]
+  unsigned long long* work;  // [1] chunk counter, zeroed by k_prep
   const int* skip;      // [P] or nullptr: base solves skip problems with skip[p] >= 0
 };
 
@@ -94,6 +100,8 @@ struct Plan {
   int O, S, W, w;       // W = Q / O quantiles per stratum, w = log2(W) <= 16
   int sh;               // 16 - w: a 16-bit field's top w bits are field >> sh
   int calls;            // ceil(S / 4) Philox calls per (candidate, outcome)
+  int Wp;               // floats per mapped outcome window: 4 + W rounded up to 4
+  long long item_floats;  // floats per item record: 2 slot_floats + O Wp
 };
 
 struct Items {
@@ -348,8 +356,10 @@ cudaError_t launch_qtable(float* qn, int Q, cudaStream_t s);
 // cap_x / tail_x [n][cells].
 cudaError_t launch_solve(const Set& set, int n, const float* cap_x, const float* tail_x,
                          fs_allocation* out, bool write_theta, LaunchCache& lc, cudaStream_t s);
+// early: the candidate ids and bounds were complete before the preceding
+// kernel started, so the bounds-only work may run before the PDL wait.
 cudaError_t launch_prep(const Set& set, const Items& it, const Plan& pl, float* tables,
-                        uint64_t* sums, LaunchCache& lc, cudaStream_t s);
+                        uint64_t* sums, bool early, LaunchCache& lc, cudaStream_t s);
 cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const float* tables,
                          uint64_t* sums, void* dump, int dump_stride, int sm_count, LaunchCache& lc,
                          cudaStream_t s);

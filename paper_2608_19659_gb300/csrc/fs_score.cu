@@ -23,6 +23,9 @@
 //
 // k_prep builds, per (candidate, realisation), the part of that table a
 // scenario can reach: Theta entries with kappa in (Cexcl, max(Cexcl, cap_hi_e)].
+// It also maps each outcome's quantile stratum into the candidate's capacity
+// interval and records where the stratum's tail values stop passing the SLO
+// (the map is monotone, so the gate of Eq. 5 is a position test).
 // k_score draws each scenario (Philox4x32-10 + quantile lookup), evaluates
 // both t* by a binary search of the staged table plus one fulfilment, and
 // sums g = rint(Gamma' 2^40) in int64. k_finalize turns the sums into
@@ -40,13 +43,17 @@ struct Eval {
   int P;   // kCostInf if no other row of class ie covers t
 };
 
-__device__ __forceinline__ Eval warp_eval_excl(float t, const float* sC, const float* sLam, const float* sRl,
-                                               const Dims& d, int rr, int ie, int lane) {
-  int R = 0;
-  bool rinf = false;
+// Evaluation of threshold t by an aligned group of gsz lanes (gsz a power of
+// two in [4, 32]); lane gl of the group takes rows gl, gl + gsz, ... The
+// per-class minimum over the four TP rows is two xor-shuffles; the other
+// classes' costs are summed with the count of uncovered classes packed
+// above bit 24 (a cost is at most G <= 32767, so 64 of them stay below 2^21).
+__device__ __forceinline__ Eval group_eval_excl(float t, const float* sC, const float* sLam, const float* sRl,
+                                                const Dims& d, int rr, int ie, int gl, int gsz) {
+  int packed = 0;
   int P = kCostInf;
-  for (int base = 0; base < d.K4; base += 32) {
-    const int rho = base + lane;
+  for (int base = 0; base < d.K4; base += gsz) {
+    const int rho = base + gl;
     int cost = kCostInf;
     if (rho < d.K4 && rho != rr) {
       const int n = min_replicas(t, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[rho & 3]);
@@ -54,15 +61,16 @@ __device__ __forceinline__ Eval warp_eval_excl(float t, const float* sC, const f
     }
     cost = min(cost, __shfl_xor_sync(0xffffffffu, cost, 1));
     cost = min(cost, __shfl_xor_sync(0xffffffffu, cost, 2));
-    const int cls = rho >> 2;
-    const bool head = rho < d.K4 && (lane & 3) == 0 && cls != ie;
-    if (__ballot_sync(0xffffffffu, head && cost >= kCostInf)) rinf = true;
-    R += __reduce_add_sync(0xffffffffu, (head && cost < kCostInf) ? cost : 0);
-    const int ibase = ie * 4;
-    if (ibase >= base && ibase < base + 32) P = __shfl_sync(0xffffffffu, cost, ibase - base);
+    const bool head = rho < d.K4 && (gl & 3) == 0 && (rho >> 2) != ie;
+    int v = head ? (cost >= kCostInf ? (1 << 24) : cost) : 0;
+    for (int off = 4; off < gsz; off <<= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+    packed += v;
+    const int ib = ie * 4;
+    const int pc = __shfl_sync(0xffffffffu, cost, (ib - base) & (gsz - 1), gsz);
+    if (ib >= base && ib < base + gsz) P = pc;
   }
   Eval e;
-  e.A = rinf ? -1 : d.G - R;
+  e.A = (packed >> 24) ? -1 : d.G - packed;
   e.P = P;
   return e;
 }
@@ -75,21 +83,52 @@ __device__ __forceinline__ bool feasible_at(const Eval& e, int m, float C, float
   return (e.P < kCostInf && e.P <= e.A) || (m >= 1 && fulfil_r((float)m, C, lam, rl) >= t);
 }
 
-__global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan pl, float* tables,
-                                                       uint64_t* sums) {
+// Index probed by group g of ng in one round of the joint search for the
+// last feasible index at Cexcl (interval (lo0, hi0)) and at max(Cexcl,
+// cap_hi) (interval (lo1, hi1)); open intervals are split evenly.
+__device__ __forceinline__ int probe_index(int g, int ng, int lo0, int hi0, int lo1, int hi1) {
+  const bool open0 = hi0 - lo0 > 1, open1 = hi1 - lo1 > 1;
+  int lo, hi, part, parts;
+  if (open0 && open1) {
+    const int half = ng >> 1;
+    const bool first = g < half;
+    lo = first ? lo0 : lo1;
+    hi = first ? hi0 : hi1;
+    parts = half + 1;
+    part = (first ? g : g - half) + 1;
+  } else {
+    lo = open0 ? lo0 : lo1;
+    hi = open0 ? hi0 : hi1;
+    parts = ng + 1;
+    part = g + 1;
+  }
+  const int k = lo + (part * (hi - lo)) / parts;
+  return max(lo + 1, min(hi - 1, k));
+}
+
+// One CTA per (candidate, realisation sigma). Before the threshold search it
+// maps the quantile strata of the outcomes o = sigma, sigma + 2, ... into the
+// candidate's record: this and Cexcl read only the bounds, so with `early`
+// they overlap the base solve that precedes this kernel.
+__global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan pl, float* rec,
+                                                       uint64_t* sums, int early) {
   extern __shared__ __align__(16) unsigned char smraw[];
   float* sC = reinterpret_cast<float*>(smraw);  // [256]
   float* sTh = sC + 256;                          // [theta_cap]
   __shared__ float s_cx, s_cmax;
-  __shared__ int s_bx;
+  __shared__ int s_bx, s_row;
+  __shared__ float sLam[FS_MAX_CLASSES], sRl[FS_MAX_CLASSES];  // demand and RN(1/demand)
+  __shared__ int s_res[2][kPrepThreads / 4];
   const Dims& d = set.d;  // kernel-parameter space: d.M[j] reads need no local copy
   const int item = blockIdx.x >> 1, sigma = blockIdx.x & 1;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = blockDim.x >> 5;
-  pdl_wait();     // thresholds, rows and the zeroed lmax come from k_solve
+  if (!early) pdl_wait();
   pdl_trigger();  // k_score may start launching; it waits for this grid to finish
   const int p = it.p ? it.p[item] : 0;
   const int cell = it.cell[item];
-  float* tab = tables + ((size_t)item * 2 + sigma) * d.slot_floats;
+  float* base_rec = rec + (size_t)item * pl.item_floats;
+  float* tab = base_rec + (size_t)sigma * d.slot_floats;
+  if (blockIdx.x == 0 && tid == 0) *set.work = 0ull;
   if (sigma == 0)
     for (int o = tid; o < pl.O; o += blockDim.x) sums[(size_t)item * pl.O + o] = 0ull;
   if (cell < 0 || cell >= d.cells) {  // device-side candidate ids are checked here
@@ -97,24 +136,21 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
       atomicOr(set.status, ST_CELL);
       for (int k = 0; k < kTableHeader; ++k) tab[k] = 0.0f;
       tab[H_BX] = __int_as_float(-1);
+      tab[H_CELL] = __int_as_float(-1);
     }
     return;
   }
   const int rr = cell / d.B, be = cell - rr * d.B, ie = rr >> 2, jr = rr & 3;
   const float lam = set.lam[ie], L = set.slo[ie], rl = __frcp_rn(lam);
-  __shared__ float sLam[FS_MAX_CLASSES], sRl[FS_MAX_CLASSES];  // demand and RN(1/demand)
   if (tid < d.K) {
     sLam[tid] = set.lam[tid];
     sRl[tid] = __frcp_rn(set.lam[tid]);
   }
-  const size_t ps = (size_t)p * 2 + sigma;
-  const int total = set.ntheta[ps];
-  const float* th_g = set.theta + ps * d.theta_cap;
-  for (int rho = tid; rho < d.K4; rho += blockDim.x) sC[rho] = set.rowC[ps * d.K4 + rho];
-  for (int k = tid; k < total; k += blockDim.x) sTh[k] = th_g[k];
   const float* bp = set.bounds + (size_t)p * 4 * d.cells;
   const float* capS = bp + (size_t)(sigma ? CAP_HI : CAP_LO) * d.cells;
   const float* tailS = bp + (size_t)(sigma ? TAIL_LO : TAIL_HI) * d.cells;
+  const float lo_c = bp[(size_t)CAP_LO * d.cells + cell], hi_c = bp[(size_t)CAP_HI * d.cells + cell];
+  const float lo_l = bp[(size_t)TAIL_LO * d.cells + cell], hi_l = bp[(size_t)TAIL_HI * d.cells + cell];
 
   // best SLO-feasible capacity of row r without bin b_e (ties: lower bin)
   if (warp == 0) {
@@ -142,65 +178,79 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
     if (lane == 0) {
       s_cx = bb >= 0 ? best : 0.0f;
       s_bx = bb;
-      s_cmax = fmaxf(s_cx, bp[(size_t)CAP_HI * d.cells + cell]);
+      s_cmax = fmaxf(s_cx, hi_c);
+      s_row = 0;
     }
   }
+
+  // Mapped strata. Window of outcome o: word 0 = the number of leading
+  // positions whose tail value passes the SLO (the mapped tails are
+  // nondecreasing in the position, so exactly one position ends the run of
+  // passes), words 4.. = the W capacities.
+  {
+    const int W = pl.W;
+    const float d_c = __fsub_rn(hi_c, lo_c), d_l = __fsub_rn(hi_l, lo_l);
+    const long long n_idx = (long long)((pl.O - sigma + 1) >> 1) * W;
+    float* wins = base_rec + 2 * (size_t)d.slot_floats;
+    // read-only loads, so that the unrolled iterations' loads are issued
+    // together rather than each behind the previous iteration's stores
+#pragma unroll 4
+    for (long long idx = tid; idx < n_idx; idx += blockDim.x) {
+      const int k = (int)(idx & (W - 1));
+      const int o = sigma + 2 * (int)(idx >> pl.w);
+      const float* q = set.qn + (size_t)o * W;
+      float* win = wins + (size_t)o * pl.Wp;
+      const float qv = __ldg(q + k);
+      const float qnext = k + 1 < W ? __ldg(q + k + 1) : 0.0f;
+      win[4 + k] = map_into(lo_c, d_c, hi_c, qv);
+      const bool pass = map_into(lo_l, d_l, hi_l, qv) <= L;
+      const bool pass_next = k + 1 < W && map_into(lo_l, d_l, hi_l, qnext) <= L;
+      if (k == 0 && !pass) win[0] = __int_as_float(0);
+      if (pass && !pass_next) win[0] = __int_as_float(k + 1);
+    }
+  }
+  if (early) pdl_wait();  // thresholds and rows come from k_solve
+
+  const size_t ps = (size_t)p * 2 + sigma;
+  const int total = set.ntheta[ps];
+  const float* th_g = set.theta + ps * d.theta_cap;
+  for (int rho = tid; rho < d.K4; rho += blockDim.x) sC[rho] = set.rowC[ps * d.K4 + rho];
+  for (int k = tid; k < total; k += blockDim.x) sTh[k] = th_g[k];
   __syncthreads();
   const float cx = s_cx, cmax = s_cmax;
   const int msent = d.K == 1 ? d.M[jr] : 0;  // above every threshold only a lone class can go on
 
   // b0: last index feasible at Cexcl; b1: last index feasible at max(Cexcl, cap_hi).
-  // Joint search: each round every warp probes one index; a probe answers for
-  // both capacities, and the warps split whichever intervals are still open.
-  __shared__ int s_iv[4], s_probe[8];
-  if (tid == 0) {
-    s_iv[0] = -1;
-    s_iv[1] = total;
-    s_iv[2] = -1;
-    s_iv[3] = total;
-  }
-  __syncthreads();
-  for (;;) {
-    const int lo0 = s_iv[0], hi0 = s_iv[1], lo1 = s_iv[2], hi1 = s_iv[3];
-    const bool open0 = hi0 - lo0 > 1, open1 = hi1 - lo1 > 1;
-    if (!open0 && !open1) break;
-    int lo, hi, part, parts;
-    if (open0 && open1) {
-      const bool first = warp < nwarp / 2;
-      lo = first ? lo0 : lo1;
-      hi = first ? hi0 : hi1;
-      parts = nwarp / 2 + 1;
-      part = (first ? warp : warp - nwarp / 2) + 1;
-    } else {
-      lo = open0 ? lo0 : lo1;
-      hi = open0 ? hi0 : hi1;
-      parts = nwarp + 1;
-      part = warp + 1;
-    }
-    int k = lo + (int)(((long long)part * (hi - lo)) / parts);
-    k = max(lo + 1, min(hi - 1, k));
-    const Eval e = warp_eval_excl(sTh[k], sC, sLam, sRl, d, rr, ie, lane);
-    const int m = replicas_left(e, jr, d);
-    if (lane == 0) {
-      s_probe[2 * warp] = k;
-      s_probe[2 * warp + 1] = (feasible_at(e, m, cx, sTh[k], lam, rl) ? 1 : 0) | (feasible_at(e, m, cmax, sTh[k], lam, rl) ? 2 : 0);
+  // Joint search: each round every group of gsz lanes probes one index and
+  // answers for both capacities; each warp merges the answers with integer
+  // max / min reductions, so a round costs one barrier.
+  int gsz = 4;
+  while (gsz < d.K4 && gsz < 32) gsz <<= 1;
+  const int ng = blockDim.x / gsz, g = tid / gsz, gl = tid & (gsz - 1);
+  int lo0 = -1, hi0 = total, lo1 = -1, hi1 = total;
+  for (int par = 0; hi0 - lo0 > 1 || hi1 - lo1 > 1; par ^= 1) {
+    const int k = probe_index(g, ng, lo0, hi0, lo1, hi1);
+    const float t = sTh[k];
+    const Eval e = group_eval_excl(t, sC, sLam, sRl, d, rr, ie, gl, gsz);
+    if (gl == 0) {
+      const int m = replicas_left(e, jr, d);
+      const int f = (feasible_at(e, m, cx, t, lam, rl) ? 1 : 0) | (feasible_at(e, m, cmax, t, lam, rl) ? 2 : 0);
+      s_res[par][g] = k | (f << 24);
     }
     __syncthreads();
-    if (tid == 0) {
-      int a0 = lo0, c0 = hi0, a1 = lo1, c1 = hi1;
-      for (int w = 0; w < nwarp; ++w) {
-        const int kk = s_probe[2 * w], f = s_probe[2 * w + 1];
-        if (f & 1) a0 = max(a0, kk); else c0 = min(c0, kk);
-        if (f & 2) a1 = max(a1, kk); else c1 = min(c1, kk);
-      }
-      s_iv[0] = a0;
-      s_iv[1] = c0;
-      s_iv[2] = a1;
-      s_iv[3] = c1;
+    int a0 = lo0, c0 = hi0, a1 = lo1, c1 = hi1;
+    if (lane < ng) {
+      const int v = s_res[par][lane];
+      const int kq = v & 0xFFFFFF, f = v >> 24;
+      if (f & 1) a0 = max(a0, kq); else c0 = min(c0, kq);
+      if (f & 2) a1 = max(a1, kq); else c1 = min(c1, kq);
     }
-    __syncthreads();
+    lo0 = __reduce_max_sync(0xffffffffu, a0);
+    hi0 = __reduce_min_sync(0xffffffffu, c0);
+    lo1 = __reduce_max_sync(0xffffffffu, a1);
+    hi1 = __reduce_min_sync(0xffffffffu, c1);
   }
-  const int b0 = s_iv[0], b1 = s_iv[2];
+  const int b0 = lo0, b1 = lo1;
   const int Lt = b1 - b0;
   // arrays padded to P = pow2 >= Lt + 1 entries (+inf beyond Lt), so the
   // scenario search needs no bound checks; at least 4 for 16-byte copies
@@ -220,7 +270,7 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
     const int k = b0 + 1 + u;
     int m;
     if (k < total) {
-      const Eval e = warp_eval_excl(sTh[k], sC, sLam, sRl, d, rr, ie, lane);
+      const Eval e = group_eval_excl(sTh[k], sC, sLam, sRl, d, rr, ie, lane, 32);
       m = replicas_left(e, jr, d);
     } else {
       m = msent;
@@ -259,6 +309,7 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
       }
     }
     if (lane == 0) {
+      if (m >= 1) s_row = 1;
       if (u == 0) tab[H_M_FIRST] = (float)m; else mn[u - 1] = (float)m;
     }
   }
@@ -267,7 +318,13 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
     tht[u] = 0.0f;
     mn[u] = 0.0f;
   }
+  __syncthreads();
   if (tid == 0) {
+    // every row-term quotient x / lambda of a scenario has x = m C' with
+    // 1 <= m <= 32767 and C' in {0} or [min(Cexcl, cap_lo), cmax]: in
+    // Markstein's range unless a positive C' can fall below 2^-60
+    const bool fast = in_markstein_range(lam) && cmax <= 0x1p44f &&
+                      (cx >= 0x1p-60f || (cx == 0.0f && (lo_c >= 0x1p-60f || hi_c == 0.0f)));
     tab[H_TH_BASE] = b0 >= 0 ? sTh[b0] : 0.0f;
     tab[H_L] = __int_as_float(Lt);
     tab[H_LPAD] = __int_as_float(Lpad);
@@ -275,32 +332,36 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
     tab[H_BX] = __int_as_float(s_bx);
     tab[H_CMAX] = cmax;
     tab[H_LAM] = lam;
-    tab[H_LO_C] = bp[(size_t)CAP_LO * d.cells + cell];
-    tab[H_HI_C] = bp[(size_t)CAP_HI * d.cells + cell];
-    tab[H_LO_L] = bp[(size_t)TAIL_LO * d.cells + cell];
-    tab[H_HI_L] = bp[(size_t)TAIL_HI * d.cells + cell];
+    tab[H_LO_C] = lo_c;
+    tab[H_HI_C] = hi_c;
+    tab[H_LO_L] = lo_l;
+    tab[H_HI_L] = hi_l;
     tab[H_SLO] = L;
     tab[H_CELL] = __int_as_float(cell);
     tab[H_P] = __int_as_float(p);
     tab[H_STEP0] = __int_as_float(Lt ? P >> 1 : 0);
-    atomicMax(set.lmax, Lpad);
+    tab[H_ROW] = __int_as_float(s_row);
+    tab[H_FAST] = __int_as_float(fast ? 1 : 0);
   }
 }
 
 // t* of one realisation with row capacity C (see the file comment). kap is
 // padded with +inf to a power of two above the entry count, so the
 // branch-free search needs no bound checks; step0 = half that power.
+// ROW = 0: no reachable threshold leaves row r a replica (m < 1 throughout),
+// so the row term is 0; ROW = 1: the quotient by Markstein's method (valid
+// for every C' of the segment); ROW = 2: the IEEE division.
+template <int ROW>
 __device__ __forceinline__ float tstar_of(float C, const float* kap, const float* tht, const float* mn,
-                                          int step0, float th_base, float m_first, float lam,
-                                          float rlam) {
+                                          int step0, float th_base, float m_first, float lam, float rlam) {
   int pos = 0;
   for (int step = step0; step > 0; step >>= 1) pos += kap[pos + step - 1] <= C ? step : 0;
   const float thb = pos ? tht[pos - 1] : th_base;
+  if (ROW == 0) return thb;
   const float m = pos ? mn[pos - 1] : m_first;
-  // the row term is rarely needed; the out-of-line IEEE divide keeps it behind
-  // the branch (an inline quotient would be computed for every scenario)
-  (void)rlam;
-  const float tr = m >= 1.0f ? fulfil(m, C, lam) : 0.0f;
+  float tr;
+  if (ROW == 1) tr = m >= 1.0f ? fulfil_fast(m, C, lam, rlam) : 0.0f;
+  else tr = m >= 1.0f ? fulfil(m, C, lam) : 0.0f;
   return tr > thb ? tr : thb;
 }
 
@@ -340,18 +401,17 @@ __device__ void dump_choices(float t, const Set& set, size_t ps, int rr, float C
 // Philox calls [q_lo, q_hi) of one (candidate, outcome) segment; call q
 // serves samples 4q..4q+3, sample 4q+h reading output word h (upper 16 bits:
 // capacity position, lower 16 bits: tail position; top log2(W) bits each).
-// h0/h1 point at the staged table headers; kap/tht/mnn at the table arrays
-// (shared memory when TS, else global). Without DUMP, sQ holds the stratum's
-// capacities already mapped into [cap_lo, cap_hi], and the tail gate of
-// Eq. 5 (l_y <= L_i) is the position test kl < kgate (the mapped tail
-// quantiles are nondecreasing in the position); with DUMP, sQ holds the raw
-// quantiles and both values are mapped per sample.
-template <bool DUMP, bool TS>
+// win is the staged window of the outcome (gate position, then the mapped
+// capacities); h0/h1 point at the staged table headers; kap/tht/mnn at the
+// table arrays (shared memory when TS, else global). The tail gate of Eq. 5
+// (l_y <= L_i) is the position test kl < kgate; in dump mode l_y itself is
+// mapped for the record and the gate compares it with the SLO.
+template <bool DUMP, bool TS, int ROW>
 __device__ __forceinline__ uint64_t run_piece(const Set& set, const Plan& pl, int item, int o, int q_lo,
-                                              int q_hi, const float* sQ, int qoff, int kgate, const float* h0,
-                                              const float* h1, const float* kap0, const float* tht0,
-                                              const float* mn0, const float* kap1, const float* tht1,
-                                              const float* mn1, unsigned char* dump, int dump_stride) {
+                                              int q_hi, const float* win, const float* h0, const float* h1,
+                                              const float* kap0, const float* tht0, const float* mn0,
+                                              const float* kap1, const float* tht1, const float* mn1,
+                                              unsigned char* dump, int dump_stride) {
   const int st0 = __float_as_int(h0[H_STEP0]), st1 = __float_as_int(h1[H_STEP0]);
   const float thb0 = h0[H_TH_BASE], mf0 = h0[H_M_FIRST], cx0 = h0[H_CX];
   const float thb1 = h1[H_TH_BASE], mf1 = h1[H_M_FIRST], cx1 = h1[H_CX];
@@ -361,7 +421,8 @@ __device__ __forceinline__ uint64_t run_piece(const Set& set, const Plan& pl, in
   const uint32_t sh = (uint32_t)pl.sh;
   const int S = pl.S;
   const uint32_t ctr1 = (uint32_t)o, ctr2 = (uint32_t)cell, ctr3 = pl.round;
-  const float* sQo = sQ + qoff;
+  const int kgate = __float_as_int(win[0]);
+  const float* sQo = win + 4;
   uint64_t acc = 0;
   for (int q = q_lo + (int)threadIdx.x; q < q_hi; q += blockDim.x) {
     const uint4 x = philox4x32_10(make_uint4((uint32_t)q, ctr1, ctr2, ctr3), keys);
@@ -371,21 +432,20 @@ __device__ __forceinline__ uint64_t run_piece(const Set& set, const Plan& pl, in
       const uint32_t word = h == 0 ? x.x : h == 1 ? x.y : h == 2 ? x.z : x.w;
       const int kc = (int)((word >> 16) >> sh);
       const int kl = (int)((word & 0xFFFFu) >> sh);
-      float cy, ly = 0.0f;
+      const float cy = sQo[kc];
+      float ly = 0.0f;
       bool gate;
       if (DUMP) {
-        const float lo_c = h0[H_LO_C], hi_c = h0[H_HI_C], lo_l = h0[H_LO_L], hi_l = h0[H_HI_L];
-        cy = map_into(lo_c, __fsub_rn(hi_c, lo_c), hi_c, sQo[kc]);
-        ly = map_into(lo_l, __fsub_rn(hi_l, lo_l), hi_l, sQo[kl]);
+        const float lo_l = h0[H_LO_L], hi_l = h0[H_HI_L];
+        ly = map_into(lo_l, __fsub_rn(hi_l, lo_l), hi_l, set.qn[(size_t)o * pl.W + kl]);
         gate = ly <= h0[H_SLO];
       } else {
-        cy = sQo[kc];
         gate = kl < kgate;
       }
       const float C0 = gate ? fmaxf(cx0, cy) : cx0;
       const float C1 = gate ? fmaxf(cx1, cy) : cx1;
-      const float t0 = tstar_of(C0, kap0, tht0, mn0, st0, thb0, mf0, lam, rlam);
-      const float t1 = tstar_of(C1, kap1, tht1, mn1, st1, thb1, mf1, lam, rlam);
+      const float t0 = tstar_of<ROW>(C0, kap0, tht0, mn0, st0, thb0, mf0, lam, rlam);
+      const float t1 = tstar_of<ROW>(C1, kap1, tht1, mn1, st1, thb1, mf1, lam, rlam);
       const uint64_t gf = fixed40(__fsub_rn(t1, t0));
       acc += (h == 0 || s < S) ? gf : 0ull;  // the last call may serve fewer than four samples
       if (DUMP && (h == 0 || s < S)) {
@@ -417,113 +477,124 @@ __device__ __forceinline__ uint64_t run_piece(const Set& set, const Plan& pl, in
   return acc;
 }
 
-// Thread 0: stage segment seg (its quantile window and both candidate tables,
-// header plus lcopy entries each) into dst, completing on bar.
-__device__ __forceinline__ void stage_segment(const Set& set, const Plan& pl, const float* tables, int seg,
-                                              float* dst, uint64_t* bar, int qwin, int tstride, int lcopy) {
-  const Dims& d = set.d;
+// Work decomposition of one k_score launch: segment = (item, outcome) with
+// pl.calls Philox calls; a chunk is up to `chunk` consecutive calls of one
+// segment, nch chunks per segment.
+struct ScoreGrid {
+  int total;        // chunks (< 2^31: the host widens chunks until they fit)
+  int chunk;        // calls per chunk (a multiple of the block size)
+  int nch;          // chunks per segment
+  int lcap_s;       // table entries staged per realisation
+  int tcopy;        // floats staged per table: header + 3 lcap_s
+  int dyn;          // 1: chunks after the first two come from the counter; 0: chunk b + k gridDim
+};
+
+// Thread 0: stage the data of segment seg (its outcome window and both
+// candidate tables, header plus lcap_s entries each) into dst, completing on bar.
+__device__ __forceinline__ void stage_segment(const Set& set, const Plan& pl, const float* rec, int seg,
+                                              float* dst, uint64_t* bar, int tcopy) {
   const int item = seg / pl.O, o = seg - item * pl.O;
-  const int q0 = (o * pl.W) & ~3;
-  const int q1 = min(((o + 1) * pl.W + 3) & ~3, d.Q);
-  const float* tab = tables + (size_t)item * 2 * d.slot_floats;
-  const uint32_t tb = (uint32_t)(kTableHeader + 3 * lcopy) * 4u;
-  const uint32_t qb = (uint32_t)(q1 - q0) * 4u;
+  const float* r = rec + (size_t)item * pl.item_floats;
+  const uint32_t tb = (uint32_t)tcopy * 4u, wb = (uint32_t)pl.Wp * 4u;
   fence_proxy_async();
-  mbar_expect_tx(bar, qb + 2 * tb);
-  bulk_g2s(dst, set.qn + q0, qb, bar);
-  bulk_g2s(dst + qwin, tab, tb, bar);
-  bulk_g2s(dst + qwin + tstride, tab + d.slot_floats, tb, bar);
+  mbar_expect_tx(bar, wb + 2 * tb);
+  bulk_g2s(dst, r + 2 * (size_t)set.d.slot_floats + (size_t)o * pl.Wp, wb, bar);
+  bulk_g2s(dst + pl.Wp, r, tb, bar);
+  bulk_g2s(dst + pl.Wp + tcopy, r + set.d.slot_floats, tb, bar);
 }
 
-// Each block owns a contiguous range of the flattened Philox-call index
-// (segment = (candidate, outcome), ceil(S/4) calls each), so the work is
-// balanced to within one call per thread. A segment's quantile window and
-// both candidate tables are staged in shared memory by TMA bulk copies,
-// double-buffered: the next segment's copies fly while this one computes.
+// Blocks take chunks until none is left: chunk blockIdx.x, then chunk
+// blockIdx.x + gridDim.x, then (with many chunks per block) chunks handed out
+// by a global counter, so segments of unequal cost (table length, row-term
+// divisions) even out across the SMs; with few chunks per block the
+// assignment stays static (every block would meet the counter at once). A chunk's data are staged in shared memory by TMA bulk copies,
+// double-buffered: thread 0 issues the next chunk's copies (and the counter
+// increment whose result names the chunk after it) before this chunk is
+// computed. The sums are integers, so the order of the chunks does not
+// change the result.
 template <bool DUMP>
-__global__ void __launch_bounds__(kScoreThreads, 5) k_score(Set set, Items it, Plan pl, const float* tables,
+__global__ void __launch_bounds__(kScoreThreads, 5) k_score(Set set, Items it, Plan pl, const float* rec,
                                                          uint64_t* sums, unsigned char* dump, int dump_stride,
-                                                         long long total_calls, int lcap_s, int qwin) {
+                                                         ScoreGrid sg) {
   extern __shared__ __align__(16) unsigned char smraw[];
   uint64_t* bar = reinterpret_cast<uint64_t*>(smraw);  // [2]
-  const int tstride = kTableHeader + 3 * lcap_s;
-  const int stage_floats = qwin + 2 * tstride;
   float* stage0 = reinterpret_cast<float*>(smraw + 16);
-  __shared__ int s_lcopy;
+  const int stage_floats = pl.Wp + 2 * sg.tcopy;
+  __shared__ int s_chunk[2];
   const Dims& d = set.d;  // kernel-parameter space: d.M[j] reads need no local copy
   const int tid = threadIdx.x, lane = tid & 31;
+  (void)it;
 
-  pdl_wait();  // tables, zeroed sums and lmax come from k_prep
-  const long long g = gridDim.x;
-  const long long r_lo = total_calls * blockIdx.x / g;
-  const long long r_hi = total_calls * (blockIdx.x + 1) / g;
-  if (r_hi <= r_lo) return;
-  const int seg_first = (int)(r_lo / pl.calls);
-  const int seg_last = (int)((r_hi - 1) / pl.calls);
-
+  pdl_wait();  // records, zeroed sums and the zeroed counter come from k_prep
+  const int g = (int)gridDim.x;
+  int next = 0;  // thread 0: the chunk to stage next
   if (tid == 0) {
-    s_lcopy = min(*set.lmax, lcap_s);
     mbar_init(&bar[0], 1);
     mbar_init(&bar[1], 1);
+    s_chunk[0] = (int)blockIdx.x;  // the grid has at most sg.total blocks
   }
   __syncthreads();
-  const int lcopy = s_lcopy;
-  if (tid == 0) stage_segment(set, pl, tables, seg_first, stage0, bar, qwin, tstride, lcopy);
+  if (tid == 0) {
+    stage_segment(set, pl, rec, (int)blockIdx.x / sg.nch, stage0, &bar[0], sg.tcopy);
+    next = (int)blockIdx.x + g;  // may pass sg.total: then the block stops after one chunk
+  }
 
-  int j = 0;
-  for (int seg = seg_first; seg <= seg_last; ++seg, ++j) {
+  for (int j = 0;; ++j) {
     const int st = j & 1;
-    if (tid == 0 && seg < seg_last)
-      stage_segment(set, pl, tables, seg + 1, stage0 + (size_t)(st ^ 1) * stage_floats, bar + (st ^ 1), qwin,
-                    tstride, lcopy);
+    const int c = s_chunk[st];
+    if (c >= sg.total) break;
+    if (tid == 0) {
+      s_chunk[st ^ 1] = next;
+      if (next < sg.total) {
+        stage_segment(set, pl, rec, next / sg.nch, stage0 + (size_t)(st ^ 1) * stage_floats, &bar[st ^ 1],
+                      sg.tcopy);
+        if (sg.dyn) {
+          // consumed one chunk later; saturates at sg.total so that it cannot wrap
+          const unsigned long long v = atomicAdd(set.work, 1ull) + 2ull * (unsigned long long)g;
+          next = v < (unsigned long long)sg.total ? (int)v : sg.total;
+        } else {
+          next = (long long)next + g < (long long)sg.total ? next + g : sg.total;
+        }
+      }
+    }
     const bool ok = mbar_wait(&bar[st], (uint32_t)((j >> 1) & 1), kWaitLimitNs);
     if (__syncthreads_or(!ok)) {
       if (tid == 0) atomicOr(set.status, ST_TIMEOUT);
       // let copies in flight land before the block exits (bounded as well)
       mbar_wait(&bar[st], (uint32_t)((j >> 1) & 1), kWaitLimitNs);
-      if (seg < seg_last) mbar_wait(&bar[st ^ 1], (uint32_t)(((j + 1) >> 1) & 1), kWaitLimitNs);
+      if (s_chunk[st ^ 1] < sg.total) mbar_wait(&bar[st ^ 1], (uint32_t)(((j + 1) >> 1) & 1), kWaitLimitNs);
       return;
     }
-    float* stg = stage0 + (size_t)st * stage_floats;
-    const float* h0 = stg + qwin;
-    const float* h1 = h0 + tstride;
+    const float* stg = stage0 + (size_t)st * stage_floats;
+    const float* h0 = stg + pl.Wp;
+    const float* h1 = h0 + sg.tcopy;
+    const int seg = c / sg.nch;
+    const int part = c - seg * sg.nch;
     const int item = seg / pl.O, o = seg - item * pl.O;
-    const long long sb = (long long)seg * pl.calls;
-    const int q_lo = (int)(max(r_lo, sb) - sb);
-    const int q_hi = (int)(min(r_hi, sb + pl.calls) - sb);
-    const int qoff = o * pl.W - ((o * pl.W) & ~3);
+    const int q_lo = part * sg.chunk;
+    const int q_hi = min(q_lo + sg.chunk, pl.calls);
     const int Lp0 = __float_as_int(h0[H_LPAD]), Lp1 = __float_as_int(h1[H_LPAD]);
     const int cell = __float_as_int(h0[H_CELL]);
     const bool cell_ok = cell >= 0 && cell < d.cells;  // a bad device-side id was flagged by k_prep
-    int kgate = 0;
-    if (!DUMP) {
-      // map the stratum's quantiles into this cell's capacity interval in place,
-      // and count the positions whose tail value passes the SLO gate
-      const float lo_c = h0[H_LO_C], hi_c = h0[H_HI_C], lo_l = h0[H_LO_L], hi_l = h0[H_HI_L];
-      const float d_c = __fsub_rn(hi_c, lo_c), d_l = __fsub_rn(hi_l, lo_l), slo = h0[H_SLO];
-      for (int k0 = 0; k0 < pl.W; k0 += blockDim.x) {
-        const int k = k0 + tid;
-        bool pass = false;
-        if (k < pl.W) {
-          const float qv = stg[qoff + k];
-          stg[qoff + k] = map_into(lo_c, d_c, hi_c, qv);
-          pass = map_into(lo_l, d_l, hi_l, qv) <= slo;
-        }
-        kgate += __syncthreads_count(pass);
-      }
-    }
     uint64_t acc = 0;
     if (cell_ok) {
-      if (Lp0 <= lcopy && Lp1 <= lcopy) {
-        acc = run_piece<DUMP, true>(set, pl, item, o, q_lo, q_hi, stg, qoff, kgate, h0, h1, h0 + kTableHeader,
-                                    h0 + kTableHeader + Lp0, h0 + kTableHeader + 2 * Lp0, h1 + kTableHeader,
-                                    h1 + kTableHeader + Lp1, h1 + kTableHeader + 2 * Lp1, dump, dump_stride);
+      const bool r0 = __float_as_int(h0[H_ROW]) != 0, r1 = __float_as_int(h1[H_ROW]) != 0;
+      const bool f0 = __float_as_int(h0[H_FAST]) != 0, f1 = __float_as_int(h1[H_FAST]) != 0;
+      const int row = DUMP ? 2 : (!r0 && !r1) ? 0 : ((!r0 || f0) && (!r1 || f1)) ? 1 : 2;
+      // the table pointers stay in one address space per branch (shared or global)
+#define FS_PIECE(TSV, ROWV)                                                                                 \
+  run_piece<DUMP, TSV, ROWV>(set, pl, item, o, q_lo, q_hi, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, \
+                             k1 + Lp1, k1 + 2 * Lp1, dump, dump_stride)
+      if (Lp0 <= sg.lcap_s && Lp1 <= sg.lcap_s) {
+        const float* k0 = h0 + kTableHeader;
+        const float* k1 = h1 + kTableHeader;
+        acc = row == 0 ? FS_PIECE(true, 0) : row == 1 ? FS_PIECE(true, 1) : FS_PIECE(true, 2);
       } else {
-        const float* g0 = tables + (size_t)item * 2 * d.slot_floats + kTableHeader;
-        const float* g1 = g0 + d.slot_floats;
-        acc = run_piece<DUMP, false>(set, pl, item, o, q_lo, q_hi, stg, qoff, kgate, h0, h1, g0, g0 + Lp0,
-                                     g0 + 2 * Lp0, g1, g1 + Lp1, g1 + 2 * Lp1, dump, dump_stride);
+        const float* k0 = rec + (size_t)item * pl.item_floats + kTableHeader;
+        const float* k1 = k0 + d.slot_floats;
+        acc = row == 0 ? FS_PIECE(false, 0) : row == 1 ? FS_PIECE(false, 1) : FS_PIECE(false, 2);
       }
+#undef FS_PIECE
     }
     for (int off = 16; off; off >>= 1) acc += __shfl_down_sync(0xffffffffu, acc, off);
     if (lane == 0 && acc)
@@ -546,7 +617,7 @@ __global__ void k_finalize(Set set, Items it, Plan pl, const uint64_t* sums, dou
 static size_t prep_smem_bytes(const Dims& d) { return (size_t)(256 + d.theta_cap) * 4; }
 
 cudaError_t launch_prep(const Set& set, const Items& it, const Plan& pl, float* tables, uint64_t* sums,
-                        LaunchCache& lc, cudaStream_t s) {
+                        bool early, LaunchCache& lc, cudaStream_t s) {
   if (it.n <= 0) return cudaSuccess;
   const size_t smem = prep_smem_bytes(set.d);
   if (smem > lc.prep_smem) {
@@ -554,22 +625,19 @@ cudaError_t launch_prep(const Set& set, const Items& it, const Plan& pl, float* 
     if (e != cudaSuccess) return e;
     lc.prep_smem = smem;
   }
-  return launch_pdl(k_prep, dim3(it.n * 2), dim3(kPrepThreads), smem, s, set, it, pl, tables, sums);
+  return launch_pdl(k_prep, dim3(it.n * 2), dim3(kPrepThreads), smem, s, set, it, pl, tables, sums,
+                    early ? 1 : 0);
 }
 
 static int score_lcap(const Dims& d) { return d.lcap < kSmemTableCap ? d.lcap : kSmemTableCap; }
 
-static int score_qwin(const Dims& d, const Plan& pl) {
-  const int w = ((pl.W + 3) & ~3) + 4;
-  return w < d.Q ? w : d.Q;
-}
-
 cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const float* tables, uint64_t* sums,
                          void* dump, int dump_stride, int sm_count, LaunchCache& lc, cudaStream_t s) {
   if (it.n <= 0) return cudaSuccess;
-  const long long total = (long long)it.n * pl.O * pl.calls;
-  const int lcap_s = score_lcap(set.d), qwin = score_qwin(set.d, pl);
-  const size_t smem = 16 + 2 * (size_t)(qwin + 2 * (kTableHeader + 3 * lcap_s)) * 4;
+  ScoreGrid sg{};
+  sg.lcap_s = score_lcap(set.d);
+  sg.tcopy = kTableHeader + 3 * sg.lcap_s;
+  const size_t smem = 16 + 2 * (size_t)(pl.Wp + 2 * sg.tcopy) * 4;
   const int v = dump ? 1 : 0;
   if (smem != lc.score_smem[v]) {
     cudaError_t e;
@@ -587,21 +655,34 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
     lc.score_smem[v] = smem;
     lc.score_blocks_per_sm[v] = per_sm < 1 ? 1 : per_sm;
   }
-  // One resident wave at least; up to four when every block still gets >= 16
-  // calls per thread, so that the block scheduler evens out segments of
-  // unequal cost (table length, fulfilment divisions).
+  // Chunks of U calls per thread: about eight chunks per resident block when
+  // the work allows, so that the counter can even out the segments' unequal
+  // costs; at most 8 calls per thread, and no more than a segment holds.
   const long long resident = (long long)lc.score_blocks_per_sm[v] * sm_count;
-  const long long by_work = total / ((long long)kScoreThreads * 16);
-  long long grid_l = by_work < 4 * resident ? by_work : 4 * resident;
-  if (grid_l < resident) grid_l = resident;
-  const long long min_blocks = (total + kScoreThreads - 1) / kScoreThreads;
-  if (grid_l > min_blocks) grid_l = min_blocks;
-  const int grid = (int)grid_l;
+  const long long total_calls = (long long)it.n * pl.O * pl.calls;
+  long long U = total_calls / ((long long)kScoreThreads * resident * 8);
+  const long long u_seg = ((long long)pl.calls + kScoreThreads - 1) / kScoreThreads;
+  if (U > 8) U = 8;
+  if (U > u_seg) U = u_seg;
+  if (U < 1) U = 1;
+  // chunk indices are 32-bit: widen the chunks until they fit (one chunk per
+  // segment gives n O <= 2^30 chunks, which the entry points guarantee)
+  long long nch = (pl.calls + kScoreThreads * U - 1) / (kScoreThreads * U);
+  while ((long long)it.n * pl.O * nch >= (1LL << 31) && U < u_seg) {
+    U *= 2;
+    nch = (pl.calls + kScoreThreads * U - 1) / (kScoreThreads * U);
+  }
+  if ((long long)it.n * pl.O * nch >= (1LL << 31)) return cudaErrorInvalidValue;
+  sg.chunk = (int)(kScoreThreads * U);
+  sg.nch = (int)nch;
+  sg.total = (int)((long long)it.n * pl.O * nch);
+  const int grid = (int)(sg.total < resident ? sg.total : resident);
+  sg.dyn = sg.total >= 4LL * grid ? 1 : 0;
   if (dump)
     return launch_pdl(k_score<true>, dim3(grid), dim3(kScoreThreads), smem, s, set, it, pl, tables, sums,
-                      (unsigned char*)dump, dump_stride, total, lcap_s, qwin);
+                      (unsigned char*)dump, dump_stride, sg);
   return launch_pdl(k_score<false>, dim3(grid), dim3(kScoreThreads), smem, s, set, it, pl, tables, sums,
-                    (unsigned char*)nullptr, 0, total, lcap_s, qwin);
+                    (unsigned char*)nullptr, 0, sg);
 }
 
 cudaError_t launch_finalize(const Set& set, const Items& it, const Plan& pl, const uint64_t* sums, double* gap,

@@ -70,7 +70,6 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   const Dims& d = set.d;  // kernel-parameter space: d.M[j] reads need no local copy
   const int r = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = blockDim.x >> 5;
-  if (r == 0 && tid == 0 && set.lmax) *set.lmax = 0;  // before any early exit
   pdl_trigger();
   if (r >= n_real) return;
 

@@ -115,12 +115,14 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
     off = up256(off + bytes);
     return o;
   };
-  const size_t o_status = take(4), o_lmax = take(4);
+  const size_t o_status = take(4), o_work = take(8);
   const size_t o_qn = quantile_dev ? 0 : take(4 * (size_t)Q);
   const size_t o_theta = take(8 * (size_t)d.theta_cap), o_nth = take(8);
   const size_t o_rowc = take(8 * (size_t)d.K4), o_rowb = take(8 * (size_t)d.K4);
   const size_t o_base = take(2 * sizeof(fs_allocation));
-  const size_t o_tab = take((size_t)std::max(n, 1) * 2 * d.slot_floats * 4);
+  const int Wq = Q / smp->O, Wp = 4 + ((Wq + 3) & ~3);
+  const size_t item_floats = 2 * (size_t)d.slot_floats + (size_t)smp->O * Wp;
+  const size_t o_tab = take((size_t)std::max(n, 1) * item_floats * 4);
   const size_t o_sums = take((size_t)std::max(n, 1) * smp->O * 8);
   if (off > kStaticScratchBytes)
     return say(FS_EINVAL,
@@ -164,7 +166,7 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
   set.rowB = reinterpret_cast<int*>(base + o_rowb);
   set.base = reinterpret_cast<fs_allocation*>(base + o_base);
   set.status = reinterpret_cast<uint32_t*>(base + o_status);
-  set.lmax = reinterpret_cast<int*>(base + o_lmax);
+  set.work = reinterpret_cast<unsigned long long*>(base + o_work);
   set.skip = nullptr;
 
   Items it{};
@@ -184,6 +186,8 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
   while ((1 << pl.w) < pl.W) ++pl.w;
   pl.sh = 16 - pl.w;
   pl.calls = (smp->S + 3) / 4;
+  pl.Wp = Wp;
+  pl.item_floats = (long long)item_floats;
 
   // --- the scoring pipeline on the caller's stream, then wait and report
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
@@ -191,7 +195,7 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
   if (e == cudaSuccess && !quantile_dev) e = launch_qtable(const_cast<float*>(set.qn), Q, s);
   if (e == cudaSuccess) e = launch_solve(set, 2, nullptr, nullptr, nullptr, true, *lc, s);
   if (e == cudaSuccess) e = launch_prep(set, it, pl, reinterpret_cast<float*>(base + o_tab),
-                                        reinterpret_cast<uint64_t*>(base + o_sums), *lc, s);
+                                        reinterpret_cast<uint64_t*>(base + o_sums), true, *lc, s);
   if (e == cudaSuccess)
     e = launch_score(set, it, pl, reinterpret_cast<const float*>(base + o_tab),
                      reinterpret_cast<uint64_t*>(base + o_sums), nullptr, 0, sm_count, *lc, s);
