@@ -45,9 +45,11 @@ struct Eval {
 
 // Evaluation of threshold t by an aligned group of gsz lanes (gsz a power of
 // two in [4, 32]); lane gl of the group takes rows gl, gl + gsz, ... The
-// per-class minimum over the four TP rows is two xor-shuffles; the other
-// classes' costs are summed with the count of uncovered classes packed
-// above bit 24 (a cost is at most G <= 32767, so 64 of them stay below 2^21).
+// per-class minimum over the four TP rows is two xor-shuffles, after which all
+// four lanes of a class hold its cost; xor-sums over the offsets 4 .. gsz/2
+// then add one lane of every class, so every lane of the group ends with the
+// other classes' total (uncovered classes counted above bit 24: a cost is at
+// most G <= 32767, so 64 of them stay below 2^21), and every lane's result is valid.
 __device__ __forceinline__ Eval group_eval_excl(float t, const float* sC, const float* sLam, const float* sRl,
                                                 const Dims& d, int rr, int ie, int gl, int gsz) {
   int packed = 0;
@@ -61,8 +63,8 @@ __device__ __forceinline__ Eval group_eval_excl(float t, const float* sC, const 
     }
     cost = min(cost, __shfl_xor_sync(0xffffffffu, cost, 1));
     cost = min(cost, __shfl_xor_sync(0xffffffffu, cost, 2));
-    const bool head = rho < d.K4 && (gl & 3) == 0 && (rho >> 2) != ie;
-    int v = head ? (cost >= kCostInf ? (1 << 24) : cost) : 0;
+    const bool other = rho < d.K4 && (rho >> 2) != ie;
+    int v = other ? (cost >= kCostInf ? (1 << 24) : cost) : 0;
     for (int off = 4; off < gsz; off <<= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
     packed += v;
     const int ib = ie * 4;

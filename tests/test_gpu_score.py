@@ -132,6 +132,39 @@ def test_large_workload_full_launch_and_dump_sample(fsb, cuda, oracle_lib, qn):
     assert np.all(full.score >= 0) and np.all(full.score <= full.gamma_t)
 
 
+def test_long_tables_read_from_global_memory(fsb, cuda, oracle_lib, qn):
+    """The 8-class workload at twice its demand has contested threshold ranges of up
+    to ~300 entries, longer than the 256 the scorer stages in shared memory: those
+    scenarios search their tables in global memory. Every candidate, few samples;
+    then denser sampling on candidates with a positive score."""
+    w = stressed(3, 2.0, O=2, S=8)
+    r = run(fsb, w)
+    ref = oracle_lib.score(w, qn)
+    assert_same(r, ref)
+    pos = np.nonzero(ref.score > 0)[0]
+    assert len(pos) > 0
+    w2 = dataclasses.replace(w, S=96)
+    cand = w.candidates[pos[:: max(1, len(pos) // 4)][:4]]
+    r2 = run(fsb, w2, cand=cand)
+    assert_same(r2, oracle_lib.score(w2, qn, candidates=cand), cand=cand)
+
+
+@pytest.mark.parametrize("cap", [0.0, 1e-20])
+def test_row_term_outside_markstein_range(fsb, cuda, oracle_lib, qn, cap):
+    """A row whose capacities under A- are zero or below 2^-60: the row-term
+    quotient of its candidates cannot use Markstein's method and goes through the
+    IEEE division; every cell is a candidate."""
+    w = stressed(0, 3.0, O=4, S=128)
+    cap_lo = w.cap_lo.copy().reshape(w.K, 4, w.B)
+    cap_lo[0, 0, :] = cap  # class 0, TP 1, every bin
+    w = dataclasses.replace(w, cap_lo=cap_lo.reshape(w.cap_lo.shape),
+                            candidates=np.arange(w.K * 4 * w.B, dtype=np.int32))
+    r = run(fsb, w)
+    ref = oracle_lib.score(w, qn)
+    assert_same(r, ref)
+    assert ref.gamma_t > 0
+
+
 @pytest.mark.parametrize("O,S", [(1, 7), (4, 1), (4096, 3), (16, 33), (2, 2)])
 def test_outcome_and_sample_edge_cases(fsb, cuda, oracle_lib, qn, O, S):
     w = stressed(0, 3.0, O=O, S=S)
