@@ -254,20 +254,23 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
   }
   const int b0 = lo0, b1 = lo1;
   const int Lt = b1 - b0;
-  // arrays padded to P = pow2 >= Lt + 1 entries (+inf beyond Lt), so the
-  // scenario search needs no bound checks; at least 4 for 16-byte copies
+  // Three arrays of Lpad = max(P, 4) entries, P = pow2 >= Lt + 1 (at least 4
+  // for 16-byte copies): kappa[u] for u < Lt, +inf beyond, so the scenario
+  // search needs no bound checks; thx[pos] = the threshold reached with pos
+  // kappa entries passed (thx[0] = theta_b0, 0 if b0 = -1) and mnx[pos] =
+  // the replicas row r may use just above it, for pos = 0..Lt.
   int P = 1;
   while (P < Lt + 1) P <<= 1;
-  const int Lpad = Lt ? max(P, 4) : 0;
+  const int Lpad = max(P, 4);
   if (Lpad > d.lcap) {  // cannot happen: Lt <= total <= theta_cap
     if (tid == 0) atomicOr(set.status, ST_TABLE);
     return;
   }
   float* kap = tab + kTableHeader;
-  float* tht = kap + Lpad;
-  float* mn = tht + Lpad;
+  float* thx = kap + Lpad;
+  float* mnx = thx + Lpad;
 
-  // u = 0..Lt: m at index b0+1+u (m_first, then m_next[u-1]); kappa for u < Lt
+  // u = 0..Lt: m at index b0+1+u; kappa for u < Lt
   for (int u = warp; u <= Lt; u += nwarp) {
     const int k = b0 + 1 + u;
     int m;
@@ -307,19 +310,23 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
       }
       if (lane == 0) {
         kap[u] = __uint_as_float(hi);
-        tht[u] = t;
+        thx[u + 1] = t;
       }
     }
     if (lane == 0) {
       if (m >= 1) s_row = 1;
-      if (u == 0) tab[H_M_FIRST] = (float)m; else mn[u - 1] = (float)m;
+      mnx[u] = (float)m;
+      if (u == 0) tab[H_M_FIRST] = (float)m;
     }
   }
   for (int u = Lt + tid; u < Lpad; u += blockDim.x) {
     kap[u] = __int_as_float(0x7f800000);
-    tht[u] = 0.0f;
-    mn[u] = 0.0f;
+    if (u > Lt) {
+      thx[u] = 0.0f;
+      mnx[u] = 0.0f;
+    }
   }
+  if (tid == 0) thx[0] = b0 >= 0 ? sTh[b0] : 0.0f;
   __syncthreads();
   if (tid == 0) {
     // every row-term quotient x / lambda of a scenario has x = m C' with
@@ -349,23 +356,47 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
 
 // t* of one realisation with row capacity C (see the file comment). kap is
 // padded with +inf to a power of two above the entry count, so the
-// branch-free search needs no bound checks; step0 = half that power.
-// ROW = 0: no reachable threshold leaves row r a replica (m < 1 throughout),
-// so the row term is 0; ROW = 1: the quotient by Markstein's method (valid
-// for every C' of the segment); ROW = 2: the IEEE division.
+// branch-free search needs no bound checks; step0 = half that power. thx[pos]
+// and mnx[pos] are the threshold and the replicas of row r once pos entries
+// are passed. ROW = 0: no reachable threshold leaves row r a replica (m < 1
+// throughout), so the row term is 0; ROW = 1: the quotient by Markstein's
+// method (valid for every C' of the segment); ROW = 2: the IEEE division.
 template <int ROW>
-__device__ __forceinline__ float tstar_of(float C, const float* kap, const float* tht, const float* mn,
-                                          int step0, float th_base, float m_first, float lam, float rlam) {
+__device__ __forceinline__ float tstar_of(float C, const float* kap, const float* thx, const float* mnx,
+                                          int step0, float lam, float rlam) {
   int pos = 0;
   for (int step = step0; step > 0; step >>= 1) pos += kap[pos + step - 1] <= C ? step : 0;
-  const float thb = pos ? tht[pos - 1] : th_base;
+  const float thb = thx[pos];
   if (ROW == 0) return thb;
-  const float m = pos ? mn[pos - 1] : m_first;
+  const float m = mnx[pos];
   float tr;
   if (ROW == 1) tr = m >= 1.0f ? fulfil_fast(m, C, lam, rlam) : 0.0f;
   else tr = m >= 1.0f ? fulfil(m, C, lam) : 0.0f;
   return tr > thb ? tr : thb;
 }
+
+// Sum of rint(g 2^40) over values 0 <= g <= 1 (every Gamma' is in [0, 1]).
+// u = RN(g + 8) - 8 is g rounded to the 2^-20 grid (the spacing of floats in
+// [8, 16)) and exact, and d = g - u is exact with |d| <= 2^-21, so
+// rint(g 2^40) = u 2^40 + rint(d 2^40) (u 2^40 is an even integer). The two
+// terms are the bit patterns of 2^23 + u 2^20 and 1.5 2^23 + d 2^40 less the
+// patterns of 2^23 and 1.5 2^23 (one FMA each; the second rounds d 2^40 to an
+// integer, ties to even); they are summed in two 32-bit words and the offsets
+// removed once: exact for up to 2048 values, with adds and FMAs only.
+struct Acc40 {
+  uint32_t h = 0, l = 0, n = 0;
+  __device__ __forceinline__ void add(float g) {
+    const float u = __fsub_rn(__fadd_rn(g, 8.0f), 8.0f);
+    const float dl = __fsub_rn(g, u);
+    h += __float_as_uint(__fmaf_rn(u, 0x1p20f, 0x1p23f));
+    l += __float_as_uint(__fmaf_rn(dl, 0x1p40f, 0x1.8p23f));
+  }
+  __device__ __forceinline__ uint64_t value() const {
+    const uint32_t H = h - n * 0x4B000000u;
+    const int32_t Lo = (int32_t)(l - n * 0x4B400000u);
+    return ((uint64_t)H << 20) + (uint64_t)(int64_t)Lo;
+  }
+};
 
 // Per-class choice of one scenario at threshold t (dump mode only): rows from
 // the base realisation except row rr, which has capacity C and bin bC.
@@ -402,78 +433,123 @@ __device__ void dump_choices(float t, const Set& set, size_t ps, int rr, float C
 
 // Philox calls [q_lo, q_hi) of one (candidate, outcome) segment; call q
 // serves samples 4q..4q+3, sample 4q+h reading output word h (upper 16 bits:
-// capacity position, lower 16 bits: tail position; top log2(W) bits each).
-// win is the staged window of the outcome (gate position, then the mapped
-// capacities); h0/h1 point at the staged table headers; kap/tht/mnn at the
-// table arrays (shared memory when TS, else global). The tail gate of Eq. 5
-// (l_y <= L_i) is the position test kl < kgate; in dump mode l_y itself is
-// mapped for the record and the gate compares it with the SLO.
-template <bool DUMP, bool TS, int ROW>
-__device__ __forceinline__ uint64_t run_piece(const Set& set, const Plan& pl, int item, int o, int q_lo,
-                                              int q_hi, const float* win, const float* h0, const float* h1,
-                                              const float* kap0, const float* tht0, const float* mn0,
-                                              const float* kap1, const float* tht1, const float* mn1,
-                                              unsigned char* dump, int dump_stride) {
+// capacity position, lower 16 bits: tail position; top w = log2(W) bits
+// each). win is the staged window of the outcome (gate position, then the
+// mapped capacities); h0/h1 point at the staged table headers; kap/thx/mnx at
+// the table arrays (shared memory when TS, else global). The capacity
+// position is umulhi(word, W) (the top w bits); the tail gate of Eq. 5
+// (l_y <= L_i), a position test kl < kgate, is the lower half compared with
+// kgate << (16 - w). With capacities >= 0, max(Cexcl, gate ? c_y : 0) is the
+// patched row capacity.
+template <bool TS, int ROW>
+__device__ __forceinline__ uint64_t run_piece(const Plan& pl, int o, int q_lo, int q_hi, const float* win,
+                                              const float* h0, const float* h1, const float* kap0,
+                                              const float* thx0, const float* mnx0, const float* kap1,
+                                              const float* thx1, const float* mnx1) {
   const int st0 = __float_as_int(h0[H_STEP0]), st1 = __float_as_int(h1[H_STEP0]);
-  const float thb0 = h0[H_TH_BASE], mf0 = h0[H_M_FIRST], cx0 = h0[H_CX];
-  const float thb1 = h1[H_TH_BASE], mf1 = h1[H_M_FIRST], cx1 = h1[H_CX];
+  const float cx0 = h0[H_CX], cx1 = h1[H_CX];
+  const float lam = h0[H_LAM], rlam = __frcp_rn(lam);
+  const int cell = __float_as_int(h0[H_CELL]), p = __float_as_int(h0[H_P]);
+  const PhiloxKeys keys = philox_keys(pl.key0, pl.key1 ^ (pl.stream_base + (uint32_t)p));
+  const uint32_t ctr1 = (uint32_t)o, ctr2 = (uint32_t)cell, ctr3 = pl.round;
+  const uint32_t W = (uint32_t)pl.W;
+  const uint32_t kgs = (uint32_t)__float_as_int(win[0]) << pl.sh;
+  const float* sQo = win + 4;
+  Acc40 acc;
+  uint64_t total = 0;
+  auto eval = [&](uint32_t word) {
+    const float cy = sQo[__umulhi(word, W)];
+    const float cyg = (word & 0xFFFFu) < kgs ? cy : 0.0f;
+    const float t0 = tstar_of<ROW>(fmaxf(cx0, cyg), kap0, thx0, mnx0, st0, lam, rlam);
+    const float t1 = tstar_of<ROW>(fmaxf(cx1, cyg), kap1, thx1, mnx1, st1, lam, rlam);
+    acc.add(__fsub_rn(t1, t0));
+  };
+  const int q_full = min(q_hi, pl.S >> 2);  // calls whose four samples all exist
+  const int step = (int)blockDim.x;
+  int q = q_lo + (int)threadIdx.x;
+  while (q < q_full) {
+    // at most 256 calls (1024 values) between flushes of the 32-bit sums
+    const int q_end = min(q_full, q + 256 * step);
+    for (; q < q_end; q += step) {
+      const uint4 x = philox4x32_10(make_uint4((uint32_t)q, ctr1, ctr2, ctr3), keys);
+      eval(x.x);
+      eval(x.y);
+      eval(x.z);
+      eval(x.w);
+      acc.n += 4;
+    }
+    if (q < q_full) {
+      total += acc.value();
+      acc = Acc40();
+    }
+  }
+  if (q < q_hi) {  // the segment's last call, serving S mod 4 samples
+    const uint4 x = philox4x32_10(make_uint4((uint32_t)q, ctr1, ctr2, ctr3), keys);
+    const int nv = pl.S - 4 * q;
+    eval(x.x);
+    if (nv > 1) eval(x.y);
+    if (nv > 2) eval(x.z);
+    acc.n += (uint32_t)nv;
+  }
+  return total + acc.value();
+}
+
+// The same calls in dump mode: every scenario also writes its record (draws,
+// both t* and the per-class choices), with l_y mapped from the raw quantile
+// and the gate compared with the SLO directly.
+template <bool TS>
+__device__ uint64_t run_piece_dump(const Set& set, const Plan& pl, int item, int o, int q_lo, int q_hi,
+                                   const float* win, const float* h0, const float* h1, const float* kap0,
+                                   const float* thx0, const float* mnx0, const float* kap1, const float* thx1,
+                                   const float* mnx1, unsigned char* dump, int dump_stride) {
+  const int st0 = __float_as_int(h0[H_STEP0]), st1 = __float_as_int(h1[H_STEP0]);
+  const float cx0 = h0[H_CX], cx1 = h1[H_CX];
   const float lam = h0[H_LAM], rlam = __frcp_rn(lam);
   const int cell = __float_as_int(h0[H_CELL]), p = __float_as_int(h0[H_P]);
   const PhiloxKeys keys = philox_keys(pl.key0, pl.key1 ^ (pl.stream_base + (uint32_t)p));
   const uint32_t sh = (uint32_t)pl.sh;
   const int S = pl.S;
   const uint32_t ctr1 = (uint32_t)o, ctr2 = (uint32_t)cell, ctr3 = pl.round;
-  const int kgate = __float_as_int(win[0]);
   const float* sQo = win + 4;
+  const float lo_l = h0[H_LO_L], hi_l = h0[H_HI_L];
   uint64_t acc = 0;
   for (int q = q_lo + (int)threadIdx.x; q < q_hi; q += blockDim.x) {
     const uint4 x = philox4x32_10(make_uint4((uint32_t)q, ctr1, ctr2, ctr3), keys);
-#pragma unroll
     for (int h = 0; h < 4; ++h) {
       const int s = 4 * q + h;
+      if (s >= S) break;  // the last call may serve fewer than four samples
       const uint32_t word = h == 0 ? x.x : h == 1 ? x.y : h == 2 ? x.z : x.w;
       const int kc = (int)((word >> 16) >> sh);
       const int kl = (int)((word & 0xFFFFu) >> sh);
       const float cy = sQo[kc];
-      float ly = 0.0f;
-      bool gate;
-      if (DUMP) {
-        const float lo_l = h0[H_LO_L], hi_l = h0[H_HI_L];
-        ly = map_into(lo_l, __fsub_rn(hi_l, lo_l), hi_l, set.qn[(size_t)o * pl.W + kl]);
-        gate = ly <= h0[H_SLO];
-      } else {
-        gate = kl < kgate;
-      }
+      const float ly = map_into(lo_l, __fsub_rn(hi_l, lo_l), hi_l, set.qn[(size_t)o * pl.W + kl]);
+      const bool gate = ly <= h0[H_SLO];
       const float C0 = gate ? fmaxf(cx0, cy) : cx0;
       const float C1 = gate ? fmaxf(cx1, cy) : cx1;
-      const float t0 = tstar_of<ROW>(C0, kap0, tht0, mn0, st0, thb0, mf0, lam, rlam);
-      const float t1 = tstar_of<ROW>(C1, kap1, tht1, mn1, st1, thb1, mf1, lam, rlam);
-      const uint64_t gf = fixed40(__fsub_rn(t1, t0));
-      acc += (h == 0 || s < S) ? gf : 0ull;  // the last call may serve fewer than four samples
-      if (DUMP && (h == 0 || s < S)) {
-        const size_t idx = ((size_t)item * pl.O + o) * pl.S + s;
-        unsigned char* rec = dump + idx * dump_stride;
-        fs_scenario_head hd;
-        hd.c_y = cy;
-        hd.l_y = ly;
-        hd.t_star[0] = t0;
-        hd.t_star[1] = t1;
-        const int rr = cell / set.d.B, be = cell - rr * set.d.B;
-        uint32_t* ch = reinterpret_cast<uint32_t*>(rec + sizeof(fs_scenario_head));
-#pragma unroll
-        for (int sg = 0; sg < 2; ++sg) {
-          const float cx = sg ? cx1 : cx0;
-          const int bx = __float_as_int(sg ? h1[H_BX] : h0[H_BX]);
-          int bC;
-          if (!gate) bC = bx;
-          else if (bx < 0 || cy > cx) bC = be;
-          else if (cy == cx) bC = min(be, bx);
-          else bC = bx;
-          dump_choices(sg ? t1 : t0, set, (size_t)p * 2 + sg, rr, sg ? C1 : C0, bC, ch + sg * set.d.K,
-                       &hd.total_gpus[sg]);
-        }
-        *reinterpret_cast<fs_scenario_head*>(rec) = hd;
+      const float t0 = tstar_of<2>(C0, kap0, thx0, mnx0, st0, lam, rlam);
+      const float t1 = tstar_of<2>(C1, kap1, thx1, mnx1, st1, lam, rlam);
+      acc += fixed40(__fsub_rn(t1, t0));
+      const size_t idx = ((size_t)item * pl.O + o) * pl.S + s;
+      unsigned char* rec = dump + idx * dump_stride;
+      fs_scenario_head hd;
+      hd.c_y = cy;
+      hd.l_y = ly;
+      hd.t_star[0] = t0;
+      hd.t_star[1] = t1;
+      const int rr = cell / set.d.B, be = cell - rr * set.d.B;
+      uint32_t* ch = reinterpret_cast<uint32_t*>(rec + sizeof(fs_scenario_head));
+      for (int sg = 0; sg < 2; ++sg) {
+        const float cx = sg ? cx1 : cx0;
+        const int bx = __float_as_int(sg ? h1[H_BX] : h0[H_BX]);
+        int bC;
+        if (!gate) bC = bx;
+        else if (bx < 0 || cy > cx) bC = be;
+        else if (cy == cx) bC = min(be, bx);
+        else bC = bx;
+        dump_choices(sg ? t1 : t0, set, (size_t)p * 2 + sg, rr, sg ? C1 : C0, bC, ch + sg * set.d.K,
+                     &hd.total_gpus[sg]);
       }
+      *reinterpret_cast<fs_scenario_head*>(rec) = hd;
     }
   }
   return acc;
@@ -515,7 +591,7 @@ __device__ __forceinline__ void stage_segment(const Set& set, const Plan& pl, co
 // computed. The sums are integers, so the order of the chunks does not
 // change the result.
 template <bool DUMP>
-__global__ void __launch_bounds__(kScoreThreads, 5) k_score(Set set, Items it, Plan pl, const float* rec,
+__global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, Plan pl, const float* rec,
                                                          uint64_t* sums, unsigned char* dump, int dump_stride,
                                                          ScoreGrid sg) {
   extern __shared__ __align__(16) unsigned char smraw[];
@@ -584,18 +660,23 @@ __global__ void __launch_bounds__(kScoreThreads, 5) k_score(Set set, Items it, P
       const bool f0 = __float_as_int(h0[H_FAST]) != 0, f1 = __float_as_int(h1[H_FAST]) != 0;
       const int row = DUMP ? 2 : (!r0 && !r1) ? 0 : ((!r0 || f0) && (!r1 || f1)) ? 1 : 2;
       // the table pointers stay in one address space per branch (shared or global)
-#define FS_PIECE(TSV, ROWV)                                                                                 \
-  run_piece<DUMP, TSV, ROWV>(set, pl, item, o, q_lo, q_hi, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, \
-                             k1 + Lp1, k1 + 2 * Lp1, dump, dump_stride)
+#define FS_PIECE(TSV, ROWV) \
+  run_piece<TSV, ROWV>(pl, o, q_lo, q_hi, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, k1 + Lp1, k1 + 2 * Lp1)
+#define FS_DUMP(TSV)                                                                                   \
+  run_piece_dump<TSV>(set, pl, item, o, q_lo, q_hi, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, k1 + Lp1, \
+                      k1 + 2 * Lp1, dump, dump_stride)
       if (Lp0 <= sg.lcap_s && Lp1 <= sg.lcap_s) {
         const float* k0 = h0 + kTableHeader;
         const float* k1 = h1 + kTableHeader;
-        acc = row == 0 ? FS_PIECE(true, 0) : row == 1 ? FS_PIECE(true, 1) : FS_PIECE(true, 2);
+        if constexpr (DUMP) acc = FS_DUMP(true);
+        else acc = row == 0 ? FS_PIECE(true, 0) : row == 1 ? FS_PIECE(true, 1) : FS_PIECE(true, 2);
       } else {
         const float* k0 = rec + (size_t)item * pl.item_floats + kTableHeader;
         const float* k1 = k0 + d.slot_floats;
-        acc = row == 0 ? FS_PIECE(false, 0) : row == 1 ? FS_PIECE(false, 1) : FS_PIECE(false, 2);
+        if constexpr (DUMP) acc = FS_DUMP(false);
+        else acc = row == 0 ? FS_PIECE(false, 0) : row == 1 ? FS_PIECE(false, 1) : FS_PIECE(false, 2);
       }
+#undef FS_DUMP
 #undef FS_PIECE
     }
     for (int off = 16; off; off >>= 1) acc += __shfl_down_sync(0xffffffffu, acc, off);
