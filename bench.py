@@ -36,18 +36,25 @@ from paper_2608_19659_gb300 import workloads  # noqa: E402
 
 METRIC = "scenario allocation-solves/s"
 UNIT = "allocation-solves/s"
-SMS = 152
 ISSUE_PER_SM_CLK = 4 * 32  # 4 schedulers x 32 lanes, one warp instruction each per clock
 
-# Algorithmic thread-operations per scenario of the Monte-Carlo kernel (the
-# instruction-level minimum of the method's arithmetic; derivation in the
-# design notes): half a Philox4x32-10 call (10 rounds x 2 wide multiplies +
-# 2 three-input XORs) = 20, two quantile positions + lookups = 4, two affine
-# maps with clamps = 8, tail gate and two row patches = 5, two fulfilments
-# f = min(1, m C / lambda) with an IEEE division (>= 7 each) and the
-# max with the table threshold (2 each) = 18, gap and fixed-point add = 5.
-# The table searches (3 per probe) are not counted: a lower bound.
-OPS_PER_SCENARIO = 60
+# Algorithmic thread-operations per scenario of the Monte-Carlo kernel: the
+# operations every scenario of the parametric re-solve performs.
+#   a quarter of one Philox4x32-10 call (10 rounds x (2 wide multiplies +
+#   2 three-input XORs), four samples per call)                          10
+#   capacity position (high multiply), its address, the lookup            3
+#   tail gate (mask, compare) and the gated capacity                      3
+#   the two patched row capacities (max with Cexcl)                       2
+#   two table searches: loop test, address, read of the reached threshold 6
+#   Gamma' = t*(A+') - t*(A-')                                             1
+#   exact fixed-point accumulation of rint(Gamma' 2^40)                   7
+# Search probes beyond the first (3 each) and row-term fulfilments (where a
+# reachable threshold leaves row r a replica) are not counted: a lower bound.
+OPS_PER_SCENARIO = 32
+
+# ncu summaries with the DRAM bytes of one k_score launch, per workload; used
+# for roofline.traffic only while the scorer source is the one profiled.
+PROFILES = {1: "k_score_paper_scale.md", 3: "k_score_large.md"}
 
 
 def _env_int(name, default):
@@ -55,6 +62,30 @@ def _env_int(name, default):
         return int(os.environ.get(name, default))
     except ValueError:
         return default
+
+
+def _profiled_traffic(workload: int):
+    """DRAM bytes (read + write) of one k_score launch from the committed ncu
+    summary of this workload, or None when there is none or the scorer source
+    changed since it was taken (its sha256 prefix is recorded in the summary)."""
+    import hashlib
+    import re
+
+    name = PROFILES.get(workload)
+    if not name:
+        return None
+    try:
+        text = open(os.path.join(ROOT, "profiles", name)).read()
+        src = open(os.path.join(ROOT, "paper_2608_19659_gb300", "csrc", "fs_score.cu"), "rb").read()
+    except OSError:
+        return None
+    m = re.search(r"sha256 prefix `([0-9a-f]+)`", text)
+    if not m or not hashlib.sha256(src).hexdigest().startswith(m.group(1)):
+        return None
+    m = re.search(r"dram__bytes_read\.sum \+ dram__bytes_write\.sum \| ([0-9,]+) B \+ ([0-9,]+) B", text)
+    if not m:
+        return None
+    return float(m.group(1).replace(",", "")) + float(m.group(2).replace(",", ""))
 
 
 def _measured_peaks():
@@ -338,16 +369,18 @@ def main(argv=None):
     peaks = _measured_peaks()
     clk = clocks.summary()
     sm_max = float(peaks.get("sm_max_mhz", 2070.0))
-    alu_peak = SMS * ISSUE_PER_SM_CLK * sm_max * 1e6  # thread-ops/s at the maximum SM clock
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    alu_peak = sms * ISSUE_PER_SM_CLK * sm_max * 1e6  # thread-ops/s at the maximum SM clock
     kern_s = kernel_ms / 1000.0 / max(kernel_n, 1)
     achieved = OPS_PER_SCENARIO * w.scenarios / kern_s if kernel_n else None
     roofline = {"bound": "alu", "kernel": "k_score (Monte-Carlo sampler + parametric re-solve)",
                 "achieved": achieved / 1e12 if achieved else None,
                 "peak": alu_peak / 1e12, "unit": "Tops/s (32-bit thread operations)",
                 "frac": (achieved / alu_peak) if achieved else None,
-                "traffic": None, "kernel_ms_per_launch": kern_s * 1000.0,
+                "traffic": _profiled_traffic(args.workload), "traffic_unit": "DRAM bytes per launch (ncu)",
+                "algorithmic_bytes": 0, "kernel_ms_per_launch": kern_s * 1000.0,
                 "ops_per_scenario": OPS_PER_SCENARIO,
-                "peak_basis": f"{SMS} SMs x 4 issue slots x 32 lanes x {sm_max:.0f} MHz (max SM clock)",
+                "peak_basis": f"{sms} SMs x 4 issue slots x 32 lanes x {sm_max:.0f} MHz (max SM clock)",
                 "kernel_share_of_step": (kernel_ms / max(sum(step_ms), 1e-9)) if kernel_n else None}
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

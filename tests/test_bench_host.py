@@ -74,3 +74,27 @@ def test_reference_arm_non_zero_ranks_exit_quietly():
     assert all(p.returncode == 0 for p in procs), [o[1] for o in outs]
     assert len([ln for ln in outs[0][0].splitlines() if ln.strip()]) == 1
     assert outs[1][0].strip() == ""
+
+
+def test_roofline_traffic_only_for_the_profiled_source(tmp_path, monkeypatch):
+    """roofline.traffic comes from the committed ncu summary while the scorer
+    source is the profiled one, and is null once that source changes."""
+    import shutil
+
+    sys.path.insert(0, ROOT)
+    import bench
+
+    got = bench._profiled_traffic(1)
+    assert got is not None and got > 0
+    assert bench._profiled_traffic(2) is None  # no summary for that workload
+    # a copy of the tree whose scorer source differs by one byte
+    (tmp_path / "profiles").mkdir()
+    shutil.copy(os.path.join(ROOT, "profiles", bench.PROFILES[1]), tmp_path / "profiles")
+    csrc = tmp_path / "paper_2608_19659_gb300" / "csrc"
+    csrc.mkdir(parents=True)
+    src = open(os.path.join(ROOT, "paper_2608_19659_gb300", "csrc", "fs_score.cu"), "rb").read()
+    (csrc / "fs_score.cu").write_bytes(src)
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    assert bench._profiled_traffic(1) == got
+    (csrc / "fs_score.cu").write_bytes(src + b"\n")
+    assert bench._profiled_traffic(1) is None
