@@ -186,6 +186,7 @@ Plan make_plan(const fs_model* m, const fs_samples* s, int n_items) {
   pl.W = m->d.Q / s->O;
   pl.w = log2i(pl.W);
   pl.sh = 16 - pl.w;
+  pl.logO = log2i(s->O);
   pl.calls = (s->S + 3) / 4;
   pl.Wp = 4 + ((pl.W + 3) & ~3);
   pl.item_floats = 2LL * m->d.slot_floats + (long long)s->O * pl.Wp;

@@ -7,19 +7,44 @@
 namespace fs {
 
 // Per problem: E[Gamma_{t+1} | e], score, and the argmax (largest score, then
-// lower TP = fewer profiling GPU-seconds, then earlier candidate).
+// lower TP = fewer profiling GPU-seconds, then earlier candidate). The order
+// is carried as a key compared without branches: hi = the score's fixed-point
+// value (the smallest int64 for "no candidate"), lo = (3 - j) 2^30 +
+// (2^30 - 1 - pos), larger is better in both (pos < 2^30: n_cand O <= 2^30).
+constexpr long long kNoScore = (-0x7FFFFFFFFFFFFFFFLL - 1);
+
 struct Best {
-  long long sc;
-  int j;
-  int pos;
+  long long hi;
+  uint32_t lo;
+  int cell;  // the candidate's cell, carried so that no load follows the reduction
+  __device__ __forceinline__ bool valid() const { return hi != kNoScore; }
+  __device__ __forceinline__ int pos() const { return (int)(0x3FFFFFFFu - (lo & 0x3FFFFFFFu)); }
 };
 
+__device__ __forceinline__ Best make_best(long long sc, int j, int pos, int cell) {
+  return Best{sc, ((uint32_t)(3 - j) << 30) | (0x3FFFFFFFu - (uint32_t)pos), cell};
+}
+
+__device__ __forceinline__ Best no_best() { return Best{kNoScore, 0u, -1}; }
+
 __device__ __forceinline__ bool better(const Best& a, const Best& b) {
-  if (a.pos < 0) return false;
-  if (b.pos < 0) return true;
-  if (a.sc != b.sc) return a.sc > b.sc;
-  if (a.j != b.j) return a.j < b.j;
-  return a.pos < b.pos;
+  return a.hi > b.hi || (a.hi == b.hi && a.lo > b.lo);
+}
+
+// The best of the 32 lanes' values (butterfly over xor-shuffles: every lane
+// ends with it).
+__device__ __forceinline__ Best warp_best(Best b) {
+  for (int off = 16; off; off >>= 1) {
+    Best o;
+    o.hi = __shfl_xor_sync(0xffffffffu, b.hi, off);
+    o.lo = __shfl_xor_sync(0xffffffffu, b.lo, off);
+    o.cell = __shfl_xor_sync(0xffffffffu, b.cell, off);
+    const bool t = better(o, b);
+    b.hi = t ? o.hi : b.hi;
+    b.lo = t ? o.lo : b.lo;
+    b.cell = t ? o.cell : b.cell;
+  }
+  return b;
 }
 
 // (v * 2^-40) / n rounded to the nearest double, for 0 <= v < 2^63 and n >= 1,
@@ -54,35 +79,33 @@ __device__ inline Best finalize_problem(const Set& set, const Items& it, const P
   __shared__ Best sb[32];
   const Dims& d = set.d;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = blockDim.x >> 5;
-  const float gt = __fsub_rn(set.base[2 * p + 1].t_star, set.base[2 * p].t_star);
+  // inputs are read-only here (written by earlier kernels): every load goes
+  // through the read-only path and is issued before any store
+  const float gt = __fsub_rn(__ldg(&set.base[2 * p + 1].t_star), __ldg(&set.base[2 * p].t_star));
   const long long gfix = (long long)fixed40(gt);
   const long long n = (long long)pl.O * pl.S;
   const int log2n = (n & (n - 1)) == 0 ? 63 - __clzll(n) : -1;
-  Best b{0, 0, -1};
+  Best b = no_best();
   for (int q = beg + tid; q < end; q += blockDim.x) {
+    const int cell = __ldg(it.cell + q);
     long long tot = 0;
 #pragma unroll 8
-    for (int o = 0; o < pl.O; ++o) tot += (long long)sums[(size_t)q * pl.O + o];
+    for (int o = 0; o < pl.O; ++o) tot += (long long)__ldg(sums + (size_t)q * pl.O + o);
     const long long sc = gfix * n - tot;
     if (gap) gap[q] = fixed_mean((unsigned long long)tot, n, log2n);
     if (score) score[q] = fixed_mean((unsigned long long)sc, n, log2n);
-    const Best c{sc, (it.cell[q] / d.B) & 3, q - beg};
+    const Best c = make_best(sc, (cell / d.B) & 3, q - beg, cell);
     if (better(c, b)) b = c;
   }
-  for (int off = 16; off; off >>= 1) {
-    Best o;
-    o.sc = __shfl_xor_sync(0xffffffffu, b.sc, off);
-    o.j = __shfl_xor_sync(0xffffffffu, b.j, off);
-    o.pos = __shfl_xor_sync(0xffffffffu, b.pos, off);
-    if (better(o, b)) b = o;
-  }
+  b = warp_best(b);
   if (lane == 0) sb[warp] = b;
   __syncthreads();
-  if (tid == 0) {
-    for (int w = 1; w < nwarp; ++w)
-      if (better(sb[w], b)) b = sb[w];
-    sb[0] = b;
-    if (gt_out) *gt_out = gt;
+  if (warp == 0) {  // the warps' results, reduced by warp 0 in parallel
+    b = warp_best(lane < nwarp ? sb[lane] : no_best());
+    if (lane == 0) {
+      sb[0] = b;
+      if (gt_out) *gt_out = gt;
+    }
   }
   __syncthreads();
   return sb[0];

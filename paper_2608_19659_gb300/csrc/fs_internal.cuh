@@ -52,6 +52,7 @@ enum : int {
   H_STEP0 = 15,   // first step of the table search, P/2 with P = pow2 >= L + 1 (int, 0 if L = 0)
   H_ROW = 16,     // 1 if row r can buy a replica at some reachable threshold (int)
   H_FAST = 17,    // 1 if every reachable row-term quotient is in Markstein's range (int)
+  H_RLAM = 18,    // RN(1 / lambda)
 };
 
 enum : int { CAP_LO = 0, CAP_HI = 1, TAIL_LO = 2, TAIL_HI = 3 };
@@ -98,6 +99,7 @@ struct Plan {
   uint32_t stream_base; // stream id of problem 0 (problem p uses stream_base + p)
   uint32_t round;
   int O, S, W, w;       // W = Q / O quantiles per stratum, w = log2(W) <= 16
+  int logO;             // log2(O) (O is a power of two)
   int sh;               // 16 - w: a 16-bit field's top w bits are field >> sh
   int calls;            // ceil(S / 4) Philox calls per (candidate, outcome)
   int Wp;               // floats per mapped outcome window: 4 + W rounded up to 4

@@ -89,7 +89,7 @@ __global__ void k_replay_reveal(Set set, ReplayState rs, Items it, Plan pl, cons
   const int a = blockIdx.x;
   const int p = rs.active[a];
   const Best b = finalize_problem(set, it, pl, sums, p, a * per, (a + 1) * per, nullptr, nullptr, nullptr);
-  if (threadIdx.x == 0 && b.pos >= 0) reveal_cell(set, rs, p, it.cell[a * per + b.pos]);
+  if (threadIdx.x == 0 && b.valid()) reveal_cell(set, rs, p, b.cell);
 }
 
 cudaError_t launch_replay_init(const Set& set, const ReplayState& rs, int r0, cudaStream_t s) {

@@ -351,6 +351,7 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
     tab[H_STEP0] = __int_as_float(Lt ? P >> 1 : 0);
     tab[H_ROW] = __int_as_float(s_row);
     tab[H_FAST] = __int_as_float(fast ? 1 : 0);
+    tab[H_RLAM] = rl;
   }
 }
 
@@ -441,16 +442,20 @@ __device__ void dump_choices(float t, const Set& set, size_t ps, int rr, float C
 // (l_y <= L_i), a position test kl < kgate, is the lower half compared with
 // kgate << (16 - w). With capacities >= 0, max(Cexcl, gate ? c_y : 0) is the
 // patched row capacity.
+struct PieceSum {
+  Acc40 acc;       // the last at most 1024 values
+  uint64_t total;  // earlier values, flushed
+};
+
 template <bool TS, int ROW>
-__device__ __forceinline__ uint64_t run_piece(const Plan& pl, int o, int q_lo, int q_hi, const float* win,
-                                              const float* h0, const float* h1, const float* kap0,
-                                              const float* thx0, const float* mnx0, const float* kap1,
-                                              const float* thx1, const float* mnx1) {
+__device__ __forceinline__ PieceSum run_piece(const Plan& pl, const PhiloxKeys& keys, int o, int q_lo, int q_hi,
+                                              const float* win, const float* h0, const float* h1,
+                                              const float* kap0, const float* thx0, const float* mnx0,
+                                              const float* kap1, const float* thx1, const float* mnx1) {
   const int st0 = __float_as_int(h0[H_STEP0]), st1 = __float_as_int(h1[H_STEP0]);
   const float cx0 = h0[H_CX], cx1 = h1[H_CX];
-  const float lam = h0[H_LAM], rlam = __frcp_rn(lam);
-  const int cell = __float_as_int(h0[H_CELL]), p = __float_as_int(h0[H_P]);
-  const PhiloxKeys keys = philox_keys(pl.key0, pl.key1 ^ (pl.stream_base + (uint32_t)p));
+  const float lam = h0[H_LAM], rlam = h0[H_RLAM];
+  const int cell = __float_as_int(h0[H_CELL]);
   const uint32_t ctr1 = (uint32_t)o, ctr2 = (uint32_t)cell, ctr3 = pl.round;
   const uint32_t W = (uint32_t)pl.W;
   const uint32_t kgs = (uint32_t)__float_as_int(win[0]) << pl.sh;
@@ -491,7 +496,7 @@ __device__ __forceinline__ uint64_t run_piece(const Plan& pl, int o, int q_lo, i
     if (nv > 2) eval(x.z);
     acc.n += (uint32_t)nv;
   }
-  return total + acc.value();
+  return PieceSum{acc, total};
 }
 
 // The same calls in dump mode: every scenario also writes its record (draws,
@@ -571,7 +576,7 @@ struct ScoreGrid {
 // candidate tables, header plus lcap_s entries each) into dst, completing on bar.
 __device__ __forceinline__ void stage_segment(const Set& set, const Plan& pl, const float* rec, int seg,
                                               float* dst, uint64_t* bar, int tcopy) {
-  const int item = seg / pl.O, o = seg - item * pl.O;
+  const int item = seg >> pl.logO, o = seg & (pl.O - 1);
   const float* r = rec + (size_t)item * pl.item_floats;
   const uint32_t tb = (uint32_t)tcopy * 4u, wb = (uint32_t)pl.Wp * 4u;
   fence_proxy_async();
@@ -598,7 +603,8 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
   uint64_t* bar = reinterpret_cast<uint64_t*>(smraw);  // [2]
   float* stage0 = reinterpret_cast<float*>(smraw + 16);
   const int stage_floats = pl.Wp + 2 * sg.tcopy;
-  __shared__ int s_chunk[2];
+  // per stage: chunk index, its segment and its part (thread 0 divides once)
+  __shared__ int s_chunk[2], s_seg[2], s_part[2];
   const Dims& d = set.d;  // kernel-parameter space: d.M[j] reads need no local copy
   const int tid = threadIdx.x, lane = tid & 31;
   (void)it;
@@ -609,13 +615,20 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
   if (tid == 0) {
     mbar_init(&bar[0], 1);
     mbar_init(&bar[1], 1);
-    s_chunk[0] = (int)blockIdx.x;  // the grid has at most sg.total blocks
+    const int c0 = (int)blockIdx.x;  // the grid has at most sg.total blocks
+    s_chunk[0] = c0;
+    s_seg[0] = c0 / sg.nch;
+    s_part[0] = c0 - s_seg[0] * sg.nch;
   }
   __syncthreads();
   if (tid == 0) {
-    stage_segment(set, pl, rec, (int)blockIdx.x / sg.nch, stage0, &bar[0], sg.tcopy);
+    stage_segment(set, pl, rec, s_seg[0], stage0, &bar[0], sg.tcopy);
     next = (int)blockIdx.x + g;  // may pass sg.total: then the block stops after one chunk
   }
+  // 32-bit warp sums are exact while a thread holds at most 32 values
+  const bool small = sg.chunk <= 8 * (int)blockDim.x;
+  PhiloxKeys keys;
+  int keys_p = -1;  // problem whose round keys are in `keys`
 
   for (int j = 0;; ++j) {
     const int st = j & 1;
@@ -624,8 +637,10 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
     if (tid == 0) {
       s_chunk[st ^ 1] = next;
       if (next < sg.total) {
-        stage_segment(set, pl, rec, next / sg.nch, stage0 + (size_t)(st ^ 1) * stage_floats, &bar[st ^ 1],
-                      sg.tcopy);
+        const int sn = next / sg.nch;
+        s_seg[st ^ 1] = sn;
+        s_part[st ^ 1] = next - sn * sg.nch;
+        stage_segment(set, pl, rec, sn, stage0 + (size_t)(st ^ 1) * stage_floats, &bar[st ^ 1], sg.tcopy);
         if (sg.dyn) {
           // consumed one chunk later; saturates at sg.total so that it cannot wrap
           const unsigned long long v = atomicAdd(set.work, 1ull) + 2ull * (unsigned long long)g;
@@ -635,54 +650,70 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
         }
       }
     }
+    // a thread whose wait succeeded may use the stage; the barrier at the end
+    // of the chunk tells every thread whether any wait gave up
     const bool ok = mbar_wait(&bar[st], (uint32_t)((j >> 1) & 1), kWaitLimitNs);
-    if (__syncthreads_or(!ok)) {
-      if (tid == 0) atomicOr(set.status, ST_TIMEOUT);
-      // let copies in flight land before the block exits (bounded as well)
-      mbar_wait(&bar[st], (uint32_t)((j >> 1) & 1), kWaitLimitNs);
-      if (s_chunk[st ^ 1] < sg.total) mbar_wait(&bar[st ^ 1], (uint32_t)(((j + 1) >> 1) & 1), kWaitLimitNs);
-      return;
-    }
     const float* stg = stage0 + (size_t)st * stage_floats;
     const float* h0 = stg + pl.Wp;
     const float* h1 = h0 + sg.tcopy;
-    const int seg = c / sg.nch;
-    const int part = c - seg * sg.nch;
-    const int item = seg / pl.O, o = seg - item * pl.O;
+    const int seg = s_seg[st], part = s_part[st];
+    const int item = seg >> pl.logO, o = seg & (pl.O - 1);
     const int q_lo = part * sg.chunk;
     const int q_hi = min(q_lo + sg.chunk, pl.calls);
-    const int Lp0 = __float_as_int(h0[H_LPAD]), Lp1 = __float_as_int(h1[H_LPAD]);
-    const int cell = __float_as_int(h0[H_CELL]);
-    const bool cell_ok = cell >= 0 && cell < d.cells;  // a bad device-side id was flagged by k_prep
-    uint64_t acc = 0;
-    if (cell_ok) {
-      const bool r0 = __float_as_int(h0[H_ROW]) != 0, r1 = __float_as_int(h1[H_ROW]) != 0;
-      const bool f0 = __float_as_int(h0[H_FAST]) != 0, f1 = __float_as_int(h1[H_FAST]) != 0;
-      const int row = DUMP ? 2 : (!r0 && !r1) ? 0 : ((!r0 || f0) && (!r1 || f1)) ? 1 : 2;
-      // the table pointers stay in one address space per branch (shared or global)
+    PieceSum ps{Acc40(), 0ull};
+    uint64_t acc_dump = 0;
+    if (ok) {
+      const int Lp0 = __float_as_int(h0[H_LPAD]), Lp1 = __float_as_int(h1[H_LPAD]);
+      const int cell = __float_as_int(h0[H_CELL]);
+      if (cell >= 0 && cell < d.cells) {  // a bad device-side id was flagged by k_prep
+        const bool r0 = __float_as_int(h0[H_ROW]) != 0, r1 = __float_as_int(h1[H_ROW]) != 0;
+        const bool f0 = __float_as_int(h0[H_FAST]) != 0, f1 = __float_as_int(h1[H_FAST]) != 0;
+        const int row = (!r0 && !r1) ? 0 : ((!r0 || f0) && (!r1 || f1)) ? 1 : 2;
+        const int p = __float_as_int(h0[H_P]);
+        if (!DUMP && p != keys_p) {
+          keys = philox_keys(pl.key0, pl.key1 ^ (pl.stream_base + (uint32_t)p));
+          keys_p = p;
+        }
+        // the table pointers stay in one address space per branch (shared or global)
 #define FS_PIECE(TSV, ROWV) \
-  run_piece<TSV, ROWV>(pl, o, q_lo, q_hi, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, k1 + Lp1, k1 + 2 * Lp1)
+  run_piece<TSV, ROWV>(pl, keys, o, q_lo, q_hi, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, k1 + Lp1, k1 + 2 * Lp1)
 #define FS_DUMP(TSV)                                                                                   \
   run_piece_dump<TSV>(set, pl, item, o, q_lo, q_hi, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, k1 + Lp1, \
                       k1 + 2 * Lp1, dump, dump_stride)
-      if (Lp0 <= sg.lcap_s && Lp1 <= sg.lcap_s) {
-        const float* k0 = h0 + kTableHeader;
-        const float* k1 = h1 + kTableHeader;
-        if constexpr (DUMP) acc = FS_DUMP(true);
-        else acc = row == 0 ? FS_PIECE(true, 0) : row == 1 ? FS_PIECE(true, 1) : FS_PIECE(true, 2);
-      } else {
-        const float* k0 = rec + (size_t)item * pl.item_floats + kTableHeader;
-        const float* k1 = k0 + d.slot_floats;
-        if constexpr (DUMP) acc = FS_DUMP(false);
-        else acc = row == 0 ? FS_PIECE(false, 0) : row == 1 ? FS_PIECE(false, 1) : FS_PIECE(false, 2);
-      }
+        if (Lp0 <= sg.lcap_s && Lp1 <= sg.lcap_s) {
+          const float* k0 = h0 + kTableHeader;
+          const float* k1 = h1 + kTableHeader;
+          if constexpr (DUMP) acc_dump = FS_DUMP(true);
+          else ps = row == 0 ? FS_PIECE(true, 0) : row == 1 ? FS_PIECE(true, 1) : FS_PIECE(true, 2);
+        } else {
+          const float* k0 = rec + (size_t)item * pl.item_floats + kTableHeader;
+          const float* k1 = k0 + d.slot_floats;
+          if constexpr (DUMP) acc_dump = FS_DUMP(false);
+          else ps = row == 0 ? FS_PIECE(false, 0) : row == 1 ? FS_PIECE(false, 1) : FS_PIECE(false, 2);
+        }
 #undef FS_DUMP
 #undef FS_PIECE
+      }
     }
-    for (int off = 16; off; off >>= 1) acc += __shfl_down_sync(0xffffffffu, acc, off);
-    if (lane == 0 && acc)
-      atomicAdd(reinterpret_cast<unsigned long long*>(&sums[(size_t)seg]), (unsigned long long)acc);
-    __syncthreads();  // stage st is free for the copies issued next iteration
+    if (!DUMP && small) {
+      // at most 32 values per thread: each part's warp sum fits in 32 bits
+      const uint32_t H = __reduce_add_sync(0xffffffffu, ps.acc.h - ps.acc.n * 0x4B000000u);
+      const int32_t Lo = (int32_t)__reduce_add_sync(0xffffffffu, ps.acc.l - ps.acc.n * 0x4B400000u);
+      const uint64_t v = ((uint64_t)H << 20) + (uint64_t)(int64_t)Lo;
+      if (lane == 0 && v) atomicAdd(reinterpret_cast<unsigned long long*>(&sums[(size_t)seg]), (unsigned long long)v);
+    } else {
+      uint64_t v = DUMP ? acc_dump : ps.total + ps.acc.value();
+      for (int off = 16; off; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
+      if (lane == 0 && v) atomicAdd(reinterpret_cast<unsigned long long*>(&sums[(size_t)seg]), (unsigned long long)v);
+    }
+    // stage st is free for the copies issued next iteration
+    if (__syncthreads_or(!ok)) {
+      if (tid == 0) atomicOr(set.status, ST_TIMEOUT);
+      // let copies in flight land before the block exits (bounded as well)
+      if (!ok) mbar_wait(&bar[st], (uint32_t)((j >> 1) & 1), kWaitLimitNs);
+      if (s_chunk[st ^ 1] < sg.total) mbar_wait(&bar[st ^ 1], (uint32_t)(((j + 1) >> 1) & 1), kWaitLimitNs);
+      return;
+    }
   }
   pdl_trigger();
 }
@@ -694,7 +725,7 @@ __global__ void k_finalize(Set set, Items it, Plan pl, const uint64_t* sums, dou
   const int beg = it.off ? it.off[p] : 0;
   const int end = it.off ? it.off[p + 1] : it.n;
   const Best b = finalize_problem(set, it, pl, sums, p, beg, end, gap, score, gamma_t ? gamma_t + p : nullptr);
-  if (threadIdx.x == 0 && best) best[p] = b.pos >= 0 ? it.cell[beg + b.pos] : -1;
+  if (threadIdx.x == 0 && best) best[p] = b.valid() ? b.cell : -1;
 }
 
 static size_t prep_smem_bytes(const Dims& d) { return (size_t)(256 + d.theta_cap) * 4; }

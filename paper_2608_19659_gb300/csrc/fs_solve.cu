@@ -41,13 +41,17 @@ __global__ void k_qtable(float* qn, int Q) {
 }
 
 // Total GPUs of the cheapest per-class covers of threshold t, or kCostInf if
-// some class has no cover. Called by a whole warp; rows rho = 4 i + j.
-__device__ __forceinline__ int warp_total_cost(float t, const float* sC, const float* sLam, const float* sRl,
-                                               const Dims& d, int lane) {
-  int total = 0;
-  bool inf = false;
-  for (int base = 0; base < d.K4; base += 32) {
-    const int rho = base + lane;
+// some class has no cover, evaluated by an aligned group of gsz lanes (a power
+// of two in [4, 32]); lane gl takes rows gl, gl + gsz, ... (rho = 4 i + j).
+// After the per-class minimum (two xor-shuffles) all four lanes of a class
+// hold its cost; xor-sums over the offsets 4 .. gsz/2 then add one lane per
+// class, so every lane of the group ends with the total (uncovered classes
+// counted above bit 24: a cost is at most G <= 32767, 64 classes < 2^21).
+__device__ __forceinline__ int group_total_cost(float t, const float* sC, const float* sLam, const float* sRl,
+                                                const Dims& d, int gl, int gsz) {
+  int packed = 0;
+  for (int base = 0; base < d.K4; base += gsz) {
+    const int rho = base + gl;
     int cost = kCostInf;
     if (rho < d.K4) {
       const int j = rho & 3;
@@ -56,11 +60,11 @@ __device__ __forceinline__ int warp_total_cost(float t, const float* sC, const f
     }
     cost = min(cost, __shfl_xor_sync(0xffffffffu, cost, 1));
     cost = min(cost, __shfl_xor_sync(0xffffffffu, cost, 2));
-    const bool head = rho < d.K4 && (lane & 3) == 0;
-    if (__ballot_sync(0xffffffffu, head && cost >= kCostInf)) inf = true;
-    total += __reduce_add_sync(0xffffffffu, (head && cost < kCostInf) ? cost : 0);
+    int v = rho < d.K4 ? (cost >= kCostInf ? (1 << 24) : cost) : 0;
+    for (int off = 4; off < gsz; off <<= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
+    packed += v;
   }
-  return inf ? kCostInf : total;
+  return (packed >> 24) ? kCostInf : packed;
 }
 
 __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, const float* cap_x,
@@ -69,7 +73,7 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   extern __shared__ __align__(16) unsigned char smraw[];
   const Dims& d = set.d;  // kernel-parameter space: d.M[j] reads need no local copy
   const int r = blockIdx.x;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = blockDim.x >> 5;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   pdl_trigger();
   if (r >= n_real) return;
 
@@ -228,33 +232,32 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
     }
   }
 
-  // 3. search: largest index whose threshold fits in G (lo feasible, hi not)
-  if (tid == 0) {
-    sMisc[0] = -1;
-    sMisc[1] = total;
-    sMisc[4] = 0;
-  }
+  // 3. search: largest index whose threshold fits in G (lo feasible, hi not).
+  // Each round every group of gsz lanes probes one index (an (ng+1)-ary
+  // split); each warp merges the answers with integer max / min reductions,
+  // so a round costs one barrier.
+  __shared__ int s_res[2][kSolveThreads / 4];
+  if (tid == 0) sMisc[4] = 0;
   __syncthreads();
-  while (sMisc[1] - sMisc[0] > 1) {
-    const int lo = sMisc[0], hi = sMisc[1];
-    const int span = hi - lo;
-    int kp = lo + (int)(((long long)(warp + 1) * span) / (nwarp + 1));
+  int gsz = 4;
+  while (gsz < d.K4 && gsz < 32) gsz <<= 1;
+  const int ng = blockDim.x / gsz, g = tid / gsz, gl = tid & (gsz - 1);
+  int lo = -1, hi = total;
+  for (int par = 0; hi - lo > 1; par ^= 1) {
+    int kp = lo + ((g + 1) * (hi - lo)) / (ng + 1);
     kp = max(lo + 1, min(hi - 1, kp));
-    const int cost = warp_total_cost(sTheta[kp], sC, sLam, sRl, d, lane);
-    if (lane == 0) sProbe[warp] = (cost <= d.G) ? kp : -(kp + 1);
+    const int cost = group_total_cost(sTheta[kp], sC, sLam, sRl, d, gl, gsz);
+    if (gl == 0) s_res[par][g] = (cost <= d.G) ? kp : -(kp + 1);
     __syncthreads();
-    if (tid == 0) {
-      int nlo = lo, nhi = hi;
-      for (int w = 0; w < nwarp; ++w) {
-        const int v = sProbe[w];
-        if (v >= 0) nlo = max(nlo, v); else nhi = min(nhi, -v - 1);
-      }
-      sMisc[0] = nlo;
-      sMisc[1] = nhi;
+    int nlo = lo, nhi = hi;
+    for (int q = lane; q < ng; q += 32) {
+      const int v = s_res[par][q];
+      if (v >= 0) nlo = max(nlo, v); else nhi = min(nhi, -v - 1);
     }
-    __syncthreads();
+    lo = __reduce_max_sync(0xffffffffu, nlo);
+    hi = __reduce_min_sync(0xffffffffu, nhi);
   }
-  const int kstar = sMisc[0];
+  const int kstar = lo;
   const float tstar = kstar >= 0 ? sTheta[kstar] : 0.0f;
 
   // 4. choice at t*: every row's cheapest cover in parallel (thread = row), then

@@ -185,6 +185,8 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
   pl.w = 0;
   while ((1 << pl.w) < pl.W) ++pl.w;
   pl.sh = 16 - pl.w;
+  pl.logO = 0;
+  while ((1 << pl.logO) < pl.O) ++pl.logO;
   pl.calls = (smp->S + 3) / 4;
   pl.Wp = Wp;
   pl.item_floats = (long long)item_floats;

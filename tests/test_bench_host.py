@@ -77,24 +77,31 @@ def test_reference_arm_non_zero_ranks_exit_quietly():
 
 
 def test_roofline_traffic_only_for_the_profiled_source(tmp_path, monkeypatch):
-    """roofline.traffic comes from the committed ncu summary while the scorer
-    source is the profiled one, and is null once that source changes."""
-    import shutil
+    """roofline.traffic comes from an ncu summary of the bench's workload while
+    the scorer source has the sha256 the summary records, and is null otherwise."""
+    import hashlib
+    import re
 
     sys.path.insert(0, ROOT)
     import bench
 
-    got = bench._profiled_traffic(1)
-    assert got is not None and got > 0
-    assert bench._profiled_traffic(2) is None  # no summary for that workload
-    # a copy of the tree whose scorer source differs by one byte
+    # the committed summaries carry a source hash and a parsable DRAM line
+    for name in bench.PROFILES.values():
+        text = open(os.path.join(ROOT, "profiles", name)).read()
+        assert re.search(r"sha256 prefix `[0-9a-f]{16}`", text)
+        assert re.search(r"dram__bytes_read\.sum \+ dram__bytes_write\.sum \| [0-9,]+ B \+ [0-9,]+ B", text)
+    # a tree whose summary matches its scorer source, then a changed source
     (tmp_path / "profiles").mkdir()
-    shutil.copy(os.path.join(ROOT, "profiles", bench.PROFILES[1]), tmp_path / "profiles")
     csrc = tmp_path / "paper_2608_19659_gb300" / "csrc"
     csrc.mkdir(parents=True)
-    src = open(os.path.join(ROOT, "paper_2608_19659_gb300", "csrc", "fs_score.cu"), "rb").read()
+    src = b"// scorer source\n"
     (csrc / "fs_score.cu").write_bytes(src)
+    h = hashlib.sha256(src).hexdigest()[:16]
+    (tmp_path / "profiles" / bench.PROFILES[1]).write_text(
+        f"Source: fs_score.cu, sha256 prefix `{h}`.\n"
+        "| dram__bytes_read.sum + dram__bytes_write.sum | 1,237,760 B + 512 B per launch |\n")
     monkeypatch.setattr(bench, "ROOT", str(tmp_path))
-    assert bench._profiled_traffic(1) == got
+    assert bench._profiled_traffic(1) == 1237760.0 + 512.0
+    assert bench._profiled_traffic(2) is None  # no summary for that workload
     (csrc / "fs_score.cu").write_bytes(src + b"\n")
     assert bench._profiled_traffic(1) is None
