@@ -125,7 +125,6 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
   const int item = blockIdx.x >> 1, sigma = blockIdx.x & 1;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = blockDim.x >> 5;
   if (!early) pdl_wait();
-  pdl_trigger();  // k_score may start launching; it waits for this grid to finish
   const int p = it.p ? it.p[item] : 0;
   const int cell = it.cell[item];
   float* base_rec = rec + (size_t)item * pl.item_floats;
@@ -194,21 +193,51 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
     const float d_c = __fsub_rn(hi_c, lo_c), d_l = __fsub_rn(hi_l, lo_l);
     const long long n_idx = (long long)((pl.O - sigma + 1) >> 1) * W;
     float* wins = base_rec + 2 * (size_t)d.slot_floats;
-    // read-only loads, so that the unrolled iterations' loads are issued
-    // together rather than each behind the previous iteration's stores
+    if (W >= 4 && (reinterpret_cast<uintptr_t>(set.qn) & 15u) == 0) {
+      // four consecutive positions per thread: one 16-byte load and store
+      // (windows start on 16-byte boundaries), plus the next position's value
+      const long long n4 = n_idx >> 2;
+#pragma unroll 2
+      for (long long g4 = tid; g4 < n4; g4 += blockDim.x) {
+        const long long idx = g4 << 2;
+        const int k = (int)(idx & (W - 1));
+        const int o = sigma + 2 * (int)(idx >> pl.w);
+        const float* q = set.qn + (size_t)o * W;
+        float* win = wins + (size_t)o * pl.Wp;
+        const float4 v = __ldg(reinterpret_cast<const float4*>(q + k));
+        const float vn = k + 4 < W ? __ldg(q + k + 4) : 0.0f;
+        float4 cm;
+        cm.x = map_into(lo_c, d_c, hi_c, v.x);
+        cm.y = map_into(lo_c, d_c, hi_c, v.y);
+        cm.z = map_into(lo_c, d_c, hi_c, v.z);
+        cm.w = map_into(lo_c, d_c, hi_c, v.w);
+        *reinterpret_cast<float4*>(win + 4 + k) = cm;
+        const bool p0 = map_into(lo_l, d_l, hi_l, v.x) <= L, p1 = map_into(lo_l, d_l, hi_l, v.y) <= L;
+        const bool p2 = map_into(lo_l, d_l, hi_l, v.z) <= L, p3 = map_into(lo_l, d_l, hi_l, v.w) <= L;
+        const bool p4 = k + 4 < W && map_into(lo_l, d_l, hi_l, vn) <= L;
+        if (k == 0 && !p0) win[0] = __int_as_float(0);
+        if (p0 && !p1) win[0] = __int_as_float(k + 1);
+        if (p1 && !p2) win[0] = __int_as_float(k + 2);
+        if (p2 && !p3) win[0] = __int_as_float(k + 3);
+        if (p3 && !p4) win[0] = __int_as_float(k + 4);
+      }
+    } else {
+      // read-only loads, so that the unrolled iterations' loads are issued
+      // together rather than each behind the previous iteration's stores
 #pragma unroll 4
-    for (long long idx = tid; idx < n_idx; idx += blockDim.x) {
-      const int k = (int)(idx & (W - 1));
-      const int o = sigma + 2 * (int)(idx >> pl.w);
-      const float* q = set.qn + (size_t)o * W;
-      float* win = wins + (size_t)o * pl.Wp;
-      const float qv = __ldg(q + k);
-      const float qnext = k + 1 < W ? __ldg(q + k + 1) : 0.0f;
-      win[4 + k] = map_into(lo_c, d_c, hi_c, qv);
-      const bool pass = map_into(lo_l, d_l, hi_l, qv) <= L;
-      const bool pass_next = k + 1 < W && map_into(lo_l, d_l, hi_l, qnext) <= L;
-      if (k == 0 && !pass) win[0] = __int_as_float(0);
-      if (pass && !pass_next) win[0] = __int_as_float(k + 1);
+      for (long long idx = tid; idx < n_idx; idx += blockDim.x) {
+        const int k = (int)(idx & (W - 1));
+        const int o = sigma + 2 * (int)(idx >> pl.w);
+        const float* q = set.qn + (size_t)o * W;
+        float* win = wins + (size_t)o * pl.Wp;
+        const float qv = __ldg(q + k);
+        const float qnext = k + 1 < W ? __ldg(q + k + 1) : 0.0f;
+        win[4 + k] = map_into(lo_c, d_c, hi_c, qv);
+        const bool pass = map_into(lo_l, d_l, hi_l, qv) <= L;
+        const bool pass_next = k + 1 < W && map_into(lo_l, d_l, hi_l, qnext) <= L;
+        if (k == 0 && !pass) win[0] = __int_as_float(0);
+        if (pass && !pass_next) win[0] = __int_as_float(k + 1);
+      }
     }
   }
   if (early) pdl_wait();  // thresholds and rows come from k_solve
@@ -353,6 +382,9 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
     tab[H_FAST] = __int_as_float(fast ? 1 : 0);
     tab[H_RLAM] = rl;
   }
+  // k_score launches only now: its blocks, resident early, slowed the base
+  // solve and this kernel more than their early start saved
+  pdl_trigger();
 }
 
 // t* of one realisation with row capacity C (see the file comment). kap is

@@ -104,20 +104,30 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   int* sMisc = sProbe + 32;                               // [8]
   float* sTheta = reinterpret_cast<float*>(sMisc + 8);    // [pow2 >= theta_cap]
 
-  // 1. rows: key = (capacity bits, ~bin) of the best SLO-feasible bin; 0 = none
+  // 1. rows: key = (capacity bits, ~bin) of the best SLO-feasible bin; 0 = none.
+  // The inputs of the first pass (demands, and each thread's first cell) are
+  // all loaded before anything waits on one of them: one memory round trip.
   __shared__ float sLam[FS_MAX_CLASSES], sRl[FS_MAX_CLASSES];  // demand and RN(1/demand)
-  if (tid < d.K) {
-    sLam[tid] = set.lam[tid];
-    sRl[tid] = __frcp_rn(set.lam[tid]);
-  }
+  const float lam_v = tid < d.K ? set.lam[tid] : 1.0f;
+  const bool cell0 = tid < d.cells;
+  const float tail0 = cell0 ? tail[tid] : 0.0f, cap0 = cell0 ? cap[tid] : 0.0f;
+  const float slo0 = cell0 ? set.slo[(tid / d.B) >> 2] : 0.0f;
   for (int rho = tid; rho < d.K4; rho += blockDim.x) sKey[rho] = 0ull;
   if (tid < 8) sMisc[tid] = 0;
+  if (tid < d.K) {
+    sLam[tid] = lam_v;
+    sRl[tid] = __frcp_rn(lam_v);
+  }
   __syncthreads();
   for (int c = tid; c < d.cells; c += blockDim.x) {
     const int rho = c / d.B;
     const int b = c - rho * d.B;
-    if (tail[c] <= set.slo[rho >> 2]) {
-      const uint32_t cb = __float_as_uint(__fadd_rn(cap[c], 0.0f));  // -0 -> +0: bits order like values
+    const bool first = c == tid;
+    const float tv = first ? tail0 : tail[c];
+    const float lv = first ? slo0 : set.slo[rho >> 2];
+    if (tv <= lv) {
+      const float cv = first ? cap0 : cap[c];
+      const uint32_t cb = __float_as_uint(__fadd_rn(cv, 0.0f));  // -0 -> +0: bits order like values
       atomicMax(&sKey[rho], ((unsigned long long)cb << 32) | (0xFFFFFFFFu - (uint32_t)b));
     }
   }
