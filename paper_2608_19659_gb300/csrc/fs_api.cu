@@ -82,6 +82,32 @@ struct Buf {
   }
 };
 
+// Page-locked host memory that grows on demand: copies to and from it are
+// asynchronous, so a call can queue them and wait once.
+struct HostBuf {
+  void* p = nullptr;
+  size_t bytes = 0;
+  int ensure(size_t want, const char* what) {
+    if (want <= bytes) return FS_OK;
+    if (p) cudaFreeHost(p);
+    p = nullptr;
+    bytes = 0;
+    size_t b = std::max<size_t>(want, 256);
+    cudaError_t e = cudaMallocHost(&p, b);
+    if (e != cudaSuccess) {
+      p = nullptr;
+      return cuda_fail(e, what);
+    }
+    bytes = b;
+    return FS_OK;
+  }
+  void release() {
+    if (p) cudaFreeHost(p);
+    p = nullptr;
+    bytes = 0;
+  }
+};
+
 }  // namespace fs
 
 using namespace fs;
@@ -100,6 +126,11 @@ struct fs_model {
   std::vector<float> h_bounds;      // [4][cells]
   std::vector<uint8_t> h_revealed;  // [cells]
   std::vector<float> h_lam, h_slo;
+  // page-locked staging: the last bounds upload (its copy may still be in
+  // flight until up_done), and a synchronous call's outputs and status word
+  HostBuf h_up, h_out;
+  cudaEvent_t up_done = nullptr;
+  bool up_pending = false;
   LaunchCache lc;
   // optional timing events: 5 per timed call (before solve, prep, score,
   // finalize, and after finalize); mode 1 records only the two around score
@@ -136,28 +167,60 @@ int check_bounds4(const float* clo, const float* chi, const float* tlo, const fl
 // +0 for -0, so that nonnegative floats order like their bit patterns.
 inline float canon(float v) { return v == 0.0f ? 0.0f : v; }
 
-int upload_bounds(fs_model* m) {
-  FS_CUDA(cudaMemcpyAsync(m->set.bounds, m->h_bounds.data(), m->h_bounds.size() * 4, cudaMemcpyHostToDevice,
-                          m->stream),
-          "upload bounds");
-  FS_CUDA(cudaMemcpyAsync(m->set.revealed, m->h_revealed.data(), m->h_revealed.size(), cudaMemcpyHostToDevice,
-                          m->stream),
-          "upload revealed");
-  FS_CUDA(cudaStreamSynchronize(m->stream), "upload sync");
+// The staging buffer of the last bounds upload is free once that copy has run.
+int wait_upload(fs_model* m) {
+  if (m->up_pending) {
+    FS_CUDA(cudaEventSynchronize(m->up_done), "wait for the bounds upload");
+    m->up_pending = false;
+  }
   return FS_OK;
 }
 
-int read_status(fs_model* m, cudaStream_t s) {
-  FS_CUDA(cudaStreamSynchronize(s), "synchronize");
-  uint32_t st = 0;
-  FS_CUDA(cudaMemcpy(&st, m->set.status, 4, cudaMemcpyDeviceToHost), "read status");
-  if (st) {
-    uint32_t z = 0;
-    cudaMemcpy(m->set.status, &z, 4, cudaMemcpyHostToDevice);
-    if (st & ST_TIMEOUT) return fail(FS_ETIMEOUT, "a device wait timed out (status 0x%x)", st);
-    return fail(FS_EDEVICE, "device status word 0x%x", st);
-  }
+// Work queued on a stream other than the model's starts after the last bounds upload.
+int order_after_upload(fs_model* m, cudaStream_t s) {
+  if (m->up_pending && s != m->stream) FS_CUDA(cudaStreamWaitEvent(s, m->up_done, 0), "order after the upload");
   return FS_OK;
+}
+
+// Queue the host mirror's bounds and revealed flags for the device (from
+// page-locked staging, without waiting): later work on the model's stream
+// is ordered after the copy, work on other streams waits for up_done.
+int upload_bounds(fs_model* m) {
+  const size_t nb = m->h_bounds.size() * 4, nr = m->h_revealed.size();
+  int rc = wait_upload(m);
+  if (rc) return rc;
+  // bounds and revealed flags lie in one span of the model's buffer (the
+  // flags after the bounds' 256-byte padding): staged alike, one copy
+  const size_t rev_off = (size_t)(reinterpret_cast<char*>(m->set.revealed) - reinterpret_cast<char*>(m->set.bounds));
+  if ((rc = m->h_up.ensure(rev_off + nr, "bounds staging"))) return rc;
+  char* h = static_cast<char*>(m->h_up.p);
+  std::memcpy(h, m->h_bounds.data(), nb);
+  std::memcpy(h + rev_off, m->h_revealed.data(), nr);
+  FS_CUDA(cudaMemcpyAsync(m->set.bounds, h, rev_off + nr, cudaMemcpyHostToDevice, m->stream), "upload bounds");
+  if (!m->up_done) FS_CUDA(cudaEventCreateWithFlags(&m->up_done, cudaEventDisableTiming), "create upload event");
+  FS_CUDA(cudaEventRecord(m->up_done, m->stream), "record upload event");
+  m->up_pending = true;
+  return FS_OK;
+}
+
+// Turn a nonzero device status word into an error (and clear it for the next call).
+int status_error(fs_model* m, uint32_t st) {
+  if (!st) return FS_OK;
+  uint32_t z = 0;
+  cudaMemcpy(m->set.status, &z, 4, cudaMemcpyHostToDevice);
+  if (st & ST_TIMEOUT) return fail(FS_ETIMEOUT, "a device wait timed out (status 0x%x)", st);
+  return fail(FS_EDEVICE, "device status word 0x%x", st);
+}
+
+// Wait for the work queued on s and check the status word: one asynchronous
+// copy into page-locked memory and one synchronisation.
+int read_status(fs_model* m, cudaStream_t s) {
+  int rc = m->h_out.ensure(64, "status staging");
+  if (rc) return rc;
+  uint32_t* hs = static_cast<uint32_t*>(m->h_out.p);
+  FS_CUDA(cudaMemcpyAsync(hs, m->set.status, 4, cudaMemcpyDeviceToHost, s), "read status");
+  FS_CUDA(cudaStreamSynchronize(s), "synchronize");
+  return status_error(m, *hs);
 }
 
 int check_samples(const fs_model* m, const fs_samples* s, bool host_cand) {
@@ -207,7 +270,7 @@ int ensure_items(fs_model* m, int n, int O) {
 
 // The scoring sequence on stream s; cand_dev holds n_cand cell ids.
 int run_score(fs_model* m, const fs_samples* smp, const int32_t* cand_dev, double* gap, double* score,
-              float* gamma_t, int32_t* best, void* dump, cudaStream_t s) {
+              float* gamma_t, int32_t* best, void* dump, cudaStream_t s, uint32_t* status_copy = nullptr) {
   const int n = smp->n_cand;
   Items it{};
   it.n = n;
@@ -236,7 +299,7 @@ int run_score(fs_model* m, const fs_samples* smp, const int32_t* cand_dev, doubl
                        fs_dump_stride(m), m->sm_count, m->lc, s),
           "launch score");
   if (timed) FS_CUDA(cudaEventRecord(ev[3], s), "record timing event");
-  FS_CUDA(launch_finalize(m->set, it, pl, (const uint64_t*)m->sums.p, gap, score, gamma_t, best, s),
+  FS_CUDA(launch_finalize(m->set, it, pl, (const uint64_t*)m->sums.p, gap, score, gamma_t, best, status_copy, s),
           "launch finalize");
   if (phases) FS_CUDA(cudaEventRecord(ev[4], s), "record timing event");
   return FS_OK;
@@ -396,15 +459,28 @@ int fs_score_candidates(fs_model* m, const fs_samples* smp, double* gap_out, dou
   cudaStream_t s = m->stream;
   if (n > 0)
     FS_CUDA(cudaMemcpyAsync(m->cand.p, smp->cand, 4 * (size_t)n, cudaMemcpyHostToDevice, s), "upload candidates");
-  rc = run_score(m, smp, (const int32_t*)m->cand.p, d_gap, d_score, d_gt, d_best, dump_dev, s);
+  // the status word joins the outputs on the device (gap, score, gamma_t,
+  // best, status are contiguous; k_finalize copies it), and one copy brings
+  // them all to staging
+  const size_t nn = (size_t)std::max(n, 1);
+  uint32_t* d_st = reinterpret_cast<uint32_t*>(d_best + 4);
+  rc = run_score(m, smp, (const int32_t*)m->cand.p, d_gap, d_score, d_gt, d_best, dump_dev, s, d_st);
   if (rc) return rc;
-  if (gap_out && n) FS_CUDA(cudaMemcpyAsync(gap_out, d_gap, 8 * (size_t)n, cudaMemcpyDeviceToHost, s), "read gap");
-  if (score_out && n) FS_CUDA(cudaMemcpyAsync(score_out, d_score, 8 * (size_t)n, cudaMemcpyDeviceToHost, s), "read score");
-  if (gamma_t) FS_CUDA(cudaMemcpyAsync(gamma_t, d_gt, 4, cudaMemcpyDeviceToHost, s), "read gamma");
-  if (best) FS_CUDA(cudaMemcpyAsync(best, d_best, 4, cudaMemcpyDeviceToHost, s), "read best");
+  const size_t out_bytes = 16 * nn + 36;
+  if ((rc = m->h_out.ensure(out_bytes, "output staging"))) return rc;
+  FS_CUDA(cudaMemcpyAsync(m->h_out.p, m->outs.p, out_bytes, cudaMemcpyDeviceToHost, s), "read outputs");
   if (sum_eo && n)
     FS_CUDA(cudaMemcpyAsync(sum_eo, m->sums.p, 8 * (size_t)n * smp->O, cudaMemcpyDeviceToHost, s), "read sums");
-  return read_status(m, s);
+  FS_CUDA(cudaStreamSynchronize(s), "synchronize");
+  const char* h = static_cast<const char*>(m->h_out.p);
+  uint32_t st;
+  std::memcpy(&st, h + 16 * nn + 32, 4);
+  if (st) return status_error(m, st);
+  if (gap_out && n) std::memcpy(gap_out, h, 8 * (size_t)n);
+  if (score_out && n) std::memcpy(score_out, h + 8 * nn, 8 * (size_t)n);
+  if (gamma_t) std::memcpy(gamma_t, h + 16 * nn, 4);
+  if (best) std::memcpy(best, h + 16 * nn + 16, 4);
+  return FS_OK;
 }
 
 int fs_score_candidates_async(fs_model* m, const fs_samples* smp, double* gap_dev, double* score_dev,
@@ -416,6 +492,7 @@ int fs_score_candidates_async(fs_model* m, const fs_samples* smp, double* gap_de
   const int n = smp->n_cand;
   if ((rc = ensure_items(m, n, smp->O))) return rc;
   cudaStream_t s = (cudaStream_t)cuda_stream;
+  if ((rc = order_after_upload(m, s))) return rc;
   rc = run_score(m, smp, smp->cand, gap_dev, score_dev, gamma_t_dev, best_dev, dump_dev, s);
   if (rc) return rc;
   if (sum_eo_dev && n)
@@ -448,6 +525,8 @@ int fs_solve_batch(fs_model* m, int32_t n, const float* cap_dev, const float* ta
   if (n < 0) return fail(FS_EINVAL, "n < 0");
   if (n == 0) return FS_OK;
   if (!cap_dev || !tail_dev || !out_dev) return fail(FS_EINVAL, "NULL device pointer");
+  int rc = order_after_upload(m, (cudaStream_t)cuda_stream);
+  if (rc) return rc;
   FS_CUDA(launch_solve(m->set, n, cap_dev, tail_dev, out_dev, false, m->lc, (cudaStream_t)cuda_stream),
           "launch solve");
   return FS_OK;
@@ -708,6 +787,9 @@ void fs_free_model(fs_model* m) {
   m->outs.release();
   m->real.release();
   for (cudaEvent_t e : m->ev) cudaEventDestroy(e);
+  if (m->up_done) cudaEventDestroy(m->up_done);
+  m->h_up.release();
+  m->h_out.release();
   delete m;
 }
 

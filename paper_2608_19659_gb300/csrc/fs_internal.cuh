@@ -365,8 +365,10 @@ cudaError_t launch_prep(const Set& set, const Items& it, const Plan& pl, float* 
 cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const float* tables,
                          uint64_t* sums, void* dump, int dump_stride, int sm_count, LaunchCache& lc,
                          cudaStream_t s);
+// status_copy (nullable): the status word as it stands after the whole call.
 cudaError_t launch_finalize(const Set& set, const Items& it, const Plan& pl, const uint64_t* sums,
-                            double* gap, double* score, float* gamma_t, int32_t* best, cudaStream_t s);
+                            double* gap, double* score, float* gamma_t, int32_t* best, uint32_t* status_copy,
+                            cudaStream_t s);
 cudaError_t launch_watchdog(uint32_t* status, uint64_t limit_ns, cudaStream_t s);
 
 // replay

@@ -255,9 +255,9 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
   // Joint search: each round every group of gsz lanes probes one index and
   // answers for both capacities; each warp merges the answers with integer
   // max / min reductions, so a round costs one barrier.
-  int gsz = 4;
-  while (gsz < d.K4 && gsz < 32) gsz <<= 1;
-  const int ng = blockDim.x / gsz, g = tid / gsz, gl = tid & (gsz - 1);
+  int lgs = 2;
+  while ((1 << lgs) < d.K4 && lgs < 5) ++lgs;
+  const int gsz = 1 << lgs, ng = (int)blockDim.x >> lgs, g = tid >> lgs, gl = tid & (gsz - 1);
   int lo0 = -1, hi0 = total, lo1 = -1, hi1 = total;
   for (int par = 0; hi0 - lo0 > 1 || hi1 - lo1 > 1; par ^= 1) {
     const int k = probe_index(g, ng, lo0, hi0, lo1, hi1);
@@ -316,7 +316,7 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
       // answer is not among them, a 32-ary search over the whole interval.
       const float t = sTh[k];
       const uint32_t bx = __float_as_uint(cx), bmax = __float_as_uint(cmax);
-      const float c0 = __fdiv_rn(__fmul_rn(t, lam), (float)m);
+      const float c0 = __fdividef(__fmul_rn(t, lam), (float)m);  // an estimate: the window is checked exactly
       const long long pl_ = (long long)__float_as_uint(c0) - 16 + lane;
       const uint32_t pt0 = pl_ < 0 ? 0u : (uint32_t)pl_;
       const bool ok0 = pt0 > bx && (pt0 >= bmax || fulfil_r((float)m, __uint_as_float(pt0), lam, rl) >= t);
@@ -751,13 +751,16 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
 }
 
 __global__ void k_finalize(Set set, Items it, Plan pl, const uint64_t* sums, double* gap, double* score,
-                           float* gamma_t, int32_t* best) {
+                           float* gamma_t, int32_t* best, uint32_t* status_copy) {
   pdl_wait();
   const int p = blockIdx.x;
   const int beg = it.off ? it.off[p] : 0;
   const int end = it.off ? it.off[p + 1] : it.n;
   const Best b = finalize_problem(set, it, pl, sums, p, beg, end, gap, score, gamma_t ? gamma_t + p : nullptr);
   if (threadIdx.x == 0 && best) best[p] = b.valid() ? b.cell : -1;
+  // every kernel of the call has finished (stream order, and the wait above):
+  // its status word can travel with the outputs
+  if (threadIdx.x == 0 && p == 0 && status_copy) *status_copy = *set.status;
 }
 
 static size_t prep_smem_bytes(const Dims& d) { return (size_t)(256 + d.theta_cap) * 4; }
@@ -832,9 +835,9 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
 }
 
 cudaError_t launch_finalize(const Set& set, const Items& it, const Plan& pl, const uint64_t* sums, double* gap,
-                            double* score, float* gamma_t, int32_t* best, cudaStream_t s) {
+                            double* score, float* gamma_t, int32_t* best, uint32_t* status_copy, cudaStream_t s) {
   return launch_pdl(k_finalize, dim3(it.off ? set.P : 1), dim3(256), 0, s, set, it, pl, sums, gap, score,
-                    gamma_t, best);
+                    gamma_t, best, status_copy);
 }
 
 }  // namespace fs

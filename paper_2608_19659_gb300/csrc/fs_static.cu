@@ -203,7 +203,7 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
                      reinterpret_cast<uint64_t*>(base + o_sums), nullptr, 0, sm_count, *lc, s);
   if (e == cudaSuccess)
     e = launch_finalize(set, it, pl, reinterpret_cast<const uint64_t*>(base + o_sums), gap_dev, score_dev,
-                        gamma_t_dev, best_dev, s);
+                        gamma_t_dev, best_dev, nullptr, s);
   if (e != cudaSuccess) return cuda_say(e, "launch (allocation-free scoring)");
   uint32_t st = 0;
   e = cudaMemcpyAsync(&st, set.status, 4, cudaMemcpyDeviceToHost, s);

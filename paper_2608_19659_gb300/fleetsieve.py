@@ -80,7 +80,7 @@ def lib():
         fp = C.POINTER(C.c_float)
         L.fs_load_model.argtypes = [C.POINTER(fs_bounds), fp, fp, C.c_int32, C.c_void_p,
                                     C.POINTER(C.c_void_p)]
-        L.fs_update_bounds.argtypes = [C.c_void_p, fp, fp, fp, fp]
+        L.fs_update_bounds.argtypes = [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]
         L.fs_dump_stride.argtypes = [C.c_void_p]
         L.fs_dump_stride.restype = C.c_int32
         L.fs_score_candidates.argtypes = [C.c_void_p, C.POINTER(fs_samples), C.c_void_p, C.c_void_p,
@@ -121,6 +121,8 @@ def _check(rc: int) -> int:
 
 
 def _f32(a) -> np.ndarray:
+    if isinstance(a, np.ndarray) and a.dtype == np.float32 and a.flags.c_contiguous:
+        return a
     return np.ascontiguousarray(np.asarray(a, dtype=np.float32).reshape(-1))
 
 
@@ -128,13 +130,13 @@ def _fp(a: np.ndarray):
     return a.ctypes.data_as(C.POINTER(C.c_float))
 
 
-def _vp(a) -> C.c_void_p | None:
-    """Address of a numpy array or torch tensor (None passes NULL)."""
+def _vp(a) -> int | None:
+    """Address of a numpy array or torch tensor for a void* argument (None passes NULL)."""
     if a is None:
         return None
     if isinstance(a, np.ndarray):
-        return C.c_void_p(a.ctypes.data)
-    return C.c_void_p(a.data_ptr())
+        return a.__array_interface__["data"][0]
+    return a.data_ptr()
 
 
 def _stream(s) -> C.c_void_p | None:
@@ -179,7 +181,7 @@ def fs_load_model(cap_lo, cap_hi, tail_lo, tail_hi, slo, demand, G: int, K: int,
 
 def fs_update_bounds(m: Model, cap_lo, cap_hi, tail_lo, tail_hi) -> None:
     arrs = [_f32(x) for x in (cap_lo, cap_hi, tail_lo, tail_hi)]
-    _check(lib().fs_update_bounds(m.handle, *[_fp(x) for x in arrs]))
+    _check(lib().fs_update_bounds(m.handle, *[_vp(x) for x in arrs]))
 
 
 def fs_dump_stride(m: Model) -> int:
@@ -209,7 +211,7 @@ def fs_score_candidates(m: Model, cand, O: int, S: int, seed: int, stream_id: in
         outputs = (np.zeros(n, np.float64), np.zeros(n, np.float64), np.zeros(1, np.float32),
                    np.zeros(1, np.int32), np.zeros((n, O), np.int64))
     gap, score, gt, best, sums = outputs
-    smp = _samples(seed, stream_id, rnd, n, O, S, cand.ctypes.data if n else None)
+    smp = _samples(seed, stream_id, rnd, n, O, S, _vp(cand) if n else None)
     _check(lib().fs_score_candidates(m.handle, C.byref(smp), _vp(gap), _vp(score), _vp(gt),
                                      _vp(best), _vp(sums), _vp(dump_dev)))
     return ScoreResult(gap, score, float(gt[0]), int(best[0]), sums)
