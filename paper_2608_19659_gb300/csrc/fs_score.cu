@@ -806,14 +806,16 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
   }
   // Chunks of U calls per thread: about eight chunks per resident block when
   // the work allows, so that the counter can even out the segments' unequal
-  // costs; at most 8 calls per thread, and no more than a segment holds.
+  // costs; at least 2 (a chunk's set-up is then paid for eight samples per
+  // thread, measured faster on small launches) and at most 8 calls per
+  // thread, and no more than a segment holds.
   const long long resident = (long long)lc.score_blocks_per_sm[v] * sm_count;
   const long long total_calls = (long long)it.n * pl.O * pl.calls;
   long long U = total_calls / ((long long)kScoreThreads * resident * 8);
   const long long u_seg = ((long long)pl.calls + kScoreThreads - 1) / kScoreThreads;
   if (U > 8) U = 8;
+  if (U < 2) U = 2;
   if (U > u_seg) U = u_seg;
-  if (U < 1) U = 1;
   // chunk indices are 32-bit: widen the chunks until they fit (one chunk per
   // segment gives n O <= 2^30 chunks, which the entry points guarantee)
   long long nch = (pl.calls + kScoreThreads * U - 1) / (kScoreThreads * U);
