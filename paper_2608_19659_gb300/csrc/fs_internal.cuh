@@ -30,7 +30,7 @@ namespace fs {
 constexpr int kT = 4;                 // TP degrees {1, 2, 4, 8}
 constexpr int kCostInf = 0x3FFFFFFF;  // "no option covers the threshold"
 constexpr int kSolveThreads = 256;
-constexpr int kPrepThreads = 128;
+constexpr int kPrepThreads = 256;
 constexpr int kScoreThreads = 256;
 constexpr int kTableHeader = 20;      // floats before the three table arrays (16-byte multiple)
 constexpr int kSmemTableCap = 256;    // table entries staged in shared memory per realisation (pow2)
