@@ -1,0 +1,90 @@
+"""Monte-Carlo scorer (fs_score_candidates) against the CPU oracle across many
+random small problems and at the extreme sizes the model accepts.
+
+Every case compares the fixed-point sums, E[Gamma_{t+1} | e], the scores,
+Gamma_t and the argmax bit for bit. The random cases vary K, B, G, demands,
+outcomes O, samples S (ragged last Philox call), seed, stream id, round and,
+for a quarter of them, the quantile table.
+"""
+
+import dataclasses
+
+import numpy as np
+import pytest
+
+from conftest import load_model
+from paper_2608_19659_gb300 import workloads
+
+pytestmark = pytest.mark.gpu
+
+
+def _score_both(fsb, oracle_lib, w, qn, cand, O, S, seed, stream_id, rnd, quantile=None):
+    with load_model(fsb, w, quantile) as m:
+        r = fsb.fs_score_candidates(m, cand, O, S, seed, stream_id, rnd)
+    ref = oracle_lib.score(w, qn, candidates=cand, seed=seed, stream_id=stream_id, rnd=rnd, O=O, S=S)
+    return r, ref
+
+
+def _assert_same(r, ref):
+    assert np.array_equal(r.sum_eo, ref.sum_eo)
+    assert np.array_equal(r.gap, ref.gap)
+    assert np.array_equal(r.score, ref.score)
+    assert r.gamma_t == ref.gamma_t
+    assert r.best == ref.best
+
+
+def _contested(oracle_lib, w):
+    """w with its demand scaled by the power of sqrt(2) that gives the widest
+    base gap Gamma_t (the oracle's), so that scores are not all zero."""
+    best_g, best_w = -1.0, w
+    for k in range(-8, 37):
+        x = dataclasses.replace(w, demand=(w.demand * np.float32(2.0 ** (k / 2))).astype(np.float32))
+        g = oracle_lib.base_gap(oracle_lib.Problem.of(x), x.cap_lo, x.cap_hi, x.tail_lo, x.tail_hi)[2]
+        if g > best_g:
+            best_g, best_w = g, x
+    return best_w
+
+
+def _random_quantiles(rng, Q):
+    """A nondecreasing table in [0, 1] with repeated values and both ends."""
+    v = np.sort(rng.random(Q).astype(np.float32))
+    v[: Q // 16] = v[0]
+    v[0], v[-1] = np.float32(0.0), np.float32(1.0)
+    return np.sort(v)
+
+
+@pytest.mark.parametrize("seed", range(16))
+def test_random_small_problems(fsb, cuda, oracle_lib, seed):
+    rng = np.random.default_rng(900 + seed)
+    K, B, G = int(rng.integers(1, 9)), int(rng.integers(1, 9)), int(rng.integers(1, 65))
+    w = workloads.random_small(rng, K, B, G)
+    if seed % 3:  # one case in three keeps its raw demand (often Gamma_t = 0 or 1)
+        w = _contested(oracle_lib, w)
+    O, S = int(2 ** rng.integers(0, 4)), int(rng.integers(1, 41))
+    s, sid, rnd = int(rng.integers(0, 2**63)), int(rng.integers(0, 1000)), int(rng.integers(0, 50))
+    if seed % 4 == 0:
+        qn = _random_quantiles(rng, int(2 ** rng.integers(4, 11)))
+        O = min(O, qn.size)
+        r, ref = _score_both(fsb, oracle_lib, w, qn, w.candidates, O, S, s, sid, rnd, quantile=qn)
+    else:
+        qn = oracle_lib.triangular_table(4096)
+        r, ref = _score_both(fsb, oracle_lib, w, qn, w.candidates, O, S, s, sid, rnd)
+    _assert_same(r, ref)
+
+
+@pytest.mark.parametrize("K,B,G,n_cand", [
+    (64, 2, 128, 24),   # 64 classes, 15360 thresholds
+    (1, 4096, 8, 24),   # 16384 cells
+    (1, 1, 1, 4),       # one GPU, one bin
+    (1, 6, 1, 24),      # one GPU, six bins
+    (3, 5, 1, 60),      # one GPU for three classes: t* = 0 on both sides
+    (1, 2, 8738, 8),    # 16383 thresholds, within one of the most a model holds
+])
+def test_extreme_sizes(fsb, cuda, oracle_lib, K, B, G, n_cand):
+    rng = np.random.default_rng(K * 7919 + B * 31 + G)
+    w = _contested(oracle_lib, workloads.random_small(rng, K, B, G))
+    cells = K * 4 * B
+    cand = np.sort(rng.choice(cells, size=min(n_cand, cells), replace=False)).astype(np.int32)
+    qn = oracle_lib.triangular_table(4096)
+    r, ref = _score_both(fsb, oracle_lib, w, qn, cand, 2, 16, 77, 3, 1)
+    _assert_same(r, ref)
