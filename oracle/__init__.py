@@ -20,12 +20,13 @@ SOLVER_FRONTIER = 1
 
 class _Problem(C.Structure):
     _fields_ = [("K", C.c_int), ("B", C.c_int), ("G", C.c_int),
-                ("demand", C.POINTER(C.c_float)), ("slo", C.POINTER(C.c_float))]
+                ("demand", C.POINTER(C.c_float)), ("slo", C.POINTER(C.c_float)),
+                ("floor", C.POINTER(C.c_float))]
 
 
 class _Alloc(C.Structure):
     _fields_ = [("t_star", C.c_float), ("total_gpus", C.c_int32), ("ok", C.c_int32),
-                ("pad", C.c_int32), ("has_option_mask", C.c_uint64),
+                ("floors_met", C.c_int32), ("has_option_mask", C.c_uint64),
                 ("tp", C.c_int32 * OR_KMAX), ("bin", C.c_int32 * OR_KMAX),
                 ("replicas", C.c_int32 * OR_KMAX), ("fulfil", C.c_float * OR_KMAX)]
 
@@ -40,13 +41,14 @@ class Allocation:
     bin: list
     replicas: list
     fulfil: list
+    floors_met: int = 1
 
     @staticmethod
     def of(a: _Alloc, K: int) -> "Allocation":
         return Allocation(float(a.t_star), int(a.total_gpus), int(a.ok), int(a.has_option_mask),
                           [int(a.tp[i]) for i in range(K)], [int(a.bin[i]) for i in range(K)],
                           [int(a.replicas[i]) for i in range(K)],
-                          [float(np.float32(a.fulfil[i])) for i in range(K)])
+                          [float(np.float32(a.fulfil[i])) for i in range(K)], int(a.floors_met))
 
 
 _lib = None
@@ -101,19 +103,23 @@ def _ptr(a: np.ndarray, ctype):
 
 
 class Problem:
-    """K classes, B bins, budget G, demands and SLOs (Section 3)."""
+    """K classes, B bins, budget G, demands, SLOs and optional critical floors
+    delta_i in [0, 1] (0 = not critical) (Section 3)."""
 
-    def __init__(self, K, B, G, demand, slo):
+    def __init__(self, K, B, G, demand, slo, floor=None):
         self.K, self.B, self.G = int(K), int(B), int(G)
         self.demand = _f32(demand)
         self.slo = _f32(slo)
+        self.floor = None if floor is None else _f32(floor)
         assert self.demand.size == self.K and self.slo.size == self.K
+        assert self.floor is None or self.floor.size == self.K
         self._s = _Problem(self.K, self.B, self.G, _ptr(self.demand, C.c_float),
-                           _ptr(self.slo, C.c_float))
+                           _ptr(self.slo, C.c_float),
+                           None if self.floor is None else _ptr(self.floor, C.c_float))
 
     @staticmethod
     def of(w) -> "Problem":
-        return Problem(w.K, w.B, w.G, w.demand, w.slo)
+        return Problem(w.K, w.B, w.G, w.demand, w.slo, getattr(w, "floor", None))
 
     @property
     def cells(self) -> int:

@@ -19,6 +19,18 @@
  * If no positive threshold fits (including when some class has no
  * SLO-feasible option at all), t* = 0 and every class gets nothing.
  * The success-rate gate of Eq. 5 is taken as satisfied (no success data).
+ *
+ * Tier 1 (critical floors): a critical class i (delta_i > 0) must reach
+ * r_i >= delta_i whenever that is possible. Its options below the floor are
+ * therefore not options at all; tier 2 is solved on what remains (the
+ * threshold rule then gives every class the cheapest cover of
+ * max(t, delta_i)). The floors are met when every critical class has an
+ * option at or above its floor and their cheapest such options fit in G
+ * together (the other classes may stay empty). When no positive threshold
+ * fits but the floors are met, each critical class still gets its cheapest
+ * option at or above its floor (same tie rules) and the others nothing; when
+ * the floors cannot be met, t* = 0 (no class can be served at a positive
+ * threshold while they hold) and every class gets nothing.
  */
 #include <stdlib.h>
 #include <string.h>
@@ -37,9 +49,17 @@ float or_fulfil(int n, float c, float lam)
 static int check_problem(const or_problem *p)
 {
     if (!p || p->K < 1 || p->K > OR_KMAX || p->B < 1 || p->G < 1) return -1;
-    for (int i = 0; i < p->K; ++i)
+    for (int i = 0; i < p->K; ++i) {
         if (!(p->demand[i] > 0.0f)) return -1;
+        if (p->floor && !(p->floor[i] >= 0.0f && p->floor[i] <= 1.0f)) return -1;
+    }
     return 0;
+}
+
+/* delta_i, the fulfilment floor of class i (0: not critical). */
+static float floor_of(const or_problem *p, int i)
+{
+    return p->floor ? p->floor[i] : 0.0f;
 }
 
 static void empty_alloc(const or_problem *p, uint64_t mask, or_alloc *out)
@@ -111,6 +131,7 @@ int or_solve_literal(const or_problem *p, const float *cap, const float *tail, o
                     o.cost = n * tau;
                     o.cap = cap[cell];
                     o.f = or_fulfil(n, cap[cell], p->demand[i]);
+                    if (o.f < floor_of(p, i)) continue;      /* tier 1: below the floor */
                     opt[n_opt++] = o;
                     if (o.f > 0.0f) theta[n_theta++] = o.f;
                 }
@@ -145,6 +166,7 @@ int or_solve_literal(const or_problem *p, const float *cap, const float *tail, o
             out->t_star = t;
             out->total_gpus = (int32_t)total;
             out->ok = 1;
+            out->floors_met = 1;
             for (int i = 0; i < K; ++i) {
                 out->tp[i] = OR_TP[chosen[i].j];
                 out->bin[i] = chosen[i].b;
@@ -153,7 +175,38 @@ int or_solve_literal(const or_problem *p, const float *cap, const float *tail, o
             }
         }
     }
-    if (!found) empty_alloc(p, mask, out);
+    if (!found) {
+        /* tier 1 alone: each critical class's preferred option (all of its
+         * remaining options are at or above its floor) */
+        long total = 0;
+        int met = 1;
+        for (int i = 0; i < K; ++i) {
+            chosen[i].n = 0;
+            if (floor_of(p, i) <= 0.0f) continue;
+            int best = -1;
+            for (int k = first[i]; k < first[i + 1]; ++k)
+                if (best < 0 || prefer(&opt[k], &opt[best])) best = k;
+            if (best < 0) {
+                met = 0;
+            } else {
+                chosen[i] = opt[best];
+                total += opt[best].cost;
+            }
+        }
+        if (total > G) met = 0;
+        empty_alloc(p, mask, out);
+        out->floors_met = met;
+        if (met) {
+            out->total_gpus = (int32_t)total;
+            for (int i = 0; i < K; ++i) {
+                if (floor_of(p, i) <= 0.0f) continue;
+                out->tp[i] = OR_TP[chosen[i].j];
+                out->bin[i] = chosen[i].b;
+                out->replicas[i] = chosen[i].n;
+                out->fulfil[i] = chosen[i].f;
+            }
+        }
+    }
     free(opt); free(theta); free(first);
     return 0;
 }
@@ -168,6 +221,29 @@ static int min_replicas(float t, float c, float lam, int M)
         if (or_fulfil(mid, c, lam) >= t) hi = mid; else lo = mid + 1;
     }
     return lo;
+}
+
+/* Cheapest cover of threshold t by class i over its rows (best bin of each
+ * TP degree): its GPU cost, or -1 if no row covers t; equal costs keep the
+ * lower TP. */
+static int cheapest_cover(const or_problem *p, const float *Ci, const int *bi, int i, float t,
+                          int *j_out, int *n_out)
+{
+    int best_cost = -1;
+    *j_out = -1;
+    *n_out = 0;
+    for (int j = 0; j < OR_T; ++j) {
+        if (bi[j] < 0) continue;
+        int n = min_replicas(t, Ci[j], p->demand[i], p->G / OR_TP[j]);
+        if (n == 0) continue;
+        int cost = n * OR_TP[j];
+        if (best_cost < 0 || cost < best_cost) {
+            best_cost = cost;
+            *j_out = j;
+            *n_out = n;
+        }
+    }
+    return best_cost;
 }
 
 /*
@@ -213,33 +289,23 @@ int or_solve_frontier(const or_problem *p, const float *cap, const float *tail, 
             int M = G / OR_TP[j];
             for (int n = 1; n <= M; ++n) {
                 float f = or_fulfil(n, C[i][j], p->demand[i]);
-                if (f > 0.0f) theta[n_theta++] = f;
+                if (f > 0.0f && f >= floor_of(p, i)) theta[n_theta++] = f;
             }
         }
     qsort(theta, n_theta, sizeof(float), cmp_desc);
 
     int found = 0;
+    int cj[OR_KMAX], cn[OR_KMAX];
     for (size_t q = 0; q < n_theta && !found; ++q) {
         if (q > 0 && theta[q] == theta[q - 1]) continue;
         float t = theta[q];
         long total = 0;
         int all = 1;
-        int cj[OR_KMAX], cn[OR_KMAX];
         for (int i = 0; i < K && all; ++i) {
-            int best_cost = -1;
-            cj[i] = -1; cn[i] = 0;
-            for (int j = 0; j < OR_T; ++j) {
-                if (bstar[i][j] < 0) continue;
-                int n = min_replicas(t, C[i][j], p->demand[i], G / OR_TP[j]);
-                if (n == 0) continue;
-                int cost = n * OR_TP[j];
-                if (best_cost < 0 || cost < best_cost) {   /* equal cost: lower TP kept */
-                    best_cost = cost;
-                    cj[i] = j;
-                    cn[i] = n;
-                }
-            }
-            if (best_cost < 0) all = 0; else total += best_cost;
+            /* class i must cover max(t, delta_i) */
+            float ti = t > floor_of(p, i) ? t : floor_of(p, i);
+            int cost = cheapest_cover(p, C[i], bstar[i], i, ti, &cj[i], &cn[i]);
+            if (cost < 0) all = 0; else total += cost;
         }
         if (all && total <= G) {
             found = 1;
@@ -247,6 +313,7 @@ int or_solve_frontier(const or_problem *p, const float *cap, const float *tail, 
             out->t_star = t;
             out->total_gpus = (int32_t)total;
             out->ok = 1;
+            out->floors_met = 1;
             for (int i = 0; i < K; ++i) {
                 int j = cj[i];
                 out->tp[i] = OR_TP[j];
@@ -256,7 +323,31 @@ int or_solve_frontier(const or_problem *p, const float *cap, const float *tail, 
             }
         }
     }
-    if (!found) empty_alloc(p, mask, out);
+    if (!found) {
+        /* tier 1 alone: each critical class's cheapest cover of its floor */
+        long total = 0;
+        int met = 1;
+        for (int i = 0; i < K; ++i) {
+            cn[i] = 0;
+            if (floor_of(p, i) <= 0.0f) continue;
+            int cost = cheapest_cover(p, C[i], bstar[i], i, floor_of(p, i), &cj[i], &cn[i]);
+            if (cost < 0) met = 0; else total += cost;
+        }
+        if (total > G) met = 0;
+        empty_alloc(p, mask, out);
+        out->floors_met = met;
+        if (met) {
+            out->total_gpus = (int32_t)total;
+            for (int i = 0; i < K; ++i) {
+                if (cn[i] <= 0) continue;
+                int j = cj[i];
+                out->tp[i] = OR_TP[j];
+                out->bin[i] = bstar[i][j];
+                out->replicas[i] = cn[i];
+                out->fulfil[i] = or_fulfil(cn[i], C[i][j], p->demand[i]);
+            }
+        }
+    }
     free(theta);
     return 0;
 }

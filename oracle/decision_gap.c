@@ -148,9 +148,11 @@ int or_score(const or_problem *p, const float *cap_lo, const float *cap_hi,
 }
 
 /*
- * Section 4.2 without critical classes: certified feasible when the gap is
- * at most eps and every cell that A- commits replicas to has been measured
- * (its tail upper bound is known; A- already keeps it within the SLO).
+ * Section 4.2: certified infeasible when even A+ cannot meet the critical
+ * floors; certified feasible when A- meets them, the gap is at most eps and
+ * every cell that A- commits replicas to has been measured (its tail upper
+ * bound is known; A- already keeps it within the SLO); otherwise undecided.
+ * Without critical classes both realisations meet the (empty) floors.
  */
 int or_certificate(const or_problem *p, const float *cap_lo, const float *cap_hi,
                    const float *tail_lo, const float *tail_hi, const uint8_t *revealed,
@@ -169,13 +171,15 @@ int or_certificate(const or_problem *p, const float *cap_lo, const float *cap_hi
         if (!revealed[cell]) committed_known = 0;
     }
     *gamma_t = gt;
-    *state = (gt <= eps && committed_known) ? 1 : 0;
+    if (!ap.floors_met) *state = 2;
+    else *state = (am.floors_met && gt <= eps && committed_known) ? 1 : 0;
     return 0;
 }
 
 /*
  * Algorithm 1 on one reveal order: common initial design (the first r0
- * cells of perm), then per round: A-, A+, certificate; stop when it fires,
+ * cells of perm), then per round: A-, A+, certificate; stop when it fires
+ * (certified feasible or certified infeasible),
  * else reveal the candidate with the largest score (ties: lower TP, then
  * earlier in perm). Revealing sets lo = hi = the hidden true value. Each
  * revealed cell costs 300 s x TP GPU-seconds (Section 5). Trajectories are
@@ -218,7 +222,7 @@ int or_replay_stream(const or_problem *p, const float *prior_cap_lo, const float
         rc = or_certificate(p, clo, chi, tlo, thi, rev, eps, solver, &z, &gt);
         if (rc) break;
         if (gamma_trace) gamma_trace[r] = gt;
-        if (z == 1) { st = 1; break; }
+        if (z != 0) { st = z; break; }
         int nc = 0;
         for (int q = 0; q < cells; ++q)
             if (!rev[perm[q]]) cand[nc++] = perm[q];

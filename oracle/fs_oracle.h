@@ -15,6 +15,7 @@
  *   Section 3, Eqs. 1-5 and the lexicographic objective: the allocation
  *     model (one homogeneous configuration per class, integer replicas,
  *     served load x_i <= n c, GPU budget G, tail gate l <= L_i, r_i = x/lambda);
+ *     tier 1, the fulfilment floors delta_i of the critical classes;
  *   Section 4.1: conservative A- (lower capacity, upper tail) and optimistic
  *     A+ (upper capacity, lower tail) realisations;
  *   Section 4.2: the allocation gap and the certificate;
@@ -43,6 +44,8 @@ typedef struct {
     int G;              /* GPU budget, Eq. 3 */
     const float *demand;/* lambda_i [K], req/s */
     const float *slo;   /* L_i [K], seconds */
+    const float *floor; /* delta_i [K] in [0, 1], tier 1 of Section 3; 0 = class i is
+                           not critical; NULL = no critical class */
 } or_problem;
 
 /* One allocation. A class with replicas[i] == 0 has tp = 0, bin = -1. */
@@ -50,7 +53,7 @@ typedef struct {
     float t_star;               /* max-min fulfilment reached, 0 if none */
     int32_t total_gpus;         /* sum of n * tau */
     int32_t ok;                 /* t_star > 0 */
-    int32_t pad;
+    int32_t floors_met;         /* every critical class can reach its floor within G */
     uint64_t has_option_mask;   /* bit i: class i has an SLO-feasible cell */
     int32_t tp[OR_KMAX];
     int32_t bin[OR_KMAX];
@@ -99,7 +102,8 @@ int or_score(const or_problem *p, const float *cap_lo, const float *cap_hi,
              int64_t *sum_eo, double *gap, double *score, int64_t *score_fixed,
              float *gamma_t, int32_t *best, float *dump_t /* [n_cand*O*S*2] or NULL */);
 
-/* Certificate (Section 4.2): 0 undecided, 1 certified feasible. */
+/* Certificate (Section 4.2): 0 undecided, 1 certified feasible, 2 certified
+ * infeasible (even A+ misses a critical floor). */
 int or_certificate(const or_problem *p, const float *cap_lo, const float *cap_hi,
                    const float *tail_lo, const float *tail_hi, const uint8_t *revealed,
                    float eps, int solver, int *state, float *gamma_t);

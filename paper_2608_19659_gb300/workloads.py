@@ -53,6 +53,7 @@ class Workload:
     seed: int
     stream_id: int = 0
     round: int = 0
+    floor: np.ndarray | None = None  # [K] float32 critical floors delta_i in [0, 1] (0 = not critical)
 
     @property
     def cells(self) -> int:

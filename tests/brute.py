@@ -39,13 +39,21 @@ def options(K, B, G, cap, tail, demand, slo):
     return out
 
 
-def best_max_min(K, B, G, cap, tail, demand, slo):
-    """Largest min_i r_i over every feasible allocation (0 if a class must be empty)."""
+def _floor_ok(combo, floor):
+    """Tier 1: every critical class (floor > 0) is served at r_i >= floor_i."""
+    if floor is None:
+        return True
+    return all(d <= 0 or (c is not None and c[5] >= np.float32(d)) for c, d in zip(combo, floor))
+
+
+def best_max_min(K, B, G, cap, tail, demand, slo, floor=None):
+    """Largest min_i r_i over every allocation within G that meets the critical
+    floors (0 if a class must be empty, or if no allocation meets the floors)."""
     opts = options(K, B, G, cap, tail, demand, slo)
     best = 0.0
     for combo in itertools.product(*[[None] + o for o in opts]):
         cost = sum(c[0] for c in combo if c is not None)
-        if cost > G:
+        if cost > G or not _floor_ok(combo, floor):
             continue
         if any(c is None for c in combo):
             val = 0.0
@@ -55,12 +63,23 @@ def best_max_min(K, B, G, cap, tail, demand, slo):
     return best
 
 
-def choice_at(K, B, G, cap, tail, demand, slo, t):
-    """Per class, the preferred option covering t: (cost, TP, n, -capacity, bin) minimal."""
+def floors_met(K, B, G, cap, tail, demand, slo, floor):
+    """Whether some allocation within G serves every critical class at its floor."""
+    opts = options(K, B, G, cap, tail, demand, slo)
+    for combo in itertools.product(*[[None] + o for o in opts]):
+        if sum(c[0] for c in combo if c is not None) <= G and _floor_ok(combo, floor):
+            return True
+    return False
+
+
+def choice_at(K, B, G, cap, tail, demand, slo, t, floor=None):
+    """Per class, the preferred option covering max(t, floor_i): (cost, TP, n,
+    -capacity, bin) minimal."""
     opts = options(K, B, G, cap, tail, demand, slo)
     res = []
-    for o in opts:
-        cov = [x for x in o if x[5] >= t]
+    for i, o in enumerate(opts):
+        ti = t if floor is None else max(np.float32(t), np.float32(floor[i]))
+        cov = [x for x in o if x[5] >= ti]
         if not cov:
             res.append(None)
             continue
