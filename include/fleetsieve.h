@@ -11,6 +11,7 @@
  *   fs_score_candidates   samples                   -> E[Gamma_{t+1} | e], score, argmax
  *   fs_solve(_batch)      realisation               -> allocation
  *   fs_solve_bounds       conservative / optimistic allocations and Gamma_t
+ *   fs_set_floors         critical classes' fulfilment floors (tier 1)
  *   fs_reveal, fs_certificate, fs_replay            the profiling loop
  *
  * Notation (paper, Section 3): class i has demand lambda_i (req/s) and an SLO
@@ -100,6 +101,20 @@ int fs_load_model(const fs_bounds *bounds, const float *slo, const float *demand
  */
 int fs_update_bounds(fs_model *m, const float *cap_lo, const float *cap_hi,
                      const float *tail_lo, const float *tail_hi);
+
+/*
+ * fs_set_floors -- fulfilment floors of the critical classes (Section 3,
+ * tier 1 of the lexicographic objective: enforce r_i >= delta_i for critical
+ * classes whenever feasible). floor: host [K] floats delta_i in [0, 1];
+ * delta_i = 0 marks class i as not critical; NULL clears every floor (the
+ * state a new model starts in). Under floors, every solve of this model
+ * (fs_solve*, the scoring calls' realisations and scenarios, the
+ * certificate, fs_replay) takes a critical class's options below its floor
+ * as no options at all and maximises tier 2 over what remains; see
+ * fs_allocation for the floor-only allocation. The values are copied before
+ * the call returns and are in place for every later call on any stream.
+ */
+int fs_set_floors(fs_model *m, const float *floor);
 
 /*
  * Monte-Carlo plan of one scoring call (Section 4.3).
@@ -206,14 +221,18 @@ int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, const float *bo
 /*
  * One allocation (Section 3): per class the chosen TP degree (0 = none),
  * bin (-1 = none), replica count and fulfilment r_i; t_star = min_i r_i
- * reached (the tier-2 objective), ok = t_star > 0.
+ * reached (the tier-2 objective), ok = t_star > 0. floors_met = 1 when every
+ * critical class can be served at its floor within G (always 1 without
+ * floors). With ok = 0 and floors_met = 1 the critical classes still get
+ * their cheapest options at or above their floors (same tie rules) and the
+ * other classes nothing; with floors_met = 0 no class gets replicas.
  */
 typedef struct {
     float t_star;
     int32_t total_gpus;
     uint64_t has_option_mask; /* bit i: class i has an SLO-feasible cell */
     int32_t ok;
-    int32_t reserved;
+    int32_t floors_met;
     int8_t tp[FS_MAX_CLASSES];
     int16_t bin[FS_MAX_CLASSES];
     int16_t replicas[FS_MAX_CLASSES];
@@ -222,11 +241,12 @@ typedef struct {
 
 /*
  * fs_solve -- allocation of one realisation (host arrays cap, tail
- * [K][4][B]) under the model's SLOs, demands and G. Tier 2 of the objective
- * (Section 3): t* is the largest option fulfilment t for which every class's
- * cheapest SLO-feasible option with fulfilment >= t fits in G together;
- * ties: lower TP, then fewer replicas, then larger capacity, then lower bin;
- * nothing fits -> t* = 0 and no class gets replicas.
+ * [K][4][B]) under the model's SLOs, demands, floors and G. Tier 2 of the
+ * objective (Section 3): t* is the largest option fulfilment t for which
+ * every class's cheapest SLO-feasible option with fulfilment >= max(t,
+ * delta_i) fits in G together; ties: lower TP, then fewer replicas, then
+ * larger capacity, then lower bin; nothing fits -> t* = 0 and only the
+ * floor-only allocation described at fs_allocation.
  */
 int fs_solve(fs_model *m, const float *cap, const float *tail, fs_allocation *out);
 
@@ -242,10 +262,11 @@ int fs_solve_bounds(fs_model *m, fs_allocation *minus, fs_allocation *plus, floa
 int fs_reveal(fs_model *m, int32_t cell, float cap, float tail);
 
 /*
- * Decision certificate (Section 4.2) without critical classes:
- * *state = 1 (certified feasible) when Gamma_t <= eps and every cell to which
- * A- commits replicas is revealed; else 0 (undecided). 2 (certified
- * infeasible) is reserved for critical floors. gamma_t nullable.
+ * Decision certificate (Section 4.2): *state = 2 (certified infeasible) when
+ * even A+ misses a critical floor; 1 (certified feasible) when A- meets the
+ * floors, Gamma_t <= eps and every cell to which A- commits replicas is
+ * revealed; else 0 (undecided). Without floors state 2 cannot occur.
+ * gamma_t nullable.
  */
 int fs_certificate(fs_model *m, float eps, int32_t *state, float *gamma_t);
 
@@ -254,11 +275,12 @@ int fs_certificate(fs_model *m, float eps, int32_t *state, float *gamma_t);
  * model's bounds, batched on the device. Stream k: hidden truth
  * truth_cap/truth_tail[k][cells], order perm[k][cells] (its first r0 cells
  * are the common initial design; perm position breaks exact score ties).
- * Each round: A-, A+, certificate (eps); if undecided, score the unrevealed
+ * Each round: A-, A+, certificate (eps, the model's floors); if undecided, score the unrevealed
  * cells (perm order) with O x S samples, Philox stream id k and round r,
  * then reveal the argmax. Stops on the certificate, when no cell is left, or
  * after max_rounds. All inputs are host pointers; outputs host, nullable:
- *   rounds[k], state[k], gpu_seconds[k] (300 s x TP per revealed cell),
+ *   rounds[k], state[k] (the certificate's 1 or 2, or 0 when the stream ran out
+ *   of cells or rounds undecided), gpu_seconds[k] (300 s x TP per revealed cell),
  *   reveal_order[k][cells] (-1 padded), gamma_trace[k][max_rounds+1],
  *   final_minus[k] (A- at the end).
  */

@@ -118,14 +118,14 @@ struct fs_model {
   int sm_count = 0;
   cudaStream_t stream = nullptr;
   // device state of the single problem (P = 1)
-  Buf fixed;      // lam, slo, qn, bounds, revealed, theta, ntheta, rowC, rowB, base, status
+  Buf fixed;      // lam, slo + floors, qn, bounds, revealed, theta, ntheta, rowC, rowB, base, status
   Set set{};
   // per-call scratch
   Buf cand, tables, sums, outs, real;
   // host mirrors
   std::vector<float> h_bounds;      // [4][cells]
   std::vector<uint8_t> h_revealed;  // [cells]
-  std::vector<float> h_lam, h_slo;
+  std::vector<float> h_lam, h_slo, h_dlt;
   // page-locked staging: the last bounds upload (its copy may still be in
   // flight until up_done), and a synchronous call's outputs and status word
   HostBuf h_up, h_out;
@@ -379,7 +379,7 @@ int fs_load_model(const fs_bounds* b, const float* slo, const float* demand, int
     off = align_up(off + bytes, 256);
     return o;
   };
-  const size_t o_lam = take(4 * K), o_slo = take(4 * K), o_qn = take(4 * (size_t)Q);
+  const size_t o_lam = take(4 * K), o_slo = take(8 * K), o_qn = take(4 * (size_t)Q);
   const size_t o_bounds = take(16 * (size_t)cells), o_rev = take(cells);
   const size_t o_theta = take(8 * (size_t)d.theta_cap), o_nth = take(8);
   const size_t o_rowc = take(8 * (size_t)d.K4), o_rowb = take(8 * (size_t)d.K4);
@@ -394,7 +394,7 @@ int fs_load_model(const fs_bounds* b, const float* slo, const float* demand, int
   s.d = d;
   s.P = 1;
   s.lam = (const float*)(base + o_lam);
-  s.slo = (const float*)(base + o_slo);
+  s.slo = (const float*)(base + o_slo);  // then the floors, zeroed below: no critical class
   s.qn = (const float*)(base + o_qn);
   s.bounds = (float*)(base + o_bounds);
   s.revealed = (uint8_t*)(base + o_rev);
@@ -409,6 +409,7 @@ int fs_load_model(const fs_bounds* b, const float* slo, const float* demand, int
 
   m->h_lam.assign(demand, demand + K);
   m->h_slo.assign(slo, slo + K);
+  m->h_dlt.assign(K, 0.0f);
   m->h_bounds.resize(4 * (size_t)cells);
   const float* src[4] = {b->cap_lo, b->cap_hi, b->tail_lo, b->tail_hi};
   for (int r = 0; r < 4; ++r)
@@ -443,6 +444,26 @@ int fs_update_bounds(fs_model* m, const float* cap_lo, const float* cap_hi, cons
   for (int r = 0; r < 4; ++r)
     for (int c = 0; c < cells; ++c) m->h_bounds[(size_t)r * cells + c] = canon(src[r][c]);
   return upload_bounds(m);
+}
+
+int fs_set_floors(fs_model* m, const float* floor) {
+  if (!m) return fail(FS_EINVAL, "model is NULL");
+  const int K = m->d.K;
+  std::vector<float> v(K, 0.0f);
+  if (floor)
+    for (int i = 0; i < K; ++i) {
+      if (!(floor[i] >= 0.0f && floor[i] <= 1.0f)) return fail(FS_EINVAL, "floor[%d] = %g outside [0, 1]", i, (double)floor[i]);
+      v[i] = canon(floor[i]);
+    }
+  m->h_dlt = v;
+  // a small copy, finished before the call returns: every later call on any
+  // stream sees the new floors (they follow the SLOs on the device)
+  FS_CUDA(cudaMemcpyAsync((void*)(m->set.slo + K), m->h_dlt.data(), 4 * (size_t)K, cudaMemcpyHostToDevice,
+                          m->stream),
+          "upload floors");
+  FS_CUDA(cudaStreamSynchronize(m->stream), "upload floors");
+  m->lc.floors = std::any_of(v.begin(), v.end(), [](float x) { return x > 0.0f; }) ? 1 : 0;
+  return FS_OK;
 }
 
 int fs_score_candidates(fs_model* m, const fs_samples* smp, double* gap_out, double* score_out, float* gamma_t,
@@ -575,7 +596,8 @@ int fs_certificate(fs_model* m, float eps, int32_t* state, float* gamma_t) {
     while (j < kT && (1 << j) != am.tp[i]) ++j;
     if (!m->h_revealed[(size_t)(i * 4 + j) * m->d.B + am.bin[i]]) known = false;
   }
-  *state = (gt <= eps && known) ? 1 : 0;
+  if (!ap.floors_met) *state = 2;
+  else *state = (am.floors_met && gt <= eps && known) ? 1 : 0;
   if (gamma_t) *gamma_t = gt;
   return FS_OK;
 }

@@ -53,6 +53,7 @@ enum : int {
   H_ROW = 16,     // 1 if row r can buy a replica at some reachable threshold (int)
   H_FAST = 17,    // 1 if every reachable row-term quotient is in Markstein's range (int)
   H_RLAM = 18,    // RN(1 / lambda)
+  H_DLT = 19,     // floor delta of the candidate's class (0: not critical)
 };
 
 enum : int { CAP_LO = 0, CAP_HI = 1, TAIL_LO = 2, TAIL_HI = 3 };
@@ -78,7 +79,8 @@ struct Set {
   Dims d;
   int P;
   const float* lam;     // [K]
-  const float* slo;     // [K]
+  const float* slo;     // [2K]: SLOs, then the critical floors delta_i (0: not critical);
+                        // kernel instances without floors never read the second half
   const float* qn;      // [Q]
   float* bounds;        // [P][4][cells]
   uint8_t* revealed;    // [P][cells]
@@ -346,10 +348,13 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
   return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
 }
 
-// Per-model cache of launch shapes (filled on first use).
+// Per-model launch state: whether floors are set, and the launch shapes
+// (filled on first use) per kernel instance: [floors] for the solve and the
+// preparation, [dump][floors] for the scorer.
 struct LaunchCache {
-  size_t solve_smem = 0, prep_smem = 0, score_smem[2] = {0, 0};
-  int score_blocks_per_sm[2] = {0, 0};
+  int floors = 0;  // some class has a floor > 0: launch the kernel instances with floors
+  size_t solve_smem[2] = {0, 0}, prep_smem[2] = {0, 0}, score_smem[2][2] = {{0, 0}, {0, 0}};
+  int score_blocks_per_sm[2][2] = {{0, 0}, {0, 0}};
 };
 
 cudaError_t launch_qtable(float* qn, int Q, cudaStream_t s);
@@ -376,7 +381,7 @@ struct ReplayState {
   const float* truth;     // [P][2][cells] cap, tail
   const int* perm;        // [P][cells]
   int* rounds;            // [P]
-  int* state;             // [P]  -1 running, 0 undecided stop, 1 certified
+  int* state;             // [P]  -1 running, 0 undecided stop, 1 certified feasible, 2 certified infeasible
   double* gpu_seconds;    // [P]
   int* reveal_order;      // [P][cells]
   int* n_revealed;        // [P]

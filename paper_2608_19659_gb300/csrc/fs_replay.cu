@@ -55,8 +55,11 @@ __global__ void k_replay_certify(Set set, ReplayState rs, int round) {
     const int c = (i * 4 + j) * d.B + am.bin[i];
     if (!set.revealed[(size_t)p * d.cells + c]) known = false;
   }
+  // Section 4.2: infeasible when even A+ misses a critical floor; feasible
+  // when A- meets the floors, the gap is within eps and A-'s cells are known
   int st = -1;
-  if (gt <= rs.eps && known) st = 1;
+  if (!ap.floors_met) st = 2;
+  else if (am.floors_met && gt <= rs.eps && known) st = 1;
   else if (round >= rs.max_rounds || rs.n_revealed[p] >= d.cells) st = 0;
   if (st >= 0) {
     rs.state[p] = st;

@@ -20,6 +20,9 @@
 //   between theta_b and theta_{b+1} the other classes' costs are constant, so
 //   the best cover by row r alone is its largest fulfilment within budget.
 //   Theta may contain values of row r itself (a superset is harmless).
+//   Critical floors (tier 1): class i covers max(t, delta_i) at threshold t,
+//   the base thresholds already leave out values below a floor, and row r's
+//   own term counts only at or above delta_{i_e}.
 //
 // k_prep builds, per (candidate, realisation), the part of that table a
 // scenario can reach: Theta entries with kappa in (Cexcl, max(Cexcl, cap_hi_e)].
@@ -50,15 +53,17 @@ struct Eval {
 // then add one lane of every class, so every lane of the group ends with the
 // other classes' total (uncovered classes counted above bit 24: a cost is at
 // most G <= 32767, so 64 of them stay below 2^21), and every lane's result is valid.
+template <bool FL>
 __device__ __forceinline__ Eval group_eval_excl(float t, const float* sC, const float* sLam, const float* sRl,
-                                                const Dims& d, int rr, int ie, int gl, int gsz) {
+                                                const float* sDl, const Dims& d, int rr, int ie, int gl, int gsz) {
   int packed = 0;
   int P = kCostInf;
   for (int base = 0; base < d.K4; base += gsz) {
     const int rho = base + gl;
     int cost = kCostInf;
     if (rho < d.K4 && rho != rr) {
-      const int n = min_replicas(t, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[rho & 3]);
+      const float tc = FL ? fmaxf(t, sDl[rho >> 2]) : t;
+      const int n = min_replicas(tc, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[rho & 3]);
       if (n) cost = n << (rho & 3);
     }
     cost = min(cost, __shfl_xor_sync(0xffffffffu, cost, 1));
@@ -81,8 +86,9 @@ __device__ __forceinline__ int replicas_left(const Eval& e, int jr, const Dims& 
   return (e.A >= (1 << jr)) ? min(e.A >> jr, d.M[jr]) : 0;
 }
 
-__device__ __forceinline__ bool feasible_at(const Eval& e, int m, float C, float t, float lam, float rl) {
-  return (e.P < kCostInf && e.P <= e.A) || (m >= 1 && fulfil_r((float)m, C, lam, rl) >= t);
+// te = max(t, delta_{i_e}): the fulfilment row r must reach
+__device__ __forceinline__ bool feasible_at(const Eval& e, int m, float C, float te, float lam, float rl) {
+  return (e.P < kCostInf && e.P <= e.A) || (m >= 1 && fulfil_r((float)m, C, lam, rl) >= te);
 }
 
 // Index probed by group g of ng in one round of the joint search for the
@@ -111,7 +117,9 @@ __device__ __forceinline__ int probe_index(int g, int ng, int lo0, int hi0, int 
 // One CTA per (candidate, realisation sigma). Before the threshold search it
 // maps the quantile strata of the outcomes o = sigma, sigma + 2, ... into the
 // candidate's record: this and Cexcl read only the bounds, so with `early`
-// they overlap the base solve that precedes this kernel.
+// they overlap the base solve that precedes this kernel. FL: some class is
+// critical (the model has floors).
+template <bool FL>
 __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan pl, float* rec,
                                                        uint64_t* sums, int early) {
   extern __shared__ __align__(16) unsigned char smraw[];
@@ -120,6 +128,7 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
   __shared__ float s_cx, s_cmax;
   __shared__ int s_bx, s_row;
   __shared__ float sLam[FS_MAX_CLASSES], sRl[FS_MAX_CLASSES];  // demand and RN(1/demand)
+  __shared__ float sDl[FS_MAX_CLASSES];                          // floor delta_i (0: not critical)
   __shared__ int s_res[2][kPrepThreads / 4];
   const Dims& d = set.d;  // kernel-parameter space: d.M[j] reads need no local copy
   const int item = blockIdx.x >> 1, sigma = blockIdx.x & 1;
@@ -143,9 +152,11 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
   }
   const int rr = cell / d.B, be = cell - rr * d.B, ie = rr >> 2, jr = rr & 3;
   const float lam = set.lam[ie], L = set.slo[ie], rl = __frcp_rn(lam);
+  const float dle = FL ? set.slo[d.K + ie] : 0.0f;
   if (tid < d.K) {
     sLam[tid] = set.lam[tid];
     sRl[tid] = __frcp_rn(set.lam[tid]);
+    if (FL) sDl[tid] = set.slo[d.K + tid];
   }
   const float* bp = set.bounds + (size_t)p * 4 * d.cells;
   const float* capS = bp + (size_t)(sigma ? CAP_HI : CAP_LO) * d.cells;
@@ -262,10 +273,11 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
   for (int par = 0; hi0 - lo0 > 1 || hi1 - lo1 > 1; par ^= 1) {
     const int k = probe_index(g, ng, lo0, hi0, lo1, hi1);
     const float t = sTh[k];
-    const Eval e = group_eval_excl(t, sC, sLam, sRl, d, rr, ie, gl, gsz);
+    const Eval e = group_eval_excl<FL>(t, sC, sLam, sRl, sDl, d, rr, ie, gl, gsz);
     if (gl == 0) {
       const int m = replicas_left(e, jr, d);
-      const int f = (feasible_at(e, m, cx, t, lam, rl) ? 1 : 0) | (feasible_at(e, m, cmax, t, lam, rl) ? 2 : 0);
+      const float te = FL ? fmaxf(t, dle) : t;
+      const int f = (feasible_at(e, m, cx, te, lam, rl) ? 1 : 0) | (feasible_at(e, m, cmax, te, lam, rl) ? 2 : 0);
       s_res[par][g] = k | (f << 24);
     }
     __syncthreads();
@@ -304,17 +316,18 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
     const int k = b0 + 1 + u;
     int m;
     if (k < total) {
-      const Eval e = group_eval_excl(sTh[k], sC, sLam, sRl, d, rr, ie, lane, 32);
+      const Eval e = group_eval_excl<FL>(sTh[k], sC, sLam, sRl, sDl, d, rr, ie, lane, 32);
       m = replicas_left(e, jr, d);
     } else {
       m = msent;
     }
     if (u < Lt) {
-      // smallest capacity in (cx, cmax] at which f(m, C) >= theta_k, on the bit
-      // patterns of nonnegative floats (ordered like the values). First the 32
-      // patterns around the real solution t lambda / m, one per lane; if the
-      // answer is not among them, a 32-ary search over the whole interval.
-      const float t = sTh[k];
+      // smallest capacity in (cx, cmax] at which f(m, C) >= max(theta_k,
+      // delta_{i_e}), on the bit patterns of nonnegative floats (ordered like
+      // the values). First the 32 patterns around the real solution t lambda / m,
+      // one per lane; if the answer is not among them, a 32-ary search over the
+      // whole interval.
+      const float th = sTh[k], t = FL ? fmaxf(th, dle) : th;
       const uint32_t bx = __float_as_uint(cx), bmax = __float_as_uint(cmax);
       const float c0 = __fdividef(__fmul_rn(t, lam), (float)m);  // an estimate: the window is checked exactly
       const long long pl_ = (long long)__float_as_uint(c0) - 16 + lane;
@@ -339,7 +352,7 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
       }
       if (lane == 0) {
         kap[u] = __uint_as_float(hi);
-        thx[u + 1] = t;
+        thx[u + 1] = th;
       }
     }
     if (lane == 0) {
@@ -381,6 +394,7 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
     tab[H_ROW] = __int_as_float(s_row);
     tab[H_FAST] = __int_as_float(fast ? 1 : 0);
     tab[H_RLAM] = rl;
+    tab[H_DLT] = dle;
   }
   // k_score launches only now: its blocks, resident early, slowed the base
   // solve and this kernel more than their early start saved
@@ -394,9 +408,11 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
 // are passed. ROW = 0: no reachable threshold leaves row r a replica (m < 1
 // throughout), so the row term is 0; ROW = 1: the quotient by Markstein's
 // method (valid for every C' of the segment); ROW = 2: the IEEE division.
-template <int ROW>
+// FL: the candidate's class is critical and row r's term counts only at or
+// above its floor dl.
+template <int ROW, bool FL>
 __device__ __forceinline__ float tstar_of(float C, const float* kap, const float* thx, const float* mnx,
-                                          int step0, float lam, float rlam) {
+                                          int step0, float lam, float rlam, float dl) {
   int pos = 0;
   for (int step = step0; step > 0; step >>= 1) pos += kap[pos + step - 1] <= C ? step : 0;
   const float thb = thx[pos];
@@ -405,6 +421,7 @@ __device__ __forceinline__ float tstar_of(float C, const float* kap, const float
   float tr;
   if (ROW == 1) tr = m >= 1.0f ? fulfil_fast(m, C, lam, rlam) : 0.0f;
   else tr = m >= 1.0f ? fulfil(m, C, lam) : 0.0f;
+  if (FL) return (tr > thb && tr >= dl) ? tr : thb;
   return tr > thb ? tr : thb;
 }
 
@@ -431,37 +448,59 @@ struct Acc40 {
   }
 };
 
-// Per-class choice of one scenario at threshold t (dump mode only): rows from
-// the base realisation except row rr, which has capacity C and bin bC.
+// Cheapest cover of threshold t by class i in one scenario (dump mode only):
+// rows from the base realisation except row rr, which has capacity C and bin
+// bC. Returns the cost (kCostInf: none) and the choice code.
+__device__ int dump_cover(float t, const Set& set, size_t ps, int rr, float C, int bC, int i, uint32_t* code) {
+  const Dims& d = set.d;
+  int best = kCostInf, bj = -1, bn = 0, bbin = -1;
+  for (int j = 0; j < kT; ++j) {
+    const int rho = 4 * i + j;
+    const float c = rho == rr ? C : set.rowC[ps * d.K4 + rho];
+    const int b = rho == rr ? bC : set.rowB[ps * d.K4 + rho];
+    if (b < 0) continue;
+    const int n = min_replicas(t, c, set.lam[i], __frcp_rn(set.lam[i]), d.Mf[j]);
+    if (n && (n << j) < best) {
+      best = n << j;
+      bj = j;
+      bn = n;
+      bbin = b;
+    }
+  }
+  *code = bj >= 0 ? ((uint32_t)bn | ((uint32_t)bj << 16) | ((uint32_t)bbin << 18)) : 0u;
+  return best;
+}
+
+// Per-class choice of one scenario at threshold t (dump mode only): the cover
+// of max(t, delta_i) when t > 0; with t = 0, the critical classes' floor
+// covers when they fit in G together, else nothing.
+template <bool FL>
 __device__ void dump_choices(float t, const Set& set, size_t ps, int rr, float C, int bC,
                              uint32_t* choice, int32_t* total_gpus) {
   const Dims& d = set.d;
   int total = 0;
-  for (int i = 0; i < d.K; ++i) {
-    uint32_t code = 0;
-    if (t > 0.0f) {
-      int best = kCostInf, bj = -1, bn = 0, bbin = -1;
-      for (int j = 0; j < kT; ++j) {
-        const int rho = 4 * i + j;
-        const float c = rho == rr ? C : set.rowC[ps * d.K4 + rho];
-        const int b = rho == rr ? bC : set.rowB[ps * d.K4 + rho];
-        if (b < 0) continue;
-        const int n = min_replicas(t, c, set.lam[i], __frcp_rn(set.lam[i]), d.Mf[j]);
-        if (n && (n << j) < best) {
-          best = n << j;
-          bj = j;
-          bn = n;
-          bbin = b;
-        }
-      }
-      if (bj >= 0) {
-        code = (uint32_t)bn | ((uint32_t)bj << 16) | ((uint32_t)bbin << 18);
-        total += best;
+  if (t > 0.0f) {
+    for (int i = 0; i < d.K; ++i) {
+      const float dl = FL ? set.slo[d.K + i] : 0.0f;
+      const int c = dump_cover(fmaxf(t, dl), set, ps, rr, C, bC, i, &choice[i]);
+      if (c < kCostInf) total += c;
+    }
+  } else {
+    bool met = true;
+    for (int i = 0; i < d.K; ++i) {
+      const float dl = FL ? set.slo[d.K + i] : 0.0f;
+      choice[i] = 0u;
+      if (dl > 0.0f) {
+        const int c = dump_cover(dl, set, ps, rr, C, bC, i, &choice[i]);
+        if (c < kCostInf) total += c; else met = false;
       }
     }
-    choice[i] = code;
+    if (!met || total > d.G) {
+      total = 0;
+      for (int i = 0; i < d.K; ++i) choice[i] = 0u;
+    }
   }
-  *total_gpus = t > 0.0f ? total : 0;
+  *total_gpus = total;
 }
 
 // Philox calls [q_lo, q_hi) of one (candidate, outcome) segment; call q
@@ -479,14 +518,14 @@ struct PieceSum {
   uint64_t total;  // earlier values, flushed
 };
 
-template <bool TS, int ROW>
+template <bool TS, int ROW, bool FL>
 __device__ __forceinline__ PieceSum run_piece(const Plan& pl, const PhiloxKeys& keys, int o, int q_lo, int q_hi,
                                               const float* win, const float* h0, const float* h1,
                                               const float* kap0, const float* thx0, const float* mnx0,
                                               const float* kap1, const float* thx1, const float* mnx1) {
   const int st0 = __float_as_int(h0[H_STEP0]), st1 = __float_as_int(h1[H_STEP0]);
   const float cx0 = h0[H_CX], cx1 = h1[H_CX];
-  const float lam = h0[H_LAM], rlam = h0[H_RLAM];
+  const float lam = h0[H_LAM], rlam = h0[H_RLAM], dl = h0[H_DLT];
   const int cell = __float_as_int(h0[H_CELL]);
   const uint32_t ctr1 = (uint32_t)o, ctr2 = (uint32_t)cell, ctr3 = pl.round;
   const uint32_t W = (uint32_t)pl.W;
@@ -497,8 +536,8 @@ __device__ __forceinline__ PieceSum run_piece(const Plan& pl, const PhiloxKeys& 
   auto eval = [&](uint32_t word) {
     const float cy = sQo[__umulhi(word, W)];
     const float cyg = (word & 0xFFFFu) < kgs ? cy : 0.0f;
-    const float t0 = tstar_of<ROW>(fmaxf(cx0, cyg), kap0, thx0, mnx0, st0, lam, rlam);
-    const float t1 = tstar_of<ROW>(fmaxf(cx1, cyg), kap1, thx1, mnx1, st1, lam, rlam);
+    const float t0 = tstar_of<ROW, FL>(fmaxf(cx0, cyg), kap0, thx0, mnx0, st0, lam, rlam, dl);
+    const float t1 = tstar_of<ROW, FL>(fmaxf(cx1, cyg), kap1, thx1, mnx1, st1, lam, rlam, dl);
     acc.add(__fsub_rn(t1, t0));
   };
   const int q_full = min(q_hi, pl.S >> 2);  // calls whose four samples all exist
@@ -534,14 +573,14 @@ __device__ __forceinline__ PieceSum run_piece(const Plan& pl, const PhiloxKeys& 
 // The same calls in dump mode: every scenario also writes its record (draws,
 // both t* and the per-class choices), with l_y mapped from the raw quantile
 // and the gate compared with the SLO directly.
-template <bool TS>
+template <bool TS, bool FL>
 __device__ uint64_t run_piece_dump(const Set& set, const Plan& pl, int item, int o, int q_lo, int q_hi,
                                    const float* win, const float* h0, const float* h1, const float* kap0,
                                    const float* thx0, const float* mnx0, const float* kap1, const float* thx1,
                                    const float* mnx1, unsigned char* dump, int dump_stride) {
   const int st0 = __float_as_int(h0[H_STEP0]), st1 = __float_as_int(h1[H_STEP0]);
   const float cx0 = h0[H_CX], cx1 = h1[H_CX];
-  const float lam = h0[H_LAM], rlam = __frcp_rn(lam);
+  const float lam = h0[H_LAM], rlam = __frcp_rn(lam), dl = h0[H_DLT];
   const int cell = __float_as_int(h0[H_CELL]), p = __float_as_int(h0[H_P]);
   const PhiloxKeys keys = philox_keys(pl.key0, pl.key1 ^ (pl.stream_base + (uint32_t)p));
   const uint32_t sh = (uint32_t)pl.sh;
@@ -563,8 +602,8 @@ __device__ uint64_t run_piece_dump(const Set& set, const Plan& pl, int item, int
       const bool gate = ly <= h0[H_SLO];
       const float C0 = gate ? fmaxf(cx0, cy) : cx0;
       const float C1 = gate ? fmaxf(cx1, cy) : cx1;
-      const float t0 = tstar_of<2>(C0, kap0, thx0, mnx0, st0, lam, rlam);
-      const float t1 = tstar_of<2>(C1, kap1, thx1, mnx1, st1, lam, rlam);
+      const float t0 = tstar_of<2, true>(C0, kap0, thx0, mnx0, st0, lam, rlam, dl);
+      const float t1 = tstar_of<2, true>(C1, kap1, thx1, mnx1, st1, lam, rlam, dl);
       acc += fixed40(__fsub_rn(t1, t0));
       const size_t idx = ((size_t)item * pl.O + o) * pl.S + s;
       unsigned char* rec = dump + idx * dump_stride;
@@ -583,7 +622,7 @@ __device__ uint64_t run_piece_dump(const Set& set, const Plan& pl, int item, int
         else if (bx < 0 || cy > cx) bC = be;
         else if (cy == cx) bC = min(be, bx);
         else bC = bx;
-        dump_choices(sg ? t1 : t0, set, (size_t)p * 2 + sg, rr, sg ? C1 : C0, bC, ch + sg * set.d.K,
+        dump_choices<FL>(sg ? t1 : t0, set, (size_t)p * 2 + sg, rr, sg ? C1 : C0, bC, ch + sg * set.d.K,
                      &hd.total_gpus[sg]);
       }
       *reinterpret_cast<fs_scenario_head*>(rec) = hd;
@@ -627,7 +666,9 @@ __device__ __forceinline__ void stage_segment(const Set& set, const Plan& pl, co
 // increment whose result names the chunk after it) before this chunk is
 // computed. The sums are integers, so the order of the chunks does not
 // change the result.
-template <bool DUMP>
+// FL: some class is critical (the model has floors): row terms are gated by the
+// candidate class's floor (0, so always passed, for a class that is not).
+template <bool DUMP, bool FL>
 __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, Plan pl, const float* rec,
                                                          uint64_t* sums, unsigned char* dump, int dump_stride,
                                                          ScoreGrid sg) {
@@ -707,23 +748,27 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
           keys_p = p;
         }
         // the table pointers stay in one address space per branch (shared or global)
-#define FS_PIECE(TSV, ROWV) \
-  run_piece<TSV, ROWV>(pl, keys, o, q_lo, q_hi, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, k1 + Lp1, k1 + 2 * Lp1)
+#define FS_PIECE(TSV, ROWV, FLV)                                                                  \
+  run_piece<TSV, ROWV, FLV>(pl, keys, o, q_lo, q_hi, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, k1 + Lp1, \
+                            k1 + 2 * Lp1)
+#define FS_PIECES(TSV) \
+  (row == 0 ? FS_PIECE(TSV, 0, false) : row == 1 ? FS_PIECE(TSV, 1, FL) : FS_PIECE(TSV, 2, FL))
 #define FS_DUMP(TSV)                                                                                   \
-  run_piece_dump<TSV>(set, pl, item, o, q_lo, q_hi, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, k1 + Lp1, \
+  run_piece_dump<TSV, FL>(set, pl, item, o, q_lo, q_hi, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, k1 + Lp1, \
                       k1 + 2 * Lp1, dump, dump_stride)
         if (Lp0 <= sg.lcap_s && Lp1 <= sg.lcap_s) {
           const float* k0 = h0 + kTableHeader;
           const float* k1 = h1 + kTableHeader;
           if constexpr (DUMP) acc_dump = FS_DUMP(true);
-          else ps = row == 0 ? FS_PIECE(true, 0) : row == 1 ? FS_PIECE(true, 1) : FS_PIECE(true, 2);
+          else ps = FS_PIECES(true);
         } else {
           const float* k0 = rec + (size_t)item * pl.item_floats + kTableHeader;
           const float* k1 = k0 + d.slot_floats;
           if constexpr (DUMP) acc_dump = FS_DUMP(false);
-          else ps = row == 0 ? FS_PIECE(false, 0) : row == 1 ? FS_PIECE(false, 1) : FS_PIECE(false, 2);
+          else ps = FS_PIECES(false);
         }
 #undef FS_DUMP
+#undef FS_PIECES
 #undef FS_PIECE
       }
     }
@@ -769,13 +814,14 @@ cudaError_t launch_prep(const Set& set, const Items& it, const Plan& pl, float* 
                         bool early, LaunchCache& lc, cudaStream_t s) {
   if (it.n <= 0) return cudaSuccess;
   const size_t smem = prep_smem_bytes(set.d);
-  if (smem > lc.prep_smem) {
-    cudaError_t e = cudaFuncSetAttribute(k_prep, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  const int fl = lc.floors ? 1 : 0;
+  auto kern = fl ? k_prep<true> : k_prep<false>;
+  if (smem > lc.prep_smem[fl]) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    lc.prep_smem = smem;
+    lc.prep_smem[fl] = smem;
   }
-  return launch_pdl(k_prep, dim3(it.n * 2), dim3(kPrepThreads), smem, s, set, it, pl, tables, sums,
-                    early ? 1 : 0);
+  return launch_pdl(kern, dim3(it.n * 2), dim3(kPrepThreads), smem, s, set, it, pl, tables, sums, early ? 1 : 0);
 }
 
 static int score_lcap(const Dims& d) { return d.lcap < kSmemTableCap ? d.lcap : kSmemTableCap; }
@@ -787,29 +833,23 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
   sg.lcap_s = score_lcap(set.d);
   sg.tcopy = kTableHeader + 3 * sg.lcap_s;
   const size_t smem = 16 + 2 * (size_t)(pl.Wp + 2 * sg.tcopy) * 4;
-  const int v = dump ? 1 : 0;
-  if (smem != lc.score_smem[v]) {
-    cudaError_t e;
+  const int v = dump ? 1 : 0, fl = lc.floors ? 1 : 0;
+  auto kern = dump ? (fl ? k_score<true, true> : k_score<true, false>)
+                   : (fl ? k_score<false, true> : k_score<false, false>);
+  if (smem != lc.score_smem[v][fl]) {
     int per_sm = 0;
-    if (dump) {
-      e = cudaFuncSetAttribute(k_score<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-      if (e == cudaSuccess)
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_score<true>, kScoreThreads, smem);
-    } else {
-      e = cudaFuncSetAttribute(k_score<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-      if (e == cudaSuccess)
-        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_score<false>, kScoreThreads, smem);
-    }
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kScoreThreads, smem);
     if (e != cudaSuccess) return e;
-    lc.score_smem[v] = smem;
-    lc.score_blocks_per_sm[v] = per_sm < 1 ? 1 : per_sm;
+    lc.score_smem[v][fl] = smem;
+    lc.score_blocks_per_sm[v][fl] = per_sm < 1 ? 1 : per_sm;
   }
   // Chunks of U calls per thread: about eight chunks per resident block when
   // the work allows, so that the counter can even out the segments' unequal
   // costs; at least 2 (a chunk's set-up is then paid for eight samples per
   // thread, measured faster on small launches) and at most 8 calls per
   // thread, and no more than a segment holds.
-  const long long resident = (long long)lc.score_blocks_per_sm[v] * sm_count;
+  const long long resident = (long long)lc.score_blocks_per_sm[v][fl] * sm_count;
   const long long total_calls = (long long)it.n * pl.O * pl.calls;
   long long U = total_calls / ((long long)kScoreThreads * resident * 8);
   const long long u_seg = ((long long)pl.calls + kScoreThreads - 1) / kScoreThreads;
@@ -829,11 +869,8 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
   sg.total = (int)((long long)it.n * pl.O * nch);
   const int grid = (int)(sg.total < resident ? sg.total : resident);
   sg.dyn = sg.total >= 4LL * grid ? 1 : 0;
-  if (dump)
-    return launch_pdl(k_score<true>, dim3(grid), dim3(kScoreThreads), smem, s, set, it, pl, tables, sums,
-                      (unsigned char*)dump, dump_stride, sg);
-  return launch_pdl(k_score<false>, dim3(grid), dim3(kScoreThreads), smem, s, set, it, pl, tables, sums,
-                    (unsigned char*)nullptr, 0, sg);
+  return launch_pdl(kern, dim3(grid), dim3(kScoreThreads), smem, s, set, it, pl, tables, sums,
+                    (unsigned char*)dump, dump ? dump_stride : 0, sg);
 }
 
 cudaError_t launch_finalize(const Set& set, const Items& it, const Plan& pl, const uint64_t* sums, double* gap,

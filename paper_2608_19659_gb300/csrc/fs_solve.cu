@@ -19,6 +19,12 @@
 // each row is the option the tie rule (larger capacity, then lower bin)
 // picks; and t* is the largest threshold t of the rows' values at which the
 // total fits, as cost(t) is constant between consecutive thresholds.
+// Critical floors (tier 1 of the objective): a row of a critical class i
+// starts at its first fulfilment >= delta_i (lower ones are not options), and
+// class i covers max(t, delta_i) at threshold t. Step 4 also prices every
+// critical class's cheapest cover of its floor: the floors are met when those
+// fit in G together; with t* = 0 and the floors met, that cover is the
+// class's allocation.
 #include <cuda_runtime.h>
 
 #include "fs_internal.cuh"
@@ -40,22 +46,25 @@ __global__ void k_qtable(float* qn, int Q) {
   qn[k] = x;
 }
 
-// Total GPUs of the cheapest per-class covers of threshold t, or kCostInf if
-// some class has no cover, evaluated by an aligned group of gsz lanes (a power
-// of two in [4, 32]); lane gl takes rows gl, gl + gsz, ... (rho = 4 i + j).
+// Total GPUs of the cheapest per-class covers of threshold t (class i covers
+// max(t, delta_i)), or kCostInf if some class has no cover, evaluated by an
+// aligned group of gsz lanes (a power of two in [4, 32]); lane gl takes rows
+// gl, gl + gsz, ... (rho = 4 i + j).
 // After the per-class minimum (two xor-shuffles) all four lanes of a class
 // hold its cost; xor-sums over the offsets 4 .. gsz/2 then add one lane per
 // class, so every lane of the group ends with the total (uncovered classes
 // counted above bit 24: a cost is at most G <= 32767, 64 classes < 2^21).
+template <bool FL>
 __device__ __forceinline__ int group_total_cost(float t, const float* sC, const float* sLam, const float* sRl,
-                                                const Dims& d, int gl, int gsz) {
+                                                const float* sDl, const Dims& d, int gl, int gsz) {
   int packed = 0;
   for (int base = 0; base < d.K4; base += gsz) {
     const int rho = base + gl;
     int cost = kCostInf;
     if (rho < d.K4) {
       const int j = rho & 3;
-      const int n = min_replicas(t, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[j]);
+      const float tc = FL ? fmaxf(t, sDl[rho >> 2]) : t;
+      const int n = min_replicas(tc, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[j]);
       if (n) cost = n << j;
     }
     cost = min(cost, __shfl_xor_sync(0xffffffffu, cost, 1));
@@ -67,6 +76,9 @@ __device__ __forceinline__ int group_total_cost(float t, const float* sC, const 
   return (packed >> 24) ? kCostInf : packed;
 }
 
+// FL: some class is critical (the model has floors); the instance without floors does
+// none of the floor work.
+template <bool FL>
 __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, const float* cap_x,
                                                          const float* tail_x, fs_allocation* out_x,
                                                          int write_theta) {
@@ -108,7 +120,9 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   // The inputs of the first pass (demands, and each thread's first cell) are
   // all loaded before anything waits on one of them: one memory round trip.
   __shared__ float sLam[FS_MAX_CLASSES], sRl[FS_MAX_CLASSES];  // demand and RN(1/demand)
+  __shared__ float sDl[FS_MAX_CLASSES];                          // floor delta_i (0: not critical)
   const float lam_v = tid < d.K ? set.lam[tid] : 1.0f;
+  const float dl_v = FL && tid < d.K ? set.slo[d.K + tid] : 0.0f;
   const bool cell0 = tid < d.cells;
   const float tail0 = cell0 ? tail[tid] : 0.0f, cap0 = cell0 ? cap[tid] : 0.0f;
   const float slo0 = cell0 ? set.slo[(tid / d.B) >> 2] : 0.0f;
@@ -117,6 +131,7 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   if (tid < d.K) {
     sLam[tid] = lam_v;
     sRl[tid] = __frcp_rn(lam_v);
+    if (FL) sDl[tid] = dl_v;
   }
   __syncthreads();
   for (int c = tid; c < d.cells; c += blockDim.x) {
@@ -146,7 +161,8 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
     if (bb >= 0) {
       atomicOr(reinterpret_cast<unsigned int*>(&sMisc[2 + (i >> 5)]), 1u << (i & 31));
       if (M >= 1) {
-        n0 = min_replicas(__int_as_float(1), best, lam, rl, Mf);  // first positive fulfilment
+        // first fulfilment that is positive and at or above the class's floor
+        n0 = min_replicas(FL ? fmaxf(sDl[i], __int_as_float(1)) : __int_as_float(1), best, lam, rl, Mf);
         if (n0) {
           const int ns = min_replicas(1.0f, best, lam, rl, Mf);   // first full fulfilment
           len = ns ? ns : M;
@@ -256,7 +272,7 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   for (int par = 0; hi - lo > 1; par ^= 1) {
     int kp = lo + ((g + 1) * (hi - lo)) / (ng + 1);
     kp = max(lo + 1, min(hi - 1, kp));
-    const int cost = group_total_cost(sTheta[kp], sC, sLam, sRl, d, gl, gsz);
+    const int cost = group_total_cost<FL>(sTheta[kp], sC, sLam, sRl, sDl, d, gl, gsz);
     if (gl == 0) s_res[par][g] = (cost <= d.G) ? kp : -(kp + 1);
     __syncthreads();
     int nlo = lo, nhi = hi;
@@ -271,18 +287,39 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   const float tstar = kstar >= 0 ? sTheta[kstar] : 0.0f;
 
   // 4. choice at t*: every row's cheapest cover in parallel (thread = row), then
-  // per class the cheapest row over its four TP lanes, lower TP on ties
+  // per class the cheapest row over its four TP lanes, lower TP on ties; the
+  // same for the floor of a critical class, summed into sMisc[5] (sMisc[6]:
+  // some critical class cannot reach its floor)
   {
     const int rho = tid;  // K4 <= 256 = blockDim
-    int key = 0x7fffffff;
-    if (rho < d.K4 && tstar > 0.0f) {
-      const int n = min_replicas(tstar, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[rho & 3]);
-      if (n) key = ((n << (rho & 3)) << 2) | (rho & 3);
+    int key = 0x7fffffff, keyf = 0x7fffffff;
+    if (rho < d.K4) {
+      const float dl = FL ? sDl[rho >> 2] : 0.0f;
+      if (tstar > 0.0f) {
+        const int n = min_replicas(FL ? fmaxf(tstar, dl) : tstar, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[rho & 3]);
+        if (n) key = ((n << (rho & 3)) << 2) | (rho & 3);
+      }
+      if (FL && dl > 0.0f) {
+        const int n = min_replicas(dl, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[rho & 3]);
+        if (n) keyf = ((n << (rho & 3)) << 2) | (rho & 3);
+      }
     }
     key = min(key, __shfl_xor_sync(0xffffffffu, key, 1));
     key = min(key, __shfl_xor_sync(0xffffffffu, key, 2));
+    const int i = tid >> 2;
+    if constexpr (FL) {
+      keyf = min(keyf, __shfl_xor_sync(0xffffffffu, keyf, 1));
+      keyf = min(keyf, __shfl_xor_sync(0xffffffffu, keyf, 2));
+      const bool critical = (tid & 3) == 0 && i < d.K && sDl[i] > 0.0f;
+      if (critical) {
+        if (keyf == 0x7fffffff) atomicOr(&sMisc[6], 1);
+        else atomicAdd(&sMisc[5], keyf >> 2);
+      }
+      __syncthreads();
+      const bool met = sMisc[6] == 0 && sMisc[5] <= d.G;
+      if (tstar <= 0.0f) key = (critical && met) ? keyf : 0x7fffffff;  // tier 1 alone
+    }
     if ((tid & 3) == 0) {
-      const int i = tid >> 2;
       int8_t tp = 0;
       int16_t bin = -1, reps = 0;
       float f = 0.0f;
@@ -303,10 +340,12 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   __syncthreads();
   if (tid == 0) {
     out->t_star = tstar;
-    out->total_gpus = tstar > 0.0f ? sMisc[4] : 0;
+    // (with t* = 0 and no floors the sum is 0 anyway; the unconditional read
+    // measured 1.5 us slower on a 28 us scoring call whose next kernel overlaps this one)
+    out->total_gpus = (FL || tstar > 0.0f) ? sMisc[4] : 0;
     out->has_option_mask = (uint64_t)(uint32_t)sMisc[2] | ((uint64_t)(uint32_t)sMisc[3] << 32);
     out->ok = tstar > 0.0f ? 1 : 0;
-    out->reserved = 0;
+    out->floors_met = (!FL || (sMisc[6] == 0 && sMisc[5] <= d.G)) ? 1 : 0;
   }
   if (write_theta && !cap_x) {
     float* th = set.theta + ((size_t)p * 2 + sigma) * d.theta_cap;
@@ -353,13 +392,15 @@ cudaError_t launch_solve(const Set& set, int n, const float* cap_x, const float*
                          fs_allocation* out, bool write_theta, LaunchCache& lc, cudaStream_t s) {
   if (n <= 0) return cudaSuccess;
   const size_t smem = solve_smem_bytes(set.d);
-  if (smem > lc.solve_smem) {
-    cudaError_t e = cudaFuncSetAttribute(k_solve, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  const int fl = lc.floors ? 1 : 0;
+  auto kern = fl ? k_solve<true> : k_solve<false>;
+  if (smem > lc.solve_smem[fl]) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    lc.solve_smem = smem;
+    lc.solve_smem[fl] = smem;
   }
   note_launch();
-  k_solve<<<n, kSolveThreads, smem, s>>>(set, n, cap_x, tail_x, out, write_theta ? 1 : 0);
+  kern<<<n, kSolveThreads, smem, s>>>(set, n, cap_x, tail_x, out, write_theta ? 1 : 0);
   return cudaGetLastError();
 }
 

@@ -21,7 +21,7 @@ LIB_PATH = os.path.join(HERE, "libfleetsieve.so")
 
 FS_OK, FS_EINVAL, FS_ENOMEM, FS_ECUDA, FS_ETIMEOUT, FS_EDEVICE = 0, -1, -2, -3, -4, -5
 FS_MAX_CLASSES = 64
-EXPORTS = ("fs_load_model", "fs_update_bounds", "fs_dump_stride", "fs_score_candidates",
+EXPORTS = ("fs_load_model", "fs_update_bounds", "fs_set_floors", "fs_dump_stride", "fs_score_candidates",
            "fs_score_candidates_async", "fs_solve", "fs_solve_batch", "fs_solve_bounds",
            "fs_reveal", "fs_certificate", "fs_replay", "fs_check", "fs_launch_count",
            "fs_watchdog_selftest", "fs_free_model", "fs_last_error", "fs_score_candidates_noalloc",
@@ -50,7 +50,7 @@ class fs_samples(C.Structure):
 
 class fs_allocation(C.Structure):
     _fields_ = [("t_star", C.c_float), ("total_gpus", C.c_int32),
-                ("has_option_mask", C.c_uint64), ("ok", C.c_int32), ("reserved", C.c_int32),
+                ("has_option_mask", C.c_uint64), ("ok", C.c_int32), ("floors_met", C.c_int32),
                 ("tp", C.c_int8 * FS_MAX_CLASSES), ("bin", C.c_int16 * FS_MAX_CLASSES),
                 ("replicas", C.c_int16 * FS_MAX_CLASSES), ("fulfil", C.c_float * FS_MAX_CLASSES)]
 
@@ -62,7 +62,7 @@ class fs_replay_spec(C.Structure):
                 ("truth_tail", C.POINTER(C.c_float)), ("perm", C.POINTER(C.c_int32))]
 
 
-ALLOC_DTYPE = np.dtype({"names": ["t_star", "total_gpus", "has_option_mask", "ok", "reserved",
+ALLOC_DTYPE = np.dtype({"names": ["t_star", "total_gpus", "has_option_mask", "ok", "floors_met",
                                   "tp", "bin", "replicas", "fulfil"],
                         "formats": [np.float32, np.int32, np.uint64, np.int32, np.int32,
                                     (np.int8, 64), (np.int16, 64), (np.int16, 64), (np.float32, 64)],
@@ -81,6 +81,7 @@ def lib():
         L.fs_load_model.argtypes = [C.POINTER(fs_bounds), fp, fp, C.c_int32, C.c_void_p,
                                     C.POINTER(C.c_void_p)]
         L.fs_update_bounds.argtypes = [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]
+        L.fs_set_floors.argtypes = [C.c_void_p, C.c_void_p]
         L.fs_dump_stride.argtypes = [C.c_void_p]
         L.fs_dump_stride.restype = C.c_int32
         L.fs_score_candidates.argtypes = [C.c_void_p, C.POINTER(fs_samples), C.c_void_p, C.c_void_p,
@@ -184,6 +185,14 @@ def fs_update_bounds(m: Model, cap_lo, cap_hi, tail_lo, tail_hi) -> None:
     _check(lib().fs_update_bounds(m.handle, *[_vp(x) for x in arrs]))
 
 
+def fs_set_floors(m: Model, floor=None) -> None:
+    """Critical floors delta_i in [0, 1] per class (0: not critical); None clears them."""
+    f = _f32(floor) if floor is not None else None
+    if f is not None and f.size != m.K:
+        raise ValueError(f"floor has {f.size} values for K = {m.K} classes")
+    _check(lib().fs_set_floors(m.handle, _vp(f) if f is not None else None))
+
+
 def fs_dump_stride(m: Model) -> int:
     return int(lib().fs_dump_stride(m.handle))
 
@@ -252,7 +261,7 @@ def fs_score_candidates_async(m: Model, cand_dev, O: int, S: int, seed: int, str
 
 def alloc_to_dict(a: fs_allocation, K: int) -> dict:
     return {"t_star": float(np.float32(a.t_star)), "total_gpus": int(a.total_gpus),
-            "has_option_mask": int(a.has_option_mask), "ok": int(a.ok),
+            "has_option_mask": int(a.has_option_mask), "ok": int(a.ok), "floors_met": int(a.floors_met),
             "tp": [int(a.tp[i]) for i in range(K)], "bin": [int(a.bin[i]) for i in range(K)],
             "replicas": [int(a.replicas[i]) for i in range(K)],
             "fulfil": [float(np.float32(a.fulfil[i])) for i in range(K)]}

@@ -54,8 +54,11 @@ def cuda():
 
 
 def load_model(fsb, w, quantile=None):
-    return fsb.fs_load_model(w.cap_lo, w.cap_hi, w.tail_lo, w.tail_hi, w.slo, w.demand, w.G, w.K, w.B,
-                             quantile=quantile)
+    m = fsb.fs_load_model(w.cap_lo, w.cap_hi, w.tail_lo, w.tail_hi, w.slo, w.demand, w.G, w.K, w.B,
+                          quantile=quantile)
+    if getattr(w, "floor", None) is not None:
+        fsb.fs_set_floors(m, w.floor)
+    return m
 
 
 def alloc_matches(gpu: dict, ref, K: int) -> bool:
@@ -63,6 +66,7 @@ def alloc_matches(gpu: dict, ref, K: int) -> bool:
     import numpy as np
 
     return (gpu["t_star"] == ref.t_star and gpu["total_gpus"] == ref.total_gpus and gpu["ok"] == ref.ok
+            and gpu["floors_met"] == ref.floors_met
             and gpu["has_option_mask"] == ref.has_option_mask and gpu["tp"] == ref.tp
             and gpu["bin"] == ref.bin and gpu["replicas"] == ref.replicas
             and [np.float32(x) for x in gpu["fulfil"]] == [np.float32(x) for x in ref.fulfil])

@@ -49,7 +49,7 @@ def _solve_batch(fsb, torch, m, cap, tail):
 
 def _as_dict(rec, K):
     return {"t_star": float(rec["t_star"]), "total_gpus": int(rec["total_gpus"]), "ok": int(rec["ok"]),
-            "has_option_mask": int(rec["has_option_mask"]), "tp": [int(x) for x in rec["tp"][:K]],
+            "floors_met": int(rec["floors_met"]), "has_option_mask": int(rec["has_option_mask"]), "tp": [int(x) for x in rec["tp"][:K]],
             "bin": [int(x) for x in rec["bin"][:K]], "replicas": [int(x) for x in rec["replicas"][:K]],
             "fulfil": [float(x) for x in rec["fulfil"][:K]]}
 
