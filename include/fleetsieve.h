@@ -278,7 +278,10 @@ int fs_certificate(fs_model *m, float eps, int32_t *state, float *gamma_t);
  * Each round: A-, A+, certificate (eps, the model's floors); if undecided, score the unrevealed
  * cells (perm order) with O x S samples, Philox stream id k and round r,
  * then reveal the argmax. Stops on the certificate, when no cell is left, or
- * after max_rounds. All inputs are host pointers; outputs host, nullable:
+ * after max_rounds. policy 1 replaces the scored choice by the next
+ * unrevealed cell of perm[k] (no scoring): the fixed-order baselines of
+ * Section 6.2 (uniform random for a random perm, fixed grid order for a perm
+ * that lists the grid), stopped by the same certificate. All inputs are host pointers; outputs host, nullable:
  *   rounds[k], state[k] (the certificate's 1 or 2, or 0 when the stream ran out
  *   of cells or rounds undecided), gpu_seconds[k] (300 s x TP per revealed cell),
  *   reveal_order[k][cells] (-1 padded), gamma_trace[k][max_rounds+1],
@@ -291,6 +294,7 @@ typedef struct {
     int32_t O;
     int32_t S;
     int32_t max_rounds;
+    int32_t policy;           /* 0: reveal the best-scored cell; 1: the next cell of perm */
     uint64_t seed;
     const float *truth_cap;
     const float *truth_tail;

@@ -88,7 +88,7 @@ def lib():
                                         C.POINTER(C.c_int), fp]
         _lib.or_replay_stream.argtypes = [C.POINTER(_Problem), fp, fp, fp, fp, fp, fp, ip,
                                           C.c_int, C.c_float, fp, C.c_int, C.c_uint64,
-                                          C.c_uint32, C.c_int, C.c_int, C.c_int, C.c_int,
+                                          C.c_uint32, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int,
                                           ip, ip, ip, C.POINTER(C.c_double), ip,
                                           C.POINTER(_Alloc), fp]
     return _lib
@@ -280,7 +280,10 @@ class ReplayResult:
 
 
 def replay_stream(rp, k: int, qn, seed: int, S=None, O=None, max_rounds=None,
-                  solver=SOLVER_FRONTIER) -> ReplayResult:
+                  solver=SOLVER_FRONTIER, policy: int = 0, perm=None) -> ReplayResult:
+    """Algorithm 1 on stream k of the replay ``rp``. policy 0: reveal the
+    best-scored cell; 1: the next unrevealed cell of ``perm`` (default: the
+    stream's own permutation)."""
     w = rp.base
     prob = Problem.of(w)
     b = _bounds(w)
@@ -288,7 +291,7 @@ def replay_stream(rp, k: int, qn, seed: int, S=None, O=None, max_rounds=None,
     cells = w.cells
     tc = _f32(rp.truth_cap[k])
     tl = _f32(rp.truth_tail[k])
-    perm = np.ascontiguousarray(rp.perm[k], np.int32)
+    perm = np.ascontiguousarray(rp.perm[k] if perm is None else perm, np.int32)
     order = np.full(cells, -1, np.int32)
     mr = rp.max_rounds if max_rounds is None else max_rounds
     trace = np.zeros(mr + 1, np.float32)
@@ -298,7 +301,7 @@ def replay_stream(rp, k: int, qn, seed: int, S=None, O=None, max_rounds=None,
     rc = lib().or_replay_stream(C.byref(prob._s), *[_ptr(x, C.c_float) for x in b],
                                 _ptr(tc, C.c_float), _ptr(tl, C.c_float), _ptr(perm, C.c_int32),
                                 rp.r0, rp.eps, _ptr(qn, C.c_float), qn.size, seed, k,
-                                w.O if O is None else O, w.S if S is None else S, mr, solver,
+                                w.O if O is None else O, w.S if S is None else S, mr, solver, policy,
                                 C.byref(rounds), _ptr(order, C.c_int32), C.byref(nrev),
                                 C.byref(gs), C.byref(st), C.byref(am), _ptr(trace, C.c_float))
     if rc:

@@ -184,18 +184,22 @@ int or_certificate(const or_problem *p, const float *cap_lo, const float *cap_hi
  * earlier in perm). Revealing sets lo = hi = the hidden true value. Each
  * revealed cell costs 300 s x TP GPU-seconds (Section 5). Trajectories are
  * parity unpinned against the paper (its measured grid is not available).
+ * policy 1 replaces the scored choice by the next unrevealed cell of perm:
+ * the fixed-order baselines of Section 6.2 (uniform random when perm is a
+ * random permutation, fixed grid order when it lists the grid), stopped by
+ * the same certificate.
  */
 int or_replay_stream(const or_problem *p, const float *prior_cap_lo, const float *prior_cap_hi,
                      const float *prior_tail_lo, const float *prior_tail_hi,
                      const float *truth_cap, const float *truth_tail, const int32_t *perm,
                      int r0, float eps, const float *qn, int Q, uint64_t seed,
-                     uint32_t stream_id, int O, int S, int max_rounds, int solver,
+                     uint32_t stream_id, int O, int S, int max_rounds, int solver, int policy,
                      int32_t *rounds, int32_t *reveal_order, int32_t *n_revealed,
                      double *gpu_seconds, int32_t *state, or_alloc *final_minus,
                      float *gamma_trace)
 {
     int cells = cells_of(p);
-    if (r0 < 0 || r0 > cells) return -1;
+    if (r0 < 0 || r0 > cells || policy < 0 || policy > 1) return -1;
     float *buf = (float *)malloc(sizeof(float) * cells * 4);
     uint8_t *rev = (uint8_t *)calloc(cells, 1);
     int32_t *cand = (int32_t *)malloc(sizeof(int32_t) * cells);
@@ -227,11 +231,13 @@ int or_replay_stream(const or_problem *p, const float *prior_cap_lo, const float
         for (int q = 0; q < cells; ++q)
             if (!rev[perm[q]]) cand[nc++] = perm[q];
         if (nc == 0 || r >= max_rounds) { st = 0; break; }
-        int32_t bestc;
-        float g2;
-        rc = or_score(p, clo, chi, tlo, thi, qn, Q, seed, stream_id, (uint32_t)r, nc, cand, O, S,
-                      solver, NULL, NULL, NULL, NULL, &g2, &bestc, NULL);
-        if (rc) break;
+        int32_t bestc = cand[0];
+        if (policy == 0) {
+            float g2;
+            rc = or_score(p, clo, chi, tlo, thi, qn, Q, seed, stream_id, (uint32_t)r, nc, cand, O, S,
+                          solver, NULL, NULL, NULL, NULL, &g2, &bestc, NULL);
+            if (rc) break;
+        }
         clo[bestc] = chi[bestc] = truth_cap[bestc];
         tlo[bestc] = thi[bestc] = truth_tail[bestc];
         rev[bestc] = 1;

@@ -108,12 +108,13 @@ int or_certificate(const or_problem *p, const float *cap_lo, const float *cap_hi
                    const float *tail_lo, const float *tail_hi, const uint8_t *revealed,
                    float eps, int solver, int *state, float *gamma_t);
 
-/* Algorithm 1 on one reveal order. */
+/* Algorithm 1 on one reveal order; policy 0 reveals the best-scored cell,
+ * policy 1 the next unrevealed cell of perm (the fixed-order baselines). */
 int or_replay_stream(const or_problem *p, const float *prior_cap_lo, const float *prior_cap_hi,
                      const float *prior_tail_lo, const float *prior_tail_hi,
                      const float *truth_cap, const float *truth_tail, const int32_t *perm,
                      int r0, float eps, const float *qn, int Q, uint64_t seed,
-                     uint32_t stream_id, int O, int S, int max_rounds, int solver,
+                     uint32_t stream_id, int O, int S, int max_rounds, int solver, int policy,
                      int32_t *rounds, int32_t *reveal_order, int32_t *n_revealed,
                      double *gpu_seconds, int32_t *state, or_alloc *final_minus,
                      float *gamma_trace);

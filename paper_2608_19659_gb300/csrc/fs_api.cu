@@ -612,6 +612,7 @@ int fs_replay(fs_model* m, const fs_replay_spec* sp, int32_t* rounds, int32_t* s
   if (sp->r0 < 0 || sp->r0 > cells) return fail(FS_EINVAL, "r0 = %d outside [0, cells]", sp->r0);
   if (sp->max_rounds < 0 || sp->max_rounds > cells) return fail(FS_EINVAL, "max_rounds outside [0, cells]");
   if (std::isnan(sp->eps)) return fail(FS_EINVAL, "eps is NaN");
+  if (sp->policy < 0 || sp->policy > 1) return fail(FS_EINVAL, "policy = %d is not 0 or 1", sp->policy);
   if (!sp->truth_cap || !sp->truth_tail || !sp->perm) return fail(FS_EINVAL, "NULL truth / perm");
   fs_samples probe{sp->seed, 0, 0, 0, sp->O, sp->S, 0, nullptr};
   int rc = check_samples(m, &probe, false);
@@ -704,6 +705,10 @@ int fs_replay(fs_model* m, const fs_replay_spec* sp, int32_t* rounds, int32_t* s
       if (n_active == 0) break;
       const int per = cells - sp->r0 - r;
       if (per <= 0) break;
+      if (sp->policy == 1) {
+        FS_CUDA(launch_replay_next(set, rs, n_active, s), "launch reveal");
+        continue;
+      }
       const int n_items = n_active * per;
       int rc2 = ensure_items(m, n_items, sp->O);
       if (rc2) return rc2;

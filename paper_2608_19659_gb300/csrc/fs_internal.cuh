@@ -398,6 +398,7 @@ cudaError_t launch_replay_init(const Set& set, const ReplayState& rs, int r0, cu
 cudaError_t launch_replay_certify(const Set& set, const ReplayState& rs, int round, cudaStream_t s);
 cudaError_t launch_replay_items(const Set& set, const ReplayState& rs, int n_active, int per,
                                 cudaStream_t s);
+cudaError_t launch_replay_next(const Set& set, const ReplayState& rs, int n_active, cudaStream_t s);
 cudaError_t launch_replay_reveal(const Set& set, const ReplayState& rs, const Items& it,
                                  const Plan& pl, const uint64_t* sums, int n_active, cudaStream_t s);
 

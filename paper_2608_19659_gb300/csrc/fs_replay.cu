@@ -5,6 +5,8 @@
 //   A-, A+ (k_solve) -> certificate (Section 4.2) -> candidate list (the
 //   unrevealed cells in the stream's reveal order) -> k_prep / k_score
 //   (Section 4.3) -> argmax -> reveal (interval collapses to the truth).
+// The fixed-order policy skips the scoring and reveals the next cell of the
+// stream's order.
 // The host only reads the number of streams still going once per round.
 #include <cuda_runtime.h>
 
@@ -88,6 +90,23 @@ __global__ void k_replay_items(Set set, ReplayState rs, int n_active, int per) {
   if (q != per) atomicOr(set.status, ST_TABLE);
 }
 
+// Fixed-order policy: running stream slot a reveals its next unrevealed cell
+// in reveal order (the candidate list's first entry).
+__global__ void k_replay_next(Set set, ReplayState rs, int n_active) {
+  const int a = blockIdx.x * blockDim.x + threadIdx.x;
+  if (a >= n_active) return;
+  const int p = rs.active[a];
+  const Dims& d = set.d;
+  for (int k = 0; k < d.cells; ++k) {
+    const int c = rs.perm[(size_t)p * d.cells + k];
+    if (!set.revealed[(size_t)p * d.cells + c]) {
+      reveal_cell(set, rs, p, c);
+      return;
+    }
+  }
+  atomicOr(set.status, ST_TABLE);  // a running stream always has an unrevealed cell
+}
+
 __global__ void k_replay_reveal(Set set, ReplayState rs, Items it, Plan pl, const uint64_t* sums, int per) {
   const int a = blockIdx.x;
   const int p = rs.active[a];
@@ -110,6 +129,12 @@ cudaError_t launch_replay_certify(const Set& set, const ReplayState& rs, int rou
 cudaError_t launch_replay_items(const Set& set, const ReplayState& rs, int n_active, int per, cudaStream_t s) {
   note_launch();
   k_replay_items<<<(n_active + 127) / 128, 128, 0, s>>>(set, rs, n_active, per);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_replay_next(const Set& set, const ReplayState& rs, int n_active, cudaStream_t s) {
+  note_launch();
+  k_replay_next<<<(n_active + 127) / 128, 128, 0, s>>>(set, rs, n_active);
   return cudaGetLastError();
 }
 

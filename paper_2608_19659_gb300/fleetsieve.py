@@ -58,7 +58,7 @@ class fs_allocation(C.Structure):
 class fs_replay_spec(C.Structure):
     _fields_ = [("n_streams", C.c_int32), ("r0", C.c_int32), ("eps", C.c_float),
                 ("O", C.c_int32), ("S", C.c_int32), ("max_rounds", C.c_int32),
-                ("seed", C.c_uint64), ("truth_cap", C.POINTER(C.c_float)),
+                ("policy", C.c_int32), ("seed", C.c_uint64), ("truth_cap", C.POINTER(C.c_float)),
                 ("truth_tail", C.POINTER(C.c_float)), ("perm", C.POINTER(C.c_int32))]
 
 
@@ -309,12 +309,13 @@ class ReplayResult:
 
 
 def fs_replay(m: Model, truth_cap, truth_tail, perm, r0: int, eps: float, O: int, S: int,
-              seed: int, max_rounds: int) -> ReplayResult:
+              seed: int, max_rounds: int, policy: int = 0) -> ReplayResult:
+    """policy 0: reveal the best-scored cell each round; 1: the next unrevealed cell of perm."""
     tc = _f32(truth_cap)
     tl = _f32(truth_tail)
     pm = np.ascontiguousarray(perm, dtype=np.int32).reshape(-1)
     n = pm.size // m.cells
-    spec = fs_replay_spec(n, int(r0), float(eps), int(O), int(S), int(max_rounds),
+    spec = fs_replay_spec(n, int(r0), float(eps), int(O), int(S), int(max_rounds), int(policy),
                           int(seed) & (2**64 - 1), _fp(tc), _fp(tl),
                           pm.ctypes.data_as(C.POINTER(C.c_int32)))
     rounds = np.zeros(n, np.int32)

@@ -79,3 +79,37 @@ def test_replay_rejects_bad_specs(fsb, cuda):
             fsb.fs_replay(m, rp.truth_cap, rp.truth_tail, bad, 6, 0.01, 8, 16, 1, 64)
         with pytest.raises(fsb.FleetSieveError):
             fsb.fs_replay(m, rp.truth_cap, rp.truth_tail, rp.perm, 6, 0.01, 3, 16, 1, 64)
+
+
+def test_fixed_order_policies_match_oracle(fsb, cuda, oracle_lib, qn):
+    """Section 6.2's fixed-order baselines (uniform random, fixed grid order) on the
+    GPU replay: same stop, state, order, GPU-seconds and final allocation as the oracle."""
+    from paper_2608_19659_gb300 import compare
+
+    rp = workloads.make_replay(n_streams=10)
+    w = rp.base
+    for perm in (rp.perm, compare.grid_order(rp.perm, rp.r0)):
+        with load_model(fsb, w) as m:
+            res = fsb.fs_replay(m, rp.truth_cap, rp.truth_tail, perm, rp.r0, rp.eps, w.O, 16, 3,
+                                rp.max_rounds, policy=1)
+        for k in range(10):
+            ref = oracle_lib.replay_stream(rp, k, qn, seed=3, S=16, policy=1, perm=perm[k])
+            _compare(fsb, res, rp, k, ref, w.K)
+
+
+def test_policy_comparison_runs(fsb, cuda):
+    from paper_2608_19659_gb300 import compare
+
+    rp = workloads.make_replay(n_streams=8)
+    w = rp.base
+    with load_model(fsb, w) as m:
+        runs = compare.run_policies(m, rp, 4, 32, 7)
+        with pytest.raises(fsb.FleetSieveError):
+            fsb.fs_replay(m, rp.truth_cap, rp.truth_tail, rp.perm, rp.r0, rp.eps, 4, 32, 7, 10, policy=2)
+    assert set(runs) == {"fleetsieve", "uniform_random", "fixed_grid"}
+    for r in runs.values():
+        assert np.all(r.state == 1)
+        assert np.allclose(r.class_seconds.sum(axis=1), r.gpu_seconds)
+    s = compare.summarise(runs["fleetsieve"], runs["uniform_random"], n_boot=200)
+    lo, hi = s["ci95"]
+    assert lo <= s["advantage"] <= hi and len(s["per_class"]) == w.K
