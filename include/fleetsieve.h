@@ -95,9 +95,11 @@ int fs_load_model(const fs_bounds *bounds, const float *slo, const float *demand
  * fs_update_bounds -- replace the four bound arrays (host, [K][4][B]) of a
  * model, e.g. after the intervals were refit (Algorithm 1, "fit joint
  * capacity and tail intervals"). Revealed flags are kept. The arrays are
- * copied before the call returns; the device copy is queued on the model's
- * stream without waiting, and every later call on the model is ordered after
- * it (work a later call queues on another stream waits for it).
+ * copied (into page-locked staging) before the call returns, which queues no
+ * device work: the next call that needs the bounds on the device queues their
+ * copy on the model's stream (work it queues on another stream waits for it),
+ * and fs_score_candidates reads freshly staged bounds where they are. Every
+ * later call on the model sees the new bounds.
  */
 int fs_update_bounds(fs_model *m, const float *cap_lo, const float *cap_hi,
                      const float *tail_lo, const float *tail_hi);
@@ -258,7 +260,7 @@ int fs_solve_batch(fs_model *m, int32_t n, const float *cap_dev, const float *ta
 int fs_solve_bounds(fs_model *m, fs_allocation *minus, fs_allocation *plus, float *gamma_t);
 
 /* Measurement of one cell: lo = hi = the measured value, marks it revealed
- * (queued for the device like fs_update_bounds). */
+ * (staged for the device like fs_update_bounds). */
 int fs_reveal(fs_model *m, int32_t cell, float cap, float tail);
 
 /*

@@ -82,20 +82,26 @@ struct Buf {
   }
 };
 
-// Page-locked host memory that grows on demand: copies to and from it are
-// asynchronous, so a call can queue them and wait once.
+// Page-locked host memory that grows on demand, mapped into the device's
+// address space: copies to and from it are asynchronous, so a call can queue
+// them and wait once, and kernels can read and write it directly (dev).
 struct HostBuf {
   void* p = nullptr;
+  void* dev = nullptr;
   size_t bytes = 0;
   int ensure(size_t want, const char* what) {
     if (want <= bytes) return FS_OK;
     if (p) cudaFreeHost(p);
     p = nullptr;
+    dev = nullptr;
     bytes = 0;
     size_t b = std::max<size_t>(want, 256);
-    cudaError_t e = cudaMallocHost(&p, b);
+    cudaError_t e = cudaHostAlloc(&p, b, cudaHostAllocMapped);
+    if (e == cudaSuccess) e = cudaHostGetDevicePointer(&dev, p, 0);
     if (e != cudaSuccess) {
+      if (p) cudaFreeHost(p);
       p = nullptr;
+      dev = nullptr;
       return cuda_fail(e, what);
     }
     bytes = b;
@@ -104,6 +110,7 @@ struct HostBuf {
   void release() {
     if (p) cudaFreeHost(p);
     p = nullptr;
+    dev = nullptr;
     bytes = 0;
   }
 };
@@ -131,6 +138,7 @@ struct fs_model {
   HostBuf h_up, h_out;
   cudaEvent_t up_done = nullptr;
   bool up_pending = false;
+  bool staged = false;  // the staging holds bounds the device copy does not have yet
   LaunchCache lc;
   // optional timing events: 5 per timed call (before solve, prep, score,
   // finalize, and after finalize); mode 1 records only the two around score
@@ -182,10 +190,12 @@ int order_after_upload(fs_model* m, cudaStream_t s) {
   return FS_OK;
 }
 
-// Queue the host mirror's bounds and revealed flags for the device (from
-// page-locked staging, without waiting): later work on the model's stream
-// is ordered after the copy, work on other streams waits for up_done.
-int upload_bounds(fs_model* m) {
+// Stage the host mirror's bounds and revealed flags in page-locked memory
+// (once the previous staging's device copy has run). No CUDA work is queued:
+// the next call that needs the bounds on the device queues the copy
+// (flush_bounds), and a synchronous scoring call reads the staged bounds
+// directly, so an update costs no copy-engine round trip of its own.
+int stage_bounds(fs_model* m) {
   const size_t nb = m->h_bounds.size() * 4, nr = m->h_revealed.size();
   int rc = wait_upload(m);
   if (rc) return rc;
@@ -196,11 +206,23 @@ int upload_bounds(fs_model* m) {
   char* h = static_cast<char*>(m->h_up.p);
   std::memcpy(h, m->h_bounds.data(), nb);
   std::memcpy(h + rev_off, m->h_revealed.data(), nr);
-  FS_CUDA(cudaMemcpyAsync(m->set.bounds, h, rev_off + nr, cudaMemcpyHostToDevice, m->stream), "upload bounds");
-  if (!m->up_done) FS_CUDA(cudaEventCreateWithFlags(&m->up_done, cudaEventDisableTiming), "create upload event");
-  FS_CUDA(cudaEventRecord(m->up_done, m->stream), "record upload event");
-  m->up_pending = true;
+  m->staged = true;
   return FS_OK;
+}
+
+// Queue the device copy of staged bounds (if any) on the model's stream without
+// waiting, and order work on stream s after the last such copy.
+int flush_bounds(fs_model* m, cudaStream_t s) {
+  if (m->staged) {
+    const size_t span = (size_t)(reinterpret_cast<char*>(m->set.revealed) - reinterpret_cast<char*>(m->set.bounds)) +
+                        m->h_revealed.size();
+    FS_CUDA(cudaMemcpyAsync(m->set.bounds, m->h_up.p, span, cudaMemcpyHostToDevice, m->stream), "upload bounds");
+    if (!m->up_done) FS_CUDA(cudaEventCreateWithFlags(&m->up_done, cudaEventDisableTiming), "create upload event");
+    FS_CUDA(cudaEventRecord(m->up_done, m->stream), "record upload event");
+    m->up_pending = true;
+    m->staged = false;
+  }
+  return order_after_upload(m, s);
 }
 
 // Turn a nonzero device status word into an error (and clear it for the next call).
@@ -269,8 +291,9 @@ int ensure_items(fs_model* m, int n, int O) {
 }
 
 // The scoring sequence on stream s; cand_dev holds n_cand cell ids.
-int run_score(fs_model* m, const fs_samples* smp, const int32_t* cand_dev, double* gap, double* score,
-              float* gamma_t, int32_t* best, void* dump, cudaStream_t s, uint32_t* status_copy = nullptr) {
+int run_score(fs_model* m, const Set& set, const fs_samples* smp, const int32_t* cand_dev, double* gap,
+              double* score, float* gamma_t, int32_t* best, void* dump, cudaStream_t s,
+              uint32_t* status_copy = nullptr) {
   const int n = smp->n_cand;
   Items it{};
   it.n = n;
@@ -291,15 +314,15 @@ int run_score(fs_model* m, const fs_samples* smp, const int32_t* cand_dev, doubl
   }
   const bool phases = timed && m->timing == 2;
   if (phases) FS_CUDA(cudaEventRecord(ev[0], s), "record timing event");
-  FS_CUDA(launch_solve(m->set, 2, nullptr, nullptr, nullptr, true, m->lc, s), "launch solve");
+  FS_CUDA(launch_solve(set, 2, nullptr, nullptr, nullptr, true, m->lc, s), "launch solve");
   if (phases) FS_CUDA(cudaEventRecord(ev[1], s), "record timing event");
-  FS_CUDA(launch_prep(m->set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, true, m->lc, s), "launch prep");
+  FS_CUDA(launch_prep(set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, true, m->lc, s), "launch prep");
   if (timed) FS_CUDA(cudaEventRecord(ev[2], s), "record timing event");
-  FS_CUDA(launch_score(m->set, it, pl, (const float*)m->tables.p, (uint64_t*)m->sums.p, dump,
+  FS_CUDA(launch_score(set, it, pl, (const float*)m->tables.p, (uint64_t*)m->sums.p, dump,
                        fs_dump_stride(m), m->sm_count, m->lc, s),
           "launch score");
   if (timed) FS_CUDA(cudaEventRecord(ev[3], s), "record timing event");
-  FS_CUDA(launch_finalize(m->set, it, pl, (const uint64_t*)m->sums.p, gap, score, gamma_t, best, status_copy, s),
+  FS_CUDA(launch_finalize(set, it, pl, (const uint64_t*)m->sums.p, gap, score, gamma_t, best, status_copy, s),
           "launch finalize");
   if (phases) FS_CUDA(cudaEventRecord(ev[4], s), "record timing event");
   return FS_OK;
@@ -428,7 +451,8 @@ int fs_load_model(const fs_bounds* b, const float* slo, const float* demand, int
     else e = launch_qtable((float*)s.qn, Q, m->stream);
   }
   if (e != cudaSuccess) return bail(cuda_fail(e, "model upload"));
-  rc = upload_bounds(m);
+  rc = stage_bounds(m);
+  if (rc == FS_OK) rc = flush_bounds(m, m->stream);
   if (rc) return bail(rc);
   *out = m;
   return FS_OK;
@@ -443,7 +467,7 @@ int fs_update_bounds(fs_model* m, const float* cap_lo, const float* cap_hi, cons
   const float* src[4] = {cap_lo, cap_hi, tail_lo, tail_hi};
   for (int r = 0; r < 4; ++r)
     for (int c = 0; c < cells; ++c) m->h_bounds[(size_t)r * cells + c] = canon(src[r][c]);
-  return upload_bounds(m);
+  return stage_bounds(m);
 }
 
 int fs_set_floors(fs_model* m, const float* floor) {
@@ -473,27 +497,32 @@ int fs_score_candidates(fs_model* m, const fs_samples* smp, double* gap_out, dou
   if (rc) return rc;
   const int n = smp->n_cand;
   if ((rc = ensure_items(m, n, smp->O))) return rc;
-  double* d_gap = (double*)m->outs.p;
-  double* d_score = d_gap + std::max(n, 1);
-  float* d_gt = (float*)(d_score + std::max(n, 1));
-  int32_t* d_best = (int32_t*)(d_gt + 4);
-  cudaStream_t s = m->stream;
-  if (n > 0)
-    FS_CUDA(cudaMemcpyAsync(m->cand.p, smp->cand, 4 * (size_t)n, cudaMemcpyHostToDevice, s), "upload candidates");
-  // the status word joins the outputs on the device (gap, score, gamma_t,
-  // best, status are contiguous; k_finalize copies it), and one copy brings
-  // them all to staging
+  // One mapped page-locked block carries the call's host data both ways: the
+  // kernels read the candidate ids from it and write gap, score, gamma_t, best
+  // and the status word into it (k_finalize copies the status word), so no
+  // copy engine sits before the first kernel or after the last one.
   const size_t nn = (size_t)std::max(n, 1);
+  const size_t out_bytes = align_up(16 * nn + 36, 16);
+  if ((rc = m->h_out.ensure(out_bytes + 4 * nn, "host staging"))) return rc;
+  char* h = static_cast<char*>(m->h_out.p);
+  char* hd = static_cast<char*>(m->h_out.dev);
+  if (n > 0) std::memcpy(h + out_bytes, smp->cand, 4 * (size_t)n);
+  double* d_gap = reinterpret_cast<double*>(hd);
+  double* d_score = d_gap + nn;
+  float* d_gt = reinterpret_cast<float*>(d_score + nn);
+  int32_t* d_best = reinterpret_cast<int32_t*>(d_gt + 4);
   uint32_t* d_st = reinterpret_cast<uint32_t*>(d_best + 4);
-  rc = run_score(m, smp, (const int32_t*)m->cand.p, d_gap, d_score, d_gt, d_best, dump_dev, s, d_st);
+  cudaStream_t s = m->stream;
+  // freshly staged bounds are read where they are (their device copy waits
+  // for the next call that needs it)
+  Set set = m->set;
+  if (m->staged) set.bounds = static_cast<float*>(m->h_up.dev);
+  rc = run_score(m, set, smp, reinterpret_cast<const int32_t*>(hd + out_bytes), d_gap, d_score, d_gt, d_best,
+                 dump_dev, s, d_st);
   if (rc) return rc;
-  const size_t out_bytes = 16 * nn + 36;
-  if ((rc = m->h_out.ensure(out_bytes, "output staging"))) return rc;
-  FS_CUDA(cudaMemcpyAsync(m->h_out.p, m->outs.p, out_bytes, cudaMemcpyDeviceToHost, s), "read outputs");
   if (sum_eo && n)
     FS_CUDA(cudaMemcpyAsync(sum_eo, m->sums.p, 8 * (size_t)n * smp->O, cudaMemcpyDeviceToHost, s), "read sums");
   FS_CUDA(cudaStreamSynchronize(s), "synchronize");
-  const char* h = static_cast<const char*>(m->h_out.p);
   uint32_t st;
   std::memcpy(&st, h + 16 * nn + 32, 4);
   if (st) return status_error(m, st);
@@ -513,8 +542,8 @@ int fs_score_candidates_async(fs_model* m, const fs_samples* smp, double* gap_de
   const int n = smp->n_cand;
   if ((rc = ensure_items(m, n, smp->O))) return rc;
   cudaStream_t s = (cudaStream_t)cuda_stream;
-  if ((rc = order_after_upload(m, s))) return rc;
-  rc = run_score(m, smp, smp->cand, gap_dev, score_dev, gamma_t_dev, best_dev, dump_dev, s);
+  if ((rc = flush_bounds(m, s))) return rc;
+  rc = run_score(m, m->set, smp, smp->cand, gap_dev, score_dev, gamma_t_dev, best_dev, dump_dev, s);
   if (rc) return rc;
   if (sum_eo_dev && n)
     FS_CUDA(cudaMemcpyAsync(sum_eo_dev, m->sums.p, 8 * (size_t)n * smp->O, cudaMemcpyDeviceToDevice, s),
@@ -546,7 +575,7 @@ int fs_solve_batch(fs_model* m, int32_t n, const float* cap_dev, const float* ta
   if (n < 0) return fail(FS_EINVAL, "n < 0");
   if (n == 0) return FS_OK;
   if (!cap_dev || !tail_dev || !out_dev) return fail(FS_EINVAL, "NULL device pointer");
-  int rc = order_after_upload(m, (cudaStream_t)cuda_stream);
+  int rc = flush_bounds(m, (cudaStream_t)cuda_stream);
   if (rc) return rc;
   FS_CUDA(launch_solve(m->set, n, cap_dev, tail_dev, out_dev, false, m->lc, (cudaStream_t)cuda_stream),
           "launch solve");
@@ -556,6 +585,8 @@ int fs_solve_batch(fs_model* m, int32_t n, const float* cap_dev, const float* ta
 int fs_solve_bounds(fs_model* m, fs_allocation* minus, fs_allocation* plus, float* gamma_t) {
   if (!m) return fail(FS_EINVAL, "model is NULL");
   cudaStream_t s = m->stream;
+  int rc0 = flush_bounds(m, s);
+  if (rc0) return rc0;
   FS_CUDA(launch_solve(m->set, 2, nullptr, nullptr, nullptr, true, m->lc, s), "launch solve");
   fs_allocation h[2];
   FS_CUDA(cudaMemcpyAsync(h, m->set.base, sizeof h, cudaMemcpyDeviceToHost, s), "read allocations");
@@ -578,7 +609,7 @@ int fs_reveal(fs_model* m, int32_t cell, float cap, float tail) {
   m->h_bounds[(size_t)TAIL_LO * cells + cell] = canon(tail);
   m->h_bounds[(size_t)TAIL_HI * cells + cell] = canon(tail);
   m->h_revealed[cell] = 1;
-  return upload_bounds(m);
+  return stage_bounds(m);
 }
 
 int fs_certificate(fs_model* m, float eps, int32_t* state, float* gamma_t) {

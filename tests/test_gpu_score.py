@@ -261,3 +261,39 @@ def test_watchdog_times_out_cleanly(fsb, cuda):
     w = workloads.make_workload(0)
     with load_model(fsb, w) as m:
         fsb.fs_score_candidates(m, w.candidates, 4, 8, 0)
+
+
+def test_staged_bounds_reach_every_later_call(fsb, cuda, oracle_lib, qn):
+    """fs_update_bounds only stages: a synchronous score reads the staged bounds,
+    every device-side call after it (asynchronous scoring on another stream,
+    bounds solves) sees them too."""
+    torch = cuda
+    w1 = stressed(0, 3.0, S=64)
+    w2 = stressed(0, 2.0, S=64, cap_lo=(workloads.make_workload(0).cap_lo * 0.9).astype(np.float32))
+    n = len(w1.candidates)
+    cand = torch.from_numpy(w1.candidates).cuda()
+    side = torch.cuda.Stream()
+
+    def score_async(m):
+        gap = torch.zeros(n, dtype=torch.float64, device="cuda")
+        sums = torch.zeros((n, w1.O), dtype=torch.int64, device="cuda")
+        with torch.cuda.stream(side):
+            fsb.fs_score_candidates_async(m, cand, w1.O, w1.S, w1.seed, gap_dev=gap, sum_eo_dev=sums, stream=side)
+        fsb.fs_check(m, side)
+        return sums.cpu().numpy()
+
+    ref1 = oracle_lib.score(w1, qn)
+    w2s = dataclasses.replace(w2, demand=w1.demand)
+    ref2 = oracle_lib.score(w2s, qn)
+    with load_model(fsb, w1) as m:
+        fsb.fs_update_bounds(m, w2.cap_lo, w2.cap_hi, w2.tail_lo, w2.tail_hi)
+        assert np.array_equal(score_async(m), ref2.sum_eo)           # straight after the update
+        fsb.fs_update_bounds(m, w1.cap_lo, w1.cap_hi, w1.tail_lo, w1.tail_hi)
+        r = fsb.fs_score_candidates(m, w1.candidates, w1.O, w1.S, w1.seed)  # reads the staging
+        assert np.array_equal(r.sum_eo, ref1.sum_eo)
+        assert np.array_equal(score_async(m), ref1.sum_eo)           # the device copy followed
+        fsb.fs_update_bounds(m, w2.cap_lo, w2.cap_hi, w2.tail_lo, w2.tail_hi)
+        gm, gp, g = fsb.fs_solve_bounds(m)
+        assert g == oracle_lib.base_gap(oracle_lib.Problem.of(w2s), w2.cap_lo, w2.cap_hi, w2.tail_lo, w2.tail_hi)[2]
+        r = fsb.fs_score_candidates(m, w1.candidates, w1.O, w1.S, w1.seed)
+        assert np.array_equal(r.sum_eo, ref2.sum_eo)
