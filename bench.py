@@ -451,7 +451,7 @@ def main(argv=None):
             "candidate_scores_per_s": len(w.candidates) * args.steps * world / (total_ms / 1000.0),
             "scenarios_per_s": scen_all / (total_ms / 1000.0),
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                    "api": "fs_update_bounds + fs_score_candidates (pinned host buffers)",
+                    "api": "fs_update_bounds + fs_score_candidates (pinned host buffers; inputs and results cross through mapped page-locked memory the kernels read and write)",
                     "best": int(res.best)},
             "gpu_launches": int(launches), "roofline": roofline, "clocks": clk,
             "cpu_baseline": cpu, "other_workloads": others}
