@@ -38,8 +38,8 @@ METRIC = "scenario allocation-solves/s"
 UNIT = "allocation-solves/s"
 ISSUE_PER_SM_CLK = 4 * 32  # 4 schedulers x 32 lanes, one warp instruction each per clock
 
-# Algorithmic thread-operations per scenario of the Monte-Carlo kernel: the
-# operations every scenario of the parametric re-solve performs.
+# Algorithmic thread-operations of the Monte-Carlo kernel. Plain path, per
+# scenario (the parametric re-solve):
 #   a quarter of one Philox4x32-10 call (10 rounds x (2 wide multiplies +
 #   2 three-input XORs), four samples per call)                          10
 #   capacity position (high multiply), its address, the lookup            3
@@ -48,9 +48,33 @@ ISSUE_PER_SM_CLK = 4 * 32  # 4 schedulers x 32 lanes, one warp instruction each 
 #   two table searches: loop test, address, read of the reached threshold 6
 #   Gamma' = t*(A+') - t*(A-')                                             1
 #   exact fixed-point accumulation of rint(Gamma' 2^40)                   7
-# Search probes beyond the first (3 each) and row-term fulfilments (where a
-# reachable threshold leaves row r a replica) are not counted: a lower bound.
+# Table path (a segment's W + 1 values of rint(Gamma' 2^40) tabulated once):
+# per scenario the Philox share (10), capacity position (1), gate mask,
+# compare and index select (3), the entry's load (1) and its two field sums
+# (2) = 17; per table entry the two patched capacities (2), two table searches
+# (6), Gamma' (1), the fixed-point conversion (5) and the store (1) = 15.
+# Search probes beyond the first (3 each) and row-term fulfilments are not
+# counted: lower bounds.
 OPS_PER_SCENARIO = 32
+OPS_PER_SCENARIO_TABLE = 17
+OPS_PER_TABLE_ENTRY = 15
+Q_TABLE = 4096  # quantile table size of the built-in triangular table
+
+
+def table_path(O: int, S: int) -> bool:
+    """Whether a launch of O outcomes x S samples takes the table path: the
+    scorer's rule (W = Q/O entries at most 4096, and 3 (W + 1) at most twice
+    the smaller of S and a minimum chunk of 2048 samples)."""
+    W = Q_TABLE // O
+    return W <= 4096 and 3 * (W + 1) <= 2 * min(S, 2048)
+
+
+def algorithmic_ops(w) -> float:
+    """Algorithmic thread-operations of one Monte-Carlo launch over workload w."""
+    if table_path(w.O, w.S):
+        W = Q_TABLE // w.O
+        return float(len(w.candidates)) * w.O * (w.S * OPS_PER_SCENARIO_TABLE + (W + 1) * OPS_PER_TABLE_ENTRY)
+    return float(OPS_PER_SCENARIO) * w.scenarios
 
 # ncu summaries with the DRAM bytes of one k_score launch, per workload; used
 # for roofline.traffic only while the scorer source is the one profiled.
@@ -248,7 +272,7 @@ def other_workload(idx: int, steps: int, warmup: int, alu_peak: float, stream_id
     fsb.fs_check(m, stream)
     fsb.fs_free_model(m)
     kern_s = kernel_ms / 1000.0 / max(kernel_n, 1)
-    achieved = OPS_PER_SCENARIO * w.scenarios / kern_s
+    achieved = algorithmic_ops(w) / kern_s
     return {"workload": w.name, "ms_per_step": step_ms, "scenarios_per_s": w.scenarios / (step_ms / 1000.0),
             "allocation_solves_per_s": 2.0 * w.scenarios / (step_ms / 1000.0),
             "candidate_scores_per_s": n / (step_ms / 1000.0),
@@ -427,14 +451,15 @@ def main(argv=None):
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     alu_peak = sms * ISSUE_PER_SM_CLK * sm_max * 1e6  # thread-ops/s at the maximum SM clock
     kern_s = kernel_ms / 1000.0 / max(kernel_n, 1)
-    achieved = OPS_PER_SCENARIO * w.scenarios / kern_s if kernel_n else None
+    achieved = algorithmic_ops(w) / kern_s if kernel_n else None
     roofline = {"bound": "alu", "kernel": "k_score (Monte-Carlo sampler + parametric re-solve)",
                 "achieved": achieved / 1e12 if achieved else None,
                 "peak": alu_peak / 1e12, "unit": "Tops/s (32-bit thread operations)",
                 "frac": (achieved / alu_peak) if achieved else None,
                 "traffic": _profiled_traffic(args.workload), "traffic_unit": "DRAM bytes per launch (ncu)",
                 "algorithmic_bytes": 0, "kernel_ms_per_launch": kern_s * 1000.0,
-                "ops_per_scenario": OPS_PER_SCENARIO,
+                "ops_per_scenario": algorithmic_ops(w) / w.scenarios,
+                "path": "table" if table_path(w.O, w.S) else "plain",
                 "peak_basis": f"{sms} SMs x 4 issue slots x 32 lanes x {sm_max:.0f} MHz (max SM clock)",
                 "kernel_share_of_step": (kernel_ms / max(sum(step_ms), 1e-9)) if kernel_n else None}
     cpu = None

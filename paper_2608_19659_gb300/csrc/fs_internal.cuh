@@ -350,11 +350,11 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
 
 // Per-model launch state: whether floors are set, and the launch shapes
 // (filled on first use) per kernel instance: [floors] for the solve and the
-// preparation, [dump][floors] for the scorer.
+// preparation, [path][floors] for the scorer (plain, dump, table).
 struct LaunchCache {
   int floors = 0;  // some class has a floor > 0: launch the kernel instances with floors
-  size_t solve_smem[2] = {0, 0}, prep_smem[2] = {0, 0}, score_smem[2][2] = {{0, 0}, {0, 0}};
-  int score_blocks_per_sm[2][2] = {{0, 0}, {0, 0}};
+  size_t solve_smem[2] = {0, 0}, prep_smem[2] = {0, 0}, score_smem[3][2] = {{0, 0}, {0, 0}, {0, 0}};
+  int score_blocks_per_sm[3][2] = {{0, 0}, {0, 0}, {0, 0}};
 };
 
 cudaError_t launch_qtable(float* qn, int Q, cudaStream_t s);

@@ -35,6 +35,8 @@
 // E[Gamma_{t+1} | e], the score and the argmax.
 #include <cuda_runtime.h>
 
+#include <algorithm>
+
 #include "fs_finalize.cuh"
 #include "fs_internal.cuh"
 
@@ -631,6 +633,82 @@ __device__ uint64_t run_piece_dump(const Set& set, const Plan& pl, int item, int
   return acc;
 }
 
+// Table path. Within a segment (candidate e, outcome o) a scenario's Gamma'
+// depends on its draw only through the capacity position k (which selects c_y
+// among the outcome's W mapped quantiles) and the tail gate (l_y <= L_i); with
+// the gate closed the row keeps Cexcl whatever k is. So the segment has at most
+// W + 1 values of rint(Gamma' 2^40): gtab[k] for an open gate at position k,
+// gtab[W] for a closed gate. The block evaluates them once per chunk (two t*
+// each, the same arithmetic as a scenario), after which a scenario costs its
+// share of the Philox call, one index and one shared-memory load. Each entry
+// holds the value's upper bits (>> 20) and lower 20 bits, summed separately.
+template <bool TS, int ROW, bool FL>
+__device__ __forceinline__ void build_gtab(uint2* gtab, int W, const float* win, const float* h0, const float* h1,
+                                           const float* kap0, const float* thx0, const float* mnx0,
+                                           const float* kap1, const float* thx1, const float* mnx1) {
+  const int st0 = __float_as_int(h0[H_STEP0]), st1 = __float_as_int(h1[H_STEP0]);
+  const float cx0 = h0[H_CX], cx1 = h1[H_CX];
+  const float lam = h0[H_LAM], rlam = h0[H_RLAM], dl = h0[H_DLT];
+  const float* capw = win + 4;
+  for (int k = threadIdx.x; k <= W; k += blockDim.x) {
+    const float cy = k < W ? capw[k] : 0.0f;  // a closed gate: the row keeps max(Cexcl, 0) = Cexcl
+    const float t0 = tstar_of<ROW, FL>(fmaxf(cx0, cy), kap0, thx0, mnx0, st0, lam, rlam, dl);
+    const float t1 = tstar_of<ROW, FL>(fmaxf(cx1, cy), kap1, thx1, mnx1, st1, lam, rlam, dl);
+    const uint64_t g = fixed40(__fsub_rn(t1, t0));
+    gtab[k] = make_uint2((uint32_t)(g >> 20), (uint32_t)g & 0xFFFFFu);
+  }
+}
+
+// Philox calls [q_lo, q_hi) of one segment on the table path: the sums of the
+// two fields of the drawn entries (each field below 2^21), flushed into a
+// 64-bit total every 256 calls so that the 32-bit sums cannot wrap. With at
+// most 32 values per thread nothing is flushed and a warp's field sums stay
+// below 2^32.
+struct GtabSum {
+  uint32_t h, l;   // the last at most 1024 values
+  uint64_t total;  // earlier values
+};
+
+__device__ __forceinline__ GtabSum sample_gtab(const Plan& pl, const PhiloxKeys& keys, int o, int cell, int q_lo,
+                                               int q_hi, const uint2* gtab, const float* win) {
+  const uint32_t ctr1 = (uint32_t)o, ctr2 = (uint32_t)cell, ctr3 = pl.round;
+  const uint32_t W = (uint32_t)pl.W;
+  const uint32_t kgs = (uint32_t)__float_as_int(win[0]) << pl.sh;
+  uint32_t gh = 0, glo = 0;
+  auto take = [&](uint32_t word) {
+    const uint32_t idx = (word & 0xFFFFu) < kgs ? __umulhi(word, W) : W;
+    const uint2 v = gtab[idx];
+    gh += v.x;
+    glo += v.y;
+  };
+  const int q_full = min(q_hi, pl.S >> 2);  // calls whose four samples all exist
+  const int step = (int)blockDim.x;
+  uint64_t total = 0;
+  int q = q_lo + (int)threadIdx.x;
+  while (q < q_full) {
+    const int q_end = min(q_full, q + 256 * step);
+    for (; q < q_end; q += step) {
+      const uint4 x = philox4x32_10(make_uint4((uint32_t)q, ctr1, ctr2, ctr3), keys);
+      take(x.x);
+      take(x.y);
+      take(x.z);
+      take(x.w);
+    }
+    if (q < q_full) {
+      total += ((uint64_t)gh << 20) + glo;
+      gh = glo = 0;
+    }
+  }
+  if (q < q_hi) {  // the segment's last call, serving S mod 4 samples
+    const uint4 x = philox4x32_10(make_uint4((uint32_t)q, ctr1, ctr2, ctr3), keys);
+    const int nv = pl.S - 4 * q;
+    take(x.x);
+    if (nv > 1) take(x.y);
+    if (nv > 2) take(x.z);
+  }
+  return GtabSum{gh, glo, total};
+}
+
 // Work decomposition of one k_score launch: segment = (item, outcome) with
 // pl.calls Philox calls; a chunk is up to `chunk` consecutive calls of one
 // segment, nch chunks per segment.
@@ -642,6 +720,9 @@ struct ScoreGrid {
   int tcopy;        // floats staged per table: header + 3 lcap_s
   int dyn;          // 1: chunks after the first two come from the counter; 0: chunk b + k gridDim
 };
+
+// Which scoring path a launch takes.
+enum : int { SCORE_PLAIN = 0, SCORE_DUMP = 1, SCORE_TABLE = 2 };
 
 // Thread 0: stage the data of segment seg (its outcome window and both
 // candidate tables, header plus lcap_s entries each) into dst, completing on bar.
@@ -668,7 +749,9 @@ __device__ __forceinline__ void stage_segment(const Set& set, const Plan& pl, co
 // change the result.
 // FL: some class is critical (the model has floors): row terms are gated by the
 // candidate class's floor (0, so always passed, for a class that is not).
-template <bool DUMP, bool FL>
+// GT: the table path (build_gtab), chosen by the host when a chunk's samples
+// outnumber a segment's W + 1 table entries; never with DUMP.
+template <bool DUMP, bool FL, bool GT>
 __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, Plan pl, const float* rec,
                                                          uint64_t* sums, unsigned char* dump, int dump_stride,
                                                          ScoreGrid sg) {
@@ -676,6 +759,7 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
   uint64_t* bar = reinterpret_cast<uint64_t*>(smraw);  // [2]
   float* stage0 = reinterpret_cast<float*>(smraw + 16);
   const int stage_floats = pl.Wp + 2 * sg.tcopy;
+  uint2* gtab = reinterpret_cast<uint2*>(smraw + 16 + (size_t)2 * stage_floats * 4);  // GT: [W + 1]
   // per stage: chunk index, its segment and its part (thread 0 divides once)
   __shared__ int s_chunk[2], s_seg[2], s_part[2];
   const Dims& d = set.d;  // kernel-parameter space: d.M[j] reads need no local copy
@@ -733,6 +817,51 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
     const int item = seg >> pl.logO, o = seg & (pl.O - 1);
     const int q_lo = part * sg.chunk;
     const int q_hi = min(q_lo + sg.chunk, pl.calls);
+    if constexpr (GT) {
+      const int cell = ok ? __float_as_int(h0[H_CELL]) : -1;
+      const bool use = cell >= 0 && cell < d.cells;  // a bad device-side id was flagged by k_prep
+      if (use) {
+        const int Lp0 = __float_as_int(h0[H_LPAD]), Lp1 = __float_as_int(h1[H_LPAD]);
+        const bool r0 = __float_as_int(h0[H_ROW]) != 0, r1 = __float_as_int(h1[H_ROW]) != 0;
+        const bool f0 = __float_as_int(h0[H_FAST]) != 0, f1 = __float_as_int(h1[H_FAST]) != 0;
+        const int row = (!r0 && !r1) ? 0 : ((!r0 || f0) && (!r1 || f1)) ? 1 : 2;
+#define FS_BUILD(TSV, ROWV, FLV) \
+  build_gtab<TSV, ROWV, FLV>(gtab, pl.W, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, k1 + Lp1, k1 + 2 * Lp1)
+#define FS_BUILDS(TSV)                       \
+  if (row == 0) FS_BUILD(TSV, 0, false);     \
+  else if (row == 1) FS_BUILD(TSV, 1, FL);   \
+  else FS_BUILD(TSV, 2, FL);
+        if (Lp0 <= sg.lcap_s && Lp1 <= sg.lcap_s) {
+          const float* k0 = h0 + kTableHeader;
+          const float* k1 = h1 + kTableHeader;
+          FS_BUILDS(true)
+        } else {
+          const float* k0 = rec + (size_t)item * pl.item_floats + kTableHeader;
+          const float* k1 = k0 + d.slot_floats;
+          FS_BUILDS(false)
+        }
+#undef FS_BUILDS
+#undef FS_BUILD
+        const int p = __float_as_int(h0[H_P]);
+        if (p != keys_p) {
+          keys = philox_keys(pl.key0, pl.key1 ^ (pl.stream_base + (uint32_t)p));
+          keys_p = p;
+        }
+      }
+      __syncthreads();  // the table is complete
+      GtabSum gs{0u, 0u, 0ull};
+      if (use) gs = sample_gtab(pl, keys, o, cell, q_lo, q_hi, gtab, stg);
+      uint64_t v;
+      if (small) {  // at most 32 values per thread: each field's warp sum fits in 32 bits
+        const uint32_t H = __reduce_add_sync(0xffffffffu, gs.h);
+        const uint32_t Lo = __reduce_add_sync(0xffffffffu, gs.l);
+        v = ((uint64_t)H << 20) + (uint64_t)Lo;
+      } else {
+        v = gs.total + ((uint64_t)gs.h << 20) + gs.l;
+        for (int off = 16; off; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
+      }
+      if (lane == 0 && v) atomicAdd(reinterpret_cast<unsigned long long*>(&sums[(size_t)seg]), (unsigned long long)v);
+    } else {
     PieceSum ps{Acc40(), 0ull};
     uint64_t acc_dump = 0;
     if (ok) {
@@ -783,6 +912,7 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
       for (int off = 16; off; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
       if (lane == 0 && v) atomicAdd(reinterpret_cast<unsigned long long*>(&sums[(size_t)seg]), (unsigned long long)v);
     }
+    }
     // stage st is free for the copies issued next iteration
     if (__syncthreads_or(!ok)) {
       if (tid == 0) atomicOr(set.status, ST_TIMEOUT);
@@ -832,10 +962,17 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
   ScoreGrid sg{};
   sg.lcap_s = score_lcap(set.d);
   sg.tcopy = kTableHeader + 3 * sg.lcap_s;
-  const size_t smem = 16 + 2 * (size_t)(pl.Wp + 2 * sg.tcopy) * 4;
-  const int v = dump ? 1 : 0, fl = lc.floors ? 1 : 0;
-  auto kern = dump ? (fl ? k_score<true, true> : k_score<true, false>)
-                   : (fl ? k_score<false, true> : k_score<false, false>);
+  // the table path when a segment's W + 1 entries cost well under a chunk's
+  // samples (an entry costs about one scenario of the plain path, a scenario
+  // about a third of one there); the smallest chunk holds 2 calls per thread
+  const long long chunk_min = std::min<long long>(pl.S, 2LL * 4 * kScoreThreads);
+  const bool table = !dump && pl.W <= 4096 && 3LL * (pl.W + 1) <= 2 * chunk_min;
+  const size_t stages = 16 + 2 * (size_t)(pl.Wp + 2 * sg.tcopy) * 4;
+  const size_t smem = stages + (table ? ((size_t)8 * (pl.W + 1) + 15) / 16 * 16 : 0);
+  const int v = dump ? SCORE_DUMP : table ? SCORE_TABLE : SCORE_PLAIN, fl = lc.floors ? 1 : 0;
+  auto kern = dump ? (fl ? k_score<true, true, false> : k_score<true, false, false>)
+          : table ? (fl ? k_score<false, true, true> : k_score<false, false, true>)
+                  : (fl ? k_score<false, true, false> : k_score<false, false, false>);
   if (smem != lc.score_smem[v][fl]) {
     int per_sm = 0;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

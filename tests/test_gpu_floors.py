@@ -242,3 +242,18 @@ def test_replay_with_floors(fsb, cuda, oracle_lib, qn):
     assert np.all(res.state == 2) and np.all(res.rounds == 0)
     ref = oracle_lib.replay_stream(dataclasses.replace(rp, base=bad), 0, qn, seed=11, S=8, max_rounds=5)
     assert ref.state == 2 and ref.rounds == 0
+
+
+def test_table_path_with_floors(fsb, cuda, oracle_lib, qn):
+    """Floors on the table path (2048 samples per outcome): the segment tables
+    gate row terms by the candidate class's floor."""
+    w = workloads.make_workload(1)
+    p = oracle_lib.Problem.of(w)
+    am, ap, _ = oracle_lib.base_gap(p, w.cap_lo, w.cap_hi, w.tail_lo, w.tail_hi)
+    d = np.float32(0.5 * (am.t_star + ap.t_star))
+    w = dataclasses.replace(w, floor=np.array([d, 0.0], np.float32), S=2048,
+                            candidates=w.candidates[::8].copy())
+    with load_model(fsb, w) as m:
+        r = fsb.fs_score_candidates(m, w.candidates, w.O, w.S, w.seed)
+    ref = oracle_lib.score(w, qn)
+    assert np.array_equal(r.sum_eo, ref.sum_eo) and r.best == ref.best

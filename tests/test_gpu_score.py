@@ -297,3 +297,16 @@ def test_staged_bounds_reach_every_later_call(fsb, cuda, oracle_lib, qn):
         assert g == oracle_lib.base_gap(oracle_lib.Problem.of(w2s), w2.cap_lo, w2.cap_hi, w2.tail_lo, w2.tail_hi)[2]
         r = fsb.fs_score_candidates(m, w1.candidates, w1.O, w1.S, w1.seed)
         assert np.array_equal(r.sum_eo, ref2.sum_eo)
+
+
+def test_table_path_with_long_tables(fsb, cuda, oracle_lib, qn):
+    """The table path on the 8-class workload at twice its demand, where some
+    candidates' contested ranges exceed the 256 entries staged in shared memory,
+    so their segment tables are built from global memory."""
+    w = stressed(3, 2.0, O=16, S=512)
+    probe = stressed(3, 2.0, O=2, S=8)
+    ref0 = oracle_lib.score(probe, qn)
+    pos = np.nonzero(ref0.score > 0)[0]
+    cand = probe.candidates[pos[:: max(1, len(pos) // 3)][:3]]
+    r = run(fsb, w, cand=cand)
+    assert_same(r, oracle_lib.score(w, qn, candidates=cand), cand=cand)

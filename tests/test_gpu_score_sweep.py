@@ -88,3 +88,20 @@ def test_extreme_sizes(fsb, cuda, oracle_lib, K, B, G, n_cand):
     qn = oracle_lib.triangular_table(4096)
     r, ref = _score_both(fsb, oracle_lib, w, qn, cand, 2, 16, 77, 3, 1)
     _assert_same(r, ref)
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_table_path_random_problems(fsb, cuda, oracle_lib, seed):
+    """Enough samples per outcome that the scorer tabulates each segment's
+    values of rint(Gamma' 2^40) (W = 4096 / O entries) and only draws indices;
+    a subset of candidates, sums compared bit for bit."""
+    rng = np.random.default_rng(1700 + seed)
+    K, B, G = int(rng.integers(1, 7)), int(rng.integers(1, 7)), int(rng.integers(2, 49))
+    w = _contested(oracle_lib, workloads.random_small(rng, K, B, G))
+    O = int(rng.choice([4, 8, 16]))
+    S = int(rng.integers(800, 2600))
+    cand = np.sort(rng.choice(w.cells, size=min(6, w.cells), replace=False)).astype(np.int32)
+    s, sid, rnd = int(rng.integers(0, 2**63)), int(rng.integers(0, 100)), int(rng.integers(0, 20))
+    qn = oracle_lib.triangular_table(4096)
+    r, ref = _score_both(fsb, oracle_lib, w, qn, cand, O, S, s, sid, rnd)
+    _assert_same(r, ref)
