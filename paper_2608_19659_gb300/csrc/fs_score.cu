@@ -670,10 +670,9 @@ struct GtabSum {
 };
 
 __device__ __forceinline__ GtabSum sample_gtab(const Plan& pl, const PhiloxKeys& keys, int o, int cell, int q_lo,
-                                               int q_hi, const uint2* gtab, const float* win) {
+                                               int q_hi, const uint2* gtab, uint32_t kgs) {
   const uint32_t ctr1 = (uint32_t)o, ctr2 = (uint32_t)cell, ctr3 = pl.round;
   const uint32_t W = (uint32_t)pl.W;
-  const uint32_t kgs = (uint32_t)__float_as_int(win[0]) << pl.sh;
   uint32_t gh = 0, glo = 0;
   auto take = [&](uint32_t word) {
     const uint32_t idx = (word & 0xFFFFu) < kgs ? __umulhi(word, W) : W;
@@ -759,7 +758,8 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
   uint64_t* bar = reinterpret_cast<uint64_t*>(smraw);  // [2]
   float* stage0 = reinterpret_cast<float*>(smraw + 16);
   const int stage_floats = pl.Wp + 2 * sg.tcopy;
-  uint2* gtab = reinterpret_cast<uint2*>(smraw + 16 + (size_t)2 * stage_floats * 4);  // GT: [W + 1]
+  // GT: two tables of W + 1 entries, used by alternate chunks
+  uint2* gtab2 = reinterpret_cast<uint2*>(smraw + 16 + (size_t)2 * stage_floats * 4);
   // per stage: chunk index, its segment and its part (thread 0 divides once)
   __shared__ int s_chunk[2], s_seg[2], s_part[2];
   const Dims& d = set.d;  // kernel-parameter space: d.M[j] reads need no local copy
@@ -782,8 +782,10 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
     stage_segment(set, pl, rec, s_seg[0], stage0, &bar[0], sg.tcopy);
     next = (int)blockIdx.x + g;  // may pass sg.total: then the block stops after one chunk
   }
-  // 32-bit warp sums are exact while a thread holds at most 32 values
+  // 32-bit warp sums are exact while a thread holds at most 32 values (the
+  // table path's fields are below 2^21: at most 64 values)
   const bool small = sg.chunk <= 8 * (int)blockDim.x;
+  const bool small_gt = sg.chunk <= 16 * (int)blockDim.x;
   PhiloxKeys keys;
   int keys_p = -1;  // problem whose round keys are in `keys`
 
@@ -818,8 +820,14 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
     const int q_lo = part * sg.chunk;
     const int q_hi = min(q_lo + sg.chunk, pl.calls);
     if constexpr (GT) {
+      // One barrier a chunk: every thread's reads of stage st (table build and
+      // the gate position) come before it, so thread 0 may refill the stage
+      // next iteration, and the next chunk builds the other table while a late
+      // thread may still draw from this one.
+      uint2* gtab = gtab2 + (size_t)(j & 1) * (pl.W + 1);
       const int cell = ok ? __float_as_int(h0[H_CELL]) : -1;
       const bool use = cell >= 0 && cell < d.cells;  // a bad device-side id was flagged by k_prep
+      const uint32_t kgs = use ? (uint32_t)__float_as_int(stg[0]) << pl.sh : 0u;
       if (use) {
         const int Lp0 = __float_as_int(h0[H_LPAD]), Lp1 = __float_as_int(h1[H_LPAD]);
         const bool r0 = __float_as_int(h0[H_ROW]) != 0, r1 = __float_as_int(h1[H_ROW]) != 0;
@@ -848,11 +856,16 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
           keys_p = p;
         }
       }
-      __syncthreads();  // the table is complete
+      if (__syncthreads_or(!ok)) {  // the table is complete; or some wait gave up
+        if (tid == 0) atomicOr(set.status, ST_TIMEOUT);
+        if (!ok) mbar_wait(&bar[st], (uint32_t)((j >> 1) & 1), kWaitLimitNs);
+        if (s_chunk[st ^ 1] < sg.total) mbar_wait(&bar[st ^ 1], (uint32_t)(((j + 1) >> 1) & 1), kWaitLimitNs);
+        return;
+      }
       GtabSum gs{0u, 0u, 0ull};
-      if (use) gs = sample_gtab(pl, keys, o, cell, q_lo, q_hi, gtab, stg);
+      if (use) gs = sample_gtab(pl, keys, o, cell, q_lo, q_hi, gtab, kgs);
       uint64_t v;
-      if (small) {  // at most 32 values per thread: each field's warp sum fits in 32 bits
+      if (small_gt) {  // at most 64 values per thread: each field's warp sum fits in 32 bits
         const uint32_t H = __reduce_add_sync(0xffffffffu, gs.h);
         const uint32_t Lo = __reduce_add_sync(0xffffffffu, gs.l);
         v = ((uint64_t)H << 20) + (uint64_t)Lo;
@@ -861,6 +874,7 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
         for (int off = 16; off; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
       }
       if (lane == 0 && v) atomicAdd(reinterpret_cast<unsigned long long*>(&sums[(size_t)seg]), (unsigned long long)v);
+      continue;
     } else {
     PieceSum ps{Acc40(), 0ull};
     uint64_t acc_dump = 0;
@@ -968,7 +982,7 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
   const long long chunk_min = std::min<long long>(pl.S, 2LL * 4 * kScoreThreads);
   const bool table = !dump && pl.W <= 4096 && 3LL * (pl.W + 1) <= 2 * chunk_min;
   const size_t stages = 16 + 2 * (size_t)(pl.Wp + 2 * sg.tcopy) * 4;
-  const size_t smem = stages + (table ? ((size_t)8 * (pl.W + 1) + 15) / 16 * 16 : 0);
+  const size_t smem = stages + (table ? ((size_t)16 * (pl.W + 1) + 15) / 16 * 16 : 0);
   const int v = dump ? SCORE_DUMP : table ? SCORE_TABLE : SCORE_PLAIN, fl = lc.floors ? 1 : 0;
   auto kern = dump ? (fl ? k_score<true, true, false> : k_score<true, false, false>)
           : table ? (fl ? k_score<false, true, true> : k_score<false, false, true>)
@@ -985,12 +999,13 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
   // the work allows, so that the counter can even out the segments' unequal
   // costs; at least 2 (a chunk's set-up is then paid for eight samples per
   // thread, measured faster on small launches) and at most 8 calls per
-  // thread, and no more than a segment holds.
+  // thread (16 on the table path, whose chunks also build a table), and no
+  // more than a segment holds.
   const long long resident = (long long)lc.score_blocks_per_sm[v][fl] * sm_count;
   const long long total_calls = (long long)it.n * pl.O * pl.calls;
   long long U = total_calls / ((long long)kScoreThreads * resident * 8);
   const long long u_seg = ((long long)pl.calls + kScoreThreads - 1) / kScoreThreads;
-  if (U > 8) U = 8;
+  if (U > (table ? 16 : 8)) U = table ? 16 : 8;
   if (U < 2) U = 2;
   if (U > u_seg) U = u_seg;
   // chunk indices are 32-bit: widen the chunks until they fit (one chunk per
