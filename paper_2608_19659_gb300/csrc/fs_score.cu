@@ -1008,6 +1008,23 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
   if (U > (table ? 16 : 8)) U = table ? 16 : 8;
   if (U < 2) U = 2;
   if (U > u_seg) U = u_seg;
+  if (table) {
+    // every chunk builds its segment's table first: pick the chunk length that
+    // minimises rounds of chunks per block x (build + draws), in units of about
+    // one thread-instruction (an entry ~60 per thread share, a call's four draws ~72)
+    const long long n_seg = (long long)it.n * pl.O;
+    const long long build = ((pl.W + 1 + kScoreThreads - 1) / kScoreThreads) * 60;
+    long long best = -1;
+    for (long long u = 2; u <= std::min<long long>(16, u_seg); ++u) {
+      const long long nch_u = (pl.calls + kScoreThreads * u - 1) / (kScoreThreads * u);
+      const long long rounds = (n_seg * nch_u + resident - 1) / resident;
+      const long long cost = rounds * (build + 72 * u);
+      if (best < 0 || cost < best) {
+        best = cost;
+        U = u;
+      }
+    }
+  }
   // chunk indices are 32-bit: widen the chunks until they fit (one chunk per
   // segment gives n O <= 2^30 chunks, which the entry points guarantee)
   long long nch = (pl.calls + kScoreThreads * U - 1) / (kScoreThreads * U);
