@@ -314,7 +314,7 @@ int run_score(fs_model* m, const Set& set, const fs_samples* smp, const int32_t*
   }
   const bool phases = timed && m->timing == 2;
   if (phases) FS_CUDA(cudaEventRecord(ev[0], s), "record timing event");
-  FS_CUDA(launch_solve(set, 2, nullptr, nullptr, nullptr, true, m->lc, s), "launch solve");
+  FS_CUDA(launch_solve(set, 2, nullptr, nullptr, nullptr, true, m->lc, s, true), "launch solve");
   if (phases) FS_CUDA(cudaEventRecord(ev[1], s), "record timing event");
   FS_CUDA(launch_prep(set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, true, m->lc, s), "launch prep");
   if (timed) FS_CUDA(cudaEventRecord(ev[2], s), "record timing event");

@@ -361,8 +361,12 @@ cudaError_t launch_qtable(float* qn, int Q, cudaStream_t s);
 // Base or explicit realisations: realisation r of `n` reads cap/tail either
 // from the problem set's bounds (explicit == nullptr: r = 2 p + sigma) or from
 // cap_x / tail_x [n][cells].
+// tstar_only: the allocations' per-class choice is not needed (the scoring
+// call reads only t* and the thresholds); total_gpus is then -1 unless the
+// model has floors.
 cudaError_t launch_solve(const Set& set, int n, const float* cap_x, const float* tail_x,
-                         fs_allocation* out, bool write_theta, LaunchCache& lc, cudaStream_t s);
+                         fs_allocation* out, bool write_theta, LaunchCache& lc, cudaStream_t s,
+                         bool tstar_only = false);
 // early: the candidate ids and bounds were complete before the preceding
 // kernel started, so the bounds-only work may run before the PDL wait.
 cudaError_t launch_prep(const Set& set, const Items& it, const Plan& pl, float* tables,

@@ -81,7 +81,11 @@ __device__ __forceinline__ int group_total_cost(float t, const float* sC, const 
 template <bool FL>
 __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, const float* cap_x,
                                                          const float* tail_x, fs_allocation* out_x,
-                                                         int write_theta) {
+                                                         int mode) {
+  const bool write_theta = (mode & 1) != 0;
+  // the per-class choice at t* (step 4); a scoring call needs only t* and the
+  // thresholds, and without floors skips it
+  const bool choice = FL || (mode & 2) == 0;
   extern __shared__ __align__(16) unsigned char smraw[];
   const Dims& d = set.d;  // kernel-parameter space: d.M[j] reads need no local copy
   const int r = blockIdx.x;
@@ -286,63 +290,65 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   const int kstar = lo;
   const float tstar = kstar >= 0 ? sTheta[kstar] : 0.0f;
 
-  // 4. choice at t*: every row's cheapest cover in parallel (thread = row), then
-  // per class the cheapest row over its four TP lanes, lower TP on ties; the
-  // same for the floor of a critical class, summed into sMisc[5] (sMisc[6]:
-  // some critical class cannot reach its floor)
-  {
-    const int rho = tid;  // K4 <= 256 = blockDim
-    int key = 0x7fffffff, keyf = 0x7fffffff;
-    if (rho < d.K4) {
-      const float dl = FL ? sDl[rho >> 2] : 0.0f;
-      if (tstar > 0.0f) {
-        const int n = min_replicas(FL ? fmaxf(tstar, dl) : tstar, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[rho & 3]);
-        if (n) key = ((n << (rho & 3)) << 2) | (rho & 3);
+  if (choice) {
+    // 4. choice at t*: every row's cheapest cover in parallel (thread = row), then
+    // per class the cheapest row over its four TP lanes, lower TP on ties; the
+    // same for the floor of a critical class, summed into sMisc[5] (sMisc[6]:
+    // some critical class cannot reach its floor)
+    {
+      const int rho = tid;  // K4 <= 256 = blockDim
+      int key = 0x7fffffff, keyf = 0x7fffffff;
+      if (rho < d.K4) {
+        const float dl = FL ? sDl[rho >> 2] : 0.0f;
+        if (tstar > 0.0f) {
+          const int n = min_replicas(FL ? fmaxf(tstar, dl) : tstar, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[rho & 3]);
+          if (n) key = ((n << (rho & 3)) << 2) | (rho & 3);
+        }
+        if (FL && dl > 0.0f) {
+          const int n = min_replicas(dl, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[rho & 3]);
+          if (n) keyf = ((n << (rho & 3)) << 2) | (rho & 3);
+        }
       }
-      if (FL && dl > 0.0f) {
-        const int n = min_replicas(dl, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[rho & 3]);
-        if (n) keyf = ((n << (rho & 3)) << 2) | (rho & 3);
+      key = min(key, __shfl_xor_sync(0xffffffffu, key, 1));
+      key = min(key, __shfl_xor_sync(0xffffffffu, key, 2));
+      const int i = tid >> 2;
+      if constexpr (FL) {
+        keyf = min(keyf, __shfl_xor_sync(0xffffffffu, keyf, 1));
+        keyf = min(keyf, __shfl_xor_sync(0xffffffffu, keyf, 2));
+        const bool critical = (tid & 3) == 0 && i < d.K && sDl[i] > 0.0f;
+        if (critical) {
+          if (keyf == 0x7fffffff) atomicOr(&sMisc[6], 1);
+          else atomicAdd(&sMisc[5], keyf >> 2);
+        }
+        __syncthreads();
+        const bool met = sMisc[6] == 0 && sMisc[5] <= d.G;
+        if (tstar <= 0.0f) key = (critical && met) ? keyf : 0x7fffffff;  // tier 1 alone
+      }
+      if ((tid & 3) == 0) {
+        int8_t tp = 0;
+        int16_t bin = -1, reps = 0;
+        float f = 0.0f;
+        if (i < d.K && key != 0x7fffffff) {
+          const int bj = key & 3, cost_i = key >> 2, bn = cost_i >> bj;
+          tp = (int8_t)(1 << bj);
+          bin = (int16_t)sB[4 * i + bj];
+          reps = (int16_t)bn;
+          f = fulfil_r((float)bn, sC[4 * i + bj], sLam[i], sRl[i]);
+          atomicAdd(&sMisc[4], cost_i);
+        }
+        out->tp[i] = tp;
+        out->bin[i] = bin;
+        out->replicas[i] = reps;
+        out->fulfil[i] = f;
       }
     }
-    key = min(key, __shfl_xor_sync(0xffffffffu, key, 1));
-    key = min(key, __shfl_xor_sync(0xffffffffu, key, 2));
-    const int i = tid >> 2;
-    if constexpr (FL) {
-      keyf = min(keyf, __shfl_xor_sync(0xffffffffu, keyf, 1));
-      keyf = min(keyf, __shfl_xor_sync(0xffffffffu, keyf, 2));
-      const bool critical = (tid & 3) == 0 && i < d.K && sDl[i] > 0.0f;
-      if (critical) {
-        if (keyf == 0x7fffffff) atomicOr(&sMisc[6], 1);
-        else atomicAdd(&sMisc[5], keyf >> 2);
-      }
-      __syncthreads();
-      const bool met = sMisc[6] == 0 && sMisc[5] <= d.G;
-      if (tstar <= 0.0f) key = (critical && met) ? keyf : 0x7fffffff;  // tier 1 alone
-    }
-    if ((tid & 3) == 0) {
-      int8_t tp = 0;
-      int16_t bin = -1, reps = 0;
-      float f = 0.0f;
-      if (i < d.K && key != 0x7fffffff) {
-        const int bj = key & 3, cost_i = key >> 2, bn = cost_i >> bj;
-        tp = (int8_t)(1 << bj);
-        bin = (int16_t)sB[4 * i + bj];
-        reps = (int16_t)bn;
-        f = fulfil_r((float)bn, sC[4 * i + bj], sLam[i], sRl[i]);
-        atomicAdd(&sMisc[4], cost_i);
-      }
-      out->tp[i] = tp;
-      out->bin[i] = bin;
-      out->replicas[i] = reps;
-      out->fulfil[i] = f;
-    }
+    __syncthreads();
   }
-  __syncthreads();
   if (tid == 0) {
     out->t_star = tstar;
     // (with t* = 0 and no floors the sum is 0 anyway; the unconditional read
     // measured 1.5 us slower on a 28 us scoring call whose next kernel overlaps this one)
-    out->total_gpus = (FL || tstar > 0.0f) ? sMisc[4] : 0;
+    out->total_gpus = !choice ? -1 : (FL || tstar > 0.0f) ? sMisc[4] : 0;  // -1: not computed
     out->has_option_mask = (uint64_t)(uint32_t)sMisc[2] | ((uint64_t)(uint32_t)sMisc[3] << 32);
     out->ok = tstar > 0.0f ? 1 : 0;
     out->floors_met = (!FL || (sMisc[6] == 0 && sMisc[5] <= d.G)) ? 1 : 0;
@@ -389,7 +395,7 @@ cudaError_t launch_qtable(float* qn, int Q, cudaStream_t s) {
 }
 
 cudaError_t launch_solve(const Set& set, int n, const float* cap_x, const float* tail_x,
-                         fs_allocation* out, bool write_theta, LaunchCache& lc, cudaStream_t s) {
+                         fs_allocation* out, bool write_theta, LaunchCache& lc, cudaStream_t s, bool tstar_only) {
   if (n <= 0) return cudaSuccess;
   const size_t smem = solve_smem_bytes(set.d);
   const int fl = lc.floors ? 1 : 0;
@@ -400,7 +406,7 @@ cudaError_t launch_solve(const Set& set, int n, const float* cap_x, const float*
     lc.solve_smem[fl] = smem;
   }
   note_launch();
-  kern<<<n, kSolveThreads, smem, s>>>(set, n, cap_x, tail_x, out, write_theta ? 1 : 0);
+  kern<<<n, kSolveThreads, smem, s>>>(set, n, cap_x, tail_x, out, (write_theta ? 1 : 0) | (tstar_only ? 2 : 0));
   return cudaGetLastError();
 }
 

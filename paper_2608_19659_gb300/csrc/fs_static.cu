@@ -195,7 +195,7 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
   e = cudaMemsetAsync(set.status, 0, 4, s);  // the array keeps the last call's status word
   if (e == cudaSuccess && !quantile_dev) e = launch_qtable(const_cast<float*>(set.qn), Q, s);
-  if (e == cudaSuccess) e = launch_solve(set, 2, nullptr, nullptr, nullptr, true, *lc, s);
+  if (e == cudaSuccess) e = launch_solve(set, 2, nullptr, nullptr, nullptr, true, *lc, s, true);
   if (e == cudaSuccess) e = launch_prep(set, it, pl, reinterpret_cast<float*>(base + o_tab),
                                         reinterpret_cast<uint64_t*>(base + o_sums), true, *lc, s);
   if (e == cudaSuccess)
