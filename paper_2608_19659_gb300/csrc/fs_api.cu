@@ -285,7 +285,8 @@ int ensure_items(fs_model* m, int n, int O) {
   const int W = m->d.Q / O, Wp = 4 + ((W + 3) & ~3);
   const size_t item_floats = 2 * (size_t)m->d.slot_floats + (size_t)O * Wp;
   if ((rc = m->tables.ensure((size_t)std::max(n, 1) * item_floats * 4, "candidate records"))) return rc;
-  if ((rc = m->sums.ensure((size_t)std::max(n, 1) * O * 8, "sums"))) return rc;
+  // sums, then the split reduction's scratch (2 words per block)
+  if ((rc = m->sums.ensure((size_t)std::max(n, 1) * O * 8 + 16 * (size_t)kFinalizeMaxBlocks, "sums"))) return rc;
   if ((rc = m->outs.ensure((size_t)std::max(n, 1) * 16 + 64, "outputs"))) return rc;
   return FS_OK;
 }
@@ -322,7 +323,8 @@ int run_score(fs_model* m, const Set& set, const fs_samples* smp, const int32_t*
                        fs_dump_stride(m), m->sm_count, m->lc, s),
           "launch score");
   if (timed) FS_CUDA(cudaEventRecord(ev[3], s), "record timing event");
-  FS_CUDA(launch_finalize(set, it, pl, (const uint64_t*)m->sums.p, gap, score, gamma_t, best, status_copy, s),
+  FS_CUDA(launch_finalize(set, it, pl, (const uint64_t*)m->sums.p, gap, score, gamma_t, best, status_copy,
+                          (uint64_t*)m->sums.p + (size_t)std::max(n, 1) * smp->O, s),
           "launch finalize");
   if (phases) FS_CUDA(cudaEventRecord(ev[4], s), "record timing event");
   return FS_OK;
@@ -406,7 +408,7 @@ int fs_load_model(const fs_bounds* b, const float* slo, const float* demand, int
   const size_t o_bounds = take(16 * (size_t)cells), o_rev = take(cells);
   const size_t o_theta = take(8 * (size_t)d.theta_cap), o_nth = take(8);
   const size_t o_rowc = take(8 * (size_t)d.K4), o_rowb = take(8 * (size_t)d.K4);
-  const size_t o_base = take(2 * sizeof(fs_allocation)), o_status = take(4), o_work = take(8);
+  const size_t o_base = take(2 * sizeof(fs_allocation)), o_status = take(4), o_work = take(16);
   rc = m->fixed.ensure(off, "model state");
   if (rc) {
     delete m;

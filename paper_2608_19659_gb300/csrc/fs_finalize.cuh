@@ -74,8 +74,11 @@ __device__ __forceinline__ double fixed_mean(unsigned long long v, long long n, 
   return __longlong_as_double((long long)(((unsigned long long)bexp << 52) | (m & ((1ull << 52) - 1ull))));
 }
 
+// Items [beg, end) of problem p, whose first item is pos0 (candidate positions,
+// for the order of equal scores, count from there).
 __device__ inline Best finalize_problem(const Set& set, const Items& it, const Plan& pl, const uint64_t* sums,
-                                 int p, int beg, int end, double* gap, double* score, float* gt_out) {
+                                 int p, int beg, int end, double* gap, double* score, float* gt_out,
+                                 int pos0) {
   __shared__ Best sb[32];
   const Dims& d = set.d;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = blockDim.x >> 5;
@@ -94,7 +97,7 @@ __device__ inline Best finalize_problem(const Set& set, const Items& it, const P
     const long long sc = gfix * n - tot;
     if (gap) gap[q] = fixed_mean((unsigned long long)tot, n, log2n);
     if (score) score[q] = fixed_mean((unsigned long long)sc, n, log2n);
-    const Best c = make_best(sc, (cell / d.B) & 3, q - beg, cell);
+    const Best c = make_best(sc, (cell / d.B) & 3, q - pos0, cell);
     if (better(c, b)) b = c;
   }
   b = warp_best(b);

@@ -10,7 +10,7 @@
 //   rowC     [P][2][K*4]   f32   best SLO-feasible capacity per (class, TP)
 //   rowB     [P][2][K*4]   i32   its bin (-1: none)
 //   base     [P][2]        fs_allocation
-//   work     [1]           u64   chunk counter of the Monte-Carlo kernel
+//   work     [2]           u64   chunk counter of the Monte-Carlo kernel, the reduction's ticket
 // Per scoring call (items = (problem, candidate cell) pairs), one record of
 // item_floats = 2 slot_floats + O Wp floats per item:
 //   [2][slot_floats] f32   threshold tables of the two realisations
@@ -90,7 +90,7 @@ struct Set {
   int* rowB;            // [P][2][K4] bin of rowC, -1 = no SLO-feasible bin
   fs_allocation* base;  // [P][2]
   uint32_t* status;
-  unsigned long long* work;  // [1] chunk counter, zeroed by k_prep
+  unsigned long long* work;  // [2] chunk counter, reduction ticket; zeroed by k_prep
   const int* skip;      // [P] or nullptr: base solves skip problems with skip[p] >= 0
 };
 
@@ -375,9 +375,12 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
                          uint64_t* sums, void* dump, int dump_stride, int sm_count, LaunchCache& lc,
                          cudaStream_t s);
 // status_copy (nullable): the status word as it stands after the whole call.
+// part: 2 finalize_blocks(it) words of scratch (nullable when that is 0).
+constexpr int kFinalizeMaxBlocks = 64;
+int finalize_blocks(const Items& it);
 cudaError_t launch_finalize(const Set& set, const Items& it, const Plan& pl, const uint64_t* sums,
                             double* gap, double* score, float* gamma_t, int32_t* best, uint32_t* status_copy,
-                            cudaStream_t s);
+                            uint64_t* part, cudaStream_t s);
 cudaError_t launch_watchdog(uint32_t* status, uint64_t limit_ns, cudaStream_t s);
 
 // replay

@@ -110,7 +110,7 @@ __global__ void k_replay_next(Set set, ReplayState rs, int n_active) {
 __global__ void k_replay_reveal(Set set, ReplayState rs, Items it, Plan pl, const uint64_t* sums, int per) {
   const int a = blockIdx.x;
   const int p = rs.active[a];
-  const Best b = finalize_problem(set, it, pl, sums, p, a * per, (a + 1) * per, nullptr, nullptr, nullptr);
+  const Best b = finalize_problem(set, it, pl, sums, p, a * per, (a + 1) * per, nullptr, nullptr, nullptr, a * per);
   if (threadIdx.x == 0 && b.valid()) reveal_cell(set, rs, p, b.cell);
 }
 

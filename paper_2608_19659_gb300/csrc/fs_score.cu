@@ -140,7 +140,10 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
   const int cell = it.cell[item];
   float* base_rec = rec + (size_t)item * pl.item_floats;
   float* tab = base_rec + (size_t)sigma * d.slot_floats;
-  if (blockIdx.x == 0 && tid == 0) *set.work = 0ull;
+  if (blockIdx.x == 0 && tid == 0) {
+    set.work[0] = 0ull;  // the Monte-Carlo kernel's chunk counter
+    set.work[1] = 0ull;  // the reduction's ticket
+  }
   if (sigma == 0)
     for (int o = tid; o < pl.O; o += blockDim.x) sums[(size_t)item * pl.O + o] = 0ull;
   if (cell < 0 || cell >= d.cells) {  // device-side candidate ids are checked here
@@ -945,11 +948,44 @@ __global__ void k_finalize(Set set, Items it, Plan pl, const uint64_t* sums, dou
   const int p = blockIdx.x;
   const int beg = it.off ? it.off[p] : 0;
   const int end = it.off ? it.off[p + 1] : it.n;
-  const Best b = finalize_problem(set, it, pl, sums, p, beg, end, gap, score, gamma_t ? gamma_t + p : nullptr);
+  const Best b = finalize_problem(set, it, pl, sums, p, beg, end, gap, score, gamma_t ? gamma_t + p : nullptr, beg);
   if (threadIdx.x == 0 && best) best[p] = b.valid() ? b.cell : -1;
   // every kernel of the call has finished (stream order, and the wait above):
   // its status word can travel with the outputs
   if (threadIdx.x == 0 && p == 0 && status_copy) *status_copy = *set.status;
+}
+
+// One problem with many candidates, split over the CTAs: each writes its
+// candidates' expectations and scores and its best entry into part[2 b ..],
+// and the last to finish (a ticket in work[1], zeroed by k_prep) reduces them.
+__global__ void k_finalize_split(Set set, Items it, Plan pl, const uint64_t* sums, double* gap, double* score,
+                                 float* gamma_t, int32_t* best, uint32_t* status_copy, uint64_t* part) {
+  pdl_wait();
+  const int nb = (int)gridDim.x, per = (it.n + nb - 1) / nb;
+  const int beg = min(it.n, (int)blockIdx.x * per), end = min(it.n, beg + per);
+  const Best b = finalize_problem(set, it, pl, sums, 0, beg, end, gap, score,
+                                  blockIdx.x == 0 ? gamma_t : nullptr, 0);
+  __shared__ int s_last;
+  if (threadIdx.x == 0) {
+    part[2 * blockIdx.x] = (uint64_t)b.hi;
+    part[2 * blockIdx.x + 1] = ((uint64_t)b.lo << 32) | (uint32_t)b.cell;
+    __threadfence();
+    s_last = atomicAdd(&set.work[1], 1ull) == (unsigned long long)(nb - 1);
+  }
+  __syncthreads();
+  if (!s_last || threadIdx.x >= 32) return;
+  __threadfence();
+  Best r = no_best();
+  for (int q = threadIdx.x; q < nb; q += 32) {
+    const uint64_t w = __ldcg(part + 2 * q + 1);
+    const Best c{(long long)__ldcg(part + 2 * q), (uint32_t)(w >> 32), (int)(uint32_t)w};
+    if (better(c, r)) r = c;
+  }
+  r = warp_best(r);
+  if (threadIdx.x == 0) {
+    if (best) *best = r.valid() ? r.cell : -1;
+    if (status_copy) *status_copy = *set.status;
+  }
 }
 
 static size_t prep_smem_bytes(const Dims& d) { return (size_t)(256 + d.theta_cap) * 4; }
@@ -1042,10 +1078,21 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
                     (unsigned char*)dump, dump ? dump_stride : 0, sg);
 }
 
+int finalize_blocks(const Items& it) {
+  if (it.off) return 0;
+  const int nb = (it.n + 255) / 256;  // one candidate per thread
+  return nb < 2 ? 0 : (nb > kFinalizeMaxBlocks ? kFinalizeMaxBlocks : nb);
+}
+
 cudaError_t launch_finalize(const Set& set, const Items& it, const Plan& pl, const uint64_t* sums, double* gap,
-                            double* score, float* gamma_t, int32_t* best, uint32_t* status_copy, cudaStream_t s) {
-  return launch_pdl(k_finalize, dim3(it.off ? set.P : 1), dim3(256), 0, s, set, it, pl, sums, gap, score,
-                    gamma_t, best, status_copy);
+                            double* score, float* gamma_t, int32_t* best, uint32_t* status_copy, uint64_t* part,
+                            cudaStream_t s) {
+  const int nb = finalize_blocks(it);
+  if (nb > 0 && part)
+    return launch_pdl(k_finalize_split, dim3(nb), dim3(256), 0, s, set, it, pl, sums, gap, score, gamma_t, best,
+                      status_copy, part);
+  return launch_pdl(k_finalize, dim3(it.off ? set.P : 1), dim3(256), 0, s, set, it, pl, sums, gap, score, gamma_t,
+                    best, status_copy);
 }
 
 }  // namespace fs

@@ -115,7 +115,7 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
     off = up256(off + bytes);
     return o;
   };
-  const size_t o_status = take(4), o_work = take(8);
+  const size_t o_status = take(4), o_work = take(16), o_part = take(16 * (size_t)kFinalizeMaxBlocks);
   const size_t o_qn = quantile_dev ? 0 : take(4 * (size_t)Q);
   const size_t o_theta = take(8 * (size_t)d.theta_cap), o_nth = take(8);
   const size_t o_rowc = take(8 * (size_t)d.K4), o_rowb = take(8 * (size_t)d.K4);
@@ -203,7 +203,7 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
                      reinterpret_cast<uint64_t*>(base + o_sums), nullptr, 0, sm_count, *lc, s);
   if (e == cudaSuccess)
     e = launch_finalize(set, it, pl, reinterpret_cast<const uint64_t*>(base + o_sums), gap_dev, score_dev,
-                        gamma_t_dev, best_dev, nullptr, s);
+                        gamma_t_dev, best_dev, nullptr, reinterpret_cast<uint64_t*>(base + o_part), s);
   if (e != cudaSuccess) return cuda_say(e, "launch (allocation-free scoring)");
   uint32_t st = 0;
   e = cudaMemcpyAsync(&st, set.status, 4, cudaMemcpyDeviceToHost, s);

@@ -310,3 +310,16 @@ def test_table_path_with_long_tables(fsb, cuda, oracle_lib, qn):
     cand = probe.candidates[pos[:: max(1, len(pos) // 3)][:3]]
     r = run(fsb, w, cand=cand)
     assert_same(r, oracle_lib.score(w, qn, candidates=cand), cand=cand)
+
+
+def test_split_reduction_keeps_candidate_order(fsb, cuda, oracle_lib, qn):
+    """More than 256 candidates: the reduction is split over several blocks and
+    the argmax is merged from their results. Every cell appears several times,
+    so equal scores must still resolve to the earliest position of the list."""
+    w = stressed(0, 3.0, O=4, S=64)
+    rng = np.random.default_rng(12)
+    cand = rng.permutation(np.tile(np.arange(w.cells, dtype=np.int32), 10))[:600].astype(np.int32)
+    r = run(fsb, w, cand=cand)
+    ref = oracle_lib.score(w, qn, candidates=cand)
+    assert_same(r, ref)
+    assert r.best == ref.best and np.sum(cand == r.best) > 1
