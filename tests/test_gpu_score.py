@@ -323,3 +323,25 @@ def test_split_reduction_keeps_candidate_order(fsb, cuda, oracle_lib, qn):
     ref = oracle_lib.score(w, qn, candidates=cand)
     assert_same(r, ref)
     assert r.best == ref.best and np.sum(cand == r.best) > 1
+
+
+def test_repeated_arrays_read_at_every_call(fsb, cuda, oracle_lib, qn):
+    """The binding reuses the addresses of arrays passed again; their contents
+    are still read at every call (bounds and candidates changed in place)."""
+    w = stressed(0, 3.0, S=64)
+    cl, ch, tl, th = (np.ascontiguousarray(getattr(w, k).reshape(-1)).copy()
+                      for k in ("cap_lo", "cap_hi", "tail_lo", "tail_hi"))
+    cand = w.candidates.copy()
+    n = len(cand)
+    outs = (np.zeros(n), np.zeros(n), np.zeros(1, np.float32), np.zeros(1, np.int32), np.zeros((n, w.O), np.int64))
+    with load_model(fsb, w) as m:
+        fsb.fs_update_bounds(m, cl, ch, tl, th)
+        r = fsb.fs_score_candidates(m, cand, w.O, w.S, w.seed, outputs=outs)
+        assert np.array_equal(r.sum_eo, oracle_lib.score(w, qn).sum_eo)
+        cl *= np.float32(0.9)  # in place: same arrays, new contents
+        cand[:] = cand[::-1]
+        fsb.fs_update_bounds(m, cl, ch, tl, th)
+        r = fsb.fs_score_candidates(m, cand, w.O, w.S, w.seed, outputs=outs)
+    w2 = dataclasses.replace(w, cap_lo=cl.reshape(w.cap_lo.shape).copy(), candidates=cand.copy())
+    ref = oracle_lib.score(w2, qn)
+    assert np.array_equal(r.sum_eo, ref.sum_eo) and r.best == ref.best
