@@ -9,6 +9,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <new>
 #include <string>
 #include <vector>
@@ -19,6 +20,23 @@ namespace fs {
 
 static std::atomic<uint64_t> g_launches{0};
 void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+
+cudaError_t raise_smem_limit(const void* func, size_t bytes) {
+  static std::mutex mu;
+  static std::vector<std::pair<const void*, size_t>> limits;  // (kernel, largest limit set)
+  std::lock_guard<std::mutex> lock(mu);
+  size_t* cur = nullptr;
+  for (auto& e : limits)
+    if (e.first == func) cur = &e.second;
+  if (!cur) {
+    limits.emplace_back(func, 0);
+    cur = &limits.back().second;
+  }
+  const size_t want = std::max(*cur, bytes);
+  const cudaError_t e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)want);
+  if (e == cudaSuccess) *cur = want;
+  return e;
+}
 
 static thread_local std::string g_err;
 
@@ -409,6 +427,7 @@ int fs_load_model(const fs_bounds* b, const float* slo, const float* demand, int
   const size_t o_theta = take(8 * (size_t)d.theta_cap), o_nth = take(8);
   const size_t o_rowc = take(8 * (size_t)d.K4), o_rowb = take(8 * (size_t)d.K4);
   const size_t o_base = take(2 * sizeof(fs_allocation)), o_status = take(4), o_work = take(16);
+  const size_t o_rtab = take(8 * (size_t)kRowTabMax);
   rc = m->fixed.ensure(off, "model state");
   if (rc) {
     delete m;
@@ -431,6 +450,7 @@ int fs_load_model(const fs_bounds* b, const float* slo, const float* demand, int
   s.status = (uint32_t*)(base + o_status);
   s.work = (unsigned long long*)(base + o_work);
   s.skip = nullptr;
+  s.rtab = (int*)(base + o_rtab);
 
   m->h_lam.assign(demand, demand + K);
   m->h_slo.assign(slo, slo + K);
@@ -679,6 +699,7 @@ int fs_replay(fs_model* m, const fs_replay_spec* sp, int32_t* rounds, int32_t* s
   const size_t o_trace = take(4 * (size_t)P * (sp->max_rounds + 1));
   const size_t o_final = take((size_t)P * sizeof(fs_allocation)), o_active = take(4 * (size_t)P), o_nact = take(4);
   const size_t o_ip = take(4 * (size_t)P * cells), o_ic = take(4 * (size_t)P * cells);
+  const size_t o_rtab = take(8 * (size_t)P * kRowTabMax);
   Buf all;
   if ((rc = all.ensure(off, "replay state"))) return rc;
   char* base = (char*)all.p;
@@ -691,6 +712,7 @@ int fs_replay(fs_model* m, const fs_replay_spec* sp, int32_t* rounds, int32_t* s
   set.rowC = (float*)(base + o_rowc);
   set.rowB = (int*)(base + o_rowb);
   set.base = (fs_allocation*)(base + o_base);
+  set.rtab = (int*)(base + o_rtab);
   ReplayState rs{};
   rs.truth = (const float*)(base + o_truth);
   rs.perm = (const int*)(base + o_perm);

@@ -34,6 +34,9 @@ constexpr int kPrepThreads = 256;
 constexpr int kScoreThreads = 256;
 constexpr int kTableHeader = 20;      // floats before the three table arrays (16-byte multiple)
 constexpr int kSmemTableCap = 256;    // table entries staged in shared memory per realisation (pow2)
+// Row table of a scoring solve: one word per (row, threshold) pair, built when
+// K4 x |Theta| is at most this (else the per-candidate preparation searches).
+constexpr int kRowTabMax = 8192;
 
 // Table header words (floats unless noted).
 enum : int {
@@ -92,6 +95,7 @@ struct Set {
   uint32_t* status;
   unsigned long long* work;  // [2] chunk counter, reduction ticket; zeroed by k_prep
   const int* skip;      // [P] or nullptr: base solves skip problems with skip[p] >= 0
+  int* rtab;            // [P][2][kRowTabMax] or nullptr: row tables of the scoring solves
 };
 
 // Scenario plan shared by a launch.
@@ -329,6 +333,12 @@ constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s
 // ---------------------------------------------------------------- launchers (host)
 
 void note_launch();
+// Raises the dynamic shared memory limit of kernel `func` to at least `bytes`.
+// The limit belongs to the function, not to a model: models of every size and
+// the allocation-free path share it, and a caller that has set it once skips
+// the call later (LaunchCache), so it is only ever raised, to the largest size
+// asked for so far.
+cudaError_t raise_smem_limit(const void* func, size_t bytes);
 // Launch with programmatic stream serialisation: the kernel may start while
 // its predecessor drains and synchronises with it through pdl_wait().
 template <typename... KArgs, typename... Args>

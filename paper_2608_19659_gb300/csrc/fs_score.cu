@@ -116,6 +116,31 @@ __device__ __forceinline__ int probe_index(int g, int ng, int lo0, int hi0, int 
   return max(lo + 1, min(hi - 1, k));
 }
 
+// Smallest bit pattern C in (bx, bmax] with fulfil(m, C) >= t, given that bmax
+// qualifies (fulfil is nondecreasing in C, and nonnegative floats order like
+// their bit patterns). From the estimate `guess` it gallops (steps 1, 2, 4,
+// ...) until the answer is bracketed, then bisects: a few evaluations when the
+// estimate is within a few units in the last place, at most about 64 for any.
+__device__ __forceinline__ uint32_t kappa_walk(float mf, float t, float lam, float rl, uint32_t bx,
+                                               uint32_t bmax, uint32_t guess) {
+  uint32_t lo = bx, hi = bmax;  // lo fails (or is Cexcl itself), hi passes
+  const uint32_t g = min(max(guess, bx + 1u), bmax);
+  const bool up = g < bmax && fulfil_r(mf, __uint_as_float(g), lam, rl) < t;
+  if (up) lo = g; else hi = g;
+  for (uint32_t step = 1; hi - lo > 1; step <<= 1) {
+    const uint32_t w = min(step, hi - lo - 1);
+    const uint32_t q = up ? lo + w : hi - w;
+    const bool ok = fulfil_r(mf, __uint_as_float(q), lam, rl) >= t;
+    if (ok) hi = q; else lo = q;
+    if (ok == up) break;  // bracketed
+  }
+  while (hi - lo > 1) {
+    const uint32_t mid = lo + ((hi - lo) >> 1);
+    if (fulfil_r(mf, __uint_as_float(mid), lam, rl) >= t) hi = mid; else lo = mid;
+  }
+  return hi;
+}
+
 // One CTA per (candidate, realisation sigma). Before the threshold search it
 // maps the quantile strata of the outcomes o = sigma, sigma + 2, ... into the
 // candidate's record: this and Cexcl read only the bounds, so with `early`
@@ -261,44 +286,75 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
   const size_t ps = (size_t)p * 2 + sigma;
   const int total = set.ntheta[ps];
   const float* th_g = set.theta + ps * d.theta_cap;
+  // the base solve's row table, this candidate's row of it, when it built one
+  const bool rtab = set.rtab != nullptr && d.K4 * total <= kRowTabMax;
+  const int* rt_g = rtab ? set.rtab + ps * kRowTabMax + (size_t)rr * total : nullptr;
+  int* sRt = reinterpret_cast<int*>(sTh + d.theta_cap);  // [min(theta_cap, kRowTabMax / 4)]
   for (int rho = tid; rho < d.K4; rho += blockDim.x) sC[rho] = set.rowC[ps * d.K4 + rho];
-  for (int k = tid; k < total; k += blockDim.x) sTh[k] = th_g[k];
+  for (int k = tid; k < total; k += blockDim.x) {
+    sTh[k] = th_g[k];
+    if (rtab) sRt[k] = rt_g[k];
+  }
   __syncthreads();
   const float cx = s_cx, cmax = s_cmax;
   const int msent = d.K == 1 ? d.M[jr] : 0;  // above every threshold only a lone class can go on
 
   // b0: last index feasible at Cexcl; b1: last index feasible at max(Cexcl, cap_hi).
-  // Joint search: each round every group of gsz lanes probes one index and
-  // answers for both capacities; each warp merges the answers with integer
-  // max / min reductions, so a round costs one barrier.
-  int lgs = 2;
-  while ((1 << lgs) < d.K4 && lgs < 5) ++lgs;
-  const int gsz = 1 << lgs, ng = (int)blockDim.x >> lgs, g = tid >> lgs, gl = tid & (gsz - 1);
-  int lo0 = -1, hi0 = total, lo1 = -1, hi1 = total;
-  for (int par = 0; hi0 - lo0 > 1 || hi1 - lo1 > 1; par ^= 1) {
-    const int k = probe_index(g, ng, lo0, hi0, lo1, hi1);
-    const float t = sTh[k];
-    const Eval e = group_eval_excl<FL>(t, sC, sLam, sRl, sDl, d, rr, ie, gl, gsz);
-    if (gl == 0) {
-      const int m = replicas_left(e, jr, d);
-      const float te = FL ? fmaxf(t, dle) : t;
-      const int f = (feasible_at(e, m, cx, te, lam, rl) ? 1 : 0) | (feasible_at(e, m, cmax, te, lam, rl) ? 2 : 0);
-      s_res[par][g] = k | (f << 24);
+  // Feasibility is nonincreasing along the sorted thresholds, so with the row
+  // table each is the count of feasible indices less one (one barrier per 256
+  // indices); without it, a joint search.
+  int b0, b1;
+  if (rtab) {
+    int n0 = 0, n1 = 0;
+    for (int k0 = 0; k0 < total; k0 += blockDim.x) {
+      const int k = k0 + tid;
+      bool f0 = false, f1 = false;
+      if (k < total) {
+        const int e = sRt[k], m = e & 0xFFFF;
+        const bool other = (e >> 16) & 1;
+        const float te = FL ? fmaxf(sTh[k], dle) : sTh[k];
+        f0 = other || (m >= 1 && fulfil_r((float)m, cx, lam, rl) >= te);
+        f1 = other || (m >= 1 && fulfil_r((float)m, cmax, lam, rl) >= te);
+      }
+      n0 += __syncthreads_count(f0);
+      n1 += __syncthreads_count(f1);
     }
-    __syncthreads();
-    int a0 = lo0, c0 = hi0, a1 = lo1, c1 = hi1;
-    if (lane < ng) {
-      const int v = s_res[par][lane];
-      const int kq = v & 0xFFFFFF, f = v >> 24;
-      if (f & 1) a0 = max(a0, kq); else c0 = min(c0, kq);
-      if (f & 2) a1 = max(a1, kq); else c1 = min(c1, kq);
+    b0 = n0 - 1;
+    b1 = n1 - 1;
+  } else {
+    // Joint search: each round every group of gsz lanes probes one index and
+    // answers for both capacities; each warp merges the answers with integer
+    // max / min reductions, so a round costs one barrier.
+    int lgs = 2;
+    while ((1 << lgs) < d.K4 && lgs < 5) ++lgs;
+    const int gsz = 1 << lgs, ng = (int)blockDim.x >> lgs, g = tid >> lgs, gl = tid & (gsz - 1);
+    int lo0 = -1, hi0 = total, lo1 = -1, hi1 = total;
+    for (int par = 0; hi0 - lo0 > 1 || hi1 - lo1 > 1; par ^= 1) {
+      const int k = probe_index(g, ng, lo0, hi0, lo1, hi1);
+      const float t = sTh[k];
+      const Eval e = group_eval_excl<FL>(t, sC, sLam, sRl, sDl, d, rr, ie, gl, gsz);
+      if (gl == 0) {
+        const int m = replicas_left(e, jr, d);
+        const float te = FL ? fmaxf(t, dle) : t;
+        const int f = (feasible_at(e, m, cx, te, lam, rl) ? 1 : 0) | (feasible_at(e, m, cmax, te, lam, rl) ? 2 : 0);
+        s_res[par][g] = k | (f << 24);
+      }
+      __syncthreads();
+      int a0 = lo0, c0 = hi0, a1 = lo1, c1 = hi1;
+      if (lane < ng) {
+        const int v = s_res[par][lane];
+        const int kq = v & 0xFFFFFF, f = v >> 24;
+        if (f & 1) a0 = max(a0, kq); else c0 = min(c0, kq);
+        if (f & 2) a1 = max(a1, kq); else c1 = min(c1, kq);
+      }
+      lo0 = __reduce_max_sync(0xffffffffu, a0);
+      hi0 = __reduce_min_sync(0xffffffffu, c0);
+      lo1 = __reduce_max_sync(0xffffffffu, a1);
+      hi1 = __reduce_min_sync(0xffffffffu, c1);
     }
-    lo0 = __reduce_max_sync(0xffffffffu, a0);
-    hi0 = __reduce_min_sync(0xffffffffu, c0);
-    lo1 = __reduce_max_sync(0xffffffffu, a1);
-    hi1 = __reduce_min_sync(0xffffffffu, c1);
+    b0 = lo0;
+    b1 = lo1;
   }
-  const int b0 = lo0, b1 = lo1;
   const int Lt = b1 - b0;
   // Three arrays of Lpad = max(P, 4) entries, P = pow2 >= Lt + 1 (at least 4
   // for 16-byte copies): kappa[u] for u < Lt, +inf beyond, so the scenario
@@ -317,53 +373,72 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
   float* mnx = thx + Lpad;
 
   // u = 0..Lt: m at index b0+1+u; kappa for u < Lt
-  for (int u = warp; u <= Lt; u += nwarp) {
-    const int k = b0 + 1 + u;
-    int m;
-    if (k < total) {
-      const Eval e = group_eval_excl<FL>(sTh[k], sC, sLam, sRl, sDl, d, rr, ie, lane, 32);
-      m = replicas_left(e, jr, d);
-    } else {
-      m = msent;
-    }
-    if (u < Lt) {
-      // smallest capacity in (cx, cmax] at which f(m, C) >= max(theta_k,
-      // delta_{i_e}), on the bit patterns of nonnegative floats (ordered like
-      // the values). First the 32 patterns around the real solution t lambda / m,
-      // one per lane; if the answer is not among them, a 32-ary search over the
-      // whole interval.
-      const float th = sTh[k], t = FL ? fmaxf(th, dle) : th;
-      const uint32_t bx = __float_as_uint(cx), bmax = __float_as_uint(cmax);
-      const float c0 = __fdividef(__fmul_rn(t, lam), (float)m);  // an estimate: the window is checked exactly
-      const long long pl_ = (long long)__float_as_uint(c0) - 16 + lane;
-      const uint32_t pt0 = pl_ < 0 ? 0u : (uint32_t)pl_;
-      const bool ok0 = pt0 > bx && (pt0 >= bmax || fulfil_r((float)m, __uint_as_float(pt0), lam, rl) >= t);
-      const uint32_t bal0 = __ballot_sync(0xffffffffu, ok0);
-      uint32_t lo = bx, hi = bmax;
-      if (bal0 != 0u && (bal0 & 1u) == 0u) {  // lane 0 fails, some lane passes: the first passing lane
-        hi = __shfl_sync(0xffffffffu, pt0, __ffs(bal0) - 1);
-        lo = hi - 1;
-      }
-      while (hi - lo > 1) {
-        const uint32_t span = hi - lo;
-        const uint32_t pt = lo + (uint32_t)(((uint64_t)(lane + 1) * span) >> 5);
-        const bool ok = fulfil_r((float)m, __uint_as_float(pt), lam, rl) >= t;
-        const uint32_t bal = __ballot_sync(0xffffffffu, ok);
-        const int l = __ffs(bal) - 1;  // lane 31 tests hi, which is feasible
-        const uint32_t nhi = __shfl_sync(0xffffffffu, pt, l);
-        const uint32_t nlo = __shfl_sync(0xffffffffu, pt, l > 0 ? l - 1 : 0);
-        if (l > 0) lo = nlo;
-        hi = nhi;
-      }
-      if (lane == 0) {
-        kap[u] = __uint_as_float(hi);
+  if (rtab) {
+    // one thread per entry, m from the row table, kappa by a walk from the
+    // estimate t lambda / m (Cexcl = -0 as +0: the same smallest capacity)
+    const uint32_t bx = __float_as_uint(cx) & 0x7fffffffu, bmax = __float_as_uint(cmax) & 0x7fffffffu;
+    for (int u = tid; u <= Lt; u += blockDim.x) {
+      const int k = b0 + 1 + u;
+      const int m = k < total ? (sRt[k] & 0xFFFF) : msent;
+      if (u < Lt) {
+        const float th = sTh[k], t = FL ? fmaxf(th, dle) : th;
+        const float c0 = __fdividef(__fmul_rn(t, lam), (float)m);  // an estimate: the walk is exact
+        kap[u] = __uint_as_float(kappa_walk((float)m, t, lam, rl, bx, bmax, __float_as_uint(c0)));
         thx[u + 1] = th;
       }
-    }
-    if (lane == 0) {
       if (m >= 1) s_row = 1;
       mnx[u] = (float)m;
       if (u == 0) tab[H_M_FIRST] = (float)m;
+    }
+  } else {
+    for (int u = warp; u <= Lt; u += nwarp) {
+      const int k = b0 + 1 + u;
+      int m;
+      if (k < total) {
+        const Eval e = group_eval_excl<FL>(sTh[k], sC, sLam, sRl, sDl, d, rr, ie, lane, 32);
+        m = replicas_left(e, jr, d);
+      } else {
+        m = msent;
+      }
+      if (u < Lt) {
+        // smallest capacity in (cx, cmax] at which f(m, C) >= max(theta_k,
+        // delta_{i_e}), on the bit patterns of nonnegative floats (ordered like
+        // the values). First the 32 patterns around the real solution t lambda / m,
+        // one per lane; if the answer is not among them, a 32-ary search over the
+        // whole interval.
+        const float th = sTh[k], t = FL ? fmaxf(th, dle) : th;
+        const uint32_t bx = __float_as_uint(cx), bmax = __float_as_uint(cmax);
+        const float c0 = __fdividef(__fmul_rn(t, lam), (float)m);  // an estimate: the window is checked exactly
+        const long long pl_ = (long long)__float_as_uint(c0) - 16 + lane;
+        const uint32_t pt0 = pl_ < 0 ? 0u : (uint32_t)pl_;
+        const bool ok0 = pt0 > bx && (pt0 >= bmax || fulfil_r((float)m, __uint_as_float(pt0), lam, rl) >= t);
+        const uint32_t bal0 = __ballot_sync(0xffffffffu, ok0);
+        uint32_t lo = bx, hi = bmax;
+        if (bal0 != 0u && (bal0 & 1u) == 0u) {  // lane 0 fails, some lane passes: the first passing lane
+          hi = __shfl_sync(0xffffffffu, pt0, __ffs(bal0) - 1);
+          lo = hi - 1;
+        }
+        while (hi - lo > 1) {
+          const uint32_t span = hi - lo;
+          const uint32_t pt = lo + (uint32_t)(((uint64_t)(lane + 1) * span) >> 5);
+          const bool ok = fulfil_r((float)m, __uint_as_float(pt), lam, rl) >= t;
+          const uint32_t bal = __ballot_sync(0xffffffffu, ok);
+          const int l = __ffs(bal) - 1;  // lane 31 tests hi, which is feasible
+          const uint32_t nhi = __shfl_sync(0xffffffffu, pt, l);
+          const uint32_t nlo = __shfl_sync(0xffffffffu, pt, l > 0 ? l - 1 : 0);
+          if (l > 0) lo = nlo;
+          hi = nhi;
+        }
+        if (lane == 0) {
+          kap[u] = __uint_as_float(hi);
+          thx[u + 1] = th;
+        }
+      }
+      if (lane == 0) {
+        if (m >= 1) s_row = 1;
+        mnx[u] = (float)m;
+        if (u == 0) tab[H_M_FIRST] = (float)m;
+      }
     }
   }
   for (int u = Lt + tid; u < Lpad; u += blockDim.x) {
@@ -988,16 +1063,20 @@ __global__ void k_finalize_split(Set set, Items it, Plan pl, const uint64_t* sum
   }
 }
 
-static size_t prep_smem_bytes(const Dims& d) { return (size_t)(256 + d.theta_cap) * 4; }
+// rowC, the thresholds and, with a row table, the candidate row's words
+static size_t prep_smem_bytes(const Set& set) {
+  const Dims& d = set.d;
+  return (size_t)(256 + d.theta_cap + (set.rtab ? std::min(d.theta_cap, kRowTabMax / 4) : 0)) * 4;
+}
 
 cudaError_t launch_prep(const Set& set, const Items& it, const Plan& pl, float* tables, uint64_t* sums,
                         bool early, LaunchCache& lc, cudaStream_t s) {
   if (it.n <= 0) return cudaSuccess;
-  const size_t smem = prep_smem_bytes(set.d);
+  const size_t smem = prep_smem_bytes(set);
   const int fl = lc.floors ? 1 : 0;
   auto kern = fl ? k_prep<true> : k_prep<false>;
   if (smem > lc.prep_smem[fl]) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(kern), smem);
     if (e != cudaSuccess) return e;
     lc.prep_smem[fl] = smem;
   }
@@ -1025,7 +1104,7 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
                   : (fl ? k_score<false, true, false> : k_score<false, false, false>);
   if (smem != lc.score_smem[v][fl]) {
     int per_sm = 0;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(kern), smem);
     if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kScoreThreads, smem);
     if (e != cudaSuccess) return e;
     lc.score_smem[v][fl] = smem;

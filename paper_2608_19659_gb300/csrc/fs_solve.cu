@@ -262,32 +262,89 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
     }
   }
 
-  // 3. search: largest index whose threshold fits in G (lo feasible, hi not).
-  // Each round every group of gsz lanes probes one index (an (ng+1)-ary
-  // split); each warp merges the answers with integer max / min reductions,
-  // so a round costs one barrier.
+  // 3. t*: the largest index whose threshold fits in G (the cheapest-cover
+  // total is nondecreasing along the sorted thresholds).
   __shared__ int s_res[2][kSolveThreads / 4];
   if (tid == 0) sMisc[4] = 0;
   __syncthreads();
-  int gsz = 4;
-  while (gsz < d.K4 && gsz < 32) gsz <<= 1;
-  const int ng = blockDim.x / gsz, g = tid / gsz, gl = tid & (gsz - 1);
-  int lo = -1, hi = total;
-  for (int par = 0; hi - lo > 1; par ^= 1) {
-    int kp = lo + ((g + 1) * (hi - lo)) / (ng + 1);
-    kp = max(lo + 1, min(hi - 1, kp));
-    const int cost = group_total_cost<FL>(sTheta[kp], sC, sLam, sRl, sDl, d, gl, gsz);
-    if (gl == 0) s_res[par][g] = (cost <= d.G) ? kp : -(kp + 1);
-    __syncthreads();
-    int nlo = lo, nhi = hi;
-    for (int q = lane; q < ng; q += 32) {
-      const int v = s_res[par][q];
-      if (v >= 0) nlo = max(nlo, v); else nhi = min(nhi, -v - 1);
+  int kstar;
+  if (write_theta && !cap_x && set.rtab && d.K4 * total <= kRowTabMax) {
+    // Row table of a scoring solve: every row's cover cost at every threshold,
+    // then per (row rho, threshold k) the word the per-candidate preparation
+    // reads for a candidate in row rho: bits 0-15 the replicas rho may use
+    // once the other classes are covered (0 if one cannot be), bit 16 set if
+    // another row of rho's class covers theta_k within that budget. t* is
+    // the count of thresholds whose total fits, less one.
+    int P2c = 1;
+    while (P2c < d.theta_cap) P2c <<= 1;
+    int* sCost = reinterpret_cast<int*>(sTheta + P2c);  // [K4][total]
+    int* sSum = sCost + d.K4 * total;                   // [total]
+    const int nx = d.K4 * total;
+    for (int x = tid; x < nx; x += blockDim.x) {
+      const int rho = x / total, k = x - rho * total;
+      const float tc = FL ? fmaxf(sTheta[k], sDl[rho >> 2]) : sTheta[k];
+      const int n = min_replicas(tc, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[rho & 3]);
+      sCost[x] = n ? n << (rho & 3) : kCostInf;
     }
-    lo = __reduce_max_sync(0xffffffffu, nlo);
-    hi = __reduce_min_sync(0xffffffffu, nhi);
+    __syncthreads();
+    // per threshold: the classes' cheapest covers summed, an uncovered class
+    // counted as 2^24 (a cost is at most G <= 32767, 64 of them stay below 2^21)
+    for (int k = tid; k < total; k += blockDim.x) {
+      int sum = 0;
+      for (int i = 0; i < d.K; ++i) {
+        const int* c = sCost + 4 * i * total + k;
+        const int cm = min(min(c[0], c[total]), min(c[2 * total], c[3 * total]));
+        sum += cm >= kCostInf ? (1 << 24) : cm;
+      }
+      sSum[k] = sum;
+    }
+    __syncthreads();
+    int* rt = set.rtab + ((size_t)p * 2 + sigma) * kRowTabMax;
+    for (int x = tid; x < nx; x += blockDim.x) {
+      const int rho = x / total, k = x - rho * total, j = rho & 3;
+      const int* c = sCost + (rho & ~3) * total + k;
+      int own = kCostInf, other = kCostInf;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int v = c[q * total];
+        own = min(own, v);
+        if (q != j) other = min(other, v);
+      }
+      const int rest = sSum[k] - (own >= kCostInf ? (1 << 24) : own);
+      const int A = (rest >> 24) ? -1 : d.G - rest;
+      const int m = A >= (1 << j) ? min(A >> j, d.M[j]) : 0;
+      rt[x] = m | ((other < kCostInf && other <= A) ? 1 << 16 : 0);
+    }
+    int cnt = 0;
+    for (int k0 = 0; k0 < total; k0 += blockDim.x) {
+      const int k = k0 + tid;
+      cnt += __syncthreads_count(k < total && sSum[k] <= d.G);
+    }
+    kstar = cnt - 1;
+  } else {
+    // Search: each round every group of gsz lanes probes one index (an
+    // (ng+1)-ary split); each warp merges the answers with integer max / min
+    // reductions, so a round costs one barrier (lo feasible, hi not).
+    int gsz = 4;
+    while (gsz < d.K4 && gsz < 32) gsz <<= 1;
+    const int ng = blockDim.x / gsz, g = tid / gsz, gl = tid & (gsz - 1);
+    int lo = -1, hi = total;
+    for (int par = 0; hi - lo > 1; par ^= 1) {
+      int kp = lo + ((g + 1) * (hi - lo)) / (ng + 1);
+      kp = max(lo + 1, min(hi - 1, kp));
+      const int cost = group_total_cost<FL>(sTheta[kp], sC, sLam, sRl, sDl, d, gl, gsz);
+      if (gl == 0) s_res[par][g] = (cost <= d.G) ? kp : -(kp + 1);
+      __syncthreads();
+      int nlo = lo, nhi = hi;
+      for (int q = lane; q < ng; q += 32) {
+        const int v = s_res[par][q];
+        if (v >= 0) nlo = max(nlo, v); else nhi = min(nhi, -v - 1);
+      }
+      lo = __reduce_max_sync(0xffffffffu, nlo);
+      hi = __reduce_min_sync(0xffffffffu, nhi);
+    }
+    kstar = lo;
   }
-  const int kstar = lo;
   const float tstar = kstar >= 0 ? sTheta[kstar] : 0.0f;
 
   if (choice) {
@@ -397,11 +454,13 @@ cudaError_t launch_qtable(float* qn, int Q, cudaStream_t s) {
 cudaError_t launch_solve(const Set& set, int n, const float* cap_x, const float* tail_x,
                          fs_allocation* out, bool write_theta, LaunchCache& lc, cudaStream_t s, bool tstar_only) {
   if (n <= 0) return cudaSuccess;
-  const size_t smem = solve_smem_bytes(set.d);
+  // a scoring solve may build the row table: K4 x |Theta| cover costs, then |Theta| sums
+  const size_t smem =
+      solve_smem_bytes(set.d) + (write_theta && set.rtab ? (size_t)(kRowTabMax + kRowTabMax / 4) * 4 : 0);
   const int fl = lc.floors ? 1 : 0;
   auto kern = fl ? k_solve<true> : k_solve<false>;
   if (smem > lc.solve_smem[fl]) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(kern), smem);
     if (e != cudaSuccess) return e;
     lc.solve_smem[fl] = smem;
   }

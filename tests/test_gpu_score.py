@@ -345,3 +345,20 @@ def test_repeated_arrays_read_at_every_call(fsb, cuda, oracle_lib, qn):
     w2 = dataclasses.replace(w, cap_lo=cl.reshape(w.cap_lo.shape).copy(), candidates=cand.copy())
     ref = oracle_lib.score(w2, qn)
     assert np.array_equal(r.sum_eo, ref.sum_eo) and r.best == ref.best
+
+
+def test_models_of_different_sizes_used_alternately(fsb, cuda, oracle_lib, qn):
+    """Kernels' shared-memory limits belong to the kernels, not to a model: a
+    smaller model scored between two calls of a larger one leaves the larger
+    one's launches valid."""
+    big, small = stressed(2, S=64), stressed(0, S=64)
+    big = dataclasses.replace(big, candidates=big.candidates[::16].copy())
+    with load_model(fsb, big) as mb:
+        first = fsb.fs_score_candidates(mb, big.candidates, big.O, big.S, big.seed)
+        with load_model(fsb, small) as ms:
+            r = fsb.fs_score_candidates(ms, small.candidates, small.O, small.S, small.seed)
+        again = fsb.fs_score_candidates(mb, big.candidates, big.O, big.S, big.seed)
+        fsb.fs_solve_bounds(mb)
+    assert np.array_equal(r.sum_eo, oracle_lib.score(small, qn).sum_eo)
+    assert np.array_equal(first.sum_eo, again.sum_eo)
+    assert np.array_equal(again.sum_eo, oracle_lib.score(big, qn).sum_eo)

@@ -79,6 +79,9 @@ def test_random_small_problems(fsb, cuda, oracle_lib, seed):
     (1, 6, 1, 24),      # one GPU, six bins
     (3, 5, 1, 60),      # one GPU for three classes: t* = 0 on both sides
     (1, 2, 8738, 8),    # 16383 thresholds, within one of the most a model holds
+    (1, 2, 1000, 16),   # 1875 thresholds: row table of 7500 words, several passes per count
+    (1, 3, 1200, 16),   # row table on one realisation only (6600 and 9000 words)
+    (8, 2, 64, 24),     # eight classes, row table of 7968 words
 ])
 def test_extreme_sizes(fsb, cuda, oracle_lib, K, B, G, n_cand):
     rng = np.random.default_rng(K * 7919 + B * 31 + G)
