@@ -200,6 +200,16 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   }
   int P2 = 1;
   while (P2 < total) P2 <<= 1;
+  // A scoring solve builds the row table (step 3) when it is small enough; its
+  // scratch follows the thresholds: cover costs [K4][total], class minima
+  // [K][total], and each row's own fulfilment values in order [total]
+  const bool row_table =
+      write_theta && !cap_x && set.rtab && d.K4 * total <= kRowTabMax && sOff[d.K4] == total;
+  int P2c = 1;
+  while (P2c < d.theta_cap) P2c <<= 1;
+  int* sCost = reinterpret_cast<int*>(sTheta + P2c);
+  int* sCmin = sCost + d.K4 * total;
+  float* sOwn = reinterpret_cast<float*>(sCmin + d.K * total);
 
   // 2. thresholds, then bitonic sort (ascending, +inf padding)
   for (int x = tid; x < P2; x += blockDim.x) {
@@ -212,6 +222,7 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
       }
       const int n = sN0[lo] + (x - sOff[lo]);
       v = fulfil_r((float)n, sC[lo], sLam[lo >> 2], sRl[lo >> 2]);
+      if (row_table) sOwn[x] = v;
     }
     sTheta[x] = v;
   }
@@ -268,57 +279,80 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   if (tid == 0) sMisc[4] = 0;
   __syncthreads();
   int kstar;
-  if (write_theta && !cap_x && set.rtab && d.K4 * total <= kRowTabMax) {
+  if (row_table) {
     // Row table of a scoring solve: every row's cover cost at every threshold,
     // then per (row rho, threshold k) the word the per-candidate preparation
     // reads for a candidate in row rho: bits 0-15 the replicas rho may use
     // once the other classes are covered (0 if one cannot be), bit 16 set if
-    // another row of rho's class covers theta_k within that budget. t* is
-    // the count of thresholds whose total fits, less one.
-    int P2c = 1;
-    while (P2c < d.theta_cap) P2c <<= 1;
-    int* sCost = reinterpret_cast<int*>(sTheta + P2c);  // [K4][total]
-    int* sSum = sCost + d.K4 * total;                   // [total]
-    const int nx = d.K4 * total;
+    // another row of rho's class covers theta_k within that budget.
+    //
+    // A row's cheapest cover of t (class i covers max(t, delta_i)) is n0 plus
+    // the number of its own values f(n0) <= ... <= f(len) below t: every n
+    // below n0 falls short of it, and past len either f(ns) >= 1 >= t or the
+    // row holds M replicas and none covers t. The values are the fulfilments
+    // the thresholds were made of, so the count is the cover min_replicas
+    // finds, without evaluating f. One thread per (class, threshold) runs the
+    // four TP rows' branch-free lower bounds side by side.
+    const int nx = d.K * total;
     for (int x = tid; x < nx; x += blockDim.x) {
-      const int rho = x / total, k = x - rho * total;
-      const float tc = FL ? fmaxf(sTheta[k], sDl[rho >> 2]) : sTheta[k];
-      const int n = min_replicas(tc, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[rho & 3]);
-      sCost[x] = n ? n << (rho & 3) : kCostInf;
-    }
-    __syncthreads();
-    // per threshold: the classes' cheapest covers summed, an uncovered class
-    // counted as 2^24 (a cost is at most G <= 32767, 64 of them stay below 2^21)
-    for (int k = tid; k < total; k += blockDim.x) {
-      int sum = 0;
-      for (int i = 0; i < d.K; ++i) {
-        const int* c = sCost + 4 * i * total + k;
-        const int cm = min(min(c[0], c[total]), min(c[2 * total], c[3 * total]));
-        sum += cm >= kCostInf ? (1 << 24) : cm;
-      }
-      sSum[k] = sum;
-    }
-    __syncthreads();
-    int* rt = set.rtab + ((size_t)p * 2 + sigma) * kRowTabMax;
-    for (int x = tid; x < nx; x += blockDim.x) {
-      const int rho = x / total, k = x - rho * total, j = rho & 3;
-      const int* c = sCost + (rho & ~3) * total + k;
-      int own = kCostInf, other = kCostInf;
+      const int i = x / total, k = x - i * total;
+      const float tc = FL ? fmaxf(sTheta[k], sDl[i]) : sTheta[k];
+      int q[4], nv[4], beg[4];  // values below tc so far, values held, first value
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int v = c[q * total];
-        own = min(own, v);
-        if (q != j) other = min(other, v);
+      for (int j = 0; j < 4; ++j) {
+        beg[j] = sOff[4 * i + j];
+        nv[j] = sOff[4 * i + j + 1] - beg[j];
+        q[j] = 0;
       }
-      const int rest = sSum[k] - (own >= kCostInf ? (1 << 24) : own);
-      const int A = (rest >> 24) ? -1 : d.G - rest;
-      const int m = A >= (1 << j) ? min(A >> j, d.M[j]) : 0;
-      rt[x] = m | ((other < kCostInf && other <= A) ? 1 << 16 : 0);
+      const int most = max(max(nv[0], nv[1]), max(nv[2], nv[3]));
+      for (int step = most ? 1 << (31 - __clz(most)) : 0; step > 0; step >>= 1) {
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          if (q[j] + step <= nv[j] && sOwn[beg[j] + q[j] + step - 1] < tc) q[j] += step;
+      }
+      int cm = kCostInf;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int c = q[j] < nv[j] ? (sN0[4 * i + j] + q[j]) << j : kCostInf;
+        sCost[(4 * i + j) * total + k] = c;
+        cm = min(cm, c);
+      }
+      sCmin[x] = cm;
     }
+    __syncthreads();
+    // per pair: the other classes' covers summed (an uncovered class counted as
+    // 2^24: a cost is at most G <= 32767, 64 of them stay below 2^21), then one
+    // word per TP row; t* = the count of thresholds whose total fits, less one
+    int* rt = set.rtab + ((size_t)p * 2 + sigma) * kRowTabMax;
     int cnt = 0;
-    for (int k0 = 0; k0 < total; k0 += blockDim.x) {
-      const int k = k0 + tid;
-      cnt += __syncthreads_count(k < total && sSum[k] <= d.G);
+    for (int x0 = 0; x0 < nx; x0 += blockDim.x) {
+      const int x = x0 + tid;
+      bool fits = false;
+      if (x < nx) {
+        const int i = x / total, k = x - i * total;
+        int sum = 0;
+        for (int q = 0; q < d.K; ++q) {
+          const int cq = sCmin[q * total + k];
+          sum += cq >= kCostInf ? (1 << 24) : cq;
+        }
+        fits = i == 0 && sum <= d.G;
+        const int own = sCmin[x];
+        const int rest = sum - (own >= kCostInf ? (1 << 24) : own);
+        const int A = (rest >> 24) ? -1 : d.G - rest;
+        int c[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) c[j] = sCost[(4 * i + j) * total + k];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          int other = kCostInf;  // cheapest cover by another row of the class
+#pragma unroll
+          for (int q = 0; q < 4; ++q)
+            if (q != j) other = min(other, c[q]);
+          const int m = A >= (1 << j) ? min(A >> j, d.M[j]) : 0;
+          rt[(4 * i + j) * total + k] = m | ((other < kCostInf && other <= A) ? 1 << 16 : 0);
+        }
+      }
+      cnt += __syncthreads_count(fits);
     }
     kstar = cnt - 1;
   } else {
@@ -454,9 +488,10 @@ cudaError_t launch_qtable(float* qn, int Q, cudaStream_t s) {
 cudaError_t launch_solve(const Set& set, int n, const float* cap_x, const float* tail_x,
                          fs_allocation* out, bool write_theta, LaunchCache& lc, cudaStream_t s, bool tstar_only) {
   if (n <= 0) return cudaSuccess;
-  // a scoring solve may build the row table: K4 x |Theta| cover costs, then |Theta| sums
+  // a scoring solve may build the row table: K4 x |Theta| cover costs, K x |Theta| class minima
+  // and |Theta| own values, with K4 x |Theta| <= kRowTabMax
   const size_t smem =
-      solve_smem_bytes(set.d) + (write_theta && set.rtab ? (size_t)(kRowTabMax + kRowTabMax / 4) * 4 : 0);
+      solve_smem_bytes(set.d) + (write_theta && set.rtab ? (size_t)(kRowTabMax + kRowTabMax / 2) * 4 : 0);
   const int fl = lc.floors ? 1 : 0;
   auto kern = fl ? k_solve<true> : k_solve<false>;
   if (smem > lc.solve_smem[fl]) {
