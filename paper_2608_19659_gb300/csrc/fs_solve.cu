@@ -4,16 +4,19 @@
 // One CTA solves one realisation (a capacity and a tail value per cell):
 //   1. rows: for every (class i, TP index j) the best SLO-feasible bin
 //      (largest capacity, then lowest bin; Eq. 5 gates l <= L_i) -> C_ij.
-//      All cells are read once, coalesced; each feasible cell folds
-//      (capacity, -bin) into its row with a 64-bit shared-memory atomicMax;
+//      All cells are read once, coalesced; a 32-bit shared-memory atomicMax
+//      of the feasible cells' capacity bits per row, then an atomicMin of the
+//      bins that hold that capacity (a 64-bit atomicMax of (capacity, -bin)
+//      is no native operation: under contention it measured 15x slower);
 //   2. thresholds: the positive fulfilments f(n, C_ij), n = 1..floor(G/tau_j)
 //      (cut at the first n with f = 1), written to shared memory and
 //      bitonic-sorted;
-//   3. search: the largest threshold t whose cheapest per-class covers fit in
-//      G. Each probe is one warp: lanes hold rows, shuffles take the per-class
-//      minimum over the four TP lanes, a ballot flags classes with no cover,
-//      and a warp reduction sums the GPUs. The CTA's eight warps probe eight
-//      points per step (a 9-ary search);
+//   3. t*: the largest threshold t whose cheapest per-class covers fit in G.
+//      A scoring solve tabulates every row's cover of every threshold (the
+//      row table the per-candidate preparation reads) and counts; otherwise a
+//      search, each probe one group of lanes (a row per lane, shuffles for the
+//      per-class minimum over the four TP lanes and the sum), the groups of the
+//      CTA probing evenly spaced points per round;
 //   4. choice at t*: per class the cheapest cover, ties to the lower TP.
 // For a fixed (TP, n) a larger capacity never lowers f, so the best bin of
 // each row is the option the tie rule (larger capacity, then lower bin)
@@ -111,8 +114,9 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
     out = set.base + r;
   }
 
-  unsigned long long* sKey = reinterpret_cast<unsigned long long*>(smraw);  // [256]
-  float* sC = reinterpret_cast<float*>(sKey + 256);       // [256]
+  uint32_t* sRowCap = reinterpret_cast<uint32_t*>(smraw);  // [256] best feasible capacity bits per row
+  uint32_t* sRowBin = sRowCap + 256;                       // [256] lowest bin holding it (~0u: none)
+  float* sC = reinterpret_cast<float*>(sRowBin + 256);    // [256]
   int* sB = reinterpret_cast<int*>(sC + 256);             // [256]
   int* sN0 = sB + 256;                                    // [256]
   int* sOff = sN0 + 256;                                  // [260]
@@ -120,9 +124,10 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   int* sMisc = sProbe + 32;                               // [8]
   float* sTheta = reinterpret_cast<float*>(sMisc + 8);    // [pow2 >= theta_cap]
 
-  // 1. rows: key = (capacity bits, ~bin) of the best SLO-feasible bin; 0 = none.
-  // The inputs of the first pass (demands, and each thread's first cell) are
-  // all loaded before anything waits on one of them: one memory round trip.
+  // 1. rows: the best SLO-feasible bin of each row (largest capacity, then
+  // lowest bin). The inputs of the first pass (demands, and each thread's
+  // first cell) are all loaded before anything waits on one of them: one
+  // memory round trip.
   __shared__ float sLam[FS_MAX_CLASSES], sRl[FS_MAX_CLASSES];  // demand and RN(1/demand)
   __shared__ float sDl[FS_MAX_CLASSES];                          // floor delta_i (0: not critical)
   const float lam_v = tid < d.K ? set.lam[tid] : 1.0f;
@@ -130,7 +135,10 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   const bool cell0 = tid < d.cells;
   const float tail0 = cell0 ? tail[tid] : 0.0f, cap0 = cell0 ? cap[tid] : 0.0f;
   const float slo0 = cell0 ? set.slo[(tid / d.B) >> 2] : 0.0f;
-  for (int rho = tid; rho < d.K4; rho += blockDim.x) sKey[rho] = 0ull;
+  for (int rho = tid; rho < d.K4; rho += blockDim.x) {
+    sRowCap[rho] = 0u;
+    sRowBin[rho] = ~0u;
+  }
   if (tid < 8) sMisc[tid] = 0;
   if (tid < d.K) {
     sLam[tid] = lam_v;
@@ -138,23 +146,28 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
     if (FL) sDl[tid] = dl_v;
   }
   __syncthreads();
+  // feasible cells: their capacity's bits (-0 -> +0: nonnegative floats order
+  // like their bit patterns), first the row maximum, then the lowest bin
+  // holding it
+  const bool ok0 = cell0 && tail0 <= slo0;
+  const uint32_t cb0 = __float_as_uint(__fadd_rn(cap0, 0.0f));
   for (int c = tid; c < d.cells; c += blockDim.x) {
     const int rho = c / d.B;
-    const int b = c - rho * d.B;
-    const bool first = c == tid;
-    const float tv = first ? tail0 : tail[c];
-    const float lv = first ? slo0 : set.slo[rho >> 2];
-    if (tv <= lv) {
-      const float cv = first ? cap0 : cap[c];
-      const uint32_t cb = __float_as_uint(__fadd_rn(cv, 0.0f));  // -0 -> +0: bits order like values
-      atomicMax(&sKey[rho], ((unsigned long long)cb << 32) | (0xFFFFFFFFu - (uint32_t)b));
-    }
+    const bool ok = c == tid ? ok0 : tail[c] <= set.slo[rho >> 2];
+    if (ok) atomicMax(&sRowCap[rho], c == tid ? cb0 : __float_as_uint(__fadd_rn(cap[c], 0.0f)));
+  }
+  __syncthreads();
+  for (int c = tid; c < d.cells; c += blockDim.x) {
+    const int rho = c / d.B;
+    const bool ok = c == tid ? ok0 : tail[c] <= set.slo[rho >> 2];
+    const uint32_t cb = c == tid ? cb0 : __float_as_uint(__fadd_rn(cap[c], 0.0f));
+    if (ok && cb == sRowCap[rho]) atomicMin(&sRowBin[rho], (uint32_t)(c - rho * d.B));
   }
   __syncthreads();
   for (int rho = tid; rho < d.K4; rho += blockDim.x) {
-    const unsigned long long key = sKey[rho];
-    const int bb = key ? (int)(0xFFFFFFFFu - (uint32_t)key) : -1;
-    const float best = key ? __uint_as_float((uint32_t)(key >> 32)) : 0.0f;
+    const uint32_t bin = sRowBin[rho];
+    const int bb = bin != ~0u ? (int)bin : -1;
+    const float best = bb >= 0 ? __uint_as_float(sRowCap[rho]) : 0.0f;
     sC[rho] = best;
     sB[rho] = bb;
     const int i = rho >> 2, j = rho & 3;
