@@ -301,6 +301,55 @@ def cpu_baseline(w, seconds_target: float = 15.0):
             "candidate_scores_per_s": n / dt}
 
 
+def _oracle_worker(widx, lo, hi, reps, barrier, out):
+    """One oracle instance on candidates [lo, hi) of workload widx, `reps` passes,
+    timed from a barrier shared with the other instances."""
+    import oracle
+
+    w = workloads.make_workload(widx)
+    qn = oracle.triangular_table(4096)
+    oracle.score(w, qn, candidates=w.candidates[lo:lo + 1])  # the library is loaded before the start
+    barrier.wait(timeout=600)
+    t0 = time.monotonic()
+    for _ in range(reps):
+        oracle.score(w, qn, candidates=w.candidates[lo:hi])
+    out.put((t0, time.monotonic()))
+
+
+def cpu_baseline_all_cores(widx: int, w, seconds_per_candidate: float, seconds_target: float = 10.0):
+    """Independent oracle instances, one process per core this process may use,
+    over contiguous candidate ranges of the same workload: the harness's
+    parallelism (the oracle itself stays single-threaded). Processes are
+    spawned, not forked (the CUDA context exists by now)."""
+    import multiprocessing as mp
+    import queue
+
+    n = len(w.candidates)
+    k = max(1, min(len(os.sched_getaffinity(0)), n))
+    bounds = [(i * n // k, (i + 1) * n // k) for i in range(k)]
+    per = max(hi - lo for lo, hi in bounds)
+    reps = max(1, int(round(seconds_target / max(seconds_per_candidate * per, 1e-6))))
+    ctx = mp.get_context("spawn")
+    barrier, out = ctx.Barrier(k), ctx.Queue()
+    procs = [ctx.Process(target=_oracle_worker, args=(widx, lo, hi, reps, barrier, out), daemon=True)
+             for lo, hi in bounds]
+    for p in procs:
+        p.start()
+    try:
+        spans = [out.get(timeout=900) for _ in procs]
+    except queue.Empty:
+        return {"unavailable": "an oracle process did not report within 900 s"}
+    finally:
+        for p in procs:
+            p.join(timeout=60)
+    wall = max(e for _, e in spans) - min(b for b, _ in spans)
+    scen = n * w.O * w.S * reps
+    return {"value": 2 * scen / wall, "unit": UNIT, "cores": k, "kind": "oracle",
+            "sample": f"all {n} candidates x {reps} passes, {k} processes over contiguous candidate "
+                      f"ranges ({wall:.3f} s)",
+            "candidate_scores_per_s": n * reps / wall}
+
+
 def run_reference(args, w, rank):
     if rank != 0:
         return 0
@@ -342,6 +391,7 @@ def main(argv=None):
     ap.add_argument("--workload", type=int, default=1)
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-all-cores", action="store_true", help="skip the all-cores oracle run")
     ap.add_argument("--no-other-workloads", action="store_true")
     args = ap.parse_args(argv)
     if args.warmup < 3:
@@ -465,6 +515,8 @@ def main(argv=None):
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(w)
+        if not args.no_all_cores:
+            cpu["all_cores"] = cpu_baseline_all_cores(args.workload, w, 1.0 / cpu["candidate_scores_per_s"])
     # the mid and large workloads, for the kernel's efficiency at scale (not the headline)
     others = []
     if world == 1 and args.workload == 1 and not args.no_other_workloads:

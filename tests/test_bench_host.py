@@ -105,3 +105,22 @@ def test_roofline_traffic_only_for_the_profiled_source(tmp_path, monkeypatch):
     assert bench._profiled_traffic(2) is None  # no summary for that workload
     (csrc / "fs_score.cu").write_bytes(src + b"\n")
     assert bench._profiled_traffic(1) is None
+
+
+def test_all_cores_oracle_baseline_counts_every_scenario():
+    """The all-cores CPU baseline: one spawned oracle process per usable core
+    over contiguous candidate ranges; its rate counts every scenario of every
+    pass once."""
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2608_19659_gb300 import workloads
+
+    w = workloads.make_workload(0)
+    r = bench.cpu_baseline_all_cores(0, w, seconds_per_candidate=0.02, seconds_target=0.2)
+    assert "unavailable" not in r, r
+    k = min(len(os.sched_getaffinity(0)), len(w.candidates))
+    assert r["cores"] == k and r["kind"] == "oracle" and r["value"] > 0
+    reps = int(r["sample"].split(" x ")[1].split()[0])
+    wall = float(r["sample"].rsplit("(", 1)[1].split(" s")[0])
+    assert reps >= 1 and wall > 0
+    assert abs(r["value"] - 2 * len(w.candidates) * w.O * w.S * reps / wall) <= 0.06 * r["value"]
