@@ -179,7 +179,9 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
       atomicOr(reinterpret_cast<unsigned int*>(&sMisc[2 + (i >> 5)]), 1u << (i & 31));
       if (M >= 1) {
         // first fulfilment that is positive and at or above the class's floor
-        n0 = min_replicas(FL ? fmaxf(sDl[i], __int_as_float(1)) : __int_as_float(1), best, lam, rl, Mf);
+        // (n = 1 unless one replica falls short of it)
+        const float lo_f = FL ? fmaxf(sDl[i], __int_as_float(1)) : __int_as_float(1);
+        n0 = fulfil_r(1.0f, best, lam, rl) >= lo_f ? 1 : min_replicas(lo_f, best, lam, rl, Mf);
         if (n0) {
           const int ns = min_replicas(1.0f, best, lam, rl, Mf);   // first full fulfilment
           len = ns ? ns : M;
@@ -320,8 +322,13 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
       const int most = max(max(nv[0], nv[1]), max(nv[2], nv[3]));
       for (int step = most ? 1 << (31 - __clz(most)) : 0; step > 0; step >>= 1) {
 #pragma unroll
-        for (int j = 0; j < 4; ++j)
-          if (q[j] + step <= nv[j] && sOwn[beg[j] + q[j] + step - 1] < tc) q[j] += step;
+        for (int j = 0; j < 4; ++j) {
+          // the four loads are issued unconditionally: the index is clamped to
+          // the row's last value, at most total - 1 (an empty row reads the word
+          // before its start, at worst the last class minimum: scratch either way)
+          const float v = sOwn[beg[j] + min(q[j] + step, nv[j]) - 1];
+          q[j] += (q[j] + step <= nv[j]) & (v < tc) ? step : 0;
+        }
       }
       int cm = kCostInf;
 #pragma unroll
