@@ -95,7 +95,8 @@ struct Set {
   uint32_t* status;
   unsigned long long* work;  // [2] chunk counter, reduction ticket; zeroed by k_prep
   const int* skip;      // [P] or nullptr: base solves skip problems with skip[p] >= 0
-  int* rtab;            // [P][2][kRowTabMax] or nullptr: row tables of the scoring solves
+  int* rtab;            // [P][2][kRowTabMax] or nullptr: row tables of the scoring solves,
+                        // word (row rho, threshold k) at k K4 + rho
 };
 
 // Scenario plan shared by a launch.

@@ -284,16 +284,34 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
   if (early) pdl_wait();  // thresholds and rows come from k_solve
 
   const size_t ps = (size_t)p * 2 + sigma;
-  const int total = set.ntheta[ps];
   const float* th_g = set.theta + ps * d.theta_cap;
-  // the base solve's row table, this candidate's row of it, when it built one
-  const bool rtab = set.rtab != nullptr && d.K4 * total <= kRowTabMax;
-  const int* rt_g = rtab ? set.rtab + ps * kRowTabMax + (size_t)rr * total : nullptr;
+  // this candidate's row of the base solve's row table (word k at k K4), when
+  // the solve built one; with at most one threshold per thread and a table
+  // that holds every threshold the model allows, each thread loads its
+  // threshold and word together with the count (one memory round trip; the
+  // entries past the count are never used)
+  const int* rt_g = set.rtab ? set.rtab + ps * kRowTabMax + rr : nullptr;
+  const bool ahead = d.theta_cap <= (int)blockDim.x && d.K4 * d.theta_cap <= kRowTabMax;
+  float th_a = 0.0f;
+  int rt_a = 0;
+  if (ahead && tid < d.theta_cap) {
+    th_a = th_g[tid];
+    if (rt_g) rt_a = rt_g[(size_t)tid * d.K4];
+  }
+  const int total = set.ntheta[ps];
+  const bool rtab = rt_g != nullptr && d.K4 * total <= kRowTabMax;
   int* sRt = reinterpret_cast<int*>(sTh + d.theta_cap);  // [min(theta_cap, kRowTabMax / 4)]
   for (int rho = tid; rho < d.K4; rho += blockDim.x) sC[rho] = set.rowC[ps * d.K4 + rho];
-  for (int k = tid; k < total; k += blockDim.x) {
-    sTh[k] = th_g[k];
-    if (rtab) sRt[k] = rt_g[k];
+  if (ahead) {
+    if (tid < total) {
+      sTh[tid] = th_a;
+      if (rtab) sRt[tid] = rt_a;  // (the words' shared array exists only with a table)
+    }
+  } else {
+    for (int k = tid; k < total; k += blockDim.x) {
+      sTh[k] = th_g[k];
+      if (rtab) sRt[k] = rt_g[(size_t)k * d.K4];
+    }
   }
   __syncthreads();
   const float cx = s_cx, cmax = s_cmax;

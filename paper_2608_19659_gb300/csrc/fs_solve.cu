@@ -297,7 +297,8 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   if (row_table) {
     // Row table of a scoring solve: every row's cover cost at every threshold,
     // then per (row rho, threshold k) the word the per-candidate preparation
-    // reads for a candidate in row rho: bits 0-15 the replicas rho may use
+    // reads for a candidate in row rho (stored threshold-major, at k K4 + rho,
+    // so that its address does not depend on the number of thresholds): bits 0-15 the replicas rho may use
     // once the other classes are covered (0 if one cannot be), bit 16 set if
     // another row of rho's class covers theta_k within that budget.
     //
@@ -359,7 +360,7 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
         const int own = sCmin[x];
         const int rest = sum - (own >= kCostInf ? (1 << 24) : own);
         const int A = (rest >> 24) ? -1 : d.G - rest;
-        int c[4];
+        int c[4], wd[4];
 #pragma unroll
         for (int j = 0; j < 4; ++j) c[j] = sCost[(4 * i + j) * total + k];
 #pragma unroll
@@ -369,8 +370,10 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
           for (int q = 0; q < 4; ++q)
             if (q != j) other = min(other, c[q]);
           const int m = A >= (1 << j) ? min(A >> j, d.M[j]) : 0;
-          rt[(4 * i + j) * total + k] = m | ((other < kCostInf && other <= A) ? 1 << 16 : 0);
+          wd[j] = m | ((other < kCostInf && other <= A) ? 1 << 16 : 0);
         }
+        // threshold-major: word (rho, k) at k K4 + rho, the class's four in one 16-byte store
+        *reinterpret_cast<int4*>(rt + (size_t)k * d.K4 + 4 * i) = make_int4(wd[0], wd[1], wd[2], wd[3]);
       }
       cnt += __syncthreads_count(fits);
     }
