@@ -257,3 +257,27 @@ def test_table_path_with_floors(fsb, cuda, oracle_lib, qn):
         r = fsb.fs_score_candidates(m, w.candidates, w.O, w.S, w.seed)
     ref = oracle_lib.score(w, qn)
     assert np.array_equal(r.sum_eo, ref.sum_eo) and r.best == ref.best
+
+
+@pytest.mark.parametrize("K,B,G", [
+    (1, 2, 1000),   # row table on both realisations (7500 words)
+    (1, 3, 1200),   # row table on one realisation only (6600 and 9000 words)
+    (2, 3, 400),    # no row table (9752 and 8712 words): the preparation searches
+    (8, 2, 64),     # eight classes, row table of 7968 words
+])
+def test_score_with_floors_near_row_table_limit(fsb, cuda, oracle_lib, qn, K, B, G):
+    """Floors on problems at the base solve's row-table limit: the floor variants
+    of the table's costs, counts and kappa walks, and of the search without it."""
+    from test_gpu_score_sweep import _contested
+
+    rng = np.random.default_rng(K * 7919 + B * 31 + G + 5)
+    w = _contested(oracle_lib, workloads.random_small(rng, K, B, G))
+    w = dataclasses.replace(w, floor=_floors(rng, w, w.cap_lo, w.tail_hi, p_crit=1.0))
+    assert np.any(w.floor > 0)
+    cells = K * 4 * B
+    cand = np.sort(rng.choice(cells, size=min(16, cells), replace=False)).astype(np.int32)
+    with load_model(fsb, w) as m:
+        r = fsb.fs_score_candidates(m, cand, 2, 16, 91, 4, 2)
+    ref = oracle_lib.score(w, qn, candidates=cand, seed=91, stream_id=4, rnd=2, O=2, S=16)
+    assert np.array_equal(r.sum_eo, ref.sum_eo) and np.array_equal(r.score, ref.score)
+    assert r.gamma_t == ref.gamma_t and r.best == ref.best
