@@ -863,6 +863,9 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
   (void)it;
 
   pdl_wait();  // records, zeroed sums and the zeroed counter come from k_prep
+  // the reduction kernel may be placed now: it waits for this grid to complete
+  // before it reads anything
+  pdl_trigger();
   const int g = (int)gridDim.x;
   int next = 0;  // thread 0: the chunk to stage next
   if (tid == 0) {
@@ -1032,7 +1035,6 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
       return;
     }
   }
-  pdl_trigger();
 }
 
 __global__ void k_finalize(Set set, Items it, Plan pl, const uint64_t* sums, double* gap, double* score,
