@@ -26,6 +26,10 @@
 //
 // k_prep builds, per (candidate, realisation), the part of that table a
 // scenario can reach: Theta entries with kappa in (Cexcl, max(Cexcl, cap_hi_e)].
+// m(t) and "P(t) <= A(t)" depend only on (r, t): a scoring solve tabulates
+// them per realisation (the row table, k_solve), and k_prep then finds the
+// range's ends as counts of feasible thresholds and each kappa by one thread;
+// without a table it searches, evaluating the rows per probe.
 // It also maps each outcome's quantile stratum into the candidate's capacity
 // interval and records where the stratum's tail values stop passing the SLO
 // (the map is monotone, so the gate of Eq. 5 is a position test).
