@@ -406,10 +406,6 @@ int fs_load_model(const fs_bounds* b, const float* slo, const float* demand, int
   d.Q = Q;
   d.cells = cells;
   d.K4 = 4 * K;
-  for (int j = 0; j < kT; ++j) {
-    d.M[j] = G >> j;
-    d.Mf[j] = (float)(G >> j);
-  }
   d.theta_cap = (int)theta_cap;
   d.lcap = 4;
   while (d.lcap < d.theta_cap + 1) d.lcap <<= 1;

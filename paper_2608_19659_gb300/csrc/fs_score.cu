@@ -69,7 +69,7 @@ __device__ __forceinline__ Eval group_eval_excl(float t, const float* sC, const 
     int cost = kCostInf;
     if (rho < d.K4 && rho != rr) {
       const float tc = FL ? fmaxf(t, sDl[rho >> 2]) : t;
-      const int n = min_replicas(tc, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[rho & 3]);
+      const int n = min_replicas(tc, sC[rho], sLam[rho >> 2], sRl[rho >> 2], rep_capf(d, rho & 3));
       if (n) cost = n << (rho & 3);
     }
     cost = min(cost, __shfl_xor_sync(0xffffffffu, cost, 1));
@@ -89,7 +89,7 @@ __device__ __forceinline__ Eval group_eval_excl(float t, const float* sC, const 
 }
 
 __device__ __forceinline__ int replicas_left(const Eval& e, int jr, const Dims& d) {
-  return (e.A >= (1 << jr)) ? min(e.A >> jr, d.M[jr]) : 0;
+  return (e.A >= (1 << jr)) ? min(e.A >> jr, rep_cap(d, jr)) : 0;
 }
 
 // te = max(t, delta_{i_e}): the fulfilment row r must reach
@@ -161,7 +161,7 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
   __shared__ float sLam[FS_MAX_CLASSES], sRl[FS_MAX_CLASSES];  // demand and RN(1/demand)
   __shared__ float sDl[FS_MAX_CLASSES];                          // floor delta_i (0: not critical)
   __shared__ int s_res[2][kPrepThreads / 4];
-  const Dims& d = set.d;  // kernel-parameter space: d.M[j] reads need no local copy
+  const Dims& d = set.d;  // kernel-parameter space: no local copy
   const int item = blockIdx.x >> 1, sigma = blockIdx.x & 1;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = blockDim.x >> 5;
   if (!early) pdl_wait();
@@ -319,7 +319,7 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
   }
   __syncthreads();
   const float cx = s_cx, cmax = s_cmax;
-  const int msent = d.K == 1 ? d.M[jr] : 0;  // above every threshold only a lone class can go on
+  const int msent = d.K == 1 ? rep_cap(d, jr) : 0;  // above every threshold only a lone class can go on
 
   // b0: last index feasible at Cexcl; b1: last index feasible at max(Cexcl, cap_hi).
   // Feasibility is nonincreasing along the sorted thresholds, so with the row
@@ -561,7 +561,7 @@ __device__ int dump_cover(float t, const Set& set, size_t ps, int rr, float C, i
     const float c = rho == rr ? C : set.rowC[ps * d.K4 + rho];
     const int b = rho == rr ? bC : set.rowB[ps * d.K4 + rho];
     if (b < 0) continue;
-    const int n = min_replicas(t, c, set.lam[i], __frcp_rn(set.lam[i]), d.Mf[j]);
+    const int n = min_replicas(t, c, set.lam[i], __frcp_rn(set.lam[i]), rep_capf(d, j));
     if (n && (n << j) < best) {
       best = n << j;
       bj = j;
@@ -862,7 +862,7 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
   uint2* gtab2 = reinterpret_cast<uint2*>(smraw + 16 + (size_t)2 * stage_floats * 4);
   // per stage: chunk index, its segment and its part (thread 0 divides once)
   __shared__ int s_chunk[2], s_seg[2], s_part[2];
-  const Dims& d = set.d;  // kernel-parameter space: d.M[j] reads need no local copy
+  const Dims& d = set.d;  // kernel-parameter space: no local copy
   const int tid = threadIdx.x, lane = tid & 31;
   (void)it;
 

@@ -67,7 +67,7 @@ __device__ __forceinline__ int group_total_cost(float t, const float* sC, const 
     if (rho < d.K4) {
       const int j = rho & 3;
       const float tc = FL ? fmaxf(t, sDl[rho >> 2]) : t;
-      const int n = min_replicas(tc, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[j]);
+      const int n = min_replicas(tc, sC[rho], sLam[rho >> 2], sRl[rho >> 2], rep_capf(d, j));
       if (n) cost = n << j;
     }
     cost = min(cost, __shfl_xor_sync(0xffffffffu, cost, 1));
@@ -90,7 +90,7 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   // thresholds, and without floors skips it
   const bool choice = FL || (mode & 2) == 0;
   extern __shared__ __align__(16) unsigned char smraw[];
-  const Dims& d = set.d;  // kernel-parameter space: d.M[j] reads need no local copy
+  const Dims& d = set.d;  // kernel-parameter space: no local copy
   const int r = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   pdl_trigger();
@@ -172,8 +172,8 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
     sB[rho] = bb;
     const int i = rho >> 2, j = rho & 3;
     const float lam = sLam[i], rl = sRl[i];
-    const int M = d.M[j];
-    const float Mf = d.Mf[j];
+    const int M = rep_cap(d, j);
+    const float Mf = rep_capf(d, j);
     int n0 = 0, len = 0;
     if (bb >= 0) {
       atomicOr(reinterpret_cast<unsigned int*>(&sMisc[2 + (i >> 5)]), 1u << (i & 31));
@@ -369,7 +369,7 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
 #pragma unroll
           for (int q = 0; q < 4; ++q)
             if (q != j) other = min(other, c[q]);
-          const int m = A >= (1 << j) ? min(A >> j, d.M[j]) : 0;
+          const int m = A >= (1 << j) ? min(A >> j, rep_cap(d, j)) : 0;
           wd[j] = m | ((other < kCostInf && other <= A) ? 1 << 16 : 0);
         }
         // threshold-major: word (rho, k) at k K4 + rho, the class's four in one 16-byte store
@@ -415,11 +415,11 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
       if (rho < d.K4) {
         const float dl = FL ? sDl[rho >> 2] : 0.0f;
         if (tstar > 0.0f) {
-          const int n = min_replicas(FL ? fmaxf(tstar, dl) : tstar, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[rho & 3]);
+          const int n = min_replicas(FL ? fmaxf(tstar, dl) : tstar, sC[rho], sLam[rho >> 2], sRl[rho >> 2], rep_capf(d, rho & 3));
           if (n) key = ((n << (rho & 3)) << 2) | (rho & 3);
         }
         if (FL && dl > 0.0f) {
-          const int n = min_replicas(dl, sC[rho], sLam[rho >> 2], sRl[rho >> 2], d.Mf[rho & 3]);
+          const int n = min_replicas(dl, sC[rho], sLam[rho >> 2], sRl[rho >> 2], rep_capf(d, rho & 3));
           if (n) keyf = ((n << (rho & 3)) << 2) | (rho & 3);
         }
       }

@@ -99,10 +99,6 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
   d.Q = Q;
   d.cells = K * 4 * B;
   d.K4 = 4 * K;
-  for (int j = 0; j < kT; ++j) {
-    d.M[j] = G >> j;
-    d.Mf[j] = (float)(G >> j);
-  }
   d.theta_cap = (int)theta_cap;
   d.lcap = 4;
   while (d.lcap < d.theta_cap + 1) d.lcap <<= 1;
