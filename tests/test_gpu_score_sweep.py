@@ -82,6 +82,8 @@ def test_random_small_problems(fsb, cuda, oracle_lib, seed):
     (1, 2, 1000, 16),   # 1875 thresholds: row table of 7500 words, several passes per count
     (1, 3, 1200, 16),   # row table on one realisation only (6600 and 9000 words)
     (8, 2, 64, 24),     # eight classes, row table of 7968 words
+    (2, 3, 69, 24),     # theta_cap = 256: the preparation loads its row words with their count
+    (2, 3, 70, 24),     # theta_cap = 260: it reads the count first
 ])
 def test_extreme_sizes(fsb, cuda, oracle_lib, K, B, G, n_cand):
     rng = np.random.default_rng(K * 7919 + B * 31 + G)
