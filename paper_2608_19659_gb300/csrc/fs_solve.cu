@@ -415,7 +415,8 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
       if (rho < d.K4) {
         const float dl = FL ? sDl[rho >> 2] : 0.0f;
         if (tstar > 0.0f) {
-          const int n = min_replicas(FL ? fmaxf(tstar, dl) : tstar, sC[rho], sLam[rho >> 2], sRl[rho >> 2], rep_capf(d, rho & 3));
+          const int n = min_replicas(FL ? fmaxf(tstar, dl) : tstar, sC[rho], sLam[rho >> 2], sRl[rho >> 2],
+                                     rep_capf(d, rho & 3));
           if (n) key = ((n << (rho & 3)) << 2) | (rho & 3);
         }
         if (FL && dl > 0.0f) {
