@@ -297,10 +297,11 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   if (row_table) {
     // Row table of a scoring solve: every row's cover cost at every threshold,
     // then per (row rho, threshold k) the word the per-candidate preparation
-    // reads for a candidate in row rho (stored threshold-major, at k K4 + rho,
-    // so that its address does not depend on the number of thresholds): bits 0-15 the replicas rho may use
-    // once the other classes are covered (0 if one cannot be), bit 16 set if
-    // another row of rho's class covers theta_k within that budget.
+    // reads for a candidate in row rho, stored threshold-major at k K4 + rho (its
+    // address does not depend on the number of thresholds): bits 0-15 the
+    // replicas rho may use once the other classes are covered (0 if one cannot
+    // be), bit 16 set if another row of rho's class covers theta_k within that
+    // budget.
     //
     // A row's cheapest cover of t (class i covers max(t, delta_i)) is n0 plus
     // the number of its own values f(n0) <= ... <= f(len) below t: every n
