@@ -83,6 +83,12 @@ def lib():
                                   C.c_uint64, C.c_uint32, C.c_uint32, C.c_int, ip, C.c_int,
                                   C.c_int, C.c_int, C.POINTER(C.c_int64), C.POINTER(C.c_double),
                                   C.POINTER(C.c_double), C.POINTER(C.c_int64), fp, ip, fp]
+        _lib.or_score_cached.argtypes = [C.POINTER(_Problem), fp, fp, fp, fp, fp, C.c_int,
+                                         C.c_uint64, C.c_uint32, C.c_uint32, C.c_int, ip, C.c_int,
+                                         C.c_int, C.c_int, C.POINTER(C.c_int64), fp]
+        _lib.or_reduce.argtypes = [C.POINTER(_Problem), C.c_int, ip, C.c_int, C.c_int, C.c_float,
+                                   C.POINTER(C.c_int64), C.POINTER(C.c_double),
+                                   C.POINTER(C.c_double), C.POINTER(C.c_int64), ip]
         _lib.or_certificate.argtypes = [C.POINTER(_Problem), fp, fp, fp, fp,
                                         C.POINTER(C.c_uint8), C.c_float, C.c_int,
                                         C.POINTER(C.c_int), fp]
@@ -254,6 +260,51 @@ def score(w, qn, candidates=None, solver=SOLVER_FRONTIER, dump=False, seed=None,
     if rc:
         raise ValueError(f"oracle score failed ({rc})")
     return ScoreResult(sum_eo, gap, sc, scf, float(np.float32(gt.value)), int(best.value), dt)
+
+
+def score_sums_cached(w, qn, candidates=None, solver=SOLVER_FRONTIER, seed=None,
+                      stream_id=None, rnd=None, O=None, S=None):
+    """Fixed-point sums [n_cand, O] of :func:`score` and Gamma_t, with each
+    candidate's solves cached by (capacity position, tail within SLO); the
+    same values as :func:`score`, for workloads too large for it."""
+    prob = Problem.of(w)
+    b = _bounds(w)
+    qn = _f32(qn)
+    cand = np.ascontiguousarray(w.candidates if candidates is None else candidates, np.int32)
+    O = w.O if O is None else O
+    S = w.S if S is None else S
+    sum_eo = np.zeros((cand.size, O), np.int64)
+    gt = C.c_float()
+    rc = lib().or_score_cached(C.byref(prob._s), *[_ptr(x, C.c_float) for x in b],
+                               _ptr(qn, C.c_float), qn.size,
+                               w.seed if seed is None else seed,
+                               w.stream_id if stream_id is None else stream_id,
+                               w.round if rnd is None else rnd, cand.size, _ptr(cand, C.c_int32),
+                               O, S, solver, _ptr(sum_eo, C.c_int64), C.byref(gt))
+    if rc:
+        raise ValueError(f"oracle cached score failed ({rc})")
+    return sum_eo, float(np.float32(gt.value))
+
+
+def reduce_sums(w, candidates, sum_eo, gamma_t, O=None, S=None) -> ScoreResult:
+    """E[Gamma_{t+1} | e], scores and the argmax from fixed-point sums."""
+    prob = Problem.of(w)
+    cand = np.ascontiguousarray(candidates, np.int32)
+    se = np.ascontiguousarray(sum_eo, np.int64)
+    O = w.O if O is None else O
+    S = w.S if S is None else S
+    assert se.shape == (cand.size, O)
+    n = cand.size
+    gap = np.zeros(n, np.float64)
+    sc = np.zeros(n, np.float64)
+    scf = np.zeros(n, np.int64)
+    best = C.c_int32()
+    rc = lib().or_reduce(C.byref(prob._s), n, _ptr(cand, C.c_int32), O, S, gamma_t,
+                         _ptr(se, C.c_int64), _ptr(gap, C.c_double), _ptr(sc, C.c_double),
+                         _ptr(scf, C.c_int64), C.byref(best))
+    if rc:
+        raise ValueError("oracle reduce failed")
+    return ScoreResult(se.copy(), gap, sc, scf, float(np.float32(gamma_t)), int(best.value), None)
 
 
 def certificate(prob: Problem, cap_lo, cap_hi, tail_lo, tail_hi, revealed, eps,

@@ -148,6 +148,113 @@ int or_score(const or_problem *p, const float *cap_lo, const float *cap_hi,
 }
 
 /*
+ * Section 4.3, the last step: from the fixed-point sums of every
+ * (candidate, outcome) pair, E[Gamma_{t+1} | e] = sum g 2^-40 / (O S), the
+ * score E[Gamma_t - Gamma_{t+1} | e] and the argmax (largest score, then
+ * fewer profiling GPU-seconds, i.e. lower TP, then earlier position). The
+ * same rules as at the end of or_score, applied to sums computed elsewhere
+ * (by or_score_cached over disjoint candidate ranges).
+ */
+int or_reduce(const or_problem *p, int n_cand, const int32_t *cand, int O, int S, float gamma_t,
+              const int64_t *sum_eo, double *gap, double *score, int64_t *score_fixed, int32_t *best)
+{
+    if (n_cand < 0 || O < 1 || S < 1) return -1;
+    const int64_t g_t = llrintf(gamma_t * 0x1p40f);
+    const int64_t n = (int64_t)O * S;
+    int best_e = -1;
+    int64_t best_sc = 0;
+    for (int e = 0; e < n_cand; ++e) {
+        int64_t tot = 0;
+        for (int o = 0; o < O; ++o) tot += sum_eo[(size_t)e * O + o];
+        int64_t sc = g_t * n - tot;
+        if (gap) gap[e] = ((double)tot * 0x1p-40) / (double)n;
+        if (score) score[e] = ((double)sc * 0x1p-40) / (double)n;
+        if (score_fixed) score_fixed[e] = sc;
+        int j = (cand[e] / p->B) % OR_T;
+        if (best_e < 0 || sc > best_sc ||
+            (sc == best_sc && j < (cand[best_e] / p->B) % OR_T)) {
+            best_e = e;
+            best_sc = sc;
+        }
+    }
+    if (best) *best = best_e >= 0 ? cand[best_e] : -1;
+    return 0;
+}
+
+/*
+ * The fixed-point sums of or_score, scenario for scenario, with each
+ * candidate's solves cached. Both solvers read a cell's tail only through
+ * the SLO test tail <= L_i (Eq. 5), and c_y is a function of the capacity
+ * position k_cap alone, so a scenario's two allocations, and its Gamma',
+ * depend on its draw only through the pair (k_cap, l_y <= L_i). A scenario
+ * whose pair was met before in the same candidate reuses that scenario's
+ * rint(Gamma' 2^40); every other step (draws, maps, patches, solves, sums)
+ * is or_score's. Used to compute expected sums of workloads too large for
+ * or_score; the tests hold the two equal wherever or_score finishes.
+ * sum_eo [n_cand][O] is required; gamma_t receives Gamma_t.
+ */
+int or_score_cached(const or_problem *p, const float *cap_lo, const float *cap_hi,
+                    const float *tail_lo, const float *tail_hi, const float *qn, int Q,
+                    uint64_t seed, uint32_t stream_id, uint32_t round,
+                    int n_cand, const int32_t *cand, int O, int S, int solver,
+                    int64_t *sum_eo, float *gamma_t)
+{
+    if (n_cand < 0 || O < 1 || S < 1 || Q < 1 || Q % O != 0 || !sum_eo) return -1;
+    if ((int64_t)O * S > ((int64_t)1 << 22)) return -1;
+    int cells = cells_of(p);
+    for (int e = 0; e < n_cand; ++e)
+        if (cand[e] < 0 || cand[e] >= cells) return -1;
+
+    or_alloc am, ap;
+    float gt;
+    int rc = or_base_gap(p, cap_lo, cap_hi, tail_lo, tail_hi, solver, &am, &ap, &gt);
+    if (rc) return rc;
+    if (gamma_t) *gamma_t = gt;
+
+    float *cm = (float *)malloc(sizeof(float) * cells * 4);
+    int64_t *memo = (int64_t *)malloc(sizeof(int64_t) * 2 * (size_t)Q);
+    uint8_t *known = (uint8_t *)malloc(2 * (size_t)Q);
+    if (!cm || !memo || !known) { free(cm); free(memo); free(known); return -2; }
+    float *tm = cm + cells, *cp = cm + 2 * cells, *tp = cm + 3 * cells;
+    memcpy(cm, cap_lo, sizeof(float) * cells);
+    memcpy(tm, tail_hi, sizeof(float) * cells);
+    memcpy(cp, cap_hi, sizeof(float) * cells);
+    memcpy(tp, tail_lo, sizeof(float) * cells);
+
+    for (int e = 0; e < n_cand; ++e) {
+        const int32_t cell = cand[e];
+        const float L = p->slo[cell / (OR_T * p->B)];
+        memset(known, 0, 2 * (size_t)Q);
+        for (int o = 0; o < O; ++o) {
+            int64_t acc = 0;
+            for (int s = 0; s < S; ++s) {
+                int32_t kc, kl;
+                or_draw_index(seed, stream_id, round, cell, Q, O, o, s, &kc, &kl);
+                float cy = or_map(cap_lo[cell], cap_hi[cell], qn[kc]);
+                float ly = or_map(tail_lo[cell], tail_hi[cell], qn[kl]);
+                size_t key = 2 * (size_t)kc + (ly <= L ? 1u : 0u);
+                if (!known[key]) {
+                    cm[cell] = cy; tm[cell] = ly;
+                    cp[cell] = cy; tp[cell] = ly;
+                    rc = solve(p, cm, tm, solver, &am);
+                    if (!rc) rc = solve(p, cp, tp, solver, &ap);
+                    if (rc) { free(cm); free(memo); free(known); return rc; }
+                    float g = ap.t_star - am.t_star;
+                    memo[key] = llrintf(g * 0x1p40f);
+                    known[key] = 1;
+                }
+                acc += memo[key];
+            }
+            sum_eo[(size_t)e * O + o] = acc;
+        }
+        cm[cell] = cap_lo[cell]; tm[cell] = tail_hi[cell];
+        cp[cell] = cap_hi[cell]; tp[cell] = tail_lo[cell];
+    }
+    free(cm); free(memo); free(known);
+    return 0;
+}
+
+/*
  * Section 4.2: certified infeasible when even A+ cannot meet the critical
  * floors; certified feasible when A- meets them, the gap is at most eps and
  * every cell that A- commits replicas to has been measured (its tail upper

@@ -102,6 +102,18 @@ int or_score(const or_problem *p, const float *cap_lo, const float *cap_hi,
              int64_t *sum_eo, double *gap, double *score, int64_t *score_fixed,
              float *gamma_t, int32_t *best, float *dump_t /* [n_cand*O*S*2] or NULL */);
 
+/* The same fixed-point sums with each candidate's solves cached by
+ * (capacity position, tail within SLO); Gamma_t into gamma_t (nullable). */
+int or_score_cached(const or_problem *p, const float *cap_lo, const float *cap_hi,
+                    const float *tail_lo, const float *tail_hi, const float *qn, int Q,
+                    uint64_t seed, uint32_t stream_id, uint32_t round,
+                    int n_cand, const int32_t *cand, int O, int S, int solver,
+                    int64_t *sum_eo /* [n_cand*O] */, float *gamma_t);
+
+/* Expectations, scores and argmax (Section 4.3) from the sums. */
+int or_reduce(const or_problem *p, int n_cand, const int32_t *cand, int O, int S, float gamma_t,
+              const int64_t *sum_eo, double *gap, double *score, int64_t *score_fixed, int32_t *best);
+
 /* Certificate (Section 4.2): 0 undecided, 1 certified feasible, 2 certified
  * infeasible (even A+ misses a critical floor). */
 int or_certificate(const or_problem *p, const float *cap_lo, const float *cap_hi,

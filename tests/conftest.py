@@ -70,3 +70,33 @@ def alloc_matches(gpu: dict, ref, K: int) -> bool:
             and gpu["has_option_mask"] == ref.has_option_mask and gpu["tp"] == ref.tp
             and gpu["bin"] == ref.bin and gpu["replicas"] == ref.replicas
             and [np.float32(x) for x in gpu["fulfil"]] == [np.float32(x) for x in ref.fulfil])
+
+
+def read_expected_sums(name):
+    """An expected-sums file written by tests/golden/make_expected_sums.py:
+    (inputs_sha256, gamma_t, best, cells [n], sum_eo [n, O])."""
+    import numpy as np
+
+    sha = None
+    gamma_t = best = None
+    cells, deficits = [], []
+    S = None
+    with open(os.path.join(GOLDEN, name)) as f:
+        for line in f:
+            if line.startswith("# inputs_sha256"):
+                sha = line.split()[2]
+                continue
+            if not line.strip() or line.startswith("#"):
+                continue
+            t = line.split()
+            if t[0] == "gamma_t":
+                gamma_t = float(np.uint32(int(t[1], 16)).view(np.float32))
+            elif t[0] == "best":
+                best = int(t[1])
+            elif t[0] == "shape":
+                S = int(t[3])
+            else:
+                cells.append(int(t[0]))
+                deficits.append([int(x) for x in t[1:]])
+    full = np.int64(S) * np.int64(np.rint(np.float64(np.float32(gamma_t)) * 2.0**40))
+    return sha, gamma_t, best, np.array(cells, np.int32), full - np.array(deficits, np.int64)

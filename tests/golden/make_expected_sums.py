@@ -1,0 +1,126 @@
+"""Write the oracle's expected fixed-point sums of the large scoring workloads.
+
+Calls only the CPU oracle (``oracle/``) and the seeded input generator
+(``paper_2608_19659_gb300/workloads.py``, inputs only). For every candidate e
+and outcome o of a workload the oracle's Monte-Carlo estimator (Section 4.3:
+draws, patched conservative and optimistic realisations, both allocations
+solved, g = rint(Gamma' 2^40) summed in int64) gives sum_eo[e][o];
+``or_score_cached`` computes the same values as ``or_score`` scenario for
+scenario, reusing a candidate's solves for repeated (capacity position, tail
+within SLO) pairs. Candidates are split into contiguous ranges, one
+single-threaded oracle process per range; the sums do not depend on the split.
+
+Usage: python tests/golden/make_expected_sums.py [--procs N] [name ...]
+with names from WORKLOADS below (default: all). Each file records:
+  * the sha256 of the workload's inputs (bounds, demands, SLOs, candidates),
+  * Gamma_t and the argmax cell,
+  * per candidate the deficits d[e][o] = S rint(Gamma_t 2^40) - sum_eo[e][o]
+    (the fixed-point score of each outcome stratum; 0 for a candidate that
+    cannot change either allocation), so that sum_eo = S rint(Gamma_t 2^40) - d.
+"""
+
+from __future__ import annotations
+
+import argparse
+import dataclasses
+import hashlib
+import multiprocessing as mp
+import os
+import sys
+import time
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+ROOT = os.path.dirname(os.path.dirname(HERE))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+# name -> (workload index, demand factor, output file)
+WORKLOADS = {
+    "large": (3, 1.0, "large_workload_sums.txt"),
+    "mid_x3": (2, 3.0, "mid_workload_x3_sums.txt"),
+}
+
+
+def workload(name):
+    from paper_2608_19659_gb300 import workloads
+
+    idx, factor, _ = WORKLOADS[name]
+    w = workloads.make_workload(idx)
+    if factor != 1.0:
+        w = dataclasses.replace(w, demand=(w.demand * np.float32(factor)).astype(np.float32))
+    return w
+
+
+def input_digest(w) -> str:
+    h = hashlib.sha256()
+    for a in (w.cap_lo, w.cap_hi, w.tail_lo, w.tail_hi, w.demand, w.slo):
+        h.update(np.ascontiguousarray(a, np.float32).tobytes())
+    h.update(np.ascontiguousarray(w.candidates, np.int32).tobytes())
+    h.update(np.array([w.K, w.B, w.G, w.O, w.S, w.seed, w.stream_id, w.round], np.int64).tobytes())
+    return h.hexdigest()
+
+
+def _range_sums(args):
+    name, lo, hi = args
+    import oracle
+
+    w = workload(name)
+    qn = oracle.triangular_table(4096)
+    se, gt = oracle.score_sums_cached(w, qn, candidates=w.candidates[lo:hi])
+    return lo, se, gt
+
+
+def compute(name, procs):
+    import oracle
+
+    w = workload(name)
+    n = len(w.candidates)
+    step = max(1, (n + 4 * procs - 1) // (4 * procs))
+    jobs = [(name, lo, min(n, lo + step)) for lo in range(0, n, step)]
+    sums = np.zeros((n, w.O), np.int64)
+    gts = set()
+    with mp.get_context("spawn").Pool(procs) as pool:
+        for lo, se, gt in pool.imap_unordered(_range_sums, jobs):
+            sums[lo:lo + se.shape[0]] = se
+            gts.add(gt)
+    assert len(gts) == 1
+    gamma_t = gts.pop()
+    res = oracle.reduce_sums(w, w.candidates, sums, gamma_t)
+    return w, sums, res
+
+
+def write(name, w, sums, res):
+    _, _, fname = WORKLOADS[name]
+    full = np.int64(w.S) * np.int64(np.rint(np.float64(np.float32(res.gamma_t)) * 2.0**40))
+    d = full - sums
+    with open(os.path.join(HERE, fname), "w") as f:
+        f.write(f"# Expected fixed-point sums of the oracle's decision-gap estimator (Section 4.3)\n")
+        f.write(f"# workload: {w.name}, demands x{WORKLOADS[name][1]}\n")
+        f.write(f"# written by tests/golden/make_expected_sums.py {name} (oracle/ only)\n")
+        f.write(f"# inputs_sha256 {input_digest(w)}\n")
+        f.write(f"# columns: cell, then O deficits d[o] = S rint(Gamma_t 2^40) - sum_eo[o]\n")
+        f.write(f"gamma_t {np.float32(res.gamma_t).view(np.uint32):08x} {res.gamma_t!r}\n")
+        f.write(f"best {res.best}\n")
+        f.write(f"shape {len(w.candidates)} {w.O} {w.S}\n")
+        for e, cell in enumerate(w.candidates):
+            f.write(f"{int(cell)} " + " ".join(str(int(x)) for x in d[e]) + "\n")
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("names", nargs="*", default=list(WORKLOADS))
+    ap.add_argument("--procs", type=int, default=len(os.sched_getaffinity(0)))
+    a = ap.parse_args()
+    for name in a.names:
+        t0 = time.time()
+        w, sums, res = compute(name, a.procs)
+        write(name, w, sums, res)
+        print(f"{name}: {len(w.candidates)} candidates, Gamma_t {res.gamma_t}, best {res.best}, "
+              f"{int((res.score > 0).sum())} with a positive score, {time.time() - t0:.0f} s "
+              f"on {a.procs} processes")
+
+
+if __name__ == "__main__":
+    main()

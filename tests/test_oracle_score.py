@@ -149,3 +149,39 @@ def test_certificate_requires_known_committed_tails(oracle_lib):
     st, g = oracle_lib.certificate(p, w.cap_lo, w.cap_hi, w.tail_lo, w.tail_hi,
                                    np.ones(w.cells, np.uint8), -1.0)
     assert st == 0
+
+
+@pytest.mark.parametrize("idx,factor,n_cand,S", [(0, 3.0, 16, 256), (1, 1.0, 12, 512), (2, 3.0, 6, 384),
+                                                 (3, 2.0, 3, 96)])
+def test_cached_sums_equal_plain_oracle(oracle_lib, idx, factor, n_cand, S):
+    """The cached scorer reuses a candidate's solves for equal (capacity position,
+    tail within SLO) pairs; its sums, Gamma_t and, through or_reduce, its
+    expectations, scores and argmax equal or_score's on every workload family."""
+    w = workloads.make_workload(idx)
+    w = dataclasses.replace(w, demand=(w.demand * np.float32(factor)).astype(np.float32), S=S)
+    qn = oracle_lib.triangular_table(4096)
+    rng = np.random.default_rng(idx)
+    cand = np.sort(rng.choice(w.candidates, n_cand, replace=False)).astype(np.int32)
+    ref = oracle_lib.score(w, qn, candidates=cand)
+    se, gt = oracle_lib.score_sums_cached(w, qn, candidates=cand)
+    assert gt == ref.gamma_t
+    assert np.array_equal(se, ref.sum_eo)
+    red = oracle_lib.reduce_sums(w, cand, se, gt)
+    assert np.array_equal(red.gap, ref.gap) and np.array_equal(red.score, ref.score)
+    assert np.array_equal(red.score_fixed, ref.score_fixed) and red.best == ref.best
+
+
+def test_cached_sums_with_tail_gate_both_ways(oracle_lib):
+    """Cells whose tail interval straddles the SLO: the cache keys on the gate, and
+    scenarios with the gate open and closed at one capacity position differ."""
+    rng = np.random.default_rng(7)
+    w = workloads.random_small(rng, 2, 3, 10)
+    L = w.slo[:, None, None] * np.ones((w.K, 4, w.B), np.float32)
+    hi = np.where(np.arange(w.cells).reshape(L.shape) % 2 == 1, 1.2, 0.9) * L
+    w = dataclasses.replace(w, tail_lo=(0.8 * L).astype(np.float32), tail_hi=hi.astype(np.float32),
+                            demand=(3 * w.demand).astype(np.float32), O=2, S=64, seed=11)
+    qn = oracle_lib.triangular_table(64)
+    ref = oracle_lib.score(w, qn, solver=LIT)
+    se, gt = oracle_lib.score_sums_cached(w, qn, solver=LIT)
+    assert np.array_equal(se, ref.sum_eo) and gt == ref.gamma_t
+    assert ref.gamma_t > 0 and np.any(ref.score_fixed > 0)
