@@ -1,11 +1,14 @@
 """Benchmark of the GB300 decision-gap scorer.
 
-One step = one fs_score_candidates pass over the paper-scale workload
-(2 classes, TP in {1,2,4,8}, G = 16, 8 load bins; 64 candidates x 8 outcomes x
-4096 samples = 2,097,152 scenarios, each solving the allocation under both
-realisations): base solves, per-candidate tables, the Monte-Carlo kernel and
-the reduction. Inputs are resident in HBM when the timed region starts; L2 is
-flushed (256 MiB write) between timed steps. Prints one JSON line.
+One step = one fs_score_candidates pass over the largest single-GPU scoring
+workload (8 classes, TP in {1,2,4,8}, G = 256, 32 load bins; 1024 candidates x
+16 outcomes x 16384 samples = 268,435,456 scenarios, each solving the
+allocation under both realisations): base solves, per-candidate tables, the
+Monte-Carlo kernel and the reduction. Inputs are resident in HBM when the
+timed region starts; L2 is flushed (256 MiB write) between timed steps. The
+paper-scale and 4-class workloads are reported beside it, and the replay
+workload (Algorithm 1 over 200 reveal orders) is timed wall-clock. Prints one
+JSON line.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload I] [--impl reference]
 
@@ -244,11 +247,12 @@ def other_workload(idx: int, steps: int, warmup: int, alu_peak: float, stream_id
     cand = torch.from_numpy(w.candidates).cuda()
     gap = torch.zeros(n, dtype=torch.float64, device="cuda")
     score = torch.zeros(n, dtype=torch.float64, device="cuda")
+    gt = torch.zeros(1, dtype=torch.float32, device="cuda")
     flush = torch.empty(64 * 1024 * 1024, dtype=torch.float32, device="cuda")
 
     def step():
         fsb.fs_score_candidates_async(m, cand, w.O, w.S, w.seed, stream_id, 0, gap_dev=gap, score_dev=score,
-                                      stream=stream)
+                                      gamma_t_dev=gt, stream=stream)
 
     for _ in range(warmup):
         flush.zero_()
@@ -273,7 +277,11 @@ def other_workload(idx: int, steps: int, warmup: int, alu_peak: float, stream_id
     fsb.fs_free_model(m)
     kern_s = kernel_ms / 1000.0 / max(kernel_n, 1)
     achieved = algorithmic_ops(w) / kern_s
+    gamma_t = float(gt.item())
     return {"workload": w.name, "ms_per_step": step_ms, "scenarios_per_s": w.scenarios / (step_ms / 1000.0),
+            "gamma_t": gamma_t,
+            "note": ("Gamma_t = 0 at these demands (spare capacity): every score is exactly 0, and the "
+                     "Monte-Carlo kernel's tables are empty" if gamma_t == 0.0 else ""),
             "allocation_solves_per_s": 2.0 * w.scenarios / (step_ms / 1000.0),
             "candidate_scores_per_s": n / (step_ms / 1000.0),
             "kernel_ms_per_launch": kern_s * 1000.0,
@@ -282,56 +290,88 @@ def other_workload(idx: int, steps: int, warmup: int, alu_peak: float, stream_id
                          "traffic": _profiled_traffic(idx)}}
 
 
-def cpu_baseline(w, seconds_target: float = 15.0):
-    """The oracle, single-threaded, on the first candidates of the workload (whole O x S each)."""
+def oracle_prefix(w, seconds_target: float):
+    """A deterministic prefix of workload w's scenarios sized to about
+    seconds_target of one core: the first n candidates, every outcome, and
+    samples 0 .. S' - 1 of each (a subset of the workload's own scenarios;
+    S' = S once whole candidates fit). Returns (n, S')."""
     import oracle
 
     qn = oracle.triangular_table(4096)
+    s1 = min(w.S, 32)
     t0 = time.perf_counter()
-    oracle.score(w, qn, candidates=w.candidates[:1])
-    one = time.perf_counter() - t0
-    n = int(max(1, min(len(w.candidates), seconds_target / max(one, 1e-6))))
+    oracle.score(w, qn, candidates=w.candidates[:1], S=s1)
+    per_scen = (time.perf_counter() - t0) / (w.O * s1)
+    s_fit = int(seconds_target / max(per_scen * w.O, 1e-9))
+    if s_fit < w.S:
+        return 1, max(1, s_fit)
+    n = int(max(1, min(len(w.candidates), seconds_target / max(per_scen * w.O * w.S, 1e-9))))
+    return n, w.S
+
+
+def _sample_text(w, n, s_pref):
+    if s_pref == w.S:
+        return f"first {n} of {len(w.candidates)} candidates, all {w.O}x{w.S} scenarios each"
+    return (f"first {n} of {len(w.candidates)} candidates, all {w.O} outcomes, samples 0..{s_pref - 1} of "
+            f"{w.S} per outcome (a prefix of the workload's scenarios; the rate extrapolates to the "
+            f"whole workload, which the oracle would take {len(w.candidates) * w.S / (n * s_pref):.0f}x as long for)")
+
+
+def cpu_baseline(w, seconds_target: float = 15.0):
+    """The oracle, single-threaded, on a deterministic prefix of the workload."""
+    import oracle
+
+    qn = oracle.triangular_table(4096)
+    n, s_pref = oracle_prefix(w, seconds_target)
     t0 = time.perf_counter()
-    oracle.score(w, qn, candidates=w.candidates[:n])
+    oracle.score(w, qn, candidates=w.candidates[:n], S=s_pref)
     dt = time.perf_counter() - t0
-    scen = n * w.O * w.S
+    scen = n * w.O * s_pref
     return {"value": 2 * scen / dt, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"first {n} of {len(w.candidates)} candidates, all {w.O}x{w.S} scenarios each "
-                      f"({scen} scenarios, {dt:.1f} s)",
-            "candidate_scores_per_s": n / dt}
+            "sample": f"{_sample_text(w, n, s_pref)} ({scen} scenarios, {dt:.1f} s)",
+            "candidate_scores_per_s": scen / dt / (w.O * w.S), "prefix": [n, s_pref]}
 
 
-def _oracle_worker(widx, lo, hi, reps, barrier, out):
-    """One oracle instance on candidates [lo, hi) of workload widx, `reps` passes,
-    timed from a barrier shared with the other instances."""
+def _oracle_worker(widx, lo, hi, s_pref, reps, barrier, out):
+    """One oracle instance on candidates [lo, hi) of workload widx (samples
+    0 .. s_pref - 1 of every outcome), `reps` passes, timed from a barrier
+    shared with the other instances."""
     import oracle
 
     w = workloads.make_workload(widx)
     qn = oracle.triangular_table(4096)
-    oracle.score(w, qn, candidates=w.candidates[lo:lo + 1])  # the library is loaded before the start
+    oracle.score(w, qn, candidates=w.candidates[lo:lo + 1], S=1)  # the library is loaded before the start
     barrier.wait(timeout=600)
     t0 = time.monotonic()
     for _ in range(reps):
-        oracle.score(w, qn, candidates=w.candidates[lo:hi])
+        oracle.score(w, qn, candidates=w.candidates[lo:hi], S=s_pref)
     out.put((t0, time.monotonic()))
 
 
-def cpu_baseline_all_cores(widx: int, w, seconds_per_candidate: float, seconds_target: float = 10.0):
+def cpu_baseline_all_cores(widx: int, w, seconds_per_scenario: float, seconds_target: float = 10.0):
     """Independent oracle instances, one process per core this process may use,
     over contiguous candidate ranges of the same workload: the harness's
-    parallelism (the oracle itself stays single-threaded). Processes are
-    spawned, not forked (the CUDA context exists by now)."""
+    parallelism (the oracle itself stays single-threaded). Each instance takes
+    the same prefix of samples per outcome as the single-core run, sized so
+    that the run lasts about seconds_target. Processes are spawned, not forked
+    (the CUDA context exists by now)."""
     import multiprocessing as mp
     import queue
 
-    n = len(w.candidates)
-    k = max(1, min(len(os.sched_getaffinity(0)), n))
+    n_all = len(w.candidates)
+    k = max(1, min(len(os.sched_getaffinity(0)), n_all))
+    s_fit = int(seconds_target / max(seconds_per_scenario * w.O, 1e-9))
+    if s_fit < w.S:  # one candidate per process, a prefix of its samples
+        s_pref, n = max(1, s_fit), k
+        reps = 1
+    else:
+        s_pref, n = w.S, n_all
+        per = (n + k - 1) // k
+        reps = max(1, int(round(seconds_target / max(seconds_per_scenario * per * w.O * w.S, 1e-9))))
     bounds = [(i * n // k, (i + 1) * n // k) for i in range(k)]
-    per = max(hi - lo for lo, hi in bounds)
-    reps = max(1, int(round(seconds_target / max(seconds_per_candidate * per, 1e-6))))
     ctx = mp.get_context("spawn")
     barrier, out = ctx.Barrier(k), ctx.Queue()
-    procs = [ctx.Process(target=_oracle_worker, args=(widx, lo, hi, reps, barrier, out), daemon=True)
+    procs = [ctx.Process(target=_oracle_worker, args=(widx, lo, hi, s_pref, reps, barrier, out), daemon=True)
              for lo, hi in bounds]
     for p in procs:
         p.start()
@@ -343,11 +383,59 @@ def cpu_baseline_all_cores(widx: int, w, seconds_per_candidate: float, seconds_t
         for p in procs:
             p.join(timeout=60)
     wall = max(e for _, e in spans) - min(b for b, _ in spans)
-    scen = n * w.O * w.S * reps
+    scen = n * w.O * s_pref * reps
     return {"value": 2 * scen / wall, "unit": UNIT, "cores": k, "kind": "oracle",
-            "sample": f"all {n} candidates x {reps} passes, {k} processes over contiguous candidate "
-                      f"ranges ({wall:.3f} s)",
-            "candidate_scores_per_s": n * reps / wall}
+            "sample": f"{_sample_text(w, n, s_pref)}, x {reps} passes, {k} processes over contiguous "
+                      f"candidate ranges ({wall:.3f} s)",
+            "candidate_scores_per_s": scen / wall / (w.O * w.S)}
+
+
+def replay_entry(stream, alu_peak):
+    """The replay workload: Algorithm 1 on 200 independent reveal orders of the
+    paper-scale grid, each round scoring every unrevealed candidate with 8 x
+    4096 samples, until the certificate fires: fs_replay batches all streams'
+    rounds into one launch sequence per round. Wall-clock per whole replay (a
+    synchronous call, timed on the host after a synchronize), and the oracle
+    on the first rounds of stream 0."""
+    import torch
+
+    import oracle
+    from paper_2608_19659_gb300 import fleetsieve as fsb
+
+    rp = workloads.make_replay()
+    w = rp.base
+    seed = 2026
+    m = fsb.fs_load_model(w.cap_lo, w.cap_hi, w.tail_lo, w.tail_hi, w.slo, w.demand, w.G, w.K, w.B,
+                          stream=stream)
+    res = fsb.fs_replay(m, rp.truth_cap, rp.truth_tail, rp.perm, rp.r0, rp.eps, w.O, w.S, seed, rp.max_rounds)
+    walls = []
+    for _ in range(3):
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        res = fsb.fs_replay(m, rp.truth_cap, rp.truth_tail, rp.perm, rp.r0, rp.eps, w.O, w.S, seed,
+                            rp.max_rounds)
+        walls.append(time.perf_counter() - t0)
+    fsb.fs_free_model(m)
+    wall = statistics.median(walls)
+    cells = w.cells
+    # scenarios scored: stream k's round r scores its cells - r0 - r unrevealed candidates
+    cand_rounds = sum(sum(cells - rp.r0 - r for r in range(int(res.rounds[k]))) for k in range(len(res.rounds)))
+    scen = cand_rounds * w.O * w.S
+    # the oracle: the first two rounds of stream 0 (same seed, same samples)
+    qn = oracle.triangular_table(4096)
+    t0 = time.perf_counter()
+    oracle.replay_stream(rp, 0, qn, seed=seed, S=w.S, max_rounds=2)
+    odt = time.perf_counter() - t0
+    o_scen = sum(cells - rp.r0 - r for r in range(2)) * w.O * w.S
+    return {"workload": f"replay: 200 reveal orders of the paper-scale grid, unrevealed candidates x "
+                        f"{w.O} x {w.S} per round, eps {rp.eps}, seeds 100-299",
+            "wall_s_per_replay": wall, "wall_s_runs": walls,
+            "streams_per_s": len(res.rounds) / wall, "rounds_total": int(res.rounds.sum()),
+            "certified": int((res.state == 1).sum()), "candidate_scores": int(cand_rounds),
+            "scenarios": int(scen), "allocation_solves_per_s": 2.0 * scen / wall,
+            "candidate_scores_per_s": cand_rounds / wall,
+            "cpu_baseline": {"value": 2.0 * o_scen / odt, "unit": UNIT, "cores": 1, "kind": "oracle",
+                             "sample": f"stream 0, rounds 0-1 ({o_scen} scenarios, {odt:.1f} s)"}}
 
 
 def run_reference(args, w, rank):
@@ -356,31 +444,32 @@ def run_reference(args, w, rank):
     import oracle
 
     qn = oracle.triangular_table(4096)
-    # a bounded sample per step: enough candidates for about 1 s of CPU work
-    t0 = time.perf_counter()
-    oracle.score(w, qn, candidates=w.candidates[:1])
-    one = time.perf_counter() - t0
-    n = int(max(1, min(len(w.candidates), 1.0 / max(one, 1e-6))))
+    # a bounded sample per step: a prefix of the workload's scenarios for about 0.5 s of CPU work
+    n, s_pref = oracle_prefix(w, 0.5)
     for _ in range(args.warmup):
-        oracle.score(w, qn, candidates=w.candidates[:n])
+        oracle.score(w, qn, candidates=w.candidates[:n], S=s_pref)
     times = []
     for _ in range(args.steps):
         t0 = time.perf_counter()
-        oracle.score(w, qn, candidates=w.candidates[:n])
+        oracle.score(w, qn, candidates=w.candidates[:n], S=s_pref)
         times.append(time.perf_counter() - t0)
     total = sum(times)
-    scen = n * w.O * w.S
+    scen = n * w.O * s_pref
     value = 2 * scen * args.steps / total
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * total / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
-            "data": "synthetic", "config": config_of(w, {"reference_sample_candidates": n}),
-            "candidate_scores_per_s": n * args.steps / total,
+            "data": "synthetic", "config": config_of(w, {"reference_sample": [n, s_pref]}),
+            "candidate_scores_per_s": scen * args.steps / total / (w.O * w.S),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
-                             "sample": f"first {n} of {len(w.candidates)} candidates per step"},
+                             "sample": f"{_sample_text(w, n, s_pref)}, per step"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
     return 0
+
+
+def step_ms_of(starts, ends):
+    return [a.elapsed_time(b) for a, b in zip(starts, ends)]
 
 
 def main(argv=None):
@@ -388,11 +477,12 @@ def main(argv=None):
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=3)
-    ap.add_argument("--workload", type=int, default=1)
+    ap.add_argument("--workload", type=int, default=3)
     ap.add_argument("--impl", default="native", choices=["native", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-all-cores", action="store_true", help="skip the all-cores oracle run")
     ap.add_argument("--no-other-workloads", action="store_true")
+    ap.add_argument("--no-replay", action="store_true", help="skip the replay workload")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         args.warmup = 3
@@ -454,15 +544,20 @@ def main(argv=None):
         fsb.fs_check(model, stream)
         # pass 2, the same steps with events around the Monte-Carlo kernel on its
         # stream, for the kernel's own duration (the roofline)
+        # (at least about a second of them, so that the clock samples taken
+        # every 200 ms see the GPU under this load)
         fsb.fs_timing_read(model)
         fsb.fs_timing_enable(model, 1)
-        for k in range(args.steps):
+        n2 = max(args.steps, min(4000, int(1.0 / max(sum(step_ms_of(starts, ends)) / 1000.0 / args.steps, 1e-6))))
+        for k in range(n2):
             flush.zero_()
             step()
+            if (k + 1) % 1000 == 0:  # the library keeps up to 4096 timed calls
+                torch.cuda.synchronize()
         torch.cuda.synchronize()
         kernel_ms, kernel_n, _ = fsb.fs_timing_read(model)
         fsb.fs_timing_enable(model, 0)
-    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    step_ms = step_ms_of(starts, ends)
     total_ms = max_over_ranks(dist, sum(step_ms), dev)
     scen_all = sum_over_ranks(dist, float(w.scenarios) * args.steps, dev)
     value = 2.0 * scen_all / (total_ms / 1000.0)
@@ -516,11 +611,16 @@ def main(argv=None):
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(w)
         if not args.no_all_cores:
-            cpu["all_cores"] = cpu_baseline_all_cores(args.workload, w, 1.0 / cpu["candidate_scores_per_s"])
-    # the mid and large workloads, for the kernel's efficiency at scale (not the headline)
+            per_scen = 1.0 / (cpu["value"] / 2.0)
+            cpu["all_cores"] = cpu_baseline_all_cores(args.workload, w, per_scen)
+    # the other scoring workloads beside the headline (not the headline), and the replay
     others = []
-    if world == 1 and args.workload == 1 and not args.no_other_workloads:
-        others = [other_workload(i, max(3, min(args.steps, 10)), args.warmup, alu_peak) for i in (2, 3)]
+    if world == 1 and not args.no_other_workloads:
+        others = [other_workload(i, max(3, min(args.steps, 10)), args.warmup, alu_peak)
+                  for i in (1, 2, 3) if i != args.workload]
+    replay = None
+    if world == 1 and not args.no_replay:
+        replay = replay_entry(stream, alu_peak)
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
@@ -531,7 +631,7 @@ def main(argv=None):
                     "api": "fs_update_bounds + fs_score_candidates (pinned host buffers; inputs and results cross through mapped page-locked memory the kernels read and write)",
                     "best": int(res.best)},
             "gpu_launches": int(launches), "roofline": roofline, "clocks": clk,
-            "cpu_baseline": cpu, "other_workloads": others}
+            "cpu_baseline": cpu, "other_workloads": others, "replay": replay}
     if rank == 0:
         print(json.dumps(line))
     fsb.fs_free_model(model)

@@ -63,10 +63,13 @@ typedef struct fs_model fs_model;
  * Per-cell uncertainty state after round t (Section 4.1): capacity interval
  * [cap_lo, cap_hi] (req/s per replica) and tail interval [tail_lo, tail_hi]
  * (s). All four arrays are host pointers to [K][4][B] floats, finite, >= 0,
- * lo <= hi. quantile: optional host table Qn[Q] in [0, 1], nondecreasing,
- * of the posterior inside an interval (value v = lo + (hi - lo) * Qn[k]);
- * NULL selects the built-in symmetric triangular table with Q = 4096.
- * Q must be a power of two >= 4.
+ * lo <= hi. revealed: optional host [K][4][B] flags (nonzero = the cell was
+ * measured, Algorithm 1's "reveal"; its bounds must then be collapsed,
+ * lo == hi, else FS_EINVAL); NULL = no cell measured yet. The certificate
+ * (Section 4.2) reads these flags. quantile: optional host table Qn[Q] in
+ * [0, 1], nondecreasing, of the posterior inside an interval (value
+ * v = lo + (hi - lo) * Qn[k]); NULL selects the built-in symmetric
+ * triangular table with Q = 4096. Q must be a power of two >= 4.
  */
 typedef struct {
     int32_t K;
@@ -75,6 +78,7 @@ typedef struct {
     const float *cap_hi;
     const float *tail_lo;
     const float *tail_hi;
+    const uint8_t *revealed;
     const float *quantile;
     int32_t Q;
     int32_t reserved;
@@ -86,7 +90,10 @@ typedef struct {
  * cuda_stream: stream used by the synchronous calls of this model (NULL =
  * default stream). Limits: 1 <= K <= 64, 1 <= B <= 4096, 1 <= G <= 32767,
  * K * (floor(G/1) + floor(G/2) + floor(G/4) + floor(G/8)) <= 16384.
- * All cells start unrevealed. *out is set only on success.
+ * Cells start revealed as bounds->revealed says (none when it is NULL), so a
+ * model saved with fs_get_state resumes where it stopped (the counter-based
+ * draws depend only on seed, stream, round and cell). *out is set only on
+ * success.
  */
 int fs_load_model(const fs_bounds *bounds, const float *slo, const float *demand, int32_t G,
                   void *cuda_stream, fs_model **out);
@@ -202,17 +209,33 @@ int fs_score_candidates_async(fs_model *m, const fs_samples *samples, double *ga
  *   gap_dev, score_dev [n_cand] doubles, gamma_t_dev [1], best_dev [1]: DEVICE
  *                outputs (each nullable)
  * The same limits as fs_load_model apply, and the values must satisfy its
- * rules (finite, >= 0, lo <= hi, SLOs and demands > 0): they are on the device
- * and are not checked here; candidate ids are range-checked by the kernels
- * (FS_EDEVICE). All intermediates live in one fixed device array of 16 MiB
- * that every GPU loading this library holds until the process exits; a call
- * needing more (roughly n_cand * (2 * (16 + 3 * p) * 4 + 8 * O) bytes, p the
- * power of two above K * sum floor(G/tau)) returns FS_EINVAL without running.
- * The first call on a device looks up the array's address for that device, so
- * make it before any stream capture. Every call shares the array: calls whose
- * GPU work overlaps (other streams or host threads) race. The call enqueues its
- * kernels on cuda_stream, waits for that stream and reports device-side errors
- * (FS_ETIMEOUT, FS_EDEVICE).
+ * rules (finite, >= 0 (-0.0 counts as 0), lo <= hi, SLOs and demands > 0):
+ * they are on the device and are not checked here; candidate ids are
+ * range-checked by the kernels (FS_EDEVICE). The kernels are the ones
+ * fs_score_candidates runs, row tables included.
+ * Scratch: all intermediates live in one fixed device array of 16 MiB
+ * (16,777,216 bytes) that every GPU loading this library holds until the
+ * process exits. A call takes the following pieces of it, each rounded up to
+ * a multiple of 256 bytes, and returns FS_EINVAL without running when their
+ * sum exceeds 16 MiB:
+ *   4, 16 and 1024 bytes (status word, counters, reduction scratch);
+ *   4 Q (only with quantile_dev NULL: the built-in table);
+ *   8 T and 8, with T = K (floor(G/1) + floor(G/2) + floor(G/4) + floor(G/8))
+ *     (thresholds and their counts);
+ *   32 K twice (best capacity and bin per (class, TP) row), 1200 (the two
+ *     base allocations), 65536 (their row tables);
+ *   4 n I with n = max(n_cand, 1), I = 2 (20 + 3 P) + O (4 + 4 ceil(W / 4)),
+ *     P the smallest power of two >= max(T + 1, 4), W = Q / O (the
+ *     candidates' threshold tables and mapped quantile windows);
+ *   8 n O (the fixed-point sums).
+ * On the paper-scale grid (K = 2, G = 16, O = 8, Q = 4096) that allows 913
+ * candidates per call.
+ * The first call on a device looks up the array's address for that device,
+ * so make it before any stream capture. Every call shares the array, which
+ * keeps the last call's contents (the kernels clear what must start at zero):
+ * calls whose GPU work overlaps (other streams or host threads) race. The
+ * call enqueues its kernels on cuda_stream, waits for that stream before it
+ * returns and reports device-side errors (FS_ETIMEOUT, FS_EDEVICE).
  */
 int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, const float *bounds_dev,
                                 const float *slo_dev, const float *demand_dev,
@@ -252,16 +275,39 @@ typedef struct {
  */
 int fs_solve(fs_model *m, const float *cap, const float *tail, fs_allocation *out);
 
-/* n realisations, device arrays cap_dev/tail_dev [n][K][4][B], out_dev [n]. */
+/*
+ * fs_solve_batch -- the allocation of Section 3 (Eqs. 1-5, the same solver
+ * and tie rules as fs_solve) for n realisations at once: device arrays
+ * cap_dev/tail_dev [n][K][4][B] (one realisation after another), out_dev [n]
+ * device allocations. Enqueued on cuda_stream; inputs are read and outputs
+ * written in stream order (the caller keeps them alive until then).
+ */
 int fs_solve_batch(fs_model *m, int32_t n, const float *cap_dev, const float *tail_dev,
                    fs_allocation *out_dev, void *cuda_stream);
 
 /* A- and A+ at the current bounds (Section 4.1) and Gamma_t (host outputs, nullable). */
 int fs_solve_bounds(fs_model *m, fs_allocation *minus, fs_allocation *plus, float *gamma_t);
 
-/* Measurement of one cell: lo = hi = the measured value, marks it revealed
- * (staged for the device like fs_update_bounds). */
+/*
+ * fs_reveal -- Algorithm 1's reveal step: cell has been measured (capacity
+ * cap req/s per replica, binding tail tail s, both finite and >= 0). Its
+ * intervals collapse to the measured values in both realisations
+ * (Section 4.1: lo = hi), and it is marked revealed, which the certificate's
+ * "committed tail upper bounds known" test reads (Section 4.2). Other cells
+ * keep their intervals. Staged for the device like fs_update_bounds.
+ */
 int fs_reveal(fs_model *m, int32_t cell, float cap, float tail);
+
+/*
+ * fs_get_state -- the model's current uncertainty state, for checkpointing
+ * the profiling loop: bounds [K][4][B] (as staged by the last fs_load_model,
+ * fs_update_bounds or fs_reveal) and revealed flags [K][4][B] (0 / 1) into
+ * host arrays (each nullable). Loading them back through fs_bounds, with the
+ * same SLOs, demands, G, quantile table and floors, gives a model whose every
+ * later call returns what this one would.
+ */
+int fs_get_state(const fs_model *m, float *cap_lo, float *cap_hi, float *tail_lo, float *tail_hi,
+                 uint8_t *revealed);
 
 /*
  * Decision certificate (Section 4.2): *state = 2 (certified infeasible) when

@@ -374,6 +374,10 @@ int fs_load_model(const fs_bounds* b, const float* slo, const float* demand, int
     return fail(FS_EINVAL, "K * sum floor(G/tau) = %lld exceeds %d", theta_cap, FS_MAX_THRESHOLDS);
   int rc = check_bounds4(b->cap_lo, b->cap_hi, b->tail_lo, b->tail_hi, cells);
   if (rc) return rc;
+  if (b->revealed)
+    for (int c = 0; c < cells; ++c)
+      if (b->revealed[c] && (b->cap_lo[c] != b->cap_hi[c] || b->tail_lo[c] != b->tail_hi[c]))
+        return fail(FS_EINVAL, "cell %d is revealed but its bounds are not collapsed (lo != hi)", c);
   if (!slo || !demand) return fail(FS_EINVAL, "slo / demand is NULL");
   for (int i = 0; i < K; ++i) {
     if (!std::isfinite(slo[i]) || !(slo[i] > 0.0f)) return fail(FS_EINVAL, "slo[%d] must be finite and > 0", i);
@@ -456,6 +460,8 @@ int fs_load_model(const fs_bounds* b, const float* slo, const float* demand, int
   for (int r = 0; r < 4; ++r)
     for (int c = 0; c < cells; ++c) m->h_bounds[(size_t)r * cells + c] = canon(src[r][c]);
   m->h_revealed.assign(cells, 0);
+  if (b->revealed)
+    for (int c = 0; c < cells; ++c) m->h_revealed[c] = b->revealed[c] ? 1 : 0;
 
   auto bail = [&](int code) {
     fs_free_model(m);
@@ -628,6 +634,17 @@ int fs_reveal(fs_model* m, int32_t cell, float cap, float tail) {
   m->h_bounds[(size_t)TAIL_HI * cells + cell] = canon(tail);
   m->h_revealed[cell] = 1;
   return stage_bounds(m);
+}
+
+int fs_get_state(const fs_model* m, float* cap_lo, float* cap_hi, float* tail_lo, float* tail_hi,
+                 uint8_t* revealed) {
+  if (!m) return fail(FS_EINVAL, "model is NULL");
+  const size_t cells = (size_t)m->d.cells;
+  float* dst[4] = {cap_lo, cap_hi, tail_lo, tail_hi};
+  for (int r = 0; r < 4; ++r)
+    if (dst[r]) std::memcpy(dst[r], m->h_bounds.data() + (size_t)r * cells, 4 * cells);
+  if (revealed) std::memcpy(revealed, m->h_revealed.data(), cells);
+  return FS_OK;
 }
 
 int fs_certificate(fs_model* m, float eps, int32_t* state, float* gamma_t) {

@@ -429,7 +429,8 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
         // one per lane; if the answer is not among them, a 32-ary search over the
         // whole interval.
         const float th = sTh[k], t = FL ? fmaxf(th, dle) : th;
-        const uint32_t bx = __float_as_uint(cx), bmax = __float_as_uint(cmax);
+        // Cexcl = -0 as +0 (the same smallest capacity), as in the table branch
+        const uint32_t bx = __float_as_uint(cx) & 0x7fffffffu, bmax = __float_as_uint(cmax) & 0x7fffffffu;
         const float c0 = __fdividef(__fmul_rn(t, lam), (float)m);  // an estimate: the window is checked exactly
         const long long pl_ = (long long)__float_as_uint(c0) - 16 + lane;
         const uint32_t pt0 = pl_ < 0 ? 0u : (uint32_t)pl_;

@@ -116,6 +116,7 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
   const size_t o_theta = take(8 * (size_t)d.theta_cap), o_nth = take(8);
   const size_t o_rowc = take(8 * (size_t)d.K4), o_rowb = take(8 * (size_t)d.K4);
   const size_t o_base = take(2 * sizeof(fs_allocation));
+  const size_t o_rtab = take(8 * (size_t)kRowTabMax);  // row tables of the two base solves
   const int Wq = Q / smp->O, Wp = 4 + ((Wq + 3) & ~3);
   const size_t item_floats = 2 * (size_t)d.slot_floats + (size_t)smp->O * Wp;
   const size_t o_tab = take((size_t)std::max(n, 1) * item_floats * 4);
@@ -132,7 +133,7 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
   if (e != cudaSuccess) return cuda_say(e, "cudaGetDevice");
   if (dev < 0 || dev >= kMaxStaticDevices) return say(FS_EINVAL, "device %d beyond %d", dev, kMaxStaticDevices);
   char* base = nullptr;
-  LaunchCache* lc = nullptr;
+  LaunchCache lc;  // this call's copy of the device's launch shapes, written back under the lock
   {
     std::lock_guard<std::mutex> lock(g_static_mu);
     if (!g_static_ptr[dev]) {
@@ -142,7 +143,7 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
       g_static_ptr[dev] = p;
     }
     base = static_cast<char*>(g_static_ptr[dev]);
-    lc = &g_static_lc[dev];
+    lc = g_static_lc[dev];
   }
   int sm_count = 0;
   e = cudaDeviceGetAttribute(&sm_count, cudaDevAttrMultiProcessorCount, dev);
@@ -164,6 +165,7 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
   set.status = reinterpret_cast<uint32_t*>(base + o_status);
   set.work = reinterpret_cast<unsigned long long*>(base + o_work);
   set.skip = nullptr;
+  set.rtab = reinterpret_cast<int*>(base + o_rtab);
 
   Items it{};
   it.n = n;
@@ -191,15 +193,30 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
   e = cudaMemsetAsync(set.status, 0, 4, s);  // the array keeps the last call's status word
   if (e == cudaSuccess && !quantile_dev) e = launch_qtable(const_cast<float*>(set.qn), Q, s);
-  if (e == cudaSuccess) e = launch_solve(set, 2, nullptr, nullptr, nullptr, true, *lc, s, true);
+  if (e == cudaSuccess) e = launch_solve(set, 2, nullptr, nullptr, nullptr, true, lc, s, true);
   if (e == cudaSuccess) e = launch_prep(set, it, pl, reinterpret_cast<float*>(base + o_tab),
-                                        reinterpret_cast<uint64_t*>(base + o_sums), true, *lc, s);
+                                        reinterpret_cast<uint64_t*>(base + o_sums), true, lc, s);
   if (e == cudaSuccess)
     e = launch_score(set, it, pl, reinterpret_cast<const float*>(base + o_tab),
-                     reinterpret_cast<uint64_t*>(base + o_sums), nullptr, 0, sm_count, *lc, s);
+                     reinterpret_cast<uint64_t*>(base + o_sums), nullptr, 0, sm_count, lc, s);
   if (e == cudaSuccess)
     e = launch_finalize(set, it, pl, reinterpret_cast<const uint64_t*>(base + o_sums), gap_dev, score_dev,
                         gamma_t_dev, best_dev, nullptr, reinterpret_cast<uint64_t*>(base + o_part), s);
+  {
+    // launch shapes only grow (a kernel's shared-memory limit is only raised):
+    // keep the larger of what this call and any concurrent one found
+    std::lock_guard<std::mutex> lock(g_static_mu);
+    LaunchCache& g = g_static_lc[dev];
+    for (int f = 0; f < 2; ++f) {
+      g.solve_smem[f] = std::max(g.solve_smem[f], lc.solve_smem[f]);
+      g.prep_smem[f] = std::max(g.prep_smem[f], lc.prep_smem[f]);
+      for (int v = 0; v < 3; ++v)
+        if (lc.score_smem[v][f] && lc.score_smem[v][f] != g.score_smem[v][f]) {
+          g.score_smem[v][f] = lc.score_smem[v][f];
+          g.score_blocks_per_sm[v][f] = lc.score_blocks_per_sm[v][f];
+        }
+    }
+  }
   if (e != cudaSuccess) return cuda_say(e, "launch (allocation-free scoring)");
   uint32_t st = 0;
   e = cudaMemcpyAsync(&st, set.status, 4, cudaMemcpyDeviceToHost, s);

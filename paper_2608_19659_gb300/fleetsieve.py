@@ -23,7 +23,7 @@ FS_OK, FS_EINVAL, FS_ENOMEM, FS_ECUDA, FS_ETIMEOUT, FS_EDEVICE = 0, -1, -2, -3, 
 FS_MAX_CLASSES = 64
 EXPORTS = ("fs_load_model", "fs_update_bounds", "fs_set_floors", "fs_dump_stride", "fs_score_candidates",
            "fs_score_candidates_async", "fs_solve", "fs_solve_batch", "fs_solve_bounds",
-           "fs_reveal", "fs_certificate", "fs_replay", "fs_check", "fs_launch_count",
+           "fs_reveal", "fs_get_state", "fs_certificate", "fs_replay", "fs_check", "fs_launch_count",
            "fs_watchdog_selftest", "fs_free_model", "fs_last_error", "fs_score_candidates_noalloc",
            "fs_timing_enable",
            "fs_timing_read")
@@ -38,8 +38,8 @@ class FleetSieveError(RuntimeError):
 class fs_bounds(C.Structure):
     _fields_ = [("K", C.c_int32), ("B", C.c_int32), ("cap_lo", C.POINTER(C.c_float)),
                 ("cap_hi", C.POINTER(C.c_float)), ("tail_lo", C.POINTER(C.c_float)),
-                ("tail_hi", C.POINTER(C.c_float)), ("quantile", C.POINTER(C.c_float)),
-                ("Q", C.c_int32), ("reserved", C.c_int32)]
+                ("tail_hi", C.POINTER(C.c_float)), ("revealed", C.c_void_p),
+                ("quantile", C.POINTER(C.c_float)), ("Q", C.c_int32), ("reserved", C.c_int32)]
 
 
 class fs_samples(C.Structure):
@@ -99,6 +99,8 @@ def lib():
         L.fs_solve_bounds.argtypes = [C.c_void_p, C.POINTER(fs_allocation),
                                       C.POINTER(fs_allocation), fp]
         L.fs_reveal.argtypes = [C.c_void_p, C.c_int32, C.c_float, C.c_float]
+        L.fs_get_state.argtypes = [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
+                                   C.c_void_p]
         L.fs_certificate.argtypes = [C.c_void_p, C.c_float, C.POINTER(C.c_int32), fp]
         L.fs_replay.argtypes = [C.c_void_p, C.POINTER(fs_replay_spec), C.c_void_p, C.c_void_p,
                                 C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p]
@@ -176,10 +178,14 @@ class Model:
 
 
 def fs_load_model(cap_lo, cap_hi, tail_lo, tail_hi, slo, demand, G: int, K: int, B: int,
-                  quantile=None, stream=None) -> Model:
+                  quantile=None, stream=None, revealed=None) -> Model:
+    """revealed: optional [K*4*B] flags of cells already measured (bounds collapsed)."""
     arrs = [_f32(x) for x in (cap_lo, cap_hi, tail_lo, tail_hi)]
     q = _f32(quantile) if quantile is not None else None
-    b = fs_bounds(K, B, *[_fp(x) for x in arrs], _fp(q) if q is not None else None,
+    rv = np.ascontiguousarray(np.asarray(revealed).reshape(-1) != 0, np.uint8) if revealed is not None else None
+    if rv is not None and rv.size != K * 4 * B:
+        raise ValueError(f"revealed has {rv.size} flags for {K * 4 * B} cells")
+    b = fs_bounds(K, B, *[_fp(x) for x in arrs], _vp(rv), _fp(q) if q is not None else None,
                   q.size if q is not None else 0, 0)
     s_ = _f32(slo)
     d_ = _f32(demand)
@@ -316,6 +322,31 @@ def fs_solve_bounds(m: Model):
 
 def fs_reveal(m: Model, cell: int, cap: float, tail: float) -> None:
     _check(lib().fs_reveal(m.handle, int(cell), float(cap), float(tail)))
+
+
+def fs_get_state(m: Model):
+    """(cap_lo, cap_hi, tail_lo, tail_hi, revealed) of the model now, each [K*4*B]."""
+    out = [np.zeros(m.cells, np.float32) for _ in range(4)] + [np.zeros(m.cells, np.uint8)]
+    _check(lib().fs_get_state(m.handle, *[_vp(x) for x in out]))
+    return tuple(out)
+
+
+def save_state(m: Model, path: str, round: int = 0, **extra) -> None:
+    """Checkpoint of the profiling loop: the model's bounds and revealed flags,
+    its K, B, G and the next round number (the draws are counter-based, so a
+    resumed loop repeats an uninterrupted one exactly), plus caller arrays."""
+    clo, chi, tlo, thi, rev = fs_get_state(m)
+    np.savez(path, cap_lo=clo, cap_hi=chi, tail_lo=tlo, tail_hi=thi, revealed=rev,
+             dims=np.array([m.K, m.B, m.G, int(round)], np.int64), **extra)
+
+
+def load_state(path: str, slo, demand, quantile=None, stream=None):
+    """A model rebuilt from :func:`save_state`'s file, its next round and the file's arrays."""
+    z = dict(np.load(path))
+    K, B, G, rnd = (int(x) for x in z.pop("dims"))
+    m = fs_load_model(z.pop("cap_lo"), z.pop("cap_hi"), z.pop("tail_lo"), z.pop("tail_hi"), slo, demand,
+                      G, K, B, quantile=quantile, stream=stream, revealed=z.pop("revealed"))
+    return m, rnd, z
 
 
 def fs_certificate(m: Model, eps: float):

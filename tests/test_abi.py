@@ -52,7 +52,7 @@ def _good(K=2, B=3):
 
 
 @pytest.mark.parametrize("case", ["nan", "neg", "lo_gt_hi", "K0", "K65", "B0", "G0", "theta",
-                                  "slo0", "demand0", "qn_bad", "qn_size"])
+                                  "slo0", "demand0", "qn_bad", "qn_size", "revealed_open"])
 def test_load_model_rejects_bad_input(fsb, case):
     K, B, G = 2, 3, 16
     clo, chi, tlo, thi, slo, lam = _good(K, B)
@@ -81,7 +81,11 @@ def test_load_model_rejects_bad_input(fsb, case):
         q = np.linspace(1.0, 0.0, 16, dtype=np.float32)
     elif case == "qn_size":
         q = np.linspace(0.0, 1.0, 12, dtype=np.float32)
+    rev = None
+    if case == "revealed_open":  # a measured cell must have collapsed bounds
+        rev = np.zeros(K * 4 * B, np.uint8)
+        rev[4] = 1
     with pytest.raises(fsb.FleetSieveError) as ei:
-        fsb.fs_load_model(clo, chi, tlo, thi, slo, lam, G, K, B, quantile=q)
+        fsb.fs_load_model(clo, chi, tlo, thi, slo, lam, G, K, B, quantile=q, revealed=rev)
     assert ei.value.code == fsb.FS_EINVAL
     assert fsb.fs_last_error()

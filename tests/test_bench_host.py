@@ -107,23 +107,48 @@ def test_roofline_traffic_only_for_the_profiled_source(tmp_path, monkeypatch):
     assert bench._profiled_traffic(1) is None
 
 
+def _passes_and_wall(r):
+    reps = int(r["sample"].split(", x ")[1].split()[0])
+    wall = float(r["sample"].rsplit("(", 1)[1].split(" s")[0])
+    return reps, wall
+
+
 def test_all_cores_oracle_baseline_counts_every_scenario():
     """The all-cores CPU baseline: one spawned oracle process per usable core
     over contiguous candidate ranges; its rate counts every scenario of every
-    pass once."""
+    pass once. Whole candidates when they fit the time target; else one
+    candidate per process with the same prefix of samples per outcome."""
     sys.path.insert(0, ROOT)
     import bench
     from paper_2608_19659_gb300 import workloads
 
     w = workloads.make_workload(0)
-    r = bench.cpu_baseline_all_cores(0, w, seconds_per_candidate=0.02, seconds_target=0.2)
-    assert "unavailable" not in r, r
     k = min(len(os.sched_getaffinity(0)), len(w.candidates))
+    r = bench.cpu_baseline_all_cores(0, w, seconds_per_scenario=1e-6, seconds_target=0.2)
+    assert "unavailable" not in r, r
     assert r["cores"] == k and r["kind"] == "oracle" and r["value"] > 0
-    reps = int(r["sample"].split(" x ")[1].split()[0])
-    wall = float(r["sample"].rsplit("(", 1)[1].split(" s")[0])
+    reps, wall = _passes_and_wall(r)
     assert reps >= 1 and wall > 0
     assert abs(r["value"] - 2 * len(w.candidates) * w.O * w.S * reps / wall) <= 0.06 * r["value"]
+    # a prefix of 16 samples per outcome: one candidate per process
+    r = bench.cpu_baseline_all_cores(0, w, seconds_per_scenario=0.2 / (w.O * 16), seconds_target=0.2)
+    reps, wall = _passes_and_wall(r)
+    assert "samples 0..15 of 256" in r["sample"] and reps == 1
+    assert abs(r["value"] - 2 * k * w.O * 16 / wall) <= 0.06 * r["value"]
+
+
+def test_oracle_prefix_is_a_prefix_of_the_workload():
+    """The single-core sample: whole candidates when they fit, else the first
+    candidate with samples 0 .. S' - 1 of every outcome."""
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2608_19659_gb300 import workloads
+
+    n, s = bench.oracle_prefix(workloads.make_workload(0), 0.5)
+    assert s == 256 and 1 <= n <= 16
+    w3 = workloads.make_workload(3)
+    n, s = bench.oracle_prefix(w3, 0.2)
+    assert n == 1 and 1 <= s < w3.S
 
 
 def test_algorithmic_counts_of_the_scorer_paths():

@@ -53,6 +53,76 @@ def test_noalloc_matches_allocating_entry_point_on_two_calls(fsb, cuda, idx, fac
         assert ref.score.max() > 0
 
 
+def _scratch_bytes(K, G, O, Q, n, builtin_table=True):
+    """The scratch a call takes, as the header states it: pieces rounded up to 256 bytes."""
+    up = lambda x: (x + 255) // 256 * 256  # noqa: E731
+    T = K * ((G >> 0) + (G >> 1) + (G >> 2) + (G >> 3))
+    P = 4
+    while P < T + 1:
+        P *= 2
+    W = Q // O
+    I = 2 * (20 + 3 * P) + O * (4 + 4 * ((W + 3) // 4))
+    n = max(n, 1)
+    parts = [4, 16, 1024] + ([4 * Q] if builtin_table else []) + [8 * T, 8, 32 * K, 32 * K, 1200, 65536,
+                                                                   4 * n * I, 8 * n * O]
+    return sum(up(p) for p in parts)
+
+
+def test_noalloc_limit_is_the_stated_formula(fsb, cuda):
+    """The largest call the header's formula allows runs (and matches the
+    allocating path); one candidate more is refused without running."""
+    torch = cuda
+    w = workloads.make_workload(1)
+    n = 1
+    while _scratch_bytes(w.K, w.G, w.O, 4096, n + 1) <= 16 << 20:
+        n += 1
+    assert n == 913  # the figure the header quotes for this grid
+    cells = np.resize(w.candidates, n + 1).astype(np.int32)
+    bounds, slo, lam, _ = _device_inputs(torch, w)
+    cand = torch.from_numpy(cells).cuda()
+    gap = torch.zeros(n, dtype=torch.float64, device="cuda")
+    best = torch.zeros(1, dtype=torch.int32, device="cuda")
+    fsb.fs_score_candidates_noalloc(w.K, w.B, w.G, bounds, slo, lam, cand[:n], w.O, 8, w.seed,
+                                    gap_dev=gap, best_dev=best)
+    with load_model(fsb, w) as m:
+        ref = fsb.fs_score_candidates(m, cells[:n], w.O, 8, w.seed)
+    assert np.array_equal(gap.cpu().numpy(), ref.gap) and int(best.item()) == ref.best
+    with pytest.raises(fsb.FleetSieveError) as ei:
+        fsb.fs_score_candidates_noalloc(w.K, w.B, w.G, bounds, slo, lam, cand, w.O, 8, w.seed, gap_dev=gap)
+    assert ei.value.code == fsb.FS_EINVAL and "scratch" in str(ei.value)
+
+
+@pytest.mark.parametrize("idx", [1, 3])
+def test_noalloc_negative_zero_capacities(fsb, cuda, idx):
+    """Device bounds are not canonicalised by this entry point: capacities of
+    -0.0 (which the rules accept as 0) must score exactly as the allocating
+    path, which stores them as +0. The 8-class workload runs the preparation
+    without a row table (too many rows x thresholds), the paper-scale one with."""
+    torch = cuda
+    w = workloads.make_workload(idx)
+    w = dataclasses.replace(w, demand=(w.demand * np.float32(2.0)).astype(np.float32), S=64)
+    clo = w.cap_lo.copy().reshape(w.K, 4, w.B)
+    chi = w.cap_hi.copy().reshape(w.K, 4, w.B)
+    clo[0, 1, :] = np.float32(-0.0)  # class 0, TP 2: lower capacity -0 in every bin
+    chi[0, 1, : w.B // 2] = np.float32(-0.0)  # and a collapsed [-0, -0] interval in half of them
+    w = dataclasses.replace(w, cap_lo=clo.reshape(w.cap_lo.shape), cap_hi=chi.reshape(w.cap_hi.shape))
+    cand_np = np.arange(w.B, 2 * w.B, dtype=np.int32)  # every cell of that row
+    cand_np = np.concatenate([cand_np, w.candidates[:: max(1, len(w.candidates) // 16)]]).astype(np.int32)
+    bounds, slo, lam, _ = _device_inputs(torch, w)
+    assert bool(torch.signbit(bounds[w.B]).item())  # the device holds -0.0
+    n = len(cand_np)
+    gap = torch.zeros(n, dtype=torch.float64, device="cuda")
+    score = torch.zeros(n, dtype=torch.float64, device="cuda")
+    gt = torch.zeros(1, dtype=torch.float32, device="cuda")
+    best = torch.zeros(1, dtype=torch.int32, device="cuda")
+    fsb.fs_score_candidates_noalloc(w.K, w.B, w.G, bounds, slo, lam, torch.from_numpy(cand_np).cuda(), w.O, w.S,
+                                    w.seed, gap_dev=gap, score_dev=score, gamma_t_dev=gt, best_dev=best)
+    with load_model(fsb, w) as m:
+        ref = fsb.fs_score_candidates(m, cand_np, w.O, w.S, w.seed)
+    assert np.array_equal(gap.cpu().numpy(), ref.gap) and np.array_equal(score.cpu().numpy(), ref.score)
+    assert float(gt.item()) == ref.gamma_t and int(best.item()) == ref.best
+
+
 def test_noalloc_refuses_calls_beyond_its_array(fsb, cuda):
     torch = cuda
     w = workloads.make_workload(3)  # 1024 candidates x 2 tables of 16 + 3 * 4096 floats: ~100 MB
