@@ -54,10 +54,13 @@ ISSUE_PER_SM_CLK = 4 * 32  # 4 schedulers x 32 lanes, one warp instruction each 
 # Table path (a segment's W + 1 values of rint(Gamma' 2^40) tabulated once):
 # per scenario the Philox share (10), capacity position (1), gate mask,
 # compare and index select (3), the entry's load (1) and its two field sums
-# (2) = 17; per table entry the two patched capacities (2), two table searches
-# (6), Gamma' (1), the fixed-point conversion (5) and the store (1) = 15.
-# Search probes beyond the first (3 each) and row-term fulfilments are not
-# counted: lower bounds.
+# (2) = 17; per table entry evaluated the two patched capacities (2), two
+# table searches (6), Gamma' (1), the fixed-point conversion (5) and the store
+# (1) = 15. A segment whose tail gate is closed at every position of its
+# stratum evaluates no entry (all equal the closed-gate value, from the
+# preparation); the library counts the entries evaluated. Search probes
+# beyond the first (3 each) and row-term fulfilments are not counted: lower
+# bounds.
 OPS_PER_SCENARIO = 32
 OPS_PER_SCENARIO_TABLE = 17
 OPS_PER_TABLE_ENTRY = 15
@@ -72,11 +75,15 @@ def table_path(O: int, S: int) -> bool:
     return W <= 4096 and 3 * (W + 1) <= 2 * min(S, 2048)
 
 
-def algorithmic_ops(w) -> float:
-    """Algorithmic thread-operations of one Monte-Carlo launch over workload w."""
+def algorithmic_ops(w, entries_per_launch=None) -> float:
+    """Algorithmic thread-operations of one Monte-Carlo launch over workload w:
+    on the table path, with the gap-table entries the launch evaluated (as the
+    library counted them; None: W entries in every segment)."""
     if table_path(w.O, w.S):
         W = Q_TABLE // w.O
-        return float(len(w.candidates)) * w.O * (w.S * OPS_PER_SCENARIO_TABLE + (W + 1) * OPS_PER_TABLE_ENTRY)
+        if entries_per_launch is None:
+            entries_per_launch = float(len(w.candidates)) * w.O * W
+        return float(OPS_PER_SCENARIO_TABLE) * w.scenarios + OPS_PER_TABLE_ENTRY * float(entries_per_launch)
     return float(OPS_PER_SCENARIO) * w.scenarios
 
 # ncu summaries with the DRAM bytes of one k_score launch, per workload; used
@@ -271,12 +278,12 @@ def other_workload(idx: int, steps: int, warmup: int, alu_peak: float, stream_id
         flush.zero_()
         step()
     torch.cuda.synchronize()
-    kernel_ms, kernel_n, _ = fsb.fs_timing_read(m)
+    kernel_ms, kernel_n, _, entries = fsb.fs_timing_read(m, with_entries=True)
     fsb.fs_timing_enable(m, 0)
     fsb.fs_check(m, stream)
     fsb.fs_free_model(m)
     kern_s = kernel_ms / 1000.0 / max(kernel_n, 1)
-    achieved = algorithmic_ops(w) / kern_s
+    achieved = algorithmic_ops(w, entries / max(kernel_n, 1)) / kern_s
     gamma_t = float(gt.item())
     return {"workload": w.name, "ms_per_step": step_ms, "scenarios_per_s": w.scenarios / (step_ms / 1000.0),
             "gamma_t": gamma_t,
@@ -386,7 +393,7 @@ def cpu_baseline_all_cores(widx: int, w, seconds_per_scenario: float, seconds_ta
     scen = n * w.O * s_pref * reps
     return {"value": 2 * scen / wall, "unit": UNIT, "cores": k, "kind": "oracle",
             "sample": f"{_sample_text(w, n, s_pref)}, x {reps} passes, {k} processes over contiguous "
-                      f"candidate ranges ({wall:.3f} s)",
+                      f"candidate ranges ({wall:.4g} s)",
             "candidate_scores_per_s": scen / wall / (w.O * w.S)}
 
 
@@ -483,6 +490,9 @@ def main(argv=None):
     ap.add_argument("--no-all-cores", action="store_true", help="skip the all-cores oracle run")
     ap.add_argument("--no-other-workloads", action="store_true")
     ap.add_argument("--no-replay", action="store_true", help="skip the replay workload")
+    ap.add_argument("--kernel-pass-s", type=float, default=1.0,
+                    help="least duration of the kernel-timing pass (0: --steps steps)")
+    ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end pass (profiling runs)")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         args.warmup = 3
@@ -547,15 +557,16 @@ def main(argv=None):
         # (at least about a second of them, so that the clock samples taken
         # every 200 ms see the GPU under this load)
         fsb.fs_timing_read(model)
-        fsb.fs_timing_enable(model, 1)
-        n2 = max(args.steps, min(4000, int(1.0 / max(sum(step_ms_of(starts, ends)) / 1000.0 / args.steps, 1e-6))))
+        fsb.fs_timing_enable(model, 1)  # (also zeroes the library's count of table entries)
+        per_step_s = max(sum(step_ms_of(starts, ends)) / 1000.0 / args.steps, 1e-6)
+        n2 = max(args.steps, min(4000, int(args.kernel_pass_s / per_step_s)))
         for k in range(n2):
             flush.zero_()
             step()
             if (k + 1) % 1000 == 0:  # the library keeps up to 4096 timed calls
                 torch.cuda.synchronize()
         torch.cuda.synchronize()
-        kernel_ms, kernel_n, _ = fsb.fs_timing_read(model)
+        kernel_ms, kernel_n, _, entries = fsb.fs_timing_read(model, with_entries=True)
         fsb.fs_timing_enable(model, 0)
     step_ms = step_ms_of(starts, ends)
     total_ms = max_over_ranks(dist, sum(step_ms), dev)
@@ -576,17 +587,20 @@ def main(argv=None):
         fsb.fs_update_bounds(model, pinned["cap_lo"], pinned["cap_hi"], pinned["tail_lo"], pinned["tail_hi"])
         return fsb.fs_score_candidates(model, cand_h, w.O, w.S, w.seed, stream_id, 0, outputs=outs)
 
-    for _ in range(args.warmup):
-        e2e_step()
-    if dist is not None:
-        dist.barrier()
-    torch.cuda.synchronize()
-    t0 = time.perf_counter()
-    for _ in range(args.steps):
-        res = e2e_step()
-    torch.cuda.synchronize()
-    e2e_s = max_over_ranks(dist, time.perf_counter() - t0, dev)
-    e2e_value = 2.0 * scen_all / e2e_s
+    e2e_value, e2e_best = None, None
+    if not args.no_e2e:
+        for _ in range(args.warmup):
+            e2e_step()
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(args.steps):
+            res = e2e_step()
+        torch.cuda.synchronize()
+        e2e_s = max_over_ranks(dist, time.perf_counter() - t0, dev)
+        e2e_value = 2.0 * scen_all / e2e_s
+        e2e_best = int(res.best)
     h2d = 16 * w.cells + w.cells + 4 * n
     d2h = 8 * n + 8 * n + 4 + 4
 
@@ -596,17 +610,20 @@ def main(argv=None):
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     alu_peak = sms * ISSUE_PER_SM_CLK * sm_max * 1e6  # thread-ops/s at the maximum SM clock
     kern_s = kernel_ms / 1000.0 / max(kernel_n, 1)
-    achieved = algorithmic_ops(w) / kern_s if kernel_n else None
+    entries_per_launch = entries / max(kernel_n, 1)
+    ops = algorithmic_ops(w, entries_per_launch)
+    achieved = ops / kern_s if kernel_n else None
     roofline = {"bound": "alu", "kernel": "k_score (Monte-Carlo sampler + parametric re-solve)",
                 "achieved": achieved / 1e12 if achieved else None,
                 "peak": alu_peak / 1e12, "unit": "Tops/s (32-bit thread operations)",
                 "frac": (achieved / alu_peak) if achieved else None,
                 "traffic": _profiled_traffic(args.workload), "traffic_unit": "DRAM bytes per launch (ncu)",
                 "algorithmic_bytes": 0, "kernel_ms_per_launch": kern_s * 1000.0,
-                "ops_per_scenario": algorithmic_ops(w) / w.scenarios,
+                "ops_per_scenario": ops / w.scenarios,
+                "table_entries_per_launch": entries_per_launch,
                 "path": "table" if table_path(w.O, w.S) else "plain",
                 "peak_basis": f"{sms} SMs x 4 issue slots x 32 lanes x {sm_max:.0f} MHz (max SM clock)",
-                "kernel_share_of_step": (kernel_ms / max(sum(step_ms), 1e-9)) if kernel_n else None}
+                "kernel_share_of_step": (kern_s * 1000.0 / (sum(step_ms) / len(step_ms))) if kernel_n else None}
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(w)
@@ -629,7 +646,7 @@ def main(argv=None):
             "scenarios_per_s": scen_all / (total_ms / 1000.0),
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                     "api": "fs_update_bounds + fs_score_candidates (pinned host buffers; inputs and results cross through mapped page-locked memory the kernels read and write)",
-                    "best": int(res.best)},
+                    "best": e2e_best},
             "gpu_launches": int(launches), "roofline": roofline, "clocks": clk,
             "cpu_baseline": cpu, "other_workloads": others, "replay": replay}
     if rank == 0:

@@ -361,14 +361,19 @@ int fs_check(fs_model *m, void *cuda_stream);
  * later scoring call of this model records CUDA events around its
  * Monte-Carlo kernel on the stream it launches on; mode 2: also around the
  * base solves, the table preparation and the reduction; 0: off (up to 4096
- * calls are kept). fs_timing_read waits for the recorded events and returns
- * the summed Monte-Carlo kernel time (ms), the number of timed calls and,
- * in mode 2, phase_ms[4] = summed (solve, prep, Monte-Carlo, reduction) time
- * (nullable); it clears the record. Events between kernels also stop the
- * next kernel from starting early, so timed calls can take a little longer.
+ * calls are kept). fs_timing_enable also zeroes the model's count of table
+ * entries evaluated. fs_timing_read waits for the recorded events and returns
+ * the summed Monte-Carlo kernel time (ms), the number of timed calls, in mode
+ * 2 phase_ms[4] = summed (solve, prep, Monte-Carlo, reduction) time, and
+ * table_entries = the gap-table entries the Monte-Carlo kernel evaluated
+ * (two t* each) on its table path since the count was last zeroed (each
+ * outputs nullable); it clears the record and the count. Events between
+ * kernels also stop the next kernel from starting early, so timed calls can
+ * take a little longer.
  */
 int fs_timing_enable(fs_model *m, int32_t mode);
-int fs_timing_read(fs_model *m, double *kernel_ms, int32_t *launches, double *phase_ms);
+int fs_timing_read(fs_model *m, double *kernel_ms, int32_t *launches, double *phase_ms,
+                   uint64_t *table_entries);
 
 /* Kernels this library has launched since it was loaded (all models). */
 uint64_t fs_launch_count(void);

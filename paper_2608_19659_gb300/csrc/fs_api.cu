@@ -293,6 +293,7 @@ Plan make_plan(const fs_model* m, const fs_samples* s, int n_items) {
   pl.calls = (s->S + 3) / 4;
   pl.Wp = 4 + ((pl.W + 3) & ~3);
   pl.item_floats = 2LL * m->d.slot_floats + (long long)s->O * pl.Wp;
+  plan_round_keys(pl);
   (void)n_items;
   return pl;
 }
@@ -426,7 +427,7 @@ int fs_load_model(const fs_bounds* b, const float* slo, const float* demand, int
   const size_t o_bounds = take(16 * (size_t)cells), o_rev = take(cells);
   const size_t o_theta = take(8 * (size_t)d.theta_cap), o_nth = take(8);
   const size_t o_rowc = take(8 * (size_t)d.K4), o_rowb = take(8 * (size_t)d.K4);
-  const size_t o_base = take(2 * sizeof(fs_allocation)), o_status = take(4), o_work = take(16);
+  const size_t o_base = take(2 * sizeof(fs_allocation)), o_status = take(4), o_work = take(24);
   const size_t o_rtab = take(8 * (size_t)kRowTabMax);
   rc = m->fixed.ensure(off, "model state");
   if (rc) {
@@ -822,16 +823,29 @@ int fs_check(fs_model* m, void* cuda_stream) {
   return read_status(m, cuda_stream ? (cudaStream_t)cuda_stream : m->stream);
 }
 
+// The table-entry count (work[2]) of the model, zeroed in stream order.
+static int zero_entry_count(fs_model* m) {
+  FS_CUDA(cudaMemsetAsync(m->set.work + 2, 0, 8, m->stream), "zero the entry count");
+  FS_CUDA(cudaStreamSynchronize(m->stream), "zero the entry count");
+  return FS_OK;
+}
+
 int fs_timing_enable(fs_model* m, int32_t on) {
   if (!m) return fail(FS_EINVAL, "model is NULL");
   if (on < 0 || on > 2) return fail(FS_EINVAL, "timing mode %d not in {0, 1, 2}", on);
   m->timing = on;
   m->ev_used = 0;
-  return FS_OK;
+  return zero_entry_count(m);
 }
 
-int fs_timing_read(fs_model* m, double* kernel_ms, int32_t* launches, double* phase_ms) {
+int fs_timing_read(fs_model* m, double* kernel_ms, int32_t* launches, double* phase_ms, uint64_t* table_entries) {
   if (!m) return fail(FS_EINVAL, "model is NULL");
+  if (table_entries) {
+    FS_CUDA(cudaDeviceSynchronize(), "wait for the scoring calls");
+    FS_CUDA(cudaMemcpy(table_entries, m->set.work + 2, 8, cudaMemcpyDeviceToHost), "read the entry count");
+    int rc = zero_entry_count(m);
+    if (rc) return rc;
+  }
   double total = 0.0, ph[4] = {0.0, 0.0, 0.0, 0.0};
   const size_t n = m->ev_used / 5;
   for (size_t k = 0; k < n; ++k) {

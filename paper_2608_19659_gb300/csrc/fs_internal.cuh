@@ -10,7 +10,8 @@
 //   rowC     [P][2][K*4]   f32   best SLO-feasible capacity per (class, TP)
 //   rowB     [P][2][K*4]   i32   its bin (-1: none)
 //   base     [P][2]        fs_allocation
-//   work     [2]           u64   chunk counter of the Monte-Carlo kernel, the reduction's ticket
+//   work     [3]           u64   chunk counter of the Monte-Carlo kernel, the reduction's ticket,
+//                                 table entries evaluated (accumulates across calls; the host zeroes it)
 // Per scoring call (items = (problem, candidate cell) pairs), one record of
 // item_floats = 2 slot_floats + O Wp floats per item:
 //   [2][slot_floats] f32   threshold tables of the two realisations
@@ -41,7 +42,7 @@ constexpr int kRowTabMax = 8192;
 // Table header words (floats unless noted).
 enum : int {
   H_TH_BASE = 0,  // threshold below the first table entry (0 if none)
-  H_M_FIRST = 1,  // replicas row r may use just above it
+  H_TCL = 1,      // t* of this realisation at row capacity Cexcl: every scenario whose tail gate is closed
   H_L = 2,        // entries (int)
   H_LPAD = 3,     // entries padded to 4 (int)
   H_CX = 4,       // best capacity of row r without the candidate's bin
@@ -91,7 +92,8 @@ struct Set {
   int* rowB;            // [P][2][K4] bin of rowC, -1 = no SLO-feasible bin
   fs_allocation* base;  // [P][2]
   uint32_t* status;
-  unsigned long long* work;  // [2] chunk counter, reduction ticket; zeroed by k_prep
+  unsigned long long* work;  // [3] chunk counter, reduction ticket (zeroed by k_prep); table entries
+                             // evaluated by the Monte-Carlo kernel (summed over calls, zeroed by the host)
   const int* skip;      // [P] or nullptr: base solves skip problems with skip[p] >= 0
   int* rtab;            // [P][2][kRowTabMax] or nullptr: row tables of the scoring solves,
                         // word (row rho, threshold k) at k K4 + rho
@@ -109,7 +111,28 @@ struct Plan {
   int calls;            // ceil(S / 4) Philox calls per (candidate, outcome)
   int Wp;               // floats per mapped outcome window: 4 + W rounded up to 4
   long long item_floats;  // floats per item record: 2 slot_floats + O Wp
+  // Philox round keys of problem 0 (key1 XOR stream_base): as kernel
+  // parameters at fixed offsets they are constant operands of the rounds'
+  // XORs and take no registers (launches over one problem use them)
+  uint32_t rk0[10], rk1[10];
+  // 65536 and 8, read from the parameters rather than known to the compiler,
+  // so that a word's low half moved to the top and an entry's byte offset are
+  // integer multiply-adds (FMA pipe) rather than shifts and masks (ALU pipe)
+  uint32_t lo16_mul, entry_bytes;
 };
+
+// Round keys of problem 0 for the plan (host).
+inline void plan_round_keys(Plan& pl) {
+  uint32_t k0 = pl.key0, k1 = pl.key1 ^ pl.stream_base;
+  for (int r = 0; r < 10; ++r) {
+    pl.rk0[r] = k0;
+    pl.rk1[r] = k1;
+    k0 += 0x9E3779B9u;
+    k1 += 0xBB67AE85u;
+  }
+  pl.lo16_mul = 65536u;
+  pl.entry_bytes = 8u;
+}
 
 struct Items {
   int n;
@@ -244,6 +267,18 @@ __device__ __forceinline__ PhiloxKeys philox_keys(uint32_t k0, uint32_t k1) {
   return k;
 }
 
+// The same rounds with the round keys of problem 0 from the plan.
+__device__ __forceinline__ uint4 philox4x32_10_plan(uint4 c, const Plan& pl) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    const uint64_t p0 = (uint64_t)0xD2511F53u * c.x;
+    const uint64_t p1 = (uint64_t)0xCD9E8D57u * c.z;
+    c = make_uint4((uint32_t)(p1 >> 32) ^ c.y ^ pl.rk0[r], (uint32_t)p1, (uint32_t)(p0 >> 32) ^ c.w ^ pl.rk1[r],
+                   (uint32_t)p0);
+  }
+  return c;
+}
+
 __device__ __forceinline__ uint4 philox4x32_10(uint4 c, const PhiloxKeys& k) {
 #pragma unroll
   for (int r = 0; r < 10; ++r) {
@@ -366,11 +401,14 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
 
 // Per-model launch state: whether floors are set, and the launch shapes
 // (filled on first use) per kernel instance: [floors] for the solve and the
-// preparation, [path][floors] for the scorer (plain, dump, table).
+// preparation, [path][floors] for the scorer (plain, dump, table over one
+// problem, table over several).
+constexpr int kScoreVariants = 4;
 struct LaunchCache {
   int floors = 0;  // some class has a floor > 0: launch the kernel instances with floors
-  size_t solve_smem[2] = {0, 0}, prep_smem[2] = {0, 0}, score_smem[3][2] = {{0, 0}, {0, 0}, {0, 0}};
-  int score_blocks_per_sm[3][2] = {{0, 0}, {0, 0}, {0, 0}};
+  size_t solve_smem[2] = {0, 0}, prep_smem[2] = {0, 0};
+  size_t score_smem[kScoreVariants][2] = {};
+  int score_blocks_per_sm[kScoreVariants][2] = {};
 };
 
 cudaError_t launch_qtable(float* qn, int Q, cudaStream_t s);

@@ -145,6 +145,11 @@ __device__ __forceinline__ uint32_t kappa_walk(float mf, float t, float lam, flo
   return hi;
 }
 
+// t* of one realisation with row capacity C (defined below, with the scorer).
+template <int ROW, bool FL>
+__device__ __forceinline__ float tstar_of(float C, const float* kap, const float* thx, const float* mnx,
+                                          int step0, float lam, float rlam, float dl);
+
 // One CTA per (candidate, realisation sigma). Before the threshold search it
 // maps the quantile strata of the outcomes o = sigma, sigma + 2, ... into the
 // candidate's record: this and Cexcl read only the bounds, so with `early`
@@ -410,7 +415,6 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
       }
       if (m >= 1) s_row = 1;
       mnx[u] = (float)m;
-      if (u == 0) tab[H_M_FIRST] = (float)m;
     }
   } else {
     for (int u = warp; u <= Lt; u += nwarp) {
@@ -460,8 +464,7 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
       if (lane == 0) {
         if (m >= 1) s_row = 1;
         mnx[u] = (float)m;
-        if (u == 0) tab[H_M_FIRST] = (float)m;
-      }
+        }
     }
   }
   for (int u = Lt + tid; u < Lpad; u += blockDim.x) {
@@ -480,6 +483,9 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
     const bool fast = in_markstein_range(lam) && cmax <= 0x1p44f &&
                       (cx >= 0x1p-60f || (cx == 0.0f && (lo_c >= 0x1p-60f || hi_c == 0.0f)));
     tab[H_TH_BASE] = b0 >= 0 ? sTh[b0] : 0.0f;
+    // t* at row capacity Cexcl (no kappa entry is at or below it): the value of
+    // every scenario of this candidate whose tail gate is closed
+    tab[H_TCL] = tstar_of<2, FL>(cx, kap, thx, mnx, Lt ? P >> 1 : 0, lam, rl, dle);
     tab[H_L] = __int_as_float(Lt);
     tab[H_LPAD] = __int_as_float(Lpad);
     tab[H_CX] = cx;
@@ -739,10 +745,12 @@ __device__ uint64_t run_piece_dump(const Set& set, const Plan& pl, int item, int
 // among the outcome's W mapped quantiles) and the tail gate (l_y <= L_i); with
 // the gate closed the row keeps Cexcl whatever k is. So the segment has at most
 // W + 1 values of rint(Gamma' 2^40): gtab[k] for an open gate at position k,
-// gtab[W] for a closed gate. The block evaluates them once per chunk (two t*
-// each, the same arithmetic as a scenario), after which a scenario costs its
-// share of the Philox call, one index and one shared-memory load. Each entry
-// holds the value's upper bits (>> 20) and lower 20 bits, summed separately.
+// gtab[W] for a closed gate. The closed-gate value comes from the two t* at
+// Cexcl that the preparation stored (H_TCL); the block evaluates the W others
+// once per chunk (two t* each, the same arithmetic as a scenario), after which
+// a scenario costs its share of the Philox call, one index and one
+// shared-memory load. Each entry holds the value's upper bits (>> 20) and
+// lower 20 bits, summed separately.
 template <bool TS, int ROW, bool FL>
 __device__ __forceinline__ void build_gtab(uint2* gtab, int W, const float* win, const float* h0, const float* h1,
                                            const float* kap0, const float* thx0, const float* mnx0,
@@ -751,8 +759,8 @@ __device__ __forceinline__ void build_gtab(uint2* gtab, int W, const float* win,
   const float cx0 = h0[H_CX], cx1 = h1[H_CX];
   const float lam = h0[H_LAM], rlam = h0[H_RLAM], dl = h0[H_DLT];
   const float* capw = win + 4;
-  for (int k = threadIdx.x; k <= W; k += blockDim.x) {
-    const float cy = k < W ? capw[k] : 0.0f;  // a closed gate: the row keeps max(Cexcl, 0) = Cexcl
+  for (int k = threadIdx.x; k < W; k += blockDim.x) {
+    const float cy = capw[k];
     const float t0 = tstar_of<ROW, FL>(fmaxf(cx0, cy), kap0, thx0, mnx0, st0, lam, rlam, dl);
     const float t1 = tstar_of<ROW, FL>(fmaxf(cx1, cy), kap1, thx1, mnx1, st1, lam, rlam, dl);
     const uint64_t g = fixed40(__fsub_rn(t1, t0));
@@ -764,22 +772,44 @@ __device__ __forceinline__ void build_gtab(uint2* gtab, int W, const float* win,
 // two fields of the drawn entries (each field below 2^21), flushed into a
 // 64-bit total every 256 calls so that the 32-bit sums cannot wrap. With at
 // most 32 values per thread nothing is flushed and a warp's field sums stay
-// below 2^32.
+// below 2^32. Per sample: the capacity position umulhi(word, W); the tail gate,
+// (word & 0xFFFF) < kgs, as (word * 65536 mod 2^32) < kgs16 with kgs16 =
+// min(kgs 2^16, 2^32 - 1) (a multiply-add and a compare); the entry's shared
+// address base + index * 8 (a multiply-add); its load and two field sums. Two
+// calls per iteration give two independent Philox chains. KC: one problem, its
+// round keys read from the plan.
 struct GtabSum {
   uint32_t h, l;   // the last at most 1024 values
   uint64_t total;  // earlier values
 };
 
+template <bool KC>
+__device__ __forceinline__ uint4 draw_call(const Plan& pl, const PhiloxKeys& keys, uint32_t q, uint32_t ctr1,
+                                           uint32_t ctr2, uint32_t ctr3) {
+  if constexpr (KC) return philox4x32_10_plan(make_uint4(q, ctr1, ctr2, ctr3), pl);
+  else return philox4x32_10(make_uint4(q, ctr1, ctr2, ctr3), keys);
+}
+
+template <bool KC>
 __device__ __forceinline__ GtabSum sample_gtab(const Plan& pl, const PhiloxKeys& keys, int o, int cell, int q_lo,
-                                               int q_hi, const uint2* gtab, uint32_t kgs) {
+                                               int q_hi, uint32_t gtab_s, uint32_t kgs16) {
   const uint32_t ctr1 = (uint32_t)o, ctr2 = (uint32_t)cell, ctr3 = pl.round;
   const uint32_t W = (uint32_t)pl.W;
+  const uint32_t mul = pl.lo16_mul, eb = pl.entry_bytes;
   uint32_t gh = 0, glo = 0;
   auto take = [&](uint32_t word) {
-    const uint32_t idx = (word & 0xFFFFu) < kgs ? __umulhi(word, W) : W;
-    const uint2 v = gtab[idx];
-    gh += v.x;
-    glo += v.y;
+    const uint32_t cap = __umulhi(word, W);
+    const uint32_t idx = word * mul < kgs16 ? cap : W;
+    uint32_t a, b;
+    asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(a), "=r"(b) : "r"(gtab_s + idx * eb));
+    gh += a;
+    glo += b;
+  };
+  auto take4 = [&](const uint4& x) {
+    take(x.x);
+    take(x.y);
+    take(x.z);
+    take(x.w);
   };
   const int q_full = min(q_hi, pl.S >> 2);  // calls whose four samples all exist
   const int step = (int)blockDim.x;
@@ -787,12 +817,15 @@ __device__ __forceinline__ GtabSum sample_gtab(const Plan& pl, const PhiloxKeys&
   int q = q_lo + (int)threadIdx.x;
   while (q < q_full) {
     const int q_end = min(q_full, q + 256 * step);
-    for (; q < q_end; q += step) {
-      const uint4 x = philox4x32_10(make_uint4((uint32_t)q, ctr1, ctr2, ctr3), keys);
-      take(x.x);
-      take(x.y);
-      take(x.z);
-      take(x.w);
+    for (; q + step < q_end; q += 2 * step) {
+      const uint4 x0 = draw_call<KC>(pl, keys, (uint32_t)q, ctr1, ctr2, ctr3);
+      const uint4 x1 = draw_call<KC>(pl, keys, (uint32_t)(q + step), ctr1, ctr2, ctr3);
+      take4(x0);
+      take4(x1);
+    }
+    if (q < q_end) {
+      take4(draw_call<KC>(pl, keys, (uint32_t)q, ctr1, ctr2, ctr3));
+      q += step;
     }
     if (q < q_full) {
       total += ((uint64_t)gh << 20) + glo;
@@ -800,7 +833,7 @@ __device__ __forceinline__ GtabSum sample_gtab(const Plan& pl, const PhiloxKeys&
     }
   }
   if (q < q_hi) {  // the segment's last call, serving S mod 4 samples
-    const uint4 x = philox4x32_10(make_uint4((uint32_t)q, ctr1, ctr2, ctr3), keys);
+    const uint4 x = draw_call<KC>(pl, keys, (uint32_t)q, ctr1, ctr2, ctr3);
     const int nv = pl.S - 4 * q;
     take(x.x);
     if (nv > 1) take(x.y);
@@ -822,7 +855,7 @@ struct ScoreGrid {
 };
 
 // Which scoring path a launch takes.
-enum : int { SCORE_PLAIN = 0, SCORE_DUMP = 1, SCORE_TABLE = 2 };
+enum : int { SCORE_PLAIN = 0, SCORE_DUMP = 1, SCORE_TABLE = 2, SCORE_TABLE_MULTI = 3 };
 
 // Thread 0: stage the data of segment seg (its outcome window and both
 // candidate tables, header plus lcap_s entries each) into dst, completing on bar.
@@ -850,8 +883,9 @@ __device__ __forceinline__ void stage_segment(const Set& set, const Plan& pl, co
 // FL: some class is critical (the model has floors): row terms are gated by the
 // candidate class's floor (0, so always passed, for a class that is not).
 // GT: the table path (build_gtab), chosen by the host when a chunk's samples
-// outnumber a segment's W + 1 table entries; never with DUMP.
-template <bool DUMP, bool FL, bool GT>
+// outnumber a segment's W + 1 table entries; never with DUMP. KC (table path,
+// one problem): Philox round keys from the plan's parameters.
+template <bool DUMP, bool FL, bool GT, bool KC>
 __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, Plan pl, const float* rec,
                                                          uint64_t* sums, unsigned char* dump, int dump_stride,
                                                          ScoreGrid sg) {
@@ -931,33 +965,51 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
       uint2* gtab = gtab2 + (size_t)(j & 1) * (pl.W + 1);
       const int cell = ok ? __float_as_int(h0[H_CELL]) : -1;
       const bool use = cell >= 0 && cell < d.cells;  // a bad device-side id was flagged by k_prep
+      // passing tail positions of the stratum, as the top bits of a 16-bit field
       const uint32_t kgs = use ? (uint32_t)__float_as_int(stg[0]) << pl.sh : 0u;
+      const uint32_t kgs16 = (uint32_t)min((unsigned long long)kgs << 16, 0xFFFFFFFFull);
       if (use) {
-        const int Lp0 = __float_as_int(h0[H_LPAD]), Lp1 = __float_as_int(h1[H_LPAD]);
-        const bool r0 = __float_as_int(h0[H_ROW]) != 0, r1 = __float_as_int(h1[H_ROW]) != 0;
-        const bool f0 = __float_as_int(h0[H_FAST]) != 0, f1 = __float_as_int(h1[H_FAST]) != 0;
-        const int row = (!r0 && !r1) ? 0 : ((!r0 || f0) && (!r1 || f1)) ? 1 : 2;
+        const uint64_t gc = fixed40(__fsub_rn(h1[H_TCL], h0[H_TCL]));
+        const uint2 closed = make_uint2((uint32_t)(gc >> 20), (uint32_t)gc & 0xFFFFFu);
+        if (kgs == 0u) {
+          // the gate is closed at every position of the stratum: every entry
+          // is the closed-gate value (each scenario still draws its position)
+          for (int k = tid; k <= pl.W; k += blockDim.x) gtab[k] = closed;
+        } else {
+          if (tid == 0) {
+            gtab[pl.W] = closed;
+            // entries evaluated, once per segment (later chunks of a segment
+            // rebuild the same table): the measurement's algorithmic count
+            if (KC && part == 0) atomicAdd(&set.work[2], (unsigned long long)pl.W);
+          }
+          const int Lp0 = __float_as_int(h0[H_LPAD]), Lp1 = __float_as_int(h1[H_LPAD]);
+          const bool r0 = __float_as_int(h0[H_ROW]) != 0, r1 = __float_as_int(h1[H_ROW]) != 0;
+          const bool f0 = __float_as_int(h0[H_FAST]) != 0, f1 = __float_as_int(h1[H_FAST]) != 0;
+          const int row = (!r0 && !r1) ? 0 : ((!r0 || f0) && (!r1 || f1)) ? 1 : 2;
 #define FS_BUILD(TSV, ROWV, FLV) \
   build_gtab<TSV, ROWV, FLV>(gtab, pl.W, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, k1 + Lp1, k1 + 2 * Lp1)
 #define FS_BUILDS(TSV)                       \
   if (row == 0) FS_BUILD(TSV, 0, false);     \
   else if (row == 1) FS_BUILD(TSV, 1, FL);   \
   else FS_BUILD(TSV, 2, FL);
-        if (Lp0 <= sg.lcap_s && Lp1 <= sg.lcap_s) {
-          const float* k0 = h0 + kTableHeader;
-          const float* k1 = h1 + kTableHeader;
-          FS_BUILDS(true)
-        } else {
-          const float* k0 = rec + (size_t)item * pl.item_floats + kTableHeader;
-          const float* k1 = k0 + d.slot_floats;
-          FS_BUILDS(false)
-        }
+          if (Lp0 <= sg.lcap_s && Lp1 <= sg.lcap_s) {
+            const float* k0 = h0 + kTableHeader;
+            const float* k1 = h1 + kTableHeader;
+            FS_BUILDS(true)
+          } else {
+            const float* k0 = rec + (size_t)item * pl.item_floats + kTableHeader;
+            const float* k1 = k0 + d.slot_floats;
+            FS_BUILDS(false)
+          }
 #undef FS_BUILDS
 #undef FS_BUILD
-        const int p = __float_as_int(h0[H_P]);
-        if (p != keys_p) {
-          keys = philox_keys(pl.key0, pl.key1 ^ (pl.stream_base + (uint32_t)p));
-          keys_p = p;
+        }
+        if (!KC) {
+          const int p = __float_as_int(h0[H_P]);
+          if (p != keys_p) {
+            keys = philox_keys(pl.key0, pl.key1 ^ (pl.stream_base + (uint32_t)p));
+            keys_p = p;
+          }
         }
       }
       if (__syncthreads_or(!ok)) {  // the table is complete; or some wait gave up
@@ -967,7 +1019,7 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
         return;
       }
       GtabSum gs{0u, 0u, 0ull};
-      if (use) gs = sample_gtab(pl, keys, o, cell, q_lo, q_hi, gtab, kgs);
+      if (use) gs = sample_gtab<KC>(pl, keys, o, cell, q_lo, q_hi, smem_u32(gtab), kgs16);
       uint64_t v;
       if (small_gt) {  // at most 64 values per thread: each field's warp sum fits in 32 bits
         const uint32_t H = __reduce_add_sync(0xffffffffu, gs.h);
@@ -1123,10 +1175,13 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
   const bool table = !dump && pl.W <= 4096 && 3LL * (pl.W + 1) <= 2 * chunk_min;
   const size_t stages = 16 + 2 * (size_t)(pl.Wp + 2 * sg.tcopy) * 4;
   const size_t smem = stages + (table ? ((size_t)16 * (pl.W + 1) + 15) / 16 * 16 : 0);
-  const int v = dump ? SCORE_DUMP : table ? SCORE_TABLE : SCORE_PLAIN, fl = lc.floors ? 1 : 0;
-  auto kern = dump ? (fl ? k_score<true, true, false> : k_score<true, false, false>)
-          : table ? (fl ? k_score<false, true, true> : k_score<false, false, true>)
-                  : (fl ? k_score<false, true, false> : k_score<false, false, false>);
+  const int v = dump ? SCORE_DUMP : table ? (it.p == nullptr ? SCORE_TABLE : SCORE_TABLE_MULTI) : SCORE_PLAIN;
+  const int fl = lc.floors ? 1 : 0;
+  const bool one = it.p == nullptr;  // every item belongs to problem 0
+  auto kern = dump ? (fl ? k_score<true, true, false, false> : k_score<true, false, false, false>)
+          : table ? (one ? (fl ? k_score<false, true, true, true> : k_score<false, false, true, true>)
+                         : (fl ? k_score<false, true, true, false> : k_score<false, false, true, false>))
+                  : (fl ? k_score<false, true, false, false> : k_score<false, false, false, false>);
   if (smem != lc.score_smem[v][fl]) {
     int per_sm = 0;
     cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(kern), smem);

@@ -111,7 +111,7 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
     off = up256(off + bytes);
     return o;
   };
-  const size_t o_status = take(4), o_work = take(16), o_part = take(16 * (size_t)kFinalizeMaxBlocks);
+  const size_t o_status = take(4), o_work = take(24), o_part = take(16 * (size_t)kFinalizeMaxBlocks);
   const size_t o_qn = quantile_dev ? 0 : take(4 * (size_t)Q);
   const size_t o_theta = take(8 * (size_t)d.theta_cap), o_nth = take(8);
   const size_t o_rowc = take(8 * (size_t)d.K4), o_rowb = take(8 * (size_t)d.K4);
@@ -188,6 +188,7 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
   pl.calls = (smp->S + 3) / 4;
   pl.Wp = Wp;
   pl.item_floats = (long long)item_floats;
+  plan_round_keys(pl);
 
   // --- the scoring pipeline on the caller's stream, then wait and report
   cudaStream_t s = static_cast<cudaStream_t>(cuda_stream);
@@ -210,7 +211,7 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
     for (int f = 0; f < 2; ++f) {
       g.solve_smem[f] = std::max(g.solve_smem[f], lc.solve_smem[f]);
       g.prep_smem[f] = std::max(g.prep_smem[f], lc.prep_smem[f]);
-      for (int v = 0; v < 3; ++v)
+      for (int v = 0; v < kScoreVariants; ++v)
         if (lc.score_smem[v][f] && lc.score_smem[v][f] != g.score_smem[v][f]) {
           g.score_smem[v][f] = lc.score_smem[v][f];
           g.score_blocks_per_sm[v][f] = lc.score_blocks_per_sm[v][f];
