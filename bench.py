@@ -88,7 +88,7 @@ def algorithmic_ops(w, entries_per_launch=None) -> float:
 
 # ncu summaries with the DRAM bytes of one k_score launch, per workload; used
 # for roofline.traffic only while the scorer source is the one profiled.
-PROFILES = {1: "k_score_paper_scale.md", 3: "k_score_large.md"}
+PROFILES = {1: "k_score_paper_scale.md", 3: "k_score_large.md"}  # sha-checked below
 
 
 def _env_int(name, default):
