@@ -21,7 +21,7 @@ SOLVER_FRONTIER = 1
 class _Problem(C.Structure):
     _fields_ = [("K", C.c_int), ("B", C.c_int), ("G", C.c_int),
                 ("demand", C.POINTER(C.c_float)), ("slo", C.POINTER(C.c_float)),
-                ("floor", C.POINTER(C.c_float))]
+                ("floor", C.POINTER(C.c_float)), ("prior", C.c_int)]
 
 
 class _Alloc(C.Structure):
@@ -86,6 +86,8 @@ def lib():
         _lib.or_score_cached.argtypes = [C.POINTER(_Problem), fp, fp, fp, fp, fp, C.c_int,
                                          C.c_uint64, C.c_uint32, C.c_uint32, C.c_int, ip, C.c_int,
                                          C.c_int, C.c_int, C.POINTER(C.c_int64), fp]
+        _lib.or_refit.argtypes = [C.POINTER(_Problem), C.c_int, C.c_int32, C.c_float, C.c_float,
+                                  fp, fp, fp, fp]
         _lib.or_reduce.argtypes = [C.POINTER(_Problem), C.c_int, ip, C.c_int, C.c_int, C.c_float,
                                    C.POINTER(C.c_int64), C.POINTER(C.c_double),
                                    C.POINTER(C.c_double), C.POINTER(C.c_int64), ip]
@@ -108,24 +110,31 @@ def _ptr(a: np.ndarray, ctype):
     return a.ctypes.data_as(C.POINTER(ctype))
 
 
+PRIOR_REVEALED = 0
+PRIOR_MONOTONE = 1
+
+
 class Problem:
     """K classes, B bins, budget G, demands, SLOs and optional critical floors
-    delta_i in [0, 1] (0 = not critical) (Section 3)."""
+    delta_i in [0, 1] (0 = not critical) (Section 3); the interval prior used
+    when a cell is measured (PRIOR_REVEALED or PRIOR_MONOTONE, Section 4.1)."""
 
-    def __init__(self, K, B, G, demand, slo, floor=None):
+    def __init__(self, K, B, G, demand, slo, floor=None, prior=PRIOR_REVEALED):
         self.K, self.B, self.G = int(K), int(B), int(G)
         self.demand = _f32(demand)
         self.slo = _f32(slo)
         self.floor = None if floor is None else _f32(floor)
         assert self.demand.size == self.K and self.slo.size == self.K
         assert self.floor is None or self.floor.size == self.K
+        self.prior = int(prior)
         self._s = _Problem(self.K, self.B, self.G, _ptr(self.demand, C.c_float),
                            _ptr(self.slo, C.c_float),
-                           None if self.floor is None else _ptr(self.floor, C.c_float))
+                           None if self.floor is None else _ptr(self.floor, C.c_float), self.prior)
 
     @staticmethod
     def of(w) -> "Problem":
-        return Problem(w.K, w.B, w.G, w.demand, w.slo, getattr(w, "floor", None))
+        return Problem(w.K, w.B, w.G, w.demand, w.slo, getattr(w, "floor", None),
+                       getattr(w, "prior", PRIOR_REVEALED))
 
     @property
     def cells(self) -> int:
@@ -305,6 +314,17 @@ def reduce_sums(w, candidates, sum_eo, gamma_t, O=None, S=None) -> ScoreResult:
     if rc:
         raise ValueError("oracle reduce failed")
     return ScoreResult(se.copy(), gap, sc, scf, float(np.float32(gamma_t)), int(best.value), None)
+
+
+def refit(prob: Problem, cell, c, l, cap_lo, cap_hi, tail_lo, tail_hi, prior=None):
+    """The four bound arrays after measuring (c, l) at cell under the prior
+    (the problem's when None); returns new arrays."""
+    arrs = [_f32(x).copy() for x in (cap_lo, cap_hi, tail_lo, tail_hi)]
+    rc = lib().or_refit(C.byref(prob._s), prob.prior if prior is None else int(prior), int(cell),
+                        float(c), float(l), *[_ptr(x, C.c_float) for x in arrs])
+    if rc:
+        raise ValueError("oracle refit failed")
+    return arrs
 
 
 def certificate(prob: Problem, cap_lo, cap_hi, tail_lo, tail_hi, revealed, eps,

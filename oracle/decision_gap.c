@@ -9,9 +9,9 @@
  * here the tier-2 objective, Gamma = t*(A+) - t*(A-) (the "max-min gap").
  * Section 4.3: score_t(e) = E[Gamma_t - Gamma_{t+1} | e]; the expectation is
  * a Monte-Carlo mean over O outcome strata x S samples. Revealing e
- * collapses its interval to the drawn point in both realisations; other
- * cells keep their intervals (the paper's interval refit of the other cells
- * is not specified).
+ * collapses its interval to the drawn point in both realisations and refits
+ * the other intervals under the problem's prior (prior.c): none under the
+ * revealed-only prior, the rest of e's row under the monotone prior.
  *
  * Sums are taken in fixed point: g = rint(Gamma' * 2^40) as int64, so the
  * result does not depend on summation order.
@@ -40,6 +40,19 @@ int or_base_gap(const or_problem *p, const float *cap_lo, const float *cap_hi,
 
 static int cells_of(const or_problem *p) { return p->K * OR_T * p->B; }
 
+/* The base bounds of cell's row back into the realisations' working arrays
+ * (cm = cap_lo, cp = cap_hi, tp = tail_lo, tm = tail_hi). */
+static void restore_row(const or_problem *p, int32_t cell, const float *cap_lo, const float *cap_hi,
+                        const float *tail_lo, const float *tail_hi,
+                        float *cm, float *cp, float *tp, float *tm)
+{
+    int first = (cell / p->B) * p->B;
+    for (int x = first; x < first + p->B; ++x) {
+        cm[x] = cap_lo[x]; cp[x] = cap_hi[x];
+        tp[x] = tail_lo[x]; tm[x] = tail_hi[x];
+    }
+}
+
 int or_scenario(const or_problem *p, const float *cap_lo, const float *cap_hi,
                 const float *tail_lo, const float *tail_hi, const float *qn, int Q,
                 uint64_t seed, uint32_t stream_id, uint32_t round, int32_t cell,
@@ -59,8 +72,8 @@ int or_scenario(const or_problem *p, const float *cap_lo, const float *cap_hi,
     memcpy(tm, tail_hi, sizeof(float) * cells);
     memcpy(cp, cap_hi, sizeof(float) * cells);
     memcpy(tp, tail_lo, sizeof(float) * cells);
-    cm[cell] = cy; tm[cell] = ly;
-    cp[cell] = cy; tp[cell] = ly;
+    /* the revealed cell at (c_y, l_y) in both realisations, the rest refit */
+    or_refit(p, p->prior, cell, cy, ly, cm, cp, tp, tm);
     int rc = solve(p, cm, tm, solver, minus);
     if (!rc) rc = solve(p, cp, tp, solver, plus);
     free(cm);
@@ -110,8 +123,8 @@ int or_score(const or_problem *p, const float *cap_lo, const float *cap_hi,
                 or_draw_index(seed, stream_id, round, cell, Q, O, o, s, &kc, &kl);
                 float cy = or_map(cap_lo[cell], cap_hi[cell], qn[kc]);
                 float ly = or_map(tail_lo[cell], tail_hi[cell], qn[kl]);
-                cm[cell] = cy; tm[cell] = ly;
-                cp[cell] = cy; tp[cell] = ly;
+                restore_row(p, cell, cap_lo, cap_hi, tail_lo, tail_hi, cm, cp, tp, tm);
+                or_refit(p, p->prior, cell, cy, ly, cm, cp, tp, tm);
                 rc = solve(p, cm, tm, solver, &am);
                 if (!rc) rc = solve(p, cp, tp, solver, &ap);
                 if (rc) { free(cm); return rc; }
@@ -126,8 +139,7 @@ int or_score(const or_problem *p, const float *cap_lo, const float *cap_hi,
             if (sum_eo) sum_eo[(size_t)e * O + o] = acc;
             tot += acc;
         }
-        cm[cell] = cap_lo[cell]; tm[cell] = tail_hi[cell];
-        cp[cell] = cap_hi[cell]; tp[cell] = tail_lo[cell];
+        restore_row(p, cell, cap_lo, cap_hi, tail_lo, tail_hi, cm, cp, tp, tm);
 
         int64_t sc = g_t * n - tot;                        /* sum of Gamma_t - Gamma_{t+1} */
         if (gap) gap[e] = ((double)tot * 0x1p-40) / (double)n;
@@ -185,8 +197,10 @@ int or_reduce(const or_problem *p, int n_cand, const int32_t *cand, int O, int S
  * The fixed-point sums of or_score, scenario for scenario, with each
  * candidate's solves cached. Both solvers read a cell's tail only through
  * the SLO test tail <= L_i (Eq. 5), and c_y is a function of the capacity
- * position k_cap alone, so a scenario's two allocations, and its Gamma',
- * depend on its draw only through the pair (k_cap, l_y <= L_i). A scenario
+ * position k_cap alone, so under the revealed-only prior a scenario's two
+ * allocations, and its Gamma', depend on its draw only through the pair
+ * (k_cap, l_y <= L_i); under the monotone prior l_y also moves the tail
+ * bounds of the row's other bins, so the key is (k_cap, k_tail). A scenario
  * whose pair was met before in the same candidate reuses that scenario's
  * rint(Gamma' 2^40); every other step (draws, maps, patches, solves, sums)
  * is or_score's. Used to compute expected sums of workloads too large for
@@ -212,8 +226,11 @@ int or_score_cached(const or_problem *p, const float *cap_lo, const float *cap_h
     if (gamma_t) *gamma_t = gt;
 
     float *cm = (float *)malloc(sizeof(float) * cells * 4);
-    int64_t *memo = (int64_t *)malloc(sizeof(int64_t) * 2 * (size_t)Q);
-    uint8_t *known = (uint8_t *)malloc(2 * (size_t)Q);
+    /* key: (k_cap, gate) under the revealed-only prior, (k_cap, k_tail
+     * within the stratum) under the monotone prior */
+    const size_t nkey = p->prior == OR_PRIOR_REVEALED ? 2 * (size_t)Q : (size_t)Q * (size_t)(Q / O);
+    int64_t *memo = (int64_t *)malloc(sizeof(int64_t) * nkey);
+    uint8_t *known = (uint8_t *)malloc(nkey);
     if (!cm || !memo || !known) { free(cm); free(memo); free(known); return -2; }
     float *tm = cm + cells, *cp = cm + 2 * cells, *tp = cm + 3 * cells;
     memcpy(cm, cap_lo, sizeof(float) * cells);
@@ -224,7 +241,7 @@ int or_score_cached(const or_problem *p, const float *cap_lo, const float *cap_h
     for (int e = 0; e < n_cand; ++e) {
         const int32_t cell = cand[e];
         const float L = p->slo[cell / (OR_T * p->B)];
-        memset(known, 0, 2 * (size_t)Q);
+        memset(known, 0, nkey);
         for (int o = 0; o < O; ++o) {
             int64_t acc = 0;
             for (int s = 0; s < S; ++s) {
@@ -232,10 +249,11 @@ int or_score_cached(const or_problem *p, const float *cap_lo, const float *cap_h
                 or_draw_index(seed, stream_id, round, cell, Q, O, o, s, &kc, &kl);
                 float cy = or_map(cap_lo[cell], cap_hi[cell], qn[kc]);
                 float ly = or_map(tail_lo[cell], tail_hi[cell], qn[kl]);
-                size_t key = 2 * (size_t)kc + (ly <= L ? 1u : 0u);
+                size_t key = p->prior == OR_PRIOR_REVEALED ? 2 * (size_t)kc + (ly <= L ? 1u : 0u)
+                                                           : (size_t)kc * (size_t)(Q / O) + (size_t)(kl % (Q / O));
                 if (!known[key]) {
-                    cm[cell] = cy; tm[cell] = ly;
-                    cp[cell] = cy; tp[cell] = ly;
+                    restore_row(p, cell, cap_lo, cap_hi, tail_lo, tail_hi, cm, cp, tp, tm);
+                    or_refit(p, p->prior, cell, cy, ly, cm, cp, tp, tm);
                     rc = solve(p, cm, tm, solver, &am);
                     if (!rc) rc = solve(p, cp, tp, solver, &ap);
                     if (rc) { free(cm); free(memo); free(known); return rc; }
@@ -247,8 +265,7 @@ int or_score_cached(const or_problem *p, const float *cap_lo, const float *cap_h
             }
             sum_eo[(size_t)e * O + o] = acc;
         }
-        cm[cell] = cap_lo[cell]; tm[cell] = tail_hi[cell];
-        cp[cell] = cap_hi[cell]; tp[cell] = tail_lo[cell];
+        restore_row(p, cell, cap_lo, cap_hi, tail_lo, tail_hi, cm, cp, tp, tm);
     }
     free(cm); free(memo); free(known);
     return 0;
@@ -320,8 +337,7 @@ int or_replay_stream(const or_problem *p, const float *prior_cap_lo, const float
     double gs = 0.0;
     for (int q = 0; q < r0; ++q) {
         int c = perm[q];
-        clo[c] = chi[c] = truth_cap[c];
-        tlo[c] = thi[c] = truth_tail[c];
+        or_refit(p, p->prior, c, truth_cap[c], truth_tail[c], clo, chi, tlo, thi);
         rev[c] = 1;
         reveal_order[nrev++] = c;
         gs += 300.0 * (double)(1 << ((c / p->B) % OR_T));
@@ -345,8 +361,7 @@ int or_replay_stream(const or_problem *p, const float *prior_cap_lo, const float
                           solver, NULL, NULL, NULL, NULL, &g2, &bestc, NULL);
             if (rc) break;
         }
-        clo[bestc] = chi[bestc] = truth_cap[bestc];
-        tlo[bestc] = thi[bestc] = truth_tail[bestc];
+        or_refit(p, p->prior, bestc, truth_cap[bestc], truth_tail[bestc], clo, chi, tlo, thi);
         rev[bestc] = 1;
         reveal_order[nrev++] = bestc;
         gs += 300.0 * (double)(1 << ((bestc / p->B) % OR_T));

@@ -46,7 +46,12 @@ typedef struct {
     const float *slo;   /* L_i [K], seconds */
     const float *floor; /* delta_i [K] in [0, 1], tier 1 of Section 3; 0 = class i is
                            not critical; NULL = no critical class */
+    int prior;          /* interval refit after a measurement (prior.c): OR_PRIOR_REVEALED
+                           or OR_PRIOR_MONOTONE */
 } or_problem;
+
+#define OR_PRIOR_REVEALED 0  /* only the measured cell collapses */
+#define OR_PRIOR_MONOTONE 1  /* and its row's other bins are refit (nondecreasing in load) */
 
 /* One allocation. A class with replicas[i] == 0 has tp = 0, bin = -1. */
 typedef struct {
@@ -113,6 +118,11 @@ int or_score_cached(const or_problem *p, const float *cap_lo, const float *cap_h
 /* Expectations, scores and argmax (Section 4.3) from the sums. */
 int or_reduce(const or_problem *p, int n_cand, const int32_t *cand, int O, int S, float gamma_t,
               const int64_t *sum_eo, double *gap, double *score, int64_t *score_fixed, int32_t *best);
+
+/* Collapse cell to the measurement (c, l) and refit the other intervals under
+ * the given prior (Section 4.1; prior.c), in place. */
+int or_refit(const or_problem *p, int prior, int32_t cell, float c, float l,
+             float *cap_lo, float *cap_hi, float *tail_lo, float *tail_hi);
 
 /* Certificate (Section 4.2): 0 undecided, 1 certified feasible, 2 certified
  * infeasible (even A+ misses a critical floor). */

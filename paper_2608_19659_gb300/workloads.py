@@ -54,6 +54,7 @@ class Workload:
     stream_id: int = 0
     round: int = 0
     floor: np.ndarray | None = None  # [K] float32 critical floors delta_i in [0, 1] (0 = not critical)
+    prior: int = 0  # interval refit after a measurement: 0 revealed cell only, 1 monotone in load bin
 
     @property
     def cells(self) -> int:
