@@ -299,6 +299,27 @@ int fs_solve_bounds(fs_model *m, fs_allocation *minus, fs_allocation *plus, floa
 int fs_reveal(fs_model *m, int32_t cell, float cap, float tail);
 
 /*
+ * fs_set_prior -- how a measurement updates the uncertainty state (Section
+ * 4.1: intervals from an interior-knee structural prior plus measured
+ * residuals; Algorithm 1 refits them after every reveal).
+ *   FS_PRIOR_REVEALED (0, the state a new model starts in): the measured
+ *     cell collapses to its values; no other cell changes (the revealed-only
+ *     prior).
+ *   FS_PRIOR_MONOTONE (1): the reading of the interior-knee prior used here:
+ *     within a (class, TP) row, capacity and binding tail are nondecreasing
+ *     in the load bin, so a measurement (c, l) of bin b also refits the row's
+ *     other bins: for bins above b, lo = min(max(lo, v), hi); for bins below
+ *     b, hi = max(min(hi, v), lo) (v = c for capacity, l for the tail); no
+ *     interval ever widens or empties, and other rows do not change.
+ * The prior applies to fs_reveal, to fs_replay's reveals and to every
+ * scoring scenario (the drawn outcome refits the candidate's row in both
+ * realisations before they are solved).
+ */
+#define FS_PRIOR_REVEALED 0
+#define FS_PRIOR_MONOTONE 1
+int fs_set_prior(fs_model *m, int32_t prior);
+
+/*
  * fs_get_state -- the model's current uncertainty state, for checkpointing
  * the profiling loop: bounds [K][4][B] (as staged by the last fs_load_model,
  * fs_update_bounds or fs_reveal) and revealed flags [K][4][B] (0 / 1) into

@@ -628,13 +628,16 @@ int fs_reveal(fs_model* m, int32_t cell, float cap, float tail) {
   if (cell < 0 || cell >= m->d.cells) return fail(FS_EINVAL, "cell %d out of range", cell);
   if (!std::isfinite(cap) || cap < 0.0f || !std::isfinite(tail) || tail < 0.0f)
     return fail(FS_EINVAL, "measured values must be finite and >= 0");
-  const int cells = m->d.cells;
-  m->h_bounds[(size_t)CAP_LO * cells + cell] = canon(cap);
-  m->h_bounds[(size_t)CAP_HI * cells + cell] = canon(cap);
-  m->h_bounds[(size_t)TAIL_LO * cells + cell] = canon(tail);
-  m->h_bounds[(size_t)TAIL_HI * cells + cell] = canon(tail);
+  refit_cell(m->h_bounds.data(), m->d.cells, m->d.B, m->set.prior, cell, canon(cap), canon(tail));
   m->h_revealed[cell] = 1;
   return stage_bounds(m);
+}
+
+int fs_set_prior(fs_model* m, int32_t prior) {
+  if (!m) return fail(FS_EINVAL, "model is NULL");
+  if (prior != FS_PRIOR_REVEALED && prior != FS_PRIOR_MONOTONE) return fail(FS_EINVAL, "prior %d is not 0 or 1", prior);
+  m->set.prior = prior;
+  return FS_OK;
 }
 
 int fs_get_state(const fs_model* m, float* cap_lo, float* cap_hi, float* tail_lo, float* tail_hi,

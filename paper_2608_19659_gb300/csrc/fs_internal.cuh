@@ -45,11 +45,17 @@ enum : int {
   H_TCL = 1,      // t* of this realisation at row capacity Cexcl: every scenario whose tail gate is closed
   H_L = 2,        // entries (int)
   H_LPAD = 3,     // entries padded to 4 (int)
-  H_CX = 4,       // best capacity of row r without the candidate's bin
-  H_BX = 5,       // its bin (int, -1 none)
-  H_CMAX = 6,     // max(Cexcl, cap_hi of the candidate)
+  // Row r's capacity C' in a scenario drawing c_y with tail gate g (Eq. 5):
+  //   C' = max(g ? max(P_open, c_y) : P_closed, min(max(c_y, F_lo), F_hi))
+  // Without the structural prior P_open = P_closed = Cexcl (the row's best
+  // SLO-feasible capacity without the candidate's bin) and F_lo = F_hi = 0;
+  // with it the row's other bins are refit by the draw (see k_prep).
+  H_CX = 4,       // P_closed
+  H_BX = 5,       // bin of Cexcl (int, -1 none; without the prior)
+  H_PO = 6,       // P_open
   H_LAM = 7,      // demand of the candidate's class
-  H_LO_C = 8, H_HI_C = 9, H_LO_L = 10, H_HI_L = 11,  // candidate cell bounds
+  H_LF = 8, H_HF = 9,  // F_lo, F_hi
+  H_LO_L = 10, H_HI_L = 11,  // candidate cell's tail bounds
   H_SLO = 12,     // SLO of the candidate's class
   H_CELL = 13,    // candidate cell (int)
   H_P = 14,       // problem (int)
@@ -97,7 +103,42 @@ struct Set {
   const int* skip;      // [P] or nullptr: base solves skip problems with skip[p] >= 0
   int* rtab;            // [P][2][kRowTabMax] or nullptr: row tables of the scoring solves,
                         // word (row rho, threshold k) at k K4 + rho
+  int prior;            // interval refit after a measurement: 0 the measured cell only,
+                        // 1 also its row's other bins (capacity and tail nondecreasing in load)
 };
+
+// The refit of one bound after a measurement v under the monotone prior: a
+// lower bound rises to v, an upper bound falls to v, clamped into [lo, hi]
+// so that the interval never empties.
+__host__ __device__ __forceinline__ float raise_lo(float lo, float hi, float v) { return fminf(fmaxf(lo, v), hi); }
+__host__ __device__ __forceinline__ float lower_hi(float lo, float hi, float v) { return fmaxf(fminf(hi, v), lo); }
+
+// Collapse cell to the measurement (c, l) in the bounds [4][cells] and, under
+// the monotone prior, refit its row: bins above it in load get lower bounds of
+// (c, l), bins below it upper bounds.
+__host__ __device__ __forceinline__ void refit_cell(float* bp, int cells, int B, int prior, int cell, float c,
+                                                    float l) {
+  bp[0 * (size_t)cells + cell] = c;
+  bp[1 * (size_t)cells + cell] = c;
+  bp[2 * (size_t)cells + cell] = l;
+  bp[3 * (size_t)cells + cell] = l;
+  if (prior != 1) return;
+  const int first = cell - cell % B, be = cell % B;
+  for (int b = 0; b < B; ++b) {
+    const size_t x = (size_t)first + b;
+    float* clo = bp + x;
+    float* chi = bp + (size_t)cells + x;
+    float* tlo = bp + 2 * (size_t)cells + x;
+    float* thi = bp + 3 * (size_t)cells + x;
+    if (b > be) {
+      *clo = raise_lo(*clo, *chi, c);
+      *tlo = raise_lo(*tlo, *thi, l);
+    } else if (b < be) {
+      *chi = lower_hi(*clo, *chi, c);
+      *thi = lower_hi(*tlo, *thi, l);
+    }
+  }
+}
 
 // Scenario plan shared by a launch.
 struct Plan {
@@ -403,12 +444,14 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
 // (filled on first use) per kernel instance: [floors] for the solve and the
 // preparation, [path][floors] for the scorer (plain, dump, table over one
 // problem, table over several).
+// The preparation's and the scorer's instances are indexed by mode = floors +
+// 2 prior (0..3).
 constexpr int kScoreVariants = 4;
 struct LaunchCache {
   int floors = 0;  // some class has a floor > 0: launch the kernel instances with floors
-  size_t solve_smem[2] = {0, 0}, prep_smem[2] = {0, 0};
-  size_t score_smem[kScoreVariants][2] = {};
-  int score_blocks_per_sm[kScoreVariants][2] = {};
+  size_t solve_smem[2] = {0, 0}, prep_smem[4] = {0, 0, 0, 0};
+  size_t score_smem[kScoreVariants][4] = {};
+  int score_blocks_per_sm[kScoreVariants][4] = {};
 };
 
 cudaError_t launch_qtable(float* qn, int Q, cudaStream_t s);

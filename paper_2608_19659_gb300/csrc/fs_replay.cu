@@ -4,7 +4,8 @@
 // and hidden truth. A round runs, for all streams still going:
 //   A-, A+ (k_solve) -> certificate (Section 4.2) -> candidate list (the
 //   unrevealed cells in the stream's reveal order) -> k_prep / k_score
-//   (Section 4.3) -> argmax -> reveal (interval collapses to the truth).
+//   (Section 4.3) -> argmax -> reveal (interval collapses to the truth; under
+//   the monotone prior the rest of its row is refit, Section 4.1).
 // The fixed-order policy skips the scoring and reveals the next cell of the
 // stream's order.
 // The host only reads the number of streams still going once per round.
@@ -20,10 +21,7 @@ __device__ __forceinline__ void reveal_cell(const Set& set, const ReplayState& r
   float* bp = set.bounds + (size_t)p * 4 * d.cells;
   const float tc = rs.truth[((size_t)p * 2) * d.cells + c];
   const float tl = rs.truth[((size_t)p * 2 + 1) * d.cells + c];
-  bp[(size_t)CAP_LO * d.cells + c] = tc;
-  bp[(size_t)CAP_HI * d.cells + c] = tc;
-  bp[(size_t)TAIL_LO * d.cells + c] = tl;
-  bp[(size_t)TAIL_HI * d.cells + c] = tl;
+  refit_cell(bp, d.cells, d.B, set.prior, c, tc, tl);  // collapse c; under the prior, refit its row
   set.revealed[(size_t)p * d.cells + c] = 1;
   const int q = rs.n_revealed[p]++;
   rs.reveal_order[(size_t)p * d.cells + q] = c;

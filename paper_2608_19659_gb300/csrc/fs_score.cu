@@ -155,13 +155,13 @@ __device__ __forceinline__ float tstar_of(float C, const float* kap, const float
 // candidate's record: this and Cexcl read only the bounds, so with `early`
 // they overlap the base solve that precedes this kernel. FL: some class is
 // critical (the model has floors).
-template <bool FL>
+template <bool FL, bool RF>
 __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan pl, float* rec,
                                                        uint64_t* sums, int early) {
   extern __shared__ __align__(16) unsigned char smraw[];
   float* sC = reinterpret_cast<float*>(smraw);  // [256]
   float* sTh = sC + 256;                          // [theta_cap]
-  __shared__ float s_cx, s_cmax;
+  __shared__ float s_cx, s_cmax, s_pc, s_po, s_lf, s_hf;
   __shared__ int s_bx, s_row;
   __shared__ float sLam[FS_MAX_CLASSES], sRl[FS_MAX_CLASSES];  // demand and RN(1/demand)
   __shared__ float sDl[FS_MAX_CLASSES];                          // floor delta_i (0: not critical)
@@ -204,7 +204,60 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
   const float lo_l = bp[(size_t)TAIL_LO * d.cells + cell], hi_l = bp[(size_t)TAIL_HI * d.cells + cell];
 
   // best SLO-feasible capacity of row r without bin b_e (ties: lower bin)
-  if (warp == 0) {
+  if (RF) {
+    // Under the monotone prior a scenario's draw (c_y, l_y) also refits row
+    // r's other bins (capacity and tail nondecreasing in the load bin). For
+    // realisation sigma the row's capacity is then
+    //   C' = max(g ? max(P_open, c_y) : P_closed, min(max(c_y, F_lo), F_hi)):
+    // A- (sigma 0): a bin below b_e keeps cap_lo and its upper tail falls to
+    //   max(min(tail_hi, l_y), tail_lo), which passes the SLO iff tail_hi <= L,
+    //   or g and tail_lo <= L (P); a bin above b_e passes iff tail_hi <= L and
+    //   its lower capacity rises to min(max(cap_lo, c_y), cap_hi), whose
+    //   maximum over such bins is min(max(c_y, max cap_lo), max cap_hi) (F).
+    // A+ (sigma 1): a bin above b_e keeps cap_hi and its lower tail rises to
+    //   min(max(tail_lo, l_y), tail_hi), which passes iff tail_hi <= L, or g
+    //   and tail_lo <= L (P); a bin below b_e passes iff tail_lo <= L and its
+    //   upper capacity falls to max(min(cap_hi, c_y), cap_lo) (F).
+    // So C' depends on the draw only through (c_y, g), as without the prior.
+    if (warp == 0) {
+      float pc = 0.0f, po = 0.0f, lf = 0.0f, hf = 0.0f;
+      const float* cl = bp + (size_t)CAP_LO * d.cells + (size_t)rr * d.B;
+      const float* ch = bp + (size_t)CAP_HI * d.cells + (size_t)rr * d.B;
+      const float* tl = bp + (size_t)TAIL_LO * d.cells + (size_t)rr * d.B;
+      const float* th = bp + (size_t)TAIL_HI * d.cells + (size_t)rr * d.B;
+      for (int b = lane; b < d.B; b += 32) {
+        if (b == be) continue;
+        const bool p_side = sigma ? b > be : b < be;  // bins refit only in their tail
+        const float cap = sigma ? ch[b] : cl[b];
+        if (p_side) {
+          if (th[b] <= L) pc = fmaxf(pc, cap);
+          if (tl[b] <= L) po = fmaxf(po, cap);
+        } else if ((sigma ? tl[b] : th[b]) <= L) {  // bins refit only in their capacity
+          lf = fmaxf(lf, cl[b]);
+          hf = fmaxf(hf, ch[b]);
+        }
+      }
+      for (int off = 16; off; off >>= 1) {
+        pc = fmaxf(pc, __shfl_xor_sync(0xffffffffu, pc, off));
+        po = fmaxf(po, __shfl_xor_sync(0xffffffffu, po, off));
+        lf = fmaxf(lf, __shfl_xor_sync(0xffffffffu, lf, off));
+        hf = fmaxf(hf, __shfl_xor_sync(0xffffffffu, hf, off));
+      }
+      if (lane == 0) {
+        po = fmaxf(po, pc);
+        // the table covers C' from its least (c_y = cap_lo, gate closed) to
+        // its largest value (c_y = cap_hi, gate open)
+        s_cx = fmaxf(pc, fminf(fmaxf(lo_c, lf), hf));
+        s_cmax = fmaxf(fmaxf(po, hi_c), fminf(fmaxf(hi_c, lf), hf));
+        s_pc = pc;
+        s_po = po;
+        s_lf = lf;
+        s_hf = hf;
+        s_bx = -1;
+        s_row = 0;
+      }
+    }
+  } else if (warp == 0) {
     float best = 0.0f;
     int bb = -1;
     for (int b = lane; b < d.B; b += 32) {
@@ -230,6 +283,8 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
       s_cx = bb >= 0 ? best : 0.0f;
       s_bx = bb;
       s_cmax = fmaxf(s_cx, hi_c);
+      s_pc = s_po = s_cx;
+      s_lf = s_hf = 0.0f;
       s_row = 0;
     }
   }
@@ -480,20 +535,21 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
     // every row-term quotient x / lambda of a scenario has x = m C' with
     // 1 <= m <= 32767 and C' in {0} or [min(Cexcl, cap_lo), cmax]: in
     // Markstein's range unless a positive C' can fall below 2^-60
+    // (under the prior every C' lies in [cx, cmax])
     const bool fast = in_markstein_range(lam) && cmax <= 0x1p44f &&
-                      (cx >= 0x1p-60f || (cx == 0.0f && (lo_c >= 0x1p-60f || hi_c == 0.0f)));
+                      (cx >= 0x1p-60f || (!RF && cx == 0.0f && (lo_c >= 0x1p-60f || hi_c == 0.0f)));
     tab[H_TH_BASE] = b0 >= 0 ? sTh[b0] : 0.0f;
     // t* at row capacity Cexcl (no kappa entry is at or below it): the value of
     // every scenario of this candidate whose tail gate is closed
     tab[H_TCL] = tstar_of<2, FL>(cx, kap, thx, mnx, Lt ? P >> 1 : 0, lam, rl, dle);
     tab[H_L] = __int_as_float(Lt);
     tab[H_LPAD] = __int_as_float(Lpad);
-    tab[H_CX] = cx;
+    tab[H_CX] = s_pc;
     tab[H_BX] = __int_as_float(s_bx);
-    tab[H_CMAX] = cmax;
+    tab[H_PO] = s_po;
     tab[H_LAM] = lam;
-    tab[H_LO_C] = lo_c;
-    tab[H_HI_C] = hi_c;
+    tab[H_LF] = s_lf;
+    tab[H_HF] = s_hf;
     tab[H_LO_L] = lo_l;
     tab[H_HI_L] = hi_l;
     tab[H_SLO] = L;
@@ -627,13 +683,26 @@ struct PieceSum {
   uint64_t total;  // earlier values, flushed
 };
 
-template <bool TS, int ROW, bool FL>
+// Row r's capacity in a scenario under the monotone prior (see k_prep):
+// max(g ? max(P_open, c_y) : P_closed, min(max(c_y, F_lo), F_hi)).
+struct RowCap {
+  float pc, po, lf, hf;
+};
+
+__device__ __forceinline__ RowCap row_cap_of(const float* h) { return RowCap{h[H_CX], h[H_PO], h[H_LF], h[H_HF]}; }
+
+__device__ __forceinline__ float row_cap(const RowCap& r, float cy, bool g) {
+  return fmaxf(g ? fmaxf(r.po, cy) : r.pc, fminf(fmaxf(cy, r.lf), r.hf));
+}
+
+template <bool TS, int ROW, bool FL, bool RF>
 __device__ __forceinline__ PieceSum run_piece(const Plan& pl, const PhiloxKeys& keys, int o, int q_lo, int q_hi,
                                               const float* win, const float* h0, const float* h1,
                                               const float* kap0, const float* thx0, const float* mnx0,
                                               const float* kap1, const float* thx1, const float* mnx1) {
   const int st0 = __float_as_int(h0[H_STEP0]), st1 = __float_as_int(h1[H_STEP0]);
   const float cx0 = h0[H_CX], cx1 = h1[H_CX];
+  const RowCap rc0 = row_cap_of(h0), rc1 = row_cap_of(h1);
   const float lam = h0[H_LAM], rlam = h0[H_RLAM], dl = h0[H_DLT];
   const int cell = __float_as_int(h0[H_CELL]);
   const uint32_t ctr1 = (uint32_t)o, ctr2 = (uint32_t)cell, ctr3 = pl.round;
@@ -644,9 +713,12 @@ __device__ __forceinline__ PieceSum run_piece(const Plan& pl, const PhiloxKeys& 
   uint64_t total = 0;
   auto eval = [&](uint32_t word) {
     const float cy = sQo[__umulhi(word, W)];
-    const float cyg = (word & 0xFFFFu) < kgs ? cy : 0.0f;
-    const float t0 = tstar_of<ROW, FL>(fmaxf(cx0, cyg), kap0, thx0, mnx0, st0, lam, rlam, dl);
-    const float t1 = tstar_of<ROW, FL>(fmaxf(cx1, cyg), kap1, thx1, mnx1, st1, lam, rlam, dl);
+    const bool g = (word & 0xFFFFu) < kgs;
+    const float cyg = g ? cy : 0.0f;
+    const float c0 = RF ? row_cap(rc0, cy, g) : fmaxf(cx0, cyg);
+    const float c1 = RF ? row_cap(rc1, cy, g) : fmaxf(cx1, cyg);
+    const float t0 = tstar_of<ROW, FL>(c0, kap0, thx0, mnx0, st0, lam, rlam, dl);
+    const float t1 = tstar_of<ROW, FL>(c1, kap1, thx1, mnx1, st1, lam, rlam, dl);
     acc.add(__fsub_rn(t1, t0));
   };
   const int q_full = min(q_hi, pl.S >> 2);  // calls whose four samples all exist
@@ -682,13 +754,46 @@ __device__ __forceinline__ PieceSum run_piece(const Plan& pl, const PhiloxKeys& 
 // The same calls in dump mode: every scenario also writes its record (draws,
 // both t* and the per-class choices), with l_y mapped from the raw quantile
 // and the gate compared with the SLO directly.
-template <bool TS, bool FL>
+// Bin of row r's capacity in one scenario under the monotone prior (dump mode
+// only): the refit row's SLO-feasible bins in realisation sg, the largest
+// capacity, ties to the lower bin; -1 when none.
+__device__ int refit_bin(const Set& set, int p, int sg, int rr, int be, float cy, float ly, float L) {
+  const Dims& d = set.d;
+  const float* bp = set.bounds + (size_t)p * 4 * d.cells + (size_t)rr * d.B;
+  const float* cl = bp + (size_t)CAP_LO * d.cells;
+  const float* ch = bp + (size_t)CAP_HI * d.cells;
+  const float* tl = bp + (size_t)TAIL_LO * d.cells;
+  const float* th = bp + (size_t)TAIL_HI * d.cells;
+  float best = 0.0f;
+  int bb = -1;
+  for (int b = 0; b < d.B; ++b) {
+    float c, t;
+    if (b == be) {
+      c = cy;
+      t = ly;
+    } else if (b > be) {  // higher load: lower bounds rise to the draw
+      c = sg ? ch[b] : raise_lo(cl[b], ch[b], cy);
+      t = sg ? raise_lo(tl[b], th[b], ly) : th[b];
+    } else {              // lower load: upper bounds fall to the draw
+      c = sg ? lower_hi(cl[b], ch[b], cy) : cl[b];
+      t = sg ? tl[b] : lower_hi(tl[b], th[b], ly);
+    }
+    if (t <= L && (bb < 0 || c > best)) {
+      best = c;
+      bb = b;
+    }
+  }
+  return bb;
+}
+
+template <bool TS, bool FL, bool RF>
 __device__ uint64_t run_piece_dump(const Set& set, const Plan& pl, int item, int o, int q_lo, int q_hi,
                                    const float* win, const float* h0, const float* h1, const float* kap0,
                                    const float* thx0, const float* mnx0, const float* kap1, const float* thx1,
                                    const float* mnx1, unsigned char* dump, int dump_stride) {
   const int st0 = __float_as_int(h0[H_STEP0]), st1 = __float_as_int(h1[H_STEP0]);
   const float cx0 = h0[H_CX], cx1 = h1[H_CX];
+  const RowCap rc0 = row_cap_of(h0), rc1 = row_cap_of(h1);
   const float lam = h0[H_LAM], rlam = __frcp_rn(lam), dl = h0[H_DLT];
   const int cell = __float_as_int(h0[H_CELL]), p = __float_as_int(h0[H_P]);
   const PhiloxKeys keys = philox_keys(pl.key0, pl.key1 ^ (pl.stream_base + (uint32_t)p));
@@ -709,8 +814,8 @@ __device__ uint64_t run_piece_dump(const Set& set, const Plan& pl, int item, int
       const float cy = sQo[kc];
       const float ly = map_into(lo_l, __fsub_rn(hi_l, lo_l), hi_l, set.qn[(size_t)o * pl.W + kl]);
       const bool gate = ly <= h0[H_SLO];
-      const float C0 = gate ? fmaxf(cx0, cy) : cx0;
-      const float C1 = gate ? fmaxf(cx1, cy) : cx1;
+      const float C0 = RF ? row_cap(rc0, cy, gate) : gate ? fmaxf(cx0, cy) : cx0;
+      const float C1 = RF ? row_cap(rc1, cy, gate) : gate ? fmaxf(cx1, cy) : cx1;
       const float t0 = tstar_of<2, true>(C0, kap0, thx0, mnx0, st0, lam, rlam, dl);
       const float t1 = tstar_of<2, true>(C1, kap1, thx1, mnx1, st1, lam, rlam, dl);
       acc += fixed40(__fsub_rn(t1, t0));
@@ -727,7 +832,8 @@ __device__ uint64_t run_piece_dump(const Set& set, const Plan& pl, int item, int
         const float cx = sg ? cx1 : cx0;
         const int bx = __float_as_int(sg ? h1[H_BX] : h0[H_BX]);
         int bC;
-        if (!gate) bC = bx;
+        if (RF) bC = refit_bin(set, p, sg, rr, be, cy, ly, h0[H_SLO]);
+        else if (!gate) bC = bx;
         else if (bx < 0 || cy > cx) bC = be;
         else if (cy == cx) bC = min(be, bx);
         else bC = bx;
@@ -751,20 +857,29 @@ __device__ uint64_t run_piece_dump(const Set& set, const Plan& pl, int item, int
 // a scenario costs its share of the Philox call, one index and one
 // shared-memory load. Each entry holds the value's upper bits (>> 20) and
 // lower 20 bits, summed separately.
-template <bool TS, int ROW, bool FL>
+// RF: under the monotone prior the closed-gate values also depend on the
+// position (the draw refits the row's other bins): entries [W, 2W) hold them,
+// evaluated when `closed` (the open half when `open`).
+template <bool TS, int ROW, bool FL, bool RF>
 __device__ __forceinline__ void build_gtab(uint2* gtab, int W, const float* win, const float* h0, const float* h1,
                                            const float* kap0, const float* thx0, const float* mnx0,
-                                           const float* kap1, const float* thx1, const float* mnx1) {
+                                           const float* kap1, const float* thx1, const float* mnx1,
+                                           bool open = true, bool closed = false) {
   const int st0 = __float_as_int(h0[H_STEP0]), st1 = __float_as_int(h1[H_STEP0]);
   const float cx0 = h0[H_CX], cx1 = h1[H_CX];
+  const RowCap rc0 = row_cap_of(h0), rc1 = row_cap_of(h1);
   const float lam = h0[H_LAM], rlam = h0[H_RLAM], dl = h0[H_DLT];
   const float* capw = win + 4;
-  for (int k = threadIdx.x; k < W; k += blockDim.x) {
-    const float cy = capw[k];
-    const float t0 = tstar_of<ROW, FL>(fmaxf(cx0, cy), kap0, thx0, mnx0, st0, lam, rlam, dl);
-    const float t1 = tstar_of<ROW, FL>(fmaxf(cx1, cy), kap1, thx1, mnx1, st1, lam, rlam, dl);
-    const uint64_t g = fixed40(__fsub_rn(t1, t0));
-    gtab[k] = make_uint2((uint32_t)(g >> 20), (uint32_t)g & 0xFFFFFu);
+  const int k0 = (RF && !open) ? W : 0, k1 = (RF && closed) ? 2 * W : W;
+  for (int k = k0 + (int)threadIdx.x; k < k1; k += blockDim.x) {
+    const bool g = k < W;
+    const float cy = capw[g ? k : k - W];
+    const float c0 = RF ? row_cap(rc0, cy, g) : fmaxf(cx0, cy);
+    const float c1 = RF ? row_cap(rc1, cy, g) : fmaxf(cx1, cy);
+    const float t0 = tstar_of<ROW, FL>(c0, kap0, thx0, mnx0, st0, lam, rlam, dl);
+    const float t1 = tstar_of<ROW, FL>(c1, kap1, thx1, mnx1, st1, lam, rlam, dl);
+    const uint64_t gv = fixed40(__fsub_rn(t1, t0));
+    gtab[k] = make_uint2((uint32_t)(gv >> 20), (uint32_t)gv & 0xFFFFFu);
   }
 }
 
@@ -790,7 +905,7 @@ __device__ __forceinline__ uint4 draw_call(const Plan& pl, const PhiloxKeys& key
   else return philox4x32_10(make_uint4(q, ctr1, ctr2, ctr3), keys);
 }
 
-template <bool KC>
+template <bool KC, bool RF>
 __device__ __forceinline__ GtabSum sample_gtab(const Plan& pl, const PhiloxKeys& keys, int o, int cell, int q_lo,
                                                int q_hi, uint32_t gtab_s, uint32_t kgs16) {
   const uint32_t ctr1 = (uint32_t)o, ctr2 = (uint32_t)cell, ctr3 = pl.round;
@@ -799,7 +914,7 @@ __device__ __forceinline__ GtabSum sample_gtab(const Plan& pl, const PhiloxKeys&
   uint32_t gh = 0, glo = 0;
   auto take = [&](uint32_t word) {
     const uint32_t cap = __umulhi(word, W);
-    const uint32_t idx = word * mul < kgs16 ? cap : W;
+    const uint32_t idx = word * mul < kgs16 ? cap : (RF ? cap + W : W);
     uint32_t a, b;
     asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(a), "=r"(b) : "r"(gtab_s + idx * eb));
     gh += a;
@@ -885,7 +1000,7 @@ __device__ __forceinline__ void stage_segment(const Set& set, const Plan& pl, co
 // GT: the table path (build_gtab), chosen by the host when a chunk's samples
 // outnumber a segment's W + 1 table entries; never with DUMP. KC (table path,
 // one problem): Philox round keys from the plan's parameters.
-template <bool DUMP, bool FL, bool GT, bool KC>
+template <bool DUMP, bool FL, bool GT, bool KC, bool RF>
 __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, Plan pl, const float* rec,
                                                          uint64_t* sums, unsigned char* dump, int dump_stride,
                                                          ScoreGrid sg) {
@@ -893,8 +1008,9 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
   uint64_t* bar = reinterpret_cast<uint64_t*>(smraw);  // [2]
   float* stage0 = reinterpret_cast<float*>(smraw + 16);
   const int stage_floats = pl.Wp + 2 * sg.tcopy;
-  // GT: two tables of W + 1 entries, used by alternate chunks
+  // GT: two tables of W + 1 entries (2W under the prior), used by alternate chunks
   uint2* gtab2 = reinterpret_cast<uint2*>(smraw + 16 + (size_t)2 * stage_floats * 4);
+  const int gt_len = RF ? 2 * pl.W : pl.W + 1;
   // per stage: chunk index, its segment and its part (thread 0 divides once)
   __shared__ int s_chunk[2], s_seg[2], s_part[2];
   const Dims& d = set.d;  // kernel-parameter space: no local copy
@@ -962,7 +1078,7 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
       // the gate position) come before it, so thread 0 may refill the stage
       // next iteration, and the next chunk builds the other table while a late
       // thread may still draw from this one.
-      uint2* gtab = gtab2 + (size_t)(j & 1) * (pl.W + 1);
+      uint2* gtab = gtab2 + (size_t)(j & 1) * gt_len;
       const int cell = ok ? __float_as_int(h0[H_CELL]) : -1;
       const bool use = cell >= 0 && cell < d.cells;  // a bad device-side id was flagged by k_prep
       // passing tail positions of the stratum, as the top bits of a 16-bit field
@@ -971,23 +1087,27 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
       if (use) {
         const uint64_t gc = fixed40(__fsub_rn(h1[H_TCL], h0[H_TCL]));
         const uint2 closed = make_uint2((uint32_t)(gc >> 20), (uint32_t)gc & 0xFFFFFu);
-        if (kgs == 0u) {
+        // under the prior: the halves the stratum's gate positions can reach
+        const bool any_open = kgs != 0u, any_closed = kgs16 != 0xFFFFFFFFu;
+        if (!RF && kgs == 0u) {
           // the gate is closed at every position of the stratum: every entry
           // is the closed-gate value (each scenario still draws its position)
           for (int k = tid; k <= pl.W; k += blockDim.x) gtab[k] = closed;
         } else {
           if (tid == 0) {
-            gtab[pl.W] = closed;
+            if (!RF) gtab[pl.W] = closed;
             // entries evaluated, once per segment (later chunks of a segment
             // rebuild the same table): the measurement's algorithmic count
-            if (KC && part == 0) atomicAdd(&set.work[2], (unsigned long long)pl.W);
+            const int halves = RF ? (any_open ? 1 : 0) + (any_closed ? 1 : 0) : 1;
+            if (KC && part == 0) atomicAdd(&set.work[2], (unsigned long long)pl.W * halves);
           }
           const int Lp0 = __float_as_int(h0[H_LPAD]), Lp1 = __float_as_int(h1[H_LPAD]);
           const bool r0 = __float_as_int(h0[H_ROW]) != 0, r1 = __float_as_int(h1[H_ROW]) != 0;
           const bool f0 = __float_as_int(h0[H_FAST]) != 0, f1 = __float_as_int(h1[H_FAST]) != 0;
           const int row = (!r0 && !r1) ? 0 : ((!r0 || f0) && (!r1 || f1)) ? 1 : 2;
-#define FS_BUILD(TSV, ROWV, FLV) \
-  build_gtab<TSV, ROWV, FLV>(gtab, pl.W, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, k1 + Lp1, k1 + 2 * Lp1)
+#define FS_BUILD(TSV, ROWV, FLV)                                                                            \
+  build_gtab<TSV, ROWV, FLV, RF>(gtab, pl.W, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, k1 + Lp1, k1 + 2 * Lp1, \
+                                 any_open, any_closed)
 #define FS_BUILDS(TSV)                       \
   if (row == 0) FS_BUILD(TSV, 0, false);     \
   else if (row == 1) FS_BUILD(TSV, 1, FL);   \
@@ -1019,7 +1139,7 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
         return;
       }
       GtabSum gs{0u, 0u, 0ull};
-      if (use) gs = sample_gtab<KC>(pl, keys, o, cell, q_lo, q_hi, smem_u32(gtab), kgs16);
+      if (use) gs = sample_gtab<KC, RF>(pl, keys, o, cell, q_lo, q_hi, smem_u32(gtab), kgs16);
       uint64_t v;
       if (small_gt) {  // at most 64 values per thread: each field's warp sum fits in 32 bits
         const uint32_t H = __reduce_add_sync(0xffffffffu, gs.h);
@@ -1047,14 +1167,14 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
           keys_p = p;
         }
         // the table pointers stay in one address space per branch (shared or global)
-#define FS_PIECE(TSV, ROWV, FLV)                                                                  \
-  run_piece<TSV, ROWV, FLV>(pl, keys, o, q_lo, q_hi, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, k1 + Lp1, \
-                            k1 + 2 * Lp1)
+#define FS_PIECE(TSV, ROWV, FLV)                                                                      \
+  run_piece<TSV, ROWV, FLV, RF>(pl, keys, o, q_lo, q_hi, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, k1 + Lp1, \
+                                k1 + 2 * Lp1)
 #define FS_PIECES(TSV) \
   (row == 0 ? FS_PIECE(TSV, 0, false) : row == 1 ? FS_PIECE(TSV, 1, FL) : FS_PIECE(TSV, 2, FL))
-#define FS_DUMP(TSV)                                                                                   \
-  run_piece_dump<TSV, FL>(set, pl, item, o, q_lo, q_hi, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, k1 + Lp1, \
-                      k1 + 2 * Lp1, dump, dump_stride)
+#define FS_DUMP(TSV)                                                                                       \
+  run_piece_dump<TSV, FL, RF>(set, pl, item, o, q_lo, q_hi, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, k1 + Lp1, \
+                              k1 + 2 * Lp1, dump, dump_stride)
         if (Lp0 <= sg.lcap_s && Lp1 <= sg.lcap_s) {
           const float* k0 = h0 + kTableHeader;
           const float* k1 = h1 + kTableHeader;
@@ -1150,12 +1270,13 @@ cudaError_t launch_prep(const Set& set, const Items& it, const Plan& pl, float* 
                         bool early, LaunchCache& lc, cudaStream_t s) {
   if (it.n <= 0) return cudaSuccess;
   const size_t smem = prep_smem_bytes(set);
-  const int fl = lc.floors ? 1 : 0;
-  auto kern = fl ? k_prep<true> : k_prep<false>;
-  if (smem > lc.prep_smem[fl]) {
+  const int fl = lc.floors ? 1 : 0, mode = fl + (set.prior == 1 ? 2 : 0);
+  auto kern = mode == 0 ? k_prep<false, false> : mode == 1 ? k_prep<true, false>
+            : mode == 2 ? k_prep<false, true> : k_prep<true, true>;
+  if (smem > lc.prep_smem[mode]) {
     cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(kern), smem);
     if (e != cudaSuccess) return e;
-    lc.prep_smem[fl] = smem;
+    lc.prep_smem[mode] = smem;
   }
   return launch_pdl(kern, dim3(it.n * 2), dim3(kPrepThreads), smem, s, set, it, pl, tables, sums, early ? 1 : 0);
 }
@@ -1173,22 +1294,27 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
   // about a third of one there); the smallest chunk holds 2 calls per thread
   const long long chunk_min = std::min<long long>(pl.S, 2LL * 4 * kScoreThreads);
   const bool table = !dump && pl.W <= 4096 && 3LL * (pl.W + 1) <= 2 * chunk_min;
+  const bool rf = set.prior == 1;
   const size_t stages = 16 + 2 * (size_t)(pl.Wp + 2 * sg.tcopy) * 4;
-  const size_t smem = stages + (table ? ((size_t)16 * (pl.W + 1) + 15) / 16 * 16 : 0);
+  const size_t gt_len = rf ? 2 * (size_t)pl.W : (size_t)pl.W + 1;
+  const size_t smem = stages + (table ? (2 * 8 * gt_len + 15) / 16 * 16 : 0);
   const int v = dump ? SCORE_DUMP : table ? (it.p == nullptr ? SCORE_TABLE : SCORE_TABLE_MULTI) : SCORE_PLAIN;
-  const int fl = lc.floors ? 1 : 0;
+  const int fl = lc.floors ? 1 : 0, mode = fl + (rf ? 2 : 0);
   const bool one = it.p == nullptr;  // every item belongs to problem 0
-  auto kern = dump ? (fl ? k_score<true, true, false, false> : k_score<true, false, false, false>)
-          : table ? (one ? (fl ? k_score<false, true, true, true> : k_score<false, false, true, true>)
-                         : (fl ? k_score<false, true, true, false> : k_score<false, false, true, false>))
-                  : (fl ? k_score<false, true, false, false> : k_score<false, false, false, false>);
-  if (smem != lc.score_smem[v][fl]) {
+#define FS_KERN(F, R)                                                                              \
+  (dump ? k_score<true, F, false, false, R>                                                         \
+        : table ? (one ? k_score<false, F, true, true, R> : k_score<false, F, true, false, R>)      \
+                : k_score<false, F, false, false, R>)
+  auto kern = mode == 0 ? FS_KERN(false, false) : mode == 1 ? FS_KERN(true, false)
+            : mode == 2 ? FS_KERN(false, true) : FS_KERN(true, true);
+#undef FS_KERN
+  if (smem != lc.score_smem[v][mode]) {
     int per_sm = 0;
     cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(kern), smem);
     if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kScoreThreads, smem);
     if (e != cudaSuccess) return e;
-    lc.score_smem[v][fl] = smem;
-    lc.score_blocks_per_sm[v][fl] = per_sm < 1 ? 1 : per_sm;
+    lc.score_smem[v][mode] = smem;
+    lc.score_blocks_per_sm[v][mode] = per_sm < 1 ? 1 : per_sm;
   }
   // Chunks of U calls per thread: about eight chunks per resident block when
   // the work allows, so that the counter can even out the segments' unequal
@@ -1196,7 +1322,7 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
   // thread, measured faster on small launches) and at most 8 calls per
   // thread (16 on the table path, whose chunks also build a table), and no
   // more than a segment holds.
-  const long long resident = (long long)lc.score_blocks_per_sm[v][fl] * sm_count;
+  const long long resident = (long long)lc.score_blocks_per_sm[v][mode] * sm_count;
   const long long total_calls = (long long)it.n * pl.O * pl.calls;
   long long U = total_calls / ((long long)kScoreThreads * resident * 8);
   const long long u_seg = ((long long)pl.calls + kScoreThreads - 1) / kScoreThreads;

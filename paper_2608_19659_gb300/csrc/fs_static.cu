@@ -166,6 +166,7 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
   set.work = reinterpret_cast<unsigned long long*>(base + o_work);
   set.skip = nullptr;
   set.rtab = reinterpret_cast<int*>(base + o_rtab);
+  set.prior = 0;  // the revealed-only prior: no cell is measured here
 
   Items it{};
   it.n = n;
@@ -208,8 +209,8 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
     // keep the larger of what this call and any concurrent one found
     std::lock_guard<std::mutex> lock(g_static_mu);
     LaunchCache& g = g_static_lc[dev];
-    for (int f = 0; f < 2; ++f) {
-      g.solve_smem[f] = std::max(g.solve_smem[f], lc.solve_smem[f]);
+    for (int f = 0; f < 2; ++f) g.solve_smem[f] = std::max(g.solve_smem[f], lc.solve_smem[f]);
+    for (int f = 0; f < 4; ++f) {
       g.prep_smem[f] = std::max(g.prep_smem[f], lc.prep_smem[f]);
       for (int v = 0; v < kScoreVariants; ++v)
         if (lc.score_smem[v][f] && lc.score_smem[v][f] != g.score_smem[v][f]) {

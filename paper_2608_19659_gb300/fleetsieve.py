@@ -23,7 +23,7 @@ FS_OK, FS_EINVAL, FS_ENOMEM, FS_ECUDA, FS_ETIMEOUT, FS_EDEVICE = 0, -1, -2, -3, 
 FS_MAX_CLASSES = 64
 EXPORTS = ("fs_load_model", "fs_update_bounds", "fs_set_floors", "fs_dump_stride", "fs_score_candidates",
            "fs_score_candidates_async", "fs_solve", "fs_solve_batch", "fs_solve_bounds",
-           "fs_reveal", "fs_get_state", "fs_certificate", "fs_replay", "fs_check", "fs_launch_count",
+           "fs_reveal", "fs_set_prior", "fs_get_state", "fs_certificate", "fs_replay", "fs_check", "fs_launch_count",
            "fs_watchdog_selftest", "fs_free_model", "fs_last_error", "fs_score_candidates_noalloc",
            "fs_timing_enable",
            "fs_timing_read")
@@ -99,6 +99,7 @@ def lib():
         L.fs_solve_bounds.argtypes = [C.c_void_p, C.POINTER(fs_allocation),
                                       C.POINTER(fs_allocation), fp]
         L.fs_reveal.argtypes = [C.c_void_p, C.c_int32, C.c_float, C.c_float]
+        L.fs_set_prior.argtypes = [C.c_void_p, C.c_int32]
         L.fs_get_state.argtypes = [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
                                    C.c_void_p]
         L.fs_certificate.argtypes = [C.c_void_p, C.c_float, C.POINTER(C.c_int32), fp]
@@ -322,6 +323,15 @@ def fs_solve_bounds(m: Model):
 
 def fs_reveal(m: Model, cell: int, cap: float, tail: float) -> None:
     _check(lib().fs_reveal(m.handle, int(cell), float(cap), float(tail)))
+
+
+FS_PRIOR_REVEALED, FS_PRIOR_MONOTONE = 0, 1
+
+
+def fs_set_prior(m: Model, prior: int) -> None:
+    """How a measurement refits the intervals: FS_PRIOR_REVEALED (the measured
+    cell only) or FS_PRIOR_MONOTONE (also its row, nondecreasing in load)."""
+    _check(lib().fs_set_prior(m.handle, int(prior)))
 
 
 def fs_get_state(m: Model):

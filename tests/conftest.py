@@ -58,6 +58,8 @@ def load_model(fsb, w, quantile=None):
                           quantile=quantile)
     if getattr(w, "floor", None) is not None:
         fsb.fs_set_floors(m, w.floor)
+    if getattr(w, "prior", 0):
+        fsb.fs_set_prior(m, w.prior)
     return m
 
 
