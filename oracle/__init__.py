@@ -86,6 +86,21 @@ def lib():
         _lib.or_score_cached.argtypes = [C.POINTER(_Problem), fp, fp, fp, fp, fp, C.c_int,
                                          C.c_uint64, C.c_uint32, C.c_uint32, C.c_int, ip, C.c_int,
                                          C.c_int, C.c_int, C.POINTER(C.c_int64), fp]
+        i64p = C.POINTER(C.c_int64)
+        _lib.or_goodput_fx.argtypes = [C.c_int, C.c_float, C.c_float]
+        _lib.or_goodput_fx.restype = C.c_int64
+        _lib.or_solve_lex.argtypes = [C.POINTER(_Problem), fp, fp, C.c_int, C.POINTER(_Alloc), i64p]
+        _lib.or_base_gap_lex.argtypes = [C.POINTER(_Problem), fp, fp, fp, fp, C.c_int,
+                                         C.POINTER(_Alloc), C.POINTER(_Alloc), i64p, i64p, fp,
+                                         C.POINTER(C.c_double)]
+        _lib.or_certificate_lex.argtypes = [C.POINTER(_Problem), fp, fp, fp, fp,
+                                            C.POINTER(C.c_uint8), C.c_float, C.c_int,
+                                            C.POINTER(C.c_int), fp, C.POINTER(C.c_double)]
+        _lib.or_score_goodput.argtypes = [C.POINTER(_Problem), fp, fp, fp, fp, fp, C.c_int,
+                                          C.c_uint64, C.c_uint32, C.c_uint32, C.c_int, ip, C.c_int,
+                                          C.c_int, C.c_int, i64p, C.POINTER(C.c_double),
+                                          C.POINTER(C.c_double), i64p, i64p,
+                                          C.POINTER(C.c_double), ip]
         _lib.or_refit.argtypes = [C.POINTER(_Problem), C.c_int, C.c_int32, C.c_float, C.c_float,
                                   fp, fp, fp, fp]
         _lib.or_reduce.argtypes = [C.POINTER(_Problem), C.c_int, ip, C.c_int, C.c_int, C.c_float,
@@ -325,6 +340,93 @@ def refit(prob: Problem, cell, c, l, cap_lo, cap_hi, tail_lo, tail_hi, prior=Non
     if rc:
         raise ValueError("oracle refit failed")
     return arrs
+
+
+def goodput_fx(n, c, lam) -> int:
+    return int(lib().or_goodput_fx(int(n), float(c), float(lam)))
+
+
+def solve_lex(prob: Problem, cap, tail, solver: int = SOLVER_FRONTIER):
+    """Tiers 1-4 of the lexicographic objective: (Allocation, goodput in 2^-20 req/s)."""
+    cap = _f32(cap)
+    tail = _f32(tail)
+    a = _Alloc()
+    g = C.c_int64()
+    rc = lib().or_solve_lex(C.byref(prob._s), _ptr(cap, C.c_float), _ptr(tail, C.c_float), solver,
+                            C.byref(a), C.byref(g))
+    if rc:
+        raise ValueError(f"oracle lexicographic solve failed ({rc})")
+    return Allocation.of(a, prob.K), int(g.value)
+
+
+def base_gap_lex(prob: Problem, cap_lo, cap_hi, tail_lo, tail_hi, solver=SOLVER_FRONTIER):
+    """(A-, A+, GP-, GP+, max-min gap, goodput gap) with both solved to tier 4."""
+    arrs = [_f32(x) for x in (cap_lo, cap_hi, tail_lo, tail_hi)]
+    am, ap = _Alloc(), _Alloc()
+    gm, gp = C.c_int64(), C.c_int64()
+    gmm = C.c_float()
+    ggp = C.c_double()
+    rc = lib().or_base_gap_lex(C.byref(prob._s), *[_ptr(x, C.c_float) for x in arrs], solver,
+                               C.byref(am), C.byref(ap), C.byref(gm), C.byref(gp), C.byref(gmm),
+                               C.byref(ggp))
+    if rc:
+        raise ValueError("oracle lexicographic base gap failed")
+    return (Allocation.of(am, prob.K), Allocation.of(ap, prob.K), int(gm.value), int(gp.value),
+            float(np.float32(gmm.value)), float(ggp.value))
+
+
+def certificate_lex(prob: Problem, cap_lo, cap_hi, tail_lo, tail_hi, revealed, eps,
+                    solver=SOLVER_FRONTIER):
+    arrs = [_f32(x) for x in (cap_lo, cap_hi, tail_lo, tail_hi)]
+    rev = np.ascontiguousarray(revealed, np.uint8).reshape(-1)
+    st = C.c_int()
+    gmm = C.c_float()
+    ggp = C.c_double()
+    rc = lib().or_certificate_lex(C.byref(prob._s), *[_ptr(x, C.c_float) for x in arrs],
+                                  _ptr(rev, C.c_uint8), eps, solver, C.byref(st), C.byref(gmm),
+                                  C.byref(ggp))
+    if rc:
+        raise ValueError("oracle lexicographic certificate failed")
+    return int(st.value), float(np.float32(gmm.value)), float(ggp.value)
+
+
+@dataclasses.dataclass
+class GoodputScore:
+    sum_eo: np.ndarray  # [n_cand, O] int64, sums of |GP+' - GP-'| in 2^-20 req/s
+    gap: np.ndarray  # [n_cand] E[Gamma_gp,t+1 | e] (fraction of total demand)
+    score: np.ndarray
+    score_fixed: np.ndarray
+    gamma_fx: int  # |GP+ - GP-| at the bounds, 2^-20 req/s
+    gamma_gp: float
+    best: int
+
+
+def score_goodput(w, qn, candidates=None, solver=SOLVER_FRONTIER, seed=None, stream_id=None,
+                  rnd=None, O=None, S=None) -> GoodputScore:
+    prob = Problem.of(w)
+    b = _bounds(w)
+    qn = _f32(qn)
+    cand = np.ascontiguousarray(w.candidates if candidates is None else candidates, np.int32)
+    O = w.O if O is None else O
+    S = w.S if S is None else S
+    n = cand.size
+    sum_eo = np.zeros((n, O), np.int64)
+    gap = np.zeros(n, np.float64)
+    sc = np.zeros(n, np.float64)
+    scf = np.zeros(n, np.int64)
+    gfx = C.c_int64()
+    ggp = C.c_double()
+    best = C.c_int32()
+    rc = lib().or_score_goodput(C.byref(prob._s), *[_ptr(x, C.c_float) for x in b],
+                                _ptr(qn, C.c_float), qn.size,
+                                w.seed if seed is None else seed,
+                                w.stream_id if stream_id is None else stream_id,
+                                w.round if rnd is None else rnd, n, _ptr(cand, C.c_int32), O, S, solver,
+                                _ptr(sum_eo, C.c_int64), _ptr(gap, C.c_double), _ptr(sc, C.c_double),
+                                _ptr(scf, C.c_int64), C.byref(gfx), C.byref(ggp), C.byref(best))
+    if rc:
+        raise ValueError(f"oracle goodput score failed ({rc})")
+    return GoodputScore(sum_eo, gap, sc, scf, int(gfx.value), float(ggp.value), int(best.value))
 
 
 def certificate(prob: Problem, cap_lo, cap_hi, tail_lo, tail_hi, revealed, eps,

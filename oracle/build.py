@@ -12,7 +12,7 @@ import subprocess
 import sys
 
 HERE = os.path.dirname(os.path.abspath(__file__))
-SOURCES = ["sampler.c", "allocation.c", "decision_gap.c", "prior.c"]
+SOURCES = ["sampler.c", "allocation.c", "decision_gap.c", "prior.c", "lexicographic.c"]
 LIB = os.path.join(HERE, "liboracle.so")
 CFLAGS = ["-O2", "-std=c11", "-ffp-contract=off", "-fno-fast-math", "-fexcess-precision=standard",
           "-fPIC", "-shared", "-Wall", "-Wextra", "-Wno-unused-parameter"]

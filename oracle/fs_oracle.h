@@ -124,6 +124,29 @@ int or_reduce(const or_problem *p, int n_cand, const int32_t *cand, int O, int S
 int or_refit(const or_problem *p, int prior, int32_t cell, float c, float l,
              float *cap_lo, float *cap_hi, float *tail_lo, float *tail_hi);
 
+/* Tiers 3-4 of the lexicographic objective (lexicographic.c): the allocation
+ * keeping tiers 1-2 optimal with the most goodput, then the fewest GPUs, then
+ * the tie rules class by class; *goodput_fx = its goodput in 2^-20 req/s. */
+int64_t or_goodput_fx(int n, float c, float lam);
+int or_solve_lex(const or_problem *p, const float *cap, const float *tail, int solver,
+                 or_alloc *out, int64_t *goodput_fx);
+/* A-, A+ to tier 4; the max-min gap and the goodput gap |GP+ - GP-| / sum lambda. */
+int or_base_gap_lex(const or_problem *p, const float *cap_lo, const float *cap_hi,
+                    const float *tail_lo, const float *tail_hi, int solver,
+                    or_alloc *minus, or_alloc *plus, int64_t *gp_minus, int64_t *gp_plus,
+                    float *gamma_mm, double *gamma_gp);
+/* Stage-wise certificate: both gaps at most eps. */
+int or_certificate_lex(const or_problem *p, const float *cap_lo, const float *cap_hi,
+                       const float *tail_lo, const float *tail_hi, const uint8_t *revealed,
+                       float eps, int solver, int *state, float *gamma_mm, double *gamma_gp);
+/* The goodput stage of the Monte-Carlo score (sums in 2^-20 req/s). */
+int or_score_goodput(const or_problem *p, const float *cap_lo, const float *cap_hi,
+                     const float *tail_lo, const float *tail_hi, const float *qn, int Q,
+                     uint64_t seed, uint32_t stream_id, uint32_t round,
+                     int n_cand, const int32_t *cand, int O, int S, int solver,
+                     int64_t *sum_eo, double *gap, double *score, int64_t *score_fixed,
+                     int64_t *gamma_fx, double *gamma_gp, int32_t *best);
+
 /* Certificate (Section 4.2): 0 undecided, 1 certified feasible, 2 certified
  * infeasible (even A+ misses a critical floor). */
 int or_certificate(const or_problem *p, const float *cap_lo, const float *cap_hi,

@@ -85,3 +85,46 @@ def choice_at(K, B, G, cap, tail, demand, slo, t, floor=None):
             continue
         res.append(min(cov, key=lambda x: (x[0], x[1], x[2], -x[3], x[4])))
     return res
+
+
+def goodput_fx(n, c, lam):
+    """rint(min(lambda, n c) 2^20): a class's served goodput (Eqs. 2, 4) in 2^-20 req/s."""
+    served = np.float32(n) * np.float32(c)
+    x = served if served < np.float32(lam) else np.float32(lam)
+    return int(np.rint(np.float64(x) * 2.0**20))
+
+
+def lexicographic(K, B, G, cap, tail, demand, slo, floor=None):
+    """The four tiers of Section 3 by enumeration: among allocations within G,
+    those meeting the critical floors when any does (else nothing is
+    allocated), then the largest min_i r_i, then the most goodput, then the
+    fewest GPUs, then class by class the option preferred by the tie rules
+    (none first, then lower TP, fewer replicas, larger capacity, lower bin).
+    Returns (t*, goodput_fx, gpus, per-class (tp, n, bin))."""
+    opts = options(K, B, G, cap, tail, demand, slo)
+    combos = [c for c in itertools.product(*[[None] + o for o in opts])
+              if sum(x[0] for x in c if x is not None) <= G]
+    empty = (0.0, 0, 0, [(0, 0, -1)] * K)
+    if floor is not None and any(d > 0 for d in floor):
+        combos = [c for c in combos if _floor_ok(c, floor)]
+        if not combos:
+            return empty
+
+    def minr(c):
+        return 0.0 if any(x is None for x in c) else min(x[5] for x in c)
+
+    t = max(minr(c) for c in combos)
+    pool = [c for c in combos if minr(c) == t]
+
+    def gp(c):
+        return sum(goodput_fx(x[2], x[3], demand[i]) for i, x in enumerate(c) if x is not None)
+
+    def gpus(c):
+        return sum(x[0] for x in c if x is not None)
+
+    def tie(c):
+        return tuple((-1,) if x is None else (x[1], x[2], -x[3], x[4]) for x in c)
+
+    best = min(pool, key=lambda c: (-gp(c), gpus(c), tie(c)))
+    choice = [(0, 0, -1) if x is None else (TP[x[1]], x[2], x[4]) for x in best]
+    return float(t), gp(best), gpus(best), choice
