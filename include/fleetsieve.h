@@ -218,11 +218,11 @@ int fs_score_candidates_async(fs_model *m, const fs_samples *samples, double *ga
  * process exits. A call takes the following pieces of it, each rounded up to
  * a multiple of 256 bytes, and returns FS_EINVAL without running when their
  * sum exceeds 16 MiB:
- *   4, 16 and 1024 bytes (status word, counters, reduction scratch);
+ *   4, 24 and 1024 bytes (status word, counters, reduction scratch);
  *   4 Q (only with quantile_dev NULL: the built-in table);
  *   8 T and 8, with T = K (floor(G/1) + floor(G/2) + floor(G/4) + floor(G/8))
  *     (thresholds and their counts);
- *   32 K twice (best capacity and bin per (class, TP) row), 1200 (the two
+ *   32 K twice (best capacity and bin per (class, TP) row), 1216 (the two
  *     base allocations), 65536 (their row tables);
  *   4 n I with n = max(n_cand, 1), I = 2 (20 + 3 P) + O (4 + 4 ceil(W / 4)),
  *     P the smallest power of two >= max(T + 1, 4), W = Q / O (the
@@ -262,6 +262,8 @@ typedef struct {
     int16_t bin[FS_MAX_CLASSES];
     int16_t replicas[FS_MAX_CLASSES];
     float fulfil[FS_MAX_CLASSES];
+    double goodput;           /* served req/s sum_i min(lambda_i, n c) in steps of 2^-20
+                                 (tier 3); filled under the lexicographic objective, else 0 */
 } fs_allocation;
 
 /*
@@ -318,6 +320,50 @@ int fs_reveal(fs_model *m, int32_t cell, float cap, float tail);
 #define FS_PRIOR_REVEALED 0
 #define FS_PRIOR_MONOTONE 1
 int fs_set_prior(fs_model *m, int32_t prior);
+
+/*
+ * fs_set_objective -- which tiers of Section 3's lexicographic objective the
+ * solves of this model optimise.
+ *   FS_OBJECTIVE_MAXMIN (0, the state a new model starts in): tiers 1-2
+ *     (floors, then max min_i r_i by the threshold rule); the allocation is
+ *     each class's cheapest cover at t*; fs_allocation.goodput is 0.
+ *   FS_OBJECTIVE_LEXICOGRAPHIC (1): all four tiers. Among the allocations
+ *     that keep tiers 1-2 optimal (every class at r_i >= max(t*, delta_i) when
+ *     t* > 0; at t* = 0 the critical classes at their floors and the others
+ *     free; nothing when the floors cannot be met): (3) the most served
+ *     goodput sum_i min(lambda_i, n c), each class's term rounded to 2^-20
+ *     req/s; (4) "minimise fragmentation" read as the fewest GPUs in use,
+ *     then class by class the tie rules (no replicas, lower TP, fewer
+ *     replicas, larger capacity, lower bin). fs_solve, fs_solve_batch and
+ *     fs_solve_bounds return that allocation with its goodput, and
+ *     fs_certificate becomes stage-wise (Section 4.2): certified feasible
+ *     also needs the goodput gap |GP(A+) - GP(A-)| / sum_i lambda_i <= eps.
+ *     Needs (K + 1)(G + 1) <= 4 Mi (FS_EINVAL otherwise). The scoring calls
+ *     and fs_replay stay on the max-min stage; fs_score_goodput scores the
+ *     goodput stage.
+ */
+#define FS_OBJECTIVE_MAXMIN 0
+#define FS_OBJECTIVE_LEXICOGRAPHIC 1
+int fs_set_objective(fs_model *m, int32_t objective);
+
+/*
+ * fs_score_goodput -- the goodput stage of Section 4.3's score (the second
+ * curve of Fig. 4a): for every candidate e, outcome o and sample s the same
+ * draw and realisations as fs_score_candidates (the model's prior and floors
+ * included), both solved to tier 4, and the scenario's goodput gap
+ * |GP(A+') - GP(A-')| summed in int64 units of 2^-20 req/s. Host outputs
+ * (each nullable):
+ *   gap_out[n_cand]   E[Gamma_gp,t+1 | e] = sum 2^-20 / (O S) / sum_i lambda_i
+ *   score_out[n_cand] (Gamma_gp,t O S - sum) 2^-20 / (O S) / sum_i lambda_i
+ *                     (Gamma_gp,t = |GP(A+) - GP(A-)| at the bounds, 2^-20 req/s)
+ *   gamma_gp[1]       Gamma_gp,t / sum_i lambda_i
+ *   best[1]           argmax: largest score, then lower TP, then earlier in cand
+ *   sum_eo[n_cand*O]  the int64 sums
+ * Needs sum_i lambda_i <= 2^20 req/s, G <= 1024 and (K + 1)(G + 1) <= 4 Mi
+ * (FS_EINVAL otherwise). Synchronous. Independent of fs_set_objective.
+ */
+int fs_score_goodput(fs_model *m, const fs_samples *samples, double *gap_out, double *score_out,
+                     double *gamma_gp, int32_t *best, int64_t *sum_eo);
 
 /*
  * fs_get_state -- the model's current uncertainty state, for checkpointing

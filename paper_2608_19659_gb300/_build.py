@@ -19,8 +19,8 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libfleetsieve.so")
-SOURCES = ["fs_api.cu", "fs_solve.cu", "fs_score.cu", "fs_replay.cu", "fs_static.cu"]
-HEADERS = ["fs_internal.cuh", "fs_finalize.cuh"]
+SOURCES = ["fs_api.cu", "fs_solve.cu", "fs_score.cu", "fs_replay.cu", "fs_static.cu", "fs_lex.cu"]
+HEADERS = ["fs_internal.cuh", "fs_finalize.cuh", "fs_sample.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-fmad=false", "-Xcompiler", "-fPIC,-O2,-ffp-contract=off",
               "-I", os.path.join(ROOT, "include")]

@@ -146,7 +146,8 @@ struct fs_model {
   Buf fixed;      // lam, slo + floors, qn, bounds, revealed, theta, ntheta, rowC, rowB, base, status
   Set set{};
   // per-call scratch
-  Buf cand, tables, sums, outs, real;
+  Buf cand, tables, sums, outs, real, lex;
+  int objective = FS_OBJECTIVE_MAXMIN;  // FS_OBJECTIVE_LEXICOGRAPHIC: fs_solve* and the certificate to tier 4
   // host mirrors
   std::vector<float> h_bounds;      // [4][cells]
   std::vector<uint8_t> h_revealed;  // [cells]
@@ -347,6 +348,25 @@ int run_score(fs_model* m, const Set& set, const fs_samples* smp, const int32_t*
           "launch finalize");
   if (phases) FS_CUDA(cudaEventRecord(ev[4], s), "record timing event");
   return FS_OK;
+}
+
+// Tiers 3-4 (fs_lex.cu) of n realisations whose tier-2 allocations are in out
+// (or the base), when the model's objective asks for them.
+int solve_lex_pass(fs_model* m, const Set& set, int n, const float* cap_x, const float* tail_x, fs_allocation* out,
+                   cudaStream_t s) {
+  if (m->objective != FS_OBJECTIVE_LEXICOGRAPHIC || n <= 0) return FS_OK;
+  const size_t per_real = lex_scratch_cells(m->d) * kLexCellBytes;
+  const int per_launch = (int)std::max<size_t>(1, std::min<size_t>((size_t)n, (64u << 20) / per_real));
+  int rc = m->lex.ensure(per_real * per_launch, "lexicographic scratch");
+  if (rc) return rc;
+  FS_CUDA(launch_solve_lex(set, n, cap_x, tail_x, out, m->lex.p, per_launch, s), "launch lexicographic solve");
+  return FS_OK;
+}
+
+double demand_sum(const fs_model* m) {
+  double t = 0.0;
+  for (float v : m->h_lam) t += (double)v;
+  return t;
 }
 
 }  // namespace
@@ -590,6 +610,7 @@ int fs_solve(fs_model* m, const float* cap, const float* tail, fs_allocation* ou
   FS_CUDA(cudaMemcpyAsync(d_cap, cap, 4 * (size_t)cells, cudaMemcpyHostToDevice, s), "upload cap");
   FS_CUDA(cudaMemcpyAsync(d_tail, tail, 4 * (size_t)cells, cudaMemcpyHostToDevice, s), "upload tail");
   FS_CUDA(launch_solve(m->set, 1, d_cap, d_tail, d_out, false, m->lc, s), "launch solve");
+  if ((rc = solve_lex_pass(m, m->set, 1, d_cap, d_tail, d_out, s))) return rc;
   FS_CUDA(cudaMemcpyAsync(out, d_out, sizeof(fs_allocation), cudaMemcpyDeviceToHost, s), "read allocation");
   return read_status(m, s);
 }
@@ -604,7 +625,7 @@ int fs_solve_batch(fs_model* m, int32_t n, const float* cap_dev, const float* ta
   if (rc) return rc;
   FS_CUDA(launch_solve(m->set, n, cap_dev, tail_dev, out_dev, false, m->lc, (cudaStream_t)cuda_stream),
           "launch solve");
-  return FS_OK;
+  return solve_lex_pass(m, m->set, n, cap_dev, tail_dev, out_dev, (cudaStream_t)cuda_stream);
 }
 
 int fs_solve_bounds(fs_model* m, fs_allocation* minus, fs_allocation* plus, float* gamma_t) {
@@ -613,6 +634,7 @@ int fs_solve_bounds(fs_model* m, fs_allocation* minus, fs_allocation* plus, floa
   int rc0 = flush_bounds(m, s);
   if (rc0) return rc0;
   FS_CUDA(launch_solve(m->set, 2, nullptr, nullptr, nullptr, true, m->lc, s), "launch solve");
+  if ((rc0 = solve_lex_pass(m, m->set, 2, nullptr, nullptr, nullptr, s))) return rc0;
   fs_allocation h[2];
   FS_CUDA(cudaMemcpyAsync(h, m->set.base, sizeof h, cudaMemcpyDeviceToHost, s), "read allocations");
   int rc = read_status(m, s);
@@ -666,10 +688,73 @@ int fs_certificate(fs_model* m, float eps, int32_t* state, float* gamma_t) {
     while (j < kT && (1 << j) != am.tp[i]) ++j;
     if (!m->h_revealed[(size_t)(i * 4 + j) * m->d.B + am.bin[i]]) known = false;
   }
+  // under the lexicographic objective the gap is stage-wise (Section 4.2):
+  // the goodput gap |GP+ - GP-| / sum lambda must be within eps as well
+  bool gp_ok = true;
+  if (m->objective == FS_OBJECTIVE_LEXICOGRAPHIC)
+    gp_ok = std::fabs(ap.goodput - am.goodput) / demand_sum(m) <= (double)eps;
   if (!ap.floors_met) *state = 2;
-  else *state = (am.floors_met && gt <= eps && known) ? 1 : 0;
+  else *state = (am.floors_met && gt <= eps && known && gp_ok) ? 1 : 0;
   if (gamma_t) *gamma_t = gt;
   return FS_OK;
+}
+
+int fs_set_objective(fs_model* m, int32_t objective) {
+  if (!m) return fail(FS_EINVAL, "model is NULL");
+  if (objective != FS_OBJECTIVE_MAXMIN && objective != FS_OBJECTIVE_LEXICOGRAPHIC)
+    return fail(FS_EINVAL, "objective %d is not 0 or 1", objective);
+  if (objective == FS_OBJECTIVE_LEXICOGRAPHIC && lex_scratch_cells(m->d) * kLexCellBytes > (64u << 20))
+    return fail(FS_EINVAL, "the lexicographic objective needs (K + 1)(G + 1) <= 4 Mi cells");
+  m->objective = objective;
+  return FS_OK;
+}
+
+int fs_score_goodput(fs_model* m, const fs_samples* smp, double* gap_out, double* score_out, double* gamma_gp,
+                     int32_t* best, int64_t* sum_eo) {
+  if (!m) return fail(FS_EINVAL, "model is NULL");
+  int rc = check_samples(m, smp, true);
+  if (rc) return rc;
+  const double lam_sum = demand_sum(m);
+  if (!(lam_sum <= 1048576.0)) return fail(FS_EINVAL, "the goodput stage needs sum lambda <= 2^20 req/s");
+  if (m->d.G > 1024) return fail(FS_EINVAL, "the goodput stage needs G <= 1024");
+  if (lex_scratch_cells(m->d) * kLexCellBytes > (64u << 20)) return fail(FS_EINVAL, "(K + 1)(G + 1) too large");
+  const int n = smp->n_cand;
+  if ((rc = ensure_items(m, n, smp->O))) return rc;
+  cudaStream_t s = m->stream;
+  if ((rc = flush_bounds(m, s))) return rc;
+  const size_t nn = (size_t)std::max(n, 1);
+  int32_t* d_cand = static_cast<int32_t*>(m->cand.p);
+  double* d_gap = static_cast<double*>(m->outs.p);
+  double* d_score = d_gap + nn;
+  // (outs holds 16 nn + 64 bytes: gap, score, then gamma and best in the tail)
+  double* d_gamma = reinterpret_cast<double*>(static_cast<char*>(m->outs.p) + 16 * nn);
+  int32_t* d_best = reinterpret_cast<int32_t*>(d_gamma + 1);
+  if (n > 0) FS_CUDA(cudaMemcpyAsync(d_cand, smp->cand, 4 * (size_t)n, cudaMemcpyHostToDevice, s), "upload cand");
+  Items it{};
+  it.n = n;
+  it.cell = d_cand;
+  const Plan pl = make_plan(m, smp, n);
+  const int saved = m->objective;
+  m->objective = FS_OBJECTIVE_LEXICOGRAPHIC;  // the base solves to tier 4 (their goodput)
+  FS_CUDA(launch_solve(m->set, 2, nullptr, nullptr, nullptr, true, m->lc, s), "launch solve");
+  rc = solve_lex_pass(m, m->set, 2, nullptr, nullptr, nullptr, s);
+  m->objective = saved;
+  if (rc) return rc;
+  uint64_t* sums = static_cast<uint64_t*>(m->sums.p);
+  FS_CUDA(launch_prep(m->set, it, pl, static_cast<float*>(m->tables.p), sums, false, m->lc, s), "launch prep");
+  FS_CUDA(launch_score_goodput(m->set, it, pl, static_cast<const float*>(m->tables.p), sums, m->lc.floors,
+                               m->sm_count, s),
+          "launch goodput scorer");
+  FS_CUDA(launch_finalize_goodput(m->set, it, pl, sums, lam_sum, d_gap, d_score, d_gamma, d_best, s),
+          "launch goodput reduction");
+  if (gap_out && n) FS_CUDA(cudaMemcpyAsync(gap_out, d_gap, 8 * (size_t)n, cudaMemcpyDeviceToHost, s), "read gap");
+  if (score_out && n)
+    FS_CUDA(cudaMemcpyAsync(score_out, d_score, 8 * (size_t)n, cudaMemcpyDeviceToHost, s), "read score");
+  if (gamma_gp) FS_CUDA(cudaMemcpyAsync(gamma_gp, d_gamma, 8, cudaMemcpyDeviceToHost, s), "read gamma");
+  if (best) FS_CUDA(cudaMemcpyAsync(best, d_best, 4, cudaMemcpyDeviceToHost, s), "read best");
+  if (sum_eo && n)
+    FS_CUDA(cudaMemcpyAsync(sum_eo, sums, 8 * (size_t)n * smp->O, cudaMemcpyDeviceToHost, s), "read sums");
+  return read_status(m, s);
 }
 
 int fs_replay(fs_model* m, const fs_replay_spec* sp, int32_t* rounds, int32_t* state, double* gpu_seconds,
@@ -898,6 +983,7 @@ void fs_free_model(fs_model* m) {
   m->sums.release();
   m->outs.release();
   m->real.release();
+  m->lex.release();
   for (cudaEvent_t e : m->ev) cudaEventDestroy(e);
   if (m->up_done) cudaEventDestroy(m->up_done);
   m->h_up.release();

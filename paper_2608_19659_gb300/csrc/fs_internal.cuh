@@ -480,6 +480,20 @@ cudaError_t launch_finalize(const Set& set, const Items& it, const Plan& pl, con
                             uint64_t* part, cudaStream_t s);
 cudaError_t launch_watchdog(uint32_t* status, uint64_t limit_ns, cudaStream_t s);
 
+// tiers 3-4 and the goodput stage (fs_lex.cu)
+constexpr size_t kLexCellBytes = 16;  // one cell of the programme over classes and GPUs
+size_t lex_scratch_cells(const Dims& d);  // (K + 1)(G + 1) cells per realisation
+// Realisations [0, n) (as launch_solve reads them; their tier-2 allocations in
+// out / the base), per_launch of them at a time through scratch.
+cudaError_t launch_solve_lex(const Set& set, int n, const float* cap_x, const float* tail_x, fs_allocation* out,
+                             void* scratch, int per_launch, cudaStream_t s);
+size_t goodput_smem_bytes(const Dims& d, const Plan& pl, bool rf);
+cudaError_t launch_score_goodput(const Set& set, const Items& it, const Plan& pl, const float* tables,
+                                 uint64_t* sums, int floors, int sm_count, cudaStream_t s);
+cudaError_t launch_finalize_goodput(const Set& set, const Items& it, const Plan& pl, const uint64_t* sums,
+                                    double lam_sum, double* gap, double* score, double* gamma, int32_t* best,
+                                    cudaStream_t s);
+
 // replay
 struct ReplayState {
   const float* truth;     // [P][2][cells] cap, tail

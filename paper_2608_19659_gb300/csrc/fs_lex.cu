@@ -1,0 +1,397 @@
+// Tiers 3 and 4 of the lexicographic objective (Section 3) and the goodput
+// gap (Fig. 4a; the third stage of Section 4.2's stage-wise gap), for sm_103a.
+//
+// Section 3 orders the objective: (1) critical floors, (2) max min_i r_i,
+// (3) maximise total served goodput, (4) minimise fragmentation. The
+// threshold solver (k_solve) settles tiers 1-2 (t*, floors met). Among the
+// allocations that keep them optimal -- every class at r_i >= max(t*,
+// delta_i) when t* > 0; at t* = 0 the critical classes at their floors and
+// the others free; nothing at all when the floors cannot be met -- tier 3
+// takes the most goodput, sum_i x_i with x_i = min(lambda_i, n c) (Eqs. 2
+// and 4), each class's term in fixed point rint(x_i 2^20) so that sums are
+// exact; tier 4 the fewest GPUs in use, then class by class the threshold
+// solver's tie rules (no replicas first, lower TP, fewer replicas; the row's
+// best bin carries the larger-capacity and lower-bin rules).
+//
+// For a fixed (TP, n) a larger capacity never lowers goodput or fulfilment,
+// so one row per (class, TP) -- its best SLO-feasible bin -- carries every
+// useful option, and replica counts past the first that serves the whole
+// demand add GPUs and no goodput. The optimum is a programme over classes and
+// GPUs left: S_i(g) = the best (goodput, -GPUs) of classes i..K-1 within g
+// GPUs, S_K = 0, S_i(g) = max over class i's options (cost <= g) of their
+// goodput plus S_{i+1}(g - cost).
+//
+// k_solve_lex: one CTA per realisation; the table S in global scratch,
+//   threads over g, one class per step; thread 0 then walks the classes
+//   forward taking the preferred option that keeps the optimum.
+// k_score_goodput: the goodput stage of the Monte-Carlo score. Within a
+//   segment (candidate e, outcome o) a scenario's goodput gap
+//   |GP(A+') - GP(A-')| depends on its draw only through (c_y position,
+//   tail gate), as its t* does: the block tabulates those values (a warp per
+//   entry: each realisation's row capacity and t* as the scorer computes
+//   them, then the programme over the classes with row r patched, lanes over
+//   g), then draws every scenario's position and sums the entries.
+// k_finalize_goodput: E[Gamma_gp,t+1 | e] = sum 2^-20 / (O S) / sum lambda,
+//   the score Gamma_gp,t - E and the argmax (same order as the max-min stage).
+#include <cuda_runtime.h>
+
+#include "fs_finalize.cuh"
+#include "fs_internal.cuh"
+#include "fs_sample.cuh"
+
+namespace fs {
+
+// A class's served goodput in 2^-20 req/s: rint(min(lambda, fl(n c)) 2^20)
+// (2^20 x is exact; the conversion rounds to nearest, ties to even).
+__device__ __forceinline__ long long goodput_fx(float n, float c, float lam) {
+  const float served = __fmul_rn(n, c);
+  const float x = served < lam ? served : lam;
+  return __float2ll_rn(__fmul_rn(x, 0x1p20f));
+}
+
+// One programme cell: goodput (-1: unreachable) and GPUs in use.
+struct LexCell {
+  long long gp;
+  int gpus;
+};
+
+__device__ __forceinline__ bool lex_better(long long gpa, int gpusa, long long gpb, int gpusb) {
+  return gpa > gpb || (gpa == gpb && gpusa < gpusb);
+}
+
+// --------------------------------------------------------------------------- tiers 3-4
+
+__global__ void __launch_bounds__(256) k_solve_lex(Set set, int n_real, const float* cap_x, const float* tail_x,
+                                                   fs_allocation* out_x, LexCell* scratch, int r0) {
+  const Dims& d = set.d;
+  const int r = r0 + blockIdx.x;
+  const int tid = threadIdx.x;
+  if (r >= n_real) return;
+  const float* cap;
+  const float* tail;
+  fs_allocation* out;
+  if (cap_x) {
+    cap = cap_x + (size_t)r * d.cells;
+    tail = tail_x + (size_t)r * d.cells;
+    out = out_x + r;
+  } else {
+    const int p = r >> 1, sigma = r & 1;
+    const float* bp = set.bounds + (size_t)p * 4 * d.cells;
+    cap = bp + (size_t)(sigma ? CAP_HI : CAP_LO) * d.cells;
+    tail = bp + (size_t)(sigma ? TAIL_LO : TAIL_HI) * d.cells;
+    out = set.base + r;
+  }
+  LexCell* S = scratch + (size_t)blockIdx.x * (size_t)(d.K + 1) * (d.G + 1);
+  __shared__ float sC[256];
+  __shared__ int sB[256];
+  __shared__ float sT[FS_MAX_CLASSES];
+  __shared__ int sEmpty[FS_MAX_CLASSES];
+  const float tstar = out->t_star;
+  const int met = out->floors_met;
+  // rows: best SLO-feasible bin (largest capacity, then lowest bin)
+  for (int rho = tid; rho < d.K4; rho += blockDim.x) {
+    const int i = rho >> 2;
+    const float L = set.slo[i];
+    float best = 0.0f;
+    int bb = -1;
+    for (int b = 0; b < d.B; ++b) {
+      const size_t c = (size_t)rho * d.B + b;
+      if (tail[c] <= L) {
+        const float v = __fadd_rn(cap[c], 0.0f);  // -0 as +0
+        if (bb < 0 || v > best) {
+          best = v;
+          bb = b;
+        }
+      }
+    }
+    sC[rho] = best;
+    sB[rho] = bb;
+  }
+  for (int i = tid; i < d.K; i += blockDim.x) {
+    const float dl = set.slo[d.K + i];  // floors follow the SLOs (0: not critical)
+    sT[i] = tstar > 0.0f ? fmaxf(tstar, dl) : dl;
+    sEmpty[i] = !(tstar > 0.0f) && !(dl > 0.0f);
+  }
+  if (!met) {  // tier 1 cannot hold: nothing is allocated (k_solve wrote the empty allocation)
+    if (tid == 0) out->goodput = 0.0;
+    return;
+  }
+  for (int g = tid; g <= d.G; g += blockDim.x) S[(size_t)d.K * (d.G + 1) + g] = LexCell{0, 0};
+  __syncthreads();
+  for (int i = d.K - 1; i >= 0; --i) {
+    const LexCell* nxt = S + (size_t)(i + 1) * (d.G + 1);
+    LexCell* cur = S + (size_t)i * (d.G + 1);
+    const float lam = set.lam[i], T = sT[i];
+    for (int g = tid; g <= d.G; g += blockDim.x) {
+      LexCell best{-1, 0};
+      if (sEmpty[i] && nxt[g].gp >= 0) best = nxt[g];
+      for (int j = 0; j < kT; ++j) {
+        if (sB[4 * i + j] < 0) continue;
+        const float C = sC[4 * i + j];
+        const int M = rep_cap(d, j);
+        for (int n = 1; n <= M && (n << j) <= g; ++n) {
+          const float nf = (float)n;
+          if (T > 0.0f && !(fulfil(nf, C, lam) >= T)) continue;
+          const LexCell pv = nxt[g - (n << j)];
+          if (pv.gp >= 0) {
+            const long long v = goodput_fx(nf, C, lam) + pv.gp;
+            const int u = (n << j) + pv.gpus;
+            if (best.gp < 0 || lex_better(v, u, best.gp, best.gpus)) best = LexCell{v, u};
+          }
+          if (!(__fmul_rn(nf, C) < lam)) break;  // the whole demand served: more replicas add nothing
+        }
+      }
+      cur[g] = best;
+    }
+    __syncthreads();
+  }
+  if (tid != 0) return;
+  // forward: class by class the preferred option that keeps the optimum
+  int left = d.G, total = 0;
+  const long long gp_all = S[d.G].gp;
+  for (int i = 0; i < d.K; ++i) {
+    const LexCell target = S[(size_t)i * (d.G + 1) + left];
+    const LexCell* nxt = S + (size_t)(i + 1) * (d.G + 1);
+    const float lam = set.lam[i], T = sT[i];
+    int cj = -1, cn = 0;
+    if (!(sEmpty[i] && nxt[left].gp == target.gp && nxt[left].gpus == target.gpus)) {
+      for (int j = 0; j < kT && cj < 0; ++j) {
+        if (sB[4 * i + j] < 0) continue;
+        const float C = sC[4 * i + j];
+        const int M = rep_cap(d, j);
+        for (int n = 1; n <= M && (n << j) <= left; ++n) {
+          const float nf = (float)n;
+          if (T > 0.0f && !(fulfil(nf, C, lam) >= T)) continue;
+          const LexCell pv = nxt[left - (n << j)];
+          if (pv.gp >= 0 && goodput_fx(nf, C, lam) + pv.gp == target.gp && (n << j) + pv.gpus == target.gpus) {
+            cj = j;
+            cn = n;
+            break;
+          }
+        }
+      }
+    }
+    out->tp[i] = (int8_t)(cj >= 0 ? 1 << cj : 0);
+    out->bin[i] = (int16_t)(cj >= 0 ? sB[4 * i + cj] : -1);
+    out->replicas[i] = (int16_t)cn;
+    out->fulfil[i] = cj >= 0 ? fulfil((float)cn, sC[4 * i + cj], lam) : 0.0f;
+    if (cj >= 0) {
+      left -= cn << cj;
+      total += cn << cj;
+    }
+  }
+  out->total_gpus = total;
+  out->goodput = (double)gp_all * 0x1p-20;
+}
+
+// --------------------------------------------------------------------------- goodput stage
+
+// Tier-3 goodput of one realisation (rows sC / sOk of realisation sigma, row
+// rr patched to capacity Cr) at tiers 1-2 value t, by one warp: dp and tmp are
+// the warp's two arrays of G + 1 cells; -1 when the floors cannot be met.
+template <bool FL>
+__device__ long long warp_goodput(const Set& set, const float* sCs, const int* sOk, const float* sLam,
+                                  const float* sDl, int rr, float Cr, float t, long long* dp, long long* tmp) {
+  const Dims& d = set.d;
+  const int lane = threadIdx.x & 31;
+  for (int g = lane; g <= d.G; g += 32) dp[g] = 0;
+  __syncwarp();
+  for (int i = d.K - 1; i >= 0; --i) {
+    const float dl = FL ? sDl[i] : 0.0f;
+    const float T = t > 0.0f ? fmaxf(t, dl) : dl;
+    const bool may_empty = !(t > 0.0f) && !(dl > 0.0f);
+    const float lam = sLam[i];
+    for (int g = lane; g <= d.G; g += 32) {
+      long long best = may_empty ? dp[g] : -1;
+      for (int j = 0; j < kT; ++j) {
+        const int rho = 4 * i + j;
+        if (rho != rr && !sOk[rho]) continue;
+        const float C = rho == rr ? Cr : sCs[rho];
+        const int M = rep_cap(d, j);
+        for (int n = 1; n <= M && (n << j) <= g; ++n) {
+          const float nf = (float)n;
+          if (T > 0.0f && !(fulfil(nf, C, lam) >= T)) continue;
+          const long long pv = dp[g - (n << j)];
+          if (pv >= 0) {
+            const long long v = goodput_fx(nf, C, lam) + pv;
+            if (v > best) best = v;
+          }
+          if (!(__fmul_rn(nf, C) < lam)) break;
+        }
+      }
+      tmp[g] = best;
+    }
+    __syncwarp();
+    for (int g = lane; g <= d.G; g += 32) dp[g] = tmp[g];
+    __syncwarp();
+  }
+  const long long r = dp[d.G];
+  __syncwarp();
+  return r;
+}
+
+// t* of realisation sigma at row capacity C, from the candidate's table in
+// global memory (the IEEE row term: every input).
+template <bool FL>
+__device__ __forceinline__ float tstar_global(const float* h, float C) {
+  const int Lp = __float_as_int(h[H_LPAD]);
+  const float* kap = h + kTableHeader;
+  const float* thx = kap + Lp;
+  const float* mnx = thx + Lp;
+  int pos = 0;
+  for (int step = __float_as_int(h[H_STEP0]); step > 0; step >>= 1) pos += kap[pos + step - 1] <= C ? step : 0;
+  const float thb = thx[pos];
+  const float m = mnx[pos];
+  const float tr = m >= 1.0f ? fulfil(m, C, h[H_LAM]) : 0.0f;
+  if (FL) return (tr > thb && tr >= h[H_DLT]) ? tr : thb;
+  return tr > thb ? tr : thb;
+}
+
+template <bool FL, bool RF>
+__global__ void __launch_bounds__(256) k_score_goodput(Set set, Items it, Plan pl, const float* rec,
+                                                       uint64_t* sums) {
+  extern __shared__ __align__(16) unsigned char smraw[];
+  const Dims& d = set.d;
+  const int W = pl.W, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = blockDim.x >> 5;
+  const int gt_len = RF ? 2 * W : W + 1;
+  uint2* gtab = reinterpret_cast<uint2*>(smraw);
+  long long* dps = reinterpret_cast<long long*>(smraw + (((size_t)gt_len * 8 + 15) & ~(size_t)15));
+  long long* dp = dps + (size_t)warp * 2 * (d.G + 1);
+  long long* tmp = dp + (d.G + 1);
+  __shared__ float sC[2][256];
+  __shared__ int sOk[2][256];
+  __shared__ float sLam[FS_MAX_CLASSES], sDl[FS_MAX_CLASSES];
+  for (int x = tid; x < 2 * d.K4; x += blockDim.x) {
+    const int sg = x / d.K4, rho = x - sg * d.K4;
+    sC[sg][rho] = set.rowC[(size_t)sg * d.K4 + rho];
+    sOk[sg][rho] = set.rowB[(size_t)sg * d.K4 + rho] >= 0;
+  }
+  for (int i = tid; i < d.K; i += blockDim.x) {
+    sLam[i] = set.lam[i];
+    sDl[i] = FL ? set.slo[d.K + i] : 0.0f;
+  }
+  __syncthreads();
+  const PhiloxKeys keys{};  // (the plan's round keys serve a one-problem launch)
+  const long long n_seg = (long long)it.n * pl.O;
+  for (long long seg = blockIdx.x; seg < n_seg; seg += gridDim.x) {
+    const int item = (int)(seg / pl.O), o = (int)(seg - (long long)item * pl.O);
+    const float* r = rec + (size_t)item * pl.item_floats;
+    const float* h0 = r;
+    const float* h1 = r + d.slot_floats;
+    const float* win = r + 2 * (size_t)d.slot_floats + (size_t)o * pl.Wp;
+    const int cell = __float_as_int(h0[H_CELL]);
+    if (cell < 0 || cell >= d.cells) continue;  // flagged by the preparation (uniform over the block)
+    const int rr = cell / d.B;
+    const uint32_t kgs = (uint32_t)__float_as_int(win[0]) << pl.sh;
+    const uint32_t kgs16 = (uint32_t)min((unsigned long long)kgs << 16, 0xFFFFFFFFull);
+    const bool any_open = kgs != 0u, any_closed = kgs16 != 0xFFFFFFFFu;
+    const RowCap a0 = row_cap_of(h0), a1 = row_cap_of(h1);
+    // entries: [0, W) open gate at position k; [W, 2W) closed (under the prior)
+    // or W (closed, one value)
+    for (int k = warp; k < gt_len; k += nwarp) {
+      const bool g = k < W;
+      if ((g && !any_open) || (!g && !any_closed)) continue;
+      const float cy = g ? win[4 + k] : (RF ? win[4 + k - W] : 0.0f);
+      const float c0 = RF ? row_cap(a0, cy, g) : (g ? fmaxf(a0.pc, cy) : a0.pc);
+      const float c1 = RF ? row_cap(a1, cy, g) : (g ? fmaxf(a1.pc, cy) : a1.pc);
+      const float t0 = tstar_global<FL>(h0, c0), t1 = tstar_global<FL>(h1, c1);
+      long long g0 = warp_goodput<FL>(set, sC[0], sOk[0], sLam, sDl, rr, c0, t0, dp, tmp);
+      long long g1 = warp_goodput<FL>(set, sC[1], sOk[1], sLam, sDl, rr, c1, t1, dp, tmp);
+      g0 = g0 < 0 ? 0 : g0;
+      g1 = g1 < 0 ? 0 : g1;
+      const unsigned long long v = (unsigned long long)(g1 > g0 ? g1 - g0 : g0 - g1);
+      if (lane == 0) gtab[k] = make_uint2((uint32_t)(v >> 20), (uint32_t)v & 0xFFFFFu);
+    }
+    __syncthreads();
+    const GtabSum gs = sample_gtab<true, RF>(pl, keys, o, cell, 0, pl.calls, smem_u32(gtab), kgs16);
+    unsigned long long v = gs.total + ((unsigned long long)gs.h << 20) + gs.l;
+    for (int off = 16; off; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
+    if (lane == 0 && v) atomicAdd(reinterpret_cast<unsigned long long*>(&sums[(size_t)seg]), v);
+    __syncthreads();  // the table is rebuilt for the next segment
+  }
+}
+
+// E, score and argmax of the goodput stage for one problem (one CTA).
+__global__ void k_finalize_goodput(Set set, Items it, Plan pl, const uint64_t* sums, double lam_sum, double* gap,
+                                   double* score, double* gamma, int32_t* best) {
+  __shared__ Best sb[32];
+  const Dims& d = set.d;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = blockDim.x >> 5;
+  const long long gm = __double2ll_rn(__dmul_rn(set.base[0].goodput, 0x1p20));
+  const long long gpl = __double2ll_rn(__dmul_rn(set.base[1].goodput, 0x1p20));
+  const long long gfix = gpl > gm ? gpl - gm : gm - gpl;
+  const long long n = (long long)pl.O * pl.S;
+  const double dn = __ll2double_rn(n);
+  Best b = no_best();
+  for (int q = tid; q < it.n; q += blockDim.x) {
+    const int cell = it.cell[q];
+    long long tot = 0;
+    for (int o = 0; o < pl.O; ++o) tot += (long long)sums[(size_t)q * pl.O + o];
+    const long long sc = gfix * n - tot;
+    if (gap) gap[q] = __ddiv_rn(__ddiv_rn(__dmul_rn(__ll2double_rn(tot), 0x1p-20), dn), lam_sum);
+    if (score) score[q] = __ddiv_rn(__ddiv_rn(__dmul_rn(__ll2double_rn(sc), 0x1p-20), dn), lam_sum);
+    const Best c = make_best(sc, (cell / d.B) & 3, q, cell);
+    if (better(c, b)) b = c;
+  }
+  b = warp_best(b);
+  if (lane == 0) sb[warp] = b;
+  __syncthreads();
+  if (warp == 0) {
+    b = warp_best(lane < nwarp ? sb[lane] : no_best());
+    if (lane == 0) {
+      if (best) *best = b.valid() ? b.cell : -1;
+      if (gamma) *gamma = __ddiv_rn(__dmul_rn(__ll2double_rn(gfix), 0x1p-20), lam_sum);
+    }
+  }
+}
+
+// --------------------------------------------------------------------------- launchers
+
+size_t lex_scratch_cells(const Dims& d) { return (size_t)(d.K + 1) * (d.G + 1); }
+
+cudaError_t launch_solve_lex(const Set& set, int n, const float* cap_x, const float* tail_x, fs_allocation* out,
+                             void* scratch, int per_launch, cudaStream_t s) {
+  for (int r0 = 0; r0 < n; r0 += per_launch) {
+    const int m = n - r0 < per_launch ? n - r0 : per_launch;
+    note_launch();
+    k_solve_lex<<<m, 256, 0, s>>>(set, n, cap_x, tail_x, out, static_cast<LexCell*>(scratch), r0);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+size_t goodput_smem_bytes(const Dims& d, const Plan& pl, bool rf) {
+  const size_t gt_len = rf ? 2 * (size_t)pl.W : (size_t)pl.W + 1;
+  return ((gt_len * 8 + 15) & ~(size_t)15) + (size_t)8 * 2 * (d.G + 1) * 8;  // 8 warps x 2 arrays
+}
+
+cudaError_t launch_score_goodput(const Set& set, const Items& it, const Plan& pl, const float* tables,
+                                 uint64_t* sums, int floors, int sm_count, cudaStream_t s) {
+  if (it.n <= 0) return cudaSuccess;
+  const bool rf = set.prior == 1;
+  const size_t smem = goodput_smem_bytes(set.d, pl, rf);
+  auto kern = floors ? (rf ? k_score_goodput<true, true> : k_score_goodput<true, false>)
+                     : (rf ? k_score_goodput<false, true> : k_score_goodput<false, false>);
+  cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(kern), smem);
+  if (e != cudaSuccess) return e;
+  int per_sm = 0;
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 256, smem);
+  if (e != cudaSuccess) return e;
+  const long long n_seg = (long long)it.n * pl.O;
+  long long grid = (long long)(per_sm < 1 ? 1 : per_sm) * sm_count;
+  if (grid > n_seg) grid = n_seg;
+  note_launch();
+  kern<<<(unsigned)grid, 256, smem, s>>>(set, it, pl, tables, sums);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_finalize_goodput(const Set& set, const Items& it, const Plan& pl, const uint64_t* sums,
+                                    double lam_sum, double* gap, double* score, double* gamma, int32_t* best,
+                                    cudaStream_t s) {
+  note_launch();
+  k_finalize_goodput<<<1, 256, 0, s>>>(set, it, pl, sums, lam_sum, gap, score, gamma, best);
+  return cudaGetLastError();
+}
+
+}  // namespace fs

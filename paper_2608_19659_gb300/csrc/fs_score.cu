@@ -43,6 +43,7 @@
 
 #include "fs_finalize.cuh"
 #include "fs_internal.cuh"
+#include "fs_sample.cuh"
 
 namespace fs {
 
@@ -683,18 +684,6 @@ struct PieceSum {
   uint64_t total;  // earlier values, flushed
 };
 
-// Row r's capacity in a scenario under the monotone prior (see k_prep):
-// max(g ? max(P_open, c_y) : P_closed, min(max(c_y, F_lo), F_hi)).
-struct RowCap {
-  float pc, po, lf, hf;
-};
-
-__device__ __forceinline__ RowCap row_cap_of(const float* h) { return RowCap{h[H_CX], h[H_PO], h[H_LF], h[H_HF]}; }
-
-__device__ __forceinline__ float row_cap(const RowCap& r, float cy, bool g) {
-  return fmaxf(g ? fmaxf(r.po, cy) : r.pc, fminf(fmaxf(cy, r.lf), r.hf));
-}
-
 template <bool TS, int ROW, bool FL, bool RF>
 __device__ __forceinline__ PieceSum run_piece(const Plan& pl, const PhiloxKeys& keys, int o, int q_lo, int q_hi,
                                               const float* win, const float* h0, const float* h1,
@@ -881,80 +870,6 @@ __device__ __forceinline__ void build_gtab(uint2* gtab, int W, const float* win,
     const uint64_t gv = fixed40(__fsub_rn(t1, t0));
     gtab[k] = make_uint2((uint32_t)(gv >> 20), (uint32_t)gv & 0xFFFFFu);
   }
-}
-
-// Philox calls [q_lo, q_hi) of one segment on the table path: the sums of the
-// two fields of the drawn entries (each field below 2^21), flushed into a
-// 64-bit total every 256 calls so that the 32-bit sums cannot wrap. With at
-// most 32 values per thread nothing is flushed and a warp's field sums stay
-// below 2^32. Per sample: the capacity position umulhi(word, W); the tail gate,
-// (word & 0xFFFF) < kgs, as (word * 65536 mod 2^32) < kgs16 with kgs16 =
-// min(kgs 2^16, 2^32 - 1) (a multiply-add and a compare); the entry's shared
-// address base + index * 8 (a multiply-add); its load and two field sums. Two
-// calls per iteration give two independent Philox chains. KC: one problem, its
-// round keys read from the plan.
-struct GtabSum {
-  uint32_t h, l;   // the last at most 1024 values
-  uint64_t total;  // earlier values
-};
-
-template <bool KC>
-__device__ __forceinline__ uint4 draw_call(const Plan& pl, const PhiloxKeys& keys, uint32_t q, uint32_t ctr1,
-                                           uint32_t ctr2, uint32_t ctr3) {
-  if constexpr (KC) return philox4x32_10_plan(make_uint4(q, ctr1, ctr2, ctr3), pl);
-  else return philox4x32_10(make_uint4(q, ctr1, ctr2, ctr3), keys);
-}
-
-template <bool KC, bool RF>
-__device__ __forceinline__ GtabSum sample_gtab(const Plan& pl, const PhiloxKeys& keys, int o, int cell, int q_lo,
-                                               int q_hi, uint32_t gtab_s, uint32_t kgs16) {
-  const uint32_t ctr1 = (uint32_t)o, ctr2 = (uint32_t)cell, ctr3 = pl.round;
-  const uint32_t W = (uint32_t)pl.W;
-  const uint32_t mul = pl.lo16_mul, eb = pl.entry_bytes;
-  uint32_t gh = 0, glo = 0;
-  auto take = [&](uint32_t word) {
-    const uint32_t cap = __umulhi(word, W);
-    const uint32_t idx = word * mul < kgs16 ? cap : (RF ? cap + W : W);
-    uint32_t a, b;
-    asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(a), "=r"(b) : "r"(gtab_s + idx * eb));
-    gh += a;
-    glo += b;
-  };
-  auto take4 = [&](const uint4& x) {
-    take(x.x);
-    take(x.y);
-    take(x.z);
-    take(x.w);
-  };
-  const int q_full = min(q_hi, pl.S >> 2);  // calls whose four samples all exist
-  const int step = (int)blockDim.x;
-  uint64_t total = 0;
-  int q = q_lo + (int)threadIdx.x;
-  while (q < q_full) {
-    const int q_end = min(q_full, q + 256 * step);
-    for (; q + step < q_end; q += 2 * step) {
-      const uint4 x0 = draw_call<KC>(pl, keys, (uint32_t)q, ctr1, ctr2, ctr3);
-      const uint4 x1 = draw_call<KC>(pl, keys, (uint32_t)(q + step), ctr1, ctr2, ctr3);
-      take4(x0);
-      take4(x1);
-    }
-    if (q < q_end) {
-      take4(draw_call<KC>(pl, keys, (uint32_t)q, ctr1, ctr2, ctr3));
-      q += step;
-    }
-    if (q < q_full) {
-      total += ((uint64_t)gh << 20) + glo;
-      gh = glo = 0;
-    }
-  }
-  if (q < q_hi) {  // the segment's last call, serving S mod 4 samples
-    const uint4 x = draw_call<KC>(pl, keys, (uint32_t)q, ctr1, ctr2, ctr3);
-    const int nv = pl.S - 4 * q;
-    take(x.x);
-    if (nv > 1) take(x.y);
-    if (nv > 2) take(x.z);
-  }
-  return GtabSum{gh, glo, total};
 }
 
 // Work decomposition of one k_score launch: segment = (item, outcome) with

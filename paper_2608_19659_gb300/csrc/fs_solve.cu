@@ -468,6 +468,7 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
     out->has_option_mask = (uint64_t)(uint32_t)sMisc[2] | ((uint64_t)(uint32_t)sMisc[3] << 32);
     out->ok = tstar > 0.0f ? 1 : 0;
     out->floors_met = (!FL || (sMisc[6] == 0 && sMisc[5] <= d.G)) ? 1 : 0;
+    out->goodput = 0.0;  // tier 3 is filled by the lexicographic solve
   }
   if (write_theta && !cap_x) {
     float* th = set.theta + ((size_t)p * 2 + sigma) * d.theta_cap;

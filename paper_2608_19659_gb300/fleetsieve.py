@@ -23,7 +23,8 @@ FS_OK, FS_EINVAL, FS_ENOMEM, FS_ECUDA, FS_ETIMEOUT, FS_EDEVICE = 0, -1, -2, -3, 
 FS_MAX_CLASSES = 64
 EXPORTS = ("fs_load_model", "fs_update_bounds", "fs_set_floors", "fs_dump_stride", "fs_score_candidates",
            "fs_score_candidates_async", "fs_solve", "fs_solve_batch", "fs_solve_bounds",
-           "fs_reveal", "fs_set_prior", "fs_get_state", "fs_certificate", "fs_replay", "fs_check", "fs_launch_count",
+           "fs_reveal", "fs_set_prior", "fs_set_objective", "fs_score_goodput", "fs_get_state",
+           "fs_certificate", "fs_replay", "fs_check", "fs_launch_count",
            "fs_watchdog_selftest", "fs_free_model", "fs_last_error", "fs_score_candidates_noalloc",
            "fs_timing_enable",
            "fs_timing_read")
@@ -52,7 +53,8 @@ class fs_allocation(C.Structure):
     _fields_ = [("t_star", C.c_float), ("total_gpus", C.c_int32),
                 ("has_option_mask", C.c_uint64), ("ok", C.c_int32), ("floors_met", C.c_int32),
                 ("tp", C.c_int8 * FS_MAX_CLASSES), ("bin", C.c_int16 * FS_MAX_CLASSES),
-                ("replicas", C.c_int16 * FS_MAX_CLASSES), ("fulfil", C.c_float * FS_MAX_CLASSES)]
+                ("replicas", C.c_int16 * FS_MAX_CLASSES), ("fulfil", C.c_float * FS_MAX_CLASSES),
+                ("goodput", C.c_double)]
 
 
 class fs_replay_spec(C.Structure):
@@ -63,10 +65,11 @@ class fs_replay_spec(C.Structure):
 
 
 ALLOC_DTYPE = np.dtype({"names": ["t_star", "total_gpus", "has_option_mask", "ok", "floors_met",
-                                  "tp", "bin", "replicas", "fulfil"],
+                                  "tp", "bin", "replicas", "fulfil", "goodput"],
                         "formats": [np.float32, np.int32, np.uint64, np.int32, np.int32,
-                                    (np.int8, 64), (np.int16, 64), (np.int16, 64), (np.float32, 64)],
-                        "offsets": [0, 4, 8, 16, 20, 24, 88, 216, 344], "itemsize": 600})
+                                    (np.int8, 64), (np.int16, 64), (np.int16, 64), (np.float32, 64),
+                                    np.float64],
+                        "offsets": [0, 4, 8, 16, 20, 24, 88, 216, 344, 600], "itemsize": 608})
 
 _lib = None
 
@@ -100,6 +103,9 @@ def lib():
                                       C.POINTER(fs_allocation), fp]
         L.fs_reveal.argtypes = [C.c_void_p, C.c_int32, C.c_float, C.c_float]
         L.fs_set_prior.argtypes = [C.c_void_p, C.c_int32]
+        L.fs_set_objective.argtypes = [C.c_void_p, C.c_int32]
+        L.fs_score_goodput.argtypes = [C.c_void_p, C.POINTER(fs_samples), C.c_void_p, C.c_void_p,
+                                       C.c_void_p, C.c_void_p, C.c_void_p]
         L.fs_get_state.argtypes = [C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p, C.c_void_p,
                                    C.c_void_p]
         L.fs_certificate.argtypes = [C.c_void_p, C.c_float, C.POINTER(C.c_int32), fp]
@@ -298,7 +304,7 @@ def alloc_to_dict(a: fs_allocation, K: int) -> dict:
             "has_option_mask": int(a.has_option_mask), "ok": int(a.ok), "floors_met": int(a.floors_met),
             "tp": [int(a.tp[i]) for i in range(K)], "bin": [int(a.bin[i]) for i in range(K)],
             "replicas": [int(a.replicas[i]) for i in range(K)],
-            "fulfil": [float(np.float32(a.fulfil[i])) for i in range(K)]}
+            "fulfil": [float(np.float32(a.fulfil[i])) for i in range(K)], "goodput": float(a.goodput)}
 
 
 def fs_solve(m: Model, cap, tail) -> dict:
@@ -309,7 +315,7 @@ def fs_solve(m: Model, cap, tail) -> dict:
 
 
 def fs_solve_batch(m: Model, n: int, cap_dev, tail_dev, out_dev, stream=None) -> None:
-    """out_dev: a torch uint8 tensor of n * 600 bytes (view it with :data:`ALLOC_DTYPE`)."""
+    """out_dev: a torch uint8 tensor of n * 608 bytes (view it with :data:`ALLOC_DTYPE`)."""
     _check(lib().fs_solve_batch(m.handle, int(n), _vp(cap_dev), _vp(tail_dev), _vp(out_dev),
                                 _stream(stream)))
 
@@ -332,6 +338,38 @@ def fs_set_prior(m: Model, prior: int) -> None:
     """How a measurement refits the intervals: FS_PRIOR_REVEALED (the measured
     cell only) or FS_PRIOR_MONOTONE (also its row, nondecreasing in load)."""
     _check(lib().fs_set_prior(m.handle, int(prior)))
+
+
+FS_OBJECTIVE_MAXMIN, FS_OBJECTIVE_LEXICOGRAPHIC = 0, 1
+
+
+def fs_set_objective(m: Model, objective: int) -> None:
+    """FS_OBJECTIVE_MAXMIN (tiers 1-2) or FS_OBJECTIVE_LEXICOGRAPHIC (tiers 1-4) for
+    the model's solves and certificate."""
+    _check(lib().fs_set_objective(m.handle, int(objective)))
+
+
+@dataclasses.dataclass
+class GoodputScore:
+    gap: np.ndarray  # [n_cand] E[Gamma_gp,t+1 | e] (fraction of total demand)
+    score: np.ndarray  # [n_cand]
+    gamma_gp: float
+    best: int
+    sum_eo: np.ndarray  # [n_cand, O] int64, 2^-20 req/s
+
+
+def fs_score_goodput(m: Model, cand, O: int, S: int, seed: int, stream_id: int = 0, rnd: int = 0) -> GoodputScore:
+    """The goodput stage of the Monte-Carlo score (host inputs and outputs)."""
+    cand = np.ascontiguousarray(cand, dtype=np.int32)
+    n = cand.size
+    gap = np.zeros(n, np.float64)
+    score = np.zeros(n, np.float64)
+    gg = np.zeros(1, np.float64)
+    best = np.zeros(1, np.int32)
+    sums = np.zeros((n, O), np.int64)
+    smp = _samples(seed, stream_id, rnd, n, O, S, _vp(cand) if n else None)
+    _check(lib().fs_score_goodput(m.handle, C.byref(smp), _vp(gap), _vp(score), _vp(gg), _vp(best), _vp(sums)))
+    return GoodputScore(gap, score, float(gg[0]), int(best[0]), sums)
 
 
 def fs_get_state(m: Model):

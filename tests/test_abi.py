@@ -40,8 +40,9 @@ def test_binding_refuses_a_missing_library(fsb, monkeypatch):
 
 
 def test_allocation_layout(fsb):
-    assert ctypes.sizeof(fsb.fs_allocation) == 600 == fsb.ALLOC_DTYPE.itemsize
+    assert ctypes.sizeof(fsb.fs_allocation) == 608 == fsb.ALLOC_DTYPE.itemsize
     assert fsb.fs_allocation.fulfil.offset == 344 and fsb.fs_allocation.bin.offset == 88
+    assert fsb.fs_allocation.goodput.offset == 600
 
 
 def _good(K=2, B=3):

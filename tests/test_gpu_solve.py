@@ -40,7 +40,7 @@ def _solve_batch(fsb, torch, m, cap, tail):
     n = cap.shape[0]
     dc = torch.from_numpy(cap).cuda()
     dt = torch.from_numpy(tail).cuda()
-    out = torch.zeros(n * 600, dtype=torch.uint8, device="cuda")
+    out = torch.zeros(n * fsb.ALLOC_DTYPE.itemsize, dtype=torch.uint8, device="cuda")
     fsb.fs_solve_batch(m, n, dc, dt, out)
     fsb.fs_check(m)
     torch.cuda.synchronize()
