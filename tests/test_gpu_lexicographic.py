@@ -100,32 +100,19 @@ def test_table3_on_the_gpu(fsb, cuda, oracle_lib):
 
 
 def test_stagewise_certificate(fsb, cuda, oracle_lib):
-    """With every cell revealed at values that leave a goodput difference only
-    through other cells' intervals, the max-min objective may certify where the
-    lexicographic one (goodput gap above eps) does not; each equals the oracle."""
-    rp = workloads.make_replay(n_streams=6)
-    w = rp.base
-    prob = oracle_lib.Problem.of(w)
-    hits = 0
-    for k in range(6):
-        rev = np.zeros(w.cells, np.uint8)
-        clo, chi = w.cap_lo.reshape(-1).copy(), w.cap_hi.reshape(-1).copy()
-        tlo, thi = w.tail_lo.reshape(-1).copy(), w.tail_hi.reshape(-1).copy()
-        for c in rp.perm[k][:40]:
-            clo[c] = chi[c] = rp.truth_cap[k][c]
-            tlo[c] = thi[c] = rp.truth_tail[k][c]
-            rev[c] = 1
-        for eps in (0.0, 0.05, 0.3):
-            with fsb.fs_load_model(clo, chi, tlo, thi, w.slo, w.demand, w.G, w.K, w.B, revealed=rev) as m:
-                fsb.fs_set_objective(m, LEX)
-                st, gt = fsb.fs_certificate(m, eps)
-                fsb.fs_set_objective(m, 0)
-                st0, _ = fsb.fs_certificate(m, eps)
-            ref = oracle_lib.certificate_lex(prob, clo, chi, tlo, thi, rev, eps)
-            ref0 = oracle_lib.certificate(prob, clo, chi, tlo, thi, rev, eps)
-            assert (st, gt) == (ref[0], ref[1]) and st0 == ref0[0]
-            hits += st0 == 1 and st == 0
-    assert hits >= 0
+    """No max-min gap but a goodput gap of 0.25: the max-min objective certifies,
+    the lexicographic one waits until eps reaches the goodput gap."""
+    from test_oracle_lexicographic import _stagewise_instance
+
+    K, B, G, lam, slo, clo, chi, tlo, thi, rev = _stagewise_instance()
+    with fsb.fs_load_model(clo, chi, tlo, thi, slo, lam, G, K, B, revealed=rev) as m:
+        assert fsb.fs_certificate(m, 0.01) == (1, 0.0)
+        fsb.fs_set_objective(m, LEX)
+        assert fsb.fs_certificate(m, 0.01) == (0, 0.0)
+        assert fsb.fs_certificate(m, 0.25) == (1, 0.0)
+        am, ap, _ = fsb.fs_solve_bounds(m)
+    assert (am["goodput"], ap["goodput"]) == (4.0, 6.0)
+    assert am["replicas"] == [1, 4] and ap["tp"] == [8, 2] and ap["replicas"] == [1, 2]
 
 
 @pytest.mark.parametrize("idx,factor,S,n_cand", [(0, 3.0, 256, None), (1, 1.0, 512, 24), (2, 3.0, 256, 12)])

@@ -156,3 +156,35 @@ def test_goodput_scenarios_match_brute_force(oracle_lib, seed):
                     res.append(brute.lexicographic(w.K, w.B, w.G, c, t, w.demand, w.slo)[1])
                 tot += abs(res[1] - res[0])
             assert r.sum_eo[e, o] == tot
+
+
+def _stagewise_instance():
+    """Class 0's only option (TP8, 2 req/s per replica, lambda 4) caps max-min at
+    0.5 in both realisations; class 1 commits to its measured TP1 cell (0.5 req/s)
+    under A- while A+ would serve it fully on an unmeasured TP2 cell ([0, 3]):
+    no max-min gap, a goodput gap of 2 req/s of 8."""
+    K, B = 2, 1
+    clo = np.zeros((K, 4, B), np.float32)
+    chi = np.zeros_like(clo)
+    tlo = np.full((K, 4, B), 1e9, np.float32)
+    thi = np.full_like(tlo, 1e9)
+    clo[0, 3, 0] = chi[0, 3, 0] = 2.0
+    tlo[0, 3, 0] = thi[0, 3, 0] = 1.0
+    clo[1, 0, 0] = chi[1, 0, 0] = 0.5
+    tlo[1, 0, 0] = thi[1, 0, 0] = 1.0
+    chi[1, 1, 0] = 3.0
+    tlo[1, 1, 0] = thi[1, 1, 0] = 1.0
+    rev = np.zeros(K * 4 * B, np.uint8)
+    rev[3] = rev[4] = 1
+    return K, B, 12, [4.0, 4.0], [10.0, 10.0], clo, chi, tlo, thi, rev
+
+
+def test_stagewise_certificate_waits_for_the_goodput_gap(oracle_lib):
+    K, B, G, lam, slo, clo, chi, tlo, thi, rev = _stagewise_instance()
+    p = oracle_lib.Problem(K, B, G, lam, slo)
+    assert oracle_lib.certificate(p, clo, chi, tlo, thi, rev, 0.01) == (1, 0.0)
+    assert oracle_lib.certificate_lex(p, clo, chi, tlo, thi, rev, 0.01) == (0, 0.0, 0.25)
+    assert oracle_lib.certificate_lex(p, clo, chi, tlo, thi, rev, 0.25)[0] == 1
+    am, ap, gm, gp, gmm, ggp = oracle_lib.base_gap_lex(p, clo, chi, tlo, thi)
+    assert (am.tp, am.replicas, gm) == ([8, 1], [1, 4], 4 * 2**20)
+    assert (ap.tp, ap.replicas, gp) == ([8, 2], [1, 2], 6 * 2**20)
