@@ -52,17 +52,20 @@ ISSUE_PER_SM_CLK = 4 * 32  # 4 schedulers x 32 lanes, one warp instruction each 
 #   Gamma' = t*(A+') - t*(A-')                                             1
 #   exact fixed-point accumulation of rint(Gamma' 2^40)                   7
 # Table path (a segment's W + 1 values of rint(Gamma' 2^40) tabulated once):
-# per scenario the Philox share (10), capacity position (1), gate mask,
-# compare and index select (3), the entry's load (1) and its two field sums
-# (2) = 17; per table entry evaluated the two patched capacities (2), two
-# table searches (6), Gamma' (1), the fixed-point conversion (5) and the store
-# (1) = 15. A segment whose tail gate is closed at every position of its
-# stratum evaluates no entry (all equal the closed-gate value, from the
-# preparation); the library counts the entries evaluated. Search probes
-# beyond the first (3 each) and row-term fulfilments are not counted: lower
-# bounds.
+# per scenario the Philox share (10), capacity position (1), the entry's load
+# (1) and its two field sums (2) = 14, plus the tail gate's test (mask,
+# compare, index select: 3) in the scenarios of strata whose tails lie on both
+# sides of the SLO (elsewhere the gate is the same at every position); per
+# table entry evaluated the two patched capacities (2), two table searches (6),
+# Gamma' (1), the fixed-point conversion (5) and the store (1) = 15. A segment
+# whose tail gate is closed at every position of its stratum evaluates no
+# entry (all equal the closed-gate value, from the preparation). The library
+# counts the entries evaluated and the scenarios that tested their gate.
+# Search probes beyond the first (3 each) and row-term fulfilments are not
+# counted: lower bounds.
 OPS_PER_SCENARIO = 32
-OPS_PER_SCENARIO_TABLE = 17
+OPS_PER_SCENARIO_TABLE = 14
+OPS_PER_GATE_TEST = 3
 OPS_PER_TABLE_ENTRY = 15
 Q_TABLE = 4096  # quantile table size of the built-in triangular table
 
@@ -75,15 +78,19 @@ def table_path(O: int, S: int) -> bool:
     return W <= 4096 and 3 * (W + 1) <= 2 * min(S, 2048)
 
 
-def algorithmic_ops(w, entries_per_launch=None) -> float:
+def algorithmic_ops(w, entries_per_launch=None, gated_per_launch=None) -> float:
     """Algorithmic thread-operations of one Monte-Carlo launch over workload w:
-    on the table path, with the gap-table entries the launch evaluated (as the
-    library counted them; None: W entries in every segment)."""
+    on the table path, with the gap-table entries the launch evaluated and the
+    scenarios that tested their tail gate (as the library counted them; None:
+    W entries and a gate test in every segment)."""
     if table_path(w.O, w.S):
         W = Q_TABLE // w.O
         if entries_per_launch is None:
             entries_per_launch = float(len(w.candidates)) * w.O * W
-        return float(OPS_PER_SCENARIO_TABLE) * w.scenarios + OPS_PER_TABLE_ENTRY * float(entries_per_launch)
+        if gated_per_launch is None:
+            gated_per_launch = float(w.scenarios)
+        return (float(OPS_PER_SCENARIO_TABLE) * w.scenarios + OPS_PER_GATE_TEST * float(gated_per_launch)
+                + OPS_PER_TABLE_ENTRY * float(entries_per_launch))
     return float(OPS_PER_SCENARIO) * w.scenarios
 
 # ncu summaries with the DRAM bytes of one k_score launch, per workload; used
@@ -278,12 +285,12 @@ def other_workload(idx: int, steps: int, warmup: int, alu_peak: float, stream_id
         flush.zero_()
         step()
     torch.cuda.synchronize()
-    kernel_ms, kernel_n, _, entries = fsb.fs_timing_read(m, with_entries=True)
+    kernel_ms, kernel_n, _, (entries, gated) = fsb.fs_timing_read(m, with_entries=True)
     fsb.fs_timing_enable(m, 0)
     fsb.fs_check(m, stream)
     fsb.fs_free_model(m)
     kern_s = kernel_ms / 1000.0 / max(kernel_n, 1)
-    achieved = algorithmic_ops(w, entries / max(kernel_n, 1)) / kern_s
+    achieved = algorithmic_ops(w, entries / max(kernel_n, 1), gated / max(kernel_n, 1)) / kern_s
     gamma_t = float(gt.item())
     return {"workload": w.name, "ms_per_step": step_ms, "scenarios_per_s": w.scenarios / (step_ms / 1000.0),
             "gamma_t": gamma_t,
@@ -630,7 +637,7 @@ def main(argv=None):
             if (k + 1) % 1000 == 0:  # the library keeps up to 4096 timed calls
                 torch.cuda.synchronize()
         torch.cuda.synchronize()
-        kernel_ms, kernel_n, _, entries = fsb.fs_timing_read(model, with_entries=True)
+        kernel_ms, kernel_n, _, (entries, gated) = fsb.fs_timing_read(model, with_entries=True)
         fsb.fs_timing_enable(model, 0)
     step_ms = step_ms_of(starts, ends)
     total_ms = max_over_ranks(dist, sum(step_ms), dev)
@@ -675,7 +682,8 @@ def main(argv=None):
     alu_peak = sms * ISSUE_PER_SM_CLK * sm_max * 1e6  # thread-ops/s at the maximum SM clock
     kern_s = kernel_ms / 1000.0 / max(kernel_n, 1)
     entries_per_launch = entries / max(kernel_n, 1)
-    ops = algorithmic_ops(w, entries_per_launch)
+    gated_per_launch = gated / max(kernel_n, 1)
+    ops = algorithmic_ops(w, entries_per_launch, gated_per_launch)
     achieved = ops / kern_s if kernel_n else None
     roofline = {"bound": "alu", "kernel": "k_score (Monte-Carlo sampler + parametric re-solve)",
                 "achieved": achieved / 1e12 if achieved else None,
@@ -685,6 +693,7 @@ def main(argv=None):
                 "algorithmic_bytes": 0, "kernel_ms_per_launch": kern_s * 1000.0,
                 "ops_per_scenario": ops / w.scenarios,
                 "table_entries_per_launch": entries_per_launch,
+                "gate_tested_scenarios_per_launch": gated_per_launch,
                 "path": "table" if table_path(w.O, w.S) else "plain",
                 "peak_basis": f"{sms} SMs x 4 issue slots x 32 lanes x {sm_max:.0f} MHz (max SM clock)",
                 "kernel_share_of_step": (kern_s * 1000.0 / (sum(step_ms) / len(step_ms))) if kernel_n else None}

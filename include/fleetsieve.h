@@ -218,7 +218,7 @@ int fs_score_candidates_async(fs_model *m, const fs_samples *samples, double *ga
  * process exits. A call takes the following pieces of it, each rounded up to
  * a multiple of 256 bytes, and returns FS_EINVAL without running when their
  * sum exceeds 16 MiB:
- *   4, 24 and 1024 bytes (status word, counters, reduction scratch);
+ *   4, 32 and 1024 bytes (status word, counters, reduction scratch);
  *   4 Q (only with quantile_dev NULL: the built-in table);
  *   8 T and 8, with T = K (floor(G/1) + floor(G/2) + floor(G/4) + floor(G/8))
  *     (thresholds and their counts);
@@ -428,19 +428,20 @@ int fs_check(fs_model *m, void *cuda_stream);
  * later scoring call of this model records CUDA events around its
  * Monte-Carlo kernel on the stream it launches on; mode 2: also around the
  * base solves, the table preparation and the reduction; 0: off (up to 4096
- * calls are kept). fs_timing_enable also zeroes the model's count of table
- * entries evaluated. fs_timing_read waits for the recorded events and returns
- * the summed Monte-Carlo kernel time (ms), the number of timed calls, in mode
- * 2 phase_ms[4] = summed (solve, prep, Monte-Carlo, reduction) time, and
- * table_entries = the gap-table entries the Monte-Carlo kernel evaluated
- * (two t* each) on its table path since the count was last zeroed (each
- * outputs nullable); it clears the record and the count. Events between
- * kernels also stop the next kernel from starting early, so timed calls can
- * take a little longer.
+ * calls are kept). fs_timing_enable also zeroes the model's work counts.
+ * fs_timing_read waits for the recorded events and returns the summed
+ * Monte-Carlo kernel time (ms), the number of timed calls, in mode 2
+ * phase_ms[4] = summed (solve, prep, Monte-Carlo, reduction) time, and
+ * work_counts[2] = what the Monte-Carlo kernel's table path did since the
+ * counts were last zeroed: the gap-table entries it evaluated (two t* each;
+ * once per segment) and the scenarios that tested their tail gate (those of
+ * strata whose tails lie on both sides of the SLO) (each output nullable); it
+ * clears the record and the counts. Events between kernels also stop the
+ * next kernel from starting early, so timed calls can take a little longer.
  */
 int fs_timing_enable(fs_model *m, int32_t mode);
 int fs_timing_read(fs_model *m, double *kernel_ms, int32_t *launches, double *phase_ms,
-                   uint64_t *table_entries);
+                   uint64_t *work_counts);
 
 /* Kernels this library has launched since it was loaded (all models). */
 uint64_t fs_launch_count(void);

@@ -447,7 +447,7 @@ int fs_load_model(const fs_bounds* b, const float* slo, const float* demand, int
   const size_t o_bounds = take(16 * (size_t)cells), o_rev = take(cells);
   const size_t o_theta = take(8 * (size_t)d.theta_cap), o_nth = take(8);
   const size_t o_rowc = take(8 * (size_t)d.K4), o_rowb = take(8 * (size_t)d.K4);
-  const size_t o_base = take(2 * sizeof(fs_allocation)), o_status = take(4), o_work = take(24);
+  const size_t o_base = take(2 * sizeof(fs_allocation)), o_status = take(4), o_work = take(32);
   const size_t o_rtab = take(8 * (size_t)kRowTabMax);
   rc = m->fixed.ensure(off, "model state");
   if (rc) {
@@ -911,9 +911,9 @@ int fs_check(fs_model* m, void* cuda_stream) {
   return read_status(m, cuda_stream ? (cudaStream_t)cuda_stream : m->stream);
 }
 
-// The table-entry count (work[2]) of the model, zeroed in stream order.
+// The work counts (work[2..3]) of the model, zeroed in stream order.
 static int zero_entry_count(fs_model* m) {
-  FS_CUDA(cudaMemsetAsync(m->set.work + 2, 0, 8, m->stream), "zero the entry count");
+  FS_CUDA(cudaMemsetAsync(m->set.work + 2, 0, 16, m->stream), "zero the entry count");
   FS_CUDA(cudaStreamSynchronize(m->stream), "zero the entry count");
   return FS_OK;
 }
@@ -926,11 +926,11 @@ int fs_timing_enable(fs_model* m, int32_t on) {
   return zero_entry_count(m);
 }
 
-int fs_timing_read(fs_model* m, double* kernel_ms, int32_t* launches, double* phase_ms, uint64_t* table_entries) {
+int fs_timing_read(fs_model* m, double* kernel_ms, int32_t* launches, double* phase_ms, uint64_t* work_counts) {
   if (!m) return fail(FS_EINVAL, "model is NULL");
-  if (table_entries) {
+  if (work_counts) {
     FS_CUDA(cudaDeviceSynchronize(), "wait for the scoring calls");
-    FS_CUDA(cudaMemcpy(table_entries, m->set.work + 2, 8, cudaMemcpyDeviceToHost), "read the entry count");
+    FS_CUDA(cudaMemcpy(work_counts, m->set.work + 2, 16, cudaMemcpyDeviceToHost), "read the work counts");
     int rc = zero_entry_count(m);
     if (rc) return rc;
   }

@@ -10,8 +10,9 @@
 //   rowC     [P][2][K*4]   f32   best SLO-feasible capacity per (class, TP)
 //   rowB     [P][2][K*4]   i32   its bin (-1: none)
 //   base     [P][2]        fs_allocation
-//   work     [3]           u64   chunk counter of the Monte-Carlo kernel, the reduction's ticket,
-//                                 table entries evaluated (accumulates across calls; the host zeroes it)
+//   work     [4]           u64   chunk counter of the Monte-Carlo kernel, the reduction's ticket,
+//                                 table entries evaluated and scenarios that tested their tail
+//                                 gate (both accumulate across calls; the host zeroes them)
 // Per scoring call (items = (problem, candidate cell) pairs), one record of
 // item_floats = 2 slot_floats + O Wp floats per item:
 //   [2][slot_floats] f32   threshold tables of the two realisations
@@ -98,8 +99,9 @@ struct Set {
   int* rowB;            // [P][2][K4] bin of rowC, -1 = no SLO-feasible bin
   fs_allocation* base;  // [P][2]
   uint32_t* status;
-  unsigned long long* work;  // [3] chunk counter, reduction ticket (zeroed by k_prep); table entries
-                             // evaluated by the Monte-Carlo kernel (summed over calls, zeroed by the host)
+  unsigned long long* work;  // [4] chunk counter, reduction ticket (zeroed by k_prep); table entries
+                             // evaluated and scenarios that tested their tail gate in the Monte-Carlo
+                             // kernel (summed over calls, zeroed by the host)
   const int* skip;      // [P] or nullptr: base solves skip problems with skip[p] >= 0
   int* rtab;            // [P][2][kRowTabMax] or nullptr: row tables of the scoring solves,
                         // word (row rho, threshold k) at k K4 + rho

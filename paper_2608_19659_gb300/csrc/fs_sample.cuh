@@ -28,7 +28,12 @@ __device__ __forceinline__ float row_cap(const RowCap& r, float cy, bool g) {
 // min(kgs 2^16, 2^32 - 1) (a multiply-add and a compare); the entry's shared
 // address base + index * 8 (a multiply-add); its load and two field sums. Two
 // calls per iteration give two independent Philox chains. KC: one problem, its
-// round keys read from the plan.
+// round keys read from the plan. GATE = false: the stratum's tail gate is the
+// same at every position (its mapped tails all pass the SLO, or none does;
+// known from the preparation's gate position), so the entry is the capacity
+// position's in the table at gtab_s (the open half, or under the prior the
+// closed half; without the prior a closed stratum's table holds the
+// closed-gate value at every position) and no scenario tests the gate.
 struct GtabSum {
   uint32_t h, l;   // the last at most 1024 values
   uint64_t total;  // earlier values
@@ -41,7 +46,7 @@ __device__ __forceinline__ uint4 draw_call(const Plan& pl, const PhiloxKeys& key
   else return philox4x32_10(make_uint4(q, ctr1, ctr2, ctr3), keys);
 }
 
-template <bool KC, bool RF>
+template <bool KC, bool RF, bool GATE = true>
 __device__ __forceinline__ GtabSum sample_gtab(const Plan& pl, const PhiloxKeys& keys, int o, int cell, int q_lo,
                                                int q_hi, uint32_t gtab_s, uint32_t kgs16) {
   const uint32_t ctr1 = (uint32_t)o, ctr2 = (uint32_t)cell, ctr3 = pl.round;
@@ -50,7 +55,7 @@ __device__ __forceinline__ GtabSum sample_gtab(const Plan& pl, const PhiloxKeys&
   uint32_t gh = 0, glo = 0;
   auto take = [&](uint32_t word) {
     const uint32_t cap = __umulhi(word, W);
-    const uint32_t idx = word * mul < kgs16 ? cap : (RF ? cap + W : W);
+    const uint32_t idx = !GATE ? cap : word * mul < kgs16 ? cap : (RF ? cap + W : W);
     uint32_t a, b;
     asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(a), "=r"(b) : "r"(gtab_s + idx * eb));
     gh += a;

@@ -1015,6 +1015,8 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
             // rebuild the same table): the measurement's algorithmic count
             const int halves = RF ? (any_open ? 1 : 0) + (any_closed ? 1 : 0) : 1;
             if (KC && part == 0) atomicAdd(&set.work[2], (unsigned long long)pl.W * halves);
+            // scenarios that test their tail gate (a stratum on both sides of the SLO)
+            if (KC && part == 0 && any_open && any_closed) atomicAdd(&set.work[3], (unsigned long long)pl.S);
           }
           const int Lp0 = __float_as_int(h0[H_LPAD]), Lp1 = __float_as_int(h1[H_LPAD]);
           const bool r0 = __float_as_int(h0[H_ROW]) != 0, r1 = __float_as_int(h1[H_ROW]) != 0;
@@ -1054,7 +1056,13 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
         return;
       }
       GtabSum gs{0u, 0u, 0ull};
-      if (use) gs = sample_gtab<KC, RF>(pl, keys, o, cell, q_lo, q_hi, smem_u32(gtab), kgs16);
+      if (use) {
+        if (kgs == 0u || kgs16 == 0xFFFFFFFFu)  // the gate is the same at every position
+          gs = sample_gtab<KC, RF, false>(pl, keys, o, cell, q_lo, q_hi,
+                                          smem_u32(gtab) + (RF && kgs == 0u ? 8u * (uint32_t)pl.W : 0u), 0u);
+        else
+          gs = sample_gtab<KC, RF, true>(pl, keys, o, cell, q_lo, q_hi, smem_u32(gtab), kgs16);
+      }
       uint64_t v;
       if (small_gt) {  // at most 64 values per thread: each field's warp sum fits in 32 bits
         const uint32_t H = __reduce_add_sync(0xffffffffu, gs.h);

@@ -111,7 +111,7 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
     off = up256(off + bytes);
     return o;
   };
-  const size_t o_status = take(4), o_work = take(24), o_part = take(16 * (size_t)kFinalizeMaxBlocks);
+  const size_t o_status = take(4), o_work = take(32), o_part = take(16 * (size_t)kFinalizeMaxBlocks);
   const size_t o_qn = quantile_dev ? 0 : take(4 * (size_t)Q);
   const size_t o_theta = take(8 * (size_t)d.theta_cap), o_nth = take(8);
   const size_t o_rowc = take(8 * (size_t)d.K4), o_rowb = take(8 * (size_t)d.K4);

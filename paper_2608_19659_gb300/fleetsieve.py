@@ -115,7 +115,7 @@ def lib():
         L.fs_launch_count.restype = C.c_uint64
         L.fs_timing_enable.argtypes = [C.c_void_p, C.c_int32]
         L.fs_timing_read.argtypes = [C.c_void_p, C.POINTER(C.c_double), C.POINTER(C.c_int32),
-                                     C.c_void_p, C.POINTER(C.c_uint64)]
+                                     C.c_void_p, C.c_void_p]
         L.fs_watchdog_selftest.argtypes = [C.c_int64]
         L.fs_free_model.argtypes = [C.c_void_p]
         L.fs_free_model.restype = None
@@ -446,15 +446,15 @@ def fs_timing_enable(m: Model, mode: int) -> None:
 
 def fs_timing_read(m: Model, with_entries: bool = False):
     """(Monte-Carlo kernel ms, timed calls, [solve, prep, Monte-Carlo, reduction] ms) since the last
-    read; with_entries adds the gap-table entries the Monte-Carlo kernel evaluated since then."""
+    read; with_entries adds the work counts since then: (gap-table entries evaluated, scenarios
+    that tested their tail gate)."""
     ms = C.c_double()
     n = C.c_int32()
     ph = np.zeros(4, np.float64)
-    ent = C.c_uint64()
-    _check(lib().fs_timing_read(m.handle, C.byref(ms), C.byref(n), _vp(ph),
-                                C.byref(ent) if with_entries else None))
+    wc = np.zeros(2, np.uint64)
+    _check(lib().fs_timing_read(m.handle, C.byref(ms), C.byref(n), _vp(ph), _vp(wc) if with_entries else None))
     if with_entries:
-        return float(ms.value), int(n.value), ph, int(ent.value)
+        return float(ms.value), int(n.value), ph, (int(wc[0]), int(wc[1]))
     return float(ms.value), int(n.value), ph
 
 

@@ -364,24 +364,29 @@ def test_models_of_different_sizes_used_alternately(fsb, cuda, oracle_lib, qn):
     assert np.array_equal(again.sum_eo, oracle_lib.score(big, qn).sum_eo)
 
 
-def test_table_entries_counted_by_the_library(fsb, cuda, oracle_lib, qn):
+def test_table_work_counted_by_the_library(fsb, cuda, oracle_lib, qn):
     """The table path evaluates W gap-table entries in each segment whose tail
     gate is open at some position of its stratum, and none where it is closed at
-    every position (all entries are the closed-gate value); the library's count,
-    which the benchmark's algorithmic work uses, must say exactly that."""
+    every position (all entries are the closed-gate value); only the scenarios of
+    strata whose tails lie on both sides of the SLO test their gate. The
+    library's counts, which the benchmark's algorithmic work uses, must say
+    exactly that."""
     w = workloads.make_workload(1)
     W = 4096 // w.O
     lo, hi = w.tail_lo.reshape(-1), w.tail_hi.reshape(-1)
     L = np.repeat(w.slo, 4 * w.B)
-    # the smallest tail value of stratum o is the map of its first quantile
-    open_segments = sum(1 for c in w.candidates for o in range(w.O)
-                        if oracle_lib.map_value(lo[c], hi[c], qn[o * W]) <= L[c])
-    assert 0 < open_segments < len(w.candidates) * w.O
+    # the smallest and largest tail values of stratum o map its first and last quantile
+    first = [[oracle_lib.map_value(lo[c], hi[c], qn[o * W]) <= L[c] for o in range(w.O)] for c in w.candidates]
+    last = [[oracle_lib.map_value(lo[c], hi[c], qn[(o + 1) * W - 1]) <= L[c] for o in range(w.O)]
+            for c in w.candidates]
+    open_segments = sum(f for row in first for f in row)
+    mixed = sum(f and not g for fr, lr in zip(first, last) for f, g in zip(fr, lr))
+    assert 0 < open_segments < len(w.candidates) * w.O and mixed > 0
     with load_model(fsb, w) as m:
         fsb.fs_timing_enable(m, 1)
         r = fsb.fs_score_candidates(m, w.candidates, w.O, w.S, w.seed)
         r = fsb.fs_score_candidates(m, w.candidates, w.O, w.S, w.seed)
-        _, n, _, entries = fsb.fs_timing_read(m, with_entries=True)
-        assert n == 2 and entries == 2 * open_segments * W
-        assert fsb.fs_timing_read(m, with_entries=True)[3] == 0
+        _, n, _, (entries, gated) = fsb.fs_timing_read(m, with_entries=True)
+        assert n == 2 and entries == 2 * open_segments * W and gated == 2 * mixed * w.S
+        assert fsb.fs_timing_read(m, with_entries=True)[3] == (0, 0)
     assert np.array_equal(r.sum_eo, oracle_lib.score(w, qn).sum_eo)

@@ -63,7 +63,7 @@ def _scratch_bytes(K, G, O, Q, n, builtin_table=True):
     W = Q // O
     I = 2 * (20 + 3 * P) + O * (4 + 4 * ((W + 3) // 4))
     n = max(n, 1)
-    parts = [4, 24, 1024] + ([4 * Q] if builtin_table else []) + [8 * T, 8, 32 * K, 32 * K, 1216, 65536,
+    parts = [4, 32, 1024] + ([4 * Q] if builtin_table else []) + [8 * T, 8, 32 * K, 32 * K, 1216, 65536,
                                                                    4 * n * I, 8 * n * O]
     return sum(up(p) for p in parts)
 
