@@ -114,6 +114,11 @@ def lib():
                                           C.c_uint32, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int,
                                           ip, ip, ip, C.POINTER(C.c_double), ip,
                                           C.POINTER(_Alloc), fp]
+        _lib.or_replay_stream_cached.argtypes = [C.POINTER(_Problem), fp, fp, fp, fp, fp, fp, ip,
+                                          C.c_int, C.c_float, fp, C.c_int, C.c_uint64,
+                                          C.c_uint32, C.c_int, C.c_int, C.c_int, C.c_int, C.c_int,
+                                          ip, ip, ip, C.POINTER(C.c_double), ip,
+                                          C.POINTER(_Alloc), fp]
     return _lib
 
 
@@ -453,10 +458,11 @@ class ReplayResult:
 
 
 def replay_stream(rp, k: int, qn, seed: int, S=None, O=None, max_rounds=None,
-                  solver=SOLVER_FRONTIER, policy: int = 0, perm=None) -> ReplayResult:
+                  solver=SOLVER_FRONTIER, policy: int = 0, perm=None, cached: bool = False) -> ReplayResult:
     """Algorithm 1 on stream k of the replay ``rp``. policy 0: reveal the
     best-scored cell; 1: the next unrevealed cell of ``perm`` (default: the
-    stream's own permutation)."""
+    stream's own permutation). cached: each round scored by the cached scorer
+    (the same sums and argmax)."""
     w = rp.base
     prob = Problem.of(w)
     b = _bounds(w)
@@ -471,7 +477,8 @@ def replay_stream(rp, k: int, qn, seed: int, S=None, O=None, max_rounds=None,
     rounds, nrev, st = C.c_int32(), C.c_int32(), C.c_int32()
     gs = C.c_double()
     am = _Alloc()
-    rc = lib().or_replay_stream(C.byref(prob._s), *[_ptr(x, C.c_float) for x in b],
+    fn = lib().or_replay_stream_cached if cached else lib().or_replay_stream
+    rc = fn(C.byref(prob._s), *[_ptr(x, C.c_float) for x in b],
                                 _ptr(tc, C.c_float), _ptr(tl, C.c_float), _ptr(perm, C.c_int32),
                                 rp.r0, rp.eps, _ptr(qn, C.c_float), qn.size, seed, k,
                                 w.O if O is None else O, w.S if S is None else S, mr, solver, policy,

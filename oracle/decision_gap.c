@@ -313,6 +313,15 @@ int or_certificate(const or_problem *p, const float *cap_lo, const float *cap_hi
  * random permutation, fixed grid order when it lists the grid), stopped by
  * the same certificate.
  */
+static int replay_impl(const or_problem *p, const float *prior_cap_lo, const float *prior_cap_hi,
+                       const float *prior_tail_lo, const float *prior_tail_hi,
+                       const float *truth_cap, const float *truth_tail, const int32_t *perm,
+                       int r0, float eps, const float *qn, int Q, uint64_t seed,
+                       uint32_t stream_id, int O, int S, int max_rounds, int solver, int policy,
+                       int cached, int32_t *rounds, int32_t *reveal_order, int32_t *n_revealed,
+                       double *gpu_seconds, int32_t *state, or_alloc *final_minus,
+                       float *gamma_trace);
+
 int or_replay_stream(const or_problem *p, const float *prior_cap_lo, const float *prior_cap_hi,
                      const float *prior_tail_lo, const float *prior_tail_hi,
                      const float *truth_cap, const float *truth_tail, const int32_t *perm,
@@ -321,6 +330,36 @@ int or_replay_stream(const or_problem *p, const float *prior_cap_lo, const float
                      int32_t *rounds, int32_t *reveal_order, int32_t *n_revealed,
                      double *gpu_seconds, int32_t *state, or_alloc *final_minus,
                      float *gamma_trace)
+{
+    return replay_impl(p, prior_cap_lo, prior_cap_hi, prior_tail_lo, prior_tail_hi, truth_cap, truth_tail,
+                       perm, r0, eps, qn, Q, seed, stream_id, O, S, max_rounds, solver, policy, 0, rounds,
+                       reveal_order, n_revealed, gpu_seconds, state, final_minus, gamma_trace);
+}
+
+/* The same replay with each round's scores from or_score_cached + or_reduce
+ * (the same sums and argmax, fewer solves); the tests hold the two equal. */
+int or_replay_stream_cached(const or_problem *p, const float *prior_cap_lo, const float *prior_cap_hi,
+                            const float *prior_tail_lo, const float *prior_tail_hi,
+                            const float *truth_cap, const float *truth_tail, const int32_t *perm,
+                            int r0, float eps, const float *qn, int Q, uint64_t seed,
+                            uint32_t stream_id, int O, int S, int max_rounds, int solver, int policy,
+                            int32_t *rounds, int32_t *reveal_order, int32_t *n_revealed,
+                            double *gpu_seconds, int32_t *state, or_alloc *final_minus,
+                            float *gamma_trace)
+{
+    return replay_impl(p, prior_cap_lo, prior_cap_hi, prior_tail_lo, prior_tail_hi, truth_cap, truth_tail,
+                       perm, r0, eps, qn, Q, seed, stream_id, O, S, max_rounds, solver, policy, 1, rounds,
+                       reveal_order, n_revealed, gpu_seconds, state, final_minus, gamma_trace);
+}
+
+static int replay_impl(const or_problem *p, const float *prior_cap_lo, const float *prior_cap_hi,
+                       const float *prior_tail_lo, const float *prior_tail_hi,
+                       const float *truth_cap, const float *truth_tail, const int32_t *perm,
+                       int r0, float eps, const float *qn, int Q, uint64_t seed,
+                       uint32_t stream_id, int O, int S, int max_rounds, int solver, int policy,
+                       int cached, int32_t *rounds, int32_t *reveal_order, int32_t *n_revealed,
+                       double *gpu_seconds, int32_t *state, or_alloc *final_minus,
+                       float *gamma_trace)
 {
     int cells = cells_of(p);
     if (r0 < 0 || r0 > cells || policy < 0 || policy > 1) return -1;
@@ -355,10 +394,19 @@ int or_replay_stream(const or_problem *p, const float *prior_cap_lo, const float
             if (!rev[perm[q]]) cand[nc++] = perm[q];
         if (nc == 0 || r >= max_rounds) { st = 0; break; }
         int32_t bestc = cand[0];
-        if (policy == 0) {
+        if (policy == 0 && !cached) {
             float g2;
             rc = or_score(p, clo, chi, tlo, thi, qn, Q, seed, stream_id, (uint32_t)r, nc, cand, O, S,
                           solver, NULL, NULL, NULL, NULL, &g2, &bestc, NULL);
+            if (rc) break;
+        } else if (policy == 0) {
+            float g2;
+            int64_t *se = (int64_t *)malloc(sizeof(int64_t) * (size_t)nc * O);
+            if (!se) { rc = -2; break; }
+            rc = or_score_cached(p, clo, chi, tlo, thi, qn, Q, seed, stream_id, (uint32_t)r, nc, cand, O, S,
+                                 solver, se, &g2);
+            if (!rc) rc = or_reduce(p, nc, cand, O, S, g2, se, NULL, NULL, NULL, &bestc);
+            free(se);
             if (rc) break;
         }
         or_refit(p, p->prior, bestc, truth_cap[bestc], truth_tail[bestc], clo, chi, tlo, thi);

@@ -164,4 +164,14 @@ int or_replay_stream(const or_problem *p, const float *prior_cap_lo, const float
                      double *gpu_seconds, int32_t *state, or_alloc *final_minus,
                      float *gamma_trace);
 
+/* The same replay with each round scored by or_score_cached + or_reduce. */
+int or_replay_stream_cached(const or_problem *p, const float *prior_cap_lo, const float *prior_cap_hi,
+                            const float *prior_tail_lo, const float *prior_tail_hi,
+                            const float *truth_cap, const float *truth_tail, const int32_t *perm,
+                            int r0, float eps, const float *qn, int Q, uint64_t seed,
+                            uint32_t stream_id, int O, int S, int max_rounds, int solver, int policy,
+                            int32_t *rounds, int32_t *reveal_order, int32_t *n_revealed,
+                            double *gpu_seconds, int32_t *state, or_alloc *final_minus,
+                            float *gamma_trace);
+
 #endif

@@ -14,9 +14,21 @@
 #include <string>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "fs_internal.cuh"
 
 namespace fs {
+
+// An NVTX range over one call of the boundary (load, base solves, scoring,
+// reveal, replay), for timeline tools; with no tool attached a push and a pop
+// are two calls through a null handler.
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
 
 static std::atomic<uint64_t> g_launches{0};
 void note_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
@@ -384,6 +396,7 @@ int32_t fs_dump_stride(const fs_model* m) {
 
 int fs_load_model(const fs_bounds* b, const float* slo, const float* demand, int32_t G, void* cuda_stream,
                   fs_model** out) {
+  NvtxRange nvtx_range("fs_load_model");
   if (!out) return fail(FS_EINVAL, "out is NULL");
   if (!b) return fail(FS_EINVAL, "bounds is NULL");
   if (b->K < 1 || b->K > FS_MAX_CLASSES) return fail(FS_EINVAL, "K = %d outside [1, %d]", b->K, FS_MAX_CLASSES);
@@ -505,6 +518,7 @@ int fs_load_model(const fs_bounds* b, const float* slo, const float* demand, int
 
 int fs_update_bounds(fs_model* m, const float* cap_lo, const float* cap_hi, const float* tail_lo,
                      const float* tail_hi) {
+  NvtxRange nvtx_range("fs_update_bounds");
   if (!m) return fail(FS_EINVAL, "model is NULL");
   const int cells = m->d.cells;
   int rc = check_bounds4(cap_lo, cap_hi, tail_lo, tail_hi, cells);
@@ -516,6 +530,7 @@ int fs_update_bounds(fs_model* m, const float* cap_lo, const float* cap_hi, cons
 }
 
 int fs_set_floors(fs_model* m, const float* floor) {
+  NvtxRange nvtx_range("fs_set_floors");
   if (!m) return fail(FS_EINVAL, "model is NULL");
   const int K = m->d.K;
   std::vector<float> v(K, 0.0f);
@@ -537,6 +552,7 @@ int fs_set_floors(fs_model* m, const float* floor) {
 
 int fs_score_candidates(fs_model* m, const fs_samples* smp, double* gap_out, double* score_out, float* gamma_t,
                         int32_t* best, int64_t* sum_eo, void* dump_dev) {
+  NvtxRange nvtx_range("fs_score_candidates");
   if (!m) return fail(FS_EINVAL, "model is NULL");
   int rc = check_samples(m, smp, true);
   if (rc) return rc;
@@ -581,6 +597,7 @@ int fs_score_candidates(fs_model* m, const fs_samples* smp, double* gap_out, dou
 int fs_score_candidates_async(fs_model* m, const fs_samples* smp, double* gap_dev, double* score_dev,
                               float* gamma_t_dev, int32_t* best_dev, int64_t* sum_eo_dev, void* dump_dev,
                               void* cuda_stream) {
+  NvtxRange nvtx_range("fs_score_candidates_async");
   if (!m) return fail(FS_EINVAL, "model is NULL");
   int rc = check_samples(m, smp, false);
   if (rc) return rc;
@@ -597,6 +614,7 @@ int fs_score_candidates_async(fs_model* m, const fs_samples* smp, double* gap_de
 }
 
 int fs_solve(fs_model* m, const float* cap, const float* tail, fs_allocation* out) {
+  NvtxRange nvtx_range("fs_solve");
   if (!m) return fail(FS_EINVAL, "model is NULL");
   if (!out) return fail(FS_EINVAL, "out is NULL");
   const int cells = m->d.cells;
@@ -617,6 +635,7 @@ int fs_solve(fs_model* m, const float* cap, const float* tail, fs_allocation* ou
 
 int fs_solve_batch(fs_model* m, int32_t n, const float* cap_dev, const float* tail_dev, fs_allocation* out_dev,
                    void* cuda_stream) {
+  NvtxRange nvtx_range("fs_solve_batch");
   if (!m) return fail(FS_EINVAL, "model is NULL");
   if (n < 0) return fail(FS_EINVAL, "n < 0");
   if (n == 0) return FS_OK;
@@ -629,6 +648,7 @@ int fs_solve_batch(fs_model* m, int32_t n, const float* cap_dev, const float* ta
 }
 
 int fs_solve_bounds(fs_model* m, fs_allocation* minus, fs_allocation* plus, float* gamma_t) {
+  NvtxRange nvtx_range("fs_solve_bounds");
   if (!m) return fail(FS_EINVAL, "model is NULL");
   cudaStream_t s = m->stream;
   int rc0 = flush_bounds(m, s);
@@ -646,6 +666,7 @@ int fs_solve_bounds(fs_model* m, fs_allocation* minus, fs_allocation* plus, floa
 }
 
 int fs_reveal(fs_model* m, int32_t cell, float cap, float tail) {
+  NvtxRange nvtx_range("fs_reveal");
   if (!m) return fail(FS_EINVAL, "model is NULL");
   if (cell < 0 || cell >= m->d.cells) return fail(FS_EINVAL, "cell %d out of range", cell);
   if (!std::isfinite(cap) || cap < 0.0f || !std::isfinite(tail) || tail < 0.0f)
@@ -674,6 +695,7 @@ int fs_get_state(const fs_model* m, float* cap_lo, float* cap_hi, float* tail_lo
 }
 
 int fs_certificate(fs_model* m, float eps, int32_t* state, float* gamma_t) {
+  NvtxRange nvtx_range("fs_certificate");
   if (!m) return fail(FS_EINVAL, "model is NULL");
   if (!state) return fail(FS_EINVAL, "state is NULL");
   if (std::isnan(eps)) return fail(FS_EINVAL, "eps is NaN");
@@ -711,6 +733,7 @@ int fs_set_objective(fs_model* m, int32_t objective) {
 
 int fs_score_goodput(fs_model* m, const fs_samples* smp, double* gap_out, double* score_out, double* gamma_gp,
                      int32_t* best, int64_t* sum_eo) {
+  NvtxRange nvtx_range("fs_score_goodput");
   if (!m) return fail(FS_EINVAL, "model is NULL");
   int rc = check_samples(m, smp, true);
   if (rc) return rc;
@@ -759,6 +782,7 @@ int fs_score_goodput(fs_model* m, const fs_samples* smp, double* gap_out, double
 
 int fs_replay(fs_model* m, const fs_replay_spec* sp, int32_t* rounds, int32_t* state, double* gpu_seconds,
               int32_t* reveal_order, float* gamma_trace, fs_allocation* final_minus) {
+  NvtxRange nvtx_range("fs_replay");
   if (!m) return fail(FS_EINVAL, "model is NULL");
   if (!sp) return fail(FS_EINVAL, "spec is NULL");
   const Dims d = m->d;

@@ -31,9 +31,10 @@ __device__ __forceinline__ float row_cap(const RowCap& r, float cy, bool g) {
 // round keys read from the plan. GATE = false: the stratum's tail gate is the
 // same at every position (its mapped tails all pass the SLO, or none does;
 // known from the preparation's gate position), so the entry is the capacity
-// position's in the table at gtab_s (the open half, or under the prior the
-// closed half; without the prior a closed stratum's table holds the
-// closed-gate value at every position) and no scenario tests the gate.
+// position's in the table at gtab_s with a stride of `stride` bytes (the open
+// half, or under the prior the closed half; without the prior a closed
+// stratum's entries are all the closed-gate value, stored once: stride 0, so
+// a warp's loads are one broadcast) and no scenario tests the gate.
 struct GtabSum {
   uint32_t h, l;   // the last at most 1024 values
   uint64_t total;  // earlier values
@@ -48,10 +49,10 @@ __device__ __forceinline__ uint4 draw_call(const Plan& pl, const PhiloxKeys& key
 
 template <bool KC, bool RF, bool GATE = true>
 __device__ __forceinline__ GtabSum sample_gtab(const Plan& pl, const PhiloxKeys& keys, int o, int cell, int q_lo,
-                                               int q_hi, uint32_t gtab_s, uint32_t kgs16) {
+                                               int q_hi, uint32_t gtab_s, uint32_t kgs16, uint32_t stride = 8u) {
   const uint32_t ctr1 = (uint32_t)o, ctr2 = (uint32_t)cell, ctr3 = pl.round;
   const uint32_t W = (uint32_t)pl.W;
-  const uint32_t mul = pl.lo16_mul, eb = pl.entry_bytes;
+  const uint32_t mul = pl.lo16_mul, eb = GATE ? pl.entry_bytes : stride;
   uint32_t gh = 0, glo = 0;
   auto take = [&](uint32_t word) {
     const uint32_t cap = __umulhi(word, W);

@@ -1006,8 +1006,9 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
         const bool any_open = kgs != 0u, any_closed = kgs16 != 0xFFFFFFFFu;
         if (!RF && kgs == 0u) {
           // the gate is closed at every position of the stratum: every entry
-          // is the closed-gate value (each scenario still draws its position)
-          for (int k = tid; k <= pl.W; k += blockDim.x) gtab[k] = closed;
+          // is the closed-gate value, stored once at W (each scenario still
+          // draws its position and loads its entry, with stride 0)
+          if (tid == 0) gtab[pl.W] = closed;
         } else {
           if (tid == 0) {
             if (!RF) gtab[pl.W] = closed;
@@ -1059,7 +1060,8 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
       if (use) {
         if (kgs == 0u || kgs16 == 0xFFFFFFFFu)  // the gate is the same at every position
           gs = sample_gtab<KC, RF, false>(pl, keys, o, cell, q_lo, q_hi,
-                                          smem_u32(gtab) + (RF && kgs == 0u ? 8u * (uint32_t)pl.W : 0u), 0u);
+                                          smem_u32(gtab) + (kgs == 0u ? 8u * (uint32_t)pl.W : 0u), 0u,
+                                          (!RF && kgs == 0u) ? 0u : pl.entry_bytes);
         else
           gs = sample_gtab<KC, RF, true>(pl, keys, o, cell, q_lo, q_hi, smem_u32(gtab), kgs16);
       }

@@ -11,12 +11,18 @@ within SLO) pairs. Candidates are split into contiguous ranges, one
 single-threaded oracle process per range; the sums do not depend on the split.
 
 Usage: python tests/golden/make_expected_sums.py [--procs N] [name ...]
-with names from WORKLOADS below (default: all). Each file records:
+with names from WORKLOADS below and "replay" (default: all). Each sums file records:
   * the sha256 of the workload's inputs (bounds, demands, SLOs, candidates),
   * Gamma_t and the argmax cell,
   * per candidate the deficits d[e][o] = S rint(Gamma_t 2^40) - sum_eo[e][o]
     (the fixed-point score of each outcome stratum; 0 for a candidate that
     cannot change either allocation), so that sum_eo = S rint(Gamma_t 2^40) - d.
+
+"replay" writes the replay workload (Algorithm 1 over 200 reveal orders of
+the paper-scale grid, 8 x 4096 samples per candidate and round, seed 2026):
+per stream its rounds, final certificate state, GPU-seconds, reveal order and
+Gamma_t trace, from the oracle's replay with each round scored by the cached
+scorer (held equal to the plain one by the tests).
 """
 
 from __future__ import annotations
@@ -108,13 +114,66 @@ def write(name, w, sums, res):
             f.write(f"{int(cell)} " + " ".join(str(int(x)) for x in d[e]) + "\n")
 
 
+REPLAY_FILE = "replay_200_streams.txt"
+REPLAY_SEED = 2026
+
+
+def _replay_stream(k):
+    import oracle
+    from paper_2608_19659_gb300 import workloads
+
+    rp = workloads.make_replay()
+    qn = oracle.triangular_table(4096)
+    r = oracle.replay_stream(rp, k, qn, seed=REPLAY_SEED, cached=True)
+    return k, r
+
+
+def replay_digest(rp) -> str:
+    h = hashlib.sha256()
+    h.update(input_digest(rp.base).encode())
+    for a in (rp.truth_cap, rp.truth_tail):
+        h.update(np.ascontiguousarray(a, np.float32).tobytes())
+    h.update(np.ascontiguousarray(rp.perm, np.int32).tobytes())
+    h.update(np.array([rp.r0, rp.max_rounds], np.int64).tobytes())
+    h.update(np.float32(rp.eps).tobytes())
+    return h.hexdigest()
+
+
+def write_replay(procs):
+    from paper_2608_19659_gb300 import workloads
+
+    rp = workloads.make_replay()
+    n = len(rp.perm)
+    res = [None] * n
+    with mp.get_context("spawn").Pool(procs) as pool:
+        for k, r in pool.imap_unordered(_replay_stream, range(n)):
+            res[k] = r
+    with open(os.path.join(HERE, REPLAY_FILE), "w") as f:
+        f.write("# Expected replay of the oracle: Algorithm 1 on 200 reveal orders of the paper-scale grid\n")
+        f.write(f"# {rp.base.O} outcomes x {rp.base.S} samples per candidate and round, eps {rp.eps}, "
+                f"seed {REPLAY_SEED}, stream k = Philox stream id k\n")
+        f.write("# written by tests/golden/make_expected_sums.py replay (oracle/ only)\n")
+        f.write(f"# inputs_sha256 {replay_digest(rp)}\n")
+        f.write("# per stream: k rounds state gpu_seconds | reveal order | Gamma_t trace (float32 bits)\n")
+        for k, r in enumerate(res):
+            trace = " ".join(f"{np.float32(x).view(np.uint32):08x}" for x in r.gamma_trace)
+            order = " ".join(str(int(c)) for c in r.reveal_order)
+            f.write(f"{k} {r.rounds} {r.state} {r.gpu_seconds!r} | {order} | {trace}\n")
+    return res
+
+
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("names", nargs="*", default=list(WORKLOADS))
+    ap.add_argument("names", nargs="*", default=list(WORKLOADS) + ["replay"])
     ap.add_argument("--procs", type=int, default=len(os.sched_getaffinity(0)))
     a = ap.parse_args()
     for name in a.names:
         t0 = time.time()
+        if name == "replay":
+            res = write_replay(a.procs)
+            print(f"replay: {len(res)} streams, {sum(r.rounds for r in res)} rounds, "
+                  f"{time.time() - t0:.0f} s on {a.procs} processes")
+            continue
         w, sums, res = compute(name, a.procs)
         write(name, w, sums, res)
         print(f"{name}: {len(w.candidates)} candidates, Gamma_t {res.gamma_t}, best {res.best}, "
