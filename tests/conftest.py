@@ -102,3 +102,23 @@ def read_expected_sums(name):
                 deficits.append([int(x) for x in t[1:]])
     full = np.int64(S) * np.int64(np.rint(np.float64(np.float32(gamma_t)) * 2.0**40))
     return sha, gamma_t, best, np.array(cells, np.int32), full - np.array(deficits, np.int64)
+
+
+def read_expected_replay():
+    """The expected replay file written by tests/golden/make_expected_sums.py:
+    (inputs_sha256, {stream: (rounds, state, gpu_seconds, reveal order, Gamma_t trace)})."""
+    import numpy as np
+
+    sha, out = None, {}
+    with open(os.path.join(GOLDEN, "replay_200_streams.txt")) as f:
+        for line in f:
+            if line.startswith("# inputs_sha256"):
+                sha = line.split()[2]
+                continue
+            if not line.strip() or line.startswith("#"):
+                continue
+            head, order, trace = line.split("|")
+            k, rounds, state, gs = head.split()
+            out[int(k)] = (int(rounds), int(state), float(gs), np.array([int(x) for x in order.split()], np.int32),
+                           np.array([int(x, 16) for x in trace.split()], np.uint32).view(np.float32))
+    return sha, out

@@ -58,13 +58,27 @@ def test_replay_round_cap_and_full_initial_design(fsb, cuda, oracle_lib, qn):
 
 
 def test_replay_full_size(fsb, cuda, oracle_lib, qn):
-    """200 reveal orders x (unrevealed x 8 x 4096) per round; stream 0 replayed by the oracle in full."""
+    """The replay workload in full: 200 reveal orders x (unrevealed x 8 x 4096)
+    per round; every stream's rounds, state, GPU-seconds, reveal order and
+    Gamma_t trace equal the oracle's stored replay (tests/golden, oracle only),
+    and stream 0 is also replayed by the oracle here."""
+    import sys
+
+    from conftest import GOLDEN, read_expected_replay
+
+    sys.path.insert(0, GOLDEN)
+    import make_expected_sums as mes
+
     rp = workloads.make_replay()
-    res = _gpu_replay(fsb, rp, S=4096, seed=2026)
+    sha, exp = read_expected_replay()
+    assert sha == mes.replay_digest(rp)
+    res = _gpu_replay(fsb, rp, S=4096, seed=mes.REPLAY_SEED)
     assert np.all(res.state == 1)
     for k in range(200):
-        tr = res.gamma_trace[k][: res.rounds[k] + 1]
-        assert np.all(np.diff(tr) <= 0) and tr[-1] <= rp.eps
+        rounds, state, gs, order, trace = exp[k]
+        assert res.rounds[k] == rounds and res.state[k] == state and res.gpu_seconds[k] == gs, k
+        assert np.array_equal(res.reveal_order[k][: len(order)], order) and np.all(res.reveal_order[k][len(order):] == -1)
+        assert np.array_equal(res.gamma_trace[k][: rounds + 1], trace), k
     ref = oracle_lib.replay_stream(rp, 0, qn, seed=2026, S=4096)
     _compare(fsb, res, rp, 0, ref, rp.base.K)
 

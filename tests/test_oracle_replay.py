@@ -58,3 +58,41 @@ def test_replay_round_cap(oracle_lib, replay):
     never = dataclasses.replace(replay, eps=-1.0)
     r = oracle_lib.replay_stream(never, 1, qn, seed=1, S=8, max_rounds=3)
     assert r.rounds == 3 and r.state == 0
+
+
+@pytest.mark.parametrize("k", [0, 2, 7, 13])
+def test_cached_replay_equals_plain(oracle_lib, k):
+    """The replay scored by the cached scorer reveals the same cells in the same
+    rounds with the same traces as the one scored scenario by scenario."""
+    rp = workloads.make_replay(n_streams=16)
+    qn = oracle_lib.triangular_table(4096)
+    a = oracle_lib.replay_stream(rp, k, qn, seed=2026, S=96)
+    b = oracle_lib.replay_stream(rp, k, qn, seed=2026, S=96, cached=True)
+    assert (a.rounds, a.state, a.gpu_seconds) == (b.rounds, b.state, b.gpu_seconds)
+    assert np.array_equal(a.reveal_order, b.reveal_order) and np.array_equal(a.gamma_trace, b.gamma_trace)
+
+
+def test_expected_replay_file(oracle_lib):
+    """The stored replay of all 200 reveal orders: the generator's inputs today,
+    every stream certified, traces nonincreasing to at most eps, and two streams
+    recomputed by the oracle."""
+    import sys
+
+    from conftest import GOLDEN, read_expected_replay
+
+    sys.path.insert(0, GOLDEN)
+    import make_expected_sums as mes
+
+    rp = workloads.make_replay()
+    sha, exp = read_expected_replay()
+    assert sha == mes.replay_digest(rp) and sorted(exp) == list(range(200))
+    for k, (rounds, state, gs, order, trace) in exp.items():
+        assert state == 1 and len(trace) == rounds + 1 and trace[-1] <= rp.eps
+        assert len(order) == rp.r0 + rounds and np.all(np.diff(trace) <= 0)
+    qn = oracle_lib.triangular_table(4096)
+    short = [k for k in range(200) if exp[k][0] <= 2][:2]
+    for k in short:
+        r = oracle_lib.replay_stream(rp, k, qn, seed=mes.REPLAY_SEED, cached=True)
+        rounds, state, gs, order, trace = exp[k]
+        assert (r.rounds, r.state, r.gpu_seconds) == (rounds, state, gs)
+        assert np.array_equal(r.reveal_order, order) and np.array_equal(r.gamma_trace, trace)
