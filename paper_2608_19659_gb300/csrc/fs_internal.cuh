@@ -162,6 +162,10 @@ struct Plan {
   // so that a word's low half moved to the top and an entry's byte offset are
   // integer multiply-adds (FMA pipe) rather than shifts and masks (ALU pipe)
   uint32_t lo16_mul, entry_bytes;
+  // 0: the entry stride of a table whose entries are all equal (stored once).
+  // A parameter like the others: every scenario still computes its position
+  // and its entry's address, and the kernel is not specialised for that table
+  uint32_t uniform_stride;
 };
 
 // Round keys of problem 0 for the plan (host).
@@ -175,6 +179,7 @@ inline void plan_round_keys(Plan& pl) {
   }
   pl.lo16_mul = 65536u;
   pl.entry_bytes = 8u;
+  pl.uniform_stride = 0u;
 }
 
 struct Items {
@@ -396,20 +401,30 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
 
 // Bounded wait for phase `parity` of bar: true when it completed, false when
 // limit_ns elapsed (or an iteration cap was hit) first.
+__device__ __forceinline__ bool mbar_try(uint32_t a, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(a), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
   const uint32_t a = smem_u32(bar);
+  if (mbar_try(a, parity)) return true;  // the common case: no clock read
   const uint64_t t0 = global_ns();
   for (uint32_t it = 0; it < (1u << 28); ++it) {
-    uint32_t ok;
-    asm volatile(
-        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
-        : "=r"(ok)
-        : "r"(a), "r"(parity)
-        : "memory");
-    if (ok) return true;
+    if (mbar_try(a, parity)) return true;
     if ((it & 15u) == 15u && global_ns() - t0 > limit_ns) return false;
   }
   return false;
+}
+
+// Plain arrival (no transaction bytes) on bar.
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
 
 constexpr uint64_t kWaitLimitNs = 2000000000ull;  // 2 s

@@ -1061,7 +1061,7 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
         if (kgs == 0u || kgs16 == 0xFFFFFFFFu)  // the gate is the same at every position
           gs = sample_gtab<KC, RF, false>(pl, keys, o, cell, q_lo, q_hi,
                                           smem_u32(gtab) + (kgs == 0u ? 8u * (uint32_t)pl.W : 0u), 0u,
-                                          (!RF && kgs == 0u) ? 0u : pl.entry_bytes);
+                                          (!RF && kgs == 0u) ? pl.uniform_stride : pl.entry_bytes);
         else
           gs = sample_gtab<KC, RF, true>(pl, keys, o, cell, q_lo, q_hi, smem_u32(gtab), kgs16);
       }
@@ -1233,10 +1233,11 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
   auto kern = mode == 0 ? FS_KERN(false, false) : mode == 1 ? FS_KERN(true, false)
             : mode == 2 ? FS_KERN(false, true) : FS_KERN(true, true);
 #undef FS_KERN
+  const void* kfun = reinterpret_cast<const void*>(kern);
   if (smem != lc.score_smem[v][mode]) {
     int per_sm = 0;
-    cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(kern), smem);
-    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kScoreThreads, smem);
+    cudaError_t e = raise_smem_limit(kfun, smem);
+    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kfun, kScoreThreads, smem);
     if (e != cudaSuccess) return e;
     lc.score_smem[v][mode] = smem;
     lc.score_blocks_per_sm[v][mode] = per_sm < 1 ? 1 : per_sm;
