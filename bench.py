@@ -45,7 +45,7 @@ ISSUE_PER_SM_CLK = 4 * 32  # 4 schedulers x 32 lanes, one warp instruction each 
 # scenario (the parametric re-solve):
 #   a quarter of one Philox4x32-10 call (10 rounds x (2 wide multiplies +
 #   2 three-input XORs), four samples per call)                          10
-#   capacity position (high multiply), its address, the lookup            3
+#   capacity position (the word's top w bits), its address, the lookup    3
 #   tail gate (mask, compare) and the gated capacity                      3
 #   the two patched row capacities (max with Cexcl)                       2
 #   two table searches: loop test, address, read of the reached threshold 6

@@ -23,7 +23,8 @@ __device__ __forceinline__ float row_cap(const RowCap& r, float cy, bool g) {
 // two fields of the drawn entries (each field below 2^21), flushed into a
 // 64-bit total every 256 calls so that the 32-bit sums cannot wrap. With at
 // most 32 values per thread nothing is flushed and a warp's field sums stay
-// below 2^32. Per sample: the capacity position umulhi(word, W); the tail gate,
+// below 2^32. Per sample: the capacity position floor(word W / 2^32), the
+// word's top w bits for W = 2^w; the tail gate,
 // (word & 0xFFFF) < kgs, as (word * 65536 mod 2^32) < kgs16 with kgs16 =
 // min(kgs 2^16, 2^32 - 1) (a multiply-add and a compare); the entry's shared
 // address base + index * 8 (a multiply-add); its load and two field sums. Two
@@ -51,11 +52,14 @@ template <bool KC, bool RF, bool GATE = true>
 __device__ __forceinline__ GtabSum sample_gtab(const Plan& pl, const PhiloxKeys& keys, int o, int cell, int q_lo,
                                                int q_hi, uint32_t gtab_s, uint32_t kgs16, uint32_t stride = 8u) {
   const uint32_t ctr1 = (uint32_t)o, ctr2 = (uint32_t)cell, ctr3 = pl.round;
-  const uint32_t W = (uint32_t)pl.W;
+  const uint32_t W = (uint32_t)pl.W, w = (uint32_t)pl.w;
   const uint32_t mul = pl.lo16_mul, eb = GATE ? pl.entry_bytes : stride;
   uint32_t gh = 0, glo = 0;
   auto take = [&](uint32_t word) {
-    const uint32_t cap = __umulhi(word, W);
+    // capacity position floor(word W / 2^32): W = 2^w, so the word's top w
+    // bits, taken by a funnel shift (0 for w = 0) on the shift unit rather
+    // than the integer multiplier, which the Philox rounds keep busy
+    const uint32_t cap = __funnelshift_lc(word, 0u, w);
     const uint32_t idx = !GATE ? cap : word * mul < kgs16 ? cap : (RF ? cap + W : W);
     uint32_t a, b;
     asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(a), "=r"(b) : "r"(gtab_s + idx * eb));

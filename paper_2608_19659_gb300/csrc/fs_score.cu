@@ -675,7 +675,7 @@ __device__ void dump_choices(float t, const Set& set, size_t ps, int rr, float C
 // each). win is the staged window of the outcome (gate position, then the
 // mapped capacities); h0/h1 point at the staged table headers; kap/thx/mnx at
 // the table arrays (shared memory when TS, else global). The capacity
-// position is umulhi(word, W) (the top w bits); the tail gate of Eq. 5
+// position is floor(word W / 2^32) (the top w bits); the tail gate of Eq. 5
 // (l_y <= L_i), a position test kl < kgate, is the lower half compared with
 // kgate << (16 - w). With capacities >= 0, max(Cexcl, gate ? c_y : 0) is the
 // patched row capacity.
@@ -695,13 +695,13 @@ __device__ __forceinline__ PieceSum run_piece(const Plan& pl, const PhiloxKeys& 
   const float lam = h0[H_LAM], rlam = h0[H_RLAM], dl = h0[H_DLT];
   const int cell = __float_as_int(h0[H_CELL]);
   const uint32_t ctr1 = (uint32_t)o, ctr2 = (uint32_t)cell, ctr3 = pl.round;
-  const uint32_t W = (uint32_t)pl.W;
+  const uint32_t w = (uint32_t)pl.w;  // W = 2^w positions
   const uint32_t kgs = (uint32_t)__float_as_int(win[0]) << pl.sh;
   const float* sQo = win + 4;
   Acc40 acc;
   uint64_t total = 0;
   auto eval = [&](uint32_t word) {
-    const float cy = sQo[__umulhi(word, W)];
+    const float cy = sQo[__funnelshift_lc(word, 0u, w)];  // floor(word W / 2^32)
     const bool g = (word & 0xFFFFu) < kgs;
     const float cyg = g ? cy : 0.0f;
     const float c0 = RF ? row_cap(rc0, cy, g) : fmaxf(cx0, cyg);
