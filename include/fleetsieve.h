@@ -359,8 +359,10 @@ int fs_set_objective(fs_model *m, int32_t objective);
  *   gamma_gp[1]       Gamma_gp,t / sum_i lambda_i
  *   best[1]           argmax: largest score, then lower TP, then earlier in cand
  *   sum_eo[n_cand*O]  the int64 sums
- * Needs sum_i lambda_i <= 2^20 req/s, G <= 1024 and (K + 1)(G + 1) <= 4 Mi
- * (FS_EINVAL otherwise). Synchronous. Independent of fs_set_objective.
+ * Needs sum_i lambda_i <= 2^20 req/s, G <= 1024, (K + 1)(G + 1) <= 4 Mi and
+ * Q / O <= 4096 (2048 under the monotone prior: a segment's table of
+ * positions lives in shared memory) (FS_EINVAL otherwise). Synchronous.
+ * Independent of fs_set_objective.
  */
 int fs_score_goodput(fs_model *m, const fs_samples *samples, double *gap_out, double *score_out,
                      double *gamma_gp, int32_t *best, int64_t *sum_eo);

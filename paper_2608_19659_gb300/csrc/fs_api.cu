@@ -757,6 +757,8 @@ int fs_score_goodput(fs_model* m, const fs_samples* smp, double* gap_out, double
   it.n = n;
   it.cell = d_cand;
   const Plan pl = make_plan(m, smp, n);
+  if (goodput_threads(m->d, pl, m->set.prior == 1, nullptr) == 0)
+    return fail(FS_EINVAL, "the goodput stage needs Q / O <= 2048 under the monotone prior, 4096 otherwise");
   const int saved = m->objective;
   m->objective = FS_OBJECTIVE_LEXICOGRAPHIC;  // the base solves to tier 4 (their goodput)
   FS_CUDA(launch_solve(m->set, 2, nullptr, nullptr, nullptr, true, m->lc, s), "launch solve");

@@ -186,46 +186,90 @@ __global__ void __launch_bounds__(256) k_solve_lex(Set set, int n_real, const fl
 
 // --------------------------------------------------------------------------- goodput stage
 
-// Tier-3 goodput of one realisation (rows sC / sOk of realisation sigma, row
-// rr patched to capacity Cr) at tiers 1-2 value t, by one warp: dp and tmp are
-// the warp's two arrays of G + 1 cells; -1 when the floors cannot be met.
+// rint(min(lambda, fl(n c)) 2^20), the same value as goodput_fx, for
+// 0 <= min(...) <= 2^20 (the host requires sum lambda <= 2^20): x 2^-20 is
+// exact there (or its rint is 0 either way), and fixed40 rounds its 2^40
+// multiple to nearest, ties to even, without a float-to-int64 conversion.
+__device__ __forceinline__ long long goodput_fx20(float n, float c, float lam) {
+  const float served = __fmul_rn(n, c);
+  const float x = served < lam ? served : lam;
+  return (long long)fixed40(__fmul_rn(x, 0x1p-20f));
+}
+
+// The options of one row in a realisation: replica counts [lo, hi] (lo = 0:
+// none) at capacity C.
+struct RowOpt {
+  float C;
+  int lo, hi;
+};
+
+// Tier-3 goodput of one realisation (rows sCs / sOk, row rr patched to
+// capacity Cr) at tiers 1-2 value t, by one warp; -1 when the floors cannot
+// be met. Class i's options on row (i, tau = 2^j) are the replica counts n in
+// [1, G / tau] whose fulfilment reaches T_i = t > 0 ? max(t, delta_i) :
+// delta_i (all of them when T_i = 0), up to the first that serves the whole
+// demand (fl(n C) >= lambda_i: more replicas add GPUs and no goodput). Both
+// ends are monotone in n, so each row's options are one range [lo, hi], found
+// once per call (the smallest feasible count by min_replicas, the first
+// saturating count by bisection); the programme over the classes then only
+// reads, adds and compares. opt: the warp's K4 row ranges; dpa, dpb: its two
+// arrays of G + 1 cells.
 template <bool FL>
-__device__ long long warp_goodput(const Set& set, const float* sCs, const int* sOk, const float* sLam,
-                                  const float* sDl, int rr, float Cr, float t, long long* dp, long long* tmp) {
-  const Dims& d = set.d;
+__device__ long long warp_goodput(const Dims& d, const float* sCs, const int* sOk, const float* sLam,
+                                  const float* sRl, const float* sDl, int rr, float Cr, float t, RowOpt* opt,
+                                  long long* dpa, long long* dpb) {
   const int lane = threadIdx.x & 31;
-  for (int g = lane; g <= d.G; g += 32) dp[g] = 0;
-  __syncwarp();
-  for (int i = d.K - 1; i >= 0; --i) {
+  for (int rho = lane; rho < d.K4; rho += 32) {
+    const int i = rho >> 2, j = rho & 3, M = d.G >> j;
+    const float C = rho == rr ? Cr : sCs[rho];
+    const float lam = sLam[i];
     const float dl = FL ? sDl[i] : 0.0f;
     const float T = t > 0.0f ? fmaxf(t, dl) : dl;
+    int lo = 0, hi = 0;
+    if ((rho == rr || sOk[rho]) && M >= 1) {
+      lo = T > 0.0f ? min_replicas(T, C, lam, sRl[i], (float)M) : 1;
+      if (lo > 0) {
+        int a = 1, b = M + 1;  // the first n in [1, M] with fl(n C) >= lambda, else M + 1
+        while (a < b) {
+          const int mid = (a + b) >> 1;
+          if (!(__fmul_rn((float)mid, C) < lam)) b = mid;
+          else a = mid + 1;
+        }
+        hi = min(M, max(lo, a));
+      }
+    }
+    opt[rho] = RowOpt{C, lo, hi};
+  }
+  for (int g = lane; g <= d.G; g += 32) dpa[g] = 0;
+  __syncwarp();
+  long long* cur = dpa;  // S_{i+1}
+  long long* nxt = dpb;
+  for (int i = d.K - 1; i >= 0; --i) {
+    const float dl = FL ? sDl[i] : 0.0f;
     const bool may_empty = !(t > 0.0f) && !(dl > 0.0f);
     const float lam = sLam[i];
     for (int g = lane; g <= d.G; g += 32) {
-      long long best = may_empty ? dp[g] : -1;
+      long long best = may_empty ? cur[g] : -1;
+#pragma unroll
       for (int j = 0; j < kT; ++j) {
-        const int rho = 4 * i + j;
-        if (rho != rr && !sOk[rho]) continue;
-        const float C = rho == rr ? Cr : sCs[rho];
-        const int M = rep_cap(d, j);
-        for (int n = 1; n <= M && (n << j) <= g; ++n) {
-          const float nf = (float)n;
-          if (T > 0.0f && !(fulfil(nf, C, lam) >= T)) continue;
-          const long long pv = dp[g - (n << j)];
+        const RowOpt ro = opt[4 * i + j];
+        const int top = min(ro.hi, g >> j);
+        for (int n = ro.lo; n <= top && n > 0; ++n) {
+          const long long pv = cur[g - (n << j)];
           if (pv >= 0) {
-            const long long v = goodput_fx(nf, C, lam) + pv;
-            if (v > best) best = v;
+            const long long v = goodput_fx20((float)n, ro.C, lam) + pv;
+            best = v > best ? v : best;
           }
-          if (!(__fmul_rn(nf, C) < lam)) break;
         }
       }
-      tmp[g] = best;
+      nxt[g] = best;
     }
     __syncwarp();
-    for (int g = lane; g <= d.G; g += 32) dp[g] = tmp[g];
-    __syncwarp();
+    long long* x = cur;
+    cur = nxt;
+    nxt = x;
   }
-  const long long r = dp[d.G];
+  const long long r = cur[d.G];
   __syncwarp();
   return r;
 }
@@ -247,20 +291,53 @@ __device__ __forceinline__ float tstar_global(const float* h, float C) {
   return tr > thb ? tr : thb;
 }
 
+// Shared memory of k_score_goodput: per table entry its gap (8 bytes), both
+// realisations' row capacities (8) and values (16: t*, then the goodput),
+// one flag byte; per warp its K4 row ranges and two programme arrays.
+struct GoodputSmem {
+  size_t gtab, cap, val, flag, warps, per_warp, total;
+};
+
+__host__ __device__ inline GoodputSmem goodput_smem(int K4, int G, int gt_len, int nwarp) {
+  GoodputSmem m{};
+  auto up = [](size_t x) { return (x + 15) & ~(size_t)15; };
+  m.gtab = 0;
+  m.cap = up(m.gtab + 8 * (size_t)gt_len);
+  m.val = up(m.cap + 8 * (size_t)gt_len);
+  m.flag = up(m.val + 16 * (size_t)gt_len);
+  m.warps = up(m.flag + (size_t)gt_len);
+  m.per_warp = up(sizeof(RowOpt) * (size_t)K4) + 16 * ((size_t)G + 1);
+  m.total = m.warps + (size_t)nwarp * m.per_warp;
+  return m;
+}
+
+// One block per segment (candidate e, outcome o) at a time. Entries: [0, W)
+// open gate at position k; [W, 2W) closed gate at position k - W (under the
+// prior), or W alone (closed, one value). A realisation's goodput depends on
+// an entry only through its patched row capacity C' (t* is a function of C'),
+// and consecutive entries often share C' (every position whose c_y lies at
+// or below Cexcl, or is clamped by the refit): a run of equal C' takes one
+// programme, by the warp that takes the run's first entry, which then writes
+// the value over the run. Then the same draws and sums as the table path.
 template <bool FL, bool RF>
-__global__ void __launch_bounds__(256) k_score_goodput(Set set, Items it, Plan pl, const float* rec,
+__global__ void __launch_bounds__(512) k_score_goodput(Set set, Items it, Plan pl, const float* rec,
                                                        uint64_t* sums) {
   extern __shared__ __align__(16) unsigned char smraw[];
   const Dims& d = set.d;
   const int W = pl.W, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = blockDim.x >> 5;
   const int gt_len = RF ? 2 * W : W + 1;
-  uint2* gtab = reinterpret_cast<uint2*>(smraw);
-  long long* dps = reinterpret_cast<long long*>(smraw + (((size_t)gt_len * 8 + 15) & ~(size_t)15));
-  long long* dp = dps + (size_t)warp * 2 * (d.G + 1);
-  long long* tmp = dp + (d.G + 1);
+  const GoodputSmem lay = goodput_smem(d.K4, d.G, gt_len, nwarp);
+  uint2* gtab = reinterpret_cast<uint2*>(smraw + lay.gtab);
+  float* cap = reinterpret_cast<float*>(smraw + lay.cap);          // [2][gt_len]
+  long long* val = reinterpret_cast<long long*>(smraw + lay.val);  // [2][gt_len]
+  uint8_t* flag = smraw + lay.flag;  // bit 0 / 1: a run starts here (realisation 0 / 1); bit 2: reachable
+  unsigned char* wbase = smraw + lay.warps + (size_t)warp * lay.per_warp;
+  RowOpt* opt = reinterpret_cast<RowOpt*>(wbase);
+  long long* dpa = reinterpret_cast<long long*>(wbase + ((sizeof(RowOpt) * (size_t)d.K4 + 15) & ~(size_t)15));
+  long long* dpb = dpa + (d.G + 1);
   __shared__ float sC[2][256];
   __shared__ int sOk[2][256];
-  __shared__ float sLam[FS_MAX_CLASSES], sDl[FS_MAX_CLASSES];
+  __shared__ float sLam[FS_MAX_CLASSES], sRl[FS_MAX_CLASSES], sDl[FS_MAX_CLASSES];
   for (int x = tid; x < 2 * d.K4; x += blockDim.x) {
     const int sg = x / d.K4, rho = x - sg * d.K4;
     sC[sg][rho] = set.rowC[(size_t)sg * d.K4 + rho];
@@ -268,6 +345,7 @@ __global__ void __launch_bounds__(256) k_score_goodput(Set set, Items it, Plan p
   }
   for (int i = tid; i < d.K; i += blockDim.x) {
     sLam[i] = set.lam[i];
+    sRl[i] = __frcp_rn(set.lam[i]);
     sDl[i] = FL ? set.slo[d.K + i] : 0.0f;
   }
   __syncthreads();
@@ -286,28 +364,69 @@ __global__ void __launch_bounds__(256) k_score_goodput(Set set, Items it, Plan p
     const uint32_t kgs16 = (uint32_t)min((unsigned long long)kgs << 16, 0xFFFFFFFFull);
     const bool any_open = kgs != 0u, any_closed = kgs16 != 0xFFFFFFFFu;
     const RowCap a0 = row_cap_of(h0), a1 = row_cap_of(h1);
-    // entries: [0, W) open gate at position k; [W, 2W) closed (under the prior)
-    // or W (closed, one value)
-    for (int k = warp; k < gt_len; k += nwarp) {
+    auto reachable = [&](int k) { return k < W ? any_open : any_closed; };
+    // each entry's patched row capacity in both realisations
+    for (int k = tid; k < gt_len; k += blockDim.x) {
       const bool g = k < W;
-      if ((g && !any_open) || (!g && !any_closed)) continue;
       const float cy = g ? win[4 + k] : (RF ? win[4 + k - W] : 0.0f);
-      const float c0 = RF ? row_cap(a0, cy, g) : (g ? fmaxf(a0.pc, cy) : a0.pc);
-      const float c1 = RF ? row_cap(a1, cy, g) : (g ? fmaxf(a1.pc, cy) : a1.pc);
-      const float t0 = tstar_global<FL>(h0, c0), t1 = tstar_global<FL>(h1, c1);
-      long long g0 = warp_goodput<FL>(set, sC[0], sOk[0], sLam, sDl, rr, c0, t0, dp, tmp);
-      long long g1 = warp_goodput<FL>(set, sC[1], sOk[1], sLam, sDl, rr, c1, t1, dp, tmp);
-      g0 = g0 < 0 ? 0 : g0;
-      g1 = g1 < 0 ? 0 : g1;
-      const unsigned long long v = (unsigned long long)(g1 > g0 ? g1 - g0 : g0 - g1);
-      if (lane == 0) gtab[k] = make_uint2((uint32_t)(v >> 20), (uint32_t)v & 0xFFFFFu);
+      cap[k] = RF ? row_cap(a0, cy, g) : (g ? fmaxf(a0.pc, cy) : a0.pc);
+      cap[gt_len + k] = RF ? row_cap(a1, cy, g) : (g ? fmaxf(a1.pc, cy) : a1.pc);
+    }
+    __syncthreads();
+    // where runs of equal capacity start, and t* there
+    for (int k = tid; k < gt_len; k += blockDim.x) {
+      uint8_t f = 0;
+      if (reachable(k)) {
+        f = 4;
+        const bool first = k == 0 || !reachable(k - 1);
+        const float c0 = cap[k], c1 = cap[gt_len + k];
+        if (first || __float_as_uint(c0) != __float_as_uint(cap[k - 1])) {
+          f |= 1;
+          val[k] = (long long)__float_as_uint(tstar_global<FL>(h0, c0));
+        }
+        if (first || __float_as_uint(c1) != __float_as_uint(cap[gt_len + k - 1])) {
+          f |= 2;
+          val[gt_len + k] = (long long)__float_as_uint(tstar_global<FL>(h1, c1));
+        }
+      }
+      flag[k] = f;
+    }
+    __syncthreads();
+    // one programme per run, its value written over the run
+    for (int k = warp; k < gt_len; k += nwarp) {
+      const int f = flag[k];
+#pragma unroll 1
+      for (int sg = 0; sg < 2; ++sg) {
+        if (!((f >> sg) & 1)) continue;
+        long long* v = val + (size_t)sg * gt_len;
+        const float c = cap[(size_t)sg * gt_len + k];
+        const float t = __uint_as_float((uint32_t)v[k]);
+        long long gv = warp_goodput<FL>(d, sC[sg], sOk[sg], sLam, sRl, sDl, rr, c, t, opt, dpa, dpb);
+        gv = gv < 0 ? 0 : gv;
+        if (lane == 0) v[k] = gv;
+        for (int base = k + 1;; base += 32) {
+          const int kk = base + lane;
+          const bool stop = kk >= gt_len || !(flag[kk] & 4) || ((flag[kk] >> sg) & 1);
+          const unsigned ball = __ballot_sync(0xffffffffu, stop);
+          const int n = ball ? __ffs(ball) - 1 : 32;
+          if (lane < n) v[kk] = gv;
+          if (ball) break;
+        }
+      }
+    }
+    __syncthreads();
+    for (int k = tid; k < gt_len; k += blockDim.x) {
+      if (!(flag[k] & 4)) continue;
+      const long long g0 = val[k], g1 = val[gt_len + k];
+      const unsigned long long gap = (unsigned long long)(g1 > g0 ? g1 - g0 : g0 - g1);
+      gtab[k] = make_uint2((uint32_t)(gap >> 20), (uint32_t)gap & 0xFFFFFu);
     }
     __syncthreads();
     const GtabSum gs = sample_gtab<true, RF>(pl, keys, o, cell, 0, pl.calls, smem_u32(gtab), kgs16);
     unsigned long long v = gs.total + ((unsigned long long)gs.h << 20) + gs.l;
     for (int off = 16; off; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
     if (lane == 0 && v) atomicAdd(reinterpret_cast<unsigned long long*>(&sums[(size_t)seg]), v);
-    __syncthreads();  // the table is rebuilt for the next segment
+    __syncthreads();  // the tables are rebuilt for the next segment
   }
 }
 
@@ -361,28 +480,37 @@ cudaError_t launch_solve_lex(const Set& set, int n, const float* cap_x, const fl
   return cudaSuccess;
 }
 
-size_t goodput_smem_bytes(const Dims& d, const Plan& pl, bool rf) {
-  const size_t gt_len = rf ? 2 * (size_t)pl.W : (size_t)pl.W + 1;
-  return ((gt_len * 8 + 15) & ~(size_t)15) + (size_t)8 * 2 * (d.G + 1) * 8;  // 8 warps x 2 arrays
+int goodput_threads(const Dims& d, const Plan& pl, bool rf, size_t* smem) {
+  const int gt_len = rf ? 2 * pl.W : pl.W + 1;
+  for (int nw = 16; nw >= 1; --nw) {
+    const GoodputSmem m = goodput_smem(d.K4, d.G, gt_len, nw);
+    if (m.total <= kGoodputSmemMax) {
+      if (smem) *smem = m.total;
+      return 32 * nw;
+    }
+  }
+  return 0;
 }
 
 cudaError_t launch_score_goodput(const Set& set, const Items& it, const Plan& pl, const float* tables,
                                  uint64_t* sums, int floors, int sm_count, cudaStream_t s) {
   if (it.n <= 0) return cudaSuccess;
   const bool rf = set.prior == 1;
-  const size_t smem = goodput_smem_bytes(set.d, pl, rf);
+  size_t smem = 0;
+  const int threads = goodput_threads(set.d, pl, rf, &smem);
+  if (threads == 0) return cudaErrorInvalidValue;  // refused by the host before this point
   auto kern = floors ? (rf ? k_score_goodput<true, true> : k_score_goodput<true, false>)
                      : (rf ? k_score_goodput<false, true> : k_score_goodput<false, false>);
   cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(kern), smem);
   if (e != cudaSuccess) return e;
   int per_sm = 0;
-  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 256, smem);
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, smem);
   if (e != cudaSuccess) return e;
   const long long n_seg = (long long)it.n * pl.O;
   long long grid = (long long)(per_sm < 1 ? 1 : per_sm) * sm_count;
   if (grid > n_seg) grid = n_seg;
   note_launch();
-  kern<<<(unsigned)grid, 256, smem, s>>>(set, it, pl, tables, sums);
+  kern<<<(unsigned)grid, threads, smem, s>>>(set, it, pl, tables, sums);
   return cudaGetLastError();
 }
 

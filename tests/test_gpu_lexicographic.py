@@ -139,3 +139,38 @@ def test_goodput_stage_with_prior_and_floors(fsb, cuda, oracle_lib, qn, prior, f
     ref = oracle_lib.score_goodput(w, qn, stream_id=3, rnd=2)
     assert np.array_equal(r.sum_eo, ref.sum_eo) and r.best == ref.best
     assert np.array_equal(r.score, ref.score) and r.gamma_gp == ref.gamma_gp
+
+
+@pytest.mark.parametrize("K,B,G,prior,factor", [(10, 4, 40, 0, 3.0), (12, 3, 100, 1, 6.0)])
+def test_goodput_stage_many_rows(fsb, cuda, oracle_lib, qn, K, B, G, prior, factor):
+    """More rows than a warp has lanes (4K = 40, 48: each lane takes two rows'
+    replica ranges) and more GPU counts than lanes (G + 1 = 41, 101: several
+    cells per lane in each class step), without and with the prior."""
+    rng = np.random.default_rng(100 + K)
+    w = workloads.random_small(rng, K, B, G)
+    cand = np.sort(rng.choice(len(w.candidates), 12, replace=False)).astype(np.int32)
+    w = dataclasses.replace(w, candidates=cand, O=8, S=64, prior=prior,
+                            demand=(w.demand * np.float32(factor)).astype(np.float32))
+    with load_model(fsb, w) as m:
+        r = fsb.fs_score_goodput(m, cand, w.O, w.S, w.seed)
+    ref = oracle_lib.score_goodput(w, qn, candidates=cand)
+    assert np.array_equal(r.sum_eo, ref.sum_eo), f"{int((r.sum_eo != ref.sum_eo).sum())} sums differ"
+    assert np.array_equal(r.score, ref.score) and r.gamma_gp == ref.gamma_gp and r.best == ref.best
+    assert ref.gamma_fx > 0 and np.all(ref.sum_eo != 0)
+
+
+def test_goodput_stage_table_limit(fsb, cuda, oracle_lib, qn):
+    """A segment's table of Q / O positions lives in shared memory: one outcome
+    (Q / O = 4096 positions) is refused under the monotone prior (8192
+    entries) and scored without it (4097 entries), equal to the oracle."""
+    w = workloads.make_workload(0)
+    w = dataclasses.replace(w, demand=(w.demand * np.float32(3.0)).astype(np.float32), O=1, S=512)
+    cand = w.candidates[:4]
+    with load_model(fsb, dataclasses.replace(w, prior=1)) as m:
+        with pytest.raises(fsb.FleetSieveError) as ei:
+            fsb.fs_score_goodput(m, cand, 1, w.S, w.seed)
+        assert ei.value.code == fsb.FS_EINVAL
+    with load_model(fsb, w) as m:
+        r = fsb.fs_score_goodput(m, cand, 1, w.S, w.seed)
+    ref = oracle_lib.score_goodput(w, qn, candidates=cand)
+    assert np.array_equal(r.sum_eo, ref.sum_eo) and r.best == ref.best and r.gamma_gp == ref.gamma_gp
