@@ -745,17 +745,22 @@ int fs_score_goodput(fs_model* m, const fs_samples* smp, double* gap_out, double
   if ((rc = ensure_items(m, n, smp->O))) return rc;
   cudaStream_t s = m->stream;
   if ((rc = flush_bounds(m, s))) return rc;
+  // as in fs_score_candidates, one mapped page-locked block carries the
+  // candidate ids in and gap, score, gamma, best and the status word out
   const size_t nn = (size_t)std::max(n, 1);
-  int32_t* d_cand = static_cast<int32_t*>(m->cand.p);
-  double* d_gap = static_cast<double*>(m->outs.p);
+  const size_t out_bytes = align_up(16 * nn + 16, 16);
+  if ((rc = m->h_out.ensure(out_bytes + 4 * nn, "host staging"))) return rc;
+  char* h = static_cast<char*>(m->h_out.p);
+  char* hd = static_cast<char*>(m->h_out.dev);
+  if (n > 0) std::memcpy(h + out_bytes, smp->cand, 4 * (size_t)n);
+  double* d_gap = reinterpret_cast<double*>(hd);
   double* d_score = d_gap + nn;
-  // (outs holds 16 nn + 64 bytes: gap, score, then gamma and best in the tail)
-  double* d_gamma = reinterpret_cast<double*>(static_cast<char*>(m->outs.p) + 16 * nn);
-  int32_t* d_best = reinterpret_cast<int32_t*>(d_gamma + 1);
-  if (n > 0) FS_CUDA(cudaMemcpyAsync(d_cand, smp->cand, 4 * (size_t)n, cudaMemcpyHostToDevice, s), "upload cand");
+  double* d_gamma = reinterpret_cast<double*>(hd + 16 * nn);
+  int32_t* d_best = reinterpret_cast<int32_t*>(hd + 16 * nn + 8);
+  uint32_t* d_st = reinterpret_cast<uint32_t*>(hd + 16 * nn + 12);
   Items it{};
   it.n = n;
-  it.cell = d_cand;
+  it.cell = reinterpret_cast<const int32_t*>(hd + out_bytes);
   const Plan pl = make_plan(m, smp, n);
   if (goodput_threads(m->d, pl, m->set.prior == 1, nullptr) == 0)
     return fail(FS_EINVAL, "the goodput stage needs Q / O <= 2048 under the monotone prior, 4096 otherwise");
@@ -770,16 +775,19 @@ int fs_score_goodput(fs_model* m, const fs_samples* smp, double* gap_out, double
   FS_CUDA(launch_score_goodput(m->set, it, pl, static_cast<const float*>(m->tables.p), sums, m->lc.floors,
                                m->sm_count, s),
           "launch goodput scorer");
-  FS_CUDA(launch_finalize_goodput(m->set, it, pl, sums, lam_sum, d_gap, d_score, d_gamma, d_best, s),
+  FS_CUDA(launch_finalize_goodput(m->set, it, pl, sums, lam_sum, d_gap, d_score, d_gamma, d_best, d_st, s),
           "launch goodput reduction");
-  if (gap_out && n) FS_CUDA(cudaMemcpyAsync(gap_out, d_gap, 8 * (size_t)n, cudaMemcpyDeviceToHost, s), "read gap");
-  if (score_out && n)
-    FS_CUDA(cudaMemcpyAsync(score_out, d_score, 8 * (size_t)n, cudaMemcpyDeviceToHost, s), "read score");
-  if (gamma_gp) FS_CUDA(cudaMemcpyAsync(gamma_gp, d_gamma, 8, cudaMemcpyDeviceToHost, s), "read gamma");
-  if (best) FS_CUDA(cudaMemcpyAsync(best, d_best, 4, cudaMemcpyDeviceToHost, s), "read best");
   if (sum_eo && n)
     FS_CUDA(cudaMemcpyAsync(sum_eo, sums, 8 * (size_t)n * smp->O, cudaMemcpyDeviceToHost, s), "read sums");
-  return read_status(m, s);
+  FS_CUDA(cudaStreamSynchronize(s), "synchronize");
+  uint32_t st;
+  std::memcpy(&st, h + 16 * nn + 12, 4);
+  if (st) return status_error(m, st);
+  if (gap_out && n) std::memcpy(gap_out, h, 8 * (size_t)n);
+  if (score_out && n) std::memcpy(score_out, h + 8 * nn, 8 * (size_t)n);
+  if (gamma_gp) std::memcpy(gamma_gp, h + 16 * nn, 8);
+  if (best) std::memcpy(best, h + 16 * nn + 8, 4);
+  return FS_OK;
 }
 
 int fs_replay(fs_model* m, const fs_replay_spec* sp, int32_t* rounds, int32_t* state, double* gpu_seconds,

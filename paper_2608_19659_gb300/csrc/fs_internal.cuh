@@ -504,7 +504,7 @@ size_t lex_scratch_cells(const Dims& d);  // (K + 1)(G + 1) cells per realisatio
 // out / the base), per_launch of them at a time through scratch.
 cudaError_t launch_solve_lex(const Set& set, int n, const float* cap_x, const float* tail_x, fs_allocation* out,
                              void* scratch, int per_launch, cudaStream_t s);
-// Threads per block of the goodput scorer (a multiple of 32, at most 512) and
+// Threads per block of the goodput scorer (a multiple of 32, at most 256) and
 // its dynamic shared memory, or 0 when one warp's share does not fit.
 constexpr size_t kGoodputSmemMax = 220 * 1024;  // of the 227 KB a block may opt into, less its static arrays
 int goodput_threads(const Dims& d, const Plan& pl, bool rf, size_t* smem);
@@ -512,7 +512,7 @@ cudaError_t launch_score_goodput(const Set& set, const Items& it, const Plan& pl
                                  uint64_t* sums, int floors, int sm_count, cudaStream_t s);
 cudaError_t launch_finalize_goodput(const Set& set, const Items& it, const Plan& pl, const uint64_t* sums,
                                     double lam_sum, double* gap, double* score, double* gamma, int32_t* best,
-                                    cudaStream_t s);
+                                    uint32_t* status_copy, cudaStream_t s);
 
 // replay
 struct ReplayState {

@@ -197,54 +197,78 @@ __device__ __forceinline__ long long goodput_fx20(float n, float c, float lam) {
 }
 
 // The options of one row in a realisation: replica counts [lo, hi] (lo = 0:
-// none) at capacity C.
+// none) at capacity C, and the thresholds T in (a, b] for which they stay so.
 struct RowOpt {
   float C;
   int lo, hi;
+  float a, b;
 };
 
-// Tier-3 goodput of one realisation (rows sCs / sOk, row rr patched to
-// capacity Cr) at tiers 1-2 value t, by one warp; -1 when the floors cannot
-// be met. Class i's options on row (i, tau = 2^j) are the replica counts n in
-// [1, G / tau] whose fulfilment reaches T_i = t > 0 ? max(t, delta_i) :
-// delta_i (all of them when T_i = 0), up to the first that serves the whole
-// demand (fl(n C) >= lambda_i: more replicas add GPUs and no goodput). Both
-// ends are monotone in n, so each row's options are one range [lo, hi], found
-// once per call (the smallest feasible count by min_replicas, the first
-// saturating count by bisection); the programme over the classes then only
-// reads, adds and compares. opt: the warp's K4 row ranges; dpa, dpb: its two
-// arrays of G + 1 cells.
+// Class i's options on row (i, tau = 2^j) at capacity C are the replica
+// counts n in [1, M = G / tau] whose fulfilment reaches T (all of them when
+// T = 0), up to the first that serves the whole demand (fl(n C) >= lambda:
+// more replicas add GPUs and no goodput). Both ends are monotone in n, so the
+// options are one range [lo, hi]: the smallest feasible count by
+// min_replicas, the first saturating count by bisection. lo = 0: none.
+__device__ __forceinline__ void row_range(float C, bool ok, int M, float T, float lam, float rl, int& lo, int& hi) {
+  lo = hi = 0;
+  if (!ok || M < 1) return;
+  lo = T > 0.0f ? min_replicas(T, C, lam, rl, (float)M) : 1;
+  if (lo == 0) return;
+  int a = 1, b = M + 1;  // the first n in [1, M] with fl(n C) >= lambda, else M + 1
+  while (a < b) {
+    const int mid = (a + b) >> 1;
+    if (!(__fmul_rn((float)mid, C) < lam)) b = mid;
+    else a = mid + 1;
+  }
+  hi = min(M, max(lo, a));
+}
+
+// The row's range and the interval of thresholds that gives the same lo (and
+// so the same hi): fulfil(lo - 1) < T <= fulfil(lo) for lo >= 1 (no lower end
+// at lo = 1), T > fulfil(M) for lo = 0 (fulfil is nondecreasing in n).
+__device__ __forceinline__ RowOpt row_opt(float C, bool ok, int M, float T, float lam, float rl) {
+  RowOpt r{C, 0, 0, -INFINITY, INFINITY};
+  row_range(C, ok, M, T, lam, rl, r.lo, r.hi);
+  if (!ok || M < 1) return r;
+  if (r.lo == 0) {
+    r.a = fulfil((float)M, C, lam);
+  } else {
+    r.b = fulfil((float)r.lo, C, lam);
+    if (r.lo > 1) r.a = fulfil((float)(r.lo - 1), C, lam);
+  }
+  return r;
+}
+
+__device__ __forceinline__ float class_threshold(float t, float dl) { return t > 0.0f ? fmaxf(t, dl) : dl; }
+
+// The best tier-3 goodput of every class but `skip` within g GPUs, for g in
+// [0, G], at tiers 1-2 value t (-1: the floors of those classes cannot be
+// met within g), by one warp: the programme over the classes (no replicas,
+// when class i may stay empty: T_i = 0 and no floor; else one range of
+// replica counts on each of its rows) with lanes over g. Also leaves in opt
+// every row's range at t (those of `skip` for warp_best_with; row `fixed`,
+// whose capacity varies, with no interval). dpa, dpb: the warp's two arrays
+// of G + 1 cells. Returns the array that holds the result.
 template <bool FL>
-__device__ long long warp_goodput(const Dims& d, const float* sCs, const int* sOk, const float* sLam,
-                                  const float* sRl, const float* sDl, int rr, float Cr, float t, RowOpt* opt,
-                                  long long* dpa, long long* dpb) {
+__device__ const long long* warp_other(const Dims& d, const float* sCs, const int* sOk, const float* sLam,
+                                       const float* sRl, const float* sDl, int skip, int fixed, float t,
+                                       RowOpt* opt, long long* dpa, long long* dpb) {
   const int lane = threadIdx.x & 31;
+  __syncwarp();  // the previous result and ranges are no longer read
   for (int rho = lane; rho < d.K4; rho += 32) {
-    const int i = rho >> 2, j = rho & 3, M = d.G >> j;
-    const float C = rho == rr ? Cr : sCs[rho];
-    const float lam = sLam[i];
-    const float dl = FL ? sDl[i] : 0.0f;
-    const float T = t > 0.0f ? fmaxf(t, dl) : dl;
-    int lo = 0, hi = 0;
-    if ((rho == rr || sOk[rho]) && M >= 1) {
-      lo = T > 0.0f ? min_replicas(T, C, lam, sRl[i], (float)M) : 1;
-      if (lo > 0) {
-        int a = 1, b = M + 1;  // the first n in [1, M] with fl(n C) >= lambda, else M + 1
-        while (a < b) {
-          const int mid = (a + b) >> 1;
-          if (!(__fmul_rn((float)mid, C) < lam)) b = mid;
-          else a = mid + 1;
-        }
-        hi = min(M, max(lo, a));
-      }
-    }
-    opt[rho] = RowOpt{C, lo, hi};
+    const int i = rho >> 2;
+    RowOpt r = row_opt(sCs[rho], sOk[rho] != 0, d.G >> (rho & 3), class_threshold(t, FL ? sDl[i] : 0.0f),
+                       sLam[i], sRl[i]);
+    if (rho == fixed) r.a = -INFINITY, r.b = INFINITY;
+    opt[rho] = r;
   }
   for (int g = lane; g <= d.G; g += 32) dpa[g] = 0;
   __syncwarp();
   long long* cur = dpa;  // S_{i+1}
   long long* nxt = dpb;
   for (int i = d.K - 1; i >= 0; --i) {
+    if (i == skip) continue;
     const float dl = FL ? sDl[i] : 0.0f;
     const bool may_empty = !(t > 0.0f) && !(dl > 0.0f);
     const float lam = sLam[i];
@@ -269,9 +293,65 @@ __device__ long long warp_goodput(const Dims& d, const float* sCs, const int* sO
     cur = nxt;
     nxt = x;
   }
-  const long long r = cur[d.G];
-  __syncwarp();
-  return r;
+  return cur;
+}
+
+// Whether the ranges in opt (left by warp_other at a value t0 with
+// (t0 > 0) = pos) hold at t as well: then so do the programme's result and
+// class i_r's other rows. One warp.
+template <bool FL>
+__device__ bool warp_ranges_hold(const Dims& d, const float* sDl, const RowOpt* opt, float t, bool pos) {
+  const int lane = threadIdx.x & 31;
+  bool ok = (t > 0.0f) == pos;
+  for (int rho = lane; rho < d.K4; rho += 32) {
+    const float T = class_threshold(t, FL ? sDl[rho >> 2] : 0.0f);
+    ok = ok && opt[rho].a < T && T <= opt[rho].b;
+  }
+  return __all_sync(0xffffffffu, ok);
+}
+
+// Tier-3 goodput of one realisation with row rr at capacity Cr (its range
+// [lor, hir] at t), at tiers 1-2 value t, given other = warp_other(..., skip
+// = class of rr, t): the best over class i_r's choices (nothing, when it may
+// stay empty; else n replicas on one of its rows) of its goodput plus the
+// others' best within the GPUs left; -1 when the floors cannot be met. Lanes
+// over the choices, one warp.
+template <bool FL>
+__device__ long long warp_best_with(const Dims& d, const float* sLam, const float* sDl, const RowOpt* opt, int rr,
+                                    float Cr, int lor, int hir, float t, const long long* other) {
+  const int lane = threadIdx.x & 31, ir = rr >> 2, jr = rr & 3;
+  const float lam = sLam[ir];
+  const float dl = FL ? sDl[ir] : 0.0f;
+  int cnt[kT], lo[kT];
+  float C[kT];
+#pragma unroll
+  for (int j = 0; j < kT; ++j) {
+    const RowOpt ro = opt[4 * ir + j];
+    lo[j] = j == jr ? lor : ro.lo;
+    const int hi = j == jr ? hir : ro.hi;
+    C[j] = j == jr ? Cr : ro.C;
+    cnt[j] = lo[j] > 0 ? hi - lo[j] + 1 : 0;
+  }
+  long long best = (!(t > 0.0f) && !(dl > 0.0f)) ? other[d.G] : -1;
+  const int e1 = cnt[0], e2 = e1 + cnt[1], e3 = e2 + cnt[2], total = e3 + cnt[3];
+  for (int x = lane; x < total; x += 32) {
+    int j, n;
+    float Cj;
+    if (x < e1) { j = 0; n = lo[0] + x; Cj = C[0]; }
+    else if (x < e2) { j = 1; n = lo[1] + (x - e1); Cj = C[1]; }
+    else if (x < e3) { j = 2; n = lo[2] + (x - e2); Cj = C[2]; }
+    else { j = 3; n = lo[3] + (x - e3); Cj = C[3]; }
+    const long long pv = other[d.G - (n << j)];
+    if (pv >= 0) {
+      const long long v = goodput_fx20((float)n, Cj, lam) + pv;
+      best = v > best ? v : best;
+    }
+  }
+  for (int off = 16; off; off >>= 1) {
+    const long long o = __shfl_xor_sync(0xffffffffu, best, off);
+    best = o > best ? o : best;
+  }
+  return best;
 }
 
 // t* of realisation sigma at row capacity C, from the candidate's table in
@@ -314,13 +394,17 @@ __host__ __device__ inline GoodputSmem goodput_smem(int K4, int G, int gt_len, i
 // One block per segment (candidate e, outcome o) at a time. Entries: [0, W)
 // open gate at position k; [W, 2W) closed gate at position k - W (under the
 // prior), or W alone (closed, one value). A realisation's goodput depends on
-// an entry only through its patched row capacity C' (t* is a function of C'),
-// and consecutive entries often share C' (every position whose c_y lies at
-// or below Cexcl, or is clamped by the refit): a run of equal C' takes one
-// programme, by the warp that takes the run's first entry, which then writes
-// the value over the run. Then the same draws and sums as the table path.
+// an entry only through its patched row capacity C' (t* is a function of
+// C'), and consecutive entries often share C' (every position whose c_y lies
+// at or below Cexcl, or is clamped by the refit): a run of equal C' takes one
+// evaluation. The evaluation splits the programme at class i_r: the other
+// classes' best within g GPUs depends on the entry only through the replica
+// ranges that t* leaves their rows, which change at few values of t* in a
+// segment, so a warp reruns that part only where a range changes and
+// otherwise only combines it with class i_r's choices. Then the same draws
+// and sums as the table path.
 template <bool FL, bool RF>
-__global__ void __launch_bounds__(512) k_score_goodput(Set set, Items it, Plan pl, const float* rec,
+__global__ void __launch_bounds__(256, 2) k_score_goodput(Set set, Items it, Plan pl, const float* rec,
                                                        uint64_t* sums) {
   extern __shared__ __align__(16) unsigned char smraw[];
   const Dims& d = set.d;
@@ -352,6 +436,9 @@ __global__ void __launch_bounds__(512) k_score_goodput(Set set, Items it, Plan p
   const PhiloxKeys keys{};  // (the plan's round keys serve a one-problem launch)
   const long long n_seg = (long long)it.n * pl.O;
   for (long long seg = blockIdx.x; seg < n_seg; seg += gridDim.x) {
+    const long long* other = nullptr;  // the warp's programme over the other classes, for this segment
+    bool other_pos = false;
+    int other_sg = 0;
     const int item = (int)(seg / pl.O), o = (int)(seg - (long long)item * pl.O);
     const float* r = rec + (size_t)item * pl.item_floats;
     const float* h0 = r;
@@ -392,26 +479,46 @@ __global__ void __launch_bounds__(512) k_score_goodput(Set set, Items it, Plan p
       flag[k] = f;
     }
     __syncthreads();
-    // one programme per run, its value written over the run
-    for (int k = warp; k < gt_len; k += nwarp) {
-      const int f = flag[k];
-#pragma unroll 1
-      for (int sg = 0; sg < 2; ++sg) {
-        if (!((f >> sg) & 1)) continue;
+    // the warps take chunks of 32 entries of one realisation in turn; a chunk's
+    // first reachable entry starts a run. Every run start's row-r range comes
+    // from its own lane; the others' programme is rerun only where a row's
+    // range changes with t*
+    {
+      const int ir = rr >> 2, jr = rr & 3;
+      const float lam_r = sLam[ir], rl_r = sRl[ir], dl_r = FL ? sDl[ir] : 0.0f;
+      const int n_chunk = (gt_len + 31) >> 5;
+      for (int task = warp; task < 2 * n_chunk; task += nwarp) {
+        const int sg = task & 1, kk = ((task >> 1) << 5) + lane;
+        const float* cs = cap + (size_t)sg * gt_len;
         long long* v = val + (size_t)sg * gt_len;
-        const float c = cap[(size_t)sg * gt_len + k];
-        const float t = __uint_as_float((uint32_t)v[k]);
-        long long gv = warp_goodput<FL>(d, sC[sg], sOk[sg], sLam, sRl, sDl, rr, c, t, opt, dpa, dpb);
-        gv = gv < 0 ? 0 : gv;
-        if (lane == 0) v[k] = gv;
-        for (int base = k + 1;; base += 32) {
-          const int kk = base + lane;
-          const bool stop = kk >= gt_len || !(flag[kk] & 4) || ((flag[kk] >> sg) & 1);
-          const unsigned ball = __ballot_sync(0xffffffffu, stop);
-          const int n = ball ? __ffs(ball) - 1 : 32;
-          if (lane < n) v[kk] = gv;
-          if (ball) break;
+        const bool reach = kk < gt_len && (flag[kk] & 4);
+        const bool start = reach && ((flag[kk] >> sg) & 1);
+        const unsigned rb = __ballot_sync(0xffffffffu, reach);
+        const bool head = start || (rb && lane == __ffs(rb) - 1);
+        float c = 0.0f, t = 0.0f;
+        int lor = 0, hir = 0;
+        if (head) {  // t* stored where a run starts, else evaluated
+          c = cs[kk];
+          t = start ? __uint_as_float((uint32_t)v[kk]) : tstar_global<FL>(sg ? h1 : h0, c);
+          row_range(c, true, d.G >> jr, class_threshold(t, dl_r), lam_r, rl_r, lor, hir);
         }
+        unsigned heads = __ballot_sync(0xffffffffu, head);
+        long long mine = 0;
+        while (heads) {
+          const int p = __ffs(heads) - 1;
+          heads &= heads - 1;
+          const float tp = __shfl_sync(0xffffffffu, t, p), cp = __shfl_sync(0xffffffffu, c, p);
+          const int lop = __shfl_sync(0xffffffffu, lor, p), hip = __shfl_sync(0xffffffffu, hir, p);
+          if (other == nullptr || other_sg != sg || !warp_ranges_hold<FL>(d, sDl, opt, tp, other_pos)) {
+            other = warp_other<FL>(d, sC[sg], sOk[sg], sLam, sRl, sDl, ir, rr, tp, opt, dpa, dpb);
+            other_pos = tp > 0.0f;
+            other_sg = sg;
+          }
+          long long gv = warp_best_with<FL>(d, sLam, sDl, opt, rr, cp, lop, hip, tp, other);
+          gv = gv < 0 ? 0 : gv;
+          if (lane >= p) mine = gv;
+        }
+        if (reach) v[kk] = mine;
       }
     }
     __syncthreads();
@@ -432,8 +539,11 @@ __global__ void __launch_bounds__(512) k_score_goodput(Set set, Items it, Plan p
 
 // E, score and argmax of the goodput stage for one problem (one CTA).
 __global__ void k_finalize_goodput(Set set, Items it, Plan pl, const uint64_t* sums, double lam_sum, double* gap,
-                                   double* score, double* gamma, int32_t* best) {
+                                   double* score, double* gamma, int32_t* best, uint32_t* status_copy) {
   __shared__ Best sb[32];
+  // every earlier kernel of the call has completed: the status word travels
+  // with the outputs
+  if (threadIdx.x == 0 && status_copy) *status_copy = *set.status;
   const Dims& d = set.d;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = blockDim.x >> 5;
   const long long gm = __double2ll_rn(__dmul_rn(set.base[0].goodput, 0x1p20));
@@ -482,7 +592,7 @@ cudaError_t launch_solve_lex(const Set& set, int n, const float* cap_x, const fl
 
 int goodput_threads(const Dims& d, const Plan& pl, bool rf, size_t* smem) {
   const int gt_len = rf ? 2 * pl.W : pl.W + 1;
-  for (int nw = 16; nw >= 1; --nw) {
+  for (int nw = 8; nw >= 1; --nw) {
     const GoodputSmem m = goodput_smem(d.K4, d.G, gt_len, nw);
     if (m.total <= kGoodputSmemMax) {
       if (smem) *smem = m.total;
@@ -503,12 +613,11 @@ cudaError_t launch_score_goodput(const Set& set, const Items& it, const Plan& pl
                      : (rf ? k_score_goodput<false, true> : k_score_goodput<false, false>);
   cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(kern), smem);
   if (e != cudaSuccess) return e;
-  int per_sm = 0;
-  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, smem);
-  if (e != cudaSuccess) return e;
+  // one block per segment: segments differ widely in cost (where row r sets
+  // t*, its ranges change often), and the block scheduler evens them out
   const long long n_seg = (long long)it.n * pl.O;
-  long long grid = (long long)(per_sm < 1 ? 1 : per_sm) * sm_count;
-  if (grid > n_seg) grid = n_seg;
+  const long long grid = n_seg < 0x7fffffffLL ? n_seg : 0x7fffffffLL;
+  (void)sm_count;
   note_launch();
   kern<<<(unsigned)grid, threads, smem, s>>>(set, it, pl, tables, sums);
   return cudaGetLastError();
@@ -516,9 +625,9 @@ cudaError_t launch_score_goodput(const Set& set, const Items& it, const Plan& pl
 
 cudaError_t launch_finalize_goodput(const Set& set, const Items& it, const Plan& pl, const uint64_t* sums,
                                     double lam_sum, double* gap, double* score, double* gamma, int32_t* best,
-                                    cudaStream_t s) {
+                                    uint32_t* status_copy, cudaStream_t s) {
   note_launch();
-  k_finalize_goodput<<<1, 256, 0, s>>>(set, it, pl, sums, lam_sum, gap, score, gamma, best);
+  k_finalize_goodput<<<1, 256, 0, s>>>(set, it, pl, sums, lam_sum, gap, score, gamma, best, status_copy);
   return cudaGetLastError();
 }
 

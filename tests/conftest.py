@@ -104,6 +104,36 @@ def read_expected_sums(name):
     return sha, gamma_t, best, np.array(cells, np.int32), full - np.array(deficits, np.int64)
 
 
+def read_expected_goodput():
+    """The goodput-stage sums file written by tests/golden/make_expected_sums.py:
+    (inputs_sha256, gamma_fx, gamma_gp, best, cells [n], sum_eo [n, O])."""
+    import numpy as np
+
+    sha = None
+    gamma_fx = gamma_gp = best = None
+    cells, sums = [], []
+    with open(os.path.join(GOLDEN, "goodput_paper_scale_sums.txt")) as f:
+        for line in f:
+            if line.startswith("# inputs_sha256"):
+                sha = line.split()[2]
+                continue
+            if not line.strip() or line.startswith("#"):
+                continue
+            t = line.split()
+            if t[0] == "gamma_fx":
+                gamma_fx = int(t[1])
+            elif t[0] == "gamma_gp":
+                gamma_gp = float(t[1])
+            elif t[0] == "best":
+                best = int(t[1])
+            elif t[0] == "shape":
+                continue
+            else:
+                cells.append(int(t[0]))
+                sums.append([int(x) for x in t[1:]])
+    return sha, gamma_fx, gamma_gp, best, np.array(cells, np.int32), np.array(sums, np.int64)
+
+
 def read_expected_replay():
     """The expected replay file written by tests/golden/make_expected_sums.py:
     (inputs_sha256, {stream: (rounds, state, gpu_seconds, reveal order, Gamma_t trace)})."""

@@ -11,12 +11,17 @@ within SLO) pairs. Candidates are split into contiguous ranges, one
 single-threaded oracle process per range; the sums do not depend on the split.
 
 Usage: python tests/golden/make_expected_sums.py [--procs N] [name ...]
-with names from WORKLOADS below and "replay" (default: all). Each sums file records:
+with names from WORKLOADS below, "replay" and "goodput" (default: all). Each sums file records:
   * the sha256 of the workload's inputs (bounds, demands, SLOs, candidates),
   * Gamma_t and the argmax cell,
   * per candidate the deficits d[e][o] = S rint(Gamma_t 2^40) - sum_eo[e][o]
     (the fixed-point score of each outcome stratum; 0 for a candidate that
     cannot change either allocation), so that sum_eo = S rint(Gamma_t 2^40) - d.
+
+"goodput" writes the goodput stage of the score (every scenario's two
+realisations solved to tier 4) on the paper-scale workload in full: per
+candidate and outcome the int64 sum, with Gamma_gp,t in 2^-20 units and the
+argmax.
 
 "replay" writes the replay workload (Algorithm 1 over 200 reveal orders of
 the paper-scale grid, 8 x 4096 samples per candidate and round, seed 2026):
@@ -114,6 +119,35 @@ def write(name, w, sums, res):
             f.write(f"{int(cell)} " + " ".join(str(int(x)) for x in d[e]) + "\n")
 
 
+GOODPUT_FILE = "goodput_paper_scale_sums.txt"
+
+
+def write_goodput():
+    """The goodput stage of the score (Section 4.3 with both realisations of
+    every scenario solved to tier 4 of Section 3's objective) on the
+    paper-scale workload in full: 64 candidates x 8 outcomes x 4096 samples,
+    one oracle call."""
+    import oracle
+    from paper_2608_19659_gb300 import workloads
+
+    w = workloads.make_workload(1)
+    qn = oracle.triangular_table(4096)
+    r = oracle.score_goodput(w, qn)
+    with open(os.path.join(HERE, GOODPUT_FILE), "w") as f:
+        f.write("# Expected int64 sums of the oracle's goodput stage (Section 4.3, tiers 1-4 of Section 3)\n")
+        f.write(f"# workload: {w.name}\n")
+        f.write("# written by tests/golden/make_expected_sums.py goodput (oracle/ only)\n")
+        f.write(f"# inputs_sha256 {input_digest(w)}\n")
+        f.write("# columns: cell, then O sums of rint(|GP(A+') - GP(A-')| 2^20) over the outcome's samples\n")
+        f.write(f"gamma_fx {r.gamma_fx}\n")
+        f.write(f"gamma_gp {r.gamma_gp!r}\n")
+        f.write(f"best {r.best}\n")
+        f.write(f"shape {len(w.candidates)} {w.O} {w.S}\n")
+        for e, cell in enumerate(w.candidates):
+            f.write(f"{int(cell)} " + " ".join(str(int(x)) for x in r.sum_eo[e]) + "\n")
+    return w, r
+
+
 REPLAY_FILE = "replay_200_streams.txt"
 REPLAY_SEED = 2026
 
@@ -164,11 +198,16 @@ def write_replay(procs):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("names", nargs="*", default=list(WORKLOADS) + ["replay"])
+    ap.add_argument("names", nargs="*", default=list(WORKLOADS) + ["replay", "goodput"])
     ap.add_argument("--procs", type=int, default=len(os.sched_getaffinity(0)))
     a = ap.parse_args()
     for name in a.names:
         t0 = time.time()
+        if name == "goodput":
+            w, r = write_goodput()
+            print(f"goodput: {len(w.candidates)} candidates, gamma_fx {r.gamma_fx}, best {r.best}, "
+                  f"{time.time() - t0:.0f} s")
+            continue
         if name == "replay":
             res = write_replay(a.procs)
             print(f"replay: {len(res)} streams, {sum(r.rounds for r in res)} rounds, "

@@ -40,3 +40,25 @@ def test_expected_sums_reproduce(oracle_lib, name):
     assert np.array_equal(se, sums[pick])
     # the estimator's invariants hold for every stored candidate: 0 <= score <= Gamma_t
     assert np.all(red.score >= 0.0) and np.all(red.score <= gamma_t)
+
+
+def test_expected_goodput_sums_reproduce(oracle_lib):
+    """The stored goodput-stage sums of the paper-scale workload: the inputs,
+    the base goodput gap, and the argmax candidate plus four others recomputed
+    by the oracle. Sums are nonnegative (a scenario's goodput gap is an
+    absolute difference; unlike the max-min gap it has no upper bound in
+    Gamma_gp,t, since tier 3 is taken at each realisation's own t*)."""
+    from conftest import read_expected_goodput
+    from paper_2608_19659_gb300 import workloads
+
+    w = workloads.make_workload(1)
+    sha, gamma_fx, gamma_gp, best, cells, sums = read_expected_goodput()
+    assert sha == mes.input_digest(w)
+    assert np.array_equal(cells, w.candidates) and sums.shape == (len(w.candidates), w.O)
+    assert np.all(sums >= 0)
+    qn = oracle_lib.triangular_table(4096)
+    e_best = int(np.nonzero(w.candidates == best)[0][0])
+    pick = np.unique([0, e_best, 17, 40, len(cells) - 1])
+    r = oracle_lib.score_goodput(w, qn, candidates=w.candidates[pick])
+    assert np.array_equal(r.sum_eo, sums[pick])
+    assert r.gamma_fx == gamma_fx and r.gamma_gp == gamma_gp

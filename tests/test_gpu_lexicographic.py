@@ -174,3 +174,24 @@ def test_goodput_stage_table_limit(fsb, cuda, oracle_lib, qn):
         r = fsb.fs_score_goodput(m, cand, 1, w.S, w.seed)
     ref = oracle_lib.score_goodput(w, qn, candidates=cand)
     assert np.array_equal(r.sum_eo, ref.sum_eo) and r.best == ref.best and r.gamma_gp == ref.gamma_gp
+
+
+def test_goodput_stage_paper_scale_full(fsb, cuda):
+    """The goodput stage on the paper-scale workload in full (64 candidates x
+    8 outcomes x 4096 samples, the bench's configuration): every int64 sum,
+    Gamma_gp,t and the argmax equal the oracle's stored values (tests/golden,
+    written by the oracle alone)."""
+    import sys
+
+    from conftest import GOLDEN, read_expected_goodput
+
+    sys.path.insert(0, GOLDEN)
+    import make_expected_sums as mes
+
+    w = workloads.make_workload(1)
+    sha, gamma_fx, gamma_gp, best, cells, sums = read_expected_goodput()
+    assert sha == mes.input_digest(w)
+    with load_model(fsb, w) as m:
+        r = fsb.fs_score_goodput(m, w.candidates, w.O, w.S, w.seed)
+    assert np.array_equal(r.sum_eo, sums), f"{int((r.sum_eo != sums).sum())} sums differ"
+    assert r.gamma_gp == gamma_gp and r.best == best

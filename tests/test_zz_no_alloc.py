@@ -1,4 +1,4 @@
-"""The allocation-free scoring entry point against the allocating one.
+"""The allocation-free scoring entry point against the allocating one and the oracle.
 
 fs_score_candidates_noalloc exists for callers that cannot allocate device
 memory while they run (memory already handed out by their own pool, or no
@@ -50,6 +50,30 @@ def test_noalloc_matches_allocating_entry_point_on_two_calls(fsb, cuda, idx, fac
             assert np.array_equal(score.cpu().numpy(), ref.score)
             assert float(gt.item()) == ref.gamma_t and int(best.item()) == ref.best
     if factor != 1.0:
+        assert ref.score.max() > 0
+
+
+def test_noalloc_matches_oracle(fsb, cuda, oracle_lib):
+    """The allocation-free entry point against the oracle directly: the tiny
+    workload at 3x demand (nonzero scores), two rounds through the shared
+    array; gap, score, Gamma_t and the argmax equal the oracle's bit for bit."""
+    torch = cuda
+    w = workloads.make_workload(0)
+    w = dataclasses.replace(w, demand=(w.demand * np.float32(3.0)).astype(np.float32))
+    bounds, slo, lam, cand = _device_inputs(torch, w)
+    n = len(w.candidates)
+    qn = oracle_lib.triangular_table(4096)
+    stream = torch.cuda.current_stream()
+    for rnd in (0, 1):
+        ref = oracle_lib.score(w, qn, rnd=rnd)
+        gap = torch.full((n,), float("nan"), dtype=torch.float64, device="cuda")
+        score = torch.full((n,), float("nan"), dtype=torch.float64, device="cuda")
+        gt = torch.full((1,), float("nan"), dtype=torch.float32, device="cuda")
+        best = torch.full((1,), -7, dtype=torch.int32, device="cuda")
+        fsb.fs_score_candidates_noalloc(w.K, w.B, w.G, bounds, slo, lam, cand, w.O, w.S, w.seed, 0, rnd,
+                                        gap_dev=gap, score_dev=score, gamma_t_dev=gt, best_dev=best, stream=stream)
+        assert np.array_equal(gap.cpu().numpy(), ref.gap) and np.array_equal(score.cpu().numpy(), ref.score)
+        assert float(gt.item()) == ref.gamma_t and int(best.item()) == ref.best
         assert ref.score.max() > 0
 
 
