@@ -105,10 +105,10 @@ def _env_int(name, default):
         return default
 
 
-def _profiled_traffic(workload: int):
-    """DRAM bytes (read + write) of one k_score launch from the committed ncu
-    summary of this workload, or None when there is none or the scorer source
-    changed since it was taken (its sha256 prefix is recorded in the summary)."""
+def _profile_text(workload: int):
+    """The committed ncu summary of this workload's k_score launch, or None
+    when there is none or the scorer source changed since it was taken (its
+    sha256 prefix is recorded in the summary)."""
     import hashlib
     import re
 
@@ -123,10 +123,47 @@ def _profiled_traffic(workload: int):
     m = re.search(r"sha256 prefix `([0-9a-f]+)`", text)
     if not m or not hashlib.sha256(src).hexdigest().startswith(m.group(1)):
         return None
-    m = re.search(r"dram__bytes_read\.sum \+ dram__bytes_write\.sum \| ([0-9,]+) B \+ ([0-9,]+) B", text)
+    return text
+
+
+def _profiled_traffic(workload: int):
+    """DRAM bytes (read + write) of one k_score launch from the committed ncu summary."""
+    import re
+
+    text = _profile_text(workload)
+    m = re.search(r"dram__bytes_read\.sum \+ dram__bytes_write\.sum \| ([0-9,]+) B \+ ([0-9,]+) B", text or "")
     if not m:
         return None
     return float(m.group(1).replace(",", "")) + float(m.group(2).replace(",", ""))
+
+
+def _profiled_pipes(workload: int):
+    """The busiest execution units of one k_score launch from the committed ncu
+    summary (fractions of their peak): the integer multiplier (fmaheavy pipe,
+    the unit Philox4x32-10's 32x32->64 products run on), the ALU pipe and the
+    issue slots. None when the summary is missing or stale."""
+    import re
+
+    text = _profile_text(workload)
+    if not text:
+        return None
+    out = {}
+    m = re.search(r"sm__pipe_fmaheavy_cycles_active \(of peak, elapsed\) \| ([0-9.]+) %", text)
+    if m:
+        out["fmaheavy_busy"] = float(m.group(1)) / 100.0
+    m = re.search(r"sm__inst_executed_pipe_alu / _fma / _lsu \(of peak, active\) \| ([0-9.]+) %", text)
+    if m:
+        out["alu_busy"] = float(m.group(1)) / 100.0
+    m = re.search(r"smsp__issue_active \(of peak, active\) \| ([0-9.]+) %", text)
+    if m:
+        out["issue_active"] = float(m.group(1)) / 100.0
+    if not out:
+        return None
+    out["source"] = f"ncu, profiles/{PROFILES[workload]}"
+    busiest = max(("integer multiplier (fmaheavy)", out.get("fmaheavy_busy", 0.0)),
+                  ("ALU", out.get("alu_busy", 0.0)), ("issue", out.get("issue_active", 0.0)), key=lambda x: x[1])
+    out["binding"] = busiest[0] if busiest[1] >= 0.5 else "latency (no unit half busy)"
+    return out
 
 
 def _measured_peaks():
@@ -301,7 +338,7 @@ def other_workload(idx: int, steps: int, warmup: int, alu_peak: float, stream_id
             "kernel_ms_per_launch": kern_s * 1000.0,
             "roofline": {"bound": "alu", "achieved": achieved / 1e12, "peak": alu_peak / 1e12,
                          "unit": "Tops/s (32-bit thread operations)", "frac": achieved / alu_peak,
-                         "traffic": _profiled_traffic(idx)}}
+                         "traffic": _profiled_traffic(idx), "pipes": _profiled_pipes(idx)}}
 
 
 def oracle_prefix(w, seconds_target: float):
@@ -696,7 +733,8 @@ def main(argv=None):
                 "gate_tested_scenarios_per_launch": gated_per_launch,
                 "path": "table" if table_path(w.O, w.S) else "plain",
                 "peak_basis": f"{sms} SMs x 4 issue slots x 32 lanes x {sm_max:.0f} MHz (max SM clock)",
-                "kernel_share_of_step": (kern_s * 1000.0 / (sum(step_ms) / len(step_ms))) if kernel_n else None}
+                "kernel_share_of_step": (kern_s * 1000.0 / (sum(step_ms) / len(step_ms))) if kernel_n else None,
+                "pipes": _profiled_pipes(args.workload)}
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(w)
