@@ -411,7 +411,7 @@ __global__ void __launch_bounds__(256, 2) k_score_goodput(Set set, Items it, Pla
   const int W = pl.W, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = blockDim.x >> 5;
   const int gt_len = RF ? 2 * W : W + 1;
   const GoodputSmem lay = goodput_smem(d.K4, d.G, gt_len, nwarp);
-  uint2* gtab = reinterpret_cast<uint2*>(smraw + lay.gtab);
+  uint64_t* gtab = reinterpret_cast<uint64_t*>(smraw + lay.gtab);
   float* cap = reinterpret_cast<float*>(smraw + lay.cap);          // [2][gt_len]
   long long* val = reinterpret_cast<long long*>(smraw + lay.val);  // [2][gt_len]
   uint8_t* flag = smraw + lay.flag;  // bit 0 / 1: a run starts here (realisation 0 / 1); bit 2: reachable
@@ -526,11 +526,10 @@ __global__ void __launch_bounds__(256, 2) k_score_goodput(Set set, Items it, Pla
       if (!(flag[k] & 4)) continue;
       const long long g0 = val[k], g1 = val[gt_len + k];
       const unsigned long long gap = (unsigned long long)(g1 > g0 ? g1 - g0 : g0 - g1);
-      gtab[k] = make_uint2((uint32_t)(gap >> 20), (uint32_t)gap & 0xFFFFFu);
+      gtab[k] = gap;
     }
     __syncthreads();
-    const GtabSum gs = sample_gtab<true, RF>(pl, keys, o, cell, 0, pl.calls, smem_u32(gtab), kgs16);
-    unsigned long long v = gs.total + ((unsigned long long)gs.h << 20) + gs.l;
+    unsigned long long v = sample_gtab<true, RF>(pl, keys, o, cell, 0, pl.calls, smem_u32(gtab), kgs16);
     for (int off = 16; off; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
     if (lane == 0 && v) atomicAdd(reinterpret_cast<unsigned long long*>(&sums[(size_t)seg]), v);
     __syncthreads();  // the tables are rebuilt for the next segment

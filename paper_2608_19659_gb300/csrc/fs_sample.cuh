@@ -19,28 +19,21 @@ __device__ __forceinline__ float row_cap(const RowCap& r, float cy, bool g) {
   return fmaxf(g ? fmaxf(r.po, cy) : r.pc, fminf(fmaxf(cy, r.lf), r.hf));
 }
 
-// Philox calls [q_lo, q_hi) of one segment on the table path: the sums of the
-// two fields of the drawn entries (each field below 2^21), flushed into a
-// 64-bit total every 256 calls so that the 32-bit sums cannot wrap. With at
-// most 32 values per thread nothing is flushed and a warp's field sums stay
-// below 2^32. Per sample: the capacity position floor(word W / 2^32), the
-// word's top w bits for W = 2^w; the tail gate,
-// (word & 0xFFFF) < kgs, as (word * 65536 mod 2^32) < kgs16 with kgs16 =
-// min(kgs 2^16, 2^32 - 1) (a multiply-add and a compare); the entry's shared
-// address base + index * 8 (a multiply-add); its load and two field sums. Two
-// calls per iteration give two independent Philox chains. KC: one problem, its
-// round keys read from the plan. GATE = false: the stratum's tail gate is the
-// same at every position (its mapped tails all pass the SLO, or none does;
-// known from the preparation's gate position), so the entry is the capacity
-// position's in the table at gtab_s with a stride of `stride` bytes (the open
-// half, or under the prior the closed half; without the prior a closed
-// stratum's entries are all the closed-gate value, stored once: stride 0, so
-// a warp's loads are one broadcast) and no scenario tests the gate.
-struct GtabSum {
-  uint32_t h, l;   // the last at most 1024 values
-  uint64_t total;  // earlier values
-};
-
+// Philox calls [q_lo, q_hi) of one segment on the table path: the sum of the
+// drawn entries (each rint(gap 2^40) <= 2^40, stored as one 64-bit word).
+// Per sample: the capacity position floor(word W / 2^32), the word's top w
+// bits for W = 2^w; the tail gate, (word & 0xFFFF) < kgs, as
+// (word * 65536 mod 2^32) < kgs16 with kgs16 = min(kgs 2^16, 2^32 - 1) (a
+// multiply-add and a compare); the entry's shared address base + index * 8 (a
+// multiply-add); its load and one 64-bit add. Two calls per iteration give two
+// independent Philox chains. KC: one problem, its round keys read from the
+// plan. GATE = false: the stratum's tail gate is the same at every position
+// (its mapped tails all pass the SLO, or none does; known from the
+// preparation's gate position), so the entry is the capacity position's in
+// the table at gtab_s with a stride of `stride` bytes (the open half, or under
+// the prior the closed half; without the prior a closed stratum's entries are
+// all the closed-gate value, stored once: stride 0, so a warp's loads are one
+// broadcast) and no scenario tests the gate.
 template <bool KC>
 __device__ __forceinline__ uint4 draw_call(const Plan& pl, const PhiloxKeys& keys, uint32_t q, uint32_t ctr1,
                                            uint32_t ctr2, uint32_t ctr3) {
@@ -49,22 +42,21 @@ __device__ __forceinline__ uint4 draw_call(const Plan& pl, const PhiloxKeys& key
 }
 
 template <bool KC, bool RF, bool GATE = true>
-__device__ __forceinline__ GtabSum sample_gtab(const Plan& pl, const PhiloxKeys& keys, int o, int cell, int q_lo,
-                                               int q_hi, uint32_t gtab_s, uint32_t kgs16, uint32_t stride = 8u) {
+__device__ __forceinline__ uint64_t sample_gtab(const Plan& pl, const PhiloxKeys& keys, int o, int cell, int q_lo,
+                                                int q_hi, uint32_t gtab_s, uint32_t kgs16, uint32_t stride = 8u) {
   const uint32_t ctr1 = (uint32_t)o, ctr2 = (uint32_t)cell, ctr3 = pl.round;
   const uint32_t W = (uint32_t)pl.W, w = (uint32_t)pl.w;
   const uint32_t mul = pl.lo16_mul, eb = GATE ? pl.entry_bytes : stride;
-  uint32_t gh = 0, glo = 0;
+  uint64_t total = 0;
   auto take = [&](uint32_t word) {
     // capacity position floor(word W / 2^32): W = 2^w, so the word's top w
     // bits, taken by a funnel shift (0 for w = 0) on the shift unit rather
     // than the integer multiplier, which the Philox rounds keep busy
     const uint32_t cap = __funnelshift_lc(word, 0u, w);
     const uint32_t idx = !GATE ? cap : word * mul < kgs16 ? cap : (RF ? cap + W : W);
-    uint32_t a, b;
-    asm volatile("ld.shared.v2.u32 {%0, %1}, [%2];" : "=r"(a), "=r"(b) : "r"(gtab_s + idx * eb));
-    gh += a;
-    glo += b;
+    uint64_t a;
+    asm volatile("ld.shared.u64 %0, [%1];" : "=l"(a) : "r"(gtab_s + idx * eb));
+    total += a;
   };
   auto take4 = [&](const uint4& x) {
     take(x.x);
@@ -74,24 +66,16 @@ __device__ __forceinline__ GtabSum sample_gtab(const Plan& pl, const PhiloxKeys&
   };
   const int q_full = min(q_hi, pl.S >> 2);  // calls whose four samples all exist
   const int step = (int)blockDim.x;
-  uint64_t total = 0;
   int q = q_lo + (int)threadIdx.x;
-  while (q < q_full) {
-    const int q_end = min(q_full, q + 256 * step);
-    for (; q + step < q_end; q += 2 * step) {
-      const uint4 x0 = draw_call<KC>(pl, keys, (uint32_t)q, ctr1, ctr2, ctr3);
-      const uint4 x1 = draw_call<KC>(pl, keys, (uint32_t)(q + step), ctr1, ctr2, ctr3);
-      take4(x0);
-      take4(x1);
-    }
-    if (q < q_end) {
-      take4(draw_call<KC>(pl, keys, (uint32_t)q, ctr1, ctr2, ctr3));
-      q += step;
-    }
-    if (q < q_full) {
-      total += ((uint64_t)gh << 20) + glo;
-      gh = glo = 0;
-    }
+  for (; q + step < q_full; q += 2 * step) {
+    const uint4 x0 = draw_call<KC>(pl, keys, (uint32_t)q, ctr1, ctr2, ctr3);
+    const uint4 x1 = draw_call<KC>(pl, keys, (uint32_t)(q + step), ctr1, ctr2, ctr3);
+    take4(x0);
+    take4(x1);
+  }
+  if (q < q_full) {
+    take4(draw_call<KC>(pl, keys, (uint32_t)q, ctr1, ctr2, ctr3));
+    q += step;
   }
   if (q < q_hi) {  // the segment's last call, serving S mod 4 samples
     const uint4 x = draw_call<KC>(pl, keys, (uint32_t)q, ctr1, ctr2, ctr3);
@@ -100,7 +84,7 @@ __device__ __forceinline__ GtabSum sample_gtab(const Plan& pl, const PhiloxKeys&
     if (nv > 1) take(x.y);
     if (nv > 2) take(x.z);
   }
-  return GtabSum{gh, glo, total};
+  return total;
 }
 
 }  // namespace fs

@@ -844,13 +844,12 @@ __device__ uint64_t run_piece_dump(const Set& set, const Plan& pl, int item, int
 // Cexcl that the preparation stored (H_TCL); the block evaluates the W others
 // once per chunk (two t* each, the same arithmetic as a scenario), after which
 // a scenario costs its share of the Philox call, one index and one
-// shared-memory load. Each entry holds the value's upper bits (>> 20) and
-// lower 20 bits, summed separately.
+// shared-memory load. Each entry is the value as one 64-bit word.
 // RF: under the monotone prior the closed-gate values also depend on the
 // position (the draw refits the row's other bins): entries [W, 2W) hold them,
 // evaluated when `closed` (the open half when `open`).
 template <bool TS, int ROW, bool FL, bool RF>
-__device__ __forceinline__ void build_gtab(uint2* gtab, int W, const float* win, const float* h0, const float* h1,
+__device__ __forceinline__ void build_gtab(uint64_t* gtab, int W, const float* win, const float* h0, const float* h1,
                                            const float* kap0, const float* thx0, const float* mnx0,
                                            const float* kap1, const float* thx1, const float* mnx1,
                                            bool open = true, bool closed = false) {
@@ -868,7 +867,7 @@ __device__ __forceinline__ void build_gtab(uint2* gtab, int W, const float* win,
     const float t0 = tstar_of<ROW, FL>(c0, kap0, thx0, mnx0, st0, lam, rlam, dl);
     const float t1 = tstar_of<ROW, FL>(c1, kap1, thx1, mnx1, st1, lam, rlam, dl);
     const uint64_t gv = fixed40(__fsub_rn(t1, t0));
-    gtab[k] = make_uint2((uint32_t)(gv >> 20), (uint32_t)gv & 0xFFFFFu);
+    gtab[k] = gv;
   }
 }
 
@@ -924,7 +923,7 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
   float* stage0 = reinterpret_cast<float*>(smraw + 16);
   const int stage_floats = pl.Wp + 2 * sg.tcopy;
   // GT: two tables of W + 1 entries (2W under the prior), used by alternate chunks
-  uint2* gtab2 = reinterpret_cast<uint2*>(smraw + 16 + (size_t)2 * stage_floats * 4);
+  uint64_t* gtab2 = reinterpret_cast<uint64_t*>(smraw + 16 + (size_t)2 * stage_floats * 4);
   const int gt_len = RF ? 2 * pl.W : pl.W + 1;
   // per stage: chunk index, its segment and its part (thread 0 divides once)
   __shared__ int s_chunk[2], s_seg[2], s_part[2];
@@ -952,9 +951,9 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
     next = (int)blockIdx.x + g;  // may pass sg.total: then the block stops after one chunk
   }
   // 32-bit warp sums are exact while a thread holds at most 32 values (the
-  // table path's fields are below 2^21: at most 64 values)
+  // table path splits its 64-bit sums: at most 128 values)
   const bool small = sg.chunk <= 8 * (int)blockDim.x;
-  const bool small_gt = sg.chunk <= 16 * (int)blockDim.x;
+  const bool small_gt = sg.chunk <= 32 * (int)blockDim.x;
   PhiloxKeys keys;
   int keys_p = -1;  // problem whose round keys are in `keys`
 
@@ -993,7 +992,7 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
       // the gate position) come before it, so thread 0 may refill the stage
       // next iteration, and the next chunk builds the other table while a late
       // thread may still draw from this one.
-      uint2* gtab = gtab2 + (size_t)(j & 1) * gt_len;
+      uint64_t* gtab = gtab2 + (size_t)(j & 1) * gt_len;
       const int cell = ok ? __float_as_int(h0[H_CELL]) : -1;
       const bool use = cell >= 0 && cell < d.cells;  // a bad device-side id was flagged by k_prep
       // passing tail positions of the stratum, as the top bits of a 16-bit field
@@ -1001,17 +1000,16 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
       const uint32_t kgs16 = (uint32_t)min((unsigned long long)kgs << 16, 0xFFFFFFFFull);
       if (use) {
         const uint64_t gc = fixed40(__fsub_rn(h1[H_TCL], h0[H_TCL]));
-        const uint2 closed = make_uint2((uint32_t)(gc >> 20), (uint32_t)gc & 0xFFFFFu);
         // under the prior: the halves the stratum's gate positions can reach
         const bool any_open = kgs != 0u, any_closed = kgs16 != 0xFFFFFFFFu;
         if (!RF && kgs == 0u) {
           // the gate is closed at every position of the stratum: every entry
           // is the closed-gate value, stored once at W (each scenario still
           // draws its position and loads its entry, with stride 0)
-          if (tid == 0) gtab[pl.W] = closed;
+          if (tid == 0) gtab[pl.W] = gc;
         } else {
           if (tid == 0) {
-            if (!RF) gtab[pl.W] = closed;
+            if (!RF) gtab[pl.W] = gc;
             // entries evaluated, once per segment (later chunks of a segment
             // rebuild the same table): the measurement's algorithmic count
             const int halves = RF ? (any_open ? 1 : 0) + (any_closed ? 1 : 0) : 1;
@@ -1056,7 +1054,7 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
         if (s_chunk[st ^ 1] < sg.total) mbar_wait(&bar[st ^ 1], (uint32_t)(((j + 1) >> 1) & 1), kWaitLimitNs);
         return;
       }
-      GtabSum gs{0u, 0u, 0ull};
+      uint64_t gs = 0;
       if (use) {
         if (kgs == 0u || kgs16 == 0xFFFFFFFFu)  // the gate is the same at every position
           gs = sample_gtab<KC, RF, false>(pl, keys, o, cell, q_lo, q_hi,
@@ -1066,12 +1064,15 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
           gs = sample_gtab<KC, RF, true>(pl, keys, o, cell, q_lo, q_hi, smem_u32(gtab), kgs16);
       }
       uint64_t v;
-      if (small_gt) {  // at most 64 values per thread: each field's warp sum fits in 32 bits
-        const uint32_t H = __reduce_add_sync(0xffffffffu, gs.h);
-        const uint32_t Lo = __reduce_add_sync(0xffffffffu, gs.l);
-        v = ((uint64_t)H << 20) + (uint64_t)Lo;
+      if (small_gt) {
+        // at most 128 values per thread (each at most 2^40): the total's bits
+        // above bit 21 are at most 2^26 and the low 21 bits below 2^21, so
+        // each part's warp sum fits in 32 bits
+        const uint32_t H = __reduce_add_sync(0xffffffffu, (uint32_t)(gs >> 21));
+        const uint32_t Lo = __reduce_add_sync(0xffffffffu, (uint32_t)gs & 0x1FFFFFu);
+        v = ((uint64_t)H << 21) + (uint64_t)Lo;
       } else {
-        v = gs.total + ((uint64_t)gs.h << 20) + gs.l;
+        v = gs;
         for (int off = 16; off; off >>= 1) v += __shfl_down_sync(0xffffffffu, v, off);
       }
       if (lane == 0 && v) atomicAdd(reinterpret_cast<unsigned long long*>(&sums[(size_t)seg]), (unsigned long long)v);
@@ -1235,57 +1236,73 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
 #undef FS_KERN
   const void* kfun = reinterpret_cast<const void*>(kern);
   if (smem != lc.score_smem[v][mode]) {
-    int per_sm = 0;
     cudaError_t e = raise_smem_limit(kfun, smem);
-    if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kfun, kScoreThreads, smem);
+    for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
+      int per_sm = 0;
+      e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kfun, kScoreThreads >> b, smem);
+      lc.score_blocks_per_sm[v][mode][b] = per_sm < 1 ? 1 : per_sm;
+    }
     if (e != cudaSuccess) return e;
     lc.score_smem[v][mode] = smem;
-    lc.score_blocks_per_sm[v][mode] = per_sm < 1 ? 1 : per_sm;
   }
   // Chunks of U calls per thread: about eight chunks per resident block when
   // the work allows, so that the counter can even out the segments' unequal
   // costs; at least 2 (a chunk's set-up is then paid for eight samples per
   // thread, measured faster on small launches) and at most 8 calls per
-  // thread (16 on the table path, whose chunks also build a table), and no
-  // more than a segment holds.
-  const long long resident = (long long)lc.score_blocks_per_sm[v][mode] * sm_count;
+  // thread, and no more than a segment holds.
+  int bt = kScoreThreads;
+  long long resident = (long long)lc.score_blocks_per_sm[v][mode][0] * sm_count;
   const long long total_calls = (long long)it.n * pl.O * pl.calls;
-  long long U = total_calls / ((long long)kScoreThreads * resident * 8);
-  const long long u_seg = ((long long)pl.calls + kScoreThreads - 1) / kScoreThreads;
-  if (U > (table ? 16 : 8)) U = table ? 16 : 8;
+  long long U = total_calls / ((long long)bt * resident * 8);
+  long long u_seg = ((long long)pl.calls + bt - 1) / bt;
+  if (U > 8) U = 8;
   if (U < 2) U = 2;
   if (U > u_seg) U = u_seg;
   if (table) {
-    // every chunk builds its segment's table first: pick the chunk length that
-    // minimises rounds of chunks per block x (build + draws), in units of about
-    // one thread-instruction (an entry ~60 per thread share, a call's four draws ~72)
+    // Every chunk pays a fixed set-up (its records' wait, header reads, the
+    // barrier, the reduction and its atomic) and builds its segment's table
+    // before it draws. Pick the block size (256 or 128 threads) and the chunk
+    // length (up to 4096 calls per chunk) that minimise rounds of chunks per
+    // block x resident threads per SM x (set-up + build + draws), in units of
+    // about one thread-instruction: set-up ~180 per thread, an entry ~60 per
+    // thread share, a call's four draws ~72. Smaller blocks give each thread
+    // more of a segment's calls, so the set-up is paid fewer times.
     const long long n_seg = (long long)it.n * pl.O;
-    const long long build = ((pl.W + 1 + kScoreThreads - 1) / kScoreThreads) * 60;
     long long best = -1;
-    for (long long u = 2; u <= std::min<long long>(16, u_seg); ++u) {
-      const long long nch_u = (pl.calls + kScoreThreads * u - 1) / (kScoreThreads * u);
-      const long long rounds = (n_seg * nch_u + resident - 1) / resident;
-      const long long cost = rounds * (build + 72 * u);
-      if (best < 0 || cost < best) {
-        best = cost;
-        U = u;
+    for (int b = 0; b < 2; ++b) {
+      const int tb = kScoreThreads >> b;
+      const long long res_b = (long long)lc.score_blocks_per_sm[v][mode][b] * sm_count;
+      const long long us_b = ((long long)pl.calls + tb - 1) / tb;
+      const long long build = ((pl.W + 1 + tb - 1) / tb) * 60;
+      const long long u_hi = std::min<long long>(4096 / tb, us_b);
+      for (long long u = std::min<long long>(2, us_b); u <= u_hi; ++u) {
+        const long long nch_u = (pl.calls + tb * u - 1) / (tb * u);
+        const long long rounds = (n_seg * nch_u + res_b - 1) / res_b;
+        const long long cost = rounds * lc.score_blocks_per_sm[v][mode][b] * tb * (180 + build + 72 * u);
+        if (best < 0 || cost < best) {
+          best = cost;
+          U = u;
+          bt = tb;
+          resident = res_b;
+          u_seg = us_b;
+        }
       }
     }
   }
   // chunk indices are 32-bit: widen the chunks until they fit (one chunk per
   // segment gives n O <= 2^30 chunks, which the entry points guarantee)
-  long long nch = (pl.calls + kScoreThreads * U - 1) / (kScoreThreads * U);
+  long long nch = (pl.calls + bt * U - 1) / (bt * U);
   while ((long long)it.n * pl.O * nch >= (1LL << 31) && U < u_seg) {
     U *= 2;
-    nch = (pl.calls + kScoreThreads * U - 1) / (kScoreThreads * U);
+    nch = (pl.calls + bt * U - 1) / (bt * U);
   }
   if ((long long)it.n * pl.O * nch >= (1LL << 31)) return cudaErrorInvalidValue;
-  sg.chunk = (int)(kScoreThreads * U);
+  sg.chunk = (int)(bt * U);
   sg.nch = (int)nch;
   sg.total = (int)((long long)it.n * pl.O * nch);
   const int grid = (int)(sg.total < resident ? sg.total : resident);
   sg.dyn = sg.total >= 4LL * grid ? 1 : 0;
-  return launch_pdl(kern, dim3(grid), dim3(kScoreThreads), smem, s, set, it, pl, tables, sums,
+  return launch_pdl(kern, dim3(grid), dim3(bt), smem, s, set, it, pl, tables, sums,
                     (unsigned char*)dump, dump ? dump_stride : 0, sg);
 }
 

@@ -215,7 +215,8 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
       for (int v = 0; v < kScoreVariants; ++v)
         if (lc.score_smem[v][f] && lc.score_smem[v][f] != g.score_smem[v][f]) {
           g.score_smem[v][f] = lc.score_smem[v][f];
-          g.score_blocks_per_sm[v][f] = lc.score_blocks_per_sm[v][f];
+          g.score_blocks_per_sm[v][f][0] = lc.score_blocks_per_sm[v][f][0];
+          g.score_blocks_per_sm[v][f][1] = lc.score_blocks_per_sm[v][f][1];
         }
     }
   }
