@@ -53,7 +53,7 @@ ISSUE_PER_SM_CLK = 4 * 32  # 4 schedulers x 32 lanes, one warp instruction each 
 #   exact fixed-point accumulation of rint(Gamma' 2^40)                   7
 # Table path (a segment's W + 1 values of rint(Gamma' 2^40) tabulated once):
 # per scenario the Philox share (10), capacity position (1), the entry's load
-# (1) and its two field sums (2) = 14, plus the tail gate's test (mask,
+# (1) and its 64-bit sum (two 32-bit adds: 2) = 14, plus the tail gate's test (mask,
 # compare, index select: 3) in the scenarios of strata whose tails lie on both
 # sides of the SLO (elsewhere the gate is the same at every position); per
 # table entry evaluated the two patched capacities (2), two table searches (6),
@@ -76,6 +76,32 @@ def table_path(O: int, S: int) -> bool:
     the smaller of S and a minimum chunk of 2048 samples)."""
     W = Q_TABLE // O
     return W <= 4096 and 3 * (W + 1) <= 2 * min(S, 2048)
+
+
+def draw_floors(w, kernel_ms: float, reps: int = 10):
+    """The Monte-Carlo kernel against measured floors of its draws: the same
+    number of Philox4x32-10 calls (counters as the scorer's) on the table
+    path's 128-thread grid, timed alone and with the table path's per-sample
+    lookup and sum (fs_draw_floor; no chunks, staging, table builds or
+    barriers), scaled to the workload's calls. Table path only."""
+    import math
+
+    from paper_2608_19659_gb300 import fleetsieve as fsb
+
+    if not table_path(w.O, w.S):
+        return None
+    calls = len(w.candidates) * w.O * ((w.S + 3) // 4)
+    wbits = int(math.log2(Q_TABLE // w.O))
+    out = {"calls_per_launch": calls, "kernel_ms": kernel_ms}
+    for mode, key in ((0, "philox_only_ms"), (1, "philox_and_lookup_ms")):
+        ms, done = fsb.fs_draw_floor(mode, wbits, calls, reps)
+        out[key] = ms * calls / done
+    out["frac_of_philox_only"] = out["philox_only_ms"] / kernel_ms
+    out["frac_of_philox_and_lookup"] = out["philox_and_lookup_ms"] / kernel_ms
+    out["basis"] = ("median of %d launches each (after 3 untimed) of fs_draw_floor mode 0 (draws alone) and "
+                    "mode 1 (draws + position, entry load and 64-bit sum from a %d-entry shared table), "
+                    "scaled from the calls one launch made to the workload's" % (reps, (Q_TABLE // w.O) + 1))
+    return out
 
 
 def algorithmic_ops(w, entries_per_launch=None, gated_per_launch=None) -> float:
@@ -601,6 +627,7 @@ def main(argv=None):
     ap.add_argument("--kernel-pass-s", type=float, default=1.0,
                     help="least duration of the kernel-timing pass (0: --steps steps)")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end pass (profiling runs)")
+    ap.add_argument("--no-floors", action="store_true", help="skip the draw-floor measurement (profiling runs)")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         args.warmup = 3
@@ -735,6 +762,9 @@ def main(argv=None):
                 "peak_basis": f"{sms} SMs x 4 issue slots x 32 lanes x {sm_max:.0f} MHz (max SM clock)",
                 "kernel_share_of_step": (kern_s * 1000.0 / (sum(step_ms) / len(step_ms))) if kernel_n else None,
                 "pipes": _profiled_pipes(args.workload)}
+    if kernel_n and not args.no_floors:
+        # the binding unit's floor: the integer multiplier serves Philox's products
+        roofline["draw_floors"] = draw_floors(w, kern_s * 1000.0)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(w)

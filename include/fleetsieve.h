@@ -445,6 +445,23 @@ int fs_timing_enable(fs_model *m, int32_t mode);
 int fs_timing_read(fs_model *m, double *kernel_ms, int32_t *launches, double *phase_ms,
                    uint64_t *work_counts);
 
+/*
+ * Measurement floor (not part of the method). Times what the table path's
+ * draws cost without the rest of the scorer, on the current device, over one
+ * wave of 128-thread blocks (the table path's shape on large launches): each
+ * block one segment, each thread an equal share of Philox4x32-10 calls
+ * (counters as the scorer's), at least `calls` calls in all. mode 0: the
+ * draws alone. mode 1: the draws with the table path's per-sample work
+ * (capacity position from the word's top w bits, entry address, shared-memory
+ * load, 64-bit sum) over a table of 2^w + 1 entries, with no chunks, staging,
+ * table builds or barriers. Synchronous; allocates and frees its output
+ * buffer. *ms = median of `reps` launches after three untimed ones;
+ * *calls_done = the calls one launch made (>= calls). FS_EINVAL for a mode
+ * other than 0/1, w outside [0, 12], calls outside [1, 2^36], reps outside
+ * [1, 1000] or a null output.
+ */
+int fs_draw_floor(int32_t mode, int32_t w, int64_t calls, int32_t reps, double *ms, int64_t *calls_done);
+
 /* Kernels this library has launched since it was loaded (all models). */
 uint64_t fs_launch_count(void);
 

@@ -992,6 +992,23 @@ int fs_timing_read(fs_model* m, double* kernel_ms, int32_t* launches, double* ph
   return FS_OK;
 }
 
+int fs_draw_floor(int32_t mode, int32_t w, int64_t calls, int32_t reps, double* ms, int64_t* calls_done) {
+  if (mode != 0 && mode != 1) return fail(FS_EINVAL, "fs_draw_floor: mode must be 0 or 1");
+  if (w < 0 || w > 12) return fail(FS_EINVAL, "fs_draw_floor: w must be in [0, 12]");
+  if (calls < 1 || calls > (1LL << 36)) return fail(FS_EINVAL, "fs_draw_floor: calls must be in [1, 2^36]");
+  if (reps < 1 || reps > 1000) return fail(FS_EINVAL, "fs_draw_floor: reps must be in [1, 1000]");
+  if (!ms || !calls_done) return fail(FS_EINVAL, "fs_draw_floor: null output");
+  int dev = 0, sms = 0;
+  FS_CUDA(cudaGetDevice(&dev), "current device");
+  FS_CUDA(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev), "SM count");
+  long long done = 0;
+  const cudaError_t e = draw_floor(mode, w, calls, reps, sms, ms, &done);
+  if (e == cudaErrorInvalidValue) return fail(FS_EINVAL, "fs_draw_floor: too many calls per thread");
+  if (e != cudaSuccess) return cuda_fail(e, "draw floor");
+  *calls_done = done;
+  return FS_OK;
+}
+
 int fs_watchdog_selftest(int64_t timeout_ns) {
   const int64_t t = std::min<int64_t>(std::max<int64_t>(timeout_ns, 1000000), 5000000000LL);
   uint32_t* st = nullptr;

@@ -497,6 +497,11 @@ cudaError_t launch_finalize(const Set& set, const Items& it, const Plan& pl, con
                             double* gap, double* score, float* gamma_t, int32_t* best, uint32_t* status_copy,
                             uint64_t* part, cudaStream_t s);
 cudaError_t launch_watchdog(uint32_t* status, uint64_t limit_ns, cudaStream_t s);
+// Measurement only: median time of `reps` launches of the table path's draws
+// alone (mode 0) or with its per-sample lookup (mode 1), W = 2^w, at least
+// `calls` Philox calls over one wave of 128-thread blocks (synchronous).
+cudaError_t draw_floor(int mode, int w, long long calls, int reps, int sm_count, double* ms_median,
+                       long long* calls_done);
 
 // tiers 3-4 and the goodput stage (fs_lex.cu)
 constexpr size_t kLexCellBytes = 16;  // one cell of the programme over classes and GPUs

@@ -40,6 +40,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <vector>
 
 #include "fs_finalize.cuh"
 #include "fs_internal.cuh"
@@ -1321,6 +1322,90 @@ cudaError_t launch_finalize(const Set& set, const Items& it, const Plan& pl, con
                       status_copy, part);
   return launch_pdl(k_finalize, dim3(it.off ? set.P : 1), dim3(256), 0, s, set, it, pl, sums, gap, score, gamma_t,
                     best, status_copy);
+}
+
+// ---------------------------------------------------------------- measurement floors (not part of the method)
+
+// What the table path's draws cost without the rest of the scorer. MODE 0:
+// Philox4x32-10 of the table path's counters alone (two chains a thread, the
+// words XORed so that none is dead). MODE 1: the same draws with the table
+// path's per-sample work, sample_gtab over a block-local table of W + 1
+// entries with the gate the same at every position (position, entry address,
+// load and 64-bit sum). No chunks, staging, table builds or barriers: each
+// block takes one segment of per_thread calls a thread. One word per thread out.
+template <int MODE>
+__global__ void __launch_bounds__(kScoreThreads) k_draw_floor(Plan pl, int per_thread, uint64_t* out) {
+  extern __shared__ __align__(16) unsigned char smraw[];
+  uint64_t* tab = reinterpret_cast<uint64_t*>(smraw);
+  for (int k = (int)threadIdx.x; k <= pl.W; k += (int)blockDim.x) tab[k] = (uint64_t)k * 977u;
+  __syncthreads();
+  const int step = (int)blockDim.x, q_hi = per_thread * step;
+  const uint32_t cell = blockIdx.x;
+  uint64_t v = 0;
+  if constexpr (MODE == 1) {
+    const PhiloxKeys keys{};  // not read: one-problem draws take the plan's round keys
+    v = sample_gtab<true, false, false>(pl, keys, 0, (int)cell, 0, q_hi, smem_u32(tab), 0u, 8u);
+  } else {
+    uint32_t acc = 0;
+    int q = (int)threadIdx.x;
+    for (; q + step < q_hi; q += 2 * step) {
+      const uint4 x0 = philox4x32_10_plan(make_uint4((uint32_t)q, 0u, cell, pl.round), pl);
+      const uint4 x1 = philox4x32_10_plan(make_uint4((uint32_t)(q + step), 0u, cell, pl.round), pl);
+      acc ^= x0.x ^ x0.y ^ x0.z ^ x0.w ^ x1.x ^ x1.y ^ x1.z ^ x1.w;
+    }
+    if (q < q_hi) {
+      const uint4 x = philox4x32_10_plan(make_uint4((uint32_t)q, 0u, cell, pl.round), pl);
+      acc ^= x.x ^ x.y ^ x.z ^ x.w;
+    }
+    v = acc;
+  }
+  out[(size_t)blockIdx.x * blockDim.x + threadIdx.x] = v;
+}
+
+cudaError_t draw_floor(int mode, int w, long long calls, int reps, int sm_count, double* ms_median,
+                       long long* calls_done) {
+  const int bt = kScoreThreads / 2;  // the table path's blocks on large launches
+  auto kern = mode == 0 ? k_draw_floor<0> : k_draw_floor<1>;
+  const size_t smem = 8 * (((size_t)1 << w) + 1);
+  int per_sm = 0;
+  cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(kern), smem);
+  if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, bt, smem);
+  if (e != cudaSuccess) return e;
+  const long long grid = (long long)(per_sm < 1 ? 1 : per_sm) * sm_count;
+  const long long per_thread = (calls + grid * bt - 1) / (grid * bt);
+  if (per_thread < 1 || 4 * per_thread * bt > 0x7FFFFFFFLL) return cudaErrorInvalidValue;
+  Plan pl{};
+  pl.key0 = 0x0F1E2D3Cu;
+  pl.key1 = 0x4B5A6978u;
+  pl.W = 1 << w;
+  pl.w = w;
+  pl.S = (int)(4 * per_thread * bt);  // every call of a segment serves four samples
+  plan_round_keys(pl);
+  uint64_t* out = nullptr;
+  cudaEvent_t a = nullptr, b = nullptr;
+  std::vector<float> t;
+  e = cudaMalloc(&out, (size_t)grid * bt * sizeof(uint64_t));
+  if (e == cudaSuccess) e = cudaEventCreate(&a);
+  if (e == cudaSuccess) e = cudaEventCreate(&b);
+  for (int i = 0; e == cudaSuccess && i < reps + 3; ++i) {  // three untimed launches first
+    e = cudaEventRecord(a, 0);
+    note_launch();
+    if (e == cudaSuccess) kern<<<(unsigned)grid, bt, smem, 0>>>(pl, (int)per_thread, out);
+    if (e == cudaSuccess) e = cudaGetLastError();
+    if (e == cudaSuccess) e = cudaEventRecord(b, 0);
+    if (e == cudaSuccess) e = cudaEventSynchronize(b);
+    float ms = 0.0f;
+    if (e == cudaSuccess) e = cudaEventElapsedTime(&ms, a, b);
+    if (e == cudaSuccess && i >= 3) t.push_back(ms);
+  }
+  if (a) cudaEventDestroy(a);
+  if (b) cudaEventDestroy(b);
+  if (out) cudaFree(out);
+  if (e != cudaSuccess) return e;
+  std::sort(t.begin(), t.end());
+  *ms_median = t[t.size() / 2];
+  *calls_done = grid * bt * per_thread;
+  return cudaSuccess;
 }
 
 }  // namespace fs

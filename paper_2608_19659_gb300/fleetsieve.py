@@ -27,7 +27,7 @@ EXPORTS = ("fs_load_model", "fs_update_bounds", "fs_set_floors", "fs_dump_stride
            "fs_certificate", "fs_replay", "fs_check", "fs_launch_count",
            "fs_watchdog_selftest", "fs_free_model", "fs_last_error", "fs_score_candidates_noalloc",
            "fs_timing_enable",
-           "fs_timing_read")
+           "fs_timing_read", "fs_draw_floor")
 
 
 class FleetSieveError(RuntimeError):
@@ -117,6 +117,8 @@ def lib():
         L.fs_timing_read.argtypes = [C.c_void_p, C.POINTER(C.c_double), C.POINTER(C.c_int32),
                                      C.c_void_p, C.c_void_p]
         L.fs_watchdog_selftest.argtypes = [C.c_int64]
+        L.fs_draw_floor.argtypes = [C.c_int32, C.c_int32, C.c_int64, C.c_int32, C.POINTER(C.c_double),
+                                    C.POINTER(C.c_int64)]
         L.fs_free_model.argtypes = [C.c_void_p]
         L.fs_free_model.restype = None
         L.fs_last_error.restype = C.c_char_p
@@ -460,6 +462,15 @@ def fs_timing_read(m: Model, with_entries: bool = False):
 
 def fs_launch_count() -> int:
     return int(lib().fs_launch_count())
+
+
+def fs_draw_floor(mode: int, w: int, calls: int, reps: int = 10):
+    """Measurement floor of the table path's draws (mode 0: Philox alone; 1:
+    with the per-sample lookup): (median ms per launch, calls per launch)."""
+    ms = C.c_double(0.0)
+    done = C.c_int64(0)
+    _check(lib().fs_draw_floor(int(mode), int(w), int(calls), int(reps), C.byref(ms), C.byref(done)))
+    return float(ms.value), int(done.value)
 
 
 def fs_watchdog_selftest(timeout_ns: int) -> int:

@@ -90,3 +90,12 @@ def test_load_model_rejects_bad_input(fsb, case):
         fsb.fs_load_model(clo, chi, tlo, thi, slo, lam, G, K, B, quantile=q, revealed=rev)
     assert ei.value.code == fsb.FS_EINVAL
     assert fsb.fs_last_error()
+
+
+@pytest.mark.parametrize("args", [(2, 8, 1024, 10), (0, 13, 1024, 10), (1, -1, 1024, 10), (0, 8, 0, 10),
+                                  (1, 8, 1 << 40, 10), (0, 8, 1024, 0), (1, 8, 1024, 1001)])
+def test_draw_floor_rejects_bad_arguments(fsb, args):
+    """The measurement floor checks its arguments before touching a device."""
+    with pytest.raises(fsb.FleetSieveError) as ei:
+        fsb.fs_draw_floor(*args)
+    assert ei.value.code == fsb.FS_EINVAL

@@ -263,6 +263,17 @@ def test_watchdog_times_out_cleanly(fsb, cuda):
         fsb.fs_score_candidates(m, w.candidates, 4, 8, 0)
 
 
+def test_draw_floor_measures_both_modes(fsb, cuda):
+    """The measurement floor of the table path's draws runs at least the calls
+    asked for in both modes and leaves the context usable."""
+    for mode in (0, 1):
+        ms, done = fsb.fs_draw_floor(mode, 8, 1 << 20, 3)
+        assert ms > 0.0 and done >= 1 << 20
+    w = workloads.make_workload(0)
+    with load_model(fsb, w) as m:
+        fsb.fs_score_candidates(m, w.candidates, 4, 8, 0)
+
+
 def test_staged_bounds_reach_every_later_call(fsb, cuda, oracle_lib, qn):
     """fs_update_bounds only stages: a synchronous score reads the staged bounds,
     every device-side call after it (asynchronous scoring on another stream,
