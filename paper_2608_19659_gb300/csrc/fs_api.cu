@@ -159,6 +159,7 @@ struct fs_model {
   Set set{};
   // per-call scratch
   Buf cand, tables, sums, outs, real, lex;
+  Buf replay;     // fs_replay's state of every stream (grown on demand, kept)
   int objective = FS_OBJECTIVE_MAXMIN;  // FS_OBJECTIVE_LEXICOGRAPHIC: fs_solve* and the certificate to tier 4
   // host mirrors
   std::vector<float> h_bounds;      // [4][cells]
@@ -349,7 +350,7 @@ int run_score(fs_model* m, const Set& set, const fs_samples* smp, const int32_t*
   if (phases) FS_CUDA(cudaEventRecord(ev[0], s), "record timing event");
   FS_CUDA(launch_solve(set, 2, nullptr, nullptr, nullptr, true, m->lc, s, true), "launch solve");
   if (phases) FS_CUDA(cudaEventRecord(ev[1], s), "record timing event");
-  FS_CUDA(launch_prep(set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, true, m->lc, s), "launch prep");
+  FS_CUDA(launch_prep(set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, true, m->sm_count, m->lc, s), "launch prep");
   if (timed) FS_CUDA(cudaEventRecord(ev[2], s), "record timing event");
   FS_CUDA(launch_score(set, it, pl, (const float*)m->tables.p, (uint64_t*)m->sums.p, dump,
                        fs_dump_stride(m), m->sm_count, m->lc, s),
@@ -771,7 +772,7 @@ int fs_score_goodput(fs_model* m, const fs_samples* smp, double* gap_out, double
   m->objective = saved;
   if (rc) return rc;
   uint64_t* sums = static_cast<uint64_t*>(m->sums.p);
-  FS_CUDA(launch_prep(m->set, it, pl, static_cast<float*>(m->tables.p), sums, false, m->lc, s), "launch prep");
+  FS_CUDA(launch_prep(m->set, it, pl, static_cast<float*>(m->tables.p), sums, false, m->sm_count, m->lc, s), "launch prep");
   FS_CUDA(launch_score_goodput(m->set, it, pl, static_cast<const float*>(m->tables.p), sums, m->lc.floors,
                                m->sm_count, s),
           "launch goodput scorer");
@@ -836,7 +837,8 @@ int fs_replay(fs_model* m, const fs_replay_spec* sp, int32_t* rounds, int32_t* s
   const size_t o_final = take((size_t)P * sizeof(fs_allocation)), o_active = take(4 * (size_t)P), o_nact = take(4);
   const size_t o_ip = take(4 * (size_t)P * cells), o_ic = take(4 * (size_t)P * cells);
   const size_t o_rtab = take(8 * (size_t)P * kRowTabMax);
-  Buf all;
+  const size_t o_prior = take(16 * (size_t)cells);
+  Buf& all = m->replay;
   if ((rc = all.ensure(off, "replay state"))) return rc;
   char* base = (char*)all.p;
   Set set = m->set;
@@ -870,11 +872,10 @@ int fs_replay(fs_model* m, const fs_replay_spec* sp, int32_t* rounds, int32_t* s
   cudaStream_t s = m->stream;
   auto run = [&]() -> int {
     FS_CUDA(cudaMemsetAsync(all.p, 0, off, s), "clear replay state");
-    for (int k = 0; k < P; ++k) {
-      FS_CUDA(cudaMemcpyAsync(set.bounds + (size_t)k * 4 * cells, m->h_bounds.data(), 16 * (size_t)cells,
-                              cudaMemcpyHostToDevice, s),
-              "upload prior");
-    }
+    // the prior once; the init kernel gives every stream its copy
+    float* prior = (float*)(base + o_prior);
+    FS_CUDA(cudaMemcpyAsync(prior, m->h_bounds.data(), 16 * (size_t)cells, cudaMemcpyHostToDevice, s),
+            "upload prior");
     std::vector<float> truth(2 * (size_t)P * cells);
     for (int k = 0; k < P; ++k) {
       std::memcpy(&truth[(2 * (size_t)k) * cells], sp->truth_cap + (size_t)k * cells, 4 * (size_t)cells);
@@ -883,7 +884,7 @@ int fs_replay(fs_model* m, const fs_replay_spec* sp, int32_t* rounds, int32_t* s
     for (auto& v : truth) v = canon(v);
     FS_CUDA(cudaMemcpyAsync((void*)rs.truth, truth.data(), 4 * truth.size(), cudaMemcpyHostToDevice, s), "upload truth");
     FS_CUDA(cudaMemcpyAsync((void*)rs.perm, sp->perm, 4 * (size_t)P * cells, cudaMemcpyHostToDevice, s), "upload perm");
-    FS_CUDA(launch_replay_init(set, rs, sp->r0, s), "launch replay init");
+    FS_CUDA(launch_replay_init(set, rs, prior, sp->r0, s), "launch replay init");
     const int rc_sync = read_status(m, s);  // truth buffer must outlive the copy
     if (rc_sync) return rc_sync;
     for (int r = 0; r <= sp->max_rounds; ++r) {
@@ -911,7 +912,7 @@ int fs_replay(fs_model* m, const fs_replay_spec* sp, int32_t* rounds, int32_t* s
       it.off = nullptr;
       fs_samples smp{sp->seed, 0, (uint32_t)r, n_items, sp->O, sp->S, 0, nullptr};
       const Plan pl = make_plan(m, &smp, n_items);
-      FS_CUDA(launch_prep(set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, false, m->lc, s), "launch prep");
+      FS_CUDA(launch_prep(set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, false, m->sm_count, m->lc, s), "launch prep");
       FS_CUDA(launch_score(set, it, pl, (const float*)m->tables.p, (uint64_t*)m->sums.p, nullptr, 0, m->sm_count,
                            m->lc, s),
               "launch score");
@@ -936,7 +937,6 @@ int fs_replay(fs_model* m, const fs_replay_spec* sp, int32_t* rounds, int32_t* s
   };
   rc = run();
   cudaStreamSynchronize(s);
-  all.release();
   return rc;
 }
 
@@ -1035,6 +1035,7 @@ void fs_free_model(fs_model* m) {
   m->outs.release();
   m->real.release();
   m->lex.release();
+  m->replay.release();
   for (cudaEvent_t e : m->ev) cudaEventDestroy(e);
   if (m->up_done) cudaEventDestroy(m->up_done);
   m->h_up.release();

@@ -484,8 +484,11 @@ cudaError_t launch_solve(const Set& set, int n, const float* cap_x, const float*
                          bool tstar_only = false);
 // early: the candidate ids and bounds were complete before the preceding
 // kernel started, so the bounds-only work may run before the PDL wait.
+// Blocks of 256 threads, or of 64 when the launch holds more than two waves
+// of 256-thread blocks (sm_count SMs): each block is mostly a chain of
+// dependent latencies, so more of them in flight per SM finish sooner.
 cudaError_t launch_prep(const Set& set, const Items& it, const Plan& pl, float* tables,
-                        uint64_t* sums, bool early, LaunchCache& lc, cudaStream_t s);
+                        uint64_t* sums, bool early, int sm_count, LaunchCache& lc, cudaStream_t s);
 cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const float* tables,
                          uint64_t* sums, void* dump, int dump_stride, int sm_count, LaunchCache& lc,
                          cudaStream_t s);
@@ -538,7 +541,9 @@ struct ReplayState {
   int max_rounds;
   float eps;
 };
-cudaError_t launch_replay_init(const Set& set, const ReplayState& rs, int r0, cudaStream_t s);
+// prior: DEVICE [4][cells] bounds every stream starts from.
+cudaError_t launch_replay_init(const Set& set, const ReplayState& rs, const float* prior, int r0,
+                               cudaStream_t s);
 cudaError_t launch_replay_certify(const Set& set, const ReplayState& rs, int round, cudaStream_t s);
 cudaError_t launch_replay_items(const Set& set, const ReplayState& rs, int n_active, int per,
                                 cudaStream_t s);

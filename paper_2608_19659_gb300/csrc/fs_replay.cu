@@ -28,15 +28,21 @@ __device__ __forceinline__ void reveal_cell(const Set& set, const ReplayState& r
   rs.gpu_seconds[p] += 300.0 * (double)(1 << ((c / d.B) & 3));  // 300 s per cell x TP GPUs
 }
 
-__global__ void k_replay_init(Set set, ReplayState rs, int r0) {
-  const int p = blockIdx.x * blockDim.x + threadIdx.x;
-  if (p >= set.P) return;
+// One block per stream: its bounds from the common prior, an empty reveal
+// order, then (thread 0) the initial design's reveals.
+__global__ void k_replay_init(Set set, ReplayState rs, const float* prior, int r0) {
+  const int p = blockIdx.x;
+  const int cells = set.d.cells;
+  float* bp = set.bounds + (size_t)p * 4 * cells;
+  for (int q = threadIdx.x; q < 4 * cells; q += blockDim.x) bp[q] = prior[q];
+  for (int q = threadIdx.x; q < cells; q += blockDim.x) rs.reveal_order[(size_t)p * cells + q] = -1;
+  __syncthreads();
+  if (threadIdx.x != 0) return;
   rs.n_revealed[p] = 0;
   rs.gpu_seconds[p] = 0.0;
   rs.rounds[p] = 0;
   rs.state[p] = -1;
-  for (int q = 0; q < set.d.cells; ++q) rs.reveal_order[(size_t)p * set.d.cells + q] = -1;
-  for (int q = 0; q < r0; ++q) reveal_cell(set, rs, p, rs.perm[(size_t)p * set.d.cells + q]);
+  for (int q = 0; q < r0; ++q) reveal_cell(set, rs, p, rs.perm[(size_t)p * cells + q]);
 }
 
 // Certificate of every running stream; collects the ones that go on.
@@ -71,21 +77,27 @@ __global__ void k_replay_certify(Set set, ReplayState rs, int round) {
 }
 
 // Candidates of running stream slot a: its unrevealed cells in reveal order.
+// One warp per slot: 32 cells of the order at a time, each lane's place in
+// the list from a ballot of the unrevealed ones before it.
 __global__ void k_replay_items(Set set, ReplayState rs, int n_active, int per) {
-  const int a = blockIdx.x * blockDim.x + threadIdx.x;
+  const int a = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
   if (a >= n_active) return;
   const int p = rs.active[a];
   const Dims& d = set.d;
   int q = 0;
-  for (int k = 0; k < d.cells && q < per; ++k) {
-    const int c = rs.perm[(size_t)p * d.cells + k];
-    if (!set.revealed[(size_t)p * d.cells + c]) {
-      rs.item_p[a * per + q] = p;
-      rs.item_cell[a * per + q] = c;
-      ++q;
+  for (int k0 = 0; k0 < d.cells && q < per; k0 += 32) {
+    const int k = k0 + lane;
+    const int c = k < d.cells ? rs.perm[(size_t)p * d.cells + k] : 0;
+    const bool open = k < d.cells && !set.revealed[(size_t)p * d.cells + c];
+    const uint32_t bal = __ballot_sync(0xffffffffu, open);
+    const int at = q + __popc(bal & ((1u << lane) - 1u));
+    if (open && at < per) {
+      rs.item_p[(size_t)a * per + at] = p;
+      rs.item_cell[(size_t)a * per + at] = c;
     }
+    q += __popc(bal);
   }
-  if (q != per) atomicOr(set.status, ST_TABLE);
+  if (lane == 0 && q < per) atomicOr(set.status, ST_TABLE);
 }
 
 // Fixed-order policy: running stream slot a reveals its next unrevealed cell
@@ -112,9 +124,10 @@ __global__ void k_replay_reveal(Set set, ReplayState rs, Items it, Plan pl, cons
   if (threadIdx.x == 0 && b.valid()) reveal_cell(set, rs, p, b.cell);
 }
 
-cudaError_t launch_replay_init(const Set& set, const ReplayState& rs, int r0, cudaStream_t s) {
+cudaError_t launch_replay_init(const Set& set, const ReplayState& rs, const float* prior, int r0,
+                               cudaStream_t s) {
   note_launch();
-  k_replay_init<<<(set.P + 127) / 128, 128, 0, s>>>(set, rs, r0);
+  k_replay_init<<<set.P, 128, 0, s>>>(set, rs, prior, r0);
   return cudaGetLastError();
 }
 
@@ -126,7 +139,7 @@ cudaError_t launch_replay_certify(const Set& set, const ReplayState& rs, int rou
 
 cudaError_t launch_replay_items(const Set& set, const ReplayState& rs, int n_active, int per, cudaStream_t s) {
   note_launch();
-  k_replay_items<<<(n_active + 127) / 128, 128, 0, s>>>(set, rs, n_active, per);
+  k_replay_items<<<(n_active + 3) / 4, 128, 0, s>>>(set, rs, n_active, per);
   return cudaGetLastError();
 }
 

@@ -1194,7 +1194,7 @@ static size_t prep_smem_bytes(const Set& set) {
 }
 
 cudaError_t launch_prep(const Set& set, const Items& it, const Plan& pl, float* tables, uint64_t* sums,
-                        bool early, LaunchCache& lc, cudaStream_t s) {
+                        bool early, int sm_count, LaunchCache& lc, cudaStream_t s) {
   if (it.n <= 0) return cudaSuccess;
   const size_t smem = prep_smem_bytes(set);
   const int fl = lc.floors ? 1 : 0, mode = fl + (set.prior == 1 ? 2 : 0);
@@ -1205,7 +1205,10 @@ cudaError_t launch_prep(const Set& set, const Items& it, const Plan& pl, float* 
     if (e != cudaSuccess) return e;
     lc.prep_smem[mode] = smem;
   }
-  return launch_pdl(kern, dim3(it.n * 2), dim3(kPrepThreads), smem, s, set, it, pl, tables, sums, early ? 1 : 0);
+  // (five 256-thread blocks fit an SM by registers; 64-thread blocks need at
+  // least 64 threads for the classes' demands, K <= 64)
+  const int tb = (long long)it.n * 2 > 2LL * 5 * sm_count ? 64 : kPrepThreads;
+  return launch_pdl(kern, dim3(it.n * 2), dim3(tb), smem, s, set, it, pl, tables, sums, early ? 1 : 0);
 }
 
 static int score_lcap(const Dims& d) { return d.lcap < kSmemTableCap ? d.lcap : kSmemTableCap; }

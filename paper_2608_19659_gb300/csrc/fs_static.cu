@@ -197,7 +197,7 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
   if (e == cudaSuccess && !quantile_dev) e = launch_qtable(const_cast<float*>(set.qn), Q, s);
   if (e == cudaSuccess) e = launch_solve(set, 2, nullptr, nullptr, nullptr, true, lc, s, true);
   if (e == cudaSuccess) e = launch_prep(set, it, pl, reinterpret_cast<float*>(base + o_tab),
-                                        reinterpret_cast<uint64_t*>(base + o_sums), true, lc, s);
+                                        reinterpret_cast<uint64_t*>(base + o_sums), true, sm_count, lc, s);
   if (e == cudaSuccess)
     e = launch_score(set, it, pl, reinterpret_cast<const float*>(base + o_tab),
                      reinterpret_cast<uint64_t*>(base + o_sums), nullptr, 0, sm_count, lc, s);
