@@ -56,17 +56,20 @@ ISSUE_PER_SM_CLK = 4 * 32  # 4 schedulers x 32 lanes, one warp instruction each 
 # (1) and its 64-bit sum (two 32-bit adds: 2) = 14, plus the tail gate's test (mask,
 # compare, index select: 3) in the scenarios of strata whose tails lie on both
 # sides of the SLO (elsewhere the gate is the same at every position); per
-# table entry evaluated the two patched capacities (2), two table searches (6),
-# Gamma' (1), the fixed-point conversion (5) and the store (1) = 15. A segment
-# whose tail gate is closed at every position of its stratum evaluates no
-# entry (all equal the closed-gate value, from the preparation). The library
-# counts the entries evaluated and the scenarios that tested their gate.
-# Search probes beyond the first (3 each) and row-term fulfilments are not
-# counted: lower bounds.
+# table entry with both t* evaluated the two patched capacities (2), two table
+# searches (6), Gamma' (1), the fixed-point conversion (5) and the store (1) =
+# 15, counted as 7.5 per t* evaluated (an entry with one t* evaluated, the
+# other taken from the closed-gate value because its capacity is at or below
+# that realisation's Cexcl, then counts 7.5 of its 11). A segment whose tail
+# gate is closed at every position of its stratum evaluates nothing (every
+# entry equals the closed-gate value, from the preparation). The library
+# counts the t* evaluated and the scenarios that tested their gate. Search
+# probes beyond the first (3 each) and row-term fulfilments are not counted:
+# lower bounds.
 OPS_PER_SCENARIO = 32
 OPS_PER_SCENARIO_TABLE = 14
 OPS_PER_GATE_TEST = 3
-OPS_PER_TABLE_ENTRY = 15
+OPS_PER_TSTAR_EVAL = 7.5  # half of a fully evaluated table entry's 15
 Q_TABLE = 4096  # quantile table size of the built-in triangular table
 
 
@@ -104,19 +107,19 @@ def draw_floors(w, kernel_ms: float, reps: int = 10):
     return out
 
 
-def algorithmic_ops(w, entries_per_launch=None, gated_per_launch=None) -> float:
+def algorithmic_ops(w, tstar_evals_per_launch=None, gated_per_launch=None) -> float:
     """Algorithmic thread-operations of one Monte-Carlo launch over workload w:
-    on the table path, with the gap-table entries the launch evaluated and the
+    on the table path, with the t* its gap-table builds evaluated and the
     scenarios that tested their tail gate (as the library counted them; None:
-    W entries and a gate test in every segment)."""
+    both t* of W entries and a gate test in every segment)."""
     if table_path(w.O, w.S):
         W = Q_TABLE // w.O
-        if entries_per_launch is None:
-            entries_per_launch = float(len(w.candidates)) * w.O * W
+        if tstar_evals_per_launch is None:
+            tstar_evals_per_launch = 2.0 * len(w.candidates) * w.O * W
         if gated_per_launch is None:
             gated_per_launch = float(w.scenarios)
         return (float(OPS_PER_SCENARIO_TABLE) * w.scenarios + OPS_PER_GATE_TEST * float(gated_per_launch)
-                + OPS_PER_TABLE_ENTRY * float(entries_per_launch))
+                + OPS_PER_TSTAR_EVAL * float(tstar_evals_per_launch))
     return float(OPS_PER_SCENARIO) * w.scenarios
 
 # ncu summaries with the DRAM bytes of one k_score launch, per workload; used
@@ -348,12 +351,12 @@ def other_workload(idx: int, steps: int, warmup: int, alu_peak: float, stream_id
         flush.zero_()
         step()
     torch.cuda.synchronize()
-    kernel_ms, kernel_n, _, (entries, gated) = fsb.fs_timing_read(m, with_entries=True)
+    kernel_ms, kernel_n, _, (evals, gated) = fsb.fs_timing_read(m, with_entries=True)
     fsb.fs_timing_enable(m, 0)
     fsb.fs_check(m, stream)
     fsb.fs_free_model(m)
     kern_s = kernel_ms / 1000.0 / max(kernel_n, 1)
-    achieved = algorithmic_ops(w, entries / max(kernel_n, 1), gated / max(kernel_n, 1)) / kern_s
+    achieved = algorithmic_ops(w, evals / max(kernel_n, 1), gated / max(kernel_n, 1)) / kern_s
     gamma_t = float(gt.item())
     return {"workload": w.name, "ms_per_step": step_ms, "scenarios_per_s": w.scenarios / (step_ms / 1000.0),
             "gamma_t": gamma_t,
@@ -575,6 +578,12 @@ def replay_entry(stream, alu_peak):
             "certified": int((res.state == 1).sum()), "candidate_scores": int(cand_rounds),
             "scenarios": int(scen), "allocation_solves_per_s": 2.0 * scen / wall,
             "candidate_scores_per_s": cand_rounds / wall,
+            "roofline": {"bound": "alu", "achieved": OPS_PER_SCENARIO_TABLE * scen / wall / 1e12,
+                         "peak": alu_peak / 1e12, "unit": "Tops/s (32-bit thread operations)",
+                         "frac": OPS_PER_SCENARIO_TABLE * scen / wall / alu_peak,
+                         "basis": "14 thread-operations per scenario (the table path's per-scenario count; "
+                                  "table builds, gate tests and every other phase of the round loop not "
+                                  "counted: a lower bound) over the whole replay's wall clock"},
             "cpu_baseline": {"value": 2.0 * o_scen / odt, "unit": UNIT, "cores": 1, "kind": "oracle",
                              "sample": f"stream 0, rounds 0-1 ({o_scen} scenarios, {odt:.1f} s)"}}
 
@@ -692,7 +701,7 @@ def main(argv=None):
         # (at least about a second of them, so that the clock samples taken
         # every 200 ms see the GPU under this load)
         fsb.fs_timing_read(model)
-        fsb.fs_timing_enable(model, 1)  # (also zeroes the library's count of table entries)
+        fsb.fs_timing_enable(model, 1)  # (also zeroes the library's work counts)
         per_step_s = max(sum(step_ms_of(starts, ends)) / 1000.0 / args.steps, 1e-6)
         n2 = max(args.steps, min(4000, int(args.kernel_pass_s / per_step_s)))
         for k in range(n2):
@@ -701,7 +710,7 @@ def main(argv=None):
             if (k + 1) % 1000 == 0:  # the library keeps up to 4096 timed calls
                 torch.cuda.synchronize()
         torch.cuda.synchronize()
-        kernel_ms, kernel_n, _, (entries, gated) = fsb.fs_timing_read(model, with_entries=True)
+        kernel_ms, kernel_n, _, (evals, gated) = fsb.fs_timing_read(model, with_entries=True)
         fsb.fs_timing_enable(model, 0)
     step_ms = step_ms_of(starts, ends)
     total_ms = max_over_ranks(dist, sum(step_ms), dev)
@@ -745,9 +754,9 @@ def main(argv=None):
     sms = torch.cuda.get_device_properties(dev).multi_processor_count
     alu_peak = sms * ISSUE_PER_SM_CLK * sm_max * 1e6  # thread-ops/s at the maximum SM clock
     kern_s = kernel_ms / 1000.0 / max(kernel_n, 1)
-    entries_per_launch = entries / max(kernel_n, 1)
+    evals_per_launch = evals / max(kernel_n, 1)
     gated_per_launch = gated / max(kernel_n, 1)
-    ops = algorithmic_ops(w, entries_per_launch, gated_per_launch)
+    ops = algorithmic_ops(w, evals_per_launch, gated_per_launch)
     achieved = ops / kern_s if kernel_n else None
     roofline = {"bound": "alu", "kernel": "k_score (Monte-Carlo sampler + parametric re-solve)",
                 "achieved": achieved / 1e12 if achieved else None,
@@ -756,7 +765,7 @@ def main(argv=None):
                 "traffic": _profiled_traffic(args.workload), "traffic_unit": "DRAM bytes per launch (ncu)",
                 "algorithmic_bytes": 0, "kernel_ms_per_launch": kern_s * 1000.0,
                 "ops_per_scenario": ops / w.scenarios,
-                "table_entries_per_launch": entries_per_launch,
+                "tstar_evaluations_per_launch": evals_per_launch,
                 "gate_tested_scenarios_per_launch": gated_per_launch,
                 "path": "table" if table_path(w.O, w.S) else "plain",
                 "peak_basis": f"{sms} SMs x 4 issue slots x 32 lanes x {sm_max:.0f} MHz (max SM clock)",

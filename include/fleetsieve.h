@@ -435,8 +435,10 @@ int fs_check(fs_model *m, void *cuda_stream);
  * Monte-Carlo kernel time (ms), the number of timed calls, in mode 2
  * phase_ms[4] = summed (solve, prep, Monte-Carlo, reduction) time, and
  * work_counts[2] = what the Monte-Carlo kernel's table path did since the
- * counts were last zeroed: the gap-table entries it evaluated (two t* each;
- * once per segment) and the scenarios that tested their tail gate (those of
+ * counts were last zeroed: the t* its gap-table builds evaluated (at most two
+ * per entry, once per segment; an entry whose capacity is at or below a
+ * realisation's Cexcl takes that realisation's closed-gate t* without
+ * evaluating it) and the scenarios that tested their tail gate (those of
  * strata whose tails lie on both sides of the SLO) (each output nullable); it
  * clears the record and the counts. Events between kernels also stop the
  * next kernel from starting early, so timed calls can take a little longer.

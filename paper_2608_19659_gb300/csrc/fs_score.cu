@@ -846,30 +846,40 @@ __device__ uint64_t run_piece_dump(const Set& set, const Plan& pl, int item, int
 // once per chunk (two t* each, the same arithmetic as a scenario), after which
 // a scenario costs its share of the Philox call, one index and one
 // shared-memory load. Each entry is the value as one 64-bit word.
+// Without the prior an entry whose capacity is at or below a realisation's
+// Cexcl leaves that row at Cexcl, so its t* is the closed-gate one (H_TCL)
+// and is not evaluated again.
 // RF: under the monotone prior the closed-gate values also depend on the
 // position (the draw refits the row's other bins): entries [W, 2W) hold them,
 // evaluated when `closed` (the open half when `open`).
+// Returns the number of t* this thread evaluated (the measurement's count).
 template <bool TS, int ROW, bool FL, bool RF>
-__device__ __forceinline__ void build_gtab(uint64_t* gtab, int W, const float* win, const float* h0, const float* h1,
+__device__ __forceinline__ int build_gtab(uint64_t* gtab, int W, const float* win, const float* h0, const float* h1,
                                            const float* kap0, const float* thx0, const float* mnx0,
                                            const float* kap1, const float* thx1, const float* mnx1,
                                            bool open = true, bool closed = false) {
   const int st0 = __float_as_int(h0[H_STEP0]), st1 = __float_as_int(h1[H_STEP0]);
   const float cx0 = h0[H_CX], cx1 = h1[H_CX];
+  const float tcl0 = h0[H_TCL], tcl1 = h1[H_TCL];
   const RowCap rc0 = row_cap_of(h0), rc1 = row_cap_of(h1);
   const float lam = h0[H_LAM], rlam = h0[H_RLAM], dl = h0[H_DLT];
   const float* capw = win + 4;
   const int k0 = (RF && !open) ? W : 0, k1 = (RF && closed) ? 2 * W : W;
+  int evals = 0;
   for (int k = k0 + (int)threadIdx.x; k < k1; k += blockDim.x) {
     const bool g = k < W;
     const float cy = capw[g ? k : k - W];
     const float c0 = RF ? row_cap(rc0, cy, g) : fmaxf(cx0, cy);
     const float c1 = RF ? row_cap(rc1, cy, g) : fmaxf(cx1, cy);
-    const float t0 = tstar_of<ROW, FL>(c0, kap0, thx0, mnx0, st0, lam, rlam, dl);
-    const float t1 = tstar_of<ROW, FL>(c1, kap1, thx1, mnx1, st1, lam, rlam, dl);
+    // at or below Cexcl the row keeps Cexcl: t* is the closed-gate one
+    const bool e0 = RF || cy > cx0, e1 = RF || cy > cx1;
+    const float t0 = e0 ? tstar_of<ROW, FL>(c0, kap0, thx0, mnx0, st0, lam, rlam, dl) : tcl0;
+    const float t1 = e1 ? tstar_of<ROW, FL>(c1, kap1, thx1, mnx1, st1, lam, rlam, dl) : tcl1;
+    evals += (int)e0 + (int)e1;
     const uint64_t gv = fixed40(__fsub_rn(t1, t0));
     gtab[k] = gv;
   }
+  return evals;
 }
 
 // Work decomposition of one k_score launch: segment = (item, outcome) with
@@ -1011,10 +1021,6 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
         } else {
           if (tid == 0) {
             if (!RF) gtab[pl.W] = gc;
-            // entries evaluated, once per segment (later chunks of a segment
-            // rebuild the same table): the measurement's algorithmic count
-            const int halves = RF ? (any_open ? 1 : 0) + (any_closed ? 1 : 0) : 1;
-            if (KC && part == 0) atomicAdd(&set.work[2], (unsigned long long)pl.W * halves);
             // scenarios that test their tail gate (a stratum on both sides of the SLO)
             if (KC && part == 0 && any_open && any_closed) atomicAdd(&set.work[3], (unsigned long long)pl.S);
           }
@@ -1022,9 +1028,10 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
           const bool r0 = __float_as_int(h0[H_ROW]) != 0, r1 = __float_as_int(h1[H_ROW]) != 0;
           const bool f0 = __float_as_int(h0[H_FAST]) != 0, f1 = __float_as_int(h1[H_FAST]) != 0;
           const int row = (!r0 && !r1) ? 0 : ((!r0 || f0) && (!r1 || f1)) ? 1 : 2;
-#define FS_BUILD(TSV, ROWV, FLV)                                                                            \
-  build_gtab<TSV, ROWV, FLV, RF>(gtab, pl.W, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, k1 + Lp1, k1 + 2 * Lp1, \
-                                 any_open, any_closed)
+          int evals;
+#define FS_BUILD(TSV, ROWV, FLV)                                                                          \
+  evals = build_gtab<TSV, ROWV, FLV, RF>(gtab, pl.W, stg, h0, h1, k0, k0 + Lp0, k0 + 2 * Lp0, k1, k1 + Lp1, \
+                                         k1 + 2 * Lp1, any_open, any_closed)
 #define FS_BUILDS(TSV)                       \
   if (row == 0) FS_BUILD(TSV, 0, false);     \
   else if (row == 1) FS_BUILD(TSV, 1, FL);   \
@@ -1040,6 +1047,12 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
           }
 #undef FS_BUILDS
 #undef FS_BUILD
+          if (KC && part == 0) {
+            // t* evaluated, once per segment (later chunks of a segment
+            // rebuild the same table): the measurement's algorithmic count
+            evals = __reduce_add_sync(0xffffffffu, evals);
+            if (lane == 0 && evals) atomicAdd(&set.work[2], (unsigned long long)evals);
+          }
         }
         if (!KC) {
           const int p = __float_as_int(h0[H_P]);

@@ -448,8 +448,8 @@ def fs_timing_enable(m: Model, mode: int) -> None:
 
 def fs_timing_read(m: Model, with_entries: bool = False):
     """(Monte-Carlo kernel ms, timed calls, [solve, prep, Monte-Carlo, reduction] ms) since the last
-    read; with_entries adds the work counts since then: (gap-table entries evaluated, scenarios
-    that tested their tail gate)."""
+    read; with_entries adds the work counts since then: (t* evaluated in gap-table builds,
+    scenarios that tested their tail gate)."""
     ms = C.c_double()
     n = C.c_int32()
     ph = np.zeros(4, np.float64)

@@ -153,7 +153,8 @@ def test_oracle_prefix_is_a_prefix_of_the_workload():
 
 def test_algorithmic_counts_of_the_scorer_paths():
     """The roofline's algorithmic thread-operations: 14 per scenario, 3 per tail-gate
-    test and 15 per table entry evaluated on the table path (at most W per segment), 32 per scenario on
+    test and 7.5 per t* evaluated in a table build on the table path (at most two per entry, W entries
+    per segment; 15 per fully evaluated entry), 32 per scenario on
     the plain path; the path rule mirrors the scorer's (3 (W + 1) at most twice
     the smaller of S and 2048)."""
     sys.path.insert(0, ROOT)
@@ -164,8 +165,8 @@ def test_algorithmic_counts_of_the_scorer_paths():
     assert bench.table_path(w1.O, w1.S) and bench.table_path(w3.O, w3.S) and not bench.table_path(w0.O, w0.S)
     assert abs(bench.algorithmic_ops(w1) / w1.scenarios - (17 + 15 * 512 / 4096)) < 1e-12
     assert abs(bench.algorithmic_ops(w3) / w3.scenarios - (17 + 15 * 256 / 16384)) < 1e-12
-    # with the library's counts: 14 per scenario, 3 per gate test, 15 per entry evaluated
-    assert bench.algorithmic_ops(w3, 1000.0, 500.0) == 14.0 * w3.scenarios + 3.0 * 500.0 + 15.0 * 1000.0
+    # with the library's counts: 14 per scenario, 3 per gate test, 7.5 per t* evaluated
+    assert bench.algorithmic_ops(w3, 1000.0, 500.0) == 14.0 * w3.scenarios + 3.0 * 500.0 + 7.5 * 1000.0
     assert bench.algorithmic_ops(w0) == 32 * w0.scenarios
     # the rule's edges: W = 512 needs 769 samples (3 * 513 <= 2 * 769), W = 4096 at most
     assert bench.table_path(8, 770) and not bench.table_path(8, 769)

@@ -376,16 +376,25 @@ def test_models_of_different_sizes_used_alternately(fsb, cuda, oracle_lib, qn):
 
 
 def test_table_work_counted_by_the_library(fsb, cuda, oracle_lib, qn):
-    """The table path evaluates W gap-table entries in each segment whose tail
+    """The table path builds W gap-table entries in each segment whose tail
     gate is open at some position of its stratum, and none where it is closed at
-    every position (all entries are the closed-gate value); only the scenarios of
-    strata whose tails lie on both sides of the SLO test their gate. The
-    library's counts, which the benchmark's algorithmic work uses, must say
-    exactly that."""
+    every position (all entries are the closed-gate value); an entry evaluates a
+    realisation's t* only where its capacity lies above that realisation's
+    Cexcl (the best SLO-feasible capacity of the candidate's row without its
+    bin; at or below it t* is the closed-gate one). Only the scenarios of strata
+    whose tails lie on both sides of the SLO test their gate. The library's
+    counts, which the benchmark's algorithmic work uses, must say exactly that."""
     w = workloads.make_workload(1)
     W = 4096 // w.O
     lo, hi = w.tail_lo.reshape(-1), w.tail_hi.reshape(-1)
+    clo, chi = w.cap_lo.reshape(-1), w.cap_hi.reshape(-1)
     L = np.repeat(w.slo, 4 * w.B)
+
+    def cexcl(c, sigma):  # A- (cap_lo, tail_hi) or A+ (cap_hi, tail_lo)
+        cap, tail = (chi, lo) if sigma else (clo, hi)
+        row = c - c % w.B
+        feas = [cap[x] for x in range(row, row + w.B) if x != c and tail[x] <= L[x]]
+        return max(feas) if feas else 0.0
     # the smallest and largest tail values of stratum o map its first and last quantile
     first = [[oracle_lib.map_value(lo[c], hi[c], qn[o * W]) <= L[c] for o in range(w.O)] for c in w.candidates]
     last = [[oracle_lib.map_value(lo[c], hi[c], qn[(o + 1) * W - 1]) <= L[c] for o in range(w.O)]
@@ -393,11 +402,19 @@ def test_table_work_counted_by_the_library(fsb, cuda, oracle_lib, qn):
     open_segments = sum(f for row in first for f in row)
     mixed = sum(f and not g for fr, lr in zip(first, last) for f, g in zip(fr, lr))
     assert 0 < open_segments < len(w.candidates) * w.O and mixed > 0
+    evals = 0
+    for c, row in zip(w.candidates, first):
+        cx = (cexcl(c, 0), cexcl(c, 1))
+        for o in range(w.O):
+            if row[o]:
+                cy = [oracle_lib.map_value(clo[c], chi[c], qn[o * W + k]) for k in range(W)]
+                evals += sum(int(y > cx[0]) + int(y > cx[1]) for y in cy)
+    assert 0 < evals < 2 * open_segments * W
     with load_model(fsb, w) as m:
         fsb.fs_timing_enable(m, 1)
         r = fsb.fs_score_candidates(m, w.candidates, w.O, w.S, w.seed)
         r = fsb.fs_score_candidates(m, w.candidates, w.O, w.S, w.seed)
         _, n, _, (entries, gated) = fsb.fs_timing_read(m, with_entries=True)
-        assert n == 2 and entries == 2 * open_segments * W and gated == 2 * mixed * w.S
+        assert n == 2 and entries == 2 * evals and gated == 2 * mixed * w.S
         assert fsb.fs_timing_read(m, with_entries=True)[3] == (0, 0)
     assert np.array_equal(r.sum_eo, oracle_lib.score(w, qn).sum_eo)
