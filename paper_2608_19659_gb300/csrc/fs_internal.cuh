@@ -468,8 +468,8 @@ struct LaunchCache {
   int floors = 0;  // some class has a floor > 0: launch the kernel instances with floors
   size_t solve_smem[2] = {0, 0}, prep_smem[4] = {0, 0, 0, 0};
   size_t score_smem[kScoreVariants][4] = {};
-  // resident blocks per SM of 256 and of 128 threads
-  int score_blocks_per_sm[kScoreVariants][4][2] = {};
+  // resident blocks per SM of 256, 128 and 64 threads
+  int score_blocks_per_sm[kScoreVariants][4][3] = {};
 };
 
 cudaError_t launch_qtable(float* qn, int Q, cudaStream_t s);

@@ -1254,7 +1254,7 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
   const void* kfun = reinterpret_cast<const void*>(kern);
   if (smem != lc.score_smem[v][mode]) {
     cudaError_t e = raise_smem_limit(kfun, smem);
-    for (int b = 0; b < 2 && e == cudaSuccess; ++b) {
+    for (int b = 0; b < 3 && e == cudaSuccess; ++b) {
       int per_sm = 0;
       e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kfun, kScoreThreads >> b, smem);
       lc.score_blocks_per_sm[v][mode][b] = per_sm < 1 ? 1 : per_sm;
@@ -1278,7 +1278,10 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
   if (table) {
     // Every chunk pays a fixed set-up (its records' wait, header reads, the
     // barrier, the reduction and its atomic) and builds its segment's table
-    // before it draws. Pick the block size (256 or 128 threads) and the chunk
+    // before it draws. Pick the block size (256 or 128 threads; also 64 over
+    // several problems, whose segments are short: on one problem's long
+    // segments 64-thread blocks, each holding a full block's shared memory,
+    // measured slower than the model says) and the chunk
     // length (up to 4096 calls per chunk) that minimise rounds of chunks per
     // block x resident threads per SM x (set-up + build + draws), in units of
     // about one thread-instruction: set-up ~180 per thread, an entry ~60 per
@@ -1286,7 +1289,7 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
     // more of a segment's calls, so the set-up is paid fewer times.
     const long long n_seg = (long long)it.n * pl.O;
     long long best = -1;
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < (one ? 2 : 3); ++b) {
       const int tb = kScoreThreads >> b;
       const long long res_b = (long long)lc.score_blocks_per_sm[v][mode][b] * sm_count;
       const long long us_b = ((long long)pl.calls + tb - 1) / tb;

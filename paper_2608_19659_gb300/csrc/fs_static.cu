@@ -217,6 +217,7 @@ extern "C" int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, cons
           g.score_smem[v][f] = lc.score_smem[v][f];
           g.score_blocks_per_sm[v][f][0] = lc.score_blocks_per_sm[v][f][0];
           g.score_blocks_per_sm[v][f][1] = lc.score_blocks_per_sm[v][f][1];
+          g.score_blocks_per_sm[v][f][2] = lc.score_blocks_per_sm[v][f][2];
         }
     }
   }
