@@ -311,15 +311,23 @@ def config_of(w, extra=None):
     return c
 
 
-def other_workload(idx: int, steps: int, warmup: int, alu_peak: float, stream_id: int = 0):
+def other_workload(idx: int, steps: int, warmup: int, alu_peak: float, stream_id: int = 0,
+                   demand_factor: float = 1.0):
     """The same device-resident measurement on another synthetic workload (the
     mid and large ones): step time with the L2 flushed between steps, the
-    Monte-Carlo kernel's own duration, and its roofline fraction."""
+    Monte-Carlo kernel's own duration, and its roofline fraction. demand_factor
+    scales the demands (the mid workload at its nominal demands has spare
+    capacity, so its gap is 0; at three times them it is not)."""
+    import dataclasses
+
     import torch
 
     from paper_2608_19659_gb300 import fleetsieve as fsb
 
     w = workloads.make_workload(idx)
+    if demand_factor != 1.0:
+        w = dataclasses.replace(w, name=f"{w.name}, demands x{demand_factor:g}",
+                                demand=(w.demand * np.float32(demand_factor)).astype(np.float32))
     stream = torch.cuda.current_stream()
     m = fsb.fs_load_model(w.cap_lo, w.cap_hi, w.tail_lo, w.tail_hi, w.slo, w.demand, w.G, w.K, w.B,
                           stream=stream)
@@ -785,6 +793,9 @@ def main(argv=None):
     if world == 1 and not args.no_other_workloads:
         others = [other_workload(i, max(3, min(args.steps, 10)), args.warmup, alu_peak)
                   for i in (1, 2, 3) if i != args.workload]
+        # the mid workload at three times its demands: a nonzero gap (its oracle
+        # sums are stored in tests/golden/mid_workload_x3_sums.txt)
+        others.append(other_workload(2, max(3, min(args.steps, 10)), args.warmup, alu_peak, demand_factor=3.0))
     replay = None
     if world == 1 and not args.no_replay:
         replay = replay_entry(stream, alu_peak)
