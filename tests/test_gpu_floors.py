@@ -281,3 +281,23 @@ def test_score_with_floors_near_row_table_limit(fsb, cuda, oracle_lib, qn, K, B,
     ref = oracle_lib.score(w, qn, candidates=cand, seed=91, stream_id=4, rnd=2, O=2, S=16)
     assert np.array_equal(r.sum_eo, ref.sum_eo) and np.array_equal(r.score, ref.score)
     assert r.gamma_t == ref.gamma_t and r.best == ref.best
+
+
+def test_large_workload_with_floors_sampled(fsb, cuda, oracle_lib, qn):
+    """Floors on the eight-class grid at twice its demands (16,384 segments of
+    512 samples: the Monte-Carlo kernel's many-segment launch shape), two
+    classes critical (A- then misses a floor: Gamma_t = 1): candidates with a
+    positive score and a few others, compared in full with the oracle."""
+    w = workloads.make_workload(3)
+    w = dataclasses.replace(w, demand=(w.demand * np.float32(2.0)).astype(np.float32), S=512)
+    fl = np.zeros(w.K, np.float32)
+    fl[0] = np.float32(0.5)
+    fl[3] = np.float32(0.25)
+    w = dataclasses.replace(w, floor=fl)
+    with load_model(fsb, w) as m:
+        full = fsb.fs_score_candidates(m, w.candidates, w.O, w.S, w.seed)
+    pos = np.nonzero(full.score > 0)[0]
+    pick = np.unique(np.concatenate([pos[:3], pos[-2:], [0, 1, len(w.candidates) // 2, len(w.candidates) - 1]]))
+    se, gt = oracle_lib.score_sums_cached(w, qn, candidates=w.candidates[pick])
+    assert gt == full.gamma_t
+    assert np.array_equal(full.sum_eo[pick], se)
