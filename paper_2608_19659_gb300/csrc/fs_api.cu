@@ -890,12 +890,13 @@ int fs_replay(fs_model* m, const fs_replay_spec* sp, int32_t* rounds, int32_t* s
     for (int r = 0; r <= sp->max_rounds; ++r) {
       FS_CUDA(launch_solve(set, 2 * P, nullptr, nullptr, nullptr, true, m->lc, s), "launch solve");
       FS_CUDA(cudaMemsetAsync(rs.n_active, 0, 4, s), "clear active");
-      FS_CUDA(launch_replay_certify(set, rs, r, s), "launch certify");
+      const int per = cells - sp->r0 - r;  // candidates of each running stream this round
+      // the certificate, and the running streams' candidate lists (scored reveals)
+      FS_CUDA(launch_replay_certify(set, rs, r, sp->policy == 0 ? per : 0, s), "launch certify");
       int n_active = 0;
       FS_CUDA(cudaMemcpyAsync(&n_active, rs.n_active, 4, cudaMemcpyDeviceToHost, s), "read active");
       FS_CUDA(cudaStreamSynchronize(s), "round sync");
       if (n_active == 0) break;
-      const int per = cells - sp->r0 - r;
       if (per <= 0) break;
       if (sp->policy == 1) {
         FS_CUDA(launch_replay_next(set, rs, n_active, s), "launch reveal");
@@ -904,7 +905,6 @@ int fs_replay(fs_model* m, const fs_replay_spec* sp, int32_t* rounds, int32_t* s
       const int n_items = n_active * per;
       int rc2 = ensure_items(m, n_items, sp->O);
       if (rc2) return rc2;
-      FS_CUDA(launch_replay_items(set, rs, n_active, per, s), "launch items");
       Items it{};
       it.n = n_items;
       it.p = rs.item_p;

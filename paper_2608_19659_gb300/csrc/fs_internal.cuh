@@ -544,9 +544,9 @@ struct ReplayState {
 // prior: DEVICE [4][cells] bounds every stream starts from.
 cudaError_t launch_replay_init(const Set& set, const ReplayState& rs, const float* prior, int r0,
                                cudaStream_t s);
-cudaError_t launch_replay_certify(const Set& set, const ReplayState& rs, int round, cudaStream_t s);
-cudaError_t launch_replay_items(const Set& set, const ReplayState& rs, int n_active, int per,
-                                cudaStream_t s);
+// Certificate of every running stream; with per > 0 also each running
+// stream's list of per candidates (items [slot][per]).
+cudaError_t launch_replay_certify(const Set& set, const ReplayState& rs, int round, int per, cudaStream_t s);
 cudaError_t launch_replay_next(const Set& set, const ReplayState& rs, int n_active, cudaStream_t s);
 cudaError_t launch_replay_reveal(const Set& set, const ReplayState& rs, const Items& it,
                                  const Plan& pl, const uint64_t* sums, int n_active, cudaStream_t s);

@@ -2,8 +2,8 @@
 //
 // Every stream k is one problem of the set: its own bounds, revealed flags
 // and hidden truth. A round runs, for all streams still going:
-//   A-, A+ (k_solve) -> certificate (Section 4.2) -> candidate list (the
-//   unrevealed cells in the stream's reveal order) -> k_prep / k_score
+//   A-, A+ (k_solve) -> certificate (Section 4.2) and candidate list (the
+//   unrevealed cells in the stream's reveal order; one kernel) -> k_prep / k_score
 //   (Section 4.3) -> argmax -> reveal (interval collapses to the truth; under
 //   the monotone prior the rest of its row is refit, Section 4.1).
 // The fixed-order policy skips the scoring and reveals the next cell of the
@@ -45,22 +45,26 @@ __global__ void k_replay_init(Set set, ReplayState rs, const float* prior, int r
   for (int q = 0; q < r0; ++q) reveal_cell(set, rs, p, rs.perm[(size_t)p * cells + q]);
 }
 
-// Certificate of every running stream; collects the ones that go on.
-__global__ void k_replay_certify(Set set, ReplayState rs, int round) {
-  const int p = blockIdx.x * blockDim.x + threadIdx.x;
-  if (p >= set.P || rs.state[p] >= 0) return;
+// Certificate of every running stream, one warp per stream; collects the ones
+// that go on, and (per > 0) writes each one's candidate list: its unrevealed
+// cells in reveal order, 32 cells of the order at a time, each lane's place in
+// the list from a ballot of the unrevealed ones before it.
+__global__ void k_replay_certify(Set set, ReplayState rs, int round, int per) {
+  const int p = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
+  if (p >= set.P || rs.state[p] >= 0) return;  // (the warp's lanes agree)
   const Dims& d = set.d;
   const fs_allocation& am = set.base[2 * p];
   const fs_allocation& ap = set.base[2 * p + 1];
   const float gt = __fsub_rn(ap.t_star, am.t_star);
-  rs.gamma_trace[(size_t)p * (rs.max_rounds + 1) + round] = gt;
-  bool known = true;
-  for (int i = 0; i < d.K; ++i) {
+  if (lane == 0) rs.gamma_trace[(size_t)p * (rs.max_rounds + 1) + round] = gt;
+  bool known = true;  // every cell A- commits replicas to is revealed
+  for (int i = lane; i < d.K; i += 32) {
     if (am.replicas[i] <= 0) continue;
     const int j = __ffs(am.tp[i]) - 1;
     const int c = (i * 4 + j) * d.B + am.bin[i];
     if (!set.revealed[(size_t)p * d.cells + c]) known = false;
   }
+  known = __all_sync(0xffffffffu, known);
   // Section 4.2: infeasible when even A+ misses a critical floor; feasible
   // when A- meets the floors, the gap is within eps and A-'s cells are known
   int st = -1;
@@ -68,22 +72,22 @@ __global__ void k_replay_certify(Set set, ReplayState rs, int round) {
   else if (am.floors_met && gt <= rs.eps && known) st = 1;
   else if (round >= rs.max_rounds || rs.n_revealed[p] >= d.cells) st = 0;
   if (st >= 0) {
-    rs.state[p] = st;
-    rs.rounds[p] = round;
-    rs.final_minus[p] = am;
-  } else {
-    rs.active[atomicAdd(rs.n_active, 1)] = p;
+    if (lane == 0) {
+      rs.state[p] = st;
+      rs.rounds[p] = round;
+    }
+    const uint32_t* src = reinterpret_cast<const uint32_t*>(&am);
+    uint32_t* dst = reinterpret_cast<uint32_t*>(rs.final_minus + p);
+    for (int w = lane; w < (int)(sizeof(fs_allocation) / 4); w += 32) dst[w] = src[w];
+    return;
   }
-}
-
-// Candidates of running stream slot a: its unrevealed cells in reveal order.
-// One warp per slot: 32 cells of the order at a time, each lane's place in
-// the list from a ballot of the unrevealed ones before it.
-__global__ void k_replay_items(Set set, ReplayState rs, int n_active, int per) {
-  const int a = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
-  if (a >= n_active) return;
-  const int p = rs.active[a];
-  const Dims& d = set.d;
+  int a = 0;
+  if (lane == 0) {
+    a = atomicAdd(rs.n_active, 1);
+    rs.active[a] = p;
+  }
+  a = __shfl_sync(0xffffffffu, a, 0);
+  if (per <= 0) return;
   int q = 0;
   for (int k0 = 0; k0 < d.cells && q < per; k0 += 32) {
     const int k = k0 + lane;
@@ -131,15 +135,9 @@ cudaError_t launch_replay_init(const Set& set, const ReplayState& rs, const floa
   return cudaGetLastError();
 }
 
-cudaError_t launch_replay_certify(const Set& set, const ReplayState& rs, int round, cudaStream_t s) {
+cudaError_t launch_replay_certify(const Set& set, const ReplayState& rs, int round, int per, cudaStream_t s) {
   note_launch();
-  k_replay_certify<<<(set.P + 127) / 128, 128, 0, s>>>(set, rs, round);
-  return cudaGetLastError();
-}
-
-cudaError_t launch_replay_items(const Set& set, const ReplayState& rs, int n_active, int per, cudaStream_t s) {
-  note_launch();
-  k_replay_items<<<(n_active + 3) / 4, 128, 0, s>>>(set, rs, n_active, per);
+  k_replay_certify<<<(set.P + 3) / 4, 128, 0, s>>>(set, rs, round, per);
   return cudaGetLastError();
 }
 
