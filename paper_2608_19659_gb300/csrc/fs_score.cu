@@ -933,7 +933,10 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
   uint64_t* bar = reinterpret_cast<uint64_t*>(smraw);  // [2]
   float* stage0 = reinterpret_cast<float*>(smraw + 16);
   const int stage_floats = pl.Wp + 2 * sg.tcopy;
-  // GT: two tables of W + 1 entries (2W under the prior), used by alternate chunks
+  // GT: two tables of W + 1 entries (2W under the prior), used by alternate
+  // chunks; over several problems (short segments, blocks of 64 threads whose
+  // count per SM shared memory limits) one table and one more barrier a chunk
+  constexpr bool kOneTable = GT && !KC;
   uint64_t* gtab2 = reinterpret_cast<uint64_t*>(smraw + 16 + (size_t)2 * stage_floats * 4);
   const int gt_len = RF ? 2 * pl.W : pl.W + 1;
   // per stage: chunk index, its segment and its part (thread 0 divides once)
@@ -1002,8 +1005,10 @@ __global__ void __launch_bounds__(kScoreThreads, 4) k_score(Set set, Items it, P
       // One barrier a chunk: every thread's reads of stage st (table build and
       // the gate position) come before it, so thread 0 may refill the stage
       // next iteration, and the next chunk builds the other table while a late
-      // thread may still draw from this one.
-      uint64_t* gtab = gtab2 + (size_t)(j & 1) * gt_len;
+      // thread may still draw from this one (with one table, a second barrier
+      // before the build).
+      uint64_t* gtab = kOneTable ? gtab2 : gtab2 + (size_t)(j & 1) * gt_len;
+      if (kOneTable) __syncthreads();  // every thread has drawn from the previous chunk's table
       const int cell = ok ? __float_as_int(h0[H_CELL]) : -1;
       const bool use = cell >= 0 && cell < d.cells;  // a bad device-side id was flagged by k_prep
       // passing tail positions of the stratum, as the top bits of a 16-bit field
@@ -1240,7 +1245,7 @@ cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const 
   const bool rf = set.prior == 1;
   const size_t stages = 16 + 2 * (size_t)(pl.Wp + 2 * sg.tcopy) * 4;
   const size_t gt_len = rf ? 2 * (size_t)pl.W : (size_t)pl.W + 1;
-  const size_t smem = stages + (table ? (2 * 8 * gt_len + 15) / 16 * 16 : 0);
+  const size_t smem = stages + (table ? ((it.p == nullptr ? 2 : 1) * 8 * gt_len + 15) / 16 * 16 : 0);
   const int v = dump ? SCORE_DUMP : table ? (it.p == nullptr ? SCORE_TABLE : SCORE_TABLE_MULTI) : SCORE_PLAIN;
   const int fl = lc.floors ? 1 : 0, mode = fl + (rf ? 2 : 0);
   const bool one = it.p == nullptr;  // every item belongs to problem 0
