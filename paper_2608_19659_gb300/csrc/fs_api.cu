@@ -350,7 +350,8 @@ int run_score(fs_model* m, const Set& set, const fs_samples* smp, const int32_t*
   if (phases) FS_CUDA(cudaEventRecord(ev[0], s), "record timing event");
   FS_CUDA(launch_solve(set, 2, nullptr, nullptr, nullptr, true, m->lc, s, true), "launch solve");
   if (phases) FS_CUDA(cudaEventRecord(ev[1], s), "record timing event");
-  FS_CUDA(launch_prep(set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, true, m->sm_count, m->lc, s), "launch prep");
+  FS_CUDA(launch_prep(set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, true, m->sm_count, m->lc, s),
+          "launch prep");
   if (timed) FS_CUDA(cudaEventRecord(ev[2], s), "record timing event");
   FS_CUDA(launch_score(set, it, pl, (const float*)m->tables.p, (uint64_t*)m->sums.p, dump,
                        fs_dump_stride(m), m->sm_count, m->lc, s),
@@ -772,7 +773,8 @@ int fs_score_goodput(fs_model* m, const fs_samples* smp, double* gap_out, double
   m->objective = saved;
   if (rc) return rc;
   uint64_t* sums = static_cast<uint64_t*>(m->sums.p);
-  FS_CUDA(launch_prep(m->set, it, pl, static_cast<float*>(m->tables.p), sums, false, m->sm_count, m->lc, s), "launch prep");
+  FS_CUDA(launch_prep(m->set, it, pl, static_cast<float*>(m->tables.p), sums, false, m->sm_count, m->lc, s),
+          "launch prep");
   FS_CUDA(launch_score_goodput(m->set, it, pl, static_cast<const float*>(m->tables.p), sums, m->lc.floors,
                                m->sm_count, s),
           "launch goodput scorer");
@@ -912,7 +914,8 @@ int fs_replay(fs_model* m, const fs_replay_spec* sp, int32_t* rounds, int32_t* s
       it.off = nullptr;
       fs_samples smp{sp->seed, 0, (uint32_t)r, n_items, sp->O, sp->S, 0, nullptr};
       const Plan pl = make_plan(m, &smp, n_items);
-      FS_CUDA(launch_prep(set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, false, m->sm_count, m->lc, s), "launch prep");
+      FS_CUDA(launch_prep(set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, false, m->sm_count, m->lc, s),
+              "launch prep");
       FS_CUDA(launch_score(set, it, pl, (const float*)m->tables.p, (uint64_t*)m->sums.p, nullptr, 0, m->sm_count,
                            m->lc, s),
               "launch score");
