@@ -915,8 +915,7 @@ __device__ __forceinline__ void stage_segment(const Set& set, const Plan& pl, co
 // blockIdx.x + gridDim.x, then (with many chunks per block) chunks handed out
 // by a global counter, so segments of unequal cost (table length, row-term
 // divisions) even out across the SMs; with few chunks per block the
-// assignment stays static (every block would meet the counter at once). A
-// chunk's data are staged in shared memory by TMA bulk copies,
+// assignment stays static (every block would meet the counter at once). A chunk's data are staged in shared memory by TMA bulk copies,
 // double-buffered: thread 0 issues the next chunk's copies (and the counter
 // increment whose result names the chunk after it) before this chunk is
 // computed. The sums are integers, so the order of the chunks does not
