@@ -110,3 +110,21 @@ def test_table_path_random_problems(fsb, cuda, oracle_lib, seed):
     qn = oracle_lib.triangular_table(4096)
     r, ref = _score_both(fsb, oracle_lib, w, qn, cand, O, S, s, sid, rnd)
     _assert_same(r, ref)
+
+
+def test_sixty_four_classes_over_every_cell(fsb, cuda, oracle_lib):
+    """64 classes (the most a model takes) with every one of their 1,024 cells a
+    candidate: 2,048 preparation blocks, so the launch takes 64-thread blocks,
+    whose threads just cover the classes' demands, and with 15,360 thresholds
+    no row table (the joint search with two probe groups a block). Sampled
+    candidates are compared with the oracle in full."""
+    rng = np.random.default_rng(4242)
+    w = _contested(oracle_lib, workloads.random_small(rng, 64, 4, 128))
+    qn = oracle_lib.triangular_table(4096)
+    cand = np.arange(w.K * 4 * w.B, dtype=np.int32)
+    with load_model(fsb, w) as m:
+        r = fsb.fs_score_candidates(m, cand, 2, 64, 7)
+    pick = np.arange(0, cand.size, 97)
+    se, gt = oracle_lib.score_sums_cached(w, qn, candidates=cand[pick], O=2, S=64, seed=7)
+    assert gt == r.gamma_t > 0
+    assert np.array_equal(r.sum_eo[pick], se)
