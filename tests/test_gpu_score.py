@@ -61,6 +61,31 @@ def test_paper_scale_workload_full(fsb, cuda, oracle_lib, qn):
     assert ref.gamma_t > 0 and (ref.score > 0).sum() > 0
 
 
+@pytest.mark.parametrize("S", [4093, 4094])
+def test_paper_scale_table_path_ragged_samples(fsb, cuda, oracle_lib, qn, S):
+    """The table path with a ragged last Philox call in every segment (S mod 4
+    samples of its four words), all 64 candidates in full."""
+    w = dataclasses.replace(workloads.make_workload(1), S=S)
+    r = run(fsb, w)
+    ref = oracle_lib.score(w, qn)
+    assert_same(r, ref)
+    assert ref.gamma_t > 0
+
+
+def test_large_workload_ragged_samples_sampled(fsb, cuda, oracle_lib, qn):
+    """The eight-class workload at S = 16,383: one problem's many-segment launch
+    (one chunk a segment) whose segments end with a call serving three
+    samples; candidates with a positive score and a few others in full."""
+    w = dataclasses.replace(workloads.make_workload(3), S=16383)
+    full = run(fsb, w)
+    pos = np.nonzero(full.score > 0)[0]
+    assert len(pos) > 0
+    pick = np.unique(np.concatenate([pos[:3], pos[-2:], [0, len(w.candidates) - 1]]))
+    se, gt = oracle_lib.score_sums_cached(w, qn, candidates=w.candidates[pick])
+    assert gt == full.gamma_t
+    assert np.array_equal(full.sum_eo[pick], se)
+
+
 @pytest.mark.parametrize("factor", [1.0, 3.0])
 def test_mid_workload_sampled_candidates(fsb, cuda, oracle_lib, qn, factor):
     w = stressed(2, factor)
