@@ -129,6 +129,24 @@ def test_goodput_stage_matches_oracle(fsb, cuda, oracle_lib, qn, idx, factor, S,
     assert ref.gamma_fx > 0 and np.any(ref.score_fixed != 0)
 
 
+def test_goodput_stage_large_workload_sampled(fsb, cuda, oracle_lib, qn):
+    """The goodput stage on the eight-class grid (G = 256: the largest programme
+    over GPUs of the workloads) at twice its demands, every candidate scored:
+    candidates with a positive goodput score and a few others against the
+    oracle in full."""
+    w = workloads.make_workload(3)
+    w = dataclasses.replace(w, demand=(w.demand * np.float32(2.0)).astype(np.float32), S=64)
+    with load_model(fsb, w) as m:
+        full = fsb.fs_score_goodput(m, w.candidates, w.O, w.S, w.seed)
+    pos = np.nonzero(full.score > 0)[0]
+    assert len(pos) > 0
+    pick = np.unique(np.concatenate([pos[:2], pos[-1:], [0, len(w.candidates) // 2]]))
+    ref = oracle_lib.score_goodput(w, qn, candidates=w.candidates[pick])
+    assert np.array_equal(full.sum_eo[pick], ref.sum_eo)
+    assert np.array_equal(full.gap[pick], ref.gap) and np.array_equal(full.score[pick], ref.score)
+    assert full.gamma_gp == ref.gamma_gp
+
+
 @pytest.mark.parametrize("prior,floor", [(1, None), (0, (0.4, 0.0)), (1, (0.0, 0.5))])
 def test_goodput_stage_with_prior_and_floors(fsb, cuda, oracle_lib, qn, prior, floor):
     w = workloads.make_workload(0)
