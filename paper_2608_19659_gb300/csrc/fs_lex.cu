@@ -403,9 +403,12 @@ __host__ __device__ inline GoodputSmem goodput_smem(int K4, int G, int gt_len, i
 // segment, so a warp reruns that part only where a range changes and
 // otherwise only combines it with class i_r's choices. Then the same draws
 // and sums as the table path.
-template <bool FL, bool RF>
-__global__ void __launch_bounds__(256, 2) k_score_goodput(Set set, Items it, Plan pl, const float* rec,
-                                                       uint64_t* sums) {
+// MINB: resident blocks per SM the registers are capped for (2, or 4 for
+// launches of many segments, whose throughput gains more from the occupancy
+// than each block loses).
+template <bool FL, bool RF, int MINB>
+__global__ void __launch_bounds__(256, MINB) k_score_goodput(Set set, Items it, Plan pl, const float* rec,
+                                                          uint64_t* sums) {
   extern __shared__ __align__(16) unsigned char smraw[];
   const Dims& d = set.d;
   const int W = pl.W, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarp = blockDim.x >> 5;
@@ -608,15 +611,22 @@ cudaError_t launch_score_goodput(const Set& set, const Items& it, const Plan& pl
   size_t smem = 0;
   const int threads = goodput_threads(set.d, pl, rf, &smem);
   if (threads == 0) return cudaErrorInvalidValue;  // refused by the host before this point
-  auto kern = floors ? (rf ? k_score_goodput<true, true> : k_score_goodput<true, false>)
-                     : (rf ? k_score_goodput<false, true> : k_score_goodput<false, false>);
+  // many segments (beyond four waves of two blocks per SM): the instance with
+  // registers for four blocks per SM (measured 5.94 -> 3.44 ms on the
+  // eight-class workload, 0.375 -> 0.325 ms on the mid one at three times its
+  // demands; the paper-scale call, one wave, slower: 0.17 -> 0.19 ms)
+  const long long n_seg = (long long)it.n * pl.O;
+  const bool wide = n_seg > 4LL * 2 * sm_count;
+#define FS_GP(MB) \
+  (floors ? (rf ? k_score_goodput<true, true, MB> : k_score_goodput<true, false, MB>) \
+          : (rf ? k_score_goodput<false, true, MB> : k_score_goodput<false, false, MB>))
+  auto kern = wide ? FS_GP(4) : FS_GP(2);
+#undef FS_GP
   cudaError_t e = raise_smem_limit(reinterpret_cast<const void*>(kern), smem);
   if (e != cudaSuccess) return e;
   // one block per segment: segments differ widely in cost (where row r sets
   // t*, its ranges change often), and the block scheduler evens them out
-  const long long n_seg = (long long)it.n * pl.O;
   const long long grid = n_seg < 0x7fffffffLL ? n_seg : 0x7fffffffLL;
-  (void)sm_count;
   note_launch();
   kern<<<(unsigned)grid, threads, smem, s>>>(set, it, pl, tables, sums);
   return cudaGetLastError();
