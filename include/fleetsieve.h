@@ -230,12 +230,12 @@ int fs_score_candidates_async(fs_model *m, const fs_samples *samples, double *ga
  *   8 n O (the fixed-point sums).
  * On the paper-scale grid (K = 2, G = 16, O = 8, Q = 4096) that allows 913
  * candidates per call.
- * The first call on a device looks up the array's address for that device,
- * so make it before any stream capture. Every call shares the array, which
- * keeps the last call's contents (the kernels clear what must start at zero):
- * calls whose GPU work overlaps (other streams or host threads) race. The
- * call enqueues its kernels on cuda_stream, waits for that stream before it
- * returns and reports device-side errors (FS_ETIMEOUT, FS_EDEVICE).
+ * Every call shares the array, which keeps the last call's contents (the
+ * kernels clear what must start at zero): calls whose GPU work overlaps
+ * (other streams or host threads) race. The call enqueues its kernels on
+ * cuda_stream, copies the status word to the host and synchronises the
+ * stream before it returns, reporting device-side errors (FS_ETIMEOUT,
+ * FS_EDEVICE); it therefore cannot be captured into a CUDA graph.
  */
 int fs_score_candidates_noalloc(int32_t K, int32_t B, int32_t G, const float *bounds_dev,
                                 const float *slo_dev, const float *demand_dev,
