@@ -171,6 +171,7 @@ struct fs_model {
   cudaEvent_t up_done = nullptr;
   bool up_pending = false;
   bool staged = false;  // the staging holds bounds the device copy does not have yet
+  int th_bound = -1;    // threshold_bound of the current bounds (-1: not computed yet)
   LaunchCache lc;
   // optional timing events: 5 per timed call (before solve, prep, score,
   // finalize, and after finalize); mode 1 records only the two around score
@@ -239,7 +240,48 @@ int stage_bounds(fs_model* m) {
   std::memcpy(h, m->h_bounds.data(), nb);
   std::memcpy(h + rev_off, m->h_revealed.data(), nr);
   m->staged = true;
+  m->th_bound = -1;
   return FS_OK;
+}
+
+// An upper bound on the number of thresholds of either base solve of the
+// current bounds. A row (class i, TP tau) whose best SLO-feasible capacity is
+// C holds at most min(floor(G / tau), n_sat) fulfilment values, n_sat the
+// first replica count whose fulfilment RN(RN(n C) / lambda_i) reaches 1: every
+// n >= lambda_i / C (1 + 2^-23) does (each RN step loses at most 2^-24
+// relatively), so n_sat <= floor(lambda_i / C (1 + 2^-18)) + 3, with margin for
+// the bound's own double arithmetic. A row without a feasible bin holds none.
+int threshold_bound(const fs_model* m) {
+  const Dims& d = m->d;
+  const int cells = d.cells, B = d.B;
+  const float* hb = m->h_bounds.data();
+  long long most = 0;
+  for (int sigma = 0; sigma < 2; ++sigma) {
+    const float* cap = hb + (size_t)(sigma ? CAP_HI : CAP_LO) * cells;
+    const float* tail = hb + (size_t)(sigma ? TAIL_LO : TAIL_HI) * cells;
+    long long tot = 0;
+    for (int rho = 0; rho < d.K4; ++rho) {
+      const int i = rho >> 2, M = d.G >> (rho & 3);
+      bool any = false;
+      float C = 0.0f;
+      for (int b = 0; b < B; ++b) {
+        const int c = rho * B + b;
+        if (tail[c] <= m->h_slo[i]) {
+          any = true;
+          C = std::max(C, cap[c]);
+        }
+      }
+      if (!any || M < 1) continue;
+      long long n = M;
+      if (C > 0.0f) {
+        const double q = (double)m->h_lam[i] / (double)C * (1.0 + 0x1p-18);
+        if (q < (double)M) n = std::min<long long>(M, (long long)q + 3);
+      }
+      tot += n;
+    }
+    most = std::max(most, tot);
+  }
+  return (int)std::min<long long>(most, d.theta_cap);
 }
 
 // Queue the device copy of staged bounds (if any) on the model's stream without
@@ -350,7 +392,9 @@ int run_score(fs_model* m, const Set& set, const fs_samples* smp, const int32_t*
   if (phases) FS_CUDA(cudaEventRecord(ev[0], s), "record timing event");
   FS_CUDA(launch_solve(set, 2, nullptr, nullptr, nullptr, true, m->lc, s, true), "launch solve");
   if (phases) FS_CUDA(cudaEventRecord(ev[1], s), "record timing event");
-  FS_CUDA(launch_prep(set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, true, m->sm_count, m->lc, s),
+  if (m->th_bound < 0) m->th_bound = threshold_bound(m);
+  FS_CUDA(launch_prep(set, it, pl, (float*)m->tables.p, (uint64_t*)m->sums.p, true, m->sm_count, m->lc, s,
+                      m->th_bound),
           "launch prep");
   if (timed) FS_CUDA(cudaEventRecord(ev[2], s), "record timing event");
   FS_CUDA(launch_score(set, it, pl, (const float*)m->tables.p, (uint64_t*)m->sums.p, dump,

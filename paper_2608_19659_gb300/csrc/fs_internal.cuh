@@ -487,8 +487,13 @@ cudaError_t launch_solve(const Set& set, int n, const float* cap_x, const float*
 // Blocks of 256 threads, or of 64 when the launch holds more than two waves
 // of 256-thread blocks (sm_count SMs): each block is mostly a chain of
 // dependent latencies, so more of them in flight per SM finish sooner.
+// th_cap > 0: a bound on both base solves' threshold counts small enough that
+// the solves build row tables (4K th_cap <= kRowTabMax); shared memory then
+// holds th_cap thresholds instead of theta_cap, so that more blocks fit an SM
+// (a count above it is reported as ST_TABLE, never read past).
 cudaError_t launch_prep(const Set& set, const Items& it, const Plan& pl, float* tables,
-                        uint64_t* sums, bool early, int sm_count, LaunchCache& lc, cudaStream_t s);
+                        uint64_t* sums, bool early, int sm_count, LaunchCache& lc, cudaStream_t s,
+                        int th_cap = 0);
 cudaError_t launch_score(const Set& set, const Items& it, const Plan& pl, const float* tables,
                          uint64_t* sums, void* dump, int dump_stride, int sm_count, LaunchCache& lc,
                          cudaStream_t s);

@@ -159,10 +159,10 @@ __device__ __forceinline__ float tstar_of(float C, const float* kap, const float
 // critical (the model has floors).
 template <bool FL, bool RF>
 __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan pl, float* rec,
-                                                       uint64_t* sums, int early) {
+                                                       uint64_t* sums, int early, int th_cap) {
   extern __shared__ __align__(16) unsigned char smraw[];
   float* sC = reinterpret_cast<float*>(smraw);  // [256]
-  float* sTh = sC + 256;                          // [theta_cap]
+  float* sTh = sC + 256;                          // [th_cap]
   __shared__ float s_cx, s_cmax, s_pc, s_po, s_lf, s_hf;
   __shared__ int s_bx, s_row;
   __shared__ float sLam[FS_MAX_CLASSES], sRl[FS_MAX_CLASSES];  // demand and RN(1/demand)
@@ -364,9 +364,12 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
     th_a = th_g[tid];
     if (rt_g) rt_a = rt_g[(size_t)tid * d.K4];
   }
-  const int total = set.ntheta[ps];
+  // a count above the launch's bound (reported below; the call then fails) is
+  // cut to it, so that no index passes the shared arrays
+  const int total_raw = set.ntheta[ps];
+  const int total = min(total_raw, th_cap);
   const bool rtab = rt_g != nullptr && d.K4 * total <= kRowTabMax;
-  int* sRt = reinterpret_cast<int*>(sTh + d.theta_cap);  // [min(theta_cap, kRowTabMax / 4)]
+  int* sRt = reinterpret_cast<int*>(sTh + th_cap);  // [min(th_cap, kRowTabMax / 4)]
   for (int rho = tid; rho < d.K4; rho += blockDim.x) sC[rho] = set.rowC[ps * d.K4 + rho];
   if (ahead) {
     if (tid < total) {
@@ -380,6 +383,7 @@ __global__ void __launch_bounds__(kPrepThreads) k_prep(Set set, Items it, Plan p
     }
   }
   __syncthreads();
+  if (total_raw > th_cap && tid == 0) atomicOr(set.status, ST_TABLE);
   const float cx = s_cx, cmax = s_cmax;
   const int msent = d.K == 1 ? rep_cap(d, jr) : 0;  // above every threshold only a lone class can go on
 
@@ -1206,15 +1210,17 @@ __global__ void k_finalize_split(Set set, Items it, Plan pl, const uint64_t* sum
 }
 
 // rowC, the thresholds and, with a row table, the candidate row's words
-static size_t prep_smem_bytes(const Set& set) {
-  const Dims& d = set.d;
-  return (size_t)(256 + d.theta_cap + (set.rtab ? std::min(d.theta_cap, kRowTabMax / 4) : 0)) * 4;
+static size_t prep_smem_bytes(const Set& set, int th_cap) {
+  return (size_t)(256 + th_cap + (set.rtab ? std::min(th_cap, kRowTabMax / 4) : 0)) * 4;
 }
 
 cudaError_t launch_prep(const Set& set, const Items& it, const Plan& pl, float* tables, uint64_t* sums,
-                        bool early, int sm_count, LaunchCache& lc, cudaStream_t s) {
+                        bool early, int sm_count, LaunchCache& lc, cudaStream_t s, int th_cap) {
   if (it.n <= 0) return cudaSuccess;
-  const size_t smem = prep_smem_bytes(set);
+  const Dims& d = set.d;
+  const int cap = th_cap > 0 && th_cap < d.theta_cap && set.rtab && d.K4 * th_cap <= kRowTabMax ? th_cap
+                                                                                                   : d.theta_cap;
+  const size_t smem = prep_smem_bytes(set, cap);
   const int fl = lc.floors ? 1 : 0, mode = fl + (set.prior == 1 ? 2 : 0);
   auto kern = mode == 0 ? k_prep<false, false> : mode == 1 ? k_prep<true, false>
             : mode == 2 ? k_prep<false, true> : k_prep<true, true>;
@@ -1226,7 +1232,7 @@ cudaError_t launch_prep(const Set& set, const Items& it, const Plan& pl, float* 
   // (five 256-thread blocks fit an SM by registers; 64-thread blocks need at
   // least 64 threads for the classes' demands, K <= 64)
   const int tb = (long long)it.n * 2 > 2LL * 5 * sm_count ? 64 : kPrepThreads;
-  return launch_pdl(kern, dim3(it.n * 2), dim3(tb), smem, s, set, it, pl, tables, sums, early ? 1 : 0);
+  return launch_pdl(kern, dim3(it.n * 2), dim3(tb), smem, s, set, it, pl, tables, sums, early ? 1 : 0, cap);
 }
 
 static int score_lcap(const Dims& d) { return d.lcap < kSmemTableCap ? d.lcap : kSmemTableCap; }

@@ -59,3 +59,36 @@ def test_cover_by_counting_own_values_equals_brute_force():
             assert _counted(tc, c, lam, M, delta) == _brute(tc, c, lam, M), (t, c, lam, M, delta)
             checked += 1
     assert checked > 5000
+
+
+def test_row_length_bound():
+    """A row holds at most min(M, n_sat) values, n_sat the first n with f(n) = 1.
+    The library sizes the preparation's shared thresholds by the bound
+    n_sat <= floor(lambda / c (1 + 2^-18)) + 3, which rests on every n >=
+    lambda / c (1 + 2^-23) reaching f(n) = 1 (two RN steps lose at most 2^-24
+    each). Both are checked with the oracle's fulfilment arithmetic, on ratios
+    lambda / c spread over many decades and on ratios at and next to integers,
+    where the rounding decides."""
+    rng = np.random.default_rng(21)
+    cases = []
+    for _ in range(1500):
+        lam = float(np.float32(10.0 ** rng.uniform(-2, 4)))
+        c = float(np.float32(lam / 10.0 ** rng.uniform(-3, 4)))
+        cases.append((c, lam))
+    for _ in range(1500):
+        lam = float(np.float32(10.0 ** rng.uniform(-2, 4)))
+        k = int(rng.integers(1, 5000))
+        c32 = np.float32(lam / k)
+        for c in (c32, np.nextafter(c32, np.float32(0)), np.nextafter(c32, np.float32(np.inf))):
+            cases.append((float(c), lam))
+    for c, lam in cases:
+        if c <= 0.0:
+            continue
+        n_tight = int(np.ceil(lam / c * (1.0 + 2.0 ** -23)))
+        n_bound = int(lam / c * (1.0 + 2.0 ** -18)) + 3
+        assert n_tight <= n_bound
+        if n_tight > 40000:  # beyond any replica cap (M <= 32767)
+            continue
+        assert oracle.fulfil(n_tight, c, lam) == 1.0, (c, lam, n_tight)
+        if n_tight > 1:  # and the first such n is not far below it
+            assert oracle.fulfil(max(1, int(lam / c * (1.0 - 2.0 ** -20)) - 1), c, lam) < 1.0, (c, lam)
