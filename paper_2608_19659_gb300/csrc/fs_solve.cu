@@ -126,15 +126,23 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
 
   // 1. rows: the best SLO-feasible bin of each row (largest capacity, then
   // lowest bin). The inputs of the first pass (demands, and each thread's
-  // first cell) are all loaded before anything waits on one of them: one
-  // memory round trip.
+  // first kPre cells, every cell of a model with at most kPre x 256) are all
+  // loaded before anything waits on one of them: one memory round trip. Both
+  // passes read those cells from registers; any further cells from memory.
   __shared__ float sLam[FS_MAX_CLASSES], sRl[FS_MAX_CLASSES];  // demand and RN(1/demand)
   __shared__ float sDl[FS_MAX_CLASSES];                          // floor delta_i (0: not critical)
+  constexpr int kPre = 4;
   const float lam_v = tid < d.K ? set.lam[tid] : 1.0f;
   const float dl_v = FL && tid < d.K ? set.slo[d.K + tid] : 0.0f;
-  const bool cell0 = tid < d.cells;
-  const float tail0 = cell0 ? tail[tid] : 0.0f, cap0 = cell0 ? cap[tid] : 0.0f;
-  const float slo0 = cell0 ? set.slo[(tid / d.B) >> 2] : 0.0f;
+  float tailp[kPre], capp[kPre], slop[kPre];
+#pragma unroll
+  for (int k = 0; k < kPre; ++k) {
+    const int c = tid + k * (int)blockDim.x;
+    const bool in = c < d.cells;
+    tailp[k] = in ? tail[c] : 0.0f;
+    capp[k] = in ? cap[c] : 0.0f;
+    slop[k] = in ? set.slo[(c / d.B) >> 2] : 0.0f;
+  }
   for (int rho = tid; rho < d.K4; rho += blockDim.x) {
     sRowCap[rho] = 0u;
     sRowBin[rho] = ~0u;
@@ -149,19 +157,32 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   // feasible cells: their capacity's bits (-0 -> +0: nonnegative floats order
   // like their bit patterns), first the row maximum, then the lowest bin
   // holding it
-  const bool ok0 = cell0 && tail0 <= slo0;
-  const uint32_t cb0 = __float_as_uint(__fadd_rn(cap0, 0.0f));
-  for (int c = tid; c < d.cells; c += blockDim.x) {
+  bool okp[kPre];
+  uint32_t cbp[kPre];
+  int rhop[kPre];
+#pragma unroll
+  for (int k = 0; k < kPre; ++k) {
+    const int c = tid + k * (int)blockDim.x;
+    rhop[k] = c < d.cells ? c / d.B : 0;
+    okp[k] = c < d.cells && tailp[k] <= slop[k];
+    cbp[k] = __float_as_uint(__fadd_rn(capp[k], 0.0f));
+    if (okp[k]) atomicMax(&sRowCap[rhop[k]], cbp[k]);
+  }
+  const int c_rest = tid + kPre * (int)blockDim.x;
+  for (int c = c_rest; c < d.cells; c += blockDim.x) {
     const int rho = c / d.B;
-    const bool ok = c == tid ? ok0 : tail[c] <= set.slo[rho >> 2];
-    if (ok) atomicMax(&sRowCap[rho], c == tid ? cb0 : __float_as_uint(__fadd_rn(cap[c], 0.0f)));
+    if (tail[c] <= set.slo[rho >> 2]) atomicMax(&sRowCap[rho], __float_as_uint(__fadd_rn(cap[c], 0.0f)));
   }
   __syncthreads();
-  for (int c = tid; c < d.cells; c += blockDim.x) {
+#pragma unroll
+  for (int k = 0; k < kPre; ++k) {
+    const int c = tid + k * (int)blockDim.x;
+    if (okp[k] && cbp[k] == sRowCap[rhop[k]]) atomicMin(&sRowBin[rhop[k]], (uint32_t)(c - rhop[k] * d.B));
+  }
+  for (int c = c_rest; c < d.cells; c += blockDim.x) {
     const int rho = c / d.B;
-    const bool ok = c == tid ? ok0 : tail[c] <= set.slo[rho >> 2];
-    const uint32_t cb = c == tid ? cb0 : __float_as_uint(__fadd_rn(cap[c], 0.0f));
-    if (ok && cb == sRowCap[rho]) atomicMin(&sRowBin[rho], (uint32_t)(c - rho * d.B));
+    const uint32_t cb = __float_as_uint(__fadd_rn(cap[c], 0.0f));
+    if (tail[c] <= set.slo[rho >> 2] && cb == sRowCap[rho]) atomicMin(&sRowBin[rho], (uint32_t)(c - rho * d.B));
   }
   __syncthreads();
   for (int rho = tid; rho < d.K4; rho += blockDim.x) {
@@ -226,7 +247,7 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
   int* sCmin = sCost + d.K4 * total;
   float* sOwn = reinterpret_cast<float*>(sCmin + d.K * total);
 
-  // 2. thresholds, then bitonic sort (ascending, +inf padding)
+  // 2. thresholds, then a sort (ascending, +inf padding)
   for (int x = tid; x < P2; x += blockDim.x) {
     float v = __int_as_float(0x7f800000);
     if (x < total) {
@@ -269,6 +290,20 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
       if (lane + 32 < P2) sTheta[lane + 32] = r[1];
     }
     __syncthreads();
+  } else if (row_table && P2 <= (int)blockDim.x) {
+    // up to one value a thread, the unsorted values in sOwn: each thread
+    // places its value at its rank (values below it, and equal values at
+    // lower indices), one pass with no barriers between stages
+    if (tid < total) {
+      const float v = sOwn[tid];
+      int rank = 0;
+#pragma unroll 4
+      for (int j = 0; j < total; ++j) {
+        const float u = sOwn[j];
+        rank += (u < v || (u == v && j < tid)) ? 1 : 0;
+      }
+      sTheta[rank] = v;
+    }
   } else {
     for (int k = 2; k <= P2; k <<= 1) {
       for (int jj = k >> 1; jj > 0; jj >>= 1) {
