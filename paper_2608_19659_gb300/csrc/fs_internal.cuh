@@ -32,6 +32,7 @@ namespace fs {
 constexpr int kT = 4;                 // TP degrees {1, 2, 4, 8}
 constexpr int kCostInf = 0x3FFFFFFF;  // "no option covers the threshold"
 constexpr int kSolveThreads = 256;
+constexpr int kSolveThreadsWide = 512;  // a scoring solve of a model with more than 256 cells
 constexpr int kPrepThreads = 256;
 constexpr int kScoreThreads = 256;
 constexpr int kTableHeader = 20;      // floats before the three table arrays (16-byte multiple)

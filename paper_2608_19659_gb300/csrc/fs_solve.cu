@@ -82,7 +82,7 @@ __device__ __forceinline__ int group_total_cost(float t, const float* sC, const 
 // FL: some class is critical (the model has floors); the instance without floors does
 // none of the floor work.
 template <bool FL>
-__global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, const float* cap_x,
+__global__ void __launch_bounds__(kSolveThreadsWide) k_solve(Set set, int n_real, const float* cap_x,
                                                          const float* tail_x, fs_allocation* out_x,
                                                          int mode) {
   const bool write_theta = (mode & 1) != 0;
@@ -290,10 +290,11 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
       if (lane + 32 < P2) sTheta[lane + 32] = r[1];
     }
     __syncthreads();
-  } else if (row_table && P2 <= (int)blockDim.x) {
+  } else if (row_table && P2 <= 256 && P2 <= (int)blockDim.x) {
     // up to one value a thread, the unsorted values in sOwn: each thread
     // places its value at its rank (values below it, and equal values at
-    // lower indices), one pass with no barriers between stages
+    // lower indices), one pass with no barriers between stages (its cost
+    // grows with the count: above 256 values the network below is faster)
     if (tid < total) {
       const float v = sOwn[tid];
       int rank = 0;
@@ -325,7 +326,7 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
 
   // 3. t*: the largest index whose threshold fits in G (the cheapest-cover
   // total is nondecreasing along the sorted thresholds).
-  __shared__ int s_res[2][kSolveThreads / 4];
+  __shared__ int s_res[2][kSolveThreadsWide / 4];
   if (tid == 0) sMisc[4] = 0;
   __syncthreads();
   int kstar;
@@ -446,7 +447,7 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
     // same for the floor of a critical class, summed into sMisc[5] (sMisc[6]:
     // some critical class cannot reach its floor)
     {
-      const int rho = tid;  // K4 <= 256 = blockDim
+      const int rho = tid;  // K4 <= 256 <= blockDim
       int key = 0x7fffffff, keyf = 0x7fffffff;
       if (rho < d.K4) {
         const float dl = FL ? sDl[rho >> 2] : 0.0f;
@@ -475,7 +476,7 @@ __global__ void __launch_bounds__(kSolveThreads) k_solve(Set set, int n_real, co
         const bool met = sMisc[6] == 0 && sMisc[5] <= d.G;
         if (tstar <= 0.0f) key = (critical && met) ? keyf : 0x7fffffff;  // tier 1 alone
       }
-      if ((tid & 3) == 0) {
+      if ((tid & 3) == 0 && i < FS_MAX_CLASSES) {  // (a 512-thread block has 128 groups of four)
         int8_t tp = 0;
         int16_t bin = -1, reps = 0;
         float f = 0.0f;
@@ -560,8 +561,11 @@ cudaError_t launch_solve(const Set& set, int n, const float* cap_x, const float*
     if (e != cudaSuccess) return e;
     lc.solve_smem[fl] = smem;
   }
+  // a scoring solve of a model with more than 256 cells takes 512 threads: its
+  // per-cell passes and row-table phases then run half the iterations each
+  const int bt = write_theta && !cap_x && set.d.cells > kSolveThreads ? kSolveThreadsWide : kSolveThreads;
   note_launch();
-  kern<<<n, kSolveThreads, smem, s>>>(set, n, cap_x, tail_x, out, (write_theta ? 1 : 0) | (tstar_only ? 2 : 0));
+  kern<<<n, bt, smem, s>>>(set, n, cap_x, tail_x, out, (write_theta ? 1 : 0) | (tstar_only ? 2 : 0));
   return cudaGetLastError();
 }
 
